@@ -1,0 +1,284 @@
+/*
+ * cacheroute.h -- C ABI of the GB300 (sm_103a) library for the data-parallel
+ * hot path of planned prefix-affinity routing (CacheRoute, arXiv 2608.19677).
+ *
+ * The method (paper sec. 3): once per control interval a planner turns the
+ * measured per-key request rates lambda_b into a routing table T: b -> a set
+ * of destinations (Eq. 1 and Algorithm 1); during the interval, a request
+ * whose key is in T goes to the least-loaded member of T(b), and any other
+ * request goes to the less loaded of two random destinations (power-of-two
+ * choices).  Before a table is enabled it is shadow-replayed and its cache
+ * hits and per-destination load are compared with cache-blind balancing
+ * (sec. 3.2, sec. 5.3).  The calls below are that path, on one GPU:
+ *
+ *   cr_hash_prefixes  request prefix span -> 64-bit routing key b
+ *   cr_build_plan     keys of one interval -> lambda_b, k_b, admission, LPT, table
+ *   cr_route_batch    keys -> one destination per (request, replica)
+ *   cr_shadow_replay  routed requests -> per-destination LRU hits and load
+ *
+ * Conventions shared by every call:
+ *   - Pointers named d_* are DEVICE pointers owned by the caller (any CUDA
+ *     allocation, e.g. a torch tensor's storage on the context's device).
+ *     Host pointers carry no prefix.  No call keeps a caller pointer after it
+ *     returns, except that work it enqueued reads and writes them later on
+ *     the context's stream: keep them alive until that work has finished.
+ *   - The library owns cr_ctx, cr_plan and cr_replay objects and every scratch
+ *     buffer behind them; it allocates device memory only inside
+ *     cr_create/cr_plan_create/cr_replay_create and when a call needs a
+ *     larger scratch buffer than it held before.
+ *   - Every call returns a status; nothing throws.  Calls are asynchronous on
+ *     the context's CUDA stream unless documented as blocking.  Device-side
+ *     checks (for example an arithmetic overflow found in a kernel) are
+ *     reported by the next blocking call (cr_sync, *_export, *_info).
+ *   - All quantities are unsigned integers: results are exact and
+ *     deterministic (bit-identical run to run).
+ */
+#ifndef CACHEROUTE_H
+#define CACHEROUTE_H
+
+#include <stdint.h>
+
+#if defined(__GNUC__)
+#define CR_API __attribute__((visibility("default")))
+#else
+#define CR_API
+#endif
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* ---- status codes ------------------------------------------------------- */
+#define CR_OK 0        /* success */
+#define CR_EINVAL 1    /* an argument is out of range or inconsistent */
+#define CR_ENOMEM 2    /* a device allocation failed */
+#define CR_ECUDA 3     /* a CUDA runtime call failed (see cr_last_error) */
+#define CR_ETIMEOUT 4  /* a bounded device-side wait gave up */
+#define CR_EOVERFLOW 5 /* a count or load exceeded its documented range */
+
+/* ---- dispatch policies (cr_replica.policy) -------------------------------- */
+#define CR_POLICY_CACHEROUTE 0 /* T(b) from an LPT plan, else P2C (Fig. 1)       */
+#define CR_POLICY_CR_NOLPT 1   /* T(b) from a random-placement plan, else P2C    */
+#define CR_POLICY_CR_NOREPL 2  /* T(b) from a single-copy LPT plan, else P2C     */
+#define CR_POLICY_P2C 3        /* power-of-two choices over all R ("Flat-LB")   */
+#define CR_POLICY_RR 4         /* round robin over the global request index      */
+#define CR_POLICY_HASH 5       /* sticky: jump consistent hash of the key        */
+
+/* ---- plan variants (cr_plan_params.variant) ------------------------------- */
+#define CR_VARIANT_LPT 0    /* Algorithm 1 as printed                            */
+#define CR_VARIANT_RANDOM 1 /* Eq. 1 replica counts, random distinct placement  */
+#define CR_VARIANT_NOREPL 2 /* k_b = 1 for every key, LPT placement              */
+
+/* ---- limits --------------------------------------------------------------- */
+#define CR_MAX_R 8192         /* destinations per plan / route call              */
+#define CR_MAX_CAP 1024       /* LRU capacity (prefix entries) per simulator     */
+#define CR_MAX_CAPS 8         /* capacities replayed together                    */
+#define CR_MAX_REPLICAS 256   /* (policy, seed) replicas per route/replay call   */
+#define CR_CTR_FIELDS 5       /* requests, hits, hit tokens, prompt, prefill     */
+
+typedef struct cr_ctx cr_ctx;
+typedef struct cr_plan cr_plan;
+typedef struct cr_replay cr_replay;
+
+/* ==== context ============================================================ */
+
+/* Create a context on CUDA device `device` that enqueues its work on
+ * `cuda_stream` (a cudaStream_t; NULL = the legacy default stream).
+ * *out receives the context.  Errors: CR_EINVAL (out NULL, bad device),
+ * CR_ECUDA, CR_ENOMEM. */
+CR_API int cr_create(cr_ctx **out, int device, void *cuda_stream);
+
+/* Destroy a context after waiting for its stream.  NULL is accepted. */
+CR_API int cr_destroy(cr_ctx *ctx);
+
+/* Switch the stream later calls enqueue on. */
+CR_API int cr_set_stream(cr_ctx *ctx, void *cuda_stream);
+
+/* Blocking: wait for the context's stream, then report any error a kernel
+ * recorded since the last blocking call (CR_EOVERFLOW, CR_ETIMEOUT) and
+ * clear it. */
+CR_API int cr_sync(cr_ctx *ctx);
+
+/* Message for the last failing call on this context (static storage; never
+ * NULL).  A NULL ctx gives the message of the last failed cr_create. */
+CR_API const char *cr_last_error(const cr_ctx *ctx);
+
+/* Number of kernel launches this context has issued since it was created. */
+CR_API uint64_t cr_launch_count(const cr_ctx *ctx);
+
+/* ==== a1: prefix-span routing key ==================================== */
+/*
+ * The paper routes on an opaque business key b, which it allows to be salted
+ * (sec. 3.1; supplement, data handling), and defines no hash.  This library
+ * derives b from the request's reusable prefix span:
+ *
+ *   b = fmix64(salt ^ P) + sum_{i < ceil(P/2)} fmix64(w_i ^ (salt + (i+1)*G))  (mod 2^64)
+ *
+ * with fmix64 the SplitMix64 finaliser, G = 0x9e3779b97f4a7c15, and
+ * w_i = (uint32)t[2i] | (uint32)t[2i+1] << 32 the i-th pair of prefix tokens
+ * (t[P] reads as 0 when P is odd).  Only the P prefix tokens are read.
+ *
+ *   d_tokens  int32 token arena (any layout: records may overlap or be padded)
+ *   d_off     uint64[n] token index of request r's first prefix token
+ *   d_plen    uint32[n] prefix length P_r in tokens (0 allowed)
+ *   n         number of requests (0 allowed: nothing is enqueued)
+ *   salt      64-bit salt
+ *   d_key_out uint64[n] receives b_r
+ * Requests whose prefix starts on a 16-byte boundary (d_off[r] % 4 == 0) take
+ * the vectorised path; any other offset is still exact, only slower.
+ * Errors: CR_EINVAL (NULL pointer with n > 0). */
+CR_API int cr_hash_prefixes(cr_ctx *ctx, const int32_t *d_tokens, const uint64_t *d_off,
+                     const uint32_t *d_plen, uint64_t n, uint64_t salt, uint64_t *d_key_out);
+
+/* ==== a2..a6: the plan (Eq. 1, Algorithm 1) ========================== */
+
+typedef struct {
+    uint32_t R;               /* destinations, 1..CR_MAX_R                          */
+    uint32_t W;               /* warm slots per destination; C = R*W (sec. 3.1)     */
+    uint64_t qcap_num;        /* q_cap = qcap_num / qcap_den requests per interval  */
+    uint64_t qcap_den;        /*   (den < 2^32, num >= 1)                            */
+    uint32_t variant;         /* CR_VARIANT_*                                        */
+    uint32_t reserved;        /* must be 0                                           */
+    uint64_t seed;            /* CR_VARIANT_RANDOM: placement stream                 */
+    uint64_t epoch;           /* CR_VARIANT_RANDOM: e.g. the interval index          */
+    const uint64_t *d_init_load; /* uint64[R] starting loads, or NULL for the
+                                    cold-tail share floor(cold requests / R)        */
+} cr_plan_params;
+
+/* Create an empty plan owned by the library (device buffers grow on demand). */
+CR_API int cr_plan_create(cr_ctx *ctx, cr_plan **out);
+/* Destroy a plan (waits for the context's stream).  NULL is accepted. */
+CR_API int cr_plan_destroy(cr_ctx *ctx, cr_plan *plan);
+
+/*
+ * Build n_plans plans from the same interval's keys d_key[n] (uint64, any
+ * order, device).  One per-key histogram (lambda_b = number of requests with
+ * key b) is shared by all of them; plan j follows params[j]:
+ *   k_b   = min(R, max(1, ceil(lambda_b * den / num)))    (Eq. 1; 1 for NOREPL)
+ *   order = keys by (lambda_b descending, b ascending)
+ *   admit the longest prefix of that order with sum k_b <= C = R*W
+ *          (Algorithm 1 admission step: stop at the first key that does not fit)
+ *   L[r]  = d_init_load[r], or floor(sum of unadmitted lambda_b / R)
+ *   LPT:    for each admitted b in order, T(b) = the k_b smallest (L[r], r),
+ *           in that order; lambda_b is split into k_b integer jobs
+ *           floor(lambda_b/k_b) (+1 for the first lambda_b mod k_b members),
+ *           added to L (Algorithm 1 placement loop).
+ *   RANDOM: T(b) = first k_b steps of a Fisher-Yates shuffle of 0..R-1 driven
+ *           by Philox4x64-10(key = (seed, 1), counter = (a, s, 1, epoch)),
+ *           a = admission position, s = step (sec. 5.2, Table 4 "+replication").
+ * The table T is then installed as a device hash table for cr_route_batch.
+ * plans[j] must be distinct objects from cr_plan_create; any previous content
+ * is replaced.  Blocking: no.  Errors: CR_EINVAL (n >= 2^32, bad params,
+ * NULL pointers), CR_ENOMEM, CR_ECUDA; CR_EOVERFLOW is reported by the next
+ * blocking call if a load L[r] reaches 2^47. */
+CR_API int cr_build_plans(cr_ctx *ctx, const uint64_t *d_key, uint64_t n, const cr_plan_params *params,
+                   uint32_t n_plans, cr_plan *const *plans);
+
+/* cr_build_plans with one plan. */
+CR_API int cr_build_plan(cr_ctx *ctx, const uint64_t *d_key, uint64_t n, const cr_plan_params *params,
+                  cr_plan *plan);
+
+typedef struct {
+    uint64_t n;      /* requests the plan was built from                     */
+    uint64_t U;      /* distinct keys                                         */
+    uint64_t n_adm;  /* admitted keys                                         */
+    uint64_t sum_k;  /* sum of k_b over admitted keys (<= C)                  */
+    uint64_t cold;   /* requests of unadmitted keys                           */
+    uint64_t max_k;  /* largest k_b among admitted keys (0 if none)           */
+    uint32_t R, W;
+} cr_plan_info;
+
+/* Blocking: plan sizes.  Errors as cr_sync. */
+CR_API int cr_plan_get_info(cr_ctx *ctx, const cr_plan *plan, cr_plan_info *out);
+
+/* Blocking: copy a plan to HOST arrays (any may be NULL to skip it), sized
+ * from cr_plan_get_info:
+ *   ukey[U], ucnt[U]           histogram, keys ascending
+ *   adm_key[n_adm], adm_cnt[n_adm], adm_k[n_adm]   admission order
+ *   koff[n_adm+1]              member offsets
+ *   members[sum_k] (uint16), jobs[sum_k]           T(b) and its expected loads
+ *   load[R]                    final L */
+CR_API int cr_plan_export(cr_ctx *ctx, const cr_plan *plan, uint64_t *ukey, uint64_t *ucnt,
+                   uint64_t *adm_key, uint64_t *adm_cnt, uint32_t *adm_k, uint32_t *koff,
+                   uint16_t *members, uint64_t *jobs, uint64_t *load);
+
+/* ==== a7: batched dispatch ========================================== */
+
+typedef struct {
+    uint32_t policy;  /* CR_POLICY_* */
+    uint32_t reserved;/* must be 0 */
+    uint64_t seed;    /* RNG / offset / hash seed of this replica */
+} cr_replica;
+
+/*
+ * Route requests d_key[n] (device, arrival order, global request indices
+ * first_req_index .. first_req_index+n-1) for n_rep replicas at once.
+ *   plans[i]  plan used by replica i (CACHEROUTE, CR_NOLPT, CR_NOREPL), or
+ *             NULL for P2C, RR and HASH.  Plans may be shared; plan R must
+ *             equal R.
+ *   reps[i]   policy and seed (host array)
+ *   batch_B   requests are taken in batches of batch_B (>= 1); every request
+ *             of a batch sees the load vector as it stood when the batch
+ *             began; the batch's requests are added to it afterwards.
+ *             batch_B = 1 is exact sequential dispatch.
+ *   d_load    uint64[n_rep][R] live load, in/out (pass zeros at the start of
+ *             an interval to count requests routed in the interval)
+ *   d_dest    uint16[n_rep][n] receives the destination of every request
+ * Rules (Fig. 1 and sec. 3.1; comparison policies of sec. 4):
+ *   CACHEROUTE-type: b in T -> member of T(b) with the smallest
+ *     (load, position in T(b)); otherwise P2C with the replica's policy id.
+ *   P2C: u = Philox4x64-10(key = (seed, policy), counter = (g, 0, 0, 0)),
+ *     d1 = floor(u0 R / 2^64), d2 = (d1 + 1 + floor(u1 (R-1) / 2^64)) mod R;
+ *     pick d1 if load[d1] <= load[d2], else d2.
+ *   RR: (g + seed) mod R.     HASH: jump_hash(fmix64(b ^ seed), R).
+ * Errors: CR_EINVAL (R == 0 or > CR_MAX_R, n_rep > CR_MAX_REPLICAS, missing
+ * or mismatched plan, batch_B == 0, n >= 2^40). */
+CR_API int cr_route_batch(cr_ctx *ctx, const cr_plan *const *plans, const cr_replica *reps,
+                   uint32_t n_rep, uint32_t R, const uint64_t *d_key, uint64_t n,
+                   uint64_t first_req_index, uint32_t batch_B, uint64_t *d_load,
+                   uint16_t *d_dest);
+
+/* ==== a8, a9: shadow replay ========================================= */
+
+/* Create replay state for n_rep replicas x R destinations x n_caps LRU
+ * capacities (caps[] host array, each 1..CR_MAX_CAP, n_caps <= CR_MAX_CAPS).
+ * Every simulator starts empty.  Errors: CR_EINVAL, CR_ENOMEM. */
+CR_API int cr_replay_create(cr_ctx *ctx, uint32_t n_rep, uint32_t R, const uint32_t *caps,
+                     uint32_t n_caps, cr_replay **out);
+/* Empty every simulator (enqueued on the stream). */
+CR_API int cr_replay_reset(cr_ctx *ctx, cr_replay *rp);
+/* Destroy (waits for the stream).  NULL is accepted. */
+CR_API int cr_replay_destroy(cr_ctx *ctx, cr_replay *rp);
+
+/*
+ * Replay n routed requests through every simulator.  For replica i the
+ * requests with d_dest[i*n + j] == r reach destination r's caches in
+ * arrival order; each (replica, capacity, destination) is a whole-prefix LRU
+ * of `cap` entries keyed by the routing key (this library's model of the
+ * engine-native prefix cache that admitted and cold-tail traffic share,
+ * sec. 3.2).  A request hits when its key is resident: it then becomes most
+ * recent and its P prefix tokens are hit tokens; otherwise it is inserted as
+ * most recent and, when the cache is full, the least recent entry leaves.
+ * State persists across calls (and plan changes) until cr_replay_reset.
+ *   d_key uint64[n], d_plen uint32[n], d_slen uint32[n]: per request
+ *   d_dest uint16[n_rep][n]: destinations (each < R, checked on device)
+ *   d_ctr  uint64[n_rep][n_caps][R][5], ACCUMULATED (+=): requests, hit
+ *          requests, hit tokens, prompt tokens (P+S), prefill tokens
+ *          (prompt - hit tokens)
+ * Errors: CR_EINVAL (NULL pointers with n > 0, n >= 2^31); a destination
+ * >= R is skipped and reported as CR_EINVAL by the next blocking call. */
+CR_API int cr_shadow_replay(cr_ctx *ctx, cr_replay *rp, const uint64_t *d_key, const uint32_t *d_plen,
+                     const uint32_t *d_slen, const uint16_t *d_dest, uint64_t n,
+                     uint64_t *d_ctr);
+
+/* Blocking: resident keys of one simulator at the largest capacity, most
+ * recent first, into keys_out[CR_MAX_CAP] (host); *fill_out = their count.
+ * The state at a smaller capacity c is the first min(c, fill) of them. */
+CR_API int cr_replay_export_state(cr_ctx *ctx, const cr_replay *rp, uint32_t rep, uint32_t r,
+                           uint64_t *keys_out, uint32_t *fill_out);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* CACHEROUTE_H */

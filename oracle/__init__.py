@@ -5,7 +5,7 @@ CPU-baseline leg of ``bench.py`` may import this package; the library under
 ``paper_2608_19677_gb300`` never does.  The C source ``cr_oracle.c`` is a plain,
 slow, single-threaded restatement of the paper's Eq. 1 and Algorithm 1, of its
 dispatch rule (Fig. 1, sec. 3.1) and of the whole-prefix LRU replay this
-library adopts for the shadow-replay gate (sec. 5).  It shares no code with
+library adopts for the shadow-replay gate (sec. 3.2, 5.3).  It shares no code with
 the CUDA path.
 
 Parity status per function (what pins it; see tests/test_oracle_*.py):

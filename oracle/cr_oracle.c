@@ -28,7 +28,7 @@
  *       comparison policies of sec. 4 (Flat-LB, sticky hashing) plus
  *       round-robin.
  *   orc_replay_* ..................... shadow replay of each destination's
- *       prefix cache as a whole-prefix LRU (sec. 5 deployment gate; the paper
+ *       prefix cache as a whole-prefix LRU (deployment gate of sec. 3.2 and 5.3; the paper
  *       replays on hardware, the LRU model is this library's reading).
  */
 #include <stdint.h>

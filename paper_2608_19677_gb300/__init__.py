@@ -1,0 +1,318 @@
+"""GB300 (sm_103a) hot path of planned prefix-affinity routing (CacheRoute, arXiv 2608.19677).
+
+Thin ctypes binding over the C ABI declared in ``include/cacheroute.h``: every
+function below only marshals torch CUDA tensors into device pointers and calls
+the library of the same name; every step of the path runs in the library's
+CUDA kernels.  There is no CPU fallback: importing works without a GPU, but
+creating a ``Context`` requires the compiled library and a CUDA device, and
+fails loudly otherwise.
+
+  hash_prefixes   request prefix spans -> routing keys          (cr_hash_prefixes)
+  build_plans     one interval's keys -> plans (Eq. 1, Alg. 1)  (cr_build_plans)
+  route_batch     keys -> destination per (request, replica)    (cr_route_batch)
+  shadow_replay   routed requests -> LRU hit / load counters    (cr_shadow_replay)
+"""
+from __future__ import annotations
+
+import ctypes as C
+import os
+from typing import List, Optional, Sequence
+
+import numpy as np
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_HERE, "libcacheroute.so")
+
+CR_OK, CR_EINVAL, CR_ENOMEM, CR_ECUDA, CR_ETIMEOUT, CR_EOVERFLOW = range(6)
+STATUS_NAMES = {0: "CR_OK", 1: "CR_EINVAL", 2: "CR_ENOMEM", 3: "CR_ECUDA", 4: "CR_ETIMEOUT",
+                5: "CR_EOVERFLOW"}
+POLICY = {"CR": 0, "CR_NOLPT": 1, "CR_NOREPL": 2, "P2C": 3, "RR": 4, "HASH": 5}
+VARIANT = {"LPT": 0, "RANDOM": 1, "NOREPL": 2}
+MAX_R, MAX_CAP, MAX_CAPS, MAX_REPLICAS, CTR_FIELDS = 8192, 1024, 8, 256, 5
+
+# every symbol the header declares (checked by the CPU test suite)
+EXPORTS = ("cr_create", "cr_destroy", "cr_set_stream", "cr_sync", "cr_last_error", "cr_launch_count",
+           "cr_hash_prefixes", "cr_plan_create", "cr_plan_destroy", "cr_build_plans", "cr_build_plan",
+           "cr_plan_get_info", "cr_plan_export", "cr_route_batch", "cr_replay_create", "cr_replay_reset",
+           "cr_replay_destroy", "cr_shadow_replay", "cr_replay_export_state")
+
+
+class CacheRouteError(RuntimeError):
+    def __init__(self, code: int, where: str, msg: str):
+        super().__init__(f"{where}: {STATUS_NAMES.get(code, code)}: {msg}")
+        self.code = code
+
+
+class PlanParams(C.Structure):
+    _fields_ = [("R", C.c_uint32), ("W", C.c_uint32), ("qcap_num", C.c_uint64),
+                ("qcap_den", C.c_uint64), ("variant", C.c_uint32), ("reserved", C.c_uint32),
+                ("seed", C.c_uint64), ("epoch", C.c_uint64), ("d_init_load", C.c_void_p)]
+
+
+class PlanInfo(C.Structure):
+    _fields_ = [("n", C.c_uint64), ("U", C.c_uint64), ("n_adm", C.c_uint64), ("sum_k", C.c_uint64),
+                ("cold", C.c_uint64), ("max_k", C.c_uint64), ("R", C.c_uint32), ("W", C.c_uint32)]
+
+
+class Replica(C.Structure):
+    _fields_ = [("policy", C.c_uint32), ("reserved", C.c_uint32), ("seed", C.c_uint64)]
+
+
+_lib = None
+
+
+def build(force: bool = False) -> str:
+    """Compile the CUDA library in-tree (nvcc, sm_103a)."""
+    from . import buildlib
+    return buildlib.build(force=force)
+
+
+def lib() -> C.CDLL:
+    """The loaded CUDA library; raises if it has not been built."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    if not os.path.exists(LIB_PATH):
+        raise ImportError(f"{LIB_PATH} is missing: build the CUDA library first "
+                          f"(python -c 'import __graft_entry__ as g; g.build()')")
+    L = C.CDLL(LIB_PATH)
+    vp, u64, u32, i32 = C.c_void_p, C.c_uint64, C.c_uint32, C.c_int
+    sig = {
+        "cr_create": ([C.POINTER(vp), i32, vp], i32),
+        "cr_destroy": ([vp], i32),
+        "cr_set_stream": ([vp, vp], i32),
+        "cr_sync": ([vp], i32),
+        "cr_last_error": ([vp], C.c_char_p),
+        "cr_launch_count": ([vp], u64),
+        "cr_hash_prefixes": ([vp, vp, vp, vp, u64, u64, vp], i32),
+        "cr_plan_create": ([vp, C.POINTER(vp)], i32),
+        "cr_plan_destroy": ([vp, vp], i32),
+        "cr_build_plans": ([vp, vp, u64, C.POINTER(PlanParams), u32, C.POINTER(vp)], i32),
+        "cr_build_plan": ([vp, vp, u64, C.POINTER(PlanParams), vp], i32),
+        "cr_plan_get_info": ([vp, vp, C.POINTER(PlanInfo)], i32),
+        "cr_plan_export": ([vp, vp] + [vp] * 9, i32),
+        "cr_route_batch": ([vp, C.POINTER(vp), C.POINTER(Replica), u32, u32, vp, u64, u64, u32, vp, vp], i32),
+        "cr_replay_create": ([vp, u32, u32, C.POINTER(C.c_uint32), u32, C.POINTER(vp)], i32),
+        "cr_replay_reset": ([vp, vp], i32),
+        "cr_replay_destroy": ([vp, vp], i32),
+        "cr_shadow_replay": ([vp, vp, vp, vp, vp, vp, u64, vp], i32),
+        "cr_replay_export_state": ([vp, vp, u32, u32, vp, C.POINTER(C.c_uint32)], i32),
+    }
+    for name, (args, res) in sig.items():
+        f = getattr(L, name)
+        f.argtypes = args
+        f.restype = res
+    _lib = L
+    return L
+
+
+def _ptr(t) -> int:
+    return 0 if t is None else int(t.data_ptr())
+
+
+def _np_ptr(a: np.ndarray):
+    return a.ctypes.data_as(C.c_void_p)
+
+
+class Context:
+    """A library context bound to one CUDA device and stream (torch's current stream by default)."""
+
+    def __init__(self, device: int = 0, stream=None):
+        import torch
+        self.device = device
+        self._stream_obj = stream if stream is not None else torch.cuda.current_stream(device)
+        h = C.c_void_p()
+        st = lib().cr_create(C.byref(h), device, C.c_void_p(self._stream_obj.cuda_stream))
+        if st != CR_OK:
+            raise CacheRouteError(st, "cr_create", lib().cr_last_error(None).decode())
+        self._h = h
+
+    @property
+    def handle(self):
+        return self._h
+
+    def check(self, st: int, where: str):
+        if st != CR_OK:
+            raise CacheRouteError(st, where, lib().cr_last_error(self._h).decode())
+
+    def sync(self):
+        self.check(lib().cr_sync(self._h), "cr_sync")
+
+    def set_stream(self, stream):
+        self._stream_obj = stream
+        self.check(lib().cr_set_stream(self._h, C.c_void_p(stream.cuda_stream)), "cr_set_stream")
+
+    @property
+    def launches(self) -> int:
+        return int(lib().cr_launch_count(self._h))
+
+    def close(self):
+        if getattr(self, "_h", None):
+            lib().cr_destroy(self._h)
+            self._h = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+
+def _need_cuda(name, t, dtype=None):
+    if not t.is_cuda or not t.is_contiguous():
+        raise ValueError(f"{name} must be a contiguous CUDA tensor")
+    if dtype is not None and t.dtype != dtype:
+        raise ValueError(f"{name} must have dtype {dtype}, got {t.dtype}")
+
+
+def hash_prefixes(ctx: Context, tokens, off, plen, salt: int = 0, out=None):
+    """Routing key per request (uint64 values in an int64 tensor)."""
+    import torch
+    n = int(off.shape[0])
+    _need_cuda("tokens", tokens, torch.int32)
+    _need_cuda("off", off, torch.int64)
+    _need_cuda("plen", plen, torch.int32)
+    if out is None:
+        out = torch.empty(n, dtype=torch.int64, device=off.device)
+    ctx.check(lib().cr_hash_prefixes(ctx.handle, _ptr(tokens), _ptr(off), _ptr(plen), n,
+                                     salt & ((1 << 64) - 1), _ptr(out)), "cr_hash_prefixes")
+    return out
+
+
+class Plan:
+    """A library-owned plan (device resident)."""
+
+    def __init__(self, ctx: Context):
+        self.ctx = ctx
+        h = C.c_void_p()
+        ctx.check(lib().cr_plan_create(ctx.handle, C.byref(h)), "cr_plan_create")
+        self._h = h
+
+    @property
+    def handle(self):
+        return self._h
+
+    def info(self) -> PlanInfo:
+        inf = PlanInfo()
+        self.ctx.check(lib().cr_plan_get_info(self.ctx.handle, self._h, C.byref(inf)), "cr_plan_get_info")
+        return inf
+
+    def export(self) -> dict:
+        inf = self.info()
+        U, na, sk, R = int(inf.U), int(inf.n_adm), int(inf.sum_k), int(inf.R)
+        a = dict(ukey=np.zeros(max(U, 1), np.uint64), ucnt=np.zeros(max(U, 1), np.uint64),
+                 adm_key=np.zeros(max(na, 1), np.uint64), adm_cnt=np.zeros(max(na, 1), np.uint64),
+                 adm_k=np.zeros(max(na, 1), np.uint32), koff=np.zeros(na + 1, np.uint32),
+                 members=np.zeros(max(sk, 1), np.uint16), jobs=np.zeros(max(sk, 1), np.uint64),
+                 load=np.zeros(R, np.uint64))
+        self.ctx.check(lib().cr_plan_export(self.ctx.handle, self._h, *[_np_ptr(a[k]) for k in
+                                                                        ("ukey", "ucnt", "adm_key", "adm_cnt",
+                                                                         "adm_k", "koff", "members", "jobs",
+                                                                         "load")]), "cr_plan_export")
+        out = dict(U=U, n_adm=na, sum_k=sk, cold=int(inf.cold), max_k=int(inf.max_k), R=R, W=int(inf.W))
+        out.update(ukey=a["ukey"][:U], ucnt=a["ucnt"][:U], adm_key=a["adm_key"][:na], adm_cnt=a["adm_cnt"][:na],
+                   adm_k=a["adm_k"][:na], koff=a["koff"], members=a["members"][:sk], jobs=a["jobs"][:sk],
+                   load=a["load"])
+        return out
+
+    def close(self):
+        if getattr(self, "_h", None):
+            lib().cr_plan_destroy(self.ctx.handle, self._h)
+            self._h = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+
+def plan_params(R: int, W: int, qcap_num: int, qcap_den: int, variant="LPT", seed: int = 0, epoch: int = 0,
+                init_load=None) -> PlanParams:
+    v = VARIANT[variant] if isinstance(variant, str) else int(variant)
+    return PlanParams(R, W, qcap_num, qcap_den, v, 0, seed & ((1 << 64) - 1), epoch, _ptr(init_load))
+
+
+def build_plans(ctx: Context, keys, params: Sequence[PlanParams], plans: Sequence[Plan]):
+    import torch
+    n = int(keys.shape[0])
+    _need_cuda("keys", keys, torch.int64)
+    arr = (PlanParams * len(params))(*params)
+    hs = (C.c_void_p * len(plans))(*[p.handle for p in plans])
+    ctx.check(lib().cr_build_plans(ctx.handle, _ptr(keys), n, arr, len(params), hs), "cr_build_plans")
+    return plans
+
+
+def build_plan(ctx: Context, keys, params: PlanParams, plan: Optional[Plan] = None) -> Plan:
+    plan = plan or Plan(ctx)
+    build_plans(ctx, keys, [params], [plan])
+    return plan
+
+
+def route_batch(ctx: Context, plans: Sequence[Optional[Plan]], policies: Sequence, seeds: Sequence[int],
+                R: int, keys, first_req_index: int, batch_B: int, load, dest=None):
+    """Destinations (uint16 values in an int16 tensor [n_rep, n]); ``load`` [n_rep, R] is updated in place."""
+    import torch
+    n_rep = len(policies)
+    n = int(keys.shape[0])
+    _need_cuda("keys", keys, torch.int64)
+    _need_cuda("load", load, torch.int64)
+    if dest is None:
+        dest = torch.empty((n_rep, n), dtype=torch.int16, device=keys.device)
+    _need_cuda("dest", dest, torch.int16)
+    reps = (Replica * n_rep)(*[Replica(POLICY[p] if isinstance(p, str) else int(p), 0,
+                                       int(s) & ((1 << 64) - 1)) for p, s in zip(policies, seeds)])
+    hs = (C.c_void_p * n_rep)(*[(p.handle if p is not None else None) for p in plans])
+    ctx.check(lib().cr_route_batch(ctx.handle, hs, reps, n_rep, R, _ptr(keys), n, first_req_index, batch_B,
+                                   _ptr(load), _ptr(dest)), "cr_route_batch")
+    return dest
+
+
+class Replay:
+    """Library-owned LRU state for n_rep x R destinations x len(caps) capacities."""
+
+    def __init__(self, ctx: Context, n_rep: int, R: int, caps: Sequence[int]):
+        self.ctx, self.n_rep, self.R, self.caps = ctx, n_rep, R, list(caps)
+        cp = (C.c_uint32 * len(caps))(*caps)
+        h = C.c_void_p()
+        ctx.check(lib().cr_replay_create(ctx.handle, n_rep, R, cp, len(caps), C.byref(h)), "cr_replay_create")
+        self._h = h
+
+    @property
+    def handle(self):
+        return self._h
+
+    def reset(self):
+        self.ctx.check(lib().cr_replay_reset(self.ctx.handle, self._h), "cr_replay_reset")
+
+    def state(self, rep: int, r: int) -> np.ndarray:
+        out = np.zeros(MAX_CAP, np.uint64)
+        fill = C.c_uint32()
+        self.ctx.check(lib().cr_replay_export_state(self.ctx.handle, self._h, rep, r, _np_ptr(out),
+                                                    C.byref(fill)), "cr_replay_export_state")
+        return out[:fill.value].copy()
+
+    def close(self):
+        if getattr(self, "_h", None):
+            lib().cr_replay_destroy(self.ctx.handle, self._h)
+            self._h = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+
+def shadow_replay(ctx: Context, replay: Replay, keys, plen, slen, dest, ctr):
+    """Accumulate counters into ``ctr`` (int64 [n_rep, n_caps, R, 5])."""
+    import torch
+    n = int(keys.shape[0])
+    _need_cuda("keys", keys, torch.int64)
+    _need_cuda("plen", plen, torch.int32)
+    _need_cuda("slen", slen, torch.int32)
+    _need_cuda("dest", dest, torch.int16)
+    _need_cuda("ctr", ctr, torch.int64)
+    ctx.check(lib().cr_shadow_replay(ctx.handle, replay.handle, _ptr(keys), _ptr(plen), _ptr(slen), _ptr(dest),
+                                     n, _ptr(ctr)), "cr_shadow_replay")
+    return ctr

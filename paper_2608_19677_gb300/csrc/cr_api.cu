@@ -1,0 +1,127 @@
+// Context, scratch memory and status handling of the C ABI (include/cacheroute.h).
+#include <stdlib.h>
+#include <string.h>
+
+#include "cr_internal.cuh"
+
+static char g_create_msg[320] = "no error";
+
+int cr_fail(cr_ctx *ctx, int code, const char *fmt, ...)
+{
+    char *dst = ctx ? ctx->msg : g_create_msg;
+    va_list ap;
+    va_start(ap, fmt);
+    vsnprintf(dst, 320, fmt, ap);
+    va_end(ap);
+    return code;
+}
+
+int cr_check_launch(cr_ctx *ctx, const char *what)
+{
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess)
+        return cr_fail(ctx, CR_ECUDA, "launch of %s failed: %s", what, cudaGetErrorString(e));
+    return CR_OK;
+}
+
+int cr_scratch(cr_ctx *ctx, int slot, size_t bytes, void **out)
+{
+    if (bytes == 0) bytes = 16;
+    if (ctx->scratch_bytes[slot] < bytes) {
+        if (ctx->scratch[slot]) {
+            // the old buffer may still be read by enqueued work
+            cudaError_t e = cudaStreamSynchronize(ctx->stream);
+            if (e != cudaSuccess) return cr_fail(ctx, CR_ECUDA, "scratch sync: %s", cudaGetErrorString(e));
+            cudaFree(ctx->scratch[slot]);
+            ctx->scratch[slot] = NULL;
+            ctx->scratch_bytes[slot] = 0;
+        }
+        size_t grow = bytes + bytes / 4;
+        grow = (grow + 255) & ~(size_t)255;
+        void *p = NULL;
+        if (cudaMalloc(&p, grow) != cudaSuccess) {
+            cudaGetLastError();
+            return cr_fail(ctx, CR_ENOMEM, "scratch slot %d: cannot allocate %zu bytes", slot, grow);
+        }
+        ctx->scratch[slot] = p;
+        ctx->scratch_bytes[slot] = grow;
+    }
+    *out = ctx->scratch[slot];
+    return CR_OK;
+}
+
+extern "C" int cr_create(cr_ctx **out, int device, void *cuda_stream)
+{
+    if (!out) return cr_fail(NULL, CR_EINVAL, "cr_create: out is NULL");
+    *out = NULL;
+    int ndev = 0;
+    if (cudaGetDeviceCount(&ndev) != cudaSuccess || device < 0 || device >= ndev) {
+        cudaGetLastError();
+        return cr_fail(NULL, CR_EINVAL, "cr_create: device %d not available (%d devices)", device, ndev);
+    }
+    if (cudaSetDevice(device) != cudaSuccess) {
+        cudaGetLastError();
+        return cr_fail(NULL, CR_ECUDA, "cr_create: cudaSetDevice(%d) failed", device);
+    }
+    cr_ctx *c = (cr_ctx *)calloc(1, sizeof(cr_ctx));
+    if (!c) return cr_fail(NULL, CR_ENOMEM, "cr_create: host allocation failed");
+    c->device = device;
+    c->stream = (cudaStream_t)cuda_stream;
+    cudaDeviceGetAttribute(&c->num_sms, cudaDevAttrMultiProcessorCount, device);
+    if (c->num_sms <= 0) c->num_sms = 1;
+    if (cudaMalloc(&c->d_status, sizeof(uint32_t)) != cudaSuccess ||
+        cudaMemset(c->d_status, 0, sizeof(uint32_t)) != cudaSuccess) {
+        cudaGetLastError();
+        free(c);
+        return cr_fail(NULL, CR_ENOMEM, "cr_create: status word allocation failed");
+    }
+    strcpy(c->msg, "no error");
+    *out = c;
+    return CR_OK;
+}
+
+extern "C" int cr_destroy(cr_ctx *ctx)
+{
+    if (!ctx) return CR_OK;
+    cudaStreamSynchronize(ctx->stream);
+    for (int i = 0; i < SCR_NUM; ++i)
+        if (ctx->scratch[i]) cudaFree(ctx->scratch[i]);
+    cudaFree(ctx->d_status);
+    free(ctx);
+    return CR_OK;
+}
+
+extern "C" int cr_set_stream(cr_ctx *ctx, void *cuda_stream)
+{
+    if (!ctx) return CR_EINVAL;
+    ctx->stream = (cudaStream_t)cuda_stream;
+    return CR_OK;
+}
+
+extern "C" int cr_sync(cr_ctx *ctx)
+{
+    if (!ctx) return CR_EINVAL;
+    CR_CUDA(ctx, cudaStreamSynchronize(ctx->stream));
+    uint32_t flags = 0;
+    CR_CUDA(ctx, cudaMemcpy(&flags, ctx->d_status, sizeof(flags), cudaMemcpyDeviceToHost));
+    if (flags) {
+        CR_CUDA(ctx, cudaMemset(ctx->d_status, 0, sizeof(uint32_t)));
+        if (flags & CR_FLAG_BADDEST)
+            return cr_fail(ctx, CR_EINVAL, "a destination index >= R reached the replay (skipped)");
+        if (flags & CR_FLAG_OVERFLOW)
+            return cr_fail(ctx, CR_EOVERFLOW, "a load or counter exceeded its documented range");
+        if (flags & CR_FLAG_TIMEOUT)
+            return cr_fail(ctx, CR_ETIMEOUT, "a bounded device-side wait gave up");
+    }
+    return CR_OK;
+}
+
+extern "C" const char *cr_last_error(const cr_ctx *ctx)
+{
+    return ctx ? ctx->msg : g_create_msg;
+}
+
+extern "C" uint64_t cr_launch_count(const cr_ctx *ctx)
+{
+    return ctx ? ctx->launches : 0;
+}

@@ -1,0 +1,112 @@
+// a1: prefix-span routing key (cr_hash_prefixes).
+//
+// The key is the wrapping sum of one SplitMix64-mixed term per 64-bit word
+// (two int32 tokens) of the prefix plus a length term, so any partition of the
+// words over lanes gives the same result.  One warp hashes one request: lanes
+// stride over the span with 16-byte streaming loads (four tokens = two words
+// per load, four loads in flight per lane), then the warp reduces its partial
+// sums.  The path is an HBM stream of 4*P bytes per request; the per-word mix
+// (about two dozen integer instructions) keeps the ALU just under that stream
+// rate on sm_103a.
+#include "cr_device.cuh"
+#include "cr_internal.cuh"
+
+namespace {
+
+constexpr int kHashBlock = 256;
+
+__device__ __forceinline__ unsigned long long word_term(uint32_t lo, uint32_t hi, unsigned long long k)
+{
+    unsigned long long w = (unsigned long long)lo | ((unsigned long long)hi << 32);
+    return cr_fmix64(w ^ k);
+}
+
+// Words [first, nw) of a span starting at `base`, one per lane, scalar loads;
+// used for unaligned spans and for the last words of aligned ones.
+__device__ __forceinline__ unsigned long long scalar_words(const int32_t *__restrict__ base, uint32_t P,
+                                                           uint32_t first, uint32_t nw,
+                                                           unsigned long long salt, uint32_t lane)
+{
+    unsigned long long acc = 0;
+    for (uint32_t i = first + lane; i < nw; i += 32) {
+        uint32_t lo = (uint32_t)__ldcs(base + 2 * i);
+        uint32_t hi = (2 * i + 1 < P) ? (uint32_t)__ldcs(base + 2 * i + 1) : 0u;
+        acc += word_term(lo, hi, salt + (unsigned long long)(i + 1) * CR_GAMMA);
+    }
+    return acc;
+}
+
+__global__ void __launch_bounds__(kHashBlock)
+k_hash_prefixes(const int32_t *__restrict__ tok, const unsigned long long *__restrict__ off,
+                const uint32_t *__restrict__ plen, unsigned long long n, unsigned long long salt,
+                unsigned long long *__restrict__ out)
+{
+    const uint32_t lane = cr_lane();
+    const unsigned long long nwarps = ((unsigned long long)gridDim.x * blockDim.x) >> 5;
+    const unsigned long long G64 = 64ull * CR_GAMMA, G128 = 128ull * CR_GAMMA,
+                             G192 = 192ull * CR_GAMMA, G256 = 256ull * CR_GAMMA;
+    for (unsigned long long r = ((unsigned long long)blockIdx.x * blockDim.x + threadIdx.x) >> 5; r < n;
+         r += nwarps) {
+        const unsigned long long o = off[r];
+        const uint32_t P = plen[r];
+        const uint32_t nw = (P + 1) >> 1;
+        const int32_t *base = tok + o;
+        unsigned long long acc = 0;
+        if ((o & 3ull) == 0) {
+            // 16-byte aligned: vector v holds words 2v and 2v+1
+            const uint32_t nvec = P >> 2;
+            const int4 *b4 = reinterpret_cast<const int4 *>(base);
+            uint32_t v = lane;
+            unsigned long long k = salt + (unsigned long long)(2 * lane + 1) * CR_GAMMA;  // key of word 2v
+            for (; v + 96 < nvec; v += 128, k += G256) {
+                int4 a = __ldcs(b4 + v), b = __ldcs(b4 + v + 32), c = __ldcs(b4 + v + 64),
+                     d = __ldcs(b4 + v + 96);
+                acc += word_term(a.x, a.y, k) + word_term(a.z, a.w, k + CR_GAMMA);
+                acc += word_term(b.x, b.y, k + G64) + word_term(b.z, b.w, k + G64 + CR_GAMMA);
+                acc += word_term(c.x, c.y, k + G128) + word_term(c.z, c.w, k + G128 + CR_GAMMA);
+                acc += word_term(d.x, d.y, k + G192) + word_term(d.z, d.w, k + G192 + CR_GAMMA);
+            }
+            for (; v < nvec; v += 32, k += G64) {
+                int4 a = __ldcs(b4 + v);
+                acc += word_term(a.x, a.y, k) + word_term(a.z, a.w, k + CR_GAMMA);
+            }
+            acc += scalar_words(base, P, 2 * nvec, nw, salt, lane);
+        } else if ((o & 1ull) == 0) {
+            // 8-byte aligned: one word per load
+            const uint32_t nfull = P >> 1;
+            const uint2 *b2 = reinterpret_cast<const uint2 *>(base);
+            uint32_t i = lane;
+            unsigned long long k = salt + (unsigned long long)(lane + 1) * CR_GAMMA;
+            const unsigned long long G32 = 32ull * CR_GAMMA;
+            for (; i + 32 < nfull; i += 64, k += G64) {
+                uint2 a = __ldcs(b2 + i), b = __ldcs(b2 + i + 32);
+                acc += word_term(a.x, a.y, k) + word_term(b.x, b.y, k + G32);
+            }
+            for (; i < nfull; i += 32, k += G32) {
+                uint2 a = __ldcs(b2 + i);
+                acc += word_term(a.x, a.y, k);
+            }
+            acc += scalar_words(base, P, nfull, nw, salt, lane);
+        } else {
+            acc = scalar_words(base, P, 0, nw, salt, lane);
+        }
+        acc = cr_warp_sum_u64(acc);
+        if (lane == 0) out[r] = cr_fmix64(salt ^ (unsigned long long)P) + acc;
+    }
+}
+
+}  // namespace
+
+extern "C" int cr_hash_prefixes(cr_ctx *ctx, const int32_t *d_tokens, const uint64_t *d_off,
+                                const uint32_t *d_plen, uint64_t n, uint64_t salt, uint64_t *d_key_out)
+{
+    if (!ctx) return CR_EINVAL;
+    if (n == 0) return CR_OK;
+    if (!d_tokens || !d_off || !d_plen || !d_key_out)
+        return cr_fail(ctx, CR_EINVAL, "cr_hash_prefixes: NULL pointer");
+    const unsigned int warps_per_block = kHashBlock / 32;
+    unsigned int grid = cr_blocks(n, warps_per_block, (unsigned int)ctx->num_sms * 8u);
+    CR_LAUNCH(ctx, k_hash_prefixes, grid, kHashBlock, 0, d_tokens, (const unsigned long long *)d_off,
+              d_plen, (unsigned long long)n, (unsigned long long)salt, (unsigned long long *)d_key_out);
+    return CR_OK;
+}

@@ -1,0 +1,126 @@
+// Internal declarations of the CUDA library (not part of the public ABI).
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdarg.h>
+#include <stdint.h>
+#include <stdio.h>
+
+#include "cacheroute.h"
+
+// ---- device error flags (a bitmask in device memory, read by cr_sync) ------
+#define CR_FLAG_OVERFLOW 1u  // a load reached 2^47, or a stamp counter overflowed
+#define CR_FLAG_BADDEST 2u   // a destination index >= R reached the replay
+#define CR_FLAG_TIMEOUT 4u   // a bounded wait gave up
+
+// ---- scratch slots owned by the context ------------------------------------
+enum cr_scratch_slot {
+    SCR_SORT_K0 = 0,   // radix-sort keys (ping)
+    SCR_SORT_K1,       // radix-sort keys (pong)
+    SCR_SORT_V0,       // radix-sort values (ping)
+    SCR_SORT_V1,       // radix-sort values (pong)
+    SCR_SORT_HIST,     // per-tile digit counts / offsets
+    SCR_SCAN,          // block partials of the device-wide scan
+    SCR_PLAN_A,        // plan-build temporaries
+    SCR_PLAN_B,
+    SCR_PLAN_C,
+    SCR_REPLAY_IDX,    // partitioned request indices
+    SCR_REPLAY_START,  // per-stream start offsets
+    SCR_ROUTE_DESC,    // per-replica route descriptors
+    SCR_NUM
+};
+
+struct cr_ctx {
+    int device;
+    int num_sms;
+    cudaStream_t stream;
+    uint32_t *d_status;          // CR_FLAG_* bits
+    uint64_t launches;
+    void *scratch[SCR_NUM];
+    size_t scratch_bytes[SCR_NUM];
+    char msg[320];
+};
+
+// Plan: every array lives on the device; capacities are host-side upper bounds.
+struct cr_plan_info_dev {
+    unsigned long long n, U, n_adm, sum_k, cold, max_k;
+};
+
+struct cr_table_slot {               // 16 bytes: one sector-aligned probe
+    unsigned long long key;
+    uint32_t koff;                   // 0xffffffff = empty
+    uint16_t k;
+    uint16_t m0;                     // first member (the destination when k == 1)
+};
+
+struct cr_plan {
+    uint32_t R, W;
+    uint64_t cap_n;                  // capacity for histogram arrays (>= n)
+    uint64_t cap_adm;                // capacity for admitted arrays (>= min(n, C))
+    uint64_t cap_mem;                // capacity for member arrays (>= C)
+    uint64_t table_slots;            // power of two
+    uint64_t n;                      // requests of the last build (host copy)
+    unsigned long long *d_ukey, *d_ucnt;
+    unsigned long long *d_adm_key, *d_adm_cnt;
+    uint32_t *d_adm_k, *d_koff;
+    uint16_t *d_members;
+    unsigned long long *d_jobs, *d_load;
+    cr_table_slot *d_table;
+    cr_plan_info_dev *d_info;
+    int built;
+};
+
+struct cr_replay {
+    uint32_t n_rep, R, n_caps, cmax;
+    uint32_t caps[CR_MAX_CAPS];
+    uint64_t n_streams;              // n_rep * R
+    unsigned long long *d_keys;      // [stream][cmax], most recent first
+    uint32_t *d_fill;                // [stream]
+};
+
+// ---- host helpers (cr_api.cu) ----------------------------------------------
+int cr_fail(cr_ctx *ctx, int code, const char *fmt, ...);
+int cr_scratch(cr_ctx *ctx, int slot, size_t bytes, void **out);
+int cr_check_launch(cr_ctx *ctx, const char *what);
+
+#define CR_TRY(expr)                 \
+    do {                             \
+        int _st = (expr);            \
+        if (_st != CR_OK) return _st; \
+    } while (0)
+
+#define CR_CUDA(ctx, expr)                                                              \
+    do {                                                                                \
+        cudaError_t _e = (expr);                                                        \
+        if (_e != cudaSuccess)                                                          \
+            return cr_fail((ctx), CR_ECUDA, "%s: %s", #expr, cudaGetErrorString(_e));   \
+    } while (0)
+
+// Launch on the context's stream and account for it.
+#define CR_LAUNCH(ctx, kern, grid, block, smem, ...)                       \
+    do {                                                                   \
+        kern<<<(grid), (block), (smem), (ctx)->stream>>>(__VA_ARGS__);     \
+        (ctx)->launches++;                                                 \
+        CR_TRY(cr_check_launch((ctx), #kern));                             \
+    } while (0)
+
+static inline unsigned int cr_blocks(uint64_t work, unsigned int per_block, unsigned int cap)
+{
+    uint64_t b = (work + per_block - 1) / per_block;
+    if (b < 1) b = 1;
+    if (b > cap) b = cap;
+    return (unsigned int)b;
+}
+
+// ---- sort and scan primitives (cr_sort.cu) -----------------------------------
+// Stable LSD radix sort of keys (and optional u32 values) on bits [0, bits).
+// Input in (k_in, v_in); the sorted result is returned through *k_out/*v_out,
+// which point at either the input buffers or the context's ping-pong scratch.
+int cr_radix_sort_u64(cr_ctx *ctx, const unsigned long long *k_in, const uint32_t *v_in, uint64_t n,
+                      int bits, const unsigned long long **k_out, const uint32_t **v_out);
+int cr_radix_sort_u32(cr_ctx *ctx, const uint32_t *k_in, const uint32_t *v_in, uint64_t n, int bits,
+                      const uint32_t **k_out, const uint32_t **v_out);
+// Exclusive scan of u32 counts into u32 offsets (in place allowed); total to *d_total if non-null.
+int cr_scan_u32(cr_ctx *ctx, const uint32_t *in, uint32_t *out, uint64_t n, uint32_t *d_total);
+// Inclusive scan of u64 values.
+int cr_scan_u64_inclusive(cr_ctx *ctx, const unsigned long long *in, unsigned long long *out, uint64_t n);

@@ -1,0 +1,270 @@
+"""GPU parity: every CUDA kernel against the CPU oracle, element by element.
+
+All quantities are integers, so the bar is bit-exact equality.  Inputs are
+seeded synthetic traces (tracegen) or seeded random arrays; nothing the oracle
+sees comes from the CUDA path.
+"""
+import numpy as np
+import pytest
+
+torch = pytest.importorskip("torch")
+if not torch.cuda.is_available():
+    pytestmark = [pytest.mark.gpu, pytest.mark.skip(reason="needs a CUDA GPU")]
+else:
+    pytestmark = pytest.mark.gpu
+
+import oracle as O
+import oracle.pipeline as OP
+import tracegen as tg
+
+DEV = torch.device("cuda", 0)
+
+
+@pytest.fixture(scope="module")
+def P():
+    import __graft_entry__
+    __graft_entry__.build()
+    import paper_2608_19677_gb300 as P
+    return P
+
+
+@pytest.fixture(scope="module")
+def ctx(P):
+    c = P.Context(0)
+    yield c
+    c.close()
+
+
+def d_u64(a):
+    return torch.from_numpy(np.ascontiguousarray(a, np.uint64).view(np.int64)).to(DEV)
+
+
+def d_u32(a):
+    return torch.from_numpy(np.ascontiguousarray(a, np.uint32).view(np.int32)).to(DEV)
+
+
+def d_u16(a):
+    return torch.from_numpy(np.ascontiguousarray(a, np.uint16).view(np.int16)).to(DEV)
+
+
+def h_u64(t):
+    return t.cpu().numpy().view(np.uint64)
+
+
+def h_u16(t):
+    return t.cpu().numpy().view(np.uint16)
+
+
+# ------------------------------------------------------------------ a1 hash ---
+@pytest.mark.parametrize("align", [1, 2, 4])
+def test_hash_trace(P, ctx, align):
+    cfg = tg.CONFIGS["70b"].scaled(3000, 1)
+    tr = tg.Trace(cfg)
+    iv = tr.interval(0)
+    tok, off = tg.arena_host(tr, iv, align)
+    ref = O.hash_prefixes(tok, off, iv.plen, salt=12345)
+    got = P.hash_prefixes(ctx, torch.from_numpy(tok).to(DEV), d_u64(off), d_u32(iv.plen), salt=12345)
+    ctx.sync()
+    assert (h_u64(got) == ref).all()
+
+
+def test_hash_edge_lengths_and_offsets(P, ctx):
+    rng = np.random.default_rng(5)
+    lens = [0, 1, 2, 3, 4, 5, 7, 8, 9, 63, 64, 65, 127, 128, 129, 255, 256, 257, 511, 512, 513, 1023,
+            1024, 1025, 4095, 4096, 4097, 16383, 16384, 32768]
+    tok = rng.integers(-2**31, 2**31, size=200_000, dtype=np.int64).astype(np.int32)
+    offs, plens = [], []
+    for o0 in range(8):               # every alignment of the span start
+        for L in lens:
+            o = int(rng.integers(0, tok.size - L - 8)) // 8 * 8 + o0
+            offs.append(o)
+            plens.append(L)
+    offs = np.array(offs, np.uint64)
+    plens = np.array(plens, np.uint32)
+    ref = O.hash_prefixes(tok, offs, plens, salt=(1 << 64) - 3)
+    got = P.hash_prefixes(ctx, torch.from_numpy(tok).to(DEV), d_u64(offs), d_u32(plens), salt=(1 << 64) - 3)
+    ctx.sync()
+    assert (h_u64(got) == ref).all()
+
+
+def test_hash_empty(P, ctx):
+    t = torch.zeros(4, dtype=torch.int32, device=DEV)
+    out = P.hash_prefixes(ctx, t, torch.zeros(0, dtype=torch.int64, device=DEV),
+                          torch.zeros(0, dtype=torch.int32, device=DEV))
+    ctx.sync()
+    assert out.numel() == 0
+
+
+# ------------------------------------------------------------------ a2..a6 ---
+def _rates_keys(rng, nkeys, total, skew=1.2):
+    w = rng.pareto(skew, size=nkeys) + 1e-3
+    c = np.maximum(1, np.round(w / w.sum() * total)).astype(np.int64)
+    ks = rng.integers(0, 2**64, size=nkeys, dtype=np.uint64)
+    keys = np.repeat(ks, c)
+    rng.shuffle(keys)
+    return keys
+
+
+def _cmp_plan(got, ref):
+    assert got["U"] == ref.U
+    assert got["n_adm"] == ref.n_adm and got["sum_k"] == ref.sum_k and got["cold"] == ref.cold
+    assert (got["adm_key"] == ref.adm_key).all()
+    assert (got["adm_cnt"] == ref.adm_cnt).all()
+    assert (got["adm_k"] == ref.adm_k).all()
+    assert (got["koff"] == ref.koff).all()
+    assert (got["members"] == ref.members).all()
+    assert (got["jobs"] == ref.jobs).all()
+    assert (got["load"] == ref.load).all()
+
+
+@pytest.mark.parametrize("seed", range(8))
+def test_plan_parity(P, ctx, seed):
+    rng = np.random.default_rng(200 + seed)
+    R = int(rng.choice([1, 2, 3, 7, 30, 64, 100, 1024]))
+    W = int(rng.integers(1, 20))
+    nkeys = int(rng.integers(1, 5000))
+    keys = _rates_keys(rng, nkeys, int(rng.integers(nkeys, 60000)))
+    n = keys.size
+    num, den = (5 * n, 4 * R) if seed % 2 == 0 else (n, 9 * R)
+    plans = [P.Plan(ctx) for _ in range(3)]
+    params = [P.plan_params(R, W, num, den, v, seed=seed, epoch=3) for v in ("LPT", "RANDOM", "NOREPL")]
+    P.build_plans(ctx, d_u64(keys), params, plans)
+    uk, uc = O.histogram(keys)
+    for pl, v in zip(plans, ("LPT", "RANDOM", "NOREPL")):
+        got = pl.export()
+        assert (got["ukey"] == uk).all() and (got["ucnt"] == uc).all()
+        _cmp_plan(got, O.build_plan(keys, R, W, num, den, variant=v, seed=seed, epoch=3))
+
+
+def test_plan_hand_example_and_init_load(P, ctx):
+    keys = np.array([1] * 21 + [2] * 6 + [3] * 3 + [4], np.uint64)
+    pl = P.build_plan(ctx, d_u64(keys), P.plan_params(3, 1, 155, 12))
+    _cmp_plan(pl.export(), O.build_plan(keys, 3, 1, 155, 12))
+    init = np.array([9, 0, 4], np.uint64)
+    pl2 = P.build_plan(ctx, d_u64(keys), P.plan_params(3, 2, 1000, 1, init_load=d_u64(init)))
+    _cmp_plan(pl2.export(), O.build_plan(keys, 3, 2, 1000, 1, init_load=init))
+
+
+def test_plan_empty_and_single(P, ctx):
+    pl = P.build_plan(ctx, torch.zeros(0, dtype=torch.int64, device=DEV), P.plan_params(4, 2, 1, 1))
+    got = pl.export()
+    assert got["U"] == 0 and got["n_adm"] == 0 and (got["load"] == 0).all()
+    keys = np.array([7, 7, 7], np.uint64)
+    pl = P.build_plan(ctx, d_u64(keys), P.plan_params(5, 1, 1, 1))   # q_cap = 1: k = min(R, 3)
+    _cmp_plan(pl.export(), O.build_plan(keys, 5, 1, 1, 1))
+
+
+def test_plan_bad_params(P, ctx):
+    keys = d_u64(np.array([1, 2], np.uint64))
+    with pytest.raises(P.CacheRouteError):
+        P.build_plan(ctx, keys, P.plan_params(0, 1, 1, 1))
+    with pytest.raises(P.CacheRouteError):
+        P.build_plan(ctx, keys, P.plan_params(4, 1, 1, 0))
+    with pytest.raises(P.CacheRouteError):
+        P.build_plan(ctx, keys, P.plan_params(P.MAX_R + 1, 1, 1, 1))
+
+
+# ------------------------------------------------------------------ a7 route ---
+@pytest.mark.parametrize("R,B", [(1, 1), (3, 1), (7, 33), (30, 1024), (64, 5000), (1024, 256)])
+def test_route_parity(P, ctx, R, B):
+    rng = np.random.default_rng(R * 7 + B)
+    keys = _rates_keys(rng, 3000, 40000)
+    n = keys.size
+    pols = ["CR", "CR_NOLPT", "CR_NOREPL", "P2C", "RR", "HASH", "CR", "P2C"]
+    seeds = [0, 1, 0, 2, 3, 4, 9, 2**63 + 5]
+    num, den = n, 6 * R            # tight: replicated keys
+    W = 4
+    oplans = {v: O.build_plan(keys, R, W, num, den, variant=v, seed=s, epoch=1)
+              for v, s in (("LPT", 0), ("RANDOM", 1), ("NOREPL", 0))}
+    dplans = {}
+    for v, s in (("LPT", 0), ("RANDOM", 1), ("NOREPL", 0)):
+        dplans[v] = P.build_plan(ctx, d_u64(keys), P.plan_params(R, W, num, den, v, seed=s, epoch=1))
+    vmap = {"CR": "LPT", "CR_NOLPT": "RANDOM", "CR_NOREPL": "NOREPL"}
+    init = rng.integers(0, 50, size=(len(pols), R)).astype(np.uint64)
+    ref_dest, ref_load = O.route([oplans.get(vmap.get(p)) for p in pols], pols, seeds, R, keys, 777, B,
+                                 load=init)
+    load = d_u64(init.reshape(-1)).view(len(pols), R).contiguous()
+    dest = P.route_batch(ctx, [dplans.get(vmap.get(p)) for p in pols], pols, seeds, R, d_u64(keys), 777, B, load)
+    ctx.sync()
+    assert (h_u16(dest) == ref_dest).all()
+    assert (h_u64(load) == ref_load).all()
+
+
+def test_route_rejects_bad_args(P, ctx):
+    keys = d_u64(np.array([1, 2, 3], np.uint64))
+    load = torch.zeros((1, 4), dtype=torch.int64, device=DEV)
+    with pytest.raises(P.CacheRouteError):
+        P.route_batch(ctx, [None], ["CR"], [0], 4, keys, 0, 16, load)       # plan missing
+    with pytest.raises(P.CacheRouteError):
+        P.route_batch(ctx, [None], ["P2C"], [0], 4, keys, 0, 0, load)       # B = 0
+    with pytest.raises(P.CacheRouteError):
+        P.route_batch(ctx, [None], ["P2C"], [0], 0, keys, 0, 4, load)       # R = 0
+
+
+# ------------------------------------------------------------------ a8, a9 ---
+@pytest.mark.parametrize("caps", [[1], [2, 16], [12], [64, 256, 1024], [5, 33, 100], [1024]])
+def test_replay_parity(P, ctx, caps):
+    rng = np.random.default_rng(sum(caps))
+    n_rep, R = 3, 5
+    n = 20000
+    keys = _rates_keys(rng, int(rng.integers(20, 3000)), n)[:n]
+    n = keys.size
+    plen = rng.integers(16, 5000, size=n).astype(np.uint32)
+    slen = np.full(n, 64, np.uint32)
+    dest = tg.random_dest(n_rep, n, R, 3)
+    orp = O.Replay(n_rep, R, caps)
+    rp = P.Replay(ctx, n_rep, R, caps)
+    ctr = torch.zeros((n_rep, len(caps), R, 5), dtype=torch.int64, device=DEV)
+    dk, dp, ds, dd = d_u64(keys), d_u32(plen), d_u32(slen), d_u16(dest)
+    # two calls: state persists across them
+    cut = n // 3
+    for a, b in ((0, cut), (cut, n)):
+        orp.step(keys[a:b], plen[a:b], slen[a:b], dest[:, a:b])
+        P.shadow_replay(ctx, rp, dk[a:b].contiguous(), dp[a:b].contiguous(), ds[a:b].contiguous(),
+                        dd[:, a:b].contiguous(), ctr)
+        ctx.sync()
+        assert (h_u64(ctr) == orp.ctr).all()
+    cmax = max(caps)
+    for rep in range(n_rep):
+        for r in range(R):
+            st = rp.state(rep, r)
+            ci = caps.index(cmax)
+            assert (st == orp.state(rep, ci, r)).all()
+            for c_i, c in enumerate(caps):
+                assert (st[:c] == orp.state(rep, c_i, r)).all()
+
+
+def test_replay_reset_and_bad_dest(P, ctx):
+    rp = P.Replay(ctx, 1, 4, [8])
+    keys = d_u64(np.arange(10, dtype=np.uint64))
+    plen = d_u32(np.full(10, 5, np.uint32))
+    dest = d_u16(np.array([[0, 1, 2, 3, 0, 1, 2, 3, 0, 9]], np.uint16))   # 9 >= R
+    ctr = torch.zeros((1, 1, 4, 5), dtype=torch.int64, device=DEV)
+    P.shadow_replay(ctx, rp, keys, plen, plen, dest, ctr)
+    with pytest.raises(P.CacheRouteError):
+        ctx.sync()
+    assert int(ctr[..., 0].sum()) == 9
+    rp.reset()
+    ctx.sync()
+    assert rp.state(0, 0).size == 0
+
+
+# ------------------------------------------------------------------ pipeline ---
+@pytest.mark.parametrize("name,n,nint", [("tiny", 20000, 1), ("70b", 30000, 3), ("8b", 6000, 4),
+                                          ("burst", 30000, 2)])
+def test_pipeline_parity(P, ctx, name, n, nint):
+    from paper_2608_19677_gb300.pipeline import Pipeline
+    cfg = tg.CONFIGS[name]
+    if name != "tiny":
+        cfg = cfg.scaled(n, nint)
+    tr = tg.Trace(cfg)
+    ref = OP.run_trace(tr, B=1024, keep=True)
+    pipe = Pipeline(ctx, cfg.R, cfg.W, cfg.caps, cfg.replicas, tr.qcap, batch_B=1024)
+    for t in range(cfg.n_intervals):
+        iv = tr.interval(t)
+        tok, off = tg.arena_host(tr, iv, 4)
+        keys = pipe.interval(t, torch.from_numpy(tok).to(DEV), d_u64(off), d_u32(iv.plen), d_u32(iv.slen), iv.g0)
+        assert (h_u64(keys) == ref["keys"][t]).all()
+        assert (h_u16(pipe.last_dest) == ref["dest"][t]).all()
+    ctx.sync()
+    assert (h_u64(pipe.ctr) == ref["ctr"]).all()

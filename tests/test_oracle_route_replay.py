@@ -2,7 +2,7 @@
 
 Dispatch follows Fig. 1 and sec. 3.1 (least-loaded member of T(b), otherwise
 power-of-two choices); the replay is this library's whole-prefix LRU reading
-of the sec. 5 shadow-replay gate.  Pins use numpy's Philox (an independent
+of the shadow-replay gate (sec. 3.2, 5.3).  Pins use numpy's Philox (an independent
 implementation) to hand-step P2C, Lamping and Veach's monotonicity property of
 jump hashing, Mattson's stack-distance characterisation of LRU computed by
 brute force, and hand-worked traces.
