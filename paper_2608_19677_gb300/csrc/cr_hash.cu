@@ -4,8 +4,9 @@
 // (two int32 tokens) of the prefix plus a length term, so any partition of the
 // words over lanes gives the same result.  One warp hashes one request: lanes
 // stride over the span with 16-byte streaming loads (four tokens = two words
-// per load, four loads in flight per lane), then the warp reduces its partial
-// sums.  The path is an HBM stream of 4*P bytes per request; the per-word mix
+// per load, up to eight loads in flight per lane: the next group of four is
+// fetched while the current one is mixed), then the warp reduces its partial
+// sums; the next request's span descriptor is fetched a request ahead.  The path is an HBM stream of 4*P bytes per request; the per-word mix
 // (about two dozen integer instructions) keeps the ALU just under that stream
 // rate on sm_103a.
 #include "cr_device.cuh"
@@ -36,6 +37,18 @@ __device__ __forceinline__ unsigned long long scalar_words(const int32_t *__rest
     return acc;
 }
 
+__device__ __forceinline__ void load4(int4 (&x)[4], const int4 *__restrict__ b4, uint32_t v, uint32_t nvec)
+{
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+        const uint32_t i = v + 32u * q;
+        if (i < nvec)
+            x[q] = __ldcs(b4 + i);
+        else
+            x[q] = make_int4(0, 0, 0, 0);
+    }
+}
+
 __global__ void __launch_bounds__(kHashBlock)
 k_hash_prefixes(const int32_t *__restrict__ tok, const unsigned long long *__restrict__ off,
                 const uint32_t *__restrict__ plen, unsigned long long n, unsigned long long salt,
@@ -43,32 +56,48 @@ k_hash_prefixes(const int32_t *__restrict__ tok, const unsigned long long *__res
 {
     const uint32_t lane = cr_lane();
     const unsigned long long nwarps = ((unsigned long long)gridDim.x * blockDim.x) >> 5;
-    const unsigned long long G64 = 64ull * CR_GAMMA, G128 = 128ull * CR_GAMMA,
-                             G192 = 192ull * CR_GAMMA, G256 = 256ull * CR_GAMMA;
-    for (unsigned long long r = ((unsigned long long)blockIdx.x * blockDim.x + threadIdx.x) >> 5; r < n;
-         r += nwarps) {
-        const unsigned long long o = off[r];
-        const uint32_t P = plen[r];
+    const unsigned long long G64 = 64ull * CR_GAMMA, G256 = 256ull * CR_GAMMA;
+    unsigned long long r = ((unsigned long long)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+    unsigned long long o_next = 0;
+    uint32_t P_next = 0;
+    if (r < n) {
+        o_next = off[r];
+        P_next = plen[r];
+    }
+    for (; r < n; r += nwarps) {
+        const unsigned long long o = o_next;
+        const uint32_t P = P_next;
+        if (r + nwarps < n) {  // the next request's span descriptor is in flight meanwhile
+            o_next = off[r + nwarps];
+            P_next = plen[r + nwarps];
+        }
         const uint32_t nw = (P + 1) >> 1;
         const int32_t *base = tok + o;
         unsigned long long acc = 0;
         if ((o & 3ull) == 0) {
-            // 16-byte aligned: vector v holds words 2v and 2v+1
+            // 16-byte aligned: vector v holds words 2v and 2v+1.  Two groups of
+            // four vectors per lane are in flight: the next group loads while
+            // the current one is mixed.
             const uint32_t nvec = P >> 2;
             const int4 *b4 = reinterpret_cast<const int4 *>(base);
             uint32_t v = lane;
             unsigned long long k = salt + (unsigned long long)(2 * lane + 1) * CR_GAMMA;  // key of word 2v
-            for (; v + 96 < nvec; v += 128, k += G256) {
-                int4 a = __ldcs(b4 + v), b = __ldcs(b4 + v + 32), c = __ldcs(b4 + v + 64),
-                     d = __ldcs(b4 + v + 96);
-                acc += word_term(a.x, a.y, k) + word_term(a.z, a.w, k + CR_GAMMA);
-                acc += word_term(b.x, b.y, k + G64) + word_term(b.z, b.w, k + G64 + CR_GAMMA);
-                acc += word_term(c.x, c.y, k + G128) + word_term(c.z, c.w, k + G128 + CR_GAMMA);
-                acc += word_term(d.x, d.y, k + G192) + word_term(d.z, d.w, k + G192 + CR_GAMMA);
-            }
-            for (; v < nvec; v += 32, k += G64) {
-                int4 a = __ldcs(b4 + v);
-                acc += word_term(a.x, a.y, k) + word_term(a.z, a.w, k + CR_GAMMA);
+            int4 cur[4];
+            load4(cur, b4, v, nvec);
+            while (v < nvec) {
+                int4 nxt[4];
+                load4(nxt, b4, v + 128u, nvec);
+#pragma unroll
+                for (int q = 0; q < 4; ++q) {
+                    if (v + 32u * q < nvec) {
+                        const unsigned long long kq = k + (unsigned long long)q * G64;
+                        acc += word_term(cur[q].x, cur[q].y, kq) + word_term(cur[q].z, cur[q].w, kq + CR_GAMMA);
+                    }
+                }
+#pragma unroll
+                for (int q = 0; q < 4; ++q) cur[q] = nxt[q];
+                v += 128u;
+                k += G256;
             }
             acc += scalar_words(base, P, 2 * nvec, nw, salt, lane);
         } else if ((o & 1ull) == 0) {

@@ -26,6 +26,8 @@ enum cr_scratch_slot {
     SCR_PLAN_C,
     SCR_REPLAY_IDX,    // partitioned request indices
     SCR_REPLAY_START,  // per-stream start offsets
+    SCR_REPLAY_REC,    // gathered (key, prefix, suffix) records in stream order
+    SCR_REPLAY_CHUNK,  // per-stream chunk counts -> offsets, and their total
     SCR_ROUTE_DESC,    // per-replica route descriptors
     SCR_NUM
 };
@@ -74,8 +76,9 @@ struct cr_replay {
     uint32_t n_rep, R, n_caps, cmax;
     uint32_t caps[CR_MAX_CAPS];
     uint64_t n_streams;              // n_rep * R
-    unsigned long long *d_keys;      // [stream][cmax], most recent first
-    uint32_t *d_fill;                // [stream]
+    unsigned long long *d_keys[2];   // [stream][cmax], most recent first; double-buffered
+    uint32_t *d_fill[2];             // [stream]
+    int cur;                         // buffer holding the current state
 };
 
 // ---- host helpers (cr_api.cu) ----------------------------------------------

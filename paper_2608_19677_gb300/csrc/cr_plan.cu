@@ -187,10 +187,24 @@ __global__ void __launch_bounds__(32) k_plan_lpt(const cr_plan_info_dev *info,
     lane_min(L, taken, R, lane, mL, mr);
     const unsigned long long na = info->n_adm;
     bool overflow = false;
+    // the admitted keys' (lambda, k, offset) are staged 32 at a time, one per lane,
+    // and broadcast with shuffles: no global-memory latency on the sequential chain
+    unsigned long long st_lam = 0;
+    uint32_t st_k = 0, st_off = 0;
     for (unsigned long long a = 0; a < na; ++a) {
-        const uint32_t k = adm_k[a], base = koff[a];
-        const unsigned long long lam = adm_cnt[a];
-        const unsigned long long q = lam / k, rem = lam % k;
+        const uint32_t slot = (uint32_t)(a & 31ull);
+        if (slot == 0) {
+            const unsigned long long ia = a + lane;
+            if (ia < na) {
+                st_lam = adm_cnt[ia];
+                st_k = adm_k[ia];
+                st_off = koff[ia];
+            }
+        }
+        const uint32_t k = __shfl_sync(0xffffffffu, st_k, slot);
+        const uint32_t base = __shfl_sync(0xffffffffu, st_off, slot);
+        const unsigned long long lam = __shfl_sync(0xffffffffu, st_lam, slot);
+        const unsigned long long q = k == 1 ? lam : lam / k, rem = k == 1 ? 0ull : lam % k;
         for (uint32_t s = 0; s < k; ++s) {
             // warp argmin of (L, r) over the lanes' cached minima
             unsigned long long bL = mL;

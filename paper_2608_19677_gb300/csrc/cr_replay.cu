@@ -61,145 +61,267 @@ __global__ void k_stream_starts(const uint32_t *__restrict__ sk, unsigned long l
     }
 }
 
-template <int E>  // entries per lane: cmax <= 32 * E
-__global__ void k_lru_replay(const replay_caps caps, uint32_t cmax, uint32_t n_rep, uint32_t R,
-                             const uint32_t *__restrict__ start, const uint32_t *__restrict__ sval,
-                             unsigned long long n, const unsigned long long *__restrict__ keys,
-                             const uint32_t *__restrict__ plen, const uint32_t *__restrict__ slen,
-                             unsigned long long *__restrict__ st_keys, uint32_t *__restrict__ st_fill,
-                             unsigned long long *__restrict__ ctr, uint32_t *status)
+struct rec16 {
+    unsigned long long key;
+    uint32_t P, S;
+};
+
+// Gather each partitioned request's (key, prefix, suffix) into stream order.
+__global__ void k_gather_records(const uint32_t *__restrict__ sval, unsigned long long m, unsigned long long n,
+                                 const unsigned long long *__restrict__ keys, const uint32_t *__restrict__ plen,
+                                 const uint32_t *__restrict__ slen, rec16 *__restrict__ rec)
+{
+    for (unsigned long long pos = (unsigned long long)blockIdx.x * blockDim.x + threadIdx.x; pos < m;
+         pos += (unsigned long long)gridDim.x * blockDim.x) {
+        const unsigned long long j = sval[pos];
+        const unsigned long long i = j % n;
+        rec16 r;
+        r.key = keys[i];
+        r.P = plen[i];
+        r.S = slen[i];
+        rec[pos] = r;
+    }
+}
+
+// Chunks per stream (an empty stream still gets one work item that carries its state over).
+__global__ void k_chunk_counts(const uint32_t *__restrict__ start, uint32_t ns, uint32_t CL, uint32_t *__restrict__ nch)
+{
+    for (uint32_t s = blockIdx.x * blockDim.x + threadIdx.x; s < ns; s += gridDim.x * blockDim.x) {
+        const uint32_t len = start[s + 1] - start[s];
+        nch[s] = len ? (len + CL - 1) / CL : 1u;
+    }
+}
+
+struct replay_state {
+    const unsigned long long *keys_in;  // [stream][cmax], most recent first
+    const uint32_t *fill_in;
+    unsigned long long *keys_out;
+    uint32_t *fill_out;
+};
+
+// One warp per (stream, chunk).  The LRU state at the chunk's first request is
+// rebuilt by walking the stream backwards (and then the state carried in from
+// the previous call) collecting distinct keys, most recent first, until cmax
+// are found: those are exactly the resident entries of an LRU of capacity
+// cmax at that point.  The chunk is then simulated forwards.
+template <int E, int NC>  // NC: capacities counted (a compile-time bound on caps.n_caps)
+__global__ void __launch_bounds__(E == 1 ? 256 : 128, E == 1 ? 4 : 1)
+k_lru_chunks(const replay_caps caps, uint32_t cmax, uint32_t R, uint32_t ns, uint32_t CL,
+             const uint32_t *__restrict__ start, const uint32_t *__restrict__ coff, const uint32_t *__restrict__ total,
+             const rec16 *__restrict__ rec, const replay_state st, unsigned long long *__restrict__ ctr)
 {
     extern __shared__ unsigned long long sm[];
     const uint32_t lane = cr_lane(), warp = threadIdx.x >> 5, wpb = blockDim.x >> 5;
     const uint32_t slots = 32u * E;
-    unsigned long long *sk = sm + (size_t)warp * slots;                                     // keys
-    uint32_t *ss = reinterpret_cast<uint32_t *>(sm + (size_t)wpb * slots) + (size_t)warp * slots;  // stamps
-    const uint32_t stream = blockIdx.x * wpb + warp;
-    if (stream >= n_rep * R) return;
-    const uint32_t rep = stream / R, r = stream % R;
-    const uint32_t b = start[stream], e = start[stream + 1];
-    if (b == e) return;
-
-    // load state: rank q (0 = most recent) gets stamp fill - q
-    uint32_t fill = st_fill[stream];
-    const unsigned long long *gk = st_keys + (unsigned long long)stream * cmax;
-    for (uint32_t q = lane; q < fill; q += 32) {
-        sk[q] = gk[q];
-        ss[q] = fill - q;
+    unsigned long long *sk = sm + (size_t)warp * slots;
+    uint32_t *ss = reinterpret_cast<uint32_t *>(sm + (size_t)wpb * slots) + (size_t)warp * slots;
+    const uint32_t w = blockIdx.x * wpb + warp;
+    if (w >= *total) return;
+    // stream of this work item: the last s with coff[s] <= w
+    uint32_t lo = 0, hi = ns;
+    while (hi - lo > 1) {
+        uint32_t mid = (lo + hi) >> 1;
+        if (coff[mid] <= w)
+            lo = mid;
+        else
+            hi = mid;
     }
+    const uint32_t s = lo, ci = w - coff[s];
+    const uint32_t b = start[s], e = start[s + 1];
+    const uint32_t p0 = b + ci * CL;
+    const uint32_t p1 = (e - p0) < CL ? e : p0 + CL;
+    const uint32_t rep = s / R, r = s % R;
+    const uint32_t fill_in = st.fill_in[s];
+    const unsigned long long *kin = st.keys_in + (unsigned long long)s * cmax;
+    const uint32_t lt = (1u << lane) - 1u;
+
+    if (b == e) {  // nothing routed here: carry the state over unchanged
+        unsigned long long *kout = st.keys_out + (unsigned long long)s * cmax;
+        for (uint32_t q = lane; q < fill_in; q += 32) kout[q] = kin[q];
+        if (lane == 0) st.fill_out[s] = fill_in;
+        return;
+    }
+
+    // ---- state at p0 -------------------------------------------------------
+    uint32_t fill = 0;
+    if (ci == 0) {
+        for (uint32_t q = lane; q < fill_in; q += 32) sk[q] = kin[q];
+        fill = fill_in;
+    } else {
+        const uint32_t back = p0 - b;            // stream positions before the chunk
+        const uint32_t vtot = back + fill_in;    // then the carried-in state
+        for (uint32_t v0 = 0; v0 < vtot && fill < cmax; v0 += 32) {
+            const uint32_t v = v0 + lane;
+            const bool valid = v < vtot;
+            unsigned long long key = 0;
+            if (valid) key = v < back ? rec[p0 - 1 - v].key : kin[v - back];
+            const uint32_t peers = __match_any_sync(0xffffffffu, key);
+            bool fresh = valid && (peers & lt) == 0;
+            for (uint32_t q = 0; q < fill; ++q)
+                if (sk[q] == key) fresh = false;
+            const uint32_t bal = __ballot_sync(0xffffffffu, fresh);
+            const uint32_t rank = __popc(bal & lt);
+            __syncwarp();
+            if (fresh && fill + rank < cmax) sk[fill + rank] = key;
+            fill = min(cmax, fill + (uint32_t)__popc(bal));
+            __syncwarp();
+        }
+    }
+    for (uint32_t q = lane; q < fill; q += 32) ss[q] = fill - q;
     __syncwarp();
     uint32_t clock = fill;
 
-    unsigned long long c_req = 0, c_prompt = 0;
-    unsigned long long c_hit[CR_MAX_CAPS], c_hit_tok[CR_MAX_CAPS];
-#pragma unroll
-    for (int c = 0; c < CR_MAX_CAPS; ++c) c_hit[c] = c_hit_tok[c] = 0;
-    const unsigned long long rep_base = (unsigned long long)rep * n;
+    // register copy of the state when it fits one entry per lane
+    unsigned long long ek = 0;
+    uint32_t es = 0;
+    if (E == 1 && lane < fill) {
+        ek = sk[lane];
+        es = ss[lane];
+    }
 
-    for (uint32_t t0 = b; t0 < e; t0 += 32) {
-        // stage up to 32 requests of the stream, one per lane
-        unsigned long long mykey = 0;
-        uint32_t myP = 0, myS = 0;
-        if (t0 + lane < e) {
-            unsigned long long i = (unsigned long long)sval[t0 + lane] - rep_base;
-            mykey = keys[i];
-            myP = plen[i];
-            myS = slen[i];
+    unsigned long long my_req = 0, my_prompt = 0;
+    unsigned long long my_hit[NC], my_tok[NC];
+#pragma unroll
+    for (int c = 0; c < NC; ++c) my_hit[c] = my_tok[c] = 0;
+
+    for (uint32_t t0 = p0; t0 < p1; t0 += 32) {
+        rec16 mine_rec = {0ull, 0u, 0u};
+        if (t0 + lane < p1) {
+            mine_rec = rec[t0 + lane];
+            my_req += 1;
+            my_prompt += (unsigned long long)mine_rec.P + mine_rec.S;
         }
-        const uint32_t cnt = (e - t0) < 32u ? (e - t0) : 32u;
+        const uint32_t cnt = (p1 - t0) < 32u ? (p1 - t0) : 32u;
+        uint32_t my_depth = 0xffffffffu;  // lanes without a request never count a hit
         for (uint32_t j = 0; j < cnt; ++j) {
-            const unsigned long long key = __shfl_sync(0xffffffffu, mykey, j);
-            const uint32_t P = __shfl_sync(0xffffffffu, myP, j);
-            const uint32_t S = __shfl_sync(0xffffffffu, myS, j);
-            // lookup
-            int mine = -1;
-#pragma unroll
-            for (int x = 0; x < E; ++x) {
-                uint32_t idx = (uint32_t)x * 32u + lane;
-                if (idx < fill && sk[idx] == key) mine = (int)idx;
-            }
-            const uint32_t hb = __ballot_sync(0xffffffffu, mine >= 0);
-            uint32_t depth = 0xffffffffu;
+            const unsigned long long key = __shfl_sync(0xffffffffu, mine_rec.key, j);
             ++clock;
-            if (hb) {
-                const uint32_t hl = __ffs(hb) - 1;
-                const uint32_t hs = (uint32_t)__shfl_sync(0xffffffffu, mine, hl);
-                const uint32_t s_hit = ss[hs];
-                uint32_t newer = 0;
-#pragma unroll
-                for (int x = 0; x < E; ++x) {
-                    uint32_t idx = (uint32_t)x * 32u + lane;
-                    if (idx < fill && ss[idx] > s_hit) ++newer;
-                }
-                depth = 1u + __reduce_add_sync(0xffffffffu, newer);
-                __syncwarp();
-                if (lane == hl) ss[hs] = clock;
-            } else if (fill < cmax) {
-                if (lane == 0) {
-                    sk[fill] = key;
-                    ss[fill] = clock;
-                }
-                ++fill;
-            } else {
-                // evict the least recent entry (stamps are unique)
-                uint32_t lmin = 0xffffffffu, lidx = 0;
-#pragma unroll
-                for (int x = 0; x < E; ++x) {
-                    uint32_t idx = (uint32_t)x * 32u + lane;
-                    if (idx < fill && ss[idx] < lmin) {
-                        lmin = ss[idx];
-                        lidx = idx;
+            uint32_t depth = 0xffffffffu;
+            if (E == 1) {
+                const bool have = lane < fill;
+                const uint32_t hb = __ballot_sync(0xffffffffu, have && ek == key);
+                if (hb) {
+                    const uint32_t hl = __ffs(hb) - 1;
+                    const uint32_t s_hit = __shfl_sync(0xffffffffu, es, hl);
+                    depth = 1u + __popc(__ballot_sync(0xffffffffu, have && es > s_hit));
+                    if (lane == hl) es = clock;
+                } else if (fill < cmax) {
+                    if (lane == fill) {
+                        ek = key;
+                        es = clock;
+                    }
+                    ++fill;
+                } else {
+                    const uint32_t mn = __reduce_min_sync(0xffffffffu, have ? es : 0xffffffffu);
+                    const uint32_t vl = __ffs(__ballot_sync(0xffffffffu, have && es == mn)) - 1;
+                    if (lane == vl) {
+                        ek = key;
+                        es = clock;
                     }
                 }
-                const uint32_t wmin = __reduce_min_sync(0xffffffffu, lmin);
-                const uint32_t vl = __ffs(__ballot_sync(0xffffffffu, lmin == wmin)) - 1;
-                const uint32_t vidx = __shfl_sync(0xffffffffu, lidx, vl);
+            } else {
+                int mine = -1;
+#pragma unroll
+                for (int x = 0; x < E; ++x) {
+                    const uint32_t idx = (uint32_t)x * 32u + lane;
+                    if (idx < fill && sk[idx] == key) mine = (int)idx;
+                }
+                const uint32_t hb = __ballot_sync(0xffffffffu, mine >= 0);
+                if (hb) {
+                    const uint32_t hl = __ffs(hb) - 1;
+                    const uint32_t hs = (uint32_t)__shfl_sync(0xffffffffu, mine, hl);
+                    const uint32_t s_hit = ss[hs];
+                    uint32_t newer = 0;
+#pragma unroll
+                    for (int x = 0; x < E; ++x) {
+                        const uint32_t idx = (uint32_t)x * 32u + lane;
+                        if (idx < fill && ss[idx] > s_hit) ++newer;
+                    }
+                    depth = 1u + __reduce_add_sync(0xffffffffu, newer);
+                    __syncwarp();
+                    if (lane == hl) ss[hs] = clock;
+                } else if (fill < cmax) {
+                    if (lane == 0) {
+                        sk[fill] = key;
+                        ss[fill] = clock;
+                    }
+                    ++fill;
+                } else {
+                    uint32_t lmin = 0xffffffffu, lidx = 0;
+#pragma unroll
+                    for (int x = 0; x < E; ++x) {
+                        const uint32_t idx = (uint32_t)x * 32u + lane;
+                        if (idx < fill && ss[idx] < lmin) {
+                            lmin = ss[idx];
+                            lidx = idx;
+                        }
+                    }
+                    const uint32_t wmin = __reduce_min_sync(0xffffffffu, lmin);
+                    const uint32_t vl = __ffs(__ballot_sync(0xffffffffu, lmin == wmin)) - 1;
+                    const uint32_t vidx = __shfl_sync(0xffffffffu, lidx, vl);
+                    __syncwarp();
+                    if (lane == 0) {
+                        sk[vidx] = key;
+                        ss[vidx] = clock;
+                    }
+                }
                 __syncwarp();
-                if (lane == 0) {
-                    sk[vidx] = key;
-                    ss[vidx] = clock;
-                }
             }
-            __syncwarp();
-            c_req += 1;
-            c_prompt += (unsigned long long)P + S;
+            // the lane that loaded request j keeps its depth
+            if (lane == j) my_depth = depth;
+        }
+        // counters of the group, each lane for its own request
 #pragma unroll
-            for (int c = 0; c < CR_MAX_CAPS; ++c) {
-                if (c < (int)caps.n_caps && depth <= caps.cap[c]) {
-                    c_hit[c] += 1;
-                    c_hit_tok[c] += P;
-                }
+        for (int c = 0; c < NC; ++c) {
+            if (c < (int)caps.n_caps && my_depth <= caps.cap[c]) {
+                my_hit[c] += 1;
+                my_tok[c] += mine_rec.P;
             }
         }
     }
-    if (clock < fill) atomicOr(status, CR_FLAG_OVERFLOW);  // stamp counter wrapped
 
-    // store state in recency order: rank = entries with a newer stamp
-    unsigned long long *gkw = st_keys + (unsigned long long)stream * cmax;
+    // ---- counters -------------------------------------------------------------
+    my_req = cr_warp_sum_u64(my_req);
+    my_prompt = cr_warp_sum_u64(my_prompt);
 #pragma unroll
-    for (int x = 0; x < E; ++x) {
-        uint32_t idx = (uint32_t)x * 32u + lane;
-        if (idx < fill) {
-            const uint32_t my = ss[idx];
-            uint32_t rank = 0;
-            for (uint32_t f = 0; f < fill; ++f) rank += (ss[f] > my) ? 1u : 0u;
-            gkw[rank] = sk[idx];
-        }
-    }
-    if (lane == 0) {
-        st_fill[stream] = fill;
-#pragma unroll
-        for (int c = 0; c < CR_MAX_CAPS; ++c) {
-            if (c < (int)caps.n_caps) {
-                unsigned long long *C =
-                    ctr + (((unsigned long long)rep * caps.n_caps + c) * R + r) * CR_CTR_FIELDS;
-                C[0] += c_req;
-                C[1] += c_hit[c];
-                C[2] += c_hit_tok[c];
-                C[3] += c_prompt;
-                C[4] += c_prompt - c_hit_tok[c];
+    for (int c = 0; c < NC; ++c) {
+        if (c < (int)caps.n_caps) {
+            const unsigned long long h = cr_warp_sum_u64(my_hit[c]);
+            const unsigned long long tk = cr_warp_sum_u64(my_tok[c]);
+            if (lane == 0) {
+                unsigned long long *C = ctr + (((unsigned long long)rep * caps.n_caps + c) * R + r) * CR_CTR_FIELDS;
+                atomicAdd(&C[0], my_req);
+                if (h) atomicAdd(&C[1], h);
+                if (tk) atomicAdd(&C[2], tk);
+                atomicAdd(&C[3], my_prompt);
+                atomicAdd(&C[4], my_prompt - tk);
             }
         }
+    }
+
+    // ---- the stream's last chunk hands the state to the next call ---------------
+    if (p1 == e) {
+        unsigned long long *kout = st.keys_out + (unsigned long long)s * cmax;
+        if (E == 1) {
+            uint32_t rank = 0;
+            for (uint32_t q = 0; q < 32; ++q) {
+                const uint32_t sq = __shfl_sync(0xffffffffu, es, q);
+                if (q < fill && sq > es) ++rank;
+            }
+            if (lane < fill) kout[rank] = ek;
+        } else {
+#pragma unroll
+            for (int x = 0; x < E; ++x) {
+                const uint32_t idx = (uint32_t)x * 32u + lane;
+                if (idx < fill) {
+                    const uint32_t my = ss[idx];
+                    uint32_t rank = 0;
+                    for (uint32_t f = 0; f < fill; ++f) rank += (ss[f] > my) ? 1u : 0u;
+                    kout[rank] = sk[idx];
+                }
+            }
+        }
+        if (lane == 0) st.fill_out[s] = fill;
     }
 }
 
@@ -210,19 +332,35 @@ int bits_for(uint64_t v)
     return b;
 }
 
-template <int E>
-int launch_replay(cr_ctx *ctx, cr_replay *rp, const replay_caps &caps, const uint32_t *start, const uint32_t *sval,
-                  uint64_t n, const uint64_t *d_key, const uint32_t *d_plen, const uint32_t *d_slen, uint64_t *d_ctr)
+template <int E, int NC>
+int launch_replay_nc(cr_ctx *ctx, cr_replay *rp, const replay_caps &caps, uint32_t CL, const uint32_t *start,
+                     const uint32_t *coff, const uint32_t *total, uint64_t m, const rec16 *rec, uint64_t *d_ctr)
 {
-    const uint32_t wpb = E >= 16 ? 4 : 8;
+    const uint32_t wpb = E == 1 ? 8 : 4;
     const size_t smem = (size_t)wpb * 32 * E * (sizeof(unsigned long long) + sizeof(uint32_t));
     if (smem > 48 * 1024)
-        CR_CUDA(ctx, cudaFuncSetAttribute(k_lru_replay<E>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
+        CR_CUDA(ctx, cudaFuncSetAttribute(k_lru_chunks<E, NC>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                          (int)smem));
     const uint32_t ns = rp->n_rep * rp->R;
-    CR_LAUNCH(ctx, k_lru_replay<E>, (ns + wpb - 1) / wpb, wpb * 32, smem, caps, rp->cmax, rp->n_rep, rp->R, start,
-              sval, (unsigned long long)n, (const unsigned long long *)d_key, d_plen, d_slen, rp->d_keys, rp->d_fill,
-              (unsigned long long *)d_ctr, ctx->d_status);
+    const uint64_t items = (uint64_t)ns + (m + CL - 1) / CL;  // upper bound on work items
+    replay_state st;
+    st.keys_in = rp->d_keys[rp->cur];
+    st.fill_in = rp->d_fill[rp->cur];
+    st.keys_out = rp->d_keys[rp->cur ^ 1];
+    st.fill_out = rp->d_fill[rp->cur ^ 1];
+    CR_LAUNCH(ctx, (k_lru_chunks<E, NC>), (unsigned int)((items + wpb - 1) / wpb), wpb * 32, smem, caps, rp->cmax,
+              rp->R, ns, CL, start, coff, total, rec, st, (unsigned long long *)d_ctr);
+    rp->cur ^= 1;
     return CR_OK;
+}
+
+template <int E>
+int launch_replay(cr_ctx *ctx, cr_replay *rp, const replay_caps &caps, uint32_t CL, const uint32_t *start,
+                  const uint32_t *coff, const uint32_t *total, uint64_t m, const rec16 *rec, uint64_t *d_ctr)
+{
+    if (caps.n_caps == 1) return launch_replay_nc<E, 1>(ctx, rp, caps, CL, start, coff, total, m, rec, d_ctr);
+    if (caps.n_caps <= 3) return launch_replay_nc<E, 3>(ctx, rp, caps, CL, start, coff, total, m, rec, d_ctr);
+    return launch_replay_nc<E, CR_MAX_CAPS>(ctx, rp, caps, CL, start, coff, total, m, rec, d_ctr);
 }
 
 }  // namespace
@@ -249,12 +387,17 @@ extern "C" int cr_replay_create(cr_ctx *ctx, uint32_t n_rep, uint32_t R, const u
     rp->cmax = cmax;
     memcpy(rp->caps, caps, n_caps * sizeof(uint32_t));
     rp->n_streams = (uint64_t)n_rep * R;
-    if (cudaMalloc(&rp->d_keys, rp->n_streams * cmax * sizeof(unsigned long long)) != cudaSuccess ||
-        cudaMalloc(&rp->d_fill, rp->n_streams * sizeof(uint32_t)) != cudaSuccess) {
-        cudaGetLastError();
-        if (rp->d_keys) cudaFree(rp->d_keys);
-        free(rp);
-        return cr_fail(ctx, CR_ENOMEM, "replay: cannot allocate state");
+    for (int b = 0; b < 2; ++b) {
+        if (cudaMalloc(&rp->d_keys[b], rp->n_streams * cmax * sizeof(unsigned long long)) != cudaSuccess ||
+            cudaMalloc(&rp->d_fill[b], rp->n_streams * sizeof(uint32_t)) != cudaSuccess) {
+            cudaGetLastError();
+            for (int x = 0; x < 2; ++x) {
+                if (rp->d_keys[x]) cudaFree(rp->d_keys[x]);
+                if (rp->d_fill[x]) cudaFree(rp->d_fill[x]);
+            }
+            free(rp);
+            return cr_fail(ctx, CR_ENOMEM, "replay: cannot allocate state");
+        }
     }
     *out = rp;
     return cr_replay_reset(ctx, rp);
@@ -263,7 +406,8 @@ extern "C" int cr_replay_create(cr_ctx *ctx, uint32_t n_rep, uint32_t R, const u
 extern "C" int cr_replay_reset(cr_ctx *ctx, cr_replay *rp)
 {
     if (!ctx || !rp) return CR_EINVAL;
-    CR_CUDA(ctx, cudaMemsetAsync(rp->d_fill, 0, rp->n_streams * sizeof(uint32_t), ctx->stream));
+    for (int b = 0; b < 2; ++b)
+        CR_CUDA(ctx, cudaMemsetAsync(rp->d_fill[b], 0, rp->n_streams * sizeof(uint32_t), ctx->stream));
     return CR_OK;
 }
 
@@ -271,8 +415,10 @@ extern "C" int cr_replay_destroy(cr_ctx *ctx, cr_replay *rp)
 {
     if (!rp) return CR_OK;
     if (ctx) cudaStreamSynchronize(ctx->stream);
-    cudaFree(rp->d_keys);
-    cudaFree(rp->d_fill);
+    for (int b = 0; b < 2; ++b) {
+        cudaFree(rp->d_keys[b]);
+        cudaFree(rp->d_fill[b]);
+    }
     free(rp);
     return CR_OK;
 }
@@ -304,13 +450,25 @@ extern "C" int cr_shadow_replay(cr_ctx *ctx, cr_replay *rp, const uint64_t *d_ke
     replay_caps caps;
     caps.n_caps = rp->n_caps;
     for (uint32_t c = 0; c < CR_MAX_CAPS; ++c) caps.cap[c] = c < rp->n_caps ? rp->caps[c] : 0;
+    // chunk length: long enough that rebuilding an LRU state of cmax entries is amortised
+    const uint32_t CL = rp->cmax * 16u > 256u ? rp->cmax * 16u : 256u;
+    const uint32_t ns = (uint32_t)rp->n_streams;
+    void *prec, *pch;
+    CR_TRY(cr_scratch(ctx, SCR_REPLAY_REC, m * sizeof(rec16), &prec));
+    CR_TRY(cr_scratch(ctx, SCR_REPLAY_CHUNK, ((size_t)ns + 2) * sizeof(uint32_t), &pch));
+    rec16 *rec = (rec16 *)prec;
+    uint32_t *coff = (uint32_t *)pch, *total = coff + ns;
+    CR_LAUNCH(ctx, k_gather_records, cr_blocks(m, 256, gcap), 256, 0, sval, (unsigned long long)m,
+              (unsigned long long)n, (const unsigned long long *)d_key, d_plen, d_slen, rec);
+    CR_LAUNCH(ctx, k_chunk_counts, cr_blocks(ns, 256, gcap), 256, 0, (const uint32_t *)start, ns, CL, coff);
+    CR_TRY(cr_scan_u32(ctx, coff, coff, ns, total));
     const uint32_t E = (rp->cmax + 31) / 32;
-    if (E <= 1) return launch_replay<1>(ctx, rp, caps, start, sval, n, d_key, d_plen, d_slen, d_ctr);
-    if (E <= 2) return launch_replay<2>(ctx, rp, caps, start, sval, n, d_key, d_plen, d_slen, d_ctr);
-    if (E <= 4) return launch_replay<4>(ctx, rp, caps, start, sval, n, d_key, d_plen, d_slen, d_ctr);
-    if (E <= 8) return launch_replay<8>(ctx, rp, caps, start, sval, n, d_key, d_plen, d_slen, d_ctr);
-    if (E <= 16) return launch_replay<16>(ctx, rp, caps, start, sval, n, d_key, d_plen, d_slen, d_ctr);
-    return launch_replay<32>(ctx, rp, caps, start, sval, n, d_key, d_plen, d_slen, d_ctr);
+    if (E <= 1) return launch_replay<1>(ctx, rp, caps, CL, start, coff, total, m, rec, d_ctr);
+    if (E <= 2) return launch_replay<2>(ctx, rp, caps, CL, start, coff, total, m, rec, d_ctr);
+    if (E <= 4) return launch_replay<4>(ctx, rp, caps, CL, start, coff, total, m, rec, d_ctr);
+    if (E <= 8) return launch_replay<8>(ctx, rp, caps, CL, start, coff, total, m, rec, d_ctr);
+    if (E <= 16) return launch_replay<16>(ctx, rp, caps, CL, start, coff, total, m, rec, d_ctr);
+    return launch_replay<32>(ctx, rp, caps, CL, start, coff, total, m, rec, d_ctr);
 }
 
 extern "C" int cr_replay_export_state(cr_ctx *ctx, const cr_replay *rp, uint32_t rep, uint32_t r,
@@ -320,10 +478,11 @@ extern "C" int cr_replay_export_state(cr_ctx *ctx, const cr_replay *rp, uint32_t
     if (rep >= rp->n_rep || r >= rp->R) return cr_fail(ctx, CR_EINVAL, "export_state: bad stream");
     const uint64_t s = (uint64_t)rep * rp->R + r;
     uint32_t fill = 0;
-    CR_CUDA(ctx, cudaMemcpyAsync(&fill, rp->d_fill + s, sizeof(uint32_t), cudaMemcpyDeviceToHost, ctx->stream));
+    CR_CUDA(ctx, cudaMemcpyAsync(&fill, rp->d_fill[rp->cur] + s, sizeof(uint32_t), cudaMemcpyDeviceToHost,
+                                 ctx->stream));
     CR_TRY(cr_sync(ctx));
     if (fill)
-        CR_CUDA(ctx, cudaMemcpyAsync(keys_out, rp->d_keys + s * rp->cmax, fill * sizeof(uint64_t),
+        CR_CUDA(ctx, cudaMemcpyAsync(keys_out, rp->d_keys[rp->cur] + s * rp->cmax, fill * sizeof(uint64_t),
                                      cudaMemcpyDeviceToHost, ctx->stream));
     *fill_out = fill;
     return cr_sync(ctx);

@@ -68,24 +68,39 @@ class Pipeline:
         self.ctr.zero_()
         self.prev_keys = None
 
-    def interval(self, t: int, tokens, off, plen, slen, g0: int):
-        """Run one control interval on device tensors; returns the interval's keys."""
+    def interval(self, t: int, tokens, off, plen, slen, g0: int, marks=None):
+        """Run one control interval on device tensors; returns the interval's keys.
+
+        ``marks``: optional list of 5 torch.cuda.Event recorded on the context's
+        stream at the stage boundaries (start, hashed, planned, routed, replayed).
+        """
         n = int(off.shape[0])
+        stream = self.ctx._stream_obj
+        if marks is not None:
+            marks[0].record(stream)
         self._alloc(n)
         keys = self._keys[self._flip][:n]
         self._flip ^= 1
         hash_prefixes(self.ctx, tokens, off, plen, self.salt, out=keys)
+        if marks is not None:
+            marks[1].record(stream)
         pk = keys if self.prev_keys is None else self.prev_keys
         if self.plans:
             num, den = self.qcap(int(pk.shape[0]))
             params = [plan_params(self.R, self.W, num, den, v, seed=s, epoch=t) for v, s in self.plan_keys]
             build_plans(self.ctx, pk, params, self.plans)
+        if marks is not None:
+            marks[2].record(stream)
         self.load.zero_()
         dest = self._dest[:, :n] if n == self._dest.shape[1] else self._dest.view(-1)[:len(self.replicas) * n].view(
             len(self.replicas), n)
         plans = [self.plans[i] if i is not None else None for i in self.rep_plan]
         route_batch(self.ctx, plans, self.policies, self.seeds, self.R, keys, g0, self.B, self.load, dest)
+        if marks is not None:
+            marks[3].record(stream)
         shadow_replay(self.ctx, self.replay, keys, plen, slen, dest, self.ctr)
+        if marks is not None:
+            marks[4].record(stream)
         self.prev_keys = keys
         self.last_dest = dest
         return keys

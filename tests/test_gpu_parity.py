@@ -165,7 +165,8 @@ def test_plan_bad_params(P, ctx):
 
 
 # ------------------------------------------------------------------ a7 route ---
-@pytest.mark.parametrize("R,B", [(1, 1), (3, 1), (7, 33), (30, 1024), (64, 5000), (1024, 256)])
+@pytest.mark.parametrize("R,B", [(1, 1), (3, 1), (7, 33), (30, 1024), (64, 5000), (1024, 256), (30, 20000),
+                                 (5, 16384), (9, 16385)])
 def test_route_parity(P, ctx, R, B):
     rng = np.random.default_rng(R * 7 + B)
     keys = _rates_keys(rng, 3000, 40000)
