@@ -45,7 +45,7 @@ struct cr_ctx {
 
 // Plan: every array lives on the device; capacities are host-side upper bounds.
 struct cr_plan_info_dev {
-    unsigned long long n, U, n_adm, sum_k, cold, max_k;
+    unsigned long long n, U, n_adm, sum_k, cold, max_k, special;
 };
 
 struct cr_table_slot {               // 16 bytes: one sector-aligned probe

@@ -28,47 +28,251 @@ __global__ void k_plan_reset(cr_plan_info_dev *info, unsigned long long n)
     info->sum_k = 0;
     info->cold = 0;
     info->max_k = 0;
+    info->special = 0;
 }
 
-__global__ void k_rle_flags(const unsigned long long *__restrict__ s, uint64_t n, uint32_t *__restrict__ flag)
-{
-    for (uint64_t i = (uint64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (uint64_t)gridDim.x * blockDim.x)
-        flag[i] = (i == 0 || s[i] != s[i - 1]) ? 1u : 0u;
-}
+// ---- histogram: counts in an L2-resident open-addressing table ----------
+// Slots hold (key, count); an empty slot holds the key 2^64-1, so requests
+// whose key is 2^64-1 itself are counted apart in info->special.
+constexpr unsigned long long kEmptyKey = ~0ull;
 
-// pos = exclusive scan of flags; every run head writes its key and position.
-__global__ void k_rle_heads(const unsigned long long *__restrict__ s, const uint32_t *__restrict__ pos, uint64_t n,
-                            unsigned long long *__restrict__ ukey, uint32_t *__restrict__ head,
-                            cr_plan_info_dev *info)
+__global__ void k_hist_insert(const unsigned long long *__restrict__ keys, uint64_t n,
+                              unsigned long long *__restrict__ tkey, uint32_t *__restrict__ tcnt, int bits,
+                              cr_plan_info_dev *info)
 {
-    for (uint64_t i = (uint64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (uint64_t)gridDim.x * blockDim.x) {
-        bool h = (i == 0 || s[i] != s[i - 1]);
-        if (h) {
-            ukey[pos[i]] = s[i];
-            head[pos[i]] = (uint32_t)i;
+    const unsigned long long mask = (1ull << bits) - 1ull;
+    const uint32_t lane = cr_lane();
+    const uint32_t lt = (1u << lane) - 1u;
+    for (uint64_t base = ((uint64_t)blockIdx.x * blockDim.x + threadIdx.x) & ~31ull; base < n;
+         base += (uint64_t)gridDim.x * blockDim.x) {
+        const uint64_t i = base + lane;
+        const bool valid = i < n;
+        const unsigned long long key = valid ? keys[i] : kEmptyKey;
+        const uint32_t vmask = __ballot_sync(0xffffffffu, valid);
+        const uint32_t peers = __match_any_sync(0xffffffffu, key) & vmask;
+        if (!valid || (peers & lt) != 0) continue;  // one leader per distinct key in the warp
+        const uint32_t c = __popc(peers);
+        if (key == kEmptyKey) {
+            atomicAdd(&info->special, (unsigned long long)c);
+            continue;
         }
-        if (i == n - 1) {
-            unsigned long long U = (unsigned long long)pos[i] + (h ? 1ull : 0ull);
-            info->U = U;
-            head[U] = (uint32_t)n;
+        unsigned long long sl = key >> (64 - bits);
+        for (;;) {
+            unsigned long long cur = tkey[sl];
+            if (cur == kEmptyKey) {
+                cur = atomicCAS(&tkey[sl], kEmptyKey, key);
+                if (cur == kEmptyKey) cur = key;
+            }
+            if (cur == key) {
+                atomicAdd(&tcnt[sl], c);
+                break;
+            }
+            sl = (sl + 1) & mask;  // at least twice as many slots as keys
         }
     }
 }
 
-// lambda_b and the sort key (n - lambda_b); entries at u >= U sort last with key n.
-__global__ void k_rle_counts(const uint32_t *__restrict__ head, uint64_t n, const cr_plan_info_dev *info,
-                             unsigned long long *__restrict__ ucnt, uint32_t *__restrict__ sortkey)
+// Occupied slots -> a dense list (order immaterial: it is sorted next).
+__global__ void k_hist_compact(const unsigned long long *__restrict__ tkey, const uint32_t *__restrict__ tcnt,
+                               uint64_t slots, unsigned long long *__restrict__ lkey, uint32_t *__restrict__ lcnt,
+                               cr_plan_info_dev *info)
 {
-    const unsigned long long U = info->U;
-    for (uint64_t u = (uint64_t)blockIdx.x * blockDim.x + threadIdx.x; u < n; u += (uint64_t)gridDim.x * blockDim.x) {
-        if (u < U) {
-            uint32_t c = head[u + 1] - head[u];
-            ucnt[u] = c;
-            sortkey[u] = (uint32_t)(n - c);
-        } else {
-            sortkey[u] = (uint32_t)n;
+    const uint32_t lane = cr_lane();
+    for (uint64_t base = ((uint64_t)blockIdx.x * blockDim.x + threadIdx.x) & ~31ull; base < slots;
+         base += (uint64_t)gridDim.x * blockDim.x) {
+        const uint64_t s = base + lane;
+        const bool occ = s < slots && tkey[s] != kEmptyKey;
+        const uint32_t bal = __ballot_sync(0xffffffffu, occ);
+        if (!bal) continue;
+        unsigned long long at = 0;
+        if (lane == 0) at = atomicAdd(&info->U, (unsigned long long)__popc(bal));
+        at = __shfl_sync(0xffffffffu, at, 0);
+        if (occ) {
+            const unsigned long long pos = at + __popc(bal & ((1u << lane) - 1u));
+            lkey[pos] = tkey[s];
+            lcnt[pos] = tcnt[s];
         }
     }
+    if (blockIdx.x == 0 && threadIdx.x == 0 && info->special) {
+        // the key 2^64-1 was counted apart; it joins the list last
+        const unsigned long long pos = atomicAdd(&info->U, 1ull);
+        lkey[pos] = kEmptyKey;
+        lcnt[pos] = (uint32_t)info->special;
+    }
+}
+
+// ---- one-CTA stable LSD radix sort of the U distinct keys --------------------
+// 1024 threads, 8-bit digits.  All passes' digit histograms are taken in one
+// sweep.  A pass walks tiles of 4096 items; warp w owns items [128w, 128w+128)
+// of a tile, ranks them in 4 rounds with __match_any_sync against warp-private
+// digit counters, and one cross-warp prefix per digit turns the counters into
+// offsets.  The next tile's items are loaded while the current one is ranked.
+constexpr int kSmallBlock = 1024;
+constexpr int kSmallWarps = kSmallBlock / 32;
+constexpr int kSmallTile = kSmallBlock * 4;
+
+struct small_sort_smem {
+    uint32_t hist[8][256];             // digit counts of every pass, then running bases
+    uint32_t wcnt[256][kSmallWarps + 1];  // per-warp digit counters of the current tile, digit-major
+                                          // (row padded to 33 words: a warp reading one digit of every
+                                          // warp, or every digit of one warp, hits 32 distinct banks)
+};
+
+template <typename K>
+__device__ void cta_histograms(const K *kin, uint32_t n, int npass, small_sort_smem &sm)
+{
+    for (uint32_t x = threadIdx.x; x < 8 * 256; x += kSmallBlock) (&sm.hist[0][0])[x] = 0;
+    __syncthreads();
+    const uint32_t lt = (1u << cr_lane()) - 1u;
+    for (uint32_t i0 = 0; i0 < n; i0 += kSmallBlock) {  // warp-uniform trip count
+        const uint32_t i = i0 + threadIdx.x;
+        const bool valid = i < n;
+        const K key = valid ? kin[i] : (K)0;
+        for (int p = 0; p < npass; ++p) {
+            // one atomic per distinct digit in the warp: skewed digits do not serialise
+            const uint32_t d = valid ? ((uint32_t)(key >> (8 * p)) & 0xffu) : 256u;
+            const uint32_t peers = __match_any_sync(0xffffffffu, d);
+            if (valid && (peers & lt) == 0) atomicAdd(&sm.hist[p][d], (uint32_t)__popc(peers));
+        }
+    }
+    __syncthreads();
+    // exclusive scan of each pass's 256 counts (warp p scans pass p, 8 digits per lane)
+    const uint32_t warp = threadIdx.x >> 5, lane = cr_lane();
+    if (warp < (uint32_t)npass) {
+        uint32_t v[8], sum = 0;
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+            v[j] = sm.hist[warp][lane * 8 + j];
+            sum += v[j];
+        }
+        uint32_t inc = sum;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            uint32_t u = __shfl_up_sync(0xffffffffu, inc, o);
+            if (lane >= (uint32_t)o) inc += u;
+        }
+        uint32_t run = inc - sum;
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+            sm.hist[warp][lane * 8 + j] = run;
+            run += v[j];
+        }
+    }
+    __syncthreads();
+}
+
+template <typename K>
+__device__ void cta_radix_pass(const K *kin, const uint32_t *vin, K *kout, uint32_t *vout, uint32_t n, int pass,
+                               small_sort_smem &sm)
+{
+    const uint32_t tid = threadIdx.x, lane = cr_lane(), warp = tid >> 5;
+    const uint32_t lt = (1u << lane) - 1u;
+    const int shift = 8 * pass;
+    uint32_t *base = sm.hist[pass];
+    K k[4];
+    uint32_t v[4];
+    auto load_tile = [&](uint32_t t0) {
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+            const uint32_t i = t0 + warp * 128 + j * 32 + lane;
+            if (i < n) {
+                k[j] = kin[i];
+                v[j] = vin ? vin[i] : i;
+            }
+        }
+    };
+    load_tile(0);
+    for (uint32_t t0 = 0; t0 < n; t0 += kSmallTile) {
+        K ck[4];
+        uint32_t cv[4];
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+            ck[j] = k[j];
+            cv[j] = v[j];
+        }
+        if (t0 + kSmallTile < n) load_tile(t0 + kSmallTile);
+        for (uint32_t x = lane; x < 256; x += 32) sm.wcnt[x][warp] = 0;
+        __syncwarp();
+        uint32_t rank[4], dig[4];
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+            const uint32_t i = t0 + warp * 128 + j * 32 + lane;
+            const bool valid = i < n;
+            const uint32_t d = valid ? ((uint32_t)(ck[j] >> shift) & 0xffu) : 256u;
+            const uint32_t peers = __match_any_sync(0xffffffffu, d);
+            const uint32_t before = valid ? sm.wcnt[d][warp] : 0u;
+            rank[j] = before + __popc(peers & lt);
+            dig[j] = d;
+            __syncwarp();
+            if (valid && (peers & lt) == 0) sm.wcnt[d][warp] = before + __popc(peers);
+            __syncwarp();
+        }
+        __syncthreads();
+        // per digit, exclusive prefix over the warps (warp w scans digits 8w..8w+7)
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+            const uint32_t dd = warp * 8 + j;
+            const uint32_t c = sm.wcnt[dd][lane];
+            uint32_t inc = c;
+#pragma unroll
+            for (int o = 1; o < 32; o <<= 1) {
+                uint32_t u = __shfl_up_sync(0xffffffffu, inc, o);
+                if (lane >= (uint32_t)o) inc += u;
+            }
+            const uint32_t b0 = base[dd];
+            sm.wcnt[dd][lane] = b0 + inc - c;
+            __syncwarp();
+            if (lane == 31) base[dd] = b0 + inc;
+        }
+        __syncthreads();
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+            if (dig[j] < 256u) {
+                const uint32_t pos = sm.wcnt[dig[j]][warp] + rank[j];
+                kout[pos] = ck[j];
+                vout[pos] = cv[j];
+            }
+        }
+        __syncthreads();
+    }
+}
+
+// Sorts the U distinct (key, count) pairs: key ascending into (ukey, ucnt), then
+// stably by (n - count) into `order` = admission order (count desc, key asc).
+__global__ void __launch_bounds__(kSmallBlock) k_plan_sort(const cr_plan_info_dev *info, unsigned long long n,
+                                                           int cbits, unsigned long long *kA, uint32_t *vA,
+                                                           unsigned long long *kB, uint32_t *vB,
+                                                           unsigned long long *__restrict__ ukey,
+                                                           unsigned long long *__restrict__ ucnt, uint32_t *s32A,
+                                                           uint32_t *s32B, uint32_t *o32A, uint32_t *o32B,
+                                                           uint32_t *__restrict__ order)
+{
+    __shared__ small_sort_smem sm;
+    const uint32_t U = (uint32_t)info->U;
+    unsigned long long *ki = kA, *ko = kB;
+    uint32_t *vi = vA, *vo = vB;
+    cta_histograms<unsigned long long>(ki, U, 8, sm);
+    for (int pass = 0; pass < 8; ++pass) {
+        cta_radix_pass<unsigned long long>(ki, vi, ko, vo, U, pass, sm);
+        unsigned long long *tk = ki; ki = ko; ko = tk;
+        uint32_t *tv = vi; vi = vo; vo = tv;
+    }
+    for (uint32_t u = threadIdx.x; u < U; u += kSmallBlock) {
+        ukey[u] = ki[u];
+        ucnt[u] = vi[u];
+        s32A[u] = (uint32_t)(n - vi[u]);
+    }
+    __syncthreads();
+    const int cpass = (cbits + 7) / 8;
+    uint32_t *si = s32A, *so = s32B, *oi = nullptr, *oo = o32A;
+    cta_histograms<uint32_t>(si, U, cpass, sm);
+    for (int pass = 0; pass < cpass; ++pass) {
+        cta_radix_pass<uint32_t>(si, oi, so, oo, U, pass, sm);
+        uint32_t *t = si; si = so; so = t;
+        oi = oo;
+        oo = (oo == o32A) ? o32B : o32A;
+    }
+    for (uint32_t u = threadIdx.x; u < U; u += kSmallBlock) order[u] = oi ? oi[u] : u;
 }
 
 // Eq. 1: k_b = min(R, max(1, ceil(lambda * den / num))); NOREPL: 1.
@@ -148,21 +352,28 @@ __global__ void k_plan_init_load(const cr_plan_info_dev *info, const unsigned lo
 }
 
 // LPT placement (Algorithm 1 placement loop) on one warp.  Lane l owns the
-// destinations r = l, l+32, ...; it caches the smallest (L[r], r) among its
-// untaken ones.  Each job is one warp argmin over the 32 cached minima.
-__device__ __forceinline__ void lane_min(const unsigned long long *L, const unsigned char *taken, uint32_t R,
-                                         uint32_t lane, unsigned long long &mL, uint32_t &mr)
+// destinations r = l, l+32, ... (their loads and "taken" flags are touched by
+// no other lane) and caches the smallest packed key (L[r] << 16 | r) among its
+// untaken ones; packing makes (L, r) order a plain integer order (L < 2^47 is
+// enforced, r < 2^13).  Each job is one warp minimum of the 32 cached keys,
+// taken with two redux.sync reductions (high word, then low word).
+__device__ __forceinline__ unsigned long long lane_min(const unsigned long long *L, const unsigned char *taken,
+                                                       uint32_t R, uint32_t lane)
 {
-    mL = ~0ull;
-    mr = 0xffffffffu;  // no eligible destination on this lane
+    unsigned long long m = ~0ull;
     for (uint32_t r = lane; r < R; r += 32) {
         if (taken[r]) continue;
-        unsigned long long v = L[r];
-        if (mr == 0xffffffffu || v < mL) {  // r ascending: ties keep the lower index
-            mL = v;
-            mr = r;
-        }
+        const unsigned long long v = (L[r] << 16) | r;
+        m = v < m ? v : m;
     }
+    return m;
+}
+
+__device__ __forceinline__ unsigned long long warp_min_u64(unsigned long long v)
+{
+    const uint32_t hi = __reduce_min_sync(0xffffffffu, (uint32_t)(v >> 32));
+    const uint32_t lo = __reduce_min_sync(0xffffffffu, (uint32_t)(v >> 32) == hi ? (uint32_t)v : 0xffffffffu);
+    return ((unsigned long long)hi << 32) | lo;
 }
 
 __global__ void __launch_bounds__(32) k_plan_lpt(const cr_plan_info_dev *info,
@@ -181,10 +392,7 @@ __global__ void __launch_bounds__(32) k_plan_lpt(const cr_plan_info_dev *info,
         L[r] = load_g[r];
         taken[r] = 0;
     }
-    __syncwarp();
-    unsigned long long mL;
-    uint32_t mr;
-    lane_min(L, taken, R, lane, mL, mr);
+    unsigned long long m = lane_min(L, taken, R, lane);
     const unsigned long long na = info->n_adm;
     bool overflow = false;
     // the admitted keys' (lambda, k, offset) are staged 32 at a time, one per lane,
@@ -205,19 +413,10 @@ __global__ void __launch_bounds__(32) k_plan_lpt(const cr_plan_info_dev *info,
         const uint32_t base = __shfl_sync(0xffffffffu, st_off, slot);
         const unsigned long long lam = __shfl_sync(0xffffffffu, st_lam, slot);
         const unsigned long long q = k == 1 ? lam : lam / k, rem = k == 1 ? 0ull : lam % k;
+        bool took = false;
         for (uint32_t s = 0; s < k; ++s) {
-            // warp argmin of (L, r) over the lanes' cached minima
-            unsigned long long bL = mL;
-            uint32_t br = mr;
-#pragma unroll
-            for (int o = 16; o > 0; o >>= 1) {
-                unsigned long long oL = __shfl_xor_sync(0xffffffffu, bL, o);
-                uint32_t orr = __shfl_xor_sync(0xffffffffu, br, o);
-                if (oL < bL || (oL == bL && orr < br)) {
-                    bL = oL;
-                    br = orr;
-                }
-            }
+            const unsigned long long best = warp_min_u64(m);
+            const uint32_t br = (uint32_t)(best & 0xffffu);
             const unsigned long long job = q + (s < rem ? 1ull : 0ull);
             if (lane == 0) {
                 members[base + s] = (uint16_t)br;
@@ -225,30 +424,99 @@ __global__ void __launch_bounds__(32) k_plan_lpt(const cr_plan_info_dev *info,
             }
             if ((br & 31u) == lane) {
                 // a chosen destination is not eligible again for this key
-                if (k > 1) taken[br] = 1;
-                unsigned long long nl = L[br] + job;
+                if (k > 1) {
+                    taken[br] = 1;
+                    took = true;
+                }
+                const unsigned long long nl = L[br] + job;
                 if (nl >= kLoadLimit) overflow = true;
                 L[br] = nl;
-                lane_min(L, taken, R, lane, mL, mr);
+                m = lane_min(L, taken, R, lane);
             }
-            __syncwarp();
         }
-        if (k > 1) {
-            // release this key's destinations for the next key
-            bool dirty = false;
-            for (uint32_t s = 0; s < k; ++s) {
-                uint32_t m = members[base + s];
-                if ((m & 31u) == lane) {
-                    taken[m] = 0;
-                    dirty = true;
-                }
-            }
-            __syncwarp();
-            if (dirty) lane_min(L, taken, R, lane, mL, mr);
-            __syncwarp();
+        if (took) {  // release this key's destinations for the next key
+            for (uint32_t r = lane; r < R; r += 32) taken[r] = 0;
+            m = lane_min(L, taken, R, lane);
         }
     }
     for (uint32_t r = lane; r < R; r += 32) load_g[r] = L[r];
+    if (__any_sync(0xffffffffu, overflow) && lane == 0) atomicOr(status, CR_FLAG_OVERFLOW);
+}
+
+// LPT for R <= 32: lane i holds the i-th smallest packed key (L << 16 | r), so
+// T(b) for a key with k_b = k is lanes 0..k-1.  After a single-copy job the
+// grown key is re-inserted with one ballot and one shuffle; after a replicated
+// key the warp is re-sorted with a bitonic network.
+__device__ __forceinline__ unsigned long long warp_bitonic_sort(unsigned long long x)
+{
+    const uint32_t lane = cr_lane();
+#pragma unroll
+    for (int size = 2; size <= 32; size <<= 1) {
+#pragma unroll
+        for (int stride = size >> 1; stride > 0; stride >>= 1) {
+            const unsigned long long y = __shfl_xor_sync(0xffffffffu, x, stride);
+            const bool up = (lane & size) == 0;
+            const bool lower = (lane & stride) == 0;
+            const unsigned long long lo = x < y ? x : y, hi = x < y ? y : x;
+            x = (lower == up) ? lo : hi;
+        }
+    }
+    return x;
+}
+
+__global__ void __launch_bounds__(32) k_plan_lpt32(const cr_plan_info_dev *info,
+                                                   const unsigned long long *__restrict__ adm_cnt,
+                                                   const uint32_t *__restrict__ adm_k,
+                                                   const uint32_t *__restrict__ koff, uint32_t R,
+                                                   unsigned long long *__restrict__ load_g,
+                                                   uint16_t *__restrict__ members,
+                                                   unsigned long long *__restrict__ jobs, uint32_t *status)
+{
+    const uint32_t lane = cr_lane();
+    unsigned long long key = lane < R ? ((load_g[lane] << 16) | lane) : ~0ull;
+    key = warp_bitonic_sort(key);
+    const unsigned long long na = info->n_adm;
+    bool overflow = false;
+    unsigned long long st_lam = 0;
+    uint32_t st_k = 0, st_off = 0;
+    for (unsigned long long a = 0; a < na; ++a) {
+        const uint32_t slot = (uint32_t)(a & 31ull);
+        if (slot == 0) {
+            const unsigned long long ia = a + lane;
+            if (ia < na) {
+                st_lam = adm_cnt[ia];
+                st_k = adm_k[ia];
+                st_off = koff[ia];
+            }
+        }
+        const uint32_t k = __shfl_sync(0xffffffffu, st_k, slot);
+        const uint32_t base = __shfl_sync(0xffffffffu, st_off, slot);
+        const unsigned long long lam = __shfl_sync(0xffffffffu, st_lam, slot);
+        if (k == 1) {
+            const unsigned long long nk = __shfl_sync(0xffffffffu, key, 0) + (lam << 16);
+            if (lane == 0) {
+                members[base] = (uint16_t)(key & 0xffffu);
+                jobs[base] = lam;
+                if ((nk >> 16) >= kLoadLimit) overflow = true;
+            }
+            // lanes 1..pos hold keys below the grown one: shift them down one lane
+            const uint32_t below = __ballot_sync(0xffffffffu, lane > 0 && key < nk);
+            const uint32_t pos = __popc(below);
+            const unsigned long long up = __shfl_down_sync(0xffffffffu, key, 1);
+            key = lane < pos ? up : (lane == pos ? nk : key);
+        } else {
+            const unsigned long long q = lam / k, rem = lam % k;
+            if (lane < k) {
+                const unsigned long long job = q + (lane < rem ? 1ull : 0ull);
+                members[base + lane] = (uint16_t)(key & 0xffffu);
+                jobs[base + lane] = job;
+                key += job << 16;
+                if ((key >> 16) >= kLoadLimit) overflow = true;
+            }
+            key = warp_bitonic_sort(key);
+        }
+    }
+    if (lane < R) load_g[key & 0xffffu] = key >> 16;
     if (__any_sync(0xffffffffu, overflow) && lane == 0) atomicOr(status, CR_FLAG_OVERFLOW);
 }
 
@@ -470,21 +738,32 @@ extern "C" int cr_build_plans(cr_ctx *ctx, const uint64_t *d_key, uint64_t n, co
     // ---- shared histogram and admission order ------------------------------
     const uint32_t *order = nullptr;
     if (n > 0) {
-        const unsigned long long *sorted = nullptr;
-        CR_TRY(cr_radix_sort_u64(ctx, (const unsigned long long *)d_key, nullptr, n, 64, &sorted, nullptr));
-        void *pa, *pb, *pc;
-        CR_TRY(cr_scratch(ctx, SCR_PLAN_A, (n + 1) * sizeof(uint32_t), &pa));
-        CR_TRY(cr_scratch(ctx, SCR_PLAN_B, (n + 2) * sizeof(uint32_t), &pb));
-        CR_TRY(cr_scratch(ctx, SCR_PLAN_C, (n + 1) * sizeof(uint32_t), &pc));
-        uint32_t *flag = (uint32_t *)pa, *head = (uint32_t *)pb, *skey = (uint32_t *)pc;
-        CR_LAUNCH(ctx, k_rle_flags, grid_n, 256, 0, sorted, n, flag);
-        CR_TRY(cr_scan_u32(ctx, flag, flag, n, nullptr));
-        CR_LAUNCH(ctx, k_rle_heads, grid_n, 256, 0, sorted, flag, n, p0->d_ukey, head, p0->d_info);
-        CR_LAUNCH(ctx, k_rle_counts, grid_n, 256, 0, head, n, (const cr_plan_info_dev *)p0->d_info, p0->d_ucnt,
-                  skey);
-        const uint32_t *sk_sorted = nullptr;
-        CR_TRY(cr_radix_sort_u32(ctx, skey, nullptr, n, bits_for(n), &sk_sorted, &order));
-        // `order` lives in radix scratch until the next sort; nothing below sorts.
+        uint64_t slots = 1024;
+        while (slots < 2 * n) slots <<= 1;
+        const int tbits = bits_for(slots - 1);
+        void *ptk, *ptc, *pk0, *pk1, *pv0, *pv1, *po;
+        CR_TRY(cr_scratch(ctx, SCR_PLAN_A, slots * sizeof(unsigned long long), &ptk));
+        CR_TRY(cr_scratch(ctx, SCR_PLAN_B, slots * sizeof(uint32_t) + 16, &ptc));
+        CR_TRY(cr_scratch(ctx, SCR_SORT_K0, n * sizeof(unsigned long long), &pk0));
+        CR_TRY(cr_scratch(ctx, SCR_SORT_K1, n * sizeof(unsigned long long), &pk1));
+        CR_TRY(cr_scratch(ctx, SCR_SORT_V0, n * sizeof(uint32_t), &pv0));
+        CR_TRY(cr_scratch(ctx, SCR_SORT_V1, n * sizeof(uint32_t), &pv1));
+        CR_TRY(cr_scratch(ctx, SCR_PLAN_C, (2 * n + 1) * sizeof(uint32_t), &po));
+        unsigned long long *tkey = (unsigned long long *)ptk;
+        uint32_t *tcnt = (uint32_t *)ptc;
+        CR_CUDA(ctx, cudaMemsetAsync(tkey, 0xff, slots * sizeof(unsigned long long), ctx->stream));
+        CR_CUDA(ctx, cudaMemsetAsync(tcnt, 0, slots * sizeof(uint32_t), ctx->stream));
+        CR_LAUNCH(ctx, k_hist_insert, grid_n, 256, 0, (const unsigned long long *)d_key, n, tkey, tcnt, tbits,
+                  p0->d_info);
+        CR_LAUNCH(ctx, k_hist_compact, cr_blocks(slots, 256, gcap), 256, 0, (const unsigned long long *)tkey,
+                  (const uint32_t *)tcnt, slots, (unsigned long long *)pk0, (uint32_t *)pv0, p0->d_info);
+        // the (n - count) keys and the order ping-pong through the now idle table memory
+        uint32_t *s32A = (uint32_t *)ptk, *s32B = s32A + n, *o32B = (uint32_t *)ptc;
+        uint32_t *ord = (uint32_t *)po;
+        CR_LAUNCH(ctx, k_plan_sort, 1, kSmallBlock, 0, (const cr_plan_info_dev *)p0->d_info, (unsigned long long)n,
+                  bits_for(n), (unsigned long long *)pk0, (uint32_t *)pv0, (unsigned long long *)pk1,
+                  (uint32_t *)pv1, p0->d_ukey, p0->d_ucnt, s32A, s32B, ord + n, o32B, ord);
+        order = ord;
     }
 
     // ---- per plan -------------------------------------------------------------
@@ -534,6 +813,12 @@ extern "C" int cr_build_plans(cr_ctx *ctx, const uint64_t *d_key, uint64_t n, co
                 if (smem > 48 * 1024)
                     CR_CUDA(ctx, cudaFuncSetAttribute(k_plan_lpt, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                                       (int)smem));
+                if (pp.R <= 32)
+                    CR_LAUNCH(ctx, k_plan_lpt32, 1, 32, 0, (const cr_plan_info_dev *)p->d_info,
+                              (const unsigned long long *)p->d_adm_cnt, (const uint32_t *)p->d_adm_k,
+                              (const uint32_t *)p->d_koff, pp.R, p->d_load, p->d_members, p->d_jobs,
+                              ctx->d_status);
+                else
                 CR_LAUNCH(ctx, k_plan_lpt, 1, 32, smem, (const cr_plan_info_dev *)p->d_info,
                           (const unsigned long long *)p->d_adm_cnt, (const uint32_t *)p->d_adm_k,
                           (const uint32_t *)p->d_koff, pp.R, p->d_load, p->d_members, p->d_jobs, ctx->d_status);

@@ -145,6 +145,20 @@ def test_plan_hand_example_and_init_load(P, ctx):
     _cmp_plan(pl2.export(), O.build_plan(keys, 3, 2, 1000, 1, init_load=init))
 
 
+@pytest.mark.parametrize("extra", [[2**64 - 1], [0], [2**64 - 1, 0, 2**64 - 1, 2**64 - 2]])
+def test_plan_extreme_keys(P, ctx, extra):
+    # the all-ones key doubles as the device table's empty marker and is counted apart
+    rng = np.random.default_rng(len(extra))
+    keys = np.concatenate([_rates_keys(rng, 500, 5000), np.array(extra * 7, np.uint64)])
+    rng.shuffle(keys)
+    R, W = 8, 4
+    pl = P.build_plan(ctx, d_u64(keys), P.plan_params(R, W, keys.size, 3 * R))
+    got = pl.export()
+    uk, uc = O.histogram(keys)
+    assert (got["ukey"] == uk).all() and (got["ucnt"] == uc).all()
+    _cmp_plan(got, O.build_plan(keys, R, W, keys.size, 3 * R))
+
+
 def test_plan_empty_and_single(P, ctx):
     pl = P.build_plan(ctx, torch.zeros(0, dtype=torch.int64, device=DEV), P.plan_params(4, 2, 1, 1))
     got = pl.export()
@@ -251,21 +265,30 @@ def test_replay_reset_and_bad_dest(P, ctx):
 
 
 # ------------------------------------------------------------------ pipeline ---
+@pytest.mark.parametrize("overlap", [False, True])
 @pytest.mark.parametrize("name,n,nint", [("tiny", 20000, 1), ("70b", 30000, 3), ("8b", 6000, 4),
                                           ("burst", 30000, 2)])
-def test_pipeline_parity(P, ctx, name, n, nint):
+def test_pipeline_parity(P, ctx, name, n, nint, overlap):
     from paper_2608_19677_gb300.pipeline import Pipeline
     cfg = tg.CONFIGS[name]
     if name != "tiny":
         cfg = cfg.scaled(n, nint)
     tr = tg.Trace(cfg)
     ref = OP.run_trace(tr, B=1024, keep=True)
-    pipe = Pipeline(ctx, cfg.R, cfg.W, cfg.caps, cfg.replicas, tr.qcap, batch_B=1024)
-    for t in range(cfg.n_intervals):
-        iv = tr.interval(t)
-        tok, off = tg.arena_host(tr, iv, 4)
-        keys = pipe.interval(t, torch.from_numpy(tok).to(DEV), d_u64(off), d_u32(iv.plen), d_u32(iv.slen), iv.g0)
-        assert (h_u64(keys) == ref["keys"][t]).all()
-        assert (h_u16(pipe.last_dest) == ref["dest"][t]).all()
-    ctx.sync()
-    assert (h_u64(pipe.ctr) == ref["ctr"]).all()
+    pipe = Pipeline(ctx, cfg.R, cfg.W, cfg.caps, cfg.replicas, tr.qcap, batch_B=1024, overlap=overlap)
+    for rep in range(2):          # twice: reset() must restore the initial state
+        pipe.reset()
+        for t in range(cfg.n_intervals):
+            iv = tr.interval(t)
+            tok, off = tg.arena_host(tr, iv, 4)
+            keys = pipe.interval(t, torch.from_numpy(tok).to(DEV), d_u64(off), d_u32(iv.plen), d_u32(iv.slen),
+                                 iv.g0, plan_next=t + 1 < cfg.n_intervals)
+            assert (h_u64(keys) == ref["keys"][t]).all()
+            assert (h_u16(pipe.last_dest) == ref["dest"][t]).all()
+            # the plans the interval was routed with equal the oracle's
+            for (v, s), pl in zip(pipe.plan_keys, pipe.last_plans):
+                opl = ref["plans"][t][(v, s)]
+                got = pl.export()
+                assert got["n_adm"] == opl.n_adm and (got["members"] == opl.members).all()
+        pipe.sync()
+        assert (h_u64(pipe.ctr) == ref["ctr"]).all()
