@@ -1,7 +1,8 @@
 // a8, a9: shadow replay (cr_shadow_replay).
 //
-//   partition  stable radix sort of (replica, destination) over every routed
-//              request: each (replica, destination) stream in arrival order
+//   partition  one stable counting sort per replica by destination: each
+//              (replica, destination) stream's (key, prefix, suffix) records
+//              in arrival order
 //   replay     one warp per stream; the stream's LRU at the LARGEST capacity
 //              lives in shared memory (key + access stamp per entry, spread
 //              over the lanes).  A hit's depth (1 + entries touched after it)
@@ -23,63 +24,117 @@ struct replay_caps {
     uint32_t cap[CR_MAX_CAPS];
 };
 
-__global__ void k_part_keys(const uint16_t *__restrict__ dest, unsigned long long n, uint32_t n_rep, uint32_t R,
-                            int dbits, uint32_t *__restrict__ ck, uint32_t *status)
-{
-    const unsigned long long total = n * n_rep;
-    bool bad = false;
-    for (unsigned long long j = (unsigned long long)blockIdx.x * blockDim.x + threadIdx.x; j < total;
-         j += (unsigned long long)gridDim.x * blockDim.x) {
-        uint32_t rep = (uint32_t)(j / n);
-        uint32_t d = dest[j];
-        if (d >= R) {
-            bad = true;
-            ck[j] = n_rep << dbits;  // sorts after every valid stream: skipped
-        } else {
-            ck[j] = (rep << dbits) | d;
-        }
-    }
-    if (__any_sync(0xffffffffu, bad) && cr_lane() == 0) atomicOr(status, CR_FLAG_BADDEST);
-}
-
-// start[s] = first position of stream s = (rep, r) in the sorted composite keys.
-__global__ void k_stream_starts(const uint32_t *__restrict__ sk, unsigned long long m, uint32_t n_rep, uint32_t R,
-                                int dbits, uint32_t *__restrict__ start)
-{
-    const uint32_t ns = n_rep * R;
-    for (uint32_t s = blockIdx.x * blockDim.x + threadIdx.x; s <= ns; s += gridDim.x * blockDim.x) {
-        uint32_t target = (s == ns) ? (n_rep << dbits) : (((s / R) << dbits) | (s % R));
-        unsigned long long lo = 0, hi = m;
-        while (lo < hi) {
-            unsigned long long mid = (lo + hi) >> 1;
-            if (sk[mid] < target)
-                lo = mid + 1;
-            else
-                hi = mid;
-        }
-        start[s] = (uint32_t)lo;
-    }
-}
-
 struct rec16 {
     unsigned long long key;
     uint32_t P, S;
 };
 
-// Gather each partitioned request's (key, prefix, suffix) into stream order.
-__global__ void k_gather_records(const uint32_t *__restrict__ sval, unsigned long long m, unsigned long long n,
-                                 const unsigned long long *__restrict__ keys, const uint32_t *__restrict__ plen,
-                                 const uint32_t *__restrict__ slen, rec16 *__restrict__ rec)
+// ---- partition: one stable counting sort per replica, by destination --------
+// Tiles of 2048 requests.  k_part_count writes each tile's destination counts
+// at [(replica * R + r) * ntiles + tile]; one exclusive scan of that array
+// gives every (stream, tile) its output base, in stream-major order.
+// k_part_scatter ranks each tile's requests stably and writes their
+// (key, prefix, suffix) records straight to their place in stream order.
+constexpr int kPartBlock = 256;
+constexpr int kPartWarps = kPartBlock / 32;
+constexpr int kPartTile = kPartBlock * 8;
+
+__global__ void __launch_bounds__(kPartBlock) k_part_count(const uint16_t *__restrict__ dest, unsigned long long n,
+                                                           uint32_t R, uint32_t ntiles, uint32_t *__restrict__ cnt,
+                                                           uint32_t *status)
 {
-    for (unsigned long long pos = (unsigned long long)blockIdx.x * blockDim.x + threadIdx.x; pos < m;
-         pos += (unsigned long long)gridDim.x * blockDim.x) {
-        const unsigned long long j = sval[pos];
-        const unsigned long long i = j % n;
-        rec16 r;
-        r.key = keys[i];
-        r.P = plen[i];
-        r.S = slen[i];
-        rec[pos] = r;
+    extern __shared__ uint32_t hist[];
+    const uint32_t rep = blockIdx.y, tile = blockIdx.x, lane = cr_lane();
+    for (uint32_t r = threadIdx.x; r < R; r += kPartBlock) hist[r] = 0;
+    __syncthreads();
+    const uint16_t *D = dest + (unsigned long long)rep * n;
+    const unsigned long long base = (unsigned long long)tile * kPartTile;
+    bool bad = false;
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+        const unsigned long long i = base + (unsigned long long)j * kPartBlock + threadIdx.x;
+        uint32_t d = i < n ? D[i] : 0xffffu;
+        if (i < n && d >= R) {
+            bad = true;
+            d = 0xffffu;  // skipped: reported through the status word
+        }
+        const uint32_t peers = __match_any_sync(0xffffffffu, d);
+        if (d != 0xffffu && (peers & ((1u << lane) - 1u)) == 0) atomicAdd(&hist[d], (uint32_t)__popc(peers));
+    }
+    __syncthreads();
+    for (uint32_t r = threadIdx.x; r < R; r += kPartBlock)
+        cnt[((unsigned long long)rep * R + r) * ntiles + tile] = hist[r];
+    if (__any_sync(0xffffffffu, bad) && lane == 0) atomicOr(status, CR_FLAG_BADDEST);
+}
+
+// start[s] = first record of stream s = (replica, r); start[ns] = number of records.
+__global__ void k_part_starts(const uint32_t *__restrict__ off, uint32_t ns, uint32_t ntiles,
+                              const uint32_t *__restrict__ total, uint32_t *__restrict__ start)
+{
+    for (uint32_t s = blockIdx.x * blockDim.x + threadIdx.x; s <= ns; s += gridDim.x * blockDim.x)
+        start[s] = s < ns ? off[(unsigned long long)s * ntiles] : *total;
+}
+
+// Warp w ranks items [256w, 256w+256) of the tile in 8 rounds against
+// warp-private counters (u16, destination-major); one pass over the
+// destinations turns them into per-warp offsets.
+__global__ void __launch_bounds__(kPartBlock) k_part_scatter(const uint16_t *__restrict__ dest, unsigned long long n,
+                                                             uint32_t R, uint32_t ntiles,
+                                                             const uint32_t *__restrict__ off,
+                                                             const unsigned long long *__restrict__ keys,
+                                                             const uint32_t *__restrict__ plen,
+                                                             const uint32_t *__restrict__ slen,
+                                                             rec16 *__restrict__ rec)
+{
+    extern __shared__ uint16_t wc[];  // [R][8]
+    const uint32_t rep = blockIdx.y, tile = blockIdx.x, lane = cr_lane(), warp = threadIdx.x >> 5;
+    const uint32_t lt = (1u << lane) - 1u;
+    uint4 *wc4 = reinterpret_cast<uint4 *>(wc);
+    for (uint32_t r = threadIdx.x; r < R; r += kPartBlock) wc4[r] = make_uint4(0, 0, 0, 0);
+    __syncthreads();
+    const uint16_t *D = dest + (unsigned long long)rep * n;
+    const unsigned long long base = (unsigned long long)tile * kPartTile + (unsigned long long)warp * 256;
+    uint32_t dig[8], rank[8];
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+        const unsigned long long i = base + (unsigned long long)j * 32 + lane;
+        uint32_t d = i < n ? D[i] : 0xffffu;
+        if (d >= R) d = 0xffffu;
+        const uint32_t peers = __match_any_sync(0xffffffffu, d);
+        const uint32_t before = d != 0xffffu ? wc[d * kPartWarps + warp] : 0u;
+        rank[j] = before + __popc(peers & lt);
+        dig[j] = d;
+        __syncwarp();
+        if (d != 0xffffu && (peers & lt) == 0) wc[d * kPartWarps + warp] = (uint16_t)(before + __popc(peers));
+        __syncwarp();
+    }
+    __syncthreads();
+    for (uint32_t r = threadIdx.x; r < R; r += kPartBlock) {  // exclusive prefix over the 8 warps
+        uint4 v = wc4[r];
+        uint16_t c[8];
+        memcpy(c, &v, 16);
+        uint16_t run = 0;
+#pragma unroll
+        for (int w = 0; w < kPartWarps; ++w) {
+            const uint16_t x = c[w];
+            c[w] = run;
+            run = (uint16_t)(run + x);
+        }
+        memcpy(&v, c, 16);
+        wc4[r] = v;
+    }
+    __syncthreads();
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+        if (dig[j] == 0xffffu) continue;
+        const unsigned long long i = base + (unsigned long long)j * 32 + lane;
+        const uint32_t pos = off[((unsigned long long)rep * R + dig[j]) * ntiles + tile] +
+                             wc[dig[j] * kPartWarps + warp] + rank[j];
+        rec16 rr;
+        rr.key = keys[i];
+        rr.P = plen[i];
+        rr.S = slen[i];
+        rec[pos] = rr;
     }
 }
 
@@ -325,13 +380,6 @@ k_lru_chunks(const replay_caps caps, uint32_t cmax, uint32_t R, uint32_t ns, uin
     }
 }
 
-int bits_for(uint64_t v)
-{
-    int b = 0;
-    while (b < 64 && (v >> b) != 0) ++b;
-    return b;
-}
-
 template <int E, int NC>
 int launch_replay_nc(cr_ctx *ctx, cr_replay *rp, const replay_caps &caps, uint32_t CL, const uint32_t *start,
                      const uint32_t *coff, const uint32_t *total, uint64_t m, const rec16 *rec, uint64_t *d_ctr)
@@ -433,33 +481,37 @@ extern "C" int cr_shadow_replay(cr_ctx *ctx, cr_replay *rp, const uint64_t *d_ke
     const uint64_t m = n * rp->n_rep;
     if (n >= (1ull << 31) || m >= 0xffffffffull)
         return cr_fail(ctx, CR_EINVAL, "cr_shadow_replay: n * n_rep must be < 2^32 - 1");
-    const int dbits = bits_for(rp->R - 1) ? bits_for(rp->R - 1) : 1;
-    const int rbits = bits_for(rp->n_rep);  // rep == n_rep marks a skipped request
-    if (dbits + rbits > 32) return cr_fail(ctx, CR_EINVAL, "cr_shadow_replay: composite key too wide");
-    void *pk, *ps;
-    CR_TRY(cr_scratch(ctx, SCR_REPLAY_IDX, m * sizeof(uint32_t), &pk));
-    CR_TRY(cr_scratch(ctx, SCR_REPLAY_START, (rp->n_streams + 1) * sizeof(uint32_t), &ps));
-    uint32_t *ck = (uint32_t *)pk, *start = (uint32_t *)ps;
+    const uint32_t R = rp->R, ns = (uint32_t)rp->n_streams;
+    const uint32_t ntiles = (uint32_t)((n + kPartTile - 1) / kPartTile);
+    const uint64_t ncnt = (uint64_t)ns * ntiles;
+    if (ncnt >= 0xffffffffull) return cr_fail(ctx, CR_EINVAL, "cr_shadow_replay: too many (stream, tile) pairs");
+    void *pk, *ps, *prec, *pch;
+    CR_TRY(cr_scratch(ctx, SCR_REPLAY_IDX, (ncnt + 2) * sizeof(uint32_t), &pk));
+    CR_TRY(cr_scratch(ctx, SCR_REPLAY_START, ((size_t)ns + 1) * sizeof(uint32_t), &ps));
+    CR_TRY(cr_scratch(ctx, SCR_REPLAY_REC, m * sizeof(rec16), &prec));
+    CR_TRY(cr_scratch(ctx, SCR_REPLAY_CHUNK, ((size_t)ns + 2) * sizeof(uint32_t), &pch));
+    uint32_t *cnt = (uint32_t *)pk, *nrec = cnt + ncnt, *start = (uint32_t *)ps;
+    rec16 *rec = (rec16 *)prec;
+    uint32_t *coff = (uint32_t *)pch, *total = coff + ns;
     const unsigned int gcap = (unsigned int)ctx->num_sms * 8u;
-    CR_LAUNCH(ctx, k_part_keys, cr_blocks(m, 256, gcap), 256, 0, d_dest, (unsigned long long)n, rp->n_rep, rp->R,
-              dbits, ck, ctx->d_status);
-    const uint32_t *sk = nullptr, *sval = nullptr;
-    CR_TRY(cr_radix_sort_u32(ctx, ck, nullptr, m, dbits + rbits, &sk, &sval));
-    CR_LAUNCH(ctx, k_stream_starts, cr_blocks(rp->n_streams + 1, 256, gcap), 256, 0, sk, (unsigned long long)m,
-              rp->n_rep, rp->R, dbits, start);
+    const dim3 pgrid(ntiles, rp->n_rep);
+    const size_t csmem = (size_t)R * sizeof(uint32_t), ssmem = (size_t)R * kPartWarps * sizeof(uint16_t);
+    if (csmem > 48 * 1024)
+        CR_CUDA(ctx, cudaFuncSetAttribute(k_part_count, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)csmem));
+    if (ssmem > 48 * 1024)
+        CR_CUDA(ctx, cudaFuncSetAttribute(k_part_scatter, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)ssmem));
+    CR_LAUNCH(ctx, k_part_count, pgrid, kPartBlock, csmem, d_dest, (unsigned long long)n, R, ntiles, cnt,
+              ctx->d_status);
+    CR_TRY(cr_scan_u32(ctx, cnt, cnt, ncnt, nrec));
+    CR_LAUNCH(ctx, k_part_starts, cr_blocks((uint64_t)ns + 1, 256, gcap), 256, 0, (const uint32_t *)cnt, ns, ntiles,
+              (const uint32_t *)nrec, start);
+    CR_LAUNCH(ctx, k_part_scatter, pgrid, kPartBlock, ssmem, d_dest, (unsigned long long)n, R, ntiles,
+              (const uint32_t *)cnt, (const unsigned long long *)d_key, d_plen, d_slen, rec);
     replay_caps caps;
     caps.n_caps = rp->n_caps;
     for (uint32_t c = 0; c < CR_MAX_CAPS; ++c) caps.cap[c] = c < rp->n_caps ? rp->caps[c] : 0;
     // chunk length: long enough that rebuilding an LRU state of cmax entries is amortised
     const uint32_t CL = rp->cmax * 16u > 256u ? rp->cmax * 16u : 256u;
-    const uint32_t ns = (uint32_t)rp->n_streams;
-    void *prec, *pch;
-    CR_TRY(cr_scratch(ctx, SCR_REPLAY_REC, m * sizeof(rec16), &prec));
-    CR_TRY(cr_scratch(ctx, SCR_REPLAY_CHUNK, ((size_t)ns + 2) * sizeof(uint32_t), &pch));
-    rec16 *rec = (rec16 *)prec;
-    uint32_t *coff = (uint32_t *)pch, *total = coff + ns;
-    CR_LAUNCH(ctx, k_gather_records, cr_blocks(m, 256, gcap), 256, 0, sval, (unsigned long long)m,
-              (unsigned long long)n, (const unsigned long long *)d_key, d_plen, d_slen, rec);
     CR_LAUNCH(ctx, k_chunk_counts, cr_blocks(ns, 256, gcap), 256, 0, (const uint32_t *)start, ns, CL, coff);
     CR_TRY(cr_scan_u32(ctx, coff, coff, ns, total));
     const uint32_t E = (rp->cmax + 31) / 32;

@@ -11,11 +11,14 @@ One control interval t:
   4. cr_shadow_replay: LRU simulators whose state and counters persist over
      intervals.
 
-With ``overlap=True`` the planner runs on its own stream and library context:
-the plans for interval t+1 depend only on interval t's keys, so they are built
-while interval t is routed and replayed and interval t+1 is hashed.  The
-planner is latency-bound on a few SMs; the other stages stream over all of
-them.  Plans and keys are double-buffered and ordered by CUDA events.
+With ``overlap=True`` the planner runs on its own high-priority stream and
+library context, ordered by CUDA events: plans(t+1) need only interval t's
+keys, so they are built on a few SMs while interval t is routed and replayed
+and interval t+1 is hashed on the main stream.  (The driver can also put
+hashing on a stream of its own; that is off because the hash kernel's CTAs
+occupy every SM and would delay the single-SM routing CTAs instead of sharing
+the machine with them.)  Keys are triple-buffered and plans double-buffered; a
+buffer is reused only after events show its last reader has finished.
 """
 from __future__ import annotations
 
@@ -25,6 +28,7 @@ from . import (Context, Plan, Replay, build_plans, hash_prefixes, plan_params, r
                shadow_replay)
 
 VARIANT_OF = {"CR": "LPT", "CR_NOLPT": "RANDOM", "CR_NOREPL": "NOREPL"}
+NKEYS = 3
 
 
 class Pipeline:
@@ -51,113 +55,180 @@ class Pipeline:
             if k not in self.plan_keys:
                 self.plan_keys.append(k)
             self.rep_plan.append(self.plan_keys.index(k))
-        self.overlap = overlap and bool(self.plan_keys)
-        if self.overlap:
-            self.pstream = torch.cuda.Stream(dev)
+        self.overlap = overlap
+        self.mstream = ctx._stream_obj
+        if overlap:
+            # Hashing stays on the main stream: its CTAs fill every SM, so a
+            # hash stream would starve the single-SM routing CTAs rather than
+            # share with them.  The planner gets its own high-priority stream.
+            lo, hi = torch.cuda.Stream.priority_range() if hasattr(torch.cuda.Stream, "priority_range") else (0, -1)
+            self.hstream, self.hctx = self.mstream, ctx
+            self.pstream = torch.cuda.Stream(dev, priority=hi)
             self.pctx = Context(ctx.device, self.pstream)
         else:
-            self.pstream, self.pctx = ctx._stream_obj, ctx
+            self.hstream = self.pstream = self.mstream
+            self.hctx = self.pctx = ctx
         self.plans = [[Plan(self.pctx) for _ in self.plan_keys] for _ in range(2)]
         self.replay = Replay(ctx, len(self.replicas), R, self.caps)
         self.ctr = torch.zeros((len(self.replicas), len(self.caps), R, 5), dtype=torch.int64, device=dev)
         self.load = torch.zeros((len(self.replicas), R), dtype=torch.int64, device=dev)
         self._dest = None
-        self._keys = [None, None]
-        self._flip = 0
+        self._keys = [None] * NKEYS
+        self._released = [[] for _ in range(NKEYS)]  # events after which a keys buffer may be rewritten
+        self._kidx = 0
         self.prev_keys = None
+        self._prev_kb = None
         self._ready = [None, None]   # event: plans buffer b is built
         self._pbuf = 0               # plans buffer used by the next interval
         self._next_built = False     # the next interval's plans are already enqueued
         self.plan_marks = []         # (start, end) events of every plan build, when marked
+        self.hash_marks = []         # (start, end) events of every hash, when marked
         if max_n:
             self._alloc(max_n)
+
+    @property
+    def contexts(self):
+        out = []
+        for c in (self.ctx, self.hctx, self.pctx):
+            if all(c is not o for o in out):
+                out.append(c)
+        return out
 
     def _alloc(self, n: int):
         import torch
         if self._dest is None or self._dest.shape[1] < n:
+            self.sync()
             self._dest = torch.empty((len(self.replicas), n), dtype=torch.int16, device=self.dev)
-            self._keys = [torch.empty(n, dtype=torch.int64, device=self.dev) for _ in range(2)]
+            self._keys = [torch.empty(n, dtype=torch.int64, device=self.dev) for _ in range(NKEYS)]
+            self._released = [[] for _ in range(NKEYS)]
 
     def reset(self):
+        """Empty the simulators and counters; later work is ordered after everything before."""
+        import torch
         self.replay.reset()
         self.ctr.zero_()
         self.prev_keys = None
+        self._prev_kb = None
         self._next_built = False
         self.plan_marks = []
+        self.hash_marks = []
+        if self.overlap:
+            start = torch.cuda.Event()
+            start.record(self.mstream)
+            self.hstream.wait_event(start)
+            self.pstream.wait_event(start)
+
+    def _event(self, stream, timing=False):
+        import torch
+        e = torch.cuda.Event(enable_timing=timing)
+        e.record(stream)
+        return e
 
     def _build(self, buf: int, keys, epoch: int, after, mark: bool):
         """Enqueue the plans of one interval into plans buffer ``buf`` from ``keys``."""
-        import torch
         if self.overlap:
             self.pstream.wait_event(after)
-        st = self.pstream
-        ev0 = torch.cuda.Event(enable_timing=True) if mark else None
-        if mark:
-            ev0.record(st)
+        ev0 = self._event(self.pstream, True) if mark else None
         num, den = self.qcap(int(keys.shape[0]))
         params = [plan_params(self.R, self.W, num, den, v, seed=s, epoch=epoch) for v, s in self.plan_keys]
         build_plans(self.pctx, keys, params, self.plans[buf])
-        ready = torch.cuda.Event(enable_timing=mark)
-        ready.record(st)
+        ready = self._event(self.pstream, mark)
         self._ready[buf] = ready
         if mark:
             self.plan_marks.append((ev0, ready))
+        return ready
 
-    def interval(self, t: int, tokens, off, plen, slen, g0: int, marks=None, plan_next: bool = True):
-        """Run one control interval on device tensors; returns the interval's keys.
+    def interval(self, t: int, tokens, off, plen, slen, g0: int, marks=None, plan_next: bool = True,
+                 inputs_ready=None):
+        """Enqueue one control interval on device tensors; returns the interval's keys.
 
         ``marks``: optional list of 5 torch.cuda.Event recorded on the main
-        stream at the stage boundaries (start, hashed, plans ready, routed,
-        replayed); plan builds are timed separately in ``plan_marks``.
-        ``plan_next``: with overlap, also enqueue the next interval's plans.
+        stream at the stage boundaries (start, keys ready, plans ready, routed,
+        replayed); hash and plan builds are timed in ``hash_marks`` and
+        ``plan_marks`` on their own streams.  ``plan_next``: with overlap, also
+        enqueue the next interval's plans.  ``inputs_ready``: event after which
+        the input tensors may be read (e.g. the end of their copy).
         """
-        import torch
         n = int(off.shape[0])
-        stream = self.ctx._stream_obj
-        if marks is not None:
-            marks[0].record(stream)
+        mark = marks is not None
+        if mark:
+            marks[0].record(self.mstream)
         self._alloc(n)
-        keys = self._keys[self._flip][:n]
-        self._flip ^= 1
-        hash_prefixes(self.ctx, tokens, off, plen, self.salt, out=keys)
-        hashed = torch.cuda.Event()
-        hashed.record(stream)
-        if marks is not None:
-            marks[1].record(stream)
+        kb = self._kidx
+        self._kidx = (self._kidx + 1) % NKEYS
+        keys = self._keys[kb][:n]
+        # ---- hash ---------------------------------------------------------------
+        for e in self._released[kb]:
+            self.hstream.wait_event(e)
+        self._released[kb] = []
+        if inputs_ready is not None:
+            self.hstream.wait_event(inputs_ready)
+        h0 = self._event(self.hstream, True) if mark else None
+        hash_prefixes(self.hctx, tokens, off, plen, self.salt, out=keys)
+        hashed = self._event(self.hstream, mark)
+        if mark:
+            self.hash_marks.append((h0, hashed))
+        # ---- plans ----------------------------------------------------------------
         cur = self._pbuf
+        plan_reader = None
         if self.plan_keys:
             if not self._next_built:
                 # nothing planned ahead: plan this interval from the previous keys (or its own)
-                pk = keys if self.prev_keys is None else self.prev_keys
-                self._build(cur, pk, t, hashed, marks is not None)
+                if self.prev_keys is None:
+                    pk, after = keys, hashed
+                else:
+                    pk, after = self.prev_keys, self._prev_hashed
+                built = self._build(cur, pk, t, after, mark)
+                if self.overlap and self.prev_keys is not None:
+                    self._released[self._prev_kb].append(built)
             if self.overlap and plan_next:
-                # the next interval plans from this interval's keys: start now
-                self._build(cur ^ 1, keys, t + 1, hashed, marks is not None)
+                # the next interval plans from this interval's keys: start as soon as they exist
+                plan_reader = self._build(cur ^ 1, keys, t + 1, hashed, mark)
                 self._next_built = True
             else:
                 self._next_built = False
-            if self.overlap:
-                stream.wait_event(self._ready[cur])
-        if marks is not None:
-            marks[2].record(stream)
+        # ---- route and replay ---------------------------------------------------------
+        if self.overlap:
+            self.mstream.wait_event(hashed)
+            if self.plan_keys:
+                self.mstream.wait_event(self._ready[cur])
+        if mark:
+            marks[1].record(self.mstream)
+            marks[2].record(self.mstream)
         self.load.zero_()
         dest = self._dest[:, :n] if n == self._dest.shape[1] else self._dest.view(-1)[:len(self.replicas) * n].view(
             len(self.replicas), n)
         plans = [self.plans[cur][i] if i is not None else None for i in self.rep_plan]
         route_batch(self.ctx, plans, self.policies, self.seeds, self.R, keys, g0, self.B, self.load, dest)
-        if marks is not None:
-            marks[3].record(stream)
+        if mark:
+            marks[3].record(self.mstream)
         shadow_replay(self.ctx, self.replay, keys, plen, slen, dest, self.ctr)
-        if marks is not None:
-            marks[4].record(stream)
+        if mark:
+            marks[4].record(self.mstream)
+        # keys buffer kb is free once this interval's replay and the next plans have read it
+        if self.overlap:
+            self._released[kb].append(self._event(self.mstream))
+            if plan_reader is not None:
+                self._released[kb].append(plan_reader)
         self.prev_keys = keys
+        self._prev_kb = kb
+        self._prev_hashed = hashed
         self.last_dest = dest
         self.last_plans = [self.plans[cur][i] for i in range(len(self.plan_keys))]
         if self.overlap and self._next_built:
             self._pbuf = cur ^ 1
         return keys
 
-    def sync(self):
-        self.ctx.sync()
+    def finish(self):
+        """Make the main stream wait for every other stream's enqueued work."""
         if self.overlap:
-            self.pctx.sync()
+            self.mstream.wait_event(self._event(self.hstream))
+            self.mstream.wait_event(self._event(self.pstream))
+
+    def sync(self):
+        for c in self.contexts:
+            c.sync()
+
+    @property
+    def launches(self) -> int:
+        return sum(c.launches for c in self.contexts)
