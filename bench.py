@@ -117,6 +117,27 @@ class ClockSampler:
                 "samples": len(sm), "reasons": sorted(reasons)}
 
 
+def hash_traffic(alg_bytes_per_launch: float):
+    """DRAM bytes per hash launch from the committed ncu capture, scaled by algorithmic
+    bytes; None when the kernel source has changed since the capture."""
+    import hashlib
+    path = os.path.join(ROOT, "profiles", "k_hash_prefixes_traffic.txt")
+    src = os.path.join(ROOT, "paper_2608_19677_gb300", "csrc", "cr_hash.cu")
+    try:
+        kv = {}
+        for line in open(path):
+            line = line.strip()
+            if line and not line.startswith("#"):
+                k, v = line.split(None, 1)
+                kv[k] = v
+        if kv.get("source_sha256") != hashlib.sha256(open(src, "rb").read()).hexdigest():
+            return None
+        ratio = (float(kv["dram_bytes_read"]) + float(kv["dram_bytes_write"])) / float(kv["algorithmic_bytes"])
+        return ratio * alg_bytes_per_launch
+    except Exception:
+        return None
+
+
 # ----------------------------------------------------------------- oracle ---
 def oracle_sample(trace, n_intervals: int = 1, B: int = 1024):
     """Time the CPU oracle (hash, plans, route, replay) on the first intervals of the trace."""
@@ -317,13 +338,7 @@ def main():
         pass
     hbm_peak = float(peaks.get("hbm_gbs", 6800.0))
     peak_src = "measured" if "hbm_gbs" in peaks else "fallback"
-    traffic = None
-    try:
-        prof = json.load(open(os.path.join(ROOT, "profiles", "hash_traffic.json")))
-        if prof.get("kernel_rev") == "k_hash_prefixes-v1":
-            traffic = prof.get("bytes_per_launch_70b_mean")
-    except Exception:
-        pass
+    traffic = hash_traffic(float(hb.mean()))
     roofline = {"kernel": "k_hash_prefixes", "bound": "hbm", "achieved": hash_gbs, "peak": hbm_peak,
                 "peak_source": peak_src, "unit": "GB/s", "frac": hash_gbs / hbm_peak, "traffic": traffic,
                 "algorithmic_bytes_per_launch_mean": float(hb.mean()),
