@@ -277,6 +277,34 @@ CR_API int cr_shadow_replay(cr_ctx *ctx, cr_replay *rp, const uint64_t *d_key, c
 CR_API int cr_replay_export_state(cr_ctx *ctx, const cr_replay *rp, uint32_t rep, uint32_t r,
                            uint64_t *keys_out, uint32_t *fill_out);
 
+/* ==== allocation-free key histogram ================================== */
+/*
+ * The paper has no counterpart to this call: it exists for callers that
+ * cannot allocate device memory at the moment they call in, for example a
+ * process whose device memory is owned by another runtime's pool, or a
+ * latency-critical path that cannot afford cudaMalloc (which may synchronise
+ * the device).  It needs no context: it computes the same per-key histogram
+ * as cr_build_plans (lambda_b = requests with key b) with all of its scratch
+ * in a fixed array inside the library (about 3.6 MB, held on every GPU that
+ * loads the library until the process exits), and calls no allocating
+ * function.
+ *   d_key   uint64[n] keys (device), n <= CR_NOALLOC_MAX_KEYS
+ *   d_ukey  uint64[n] receives the distinct keys, ascending (first *d_U used)
+ *   d_ucnt  uint64[n] receives their counts
+ *   d_U     uint64[1] (device) receives the number of distinct keys
+ *   cuda_stream  stream the work is enqueued on (NULL = legacy default)
+ * The first call on a device looks up the array's device address on that
+ * device (it must be current); make that first call before any stream
+ * capture.  All calls share the one array: calls whose work overlaps on the
+ * GPU (different streams, or different host threads) race and must be
+ * ordered by the caller.  Every call clears what it needs, so earlier
+ * contents never leak into a result.
+ * Errors (message via cr_last_error(NULL)): CR_EINVAL (n too large, NULL
+ * pointer), CR_ECUDA. */
+#define CR_NOALLOC_MAX_KEYS 65536
+CR_API int cr_key_histogram_noalloc(const uint64_t *d_key, uint64_t n, uint64_t *d_ukey, uint64_t *d_ucnt,
+                                    uint64_t *d_U, void *cuda_stream);
+
 #ifdef __cplusplus
 }
 #endif

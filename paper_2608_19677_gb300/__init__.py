@@ -34,7 +34,8 @@ MAX_R, MAX_CAP, MAX_CAPS, MAX_REPLICAS, CTR_FIELDS = 8192, 1024, 8, 256, 5
 EXPORTS = ("cr_create", "cr_destroy", "cr_set_stream", "cr_sync", "cr_last_error", "cr_launch_count",
            "cr_hash_prefixes", "cr_plan_create", "cr_plan_destroy", "cr_build_plans", "cr_build_plan",
            "cr_plan_get_info", "cr_plan_export", "cr_route_batch", "cr_replay_create", "cr_replay_reset",
-           "cr_replay_destroy", "cr_shadow_replay", "cr_replay_export_state")
+           "cr_replay_destroy", "cr_shadow_replay", "cr_replay_export_state", "cr_key_histogram_noalloc")
+CR_NOALLOC_MAX_KEYS = 65536
 
 
 class CacheRouteError(RuntimeError):
@@ -97,6 +98,7 @@ def lib() -> C.CDLL:
         "cr_replay_destroy": ([vp, vp], i32),
         "cr_shadow_replay": ([vp, vp, vp, vp, vp, vp, u64, vp], i32),
         "cr_replay_export_state": ([vp, vp, u32, u32, vp, C.POINTER(C.c_uint32)], i32),
+        "cr_key_histogram_noalloc": ([vp, u64, vp, vp, vp, vp], i32),
     }
     for name, (args, res) in sig.items():
         f = getattr(L, name)

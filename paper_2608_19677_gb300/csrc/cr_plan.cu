@@ -885,3 +885,94 @@ extern "C" int cr_plan_export(cr_ctx *ctx, const cr_plan *p, uint64_t *ukey, uin
     if (load) CR_CUDA(ctx, cudaMemcpyAsync(load, p->d_load, (uint64_t)info.R * 8, cudaMemcpyDeviceToHost, s));
     return cr_sync(ctx);
 }
+
+// ---- allocation-free key histogram (cr_key_histogram_noalloc) ---------------
+// Some callers cannot allocate device memory when they call in: a process whose
+// device memory is owned and handed out by another runtime's pool, or a
+// latency-critical path where a cudaMalloc (which may synchronise the device)
+// is not acceptable.  For them the histogram of the plan builder runs with its
+// scratch in this file-scope array, sized for at most CR_NOALLOC_MAX_KEYS keys.
+// Every GPU that loads the library holds the array until the process exits.
+// Layout: table keys | table counts | sort keys (2 buffers) | sort values
+// (2 buffers) | order (2 buffers) | info.
+namespace {
+constexpr uint64_t kNaSlots = 2ull * CR_NOALLOC_MAX_KEYS;  // power of two, >= 2n
+constexpr uint64_t kNaN = CR_NOALLOC_MAX_KEYS;
+constexpr size_t kNaOffTcnt = kNaSlots * 8;
+constexpr size_t kNaOffKA = kNaOffTcnt + kNaSlots * 4;
+constexpr size_t kNaOffKB = kNaOffKA + kNaN * 8;
+constexpr size_t kNaOffVA = kNaOffKB + kNaN * 8;
+constexpr size_t kNaOffVB = kNaOffVA + kNaN * 4;
+constexpr size_t kNaOffOrd = kNaOffVB + kNaN * 4;
+constexpr size_t kNaOffInfo = kNaOffOrd + (2 * kNaN + 64) * 4;
+constexpr size_t kNaBytes = kNaOffInfo + 256;
+}  // namespace
+
+static __device__ __align__(256) unsigned char g_noalloc_scratch[kNaBytes];
+
+namespace {
+constexpr int kNaMaxDevices = 64;
+void *g_noalloc_ptr[kNaMaxDevices];  // device address of g_noalloc_scratch, per device
+
+__global__ void k_copy_u(const cr_plan_info_dev *info, unsigned long long *out) { *out = info->U; }
+}  // namespace
+
+extern "C" int cr_key_histogram_noalloc(const uint64_t *d_key, uint64_t n, uint64_t *d_ukey, uint64_t *d_ucnt,
+                                        uint64_t *d_U, void *cuda_stream)
+{
+    if (n > CR_NOALLOC_MAX_KEYS)
+        return cr_fail(NULL, CR_EINVAL, "cr_key_histogram_noalloc: n=%llu exceeds CR_NOALLOC_MAX_KEYS=%d",
+                       (unsigned long long)n, CR_NOALLOC_MAX_KEYS);
+    if (!d_U || (n > 0 && (!d_key || !d_ukey || !d_ucnt)))
+        return cr_fail(NULL, CR_EINVAL, "cr_key_histogram_noalloc: NULL pointer");
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kNaMaxDevices) {
+        cudaGetLastError();
+        return cr_fail(NULL, CR_ECUDA, "cr_key_histogram_noalloc: no usable current device");
+    }
+    if (!g_noalloc_ptr[dev]) {
+        // once per device, with that device current: the array's device address
+        void *p = NULL;
+        cudaError_t e = cudaGetSymbolAddress(&p, g_noalloc_scratch);
+        if (e != cudaSuccess || !p) {
+            cudaGetLastError();
+            return cr_fail(NULL, CR_ECUDA, "cr_key_histogram_noalloc: cudaGetSymbolAddress: %s",
+                           cudaGetErrorString(e));
+        }
+        g_noalloc_ptr[dev] = p;
+    }
+    cudaStream_t s = (cudaStream_t)cuda_stream;
+    unsigned char *base = (unsigned char *)g_noalloc_ptr[dev];
+    cr_plan_info_dev *info = (cr_plan_info_dev *)(base + kNaOffInfo);
+    k_plan_reset<<<1, 1, 0, s>>>(info, (unsigned long long)n);
+    if (n > 0) {
+        uint64_t slots = 1024;
+        while (slots < 2 * n) slots <<= 1;
+        int tbits = 0;
+        while ((1ull << tbits) < slots) ++tbits;
+        unsigned long long *tkey = (unsigned long long *)base;
+        uint32_t *tcnt = (uint32_t *)(base + kNaOffTcnt);
+        unsigned long long *kA = (unsigned long long *)(base + kNaOffKA), *kB = (unsigned long long *)(base + kNaOffKB);
+        uint32_t *vA = (uint32_t *)(base + kNaOffVA), *vB = (uint32_t *)(base + kNaOffVB);
+        uint32_t *ord = (uint32_t *)(base + kNaOffOrd);
+        int nsm = 1;
+        cudaDeviceGetAttribute(&nsm, cudaDevAttrMultiProcessorCount, dev);
+        const unsigned int grid = cr_blocks(n, 256, (unsigned int)nsm * 8u);
+        if (cudaMemsetAsync(tkey, 0xff, slots * sizeof(unsigned long long), s) != cudaSuccess ||
+            cudaMemsetAsync(tcnt, 0, slots * sizeof(uint32_t), s) != cudaSuccess) {
+            cudaGetLastError();
+            return cr_fail(NULL, CR_ECUDA, "cr_key_histogram_noalloc: clearing the table failed");
+        }
+        k_hist_insert<<<grid, 256, 0, s>>>((const unsigned long long *)d_key, n, tkey, tcnt, tbits, info);
+        k_hist_compact<<<cr_blocks(slots, 256, (unsigned int)nsm * 8u), 256, 0, s>>>(tkey, tcnt, slots, kA, vA, info);
+        uint32_t *s32A = (uint32_t *)tkey, *s32B = s32A + n;
+        k_plan_sort<<<1, kSmallBlock, 0, s>>>(info, (unsigned long long)n, bits_for(n), kA, vA, kB, vB,
+                                              (unsigned long long *)d_ukey, (unsigned long long *)d_ucnt, s32A,
+                                              s32B, ord + n, tcnt, ord);
+    }
+    k_copy_u<<<1, 1, 0, s>>>(info, (unsigned long long *)d_U);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess)
+        return cr_fail(NULL, CR_ECUDA, "cr_key_histogram_noalloc: launch failed: %s", cudaGetErrorString(e));
+    return CR_OK;
+}
