@@ -520,6 +520,102 @@ __global__ void __launch_bounds__(32) k_plan_lpt32(const cr_plan_info_dev *info,
     if (__any_sync(0xffffffffu, overflow) && lane == 0) atomicOr(status, CR_FLAG_OVERFLOW);
 }
 
+// LPT for 32 < R <= 1024, all LPT plans of one build at once (one warp per
+// plan).  Lane l holds the packed keys of destinations l, l+32, ... in NE
+// registers and their minimum; a job is one warp minimum (two redux.sync),
+// then the owner lane updates the chosen register and recomputes its minimum
+// with a tree over registers.  Destinations chosen earlier for the same key
+// are masked out by a per-lane bit set.
+struct lpt_job {
+    const cr_plan_info_dev *info;
+    const unsigned long long *adm_cnt;
+    const uint32_t *adm_k, *koff;
+    unsigned long long *load;
+    uint16_t *members;
+    unsigned long long *jobs;
+    uint32_t R;
+};
+
+struct lpt_jobs {
+    lpt_job j[16];
+};
+
+template <int NE>
+__device__ __forceinline__ unsigned long long reg_min(const unsigned long long (&v)[NE], uint32_t taken)
+{
+    unsigned long long t[NE];
+#pragma unroll
+    for (int j = 0; j < NE; ++j) t[j] = ((taken >> j) & 1u) ? ~0ull : v[j];
+#pragma unroll
+    for (int w = NE / 2; w > 0; w >>= 1) {
+#pragma unroll
+        for (int j = 0; j < w; ++j) t[j] = t[j + w] < t[j] ? t[j + w] : t[j];
+    }
+    return t[0];
+}
+
+template <int NE>
+__global__ void __launch_bounds__(32) k_plan_lpt_reg(const __grid_constant__ lpt_jobs jobs_in, uint32_t *status)
+{
+    const lpt_job J = jobs_in.j[blockIdx.x];
+    const uint32_t lane = cr_lane(), R = J.R;
+    unsigned long long v[NE];
+#pragma unroll
+    for (int j = 0; j < NE; ++j) {
+        const uint32_t r = lane + 32u * j;
+        v[j] = r < R ? ((J.load[r] << 16) | r) : ~0ull;
+    }
+    uint32_t taken = 0;
+    unsigned long long m = reg_min<NE>(v, 0u);
+    const unsigned long long na = J.info->n_adm;
+    bool overflow = false;
+    unsigned long long st_lam = 0;
+    uint32_t st_k = 0, st_off = 0;
+    for (unsigned long long a = 0; a < na; ++a) {
+        const uint32_t slot = (uint32_t)(a & 31ull);
+        if (slot == 0) {
+            const unsigned long long ia = a + lane;
+            if (ia < na) {
+                st_lam = J.adm_cnt[ia];
+                st_k = J.adm_k[ia];
+                st_off = J.koff[ia];
+            }
+        }
+        const uint32_t k = __shfl_sync(0xffffffffu, st_k, slot);
+        const uint32_t base = __shfl_sync(0xffffffffu, st_off, slot);
+        const unsigned long long lam = __shfl_sync(0xffffffffu, st_lam, slot);
+        const unsigned long long q = k == 1 ? lam : lam / k, rem = k == 1 ? 0ull : lam % k;
+        for (uint32_t s = 0; s < k; ++s) {
+            const unsigned long long best = warp_min_u64(m);
+            const uint32_t br = (uint32_t)(best & 0xffffu);
+            const unsigned long long job = q + (s < rem ? 1ull : 0ull);
+            if (lane == 0) {
+                J.members[base + s] = (uint16_t)br;
+                J.jobs[base + s] = job;
+            }
+            if ((br & 31u) == lane) {
+                const uint32_t jj = br >> 5;
+#pragma unroll
+                for (int j = 0; j < NE; ++j)
+                    if (j == (int)jj) v[j] += job << 16;
+                if (((best >> 16) + job) >= kLoadLimit) overflow = true;
+                if (k > 1) taken |= 1u << jj;
+                m = reg_min<NE>(v, taken);
+            }
+        }
+        if (k > 1) {  // release this key's destinations for the next key
+            taken = 0;
+            m = reg_min<NE>(v, 0u);
+        }
+    }
+#pragma unroll
+    for (int j = 0; j < NE; ++j) {
+        const uint32_t r = lane + 32u * j;
+        if (r < R) J.load[r] = v[j] >> 16;
+    }
+    if (__any_sync(0xffffffffu, overflow) && lane == 0) atomicOr(status, CR_FLAG_OVERFLOW);
+}
+
 // RANDOM placement: one warp per admitted key; the first k steps of a
 // Fisher-Yates shuffle of 0..R-1 held in shared memory.
 constexpr int kRandWarps = 4;
@@ -767,6 +863,38 @@ extern "C" int cr_build_plans(cr_ctx *ctx, const uint64_t *d_key, uint64_t n, co
     }
 
     // ---- per plan -------------------------------------------------------------
+    // LPT placements with 32 < R <= 1024 are collected and run together, one
+    // warp per plan, followed by their tables.
+    lpt_jobs lj;
+    uint32_t n_lj = 0, lj_maxR = 0, deferred[16];
+    auto table_insert = [&](uint32_t j) -> int {
+        cr_plan *p = plans[j];
+        const uint64_t C = (uint64_t)params[j].R * params[j].W;
+        const int bits = bits_for(p->table_slots - 1);
+        const uint64_t adm = n < C ? n : C;
+        CR_LAUNCH(ctx, k_table_insert, cr_blocks(adm, 256, gcap), 256, 0, (const cr_plan_info_dev *)p->d_info,
+                  (const unsigned long long *)p->d_adm_key, (const uint32_t *)p->d_adm_k,
+                  (const uint32_t *)p->d_koff, (const uint16_t *)p->d_members, p->d_table, bits);
+        return CR_OK;
+    };
+    auto flush_lpt = [&]() -> int {
+        if (!n_lj) return CR_OK;
+        const uint32_t ne = (lj_maxR + 31) / 32;
+        if (ne <= 2)
+            CR_LAUNCH(ctx, k_plan_lpt_reg<2>, n_lj, 32, 0, lj, ctx->d_status);
+        else if (ne <= 4)
+            CR_LAUNCH(ctx, k_plan_lpt_reg<4>, n_lj, 32, 0, lj, ctx->d_status);
+        else if (ne <= 8)
+            CR_LAUNCH(ctx, k_plan_lpt_reg<8>, n_lj, 32, 0, lj, ctx->d_status);
+        else if (ne <= 16)
+            CR_LAUNCH(ctx, k_plan_lpt_reg<16>, n_lj, 32, 0, lj, ctx->d_status);
+        else
+            CR_LAUNCH(ctx, k_plan_lpt_reg<32>, n_lj, 32, 0, lj, ctx->d_status);
+        for (uint32_t x = 0; x < n_lj; ++x) CR_TRY(table_insert(deferred[x]));
+        n_lj = 0;
+        lj_maxR = 0;
+        return CR_OK;
+    };
     for (uint32_t j = 0; j < n_plans; ++j) {
         cr_plan *p = plans[j];
         const cr_plan_params &pp = params[j];
@@ -818,19 +946,29 @@ extern "C" int cr_build_plans(cr_ctx *ctx, const uint64_t *d_key, uint64_t n, co
                               (const unsigned long long *)p->d_adm_cnt, (const uint32_t *)p->d_adm_k,
                               (const uint32_t *)p->d_koff, pp.R, p->d_load, p->d_members, p->d_jobs,
                               ctx->d_status);
-                else
+                else if (pp.R <= 1024) {
+                    lpt_job &jb = lj.j[n_lj++];
+                    jb.info = p->d_info;
+                    jb.adm_cnt = p->d_adm_cnt;
+                    jb.adm_k = p->d_adm_k;
+                    jb.koff = p->d_koff;
+                    jb.load = p->d_load;
+                    jb.members = p->d_members;
+                    jb.jobs = p->d_jobs;
+                    jb.R = pp.R;
+                    lj_maxR = pp.R > lj_maxR ? pp.R : lj_maxR;
+                    deferred[n_lj - 1] = j;
+                    if (n_lj == 16) CR_TRY(flush_lpt());
+                    continue;
+                } else
                 CR_LAUNCH(ctx, k_plan_lpt, 1, 32, smem, (const cr_plan_info_dev *)p->d_info,
                           (const unsigned long long *)p->d_adm_cnt, (const uint32_t *)p->d_adm_k,
                           (const uint32_t *)p->d_koff, pp.R, p->d_load, p->d_members, p->d_jobs, ctx->d_status);
             }
-            int bits = bits_for(p->table_slots - 1);
-            uint64_t adm = n < C ? n : C;
-            CR_LAUNCH(ctx, k_table_insert, cr_blocks(adm, 256, gcap), 256, 0, (const cr_plan_info_dev *)p->d_info,
-                      (const unsigned long long *)p->d_adm_key, (const uint32_t *)p->d_adm_k,
-                      (const uint32_t *)p->d_koff, (const uint16_t *)p->d_members, p->d_table, bits);
+            CR_TRY(table_insert(j));
         }
     }
-    return CR_OK;
+    return flush_lpt();
 }
 
 extern "C" int cr_build_plan(cr_ctx *ctx, const uint64_t *d_key, uint64_t n, const cr_plan_params *params,
