@@ -139,7 +139,7 @@ class Pipeline:
         return ready
 
     def interval(self, t: int, tokens, off, plen, slen, g0: int, marks=None, plan_next: bool = True,
-                 inputs_ready=None):
+                 inputs_ready=None, keys=None):
         """Enqueue one control interval on device tensors; returns the interval's keys.
 
         ``marks``: optional list of 5 torch.cuda.Event recorded on the main
@@ -147,27 +147,32 @@ class Pipeline:
         replayed); hash and plan builds are timed in ``hash_marks`` and
         ``plan_marks`` on their own streams.  ``plan_next``: with overlap, also
         enqueue the next interval's plans.  ``inputs_ready``: event after which
-        the input tensors may be read (e.g. the end of their copy).
+        the input tensors may be read (e.g. the end of their copy).  ``keys``:
+        the interval's routing keys when they were computed beforehand (the
+        token arena is then not read and may be None).
         """
-        n = int(off.shape[0])
+        n = int(keys.shape[0]) if keys is not None else int(off.shape[0])
         mark = marks is not None
         if mark:
             marks[0].record(self.mstream)
         self._alloc(n)
         kb = self._kidx
         self._kidx = (self._kidx + 1) % NKEYS
-        keys = self._keys[kb][:n]
         # ---- hash ---------------------------------------------------------------
         for e in self._released[kb]:
             self.hstream.wait_event(e)
         self._released[kb] = []
         if inputs_ready is not None:
             self.hstream.wait_event(inputs_ready)
-        h0 = self._event(self.hstream, True) if mark else None
-        hash_prefixes(self.hctx, tokens, off, plen, self.salt, out=keys)
-        hashed = self._event(self.hstream, mark)
-        if mark:
-            self.hash_marks.append((h0, hashed))
+        if keys is None:
+            keys = self._keys[kb][:n]
+            h0 = self._event(self.hstream, True) if mark else None
+            hash_prefixes(self.hctx, tokens, off, plen, self.salt, out=keys)
+            hashed = self._event(self.hstream, mark)
+            if mark:
+                self.hash_marks.append((h0, hashed))
+        else:
+            hashed = self._event(self.hstream)
         # ---- plans ----------------------------------------------------------------
         cur = self._pbuf
         plan_reader = None

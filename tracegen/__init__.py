@@ -328,6 +328,42 @@ def arena_device(trace: Trace, iv: Interval, align: int = 4, device="cuda", chun
     return out, torch.as_tensor(off.view(np.int64), device=device)
 
 
+_ctok = None
+
+
+def _tokens_lib():
+    """The C token generator (compiled on first use with the host C compiler)."""
+    global _ctok
+    if _ctok is None:
+        import ctypes
+        import os
+        import subprocess
+        here = os.path.dirname(os.path.abspath(__file__))
+        src, lib = os.path.join(here, "_tokens.c"), os.path.join(here, "_tokens.so")
+        if not os.path.exists(lib) or os.path.getmtime(lib) < os.path.getmtime(src):
+            tmp = lib + f".tmp{os.getpid()}"
+            subprocess.check_call(["gcc", "-std=c11", "-O2", "-fPIC", "-shared", "-o", tmp, src])
+            os.replace(tmp, lib)
+        L = ctypes.CDLL(lib)
+        L.tg_prefix_tokens.restype = None
+        L.tg_prefix_tokens.argtypes = [ctypes.c_void_p, ctypes.c_void_p, ctypes.c_uint64, ctypes.c_int64,
+                                       ctypes.c_int64, ctypes.c_void_p, ctypes.c_void_p]
+        _ctok = L
+    return _ctok
+
+
+def prefix_spans(trace: Trace, key_ids) -> Tuple[np.ndarray, np.ndarray, np.ndarray]:
+    """Prefix spans of many keys packed back to back: (tokens int32, off uint64, plen uint32)."""
+    ids = np.ascontiguousarray(key_ids, dtype=np.int64)
+    pl = np.ascontiguousarray(trace.key_plen[ids], dtype=np.uint32)
+    total = int(pl.astype(np.int64).sum())
+    tok = np.empty(max(total, 1), dtype=np.int32)
+    off = np.empty(max(ids.size, 1), dtype=np.uint64)
+    _tokens_lib().tg_prefix_tokens(ids.ctypes.data, pl.ctypes.data, ids.size, trace.cfg.trace_seed,
+                                   trace.cfg.vocab, tok.ctypes.data, off.ctypes.data)
+    return tok[:total], off[:ids.size], pl
+
+
 def prefix_tokens(trace: Trace, key_id: int) -> np.ndarray:
     """The prefix token span of one business key (host)."""
     p = int(trace.key_plen[key_id])
