@@ -380,6 +380,291 @@ k_lru_chunks(const replay_caps caps, uint32_t cmax, uint32_t R, uint32_t ns, uin
     }
 }
 
+// ---- capacities above 32: linked-list LRU with a hash index -----------------
+// One warp per (stream, chunk); lane 0 runs the simulator, the warp helps to
+// load and rebuild states.  Shared memory per warp: keys, prev/next links in
+// recency order (most recent at the head), a segment id per entry and an
+// open-addressing index key -> entry.  With the distinct capacities sorted
+// c_0 < c_1 < ... < c_{m-1} = cmax, segment j holds recency positions
+// (c_{j-1}, c_j] and B[j] is the entry at position c_j: an access at segment
+// s hits every capacity c_j with j >= s (LRU inclusion).  Moving an entry to
+// the front shifts the last entry of each earlier segment into the next one,
+// so every access costs O(m) pointer updates, independent of cmax.
+struct list_caps {
+    uint32_t m;                 // distinct capacities
+    uint32_t c[CR_MAX_CAPS];    // ascending
+    uint32_t out[CR_MAX_CAPS];  // counter index (position in the caller's caps) of c[j]
+    uint32_t n_out;             // caller's capacity count
+    uint32_t seg_of[CR_MAX_CAPS];  // for each caller index: its segment j
+};
+
+constexpr uint16_t kNil = 0xffffu;
+
+struct lru_list {
+    unsigned long long *key;
+    uint16_t *prev, *next;
+    uint8_t *seg;
+    uint32_t *tab;  // entry + 1; 0 = empty
+    uint32_t mask;
+    int tbits;
+};
+
+__device__ __forceinline__ uint32_t home_slot(unsigned long long key, int tbits) { return (uint32_t)(key >> (64 - tbits)); }
+
+__device__ __forceinline__ int list_find(const lru_list &L, unsigned long long key)
+{
+    uint32_t s = home_slot(key, L.tbits);
+    for (;;) {
+        const uint32_t e = L.tab[s];
+        if (e == 0) return -1;
+        if (L.key[e - 1] == key) return (int)(e - 1);
+        s = (s + 1) & L.mask;
+    }
+}
+
+__device__ __forceinline__ void list_insert_index(const lru_list &L, unsigned long long key, uint32_t node)
+{
+    uint32_t s = home_slot(key, L.tbits);
+    while (atomicCAS(&L.tab[s], 0u, node + 1) != 0u) s = (s + 1) & L.mask;
+}
+
+// Remove the index entry of `node` (key `key`): backward-shift deletion for linear probing.
+__device__ __forceinline__ void list_erase_index(const lru_list &L, unsigned long long key, uint32_t node)
+{
+    uint32_t i = home_slot(key, L.tbits);
+    while (L.tab[i] != node + 1) i = (i + 1) & L.mask;
+    uint32_t j = i;
+    for (;;) {
+        j = (j + 1) & L.mask;
+        const uint32_t e = L.tab[j];
+        if (e == 0) break;
+        const uint32_t k = home_slot(L.key[e - 1], L.tbits);
+        const bool stays = (i <= j) ? (i < k && k <= j) : (i < k || k <= j);
+        if (stays) continue;
+        L.tab[i] = e;
+        i = j;
+    }
+    L.tab[i] = 0;
+}
+
+template <int NC>
+__global__ void __launch_bounds__(128)
+k_lru_list(const list_caps lc, uint32_t cmax, uint32_t R, uint32_t ns, uint32_t CL, int tbits,
+           const uint32_t *__restrict__ start, const uint32_t *__restrict__ coff, const uint32_t *__restrict__ total,
+           const rec16 *__restrict__ rec, const replay_state st, unsigned long long *__restrict__ ctr)
+{
+    extern __shared__ unsigned long long smw[];
+    const uint32_t lane = cr_lane(), warp = threadIdx.x >> 5, wpb = blockDim.x >> 5;
+    const uint32_t tsz = 1u << tbits;
+    // per-warp region, 8-byte aligned pieces
+    const size_t per_warp = (size_t)cmax * 8 + (size_t)tsz * 4 + (((size_t)cmax * 5 + 7) & ~(size_t)7);
+    unsigned char *base = reinterpret_cast<unsigned char *>(smw) + per_warp * warp;
+    lru_list L;
+    L.key = reinterpret_cast<unsigned long long *>(base);
+    L.tab = reinterpret_cast<uint32_t *>(base + (size_t)cmax * 8);
+    L.prev = reinterpret_cast<uint16_t *>(base + (size_t)cmax * 8 + (size_t)tsz * 4);
+    L.next = L.prev + cmax;
+    L.seg = reinterpret_cast<uint8_t *>(L.next + cmax);
+    L.mask = tsz - 1;
+    L.tbits = tbits;
+
+    const uint32_t w = blockIdx.x * wpb + warp;
+    if (w >= *total) return;
+    uint32_t lo = 0, hi = ns;
+    while (hi - lo > 1) {
+        const uint32_t mid = (lo + hi) >> 1;
+        if (coff[mid] <= w)
+            lo = mid;
+        else
+            hi = mid;
+    }
+    const uint32_t s = lo, ci = w - coff[s];
+    const uint32_t b = start[s], e = start[s + 1];
+    const uint32_t p0 = b + ci * CL;
+    const uint32_t p1 = (e - p0) < CL ? e : p0 + CL;
+    const uint32_t rep = s / R, r = s % R;
+    const uint32_t fill_in = st.fill_in[s];
+    const unsigned long long *kin = st.keys_in + (unsigned long long)s * cmax;
+    const uint32_t lt = (1u << lane) - 1u;
+
+    if (b == e) {  // nothing routed here: carry the state over unchanged
+        unsigned long long *kout = st.keys_out + (unsigned long long)s * cmax;
+        for (uint32_t q = lane; q < fill_in; q += 32) kout[q] = kin[q];
+        if (lane == 0) st.fill_out[s] = fill_in;
+        return;
+    }
+
+    // ---- state at p0, as keys in recency order in L.key[0..fill) ---------------
+    for (uint32_t x = lane; x < tsz; x += 32) L.tab[x] = 0;
+    __syncwarp();
+    uint32_t fill = 0;
+    if (ci == 0) {
+        for (uint32_t q = lane; q < fill_in; q += 32) {
+            L.key[q] = kin[q];
+            list_insert_index(L, kin[q], q);
+        }
+        fill = fill_in;
+    } else {
+        const uint32_t back = p0 - b;
+        const uint32_t vtot = back + fill_in;
+        for (uint32_t v0 = 0; v0 < vtot && fill < cmax; v0 += 32) {
+            const uint32_t v = v0 + lane;
+            const bool valid = v < vtot;
+            unsigned long long key = 0;
+            if (valid) key = v < back ? rec[p0 - 1 - v].key : kin[v - back];
+            const uint32_t peers = __match_any_sync(0xffffffffu, key);
+            const bool fresh = valid && (peers & lt) == 0 && list_find(L, key) < 0;
+            const uint32_t bal = __ballot_sync(0xffffffffu, fresh);
+            const uint32_t rank = __popc(bal & lt);
+            __syncwarp();
+            if (fresh && fill + rank < cmax) {
+                L.key[fill + rank] = key;
+                list_insert_index(L, key, fill + rank);
+            }
+            fill = min(cmax, fill + (uint32_t)__popc(bal));
+            __syncwarp();
+        }
+    }
+    // links and segments of the recency order 0..fill-1
+    for (uint32_t q = lane; q < fill; q += 32) {
+        L.prev[q] = q == 0 ? kNil : (uint16_t)(q - 1);
+        L.next[q] = q + 1 == fill ? kNil : (uint16_t)(q + 1);
+        uint32_t sg = 0;
+        while (sg + 1 < lc.m && q + 1 > lc.c[sg]) ++sg;
+        L.seg[q] = (uint8_t)sg;
+    }
+    __syncwarp();
+
+    unsigned long long my_req = 0, my_prompt = 0;
+    unsigned long long hitc[NC], hitt[NC];
+#pragma unroll
+    for (int j = 0; j < NC; ++j) hitc[j] = hitt[j] = 0;
+    // simulator registers (meaningful in lane 0)
+    uint32_t head = fill ? 0u : kNil, tail = fill ? fill - 1 : kNil;
+    uint32_t B[NC];
+#pragma unroll
+    for (int j = 0; j < NC; ++j) B[j] = (j + 1 < (int)lc.m && fill >= lc.c[j]) ? lc.c[j] - 1 : kNil;
+
+    for (uint32_t t0 = p0; t0 < p1; t0 += 32) {
+        // the warp stages 32 requests; lane 0 simulates them in order
+        rec16 mine = {0ull, 0u, 0u};
+        if (t0 + lane < p1) {
+            mine = rec[t0 + lane];
+            my_req += 1;
+            my_prompt += (unsigned long long)mine.P + mine.S;
+        }
+        const uint32_t cnt = (p1 - t0) < 32u ? (p1 - t0) : 32u;
+        for (uint32_t jq = 0; jq < cnt; ++jq) {
+            const unsigned long long key = __shfl_sync(0xffffffffu, mine.key, jq);
+            const uint32_t P = __shfl_sync(0xffffffffu, mine.P, jq);
+            if (lane == 0) {
+                const int n = list_find(L, key);
+                if (n >= 0) {
+                    const uint32_t sg = L.seg[n];
+#pragma unroll
+                    for (int j = 0; j < NC; ++j) {
+                        if (j < (int)lc.m && (uint32_t)j >= sg) {
+                            hitc[j] += 1;
+                            hitt[j] += P;
+                        }
+                    }
+                    if ((uint32_t)n != head) {
+                        const uint32_t pn = L.prev[n];
+#pragma unroll
+                        for (int j = 0; j < NC; ++j) {
+                            if (j + 1 < (int)lc.m) {
+                                if ((uint32_t)j < sg) {
+                                    L.seg[B[j]] = (uint8_t)(j + 1);
+                                    B[j] = lc.c[j] == 1 ? (uint32_t)n : L.prev[B[j]];
+                                } else if ((uint32_t)j == sg && B[j] == (uint32_t)n) {
+                                    B[j] = pn;
+                                }
+                            }
+                        }
+                        // unlink n, push it to the front
+                        const uint32_t nx = L.next[n];
+                        L.next[pn] = (uint16_t)nx;
+                        if (nx != kNil)
+                            L.prev[nx] = (uint16_t)pn;
+                        else
+                            tail = pn;
+                        L.prev[n] = kNil;
+                        L.next[n] = (uint16_t)head;
+                        L.prev[head] = (uint16_t)n;
+                        head = (uint32_t)n;
+                        L.seg[n] = 0;
+                    }
+                } else {
+                    uint32_t node;
+                    const uint32_t old_fill = fill;
+                    // every resident entry moves back one position
+#pragma unroll
+                    for (int j = 0; j < NC; ++j) {
+                        if (j + 1 < (int)lc.m && B[j] != kNil) {
+                            L.seg[B[j]] = (uint8_t)(j + 1);
+                            B[j] = L.prev[B[j]];  // kNil when c_j == 1: the new entry, set below
+                        }
+                    }
+                    if (fill == cmax) {
+                        node = tail;
+                        list_erase_index(L, L.key[node], node);
+                        tail = L.prev[node];
+                        if (tail != kNil) L.next[tail] = kNil;
+                        if (head == node) head = kNil;
+                    } else {
+                        node = fill++;
+                    }
+                    L.key[node] = key;
+                    L.seg[node] = 0;
+                    L.prev[node] = kNil;
+                    L.next[node] = (uint16_t)head;
+                    if (head != kNil) L.prev[head] = (uint16_t)node;
+                    head = node;
+                    if (tail == kNil) tail = node;
+                    list_insert_index(L, key, node);
+#pragma unroll
+                    for (int j = 0; j < NC; ++j) {
+                        if (j + 1 < (int)lc.m) {
+                            if (B[j] == kNil && old_fill >= lc.c[j]) B[j] = node;    // c_j == 1
+                            if (old_fill < lc.c[j] && fill == lc.c[j]) B[j] = tail;  // boundary now defined
+                        }
+                    }
+                }
+            }
+            __syncwarp();
+        }
+    }
+
+    // ---- counters -------------------------------------------------------------
+    my_req = cr_warp_sum_u64(my_req);
+    my_prompt = cr_warp_sum_u64(my_prompt);
+    if (lane == 0) {
+        // hand the state to the next call, most recent first
+        if (p1 == e) {
+            unsigned long long *kout = st.keys_out + (unsigned long long)s * cmax;
+            uint32_t q = 0;
+            for (uint32_t x = head; x != kNil; x = L.next[x]) kout[q++] = L.key[x];
+            st.fill_out[s] = fill;
+        }
+        for (uint32_t oi = 0; oi < lc.n_out; ++oi) {
+            const uint32_t j = lc.seg_of[oi];
+            unsigned long long h = 0, tk = 0;
+#pragma unroll
+            for (int jj = 0; jj < NC; ++jj)
+                if ((uint32_t)jj == j) {
+                    h = hitc[jj];
+                    tk = hitt[jj];
+                }
+            unsigned long long *C = ctr + (((unsigned long long)rep * lc.n_out + oi) * R + r) * CR_CTR_FIELDS;
+            atomicAdd(&C[0], my_req);
+            if (h) atomicAdd(&C[1], h);
+            if (tk) atomicAdd(&C[2], tk);
+            atomicAdd(&C[3], my_prompt);
+            atomicAdd(&C[4], my_prompt - tk);
+        }
+    }
+}
+
 template <int E, int NC>
 int launch_replay_nc(cr_ctx *ctx, cr_replay *rp, const replay_caps &caps, uint32_t CL, const uint32_t *start,
                      const uint32_t *coff, const uint32_t *total, uint64_t m, const rec16 *rec, uint64_t *d_ctr)
@@ -409,6 +694,61 @@ int launch_replay(cr_ctx *ctx, cr_replay *rp, const replay_caps &caps, uint32_t 
     if (caps.n_caps == 1) return launch_replay_nc<E, 1>(ctx, rp, caps, CL, start, coff, total, m, rec, d_ctr);
     if (caps.n_caps <= 3) return launch_replay_nc<E, 3>(ctx, rp, caps, CL, start, coff, total, m, rec, d_ctr);
     return launch_replay_nc<E, CR_MAX_CAPS>(ctx, rp, caps, CL, start, coff, total, m, rec, d_ctr);
+}
+
+template <int NC>
+int launch_list_nc(cr_ctx *ctx, cr_replay *rp, const list_caps &lc, uint32_t CL, int tbits, const uint32_t *start,
+                   const uint32_t *coff, const uint32_t *total, uint64_t m, const rec16 *rec, uint64_t *d_ctr)
+{
+    const uint32_t cmax = rp->cmax, tsz = 1u << tbits;
+    const size_t per_warp = (size_t)cmax * 8 + (size_t)tsz * 4 + (((size_t)cmax * 5 + 7) & ~(size_t)7);
+    uint32_t wpb = 4;
+    while (wpb > 1 && per_warp * wpb > 200 * 1024) wpb >>= 1;
+    const size_t smem = per_warp * wpb;
+    if (smem > 48 * 1024)
+        CR_CUDA(ctx, cudaFuncSetAttribute(k_lru_list<NC>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
+    const uint32_t ns = rp->n_rep * rp->R;
+    const uint64_t items = (uint64_t)ns + (m + CL - 1) / CL;
+    replay_state st;
+    st.keys_in = rp->d_keys[rp->cur];
+    st.fill_in = rp->d_fill[rp->cur];
+    st.keys_out = rp->d_keys[rp->cur ^ 1];
+    st.fill_out = rp->d_fill[rp->cur ^ 1];
+    CR_LAUNCH(ctx, k_lru_list<NC>, (unsigned int)((items + wpb - 1) / wpb), wpb * 32, smem, lc, cmax, rp->R, ns, CL,
+              tbits, start, coff, total, rec, st, (unsigned long long *)d_ctr);
+    rp->cur ^= 1;
+    return CR_OK;
+}
+
+int launch_list(cr_ctx *ctx, cr_replay *rp, uint32_t CL, const uint32_t *start, const uint32_t *coff,
+                const uint32_t *total, uint64_t m, const rec16 *rec, uint64_t *d_ctr)
+{
+    list_caps lc;
+    memset(&lc, 0, sizeof(lc));
+    uint32_t sorted[CR_MAX_CAPS];
+    uint32_t ns_ = 0;
+    for (uint32_t i = 0; i < rp->n_caps; ++i) {
+        bool dup = false;
+        for (uint32_t j = 0; j < ns_; ++j) dup |= sorted[j] == rp->caps[i];
+        if (!dup) sorted[ns_++] = rp->caps[i];
+    }
+    for (uint32_t i = 1; i < ns_; ++i)
+        for (uint32_t j = i; j > 0 && sorted[j - 1] > sorted[j]; --j) {
+            uint32_t t = sorted[j];
+            sorted[j] = sorted[j - 1];
+            sorted[j - 1] = t;
+        }
+    lc.m = ns_;
+    for (uint32_t j = 0; j < ns_; ++j) lc.c[j] = sorted[j];
+    lc.n_out = rp->n_caps;
+    for (uint32_t i = 0; i < rp->n_caps; ++i)
+        for (uint32_t j = 0; j < ns_; ++j)
+            if (sorted[j] == rp->caps[i]) lc.seg_of[i] = j;
+    int tbits = 0;
+    while ((1u << tbits) < 2 * rp->cmax) ++tbits;
+    if (lc.m <= 1) return launch_list_nc<1>(ctx, rp, lc, CL, tbits, start, coff, total, m, rec, d_ctr);
+    if (lc.m <= 3) return launch_list_nc<3>(ctx, rp, lc, CL, tbits, start, coff, total, m, rec, d_ctr);
+    return launch_list_nc<CR_MAX_CAPS>(ctx, rp, lc, CL, tbits, start, coff, total, m, rec, d_ctr);
 }
 
 }  // namespace
@@ -515,12 +855,9 @@ extern "C" int cr_shadow_replay(cr_ctx *ctx, cr_replay *rp, const uint64_t *d_ke
     CR_LAUNCH(ctx, k_chunk_counts, cr_blocks(ns, 256, gcap), 256, 0, (const uint32_t *)start, ns, CL, coff);
     CR_TRY(cr_scan_u32(ctx, coff, coff, ns, total));
     const uint32_t E = (rp->cmax + 31) / 32;
-    if (E <= 1) return launch_replay<1>(ctx, rp, caps, CL, start, coff, total, m, rec, d_ctr);
-    if (E <= 2) return launch_replay<2>(ctx, rp, caps, CL, start, coff, total, m, rec, d_ctr);
-    if (E <= 4) return launch_replay<4>(ctx, rp, caps, CL, start, coff, total, m, rec, d_ctr);
-    if (E <= 8) return launch_replay<8>(ctx, rp, caps, CL, start, coff, total, m, rec, d_ctr);
-    if (E <= 16) return launch_replay<16>(ctx, rp, caps, CL, start, coff, total, m, rec, d_ctr);
-    return launch_replay<32>(ctx, rp, caps, CL, start, coff, total, m, rec, d_ctr);
+    // capacities up to 32: one entry per lane in registers; above: linked list + hash index
+    if (E > 1) return launch_list(ctx, rp, CL, start, coff, total, m, rec, d_ctr);
+    return launch_replay<1>(ctx, rp, caps, CL, start, coff, total, m, rec, d_ctr);
 }
 
 extern "C" int cr_replay_export_state(cr_ctx *ctx, const cr_replay *rp, uint32_t rep, uint32_t r,

@@ -217,7 +217,8 @@ def test_route_rejects_bad_args(P, ctx):
 
 
 # ------------------------------------------------------------------ a8, a9 ---
-@pytest.mark.parametrize("caps", [[1], [2, 16], [12], [64, 256, 1024], [5, 33, 100], [1024]])
+@pytest.mark.parametrize("caps", [[1], [2, 16], [12], [32], [33], [64, 256, 1024], [5, 33, 100], [1024],
+                                  [1, 40, 64], [2, 2, 50], [256, 64], [1, 2, 3, 4, 5, 6, 7, 40]])
 def test_replay_parity(P, ctx, caps):
     rng = np.random.default_rng(sum(caps))
     n_rep, R = 3, 5
