@@ -380,93 +380,94 @@ k_lru_chunks(const replay_caps caps, uint32_t cmax, uint32_t R, uint32_t ns, uin
     }
 }
 
-// ---- capacities above 32: linked-list LRU with a hash index -----------------
-// One warp per (stream, chunk); lane 0 runs the simulator, the warp helps to
-// load and rebuild states.  Shared memory per warp: keys, prev/next links in
-// recency order (most recent at the head), a segment id per entry and an
-// open-addressing index key -> entry.  With the distinct capacities sorted
-// c_0 < c_1 < ... < c_{m-1} = cmax, segment j holds recency positions
-// (c_{j-1}, c_j] and B[j] is the entry at position c_j: an access at segment
-// s hits every capacity c_j with j >= s (LRU inclusion).  Moving an entry to
-// the front shifts the last entry of each earlier segment into the next one,
-// so every access costs O(m) pointer updates, independent of cmax.
-struct list_caps {
-    uint32_t m;                 // distinct capacities
-    uint32_t c[CR_MAX_CAPS];    // ascending
-    uint32_t out[CR_MAX_CAPS];  // counter index (position in the caller's caps) of c[j]
-    uint32_t n_out;             // caller's capacity count
-    uint32_t seg_of[CR_MAX_CAPS];  // for each caller index: its segment j
-};
+// ---- capacities above 32: batched stack distances ---------------------------
+// One warp per (stream, chunk) holds the LRU of the largest capacity as keys in
+// recency order, K[0] most recent, in shared memory, with an open-addressing
+// index key -> position (u16, position + 1, 0 = empty) rebuilt after every
+// batch.  A batch is 32 consecutive requests, one per lane.  The depth of
+// request i (its LRU stack distance, Mattson et al. 1970) follows from the
+// state before the batch and the batch itself:
+//   - key seen earlier in the batch, last at lane j: 1 + the number of
+//     distinct keys among lanes (j, i);
+//   - first time in the batch, at position d0 before it: d0 + 1 + the number
+//     of distinct keys among lanes < i that were deeper than d0 or absent;
+//   - absent before the batch: a miss at every capacity.
+// A request hits capacity c iff its depth <= c.  The state after the batch is
+// the batch's distinct keys by last access (latest first) followed by the
+// untouched old keys in their old order, cut at cmax.
+constexpr uint32_t kNone = 0xffffffffu;
+constexpr uint16_t kTomb = 0xffffu;  // index slot whose key was evicted
 
-constexpr uint16_t kNil = 0xffffu;
-
-struct lru_list {
-    unsigned long long *key;
-    uint16_t *prev, *next;
-    uint8_t *seg;
-    uint32_t *tab;  // entry + 1; 0 = empty
+struct lru_index {
+    unsigned long long *K;  // [cmax] keys, recency order
+    uint16_t *TS;           // [cmax] index slot of the key at each position
+    uint16_t *tab;          // [tsz] position + 1; 0 = empty, kTomb = evicted
+    uint32_t *bm;           // [32] bitmap of old positions touched by the batch
     uint32_t mask;
     int tbits;
 };
 
-__device__ __forceinline__ uint32_t home_slot(unsigned long long key, int tbits) { return (uint32_t)(key >> (64 - tbits)); }
+__device__ __forceinline__ uint32_t lru_home(unsigned long long key, int tbits) { return (uint32_t)(key >> (64 - tbits)); }
 
-__device__ __forceinline__ int list_find(const lru_list &L, unsigned long long key)
+// Position of `key` (kNone if absent); *slot gets its index slot.
+__device__ __forceinline__ uint32_t lru_lookup(const lru_index &X, unsigned long long key, uint32_t *slot)
 {
-    uint32_t s = home_slot(key, L.tbits);
+    uint32_t s = lru_home(key, X.tbits);
     for (;;) {
-        const uint32_t e = L.tab[s];
-        if (e == 0) return -1;
-        if (L.key[e - 1] == key) return (int)(e - 1);
-        s = (s + 1) & L.mask;
+        const uint32_t e = X.tab[s];
+        if (e == 0) return kNone;
+        if (e != kTomb && X.K[e - 1] == key) {
+            *slot = s;
+            return e - 1;
+        }
+        s = (s + 1) & X.mask;
     }
 }
 
-__device__ __forceinline__ void list_insert_index(const lru_list &L, unsigned long long key, uint32_t node)
+// Claim an empty or evicted slot for an absent key; returns the slot.
+__device__ __forceinline__ uint32_t lru_insert(const lru_index &X, unsigned long long key, uint32_t pos)
 {
-    uint32_t s = home_slot(key, L.tbits);
-    while (atomicCAS(&L.tab[s], 0u, node + 1) != 0u) s = (s + 1) & L.mask;
+    unsigned short *t = reinterpret_cast<unsigned short *>(X.tab);
+    uint32_t s = lru_home(key, X.tbits);
+    for (;;) {
+        const unsigned short v = t[s];
+        if (v == 0 || v == kTomb) {
+            if (atomicCAS(&t[s], v, (unsigned short)(pos + 1)) == v) return s;
+            continue;  // lost the slot to another lane: look at it again
+        }
+        s = (s + 1) & X.mask;
+    }
 }
 
-// Remove the index entry of `node` (key `key`): backward-shift deletion for linear probing.
-__device__ __forceinline__ void list_erase_index(const lru_list &L, unsigned long long key, uint32_t node)
+// Index of K[0..fill) from scratch (warp-cooperative); clears every tombstone.
+__device__ __forceinline__ void lru_reindex(const lru_index &X, uint32_t fill, uint32_t lane)
 {
-    uint32_t i = home_slot(key, L.tbits);
-    while (L.tab[i] != node + 1) i = (i + 1) & L.mask;
-    uint32_t j = i;
-    for (;;) {
-        j = (j + 1) & L.mask;
-        const uint32_t e = L.tab[j];
-        if (e == 0) break;
-        const uint32_t k = home_slot(L.key[e - 1], L.tbits);
-        const bool stays = (i <= j) ? (i < k && k <= j) : (i < k || k <= j);
-        if (stays) continue;
-        L.tab[i] = e;
-        i = j;
-    }
-    L.tab[i] = 0;
+    uint4 *t4 = reinterpret_cast<uint4 *>(X.tab);
+    for (uint32_t x = lane; x < (X.mask + 1) / 8; x += 32) t4[x] = make_uint4(0, 0, 0, 0);
+    __syncwarp();
+    for (uint32_t p = lane; p < fill; p += 32) X.TS[p] = (uint16_t)lru_insert(X, X.K[p], p);
+    __syncwarp();
 }
 
 template <int NC>
 __global__ void __launch_bounds__(128)
-k_lru_list(const list_caps lc, uint32_t cmax, uint32_t R, uint32_t ns, uint32_t CL, int tbits,
-           const uint32_t *__restrict__ start, const uint32_t *__restrict__ coff, const uint32_t *__restrict__ total,
-           const rec16 *__restrict__ rec, const replay_state st, unsigned long long *__restrict__ ctr)
+k_lru_batch(const replay_caps caps, uint32_t cmax, uint32_t R, uint32_t ns, uint32_t CL, int tbits,
+            const uint32_t *__restrict__ start, const uint32_t *__restrict__ coff, const uint32_t *__restrict__ total,
+            const rec16 *__restrict__ rec, const replay_state st, unsigned long long *__restrict__ ctr)
 {
-    extern __shared__ unsigned long long smw[];
+    extern __shared__ uint4 smb[];
     const uint32_t lane = cr_lane(), warp = threadIdx.x >> 5, wpb = blockDim.x >> 5;
     const uint32_t tsz = 1u << tbits;
-    // per-warp region, 8-byte aligned pieces
-    const size_t per_warp = (size_t)cmax * 8 + (size_t)tsz * 4 + (((size_t)cmax * 5 + 7) & ~(size_t)7);
-    unsigned char *base = reinterpret_cast<unsigned char *>(smw) + per_warp * warp;
-    lru_list L;
-    L.key = reinterpret_cast<unsigned long long *>(base);
-    L.tab = reinterpret_cast<uint32_t *>(base + (size_t)cmax * 8);
-    L.prev = reinterpret_cast<uint16_t *>(base + (size_t)cmax * 8 + (size_t)tsz * 4);
-    L.next = L.prev + cmax;
-    L.seg = reinterpret_cast<uint8_t *>(L.next + cmax);
-    L.mask = tsz - 1;
-    L.tbits = tbits;
+    // per-warp region: index (2*tsz bytes), bitmap (128), keys (8*cmax), slots (2*cmax)
+    const size_t per_warp = ((size_t)tsz * 2 + 128 + (size_t)cmax * 10 + 15) & ~(size_t)15;
+    unsigned char *base = reinterpret_cast<unsigned char *>(smb) + per_warp * warp;
+    lru_index X;
+    X.tab = reinterpret_cast<uint16_t *>(base);
+    X.bm = reinterpret_cast<uint32_t *>(base + (size_t)tsz * 2);
+    X.K = reinterpret_cast<unsigned long long *>(base + (size_t)tsz * 2 + 128);
+    X.TS = reinterpret_cast<uint16_t *>(base + (size_t)tsz * 2 + 128 + (size_t)cmax * 8);
+    X.mask = tsz - 1;
+    X.tbits = tbits;
 
     const uint32_t w = blockIdx.x * wpb + warp;
     if (w >= *total) return;
@@ -485,7 +486,7 @@ k_lru_list(const list_caps lc, uint32_t cmax, uint32_t R, uint32_t ns, uint32_t 
     const uint32_t rep = s / R, r = s % R;
     const uint32_t fill_in = st.fill_in[s];
     const unsigned long long *kin = st.keys_in + (unsigned long long)s * cmax;
-    const uint32_t lt = (1u << lane) - 1u;
+    const uint32_t lt = (1u << lane) - 1u, gt = ~(lt | (1u << lane));
 
     if (b == e) {  // nothing routed here: carry the state over unchanged
         unsigned long long *kout = st.keys_out + (unsigned long long)s * cmax;
@@ -494,17 +495,16 @@ k_lru_list(const list_caps lc, uint32_t cmax, uint32_t R, uint32_t ns, uint32_t 
         return;
     }
 
-    // ---- state at p0, as keys in recency order in L.key[0..fill) ---------------
-    for (uint32_t x = lane; x < tsz; x += 32) L.tab[x] = 0;
-    __syncwarp();
+    // ---- state at p0 ------------------------------------------------------------
     uint32_t fill = 0;
     if (ci == 0) {
-        for (uint32_t q = lane; q < fill_in; q += 32) {
-            L.key[q] = kin[q];
-            list_insert_index(L, kin[q], q);
-        }
+        for (uint32_t q = lane; q < fill_in; q += 32) X.K[q] = kin[q];
         fill = fill_in;
+        __syncwarp();
+        lru_reindex(X, fill, lane);
     } else {
+        // walk backwards collecting distinct keys, most recent first
+        lru_reindex(X, 0, lane);
         const uint32_t back = p0 - b;
         const uint32_t vtot = back + fill_in;
         for (uint32_t v0 = 0; v0 < vtot && fill < cmax; v0 += 32) {
@@ -512,156 +512,165 @@ k_lru_list(const list_caps lc, uint32_t cmax, uint32_t R, uint32_t ns, uint32_t 
             const bool valid = v < vtot;
             unsigned long long key = 0;
             if (valid) key = v < back ? rec[p0 - 1 - v].key : kin[v - back];
-            const uint32_t peers = __match_any_sync(0xffffffffu, key);
-            const bool fresh = valid && (peers & lt) == 0 && list_find(L, key) < 0;
+            const uint32_t vm = __ballot_sync(0xffffffffu, valid);
+            const uint32_t peers = __match_any_sync(0xffffffffu, key) & vm;
+            uint32_t sl;
+            const bool fresh = valid && (peers & lt) == 0 && lru_lookup(X, key, &sl) == kNone;
             const uint32_t bal = __ballot_sync(0xffffffffu, fresh);
-            const uint32_t rank = __popc(bal & lt);
+            const uint32_t pos = fill + __popc(bal & lt);
             __syncwarp();
-            if (fresh && fill + rank < cmax) {
-                L.key[fill + rank] = key;
-                list_insert_index(L, key, fill + rank);
+            if (fresh && pos < cmax) {
+                X.K[pos] = key;
+                X.TS[pos] = (uint16_t)lru_insert(X, key, pos);
             }
             fill = min(cmax, fill + (uint32_t)__popc(bal));
             __syncwarp();
         }
     }
-    // links and segments of the recency order 0..fill-1
-    for (uint32_t q = lane; q < fill; q += 32) {
-        L.prev[q] = q == 0 ? kNil : (uint16_t)(q - 1);
-        L.next[q] = q + 1 == fill ? kNil : (uint16_t)(q + 1);
-        uint32_t sg = 0;
-        while (sg + 1 < lc.m && q + 1 > lc.c[sg]) ++sg;
-        L.seg[q] = (uint8_t)sg;
-    }
-    __syncwarp();
 
     unsigned long long my_req = 0, my_prompt = 0;
-    unsigned long long hitc[NC], hitt[NC];
+    unsigned long long my_hit[NC], my_tok[NC];
 #pragma unroll
-    for (int j = 0; j < NC; ++j) hitc[j] = hitt[j] = 0;
-    // simulator registers (meaningful in lane 0)
-    uint32_t head = fill ? 0u : kNil, tail = fill ? fill - 1 : kNil;
-    uint32_t B[NC];
-#pragma unroll
-    for (int j = 0; j < NC; ++j) B[j] = (j + 1 < (int)lc.m && fill >= lc.c[j]) ? lc.c[j] - 1 : kNil;
+    for (int c = 0; c < NC; ++c) my_hit[c] = my_tok[c] = 0;
+    const uint32_t nwords = (cmax + 31) / 32;
+    uint32_t tomb = 0;  // tombstones in the index
 
     for (uint32_t t0 = p0; t0 < p1; t0 += 32) {
-        // the warp stages 32 requests; lane 0 simulates them in order
+        const uint32_t cnt = (p1 - t0) < 32u ? (p1 - t0) : 32u;
+        const bool valid = lane < cnt;
         rec16 mine = {0ull, 0u, 0u};
-        if (t0 + lane < p1) {
+        if (valid) {
             mine = rec[t0 + lane];
             my_req += 1;
             my_prompt += (unsigned long long)mine.P + mine.S;
         }
-        const uint32_t cnt = (p1 - t0) < 32u ? (p1 - t0) : 32u;
-        for (uint32_t jq = 0; jq < cnt; ++jq) {
-            const unsigned long long key = __shfl_sync(0xffffffffu, mine.key, jq);
-            const uint32_t P = __shfl_sync(0xffffffffu, mine.P, jq);
-            if (lane == 0) {
-                const int n = list_find(L, key);
-                if (n >= 0) {
-                    const uint32_t sg = L.seg[n];
+        const uint32_t vm = cnt == 32 ? 0xffffffffu : (1u << cnt) - 1u;
+        const uint32_t grp = __match_any_sync(0xffffffffu, mine.key) & vm;
+        const uint32_t below = grp & lt, above = grp & gt;
+        const bool first = valid && below == 0;
+        const uint32_t next = above ? (uint32_t)__ffs(above) - 1u : 32u;
+        uint32_t slot0 = kNone;
+        const uint32_t d0 = first ? lru_lookup(X, mine.key, &slot0) : kNone;
+        // one ballot per request whose depth is finite: lanes that push it deeper
+        const uint32_t need = __ballot_sync(0xffffffffu, valid && (!first || d0 != kNone));
+        const uint32_t enc = first ? d0 : kNone;  // kNone: a repeat within the batch
+        uint32_t pushed = 0;
+        for (uint32_t m = need; m; m &= m - 1) {
+            const uint32_t i = (uint32_t)__ffs(m) - 1u;
+            const uint32_t di = __shfl_sync(0xffffffffu, enc, i);
+            const bool pr = di == kNone ? next > i : (first && d0 > di);
+            const uint32_t bl = __ballot_sync(0xffffffffu, pr);
+            if (lane == i) pushed = bl;
+        }
+        uint32_t depth = kNone;
+        if (valid) {
+            if (!first) {
+                const uint32_t prev = 31u - (uint32_t)__clz(below);
+                depth = 1u + (uint32_t)__popc(pushed & lt & ~((2u << prev) - 1u));
+            } else if (d0 != kNone) {
+                depth = d0 + 1u + (uint32_t)__popc(pushed & lt);
+            }
+        }
 #pragma unroll
-                    for (int j = 0; j < NC; ++j) {
-                        if (j < (int)lc.m && (uint32_t)j >= sg) {
-                            hitc[j] += 1;
-                            hitt[j] += P;
-                        }
-                    }
-                    if ((uint32_t)n != head) {
-                        const uint32_t pn = L.prev[n];
+        for (int c = 0; c < NC; ++c) {
+            if (c < (int)caps.n_caps && depth <= caps.cap[c]) {
+                my_hit[c] += 1;
+                my_tok[c] += mine.P;
+            }
+        }
+
+        // ---- state after the batch ------------------------------------------------
+        const uint32_t lastm = __ballot_sync(0xffffffffu, valid && above == 0);
+        const uint32_t u = (uint32_t)__popc(lastm);
+        if (lane < nwords) X.bm[lane] = 0;
+        __syncwarp();
+        if (d0 != kNone) atomicOr(&X.bm[d0 >> 5], 1u << (d0 & 31));
+        __syncwarp();
+        const uint32_t wv = lane < nwords ? X.bm[lane] : 0u;
+        uint32_t pre = (uint32_t)__popc(wv);  // inclusive prefix over words
 #pragma unroll
-                        for (int j = 0; j < NC; ++j) {
-                            if (j + 1 < (int)lc.m) {
-                                if ((uint32_t)j < sg) {
-                                    L.seg[B[j]] = (uint8_t)(j + 1);
-                                    B[j] = lc.c[j] == 1 ? (uint32_t)n : L.prev[B[j]];
-                                } else if ((uint32_t)j == sg && B[j] == (uint32_t)n) {
-                                    B[j] = pn;
-                                }
-                            }
-                        }
-                        // unlink n, push it to the front
-                        const uint32_t nx = L.next[n];
-                        L.next[pn] = (uint16_t)nx;
-                        if (nx != kNil)
-                            L.prev[nx] = (uint16_t)pn;
-                        else
-                            tail = pn;
-                        L.prev[n] = kNil;
-                        L.next[n] = (uint16_t)head;
-                        L.prev[head] = (uint16_t)n;
-                        head = (uint32_t)n;
-                        L.seg[n] = 0;
-                    }
-                } else {
-                    uint32_t node;
-                    const uint32_t old_fill = fill;
-                    // every resident entry moves back one position
-#pragma unroll
-                    for (int j = 0; j < NC; ++j) {
-                        if (j + 1 < (int)lc.m && B[j] != kNil) {
-                            L.seg[B[j]] = (uint8_t)(j + 1);
-                            B[j] = L.prev[B[j]];  // kNil when c_j == 1: the new entry, set below
-                        }
-                    }
-                    if (fill == cmax) {
-                        node = tail;
-                        list_erase_index(L, L.key[node], node);
-                        tail = L.prev[node];
-                        if (tail != kNil) L.next[tail] = kNil;
-                        if (head == node) head = kNil;
-                    } else {
-                        node = fill++;
-                    }
-                    L.key[node] = key;
-                    L.seg[node] = 0;
-                    L.prev[node] = kNil;
-                    L.next[node] = (uint16_t)head;
-                    if (head != kNil) L.prev[head] = (uint16_t)node;
-                    head = node;
-                    if (tail == kNil) tail = node;
-                    list_insert_index(L, key, node);
-#pragma unroll
-                    for (int j = 0; j < NC; ++j) {
-                        if (j + 1 < (int)lc.m) {
-                            if (B[j] == kNil && old_fill >= lc.c[j]) B[j] = node;    // c_j == 1
-                            if (old_fill < lc.c[j] && fill == lc.c[j]) B[j] = tail;  // boundary now defined
-                        }
-                    }
-                }
+        for (int o = 1; o < 32; o <<= 1) {
+            const uint32_t y = __shfl_up_sync(0xffffffffu, pre, o);
+            if (lane >= (uint32_t)o) pre += y;
+        }
+        const uint32_t touched = __shfl_sync(0xffffffffu, pre, 31);
+        pre -= (uint32_t)__popc(wv);  // exclusive
+        // untouched old keys move back (never forward): highest block first, in
+        // place; each rewrites its index slot, evicted ones leave a tombstone
+        uint32_t evicted = 0;
+        for (int tb = (int)((fill + 31) / 32) - 1; tb >= 0; --tb) {
+            const uint32_t p = (uint32_t)tb * 32u + lane;
+            const uint32_t wt = __shfl_sync(0xffffffffu, wv, tb), pt = __shfl_sync(0xffffffffu, pre, tb);
+            unsigned long long v = 0;
+            uint32_t np = kNone, ts = 0;
+            if (p < fill && !((wt >> lane) & 1u)) {
+                v = X.K[p];
+                ts = X.TS[p];
+                np = p + u - (pt + (uint32_t)__popc(wt & lt));
             }
             __syncwarp();
+            if (np < cmax) {
+                X.K[np] = v;
+                X.TS[np] = (uint16_t)ts;
+                X.tab[ts] = (uint16_t)(np + 1);
+            } else if (np != kNone) {
+                X.tab[ts] = kTomb;
+                ++evicted;
+            }
+        }
+        __syncwarp();
+        // the batch's distinct keys go to the front; a key already resident keeps
+        // its slot (taken from the lane of its first occurrence), a new one claims one
+        const uint32_t fl = (uint32_t)__ffs(grp ? grp : 1u) - 1u;
+        const uint32_t kslot = __shfl_sync(0xffffffffu, slot0, fl);
+        const uint32_t rank = (uint32_t)__popc(lastm & gt);
+        if (valid && above == 0) {
+            if (kslot != kNone) {
+                if (rank < cmax) {
+                    X.K[rank] = mine.key;
+                    X.TS[rank] = (uint16_t)kslot;
+                    X.tab[kslot] = (uint16_t)(rank + 1);
+                } else {
+                    X.tab[kslot] = kTomb;
+                    ++evicted;
+                }
+            } else if (rank < cmax) {
+                X.K[rank] = mine.key;
+                X.TS[rank] = (uint16_t)lru_insert(X, mine.key, rank);
+            }
+        }
+        fill = min(cmax, fill - touched + u);
+        tomb += __reduce_add_sync(0xffffffffu, evicted);
+        __syncwarp();
+        if (4 * (fill + tomb) > 3 * (X.mask + 1)) {  // too many tombstones: index afresh
+            lru_reindex(X, fill, lane);
+            tomb = 0;
         }
     }
 
     // ---- counters -------------------------------------------------------------
     my_req = cr_warp_sum_u64(my_req);
     my_prompt = cr_warp_sum_u64(my_prompt);
-    if (lane == 0) {
-        // hand the state to the next call, most recent first
-        if (p1 == e) {
-            unsigned long long *kout = st.keys_out + (unsigned long long)s * cmax;
-            uint32_t q = 0;
-            for (uint32_t x = head; x != kNil; x = L.next[x]) kout[q++] = L.key[x];
-            st.fill_out[s] = fill;
-        }
-        for (uint32_t oi = 0; oi < lc.n_out; ++oi) {
-            const uint32_t j = lc.seg_of[oi];
-            unsigned long long h = 0, tk = 0;
 #pragma unroll
-            for (int jj = 0; jj < NC; ++jj)
-                if ((uint32_t)jj == j) {
-                    h = hitc[jj];
-                    tk = hitt[jj];
-                }
-            unsigned long long *C = ctr + (((unsigned long long)rep * lc.n_out + oi) * R + r) * CR_CTR_FIELDS;
-            atomicAdd(&C[0], my_req);
-            if (h) atomicAdd(&C[1], h);
-            if (tk) atomicAdd(&C[2], tk);
-            atomicAdd(&C[3], my_prompt);
-            atomicAdd(&C[4], my_prompt - tk);
+    for (int c = 0; c < NC; ++c) {
+        if (c < (int)caps.n_caps) {
+            const unsigned long long h = cr_warp_sum_u64(my_hit[c]);
+            const unsigned long long tk = cr_warp_sum_u64(my_tok[c]);
+            if (lane == 0) {
+                unsigned long long *C = ctr + (((unsigned long long)rep * caps.n_caps + c) * R + r) * CR_CTR_FIELDS;
+                atomicAdd(&C[0], my_req);
+                if (h) atomicAdd(&C[1], h);
+                if (tk) atomicAdd(&C[2], tk);
+                atomicAdd(&C[3], my_prompt);
+                atomicAdd(&C[4], my_prompt - tk);
+            }
         }
+    }
+    // ---- the stream's last chunk hands the state to the next call, most recent first
+    if (p1 == e) {
+        unsigned long long *kout = st.keys_out + (unsigned long long)s * cmax;
+        for (uint32_t q = lane; q < fill; q += 32) kout[q] = X.K[q];
+        if (lane == 0) st.fill_out[s] = fill;
     }
 }
 
@@ -697,58 +706,36 @@ int launch_replay(cr_ctx *ctx, cr_replay *rp, const replay_caps &caps, uint32_t 
 }
 
 template <int NC>
-int launch_list_nc(cr_ctx *ctx, cr_replay *rp, const list_caps &lc, uint32_t CL, int tbits, const uint32_t *start,
-                   const uint32_t *coff, const uint32_t *total, uint64_t m, const rec16 *rec, uint64_t *d_ctr)
+int launch_batch_nc(cr_ctx *ctx, cr_replay *rp, const replay_caps &caps, uint32_t CL, const uint32_t *start,
+                    const uint32_t *coff, const uint32_t *total, uint64_t m, const rec16 *rec, uint64_t *d_ctr)
 {
-    const uint32_t cmax = rp->cmax, tsz = 1u << tbits;
-    const size_t per_warp = (size_t)cmax * 8 + (size_t)tsz * 4 + (((size_t)cmax * 5 + 7) & ~(size_t)7);
-    uint32_t wpb = 4;
-    while (wpb > 1 && per_warp * wpb > 200 * 1024) wpb >>= 1;
+    const uint32_t cmax = rp->cmax;
+    int tbits = 6;
+    while ((1u << tbits) < 2 * cmax) ++tbits;
+    const size_t per_warp = ((size_t)(1u << tbits) * 2 + 128 + (size_t)cmax * 10 + 15) & ~(size_t)15;
+    const uint32_t wpb = 4;
     const size_t smem = per_warp * wpb;
     if (smem > 48 * 1024)
-        CR_CUDA(ctx, cudaFuncSetAttribute(k_lru_list<NC>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
+        CR_CUDA(ctx, cudaFuncSetAttribute(k_lru_batch<NC>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
     const uint32_t ns = rp->n_rep * rp->R;
-    const uint64_t items = (uint64_t)ns + (m + CL - 1) / CL;
+    const uint64_t items = (uint64_t)ns + (m + CL - 1) / CL;  // upper bound on work items
     replay_state st;
     st.keys_in = rp->d_keys[rp->cur];
     st.fill_in = rp->d_fill[rp->cur];
     st.keys_out = rp->d_keys[rp->cur ^ 1];
     st.fill_out = rp->d_fill[rp->cur ^ 1];
-    CR_LAUNCH(ctx, k_lru_list<NC>, (unsigned int)((items + wpb - 1) / wpb), wpb * 32, smem, lc, cmax, rp->R, ns, CL,
-              tbits, start, coff, total, rec, st, (unsigned long long *)d_ctr);
+    CR_LAUNCH(ctx, k_lru_batch<NC>, (unsigned int)((items + wpb - 1) / wpb), wpb * 32, smem, caps, cmax, rp->R, ns,
+              CL, tbits, start, coff, total, rec, st, (unsigned long long *)d_ctr);
     rp->cur ^= 1;
     return CR_OK;
 }
 
-int launch_list(cr_ctx *ctx, cr_replay *rp, uint32_t CL, const uint32_t *start, const uint32_t *coff,
-                const uint32_t *total, uint64_t m, const rec16 *rec, uint64_t *d_ctr)
+int launch_batch(cr_ctx *ctx, cr_replay *rp, const replay_caps &caps, uint32_t CL, const uint32_t *start,
+                 const uint32_t *coff, const uint32_t *total, uint64_t m, const rec16 *rec, uint64_t *d_ctr)
 {
-    list_caps lc;
-    memset(&lc, 0, sizeof(lc));
-    uint32_t sorted[CR_MAX_CAPS];
-    uint32_t ns_ = 0;
-    for (uint32_t i = 0; i < rp->n_caps; ++i) {
-        bool dup = false;
-        for (uint32_t j = 0; j < ns_; ++j) dup |= sorted[j] == rp->caps[i];
-        if (!dup) sorted[ns_++] = rp->caps[i];
-    }
-    for (uint32_t i = 1; i < ns_; ++i)
-        for (uint32_t j = i; j > 0 && sorted[j - 1] > sorted[j]; --j) {
-            uint32_t t = sorted[j];
-            sorted[j] = sorted[j - 1];
-            sorted[j - 1] = t;
-        }
-    lc.m = ns_;
-    for (uint32_t j = 0; j < ns_; ++j) lc.c[j] = sorted[j];
-    lc.n_out = rp->n_caps;
-    for (uint32_t i = 0; i < rp->n_caps; ++i)
-        for (uint32_t j = 0; j < ns_; ++j)
-            if (sorted[j] == rp->caps[i]) lc.seg_of[i] = j;
-    int tbits = 0;
-    while ((1u << tbits) < 2 * rp->cmax) ++tbits;
-    if (lc.m <= 1) return launch_list_nc<1>(ctx, rp, lc, CL, tbits, start, coff, total, m, rec, d_ctr);
-    if (lc.m <= 3) return launch_list_nc<3>(ctx, rp, lc, CL, tbits, start, coff, total, m, rec, d_ctr);
-    return launch_list_nc<CR_MAX_CAPS>(ctx, rp, lc, CL, tbits, start, coff, total, m, rec, d_ctr);
+    if (caps.n_caps == 1) return launch_batch_nc<1>(ctx, rp, caps, CL, start, coff, total, m, rec, d_ctr);
+    if (caps.n_caps <= 3) return launch_batch_nc<3>(ctx, rp, caps, CL, start, coff, total, m, rec, d_ctr);
+    return launch_batch_nc<CR_MAX_CAPS>(ctx, rp, caps, CL, start, coff, total, m, rec, d_ctr);
 }
 
 }  // namespace
@@ -855,8 +842,8 @@ extern "C" int cr_shadow_replay(cr_ctx *ctx, cr_replay *rp, const uint64_t *d_ke
     CR_LAUNCH(ctx, k_chunk_counts, cr_blocks(ns, 256, gcap), 256, 0, (const uint32_t *)start, ns, CL, coff);
     CR_TRY(cr_scan_u32(ctx, coff, coff, ns, total));
     const uint32_t E = (rp->cmax + 31) / 32;
-    // capacities up to 32: one entry per lane in registers; above: linked list + hash index
-    if (E > 1) return launch_list(ctx, rp, CL, start, coff, total, m, rec, d_ctr);
+    // capacities up to 32: one entry per lane in registers; above: batched stack distances
+    if (E > 1) return launch_batch(ctx, rp, caps, CL, start, coff, total, m, rec, d_ctr);
     return launch_replay<1>(ctx, rp, caps, CL, start, coff, total, m, rec, d_ctr);
 }
 
