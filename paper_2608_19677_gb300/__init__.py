@@ -232,7 +232,9 @@ class Plan:
 def plan_params(R: int, W: int, qcap_num: int, qcap_den: int, variant="LPT", seed: int = 0, epoch: int = 0,
                 init_load=None) -> PlanParams:
     v = VARIANT[variant] if isinstance(variant, str) else int(variant)
-    return PlanParams(R, W, qcap_num, qcap_den, v, 0, seed & ((1 << 64) - 1), epoch, _ptr(init_load))
+    p = PlanParams(R, W, qcap_num, qcap_den, v, 0, seed & ((1 << 64) - 1), epoch, _ptr(init_load))
+    p._init_load = init_load  # the device vector must outlive the parameters that point at it
+    return p
 
 
 def build_plans(ctx: Context, keys, params: Sequence[PlanParams], plans: Sequence[Plan]):

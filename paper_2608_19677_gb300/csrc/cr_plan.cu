@@ -554,6 +554,147 @@ __device__ __forceinline__ unsigned long long reg_min(const unsigned long long (
     return t[0];
 }
 
+// Runs of keys with k_b = 1 and equal λ = q (Algorithm 1's loop over such a
+// run, done at once).  Each greedy pick is a current minimum (L_r, r) and
+// raising it by q keeps later picks no smaller, so the m picks are the m
+// smallest pairs (L_r + j q, r), j >= 0.  With L_r = q l_r + f_r (0 <= f_r < q)
+// pair (r, j) sorts by (l_r + j, f_r, r): picks come in rounds t = l_r + j,
+// each visiting {r : l_r <= t} in (f_r, r) order.  Between two consecutive
+// distinct levels l the visited set is fixed, so that stretch of rounds cycles
+// through it.  Cost: one pass over R per distinct level reached, plus the
+// output writes, instead of one warp minimum per key.
+struct lpt_run_smem {
+    uint16_t order[1024];  // destinations by (f_r, r)
+    uint16_t cyc[1024];    // destinations visited in the current stretch, in that order
+    uint32_t lev[1024];    // l_r
+    uint32_t add[1024];    // jobs given to r in this run; first q buckets reused for the sort
+};
+
+template <int NE>
+__device__ __forceinline__ bool lpt_equal_run(unsigned long long (&v)[NE], uint32_t R, unsigned long long q,
+                                              unsigned long long m, uint32_t base, uint16_t *__restrict__ members,
+                                              unsigned long long *__restrict__ jobs, lpt_run_smem &S,
+                                              bool &overflow)
+{
+    const uint32_t lane = cr_lane(), lt = (1u << lane) - 1u;
+    if (q == 0 || q > 1024) return false;
+    unsigned long long lmax = 0;
+#pragma unroll
+    for (int j = 0; j < NE; ++j)
+        if (lane + 32u * j < R) lmax = max(lmax, v[j] >> 16);
+    if (~cr_warp_min_u64(~lmax) >= (1ull << 31)) return false;  // levels in 32 bits
+    const uint32_t q32 = (uint32_t)q;
+    // counting sort by phase f_r, stable in r
+    for (uint32_t x = lane; x < q32; x += 32) S.add[x] = 0;
+    __syncwarp();
+#pragma unroll
+    for (int j = 0; j < NE; ++j) {
+        const uint32_t r = lane + 32u * j;
+        if (r < R) {
+            const uint32_t L = (uint32_t)(v[j] >> 16);
+            S.lev[r] = L / q32;
+            atomicAdd(&S.add[L % q32], 1u);
+        }
+    }
+    __syncwarp();
+    {
+        const uint32_t per = (q32 + 31) / 32, x0 = lane * per;
+        uint32_t run = 0;
+        for (uint32_t x = x0; x < x0 + per && x < q32; ++x) run += S.add[x];
+        uint32_t inc = run;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const uint32_t y = __shfl_up_sync(0xffffffffu, inc, o);
+            if (lane >= (uint32_t)o) inc += y;
+        }
+        uint32_t off = inc - run;
+        __syncwarp();
+        for (uint32_t x = x0; x < x0 + per && x < q32; ++x) {
+            const uint32_t c = S.add[x];
+            S.add[x] = off;
+            off += c;
+        }
+    }
+    __syncwarp();
+#pragma unroll
+    for (int j = 0; j < NE; ++j) {
+        const uint32_t r = lane + 32u * j;
+        const uint32_t f = r < R ? (uint32_t)(v[j] >> 16) % q32 : 0xffffffffu;
+        const uint32_t peers = __match_any_sync(0xffffffffu, f);
+        const uint32_t at = r < R ? S.add[f] : 0u;
+        __syncwarp();
+        if (r < R) {
+            S.order[at + __popc(peers & lt)] = (uint16_t)r;
+            if ((peers & lt) == 0) S.add[f] = at + __popc(peers);
+        }
+        __syncwarp();
+    }
+    for (uint32_t x = lane; x < R; x += 32) S.add[x] = 0;
+    __syncwarp();
+    // stretches of rounds between consecutive distinct levels
+    uint32_t T = 0xffffffffu;
+#pragma unroll
+    for (int j = 0; j < NE; ++j)
+        if (lane + 32u * j < R) T = min(T, S.lev[lane + 32u * j]);
+    T = __reduce_min_sync(0xffffffffu, T);
+    unsigned long long left = m, done = 0;
+    while (left) {
+        uint32_t n_in = 0, nxt = 0xffffffffu;
+#pragma unroll
+        for (int j = 0; j < NE; ++j) {
+            const uint32_t r = lane + 32u * j;
+            if (r < R) {
+                const uint32_t l = S.lev[r];
+                n_in += l <= T ? 1u : 0u;
+                if (l > T) nxt = min(nxt, l);
+            }
+        }
+        n_in = __reduce_add_sync(0xffffffffu, n_in);
+        nxt = __reduce_min_sync(0xffffffffu, nxt);
+        unsigned long long cnt = left;
+        if (nxt != 0xffffffffu && (unsigned long long)n_in * (nxt - T) < left)
+            cnt = (unsigned long long)n_in * (nxt - T);
+        const unsigned long long full = cnt / n_in;
+        const uint32_t part = (uint32_t)(cnt % n_in);
+        uint32_t seen = 0;
+        for (uint32_t p0 = 0; p0 < R; p0 += 32) {
+            const uint32_t p = p0 + lane;
+            const uint32_t r = p < R ? S.order[p] : 0u;
+            const bool in = p < R && S.lev[r] <= T;
+            const uint32_t bal = __ballot_sync(0xffffffffu, in);
+            if (in) {
+                const uint32_t k = seen + __popc(bal & lt);
+                S.cyc[k] = (uint16_t)r;
+                S.add[r] += (uint32_t)full + (k < part ? 1u : 0u);
+            }
+            seen += __popc(bal);
+        }
+        __syncwarp();
+        unsigned long long i = lane, ci = lane % n_in;
+        const uint32_t step = 32u % n_in;
+        for (; i < cnt; i += 32) {
+            members[base + done + i] = S.cyc[ci];
+            jobs[base + done + i] = q;
+            ci += step;
+            if (ci >= n_in) ci -= n_in;
+        }
+        __syncwarp();
+        done += cnt;
+        left -= cnt;
+        T = nxt;
+    }
+#pragma unroll
+    for (int j = 0; j < NE; ++j) {
+        const uint32_t r = lane + 32u * j;
+        if (r < R) {
+            v[j] += ((unsigned long long)S.add[r] * q) << 16;
+            if ((v[j] >> 16) >= kLoadLimit) overflow = true;
+        }
+    }
+    __syncwarp();
+    return true;
+}
+
 template <int NE>
 __global__ void __launch_bounds__(32) k_plan_lpt_reg(const __grid_constant__ lpt_jobs jobs_in, uint32_t *status)
 {
@@ -571,16 +712,48 @@ __global__ void __launch_bounds__(32) k_plan_lpt_reg(const __grid_constant__ lpt
     bool overflow = false;
     unsigned long long st_lam = 0;
     uint32_t st_k = 0, st_off = 0;
+    __shared__ lpt_run_smem S;
+    unsigned long long stage = 0;  // first key of the 32 staged in st_*
     for (unsigned long long a = 0; a < na; ++a) {
-        const uint32_t slot = (uint32_t)(a & 31ull);
-        if (slot == 0) {
+        if (a == 0 || a - stage >= 32) {
+            stage = a;
             const unsigned long long ia = a + lane;
             if (ia < na) {
                 st_lam = J.adm_cnt[ia];
                 st_k = J.adm_k[ia];
                 st_off = J.koff[ia];
             }
+            // a run of >= 32 keys with k = 1 and equal λ starts here: place it at once
+            const uint32_t k0 = __shfl_sync(0xffffffffu, st_k, 0);
+            const unsigned long long l0 = __shfl_sync(0xffffffffu, st_lam, 0);
+            const unsigned long long l31 = __shfl_sync(0xffffffffu, st_lam, 31);
+            if (k0 == 1 && a + 31 < na && l31 == l0) {
+                // end of the run: first index after a whose λ differs (λ is non-increasing)
+                unsigned long long lo = a + 31, hi = na;  // adm_cnt[lo] == l0; answer in (lo, hi]
+                while (hi - lo > 1) {
+                    const unsigned long long span = hi - lo;
+                    const unsigned long long pr = lo + 1 + (span - 1) * lane / 32;  // 32 probes in (lo, hi)
+                    const bool differs = J.adm_cnt[pr] != l0;
+                    const uint32_t bl = __ballot_sync(0xffffffffu, differs);
+                    if (!bl) {
+                        lo = __shfl_sync(0xffffffffu, pr, 31);
+                    } else {
+                        const uint32_t f = __ffs(bl) - 1;
+                        hi = __shfl_sync(0xffffffffu, pr, f);
+                        if (f > 0) lo = __shfl_sync(0xffffffffu, pr, f - 1);
+                    }
+                }
+                const unsigned long long runm = hi - a;
+                const uint32_t base0 = __shfl_sync(0xffffffffu, st_off, 0);
+                if (lpt_equal_run<NE>(v, R, l0, runm, base0, J.members, J.jobs, S, overflow)) {
+                    a = hi - 1;      // the loop's ++a moves to the first key after the run
+                    stage = a + 1 - 32;  // forces a restage at hi
+                    m = reg_min<NE>(v, 0u);
+                    continue;
+                }
+            }
         }
+        const uint32_t slot = (uint32_t)(a - stage);
         const uint32_t k = __shfl_sync(0xffffffffu, st_k, slot);
         const uint32_t base = __shfl_sync(0xffffffffu, st_off, slot);
         const unsigned long long lam = __shfl_sync(0xffffffffu, st_lam, slot);

@@ -136,6 +136,30 @@ def test_plan_parity(P, ctx, seed):
         _cmp_plan(got, O.build_plan(keys, R, W, num, den, variant=v, seed=seed, epoch=3))
 
 
+@pytest.mark.parametrize("R,spread", [(33, 0), (64, 50), (257, 3), (1024, 0), (1024, 400)])
+def test_plan_equal_rate_runs(P, ctx, R, spread):
+    # long runs of keys with the same count and k = 1 (placed a run at a time on
+    # the device), hot replicated keys before them, short runs, runs with
+    # counts above 1024, and uneven starting loads
+    rng = np.random.default_rng(R + spread)
+    counts = [3000] * 2 + [1500] * 3 + [1100] * 40 + [37] * 70 + [5] * 300 + [2] * 900 + [1] * 5000
+    counts += list(rng.integers(1, 60, size=200))
+    ks = np.unique(rng.integers(0, 2**64 - 1, size=len(counts) + 64, dtype=np.uint64))[:len(counts)]
+    rng.shuffle(ks)
+    keys = np.repeat(ks, counts)
+    rng.shuffle(keys)
+    init = None
+    if spread:
+        init = rng.integers(0, spread + 1, size=R).astype(np.uint64)
+    W = 2 + 6500 // R
+    params = [P.plan_params(R, W, 2000, 1, v, init_load=None if init is None else d_u64(init))
+              for v in ("LPT", "NOREPL")]
+    plans = [P.Plan(ctx) for _ in params]
+    P.build_plans(ctx, d_u64(keys), params, plans)
+    for pl, v in zip(plans, ("LPT", "NOREPL")):
+        _cmp_plan(pl.export(), O.build_plan(keys, R, W, 2000, 1, variant=v, init_load=init))
+
+
 def test_plan_hand_example_and_init_load(P, ctx):
     keys = np.array([1] * 21 + [2] * 6 + [3] * 3 + [4], np.uint64)
     pl = P.build_plan(ctx, d_u64(keys), P.plan_params(3, 1, 155, 12))
