@@ -535,12 +535,14 @@ k_lru_batch(const replay_caps caps, uint32_t cmax, uint32_t R, uint32_t ns, uint
     const uint32_t nwords = (cmax + 31) / 32;
     uint32_t tomb = 0;  // tombstones in the index
 
+    rec16 ahead = {0ull, 0u, 0u};  // the next batch's records, loaded one batch early
+    if (p0 + lane < p1) ahead = rec[p0 + lane];
     for (uint32_t t0 = p0; t0 < p1; t0 += 32) {
         const uint32_t cnt = (p1 - t0) < 32u ? (p1 - t0) : 32u;
         const bool valid = lane < cnt;
-        rec16 mine = {0ull, 0u, 0u};
+        const rec16 mine = ahead;
+        if (t0 + 32u + lane < p1) ahead = rec[t0 + 32u + lane];
         if (valid) {
-            mine = rec[t0 + lane];
             my_req += 1;
             my_prompt += (unsigned long long)mine.P + mine.S;
         }
@@ -551,26 +553,33 @@ k_lru_batch(const replay_caps caps, uint32_t cmax, uint32_t R, uint32_t ns, uint
         const uint32_t next = above ? (uint32_t)__ffs(above) - 1u : 32u;
         uint32_t slot0 = kNone;
         const uint32_t d0 = first ? lru_lookup(X, mine.key, &slot0) : kNone;
-        // one ballot per request whose depth is finite: lanes that push it deeper
-        const uint32_t need = __ballot_sync(0xffffffffu, valid && (!first || d0 != kNone));
-        const uint32_t enc = first ? d0 : kNone;  // kNone: a repeat within the batch
-        uint32_t pushed = 0;
-        for (uint32_t m = need; m; m &= m - 1) {
-            const uint32_t i = (uint32_t)__ffs(m) - 1u;
-            const uint32_t di = __shfl_sync(0xffffffffu, enc, i);
-            const bool pr = di == kNone ? next > i : (first && d0 > di);
-            const uint32_t bl = __ballot_sync(0xffffffffu, pr);
-            if (lane == i) pushed = bl;
-        }
-        uint32_t depth = kNone;
-        if (valid) {
-            if (!first) {
-                const uint32_t prev = 31u - (uint32_t)__clz(below);
-                depth = 1u + (uint32_t)__popc(pushed & lt & ~((2u << prev) - 1u));
-            } else if (d0 != kNone) {
-                depth = d0 + 1u + (uint32_t)__popc(pushed & lt);
+        // lanes that push request i deeper, for every lane at once, by comparing
+        // bit-sliced values from the most significant bit down (per bit: lanes
+        // still equal keep the ones with the same bit; a lane whose bit is 1
+        // where this lane's is 0 is decided greater):
+        //   repeat i: lanes whose key does not recur before i (next_l > i);
+        //   first i:  first occurrences whose old position is deeper (D_l > D_i)
+        const uint32_t D = first ? (d0 < cmax ? d0 : 2047u) : 2047u;  // 2047: absent
+        uint32_t gN = 0, eN = 0xffffffffu, gD = 0, eD = 0xffffffffu;
+#pragma unroll
+        for (int bt = 10; bt >= 0; --bt) {
+            const uint32_t BD = __ballot_sync(0xffffffffu, (D >> bt) & 1u);
+            const uint32_t MD = 0u - ((D >> bt) & 1u);
+            gD |= eD & BD & ~MD;
+            eD &= ~(BD ^ MD);
+            if (bt <= 5) {
+                const uint32_t BN = __ballot_sync(0xffffffffu, (next >> bt) & 1u);
+                const uint32_t MN = 0u - ((lane >> bt) & 1u);
+                gN |= eN & BN & ~MN;
+                eN &= ~(BN ^ MN);
             }
         }
+        const uint32_t firstm = __ballot_sync(0xffffffffu, first);
+        // repeat: lanes strictly between the previous occurrence and this one
+        const uint32_t win = lt & ~((2u << (31u - (uint32_t)__clz(below | 1u))) - 1u);
+        const uint32_t dep_rep = 1u + (uint32_t)__popc(gN & win);
+        const uint32_t dep_first = d0 < cmax ? d0 + 1u + (uint32_t)__popc(gD & firstm & lt) : kNone;
+        const uint32_t depth = !valid ? kNone : (first ? dep_first : dep_rep);
 #pragma unroll
         for (int c = 0; c < NC; ++c) {
             if (c < (int)caps.n_caps && depth <= caps.cap[c]) {
@@ -713,7 +722,17 @@ int launch_batch_nc(cr_ctx *ctx, cr_replay *rp, const replay_caps &caps, uint32_
     int tbits = 6;
     while ((1u << tbits) < 2 * cmax) ++tbits;
     const size_t per_warp = ((size_t)(1u << tbits) * 2 + 128 + (size_t)cmax * 10 + 15) & ~(size_t)15;
-    const uint32_t wpb = 4;
+    // warps per block: the most warps per SM that shared memory allows
+    const size_t sm_bytes = 227 * 1024;
+    uint32_t wpb = 4, best = 0;
+    for (uint32_t x = 4; x >= 1; --x) {
+        const size_t blk = per_warp * x + 1024;
+        const uint32_t nb = blk <= sm_bytes ? (uint32_t)(sm_bytes / blk) : 0u;
+        if (nb * x > best) {
+            best = nb * x;
+            wpb = x;
+        }
+    }
     const size_t smem = per_warp * wpb;
     if (smem > 48 * 1024)
         CR_CUDA(ctx, cudaFuncSetAttribute(k_lru_batch<NC>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
