@@ -275,6 +275,33 @@ __global__ void __launch_bounds__(kSmallBlock) k_plan_sort(const cr_plan_info_de
     for (uint32_t u = threadIdx.x; u < U; u += kSmallBlock) order[u] = oi ? oi[u] : u;
 }
 
+// Up to this many requests the histogram is sorted by one CTA (fewer launches);
+// above it by device-wide radix passes.
+constexpr uint64_t kPlanSortOneCta = 65536;
+
+// Large histograms (multi-CTA passes): after the key sort, the per-key output
+// and the count-descending sort key n - count.
+__global__ void k_plan_sorted_keys(const cr_plan_info_dev *info, unsigned long long n,
+                                   const unsigned long long *__restrict__ k, const uint32_t *__restrict__ c,
+                                   unsigned long long *__restrict__ ukey, unsigned long long *__restrict__ ucnt,
+                                   uint32_t *__restrict__ s32)
+{
+    const unsigned long long U = info->U;
+    for (uint64_t u = (uint64_t)blockIdx.x * blockDim.x + threadIdx.x; u < U; u += (uint64_t)gridDim.x * blockDim.x) {
+        ukey[u] = k[u];
+        ucnt[u] = c[u];
+        s32[u] = (uint32_t)(n - c[u]);
+    }
+}
+
+__global__ void k_plan_copy_order(const cr_plan_info_dev *info, const uint32_t *__restrict__ src,
+                                  uint32_t *__restrict__ order)
+{
+    const unsigned long long U = info->U;
+    for (uint64_t u = (uint64_t)blockIdx.x * blockDim.x + threadIdx.x; u < U; u += (uint64_t)gridDim.x * blockDim.x)
+        order[u] = src[u];
+}
+
 // Eq. 1: k_b = min(R, max(1, ceil(lambda * den / num))); NOREPL: 1.
 __device__ __forceinline__ uint32_t eq1_kb(unsigned long long lam, unsigned long long num, unsigned long long den,
                                            uint32_t R)
@@ -1029,9 +1056,25 @@ extern "C" int cr_build_plans(cr_ctx *ctx, const uint64_t *d_key, uint64_t n, co
         // the (n - count) keys and the order ping-pong through the now idle table memory
         uint32_t *s32A = (uint32_t *)ptk, *s32B = s32A + n, *o32B = (uint32_t *)ptc;
         uint32_t *ord = (uint32_t *)po;
-        CR_LAUNCH(ctx, k_plan_sort, 1, kSmallBlock, 0, (const cr_plan_info_dev *)p0->d_info, (unsigned long long)n,
-                  bits_for(n), (unsigned long long *)pk0, (uint32_t *)pv0, (unsigned long long *)pk1,
-                  (uint32_t *)pv1, p0->d_ukey, p0->d_ucnt, s32A, s32B, ord + n, o32B, ord);
+        if (n <= kPlanSortOneCta) {
+            CR_LAUNCH(ctx, k_plan_sort, 1, kSmallBlock, 0, (const cr_plan_info_dev *)p0->d_info,
+                      (unsigned long long)n, bits_for(n), (unsigned long long *)pk0, (uint32_t *)pv0,
+                      (unsigned long long *)pk1, (uint32_t *)pv1, p0->d_ukey, p0->d_ucnt, s32A, s32B, ord + n, o32B,
+                      ord);
+        } else {
+            // same two sorts in device-wide passes, the key count read on the device
+            const unsigned long long *dU = &p0->d_info->U;
+            int in1 = 0;
+            CR_TRY(cr_radix_pairs_u64_dev(ctx, (unsigned long long *)pk0, (uint32_t *)pv0, (unsigned long long *)pk1,
+                                          (uint32_t *)pv1, n, dU, 64, 0, &in1));
+            CR_LAUNCH(ctx, k_plan_sorted_keys, grid_n, 256, 0, (const cr_plan_info_dev *)p0->d_info,
+                      (unsigned long long)n, (const unsigned long long *)(in1 ? pk1 : pk0),
+                      (const uint32_t *)(in1 ? pv1 : pv0), p0->d_ukey, p0->d_ucnt, s32A);
+            uint32_t *o32A = (uint32_t *)pv0;  // free again after the key sort's results were copied out
+            CR_TRY(cr_radix_pairs_u32_dev(ctx, s32A, o32A, s32B, o32B, n, dU, bits_for(n), 1, &in1));
+            CR_LAUNCH(ctx, k_plan_copy_order, grid_n, 256, 0, (const cr_plan_info_dev *)p0->d_info,
+                      (const uint32_t *)(in1 ? o32B : o32A), ord);
+        }
         order = ord;
     }
 

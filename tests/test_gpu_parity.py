@@ -136,6 +136,22 @@ def test_plan_parity(P, ctx, seed):
         _cmp_plan(got, O.build_plan(keys, R, W, num, den, variant=v, seed=seed, epoch=3))
 
 
+@pytest.mark.parametrize("R,nkeys,total", [(30, 150000, 400000), (1024, 300000, 1200000)])
+def test_plan_parity_large_histogram(P, ctx, R, nkeys, total):
+    # histograms far above the one-CTA sort size (device-wide radix passes)
+    rng = np.random.default_rng(nkeys)
+    keys = _rates_keys(rng, nkeys, total, skew=0.9)
+    n = keys.size
+    params = [P.plan_params(R, 64, 5 * n, 4 * R, v, seed=3, epoch=1) for v in ("LPT", "RANDOM", "NOREPL")]
+    plans = [P.Plan(ctx) for _ in params]
+    P.build_plans(ctx, d_u64(keys), params, plans)
+    uk, uc = O.histogram(keys)
+    for pl, v in zip(plans, ("LPT", "RANDOM", "NOREPL")):
+        got = pl.export()
+        assert (got["ukey"] == uk).all() and (got["ucnt"] == uc).all()
+        _cmp_plan(got, O.build_plan(keys, R, 64, 5 * n, 4 * R, variant=v, seed=3, epoch=1))
+
+
 @pytest.mark.parametrize("R,spread", [(33, 0), (64, 50), (257, 3), (1024, 0), (1024, 400)])
 def test_plan_equal_rate_runs(P, ctx, R, spread):
     # long runs of keys with the same count and k = 1 (placed a run at a time on
