@@ -126,12 +126,15 @@ int cr_radix_sort_u32(cr_ctx *ctx, const uint32_t *k_in, const uint32_t *v_in, u
 // Exclusive scan of u32 counts into u32 offsets (in place allowed); total to *d_total if non-null.
 // Radix sort of (key, value) pairs by bits [0, bits), ping-ponging between the
 // caller's buffers 0 and 1; the item count is read from n_dev (grid sized by
-// n_max).  With iota the values start as the items' positions.  *in1 tells
-// whether the result ended in buffers 1.
+// n_max); a count <= skip_le leaves everything untouched.  With iota the
+// values start as the items' positions.  *in1 tells whether the result ended
+// in buffers 1.
 int cr_radix_pairs_u64_dev(cr_ctx *ctx, unsigned long long *k0, uint32_t *v0, unsigned long long *k1, uint32_t *v1,
-                           uint64_t n_max, const unsigned long long *n_dev, int bits, int iota, int *in1);
+                           uint64_t n_max, const unsigned long long *n_dev, unsigned long long skip_le, int bits,
+                           int iota, int *in1);
 int cr_radix_pairs_u32_dev(cr_ctx *ctx, uint32_t *k0, uint32_t *v0, uint32_t *k1, uint32_t *v1, uint64_t n_max,
-                           const unsigned long long *n_dev, int bits, int iota, int *in1);
+                           const unsigned long long *n_dev, unsigned long long skip_le, int bits, int iota,
+                           int *in1);
 int cr_scan_u32(cr_ctx *ctx, const uint32_t *in, uint32_t *out, uint64_t n, uint32_t *d_total);
 // Inclusive scan of u64 values.
 int cr_scan_u64_inclusive(cr_ctx *ctx, const unsigned long long *in, unsigned long long *out, uint64_t n);

@@ -245,9 +245,10 @@ __global__ void __launch_bounds__(kSmallBlock) k_plan_sort(const cr_plan_info_de
                                                            unsigned long long *__restrict__ ukey,
                                                            unsigned long long *__restrict__ ucnt, uint32_t *s32A,
                                                            uint32_t *s32B, uint32_t *o32A, uint32_t *o32B,
-                                                           uint32_t *__restrict__ order)
+                                                           uint32_t *__restrict__ order, unsigned long long max_u)
 {
     __shared__ small_sort_smem sm;
+    if (info->U > max_u) return;  // sorted by the device-wide passes instead
     const uint32_t U = (uint32_t)info->U;
     unsigned long long *ki = kA, *ko = kB;
     uint32_t *vi = vA, *vo = vB;
@@ -275,9 +276,10 @@ __global__ void __launch_bounds__(kSmallBlock) k_plan_sort(const cr_plan_info_de
     for (uint32_t u = threadIdx.x; u < U; u += kSmallBlock) order[u] = oi ? oi[u] : u;
 }
 
-// Up to this many requests the histogram is sorted by one CTA (fewer launches);
-// above it by device-wide radix passes.
-constexpr uint64_t kPlanSortOneCta = 65536;
+// Intervals of up to this many requests sort their histogram in one CTA (one
+// launch, one SM, so the planner barely touches the SMs the overlapped main
+// stream uses); larger ones in device-wide radix passes.
+constexpr uint64_t kPlanSortOneCta = 524288;
 
 // Large histograms (multi-CTA passes): after the key sort, the per-key output
 // and the count-descending sort key n - count.
@@ -1060,18 +1062,18 @@ extern "C" int cr_build_plans(cr_ctx *ctx, const uint64_t *d_key, uint64_t n, co
             CR_LAUNCH(ctx, k_plan_sort, 1, kSmallBlock, 0, (const cr_plan_info_dev *)p0->d_info,
                       (unsigned long long)n, bits_for(n), (unsigned long long *)pk0, (uint32_t *)pv0,
                       (unsigned long long *)pk1, (uint32_t *)pv1, p0->d_ukey, p0->d_ucnt, s32A, s32B, ord + n, o32B,
-                      ord);
+                      ord, ~0ull);
         } else {
-            // same two sorts in device-wide passes, the key count read on the device
+            // the same two sorts in device-wide passes, the key count read on the device
             const unsigned long long *dU = &p0->d_info->U;
             int in1 = 0;
             CR_TRY(cr_radix_pairs_u64_dev(ctx, (unsigned long long *)pk0, (uint32_t *)pv0, (unsigned long long *)pk1,
-                                          (uint32_t *)pv1, n, dU, 64, 0, &in1));
+                                          (uint32_t *)pv1, n, dU, 0ull, 64, 0, &in1));
             CR_LAUNCH(ctx, k_plan_sorted_keys, grid_n, 256, 0, (const cr_plan_info_dev *)p0->d_info,
                       (unsigned long long)n, (const unsigned long long *)(in1 ? pk1 : pk0),
                       (const uint32_t *)(in1 ? pv1 : pv0), p0->d_ukey, p0->d_ucnt, s32A);
             uint32_t *o32A = (uint32_t *)pv0;  // free again after the key sort's results were copied out
-            CR_TRY(cr_radix_pairs_u32_dev(ctx, s32A, o32A, s32B, o32B, n, dU, bits_for(n), 1, &in1));
+            CR_TRY(cr_radix_pairs_u32_dev(ctx, s32A, o32A, s32B, o32B, n, dU, 0ull, bits_for(n), 1, &in1));
             CR_LAUNCH(ctx, k_plan_copy_order, grid_n, 256, 0, (const cr_plan_info_dev *)p0->d_info,
                       (const uint32_t *)(in1 ? o32B : o32A), ord);
         }
@@ -1322,7 +1324,7 @@ extern "C" int cr_key_histogram_noalloc(const uint64_t *d_key, uint64_t n, uint6
         uint32_t *s32A = (uint32_t *)tkey, *s32B = s32A + n;
         k_plan_sort<<<1, kSmallBlock, 0, s>>>(info, (unsigned long long)n, bits_for(n), kA, vA, kB, vB,
                                               (unsigned long long *)d_ukey, (unsigned long long *)d_ucnt, s32A,
-                                              s32B, ord + n, tcnt, ord);
+                                              s32B, ord + n, tcnt, ord, ~0ull);
     }
     k_copy_u<<<1, 1, 0, s>>>(info, (unsigned long long *)d_U);
     cudaError_t e = cudaGetLastError();

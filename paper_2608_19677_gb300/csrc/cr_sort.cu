@@ -136,11 +136,14 @@ int scan_impl(cr_ctx *ctx, const T *in, T *out, uint64_t n, int inclusive, T *d_
 // ---------------------------------------------------------- radix sort ----
 // n_dev (optional): the item count in device memory; n is then an upper bound
 // that sized the grid and the histogram, and tiles past the count stay empty.
+// A count <= skip_le makes the pass a no-op (another path sorts those).
 template <typename K>
 __global__ void __launch_bounds__(kSortBlock) k_radix_upsweep(const K *__restrict__ keys, uint64_t n, int shift,
                                                               uint32_t ntiles, uint32_t *__restrict__ hist,
-                                                              const unsigned long long *n_dev)
+                                                              const unsigned long long *n_dev,
+                                                              unsigned long long skip_le)
 {
+    if (n_dev && *n_dev <= skip_le) return;
     if (n_dev && *n_dev < n) n = *n_dev;
     __shared__ uint32_t cnt[256];
     cnt[threadIdx.x] = 0;
@@ -161,8 +164,10 @@ __global__ void __launch_bounds__(kSortBlock) k_radix_downsweep(const K *__restr
                                                                 K *__restrict__ kout, uint32_t *__restrict__ vout,
                                                                 uint64_t n, int shift, uint32_t ntiles,
                                                                 const uint32_t *__restrict__ offs,
-                                                                const unsigned long long *n_dev)
+                                                                const unsigned long long *n_dev,
+                                                                unsigned long long skip_le)
 {
+    if (n_dev && *n_dev <= skip_le) return;
     if (n_dev && *n_dev < n) n = *n_dev;
     constexpr int kWarps = kSortBlock / 32;
     __shared__ uint32_t base_s[256];
@@ -228,11 +233,11 @@ int radix_impl(cr_ctx *ctx, const K *k_in, const uint32_t *v_in, uint64_t n, int
         K *kdst = reinterpret_cast<K *>((pass & 1) ? kb1 : kb0);
         uint32_t *vdst = want_vals ? reinterpret_cast<uint32_t *>((pass & 1) ? vb1 : vb0) : nullptr;
         CR_LAUNCH(ctx, k_radix_upsweep<K>, ntiles, kSortBlock, 0, ksrc, n, shift, ntiles, (uint32_t *)hist,
-                  (const unsigned long long *)nullptr);
+                  (const unsigned long long *)nullptr, 0ull);
         CR_TRY(scan_impl<uint32_t>(ctx, (const uint32_t *)hist, (uint32_t *)hist, (uint64_t)256 * ntiles, 0,
                                    (uint32_t *)nullptr));
         CR_LAUNCH(ctx, k_radix_downsweep<K>, ntiles, kSortBlock, 0, ksrc, vsrc, kdst, vdst, n, shift, ntiles,
-                  (const uint32_t *)hist, (const unsigned long long *)nullptr);
+                  (const uint32_t *)hist, (const unsigned long long *)nullptr, 0ull);
         ksrc = kdst;
         vsrc = vdst;
     }
@@ -246,7 +251,7 @@ int radix_impl(cr_ctx *ctx, const K *k_in, const uint32_t *v_in, uint64_t n, int
 // With iota the input values are not read: they are the items' positions.
 template <typename K>
 int radix_pairs_dev(cr_ctx *ctx, K *k0, uint32_t *v0, K *k1, uint32_t *v1, uint64_t n_max,
-                    const unsigned long long *n_dev, int bits, int iota, int *in1)
+                    const unsigned long long *n_dev, unsigned long long skip_le, int bits, int iota, int *in1)
 {
     *in1 = 0;
     if (n_max == 0 || bits <= 0) return CR_OK;
@@ -260,11 +265,11 @@ int radix_pairs_dev(cr_ctx *ctx, K *k0, uint32_t *v0, K *k1, uint32_t *v1, uint6
         const uint32_t *vs = (shift == 0 && iota) ? nullptr : (cur ? v1 : v0);
         uint32_t *vd = cur ? v0 : v1;
         CR_LAUNCH(ctx, k_radix_upsweep<K>, ntiles, kSortBlock, 0, (const K *)ks, n_max, shift, ntiles,
-                  (uint32_t *)hist, n_dev);
+                  (uint32_t *)hist, n_dev, skip_le);
         CR_TRY(scan_impl<uint32_t>(ctx, (const uint32_t *)hist, (uint32_t *)hist, (uint64_t)256 * ntiles, 0,
                                    (uint32_t *)nullptr));
         CR_LAUNCH(ctx, k_radix_downsweep<K>, ntiles, kSortBlock, 0, (const K *)ks, vs, kd, vd, n_max, shift, ntiles,
-                  (const uint32_t *)hist, n_dev);
+                  (const uint32_t *)hist, n_dev, skip_le);
         cur ^= 1;
     }
     *in1 = cur;
@@ -274,15 +279,17 @@ int radix_pairs_dev(cr_ctx *ctx, K *k0, uint32_t *v0, K *k1, uint32_t *v1, uint6
 }  // namespace
 
 int cr_radix_pairs_u64_dev(cr_ctx *ctx, unsigned long long *k0, uint32_t *v0, unsigned long long *k1, uint32_t *v1,
-                           uint64_t n_max, const unsigned long long *n_dev, int bits, int iota, int *in1)
+                           uint64_t n_max, const unsigned long long *n_dev, unsigned long long skip_le, int bits,
+                           int iota, int *in1)
 {
-    return radix_pairs_dev<unsigned long long>(ctx, k0, v0, k1, v1, n_max, n_dev, bits, iota, in1);
+    return radix_pairs_dev<unsigned long long>(ctx, k0, v0, k1, v1, n_max, n_dev, skip_le, bits, iota, in1);
 }
 
 int cr_radix_pairs_u32_dev(cr_ctx *ctx, uint32_t *k0, uint32_t *v0, uint32_t *k1, uint32_t *v1, uint64_t n_max,
-                           const unsigned long long *n_dev, int bits, int iota, int *in1)
+                           const unsigned long long *n_dev, unsigned long long skip_le, int bits, int iota,
+                           int *in1)
 {
-    return radix_pairs_dev<uint32_t>(ctx, k0, v0, k1, v1, n_max, n_dev, bits, iota, in1);
+    return radix_pairs_dev<uint32_t>(ctx, k0, v0, k1, v1, n_max, n_dev, skip_le, bits, iota, in1);
 }
 
 int cr_scan_u32(cr_ctx *ctx, const uint32_t *in, uint32_t *out, uint64_t n, uint32_t *d_total)
