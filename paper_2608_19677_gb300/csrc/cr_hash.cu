@@ -136,7 +136,9 @@ extern "C" int cr_hash_prefixes(cr_ctx *ctx, const int32_t *d_tokens, const uint
     if (!d_tokens || !d_off || !d_plen || !d_key_out)
         return cr_fail(ctx, CR_EINVAL, "cr_hash_prefixes: NULL pointer");
     const unsigned int warps_per_block = kHashBlock / 32;
-    unsigned int grid = cr_blocks(n, warps_per_block, (unsigned int)ctx->num_sms * 8u);
+    // many more blocks than fit at once (32 per SM): blocks start as others
+    // finish, which evens out the widely varying span lengths across the SMs
+    unsigned int grid = cr_blocks(n, warps_per_block, (unsigned int)ctx->num_sms * 32u);
     CR_LAUNCH(ctx, k_hash_prefixes, grid, kHashBlock, 0, d_tokens, (const unsigned long long *)d_off,
               d_plen, (unsigned long long)n, (unsigned long long)salt, (unsigned long long *)d_key_out);
     return CR_OK;
