@@ -45,6 +45,9 @@ def parse_args():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-overlap", action="store_true", help="build plans in line instead of on a second stream")
     ap.add_argument("--e2e-steps", type=int, default=2)
+    ap.add_argument("--keys-mode", action="store_true",
+                    help="hash each interval's arena on its own and time plans + route + replay over resident keys "
+                         "(automatic when the arenas do not fit in HBM)")
     ap.add_argument("--intervals", type=int, default=0,
                     help="profiling aid: run only the first N intervals (the JSON line says so)")
     return ap.parse_args()
@@ -255,7 +258,7 @@ def main():
     rec_tokens = float(trace.key_plen.astype(np.float64).mean()) + cfg.suffix + 3
     tok_bytes = 4.0 * rec_tokens * float(sum(trace.counts[:cfg.n_intervals]))
     free, _total = torch.cuda.mem_get_info(dev)
-    if tok_bytes > 0.6 * free:
+    if args.keys_mode or tok_bytes > 0.6 * free:
         return run_keys_mode(args, cfg, trace, dev, stream, world, rank, barrier)
 
     # inputs resident in HBM (generated on the device, untimed)
@@ -421,6 +424,7 @@ def run_keys_mode(args, cfg, trace, dev, stream, world, rank, barrier):
         ns.append(iv.n)
         del tok, off
     torch.cuda.synchronize()
+    torch.cuda.empty_cache()  # the arenas are gone: only keys and lengths stay on the device
     n_step = sum(ns)
     pipe = Pipeline(ctx, cfg.R, cfg.W, cfg.caps, cfg.replicas, trace.qcap, batch_B=args.batch, max_n=max(ns),
                     overlap=not args.no_overlap)
