@@ -561,7 +561,7 @@ def e2e(args, ctx, pipe, inputs, dev, stream, n_step, world):
             dtok, doff, dpl, dsl = bufs[b]
             pipe.interval(t, dtok[:h[0].numel()], doff[:n], dpl[:n], dsl[:n], g0, plan_next=i + 1 < len(host),
                           inputs_ready=ready[b])
-            done[b].record(stream)   # after this interval's replay, which follows its hash
+            done[b] = pipe.inputs_free   # after this interval's replay, the last reader of its inputs
         pipe.finish()
         out.copy_(pipe.ctr, non_blocking=True)
 

@@ -45,7 +45,10 @@ struct cr_ctx {
 
 // Plan: every array lives on the device; capacities are host-side upper bounds.
 struct cr_plan_info_dev {
-    unsigned long long n, U, n_adm, sum_k, cold, max_k, special;
+    unsigned long long n, U;
+    unsigned long long S;        // admission candidates ordered by (count desc, key asc): order[0..S)
+    unsigned long long n_adm, sum_k, cold, max_k, special;
+    unsigned long long adm_lam;  // requests of the admitted keys
 };
 
 struct cr_table_slot {               // 16 bytes: one sector-aligned probe

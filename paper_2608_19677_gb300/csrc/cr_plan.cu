@@ -24,6 +24,8 @@ __global__ void k_plan_reset(cr_plan_info_dev *info, unsigned long long n)
 {
     info->n = n;
     info->U = 0;
+    info->S = 0;
+    info->adm_lam = 0;
     info->n_adm = 0;
     info->sum_k = 0;
     info->cold = 0;
@@ -239,19 +241,16 @@ __device__ void cta_radix_pass(const K *kin, const uint32_t *vin, K *kout, uint3
 
 // Sorts the U distinct (key, count) pairs: key ascending into (ukey, ucnt), then
 // stably by (n - count) into `order` = admission order (count desc, key asc).
-__global__ void __launch_bounds__(kSmallBlock) k_plan_sort(const cr_plan_info_dev *info, unsigned long long n,
-                                                           int cbits, unsigned long long *kA, uint32_t *vA,
-                                                           unsigned long long *kB, uint32_t *vB,
-                                                           unsigned long long *__restrict__ ukey,
-                                                           unsigned long long *__restrict__ ucnt, uint32_t *s32A,
-                                                           uint32_t *s32B, uint32_t *o32A, uint32_t *o32B,
-                                                           uint32_t *__restrict__ order, unsigned long long max_u)
+// Stable LSD sort of U (key, count) pairs in one CTA: by key (8 passes), the
+// sorted pairs written to ukey/ucnt, then by n - count (ceil(cbits/8) passes)
+// giving order = positions in ukey/ucnt by (count desc, key asc).  The pairs
+// start in (ki, vi) and ping-pong with (ko, vo).
+__device__ __forceinline__ void small_sort(small_sort_smem &sm, uint32_t U, unsigned long long n, int cbits,
+                                           unsigned long long *ki, uint32_t *vi, unsigned long long *ko,
+                                           uint32_t *vo, unsigned long long *__restrict__ ukey,
+                                           unsigned long long *__restrict__ ucnt, uint32_t *s32A, uint32_t *s32B,
+                                           uint32_t *o32A, uint32_t *o32B, uint32_t *__restrict__ order)
 {
-    __shared__ small_sort_smem sm;
-    if (info->U > max_u) return;  // sorted by the device-wide passes instead
-    const uint32_t U = (uint32_t)info->U;
-    unsigned long long *ki = kA, *ko = kB;
-    uint32_t *vi = vA, *vo = vB;
     cta_histograms<unsigned long long>(ki, U, 8, sm);
     for (int pass = 0; pass < 8; ++pass) {
         cta_radix_pass<unsigned long long>(ki, vi, ko, vo, U, pass, sm);
@@ -276,6 +275,138 @@ __global__ void __launch_bounds__(kSmallBlock) k_plan_sort(const cr_plan_info_de
     for (uint32_t u = threadIdx.x; u < U; u += kSmallBlock) order[u] = oi ? oi[u] : u;
 }
 
+__global__ void __launch_bounds__(kSmallBlock) k_plan_sort(const cr_plan_info_dev *info, unsigned long long n,
+                                                           int cbits, unsigned long long *kA, uint32_t *vA,
+                                                           unsigned long long *kB, uint32_t *vB,
+                                                           unsigned long long *__restrict__ ukey,
+                                                           unsigned long long *__restrict__ ucnt, uint32_t *s32A,
+                                                           uint32_t *s32B, uint32_t *o32A, uint32_t *o32B,
+                                                           uint32_t *__restrict__ order)
+{
+    __shared__ small_sort_smem sm;
+    small_sort(sm, (uint32_t)info->U, n, cbits, kA, vA, kB, vB, ukey, ucnt, s32A, s32B, o32A, o32B, order);
+}
+
+// Admission reads only the first keys of the (count desc, key asc) order: at
+// most C = R*W of them, since every k_b >= 1.  One CTA finds the count lam_C
+// of the C-th largest count (two-level radix select over the counts), moves
+// the keys with count >= lam_C (ties at lam_C included) to the front, sorts
+// only those, and writes the other keys after them in table order.  order then
+// covers the S candidates, every key admission can reach; the plan's per-key
+// arrays still hold all U keys.
+__device__ __forceinline__ void select_from_top(const uint32_t *hist, uint32_t nbk, unsigned long long want,
+                                                uint32_t *res)
+{
+    // lane l sums buckets [nbk - (l+1) per, nbk - l per): lane 0 holds the top
+    const uint32_t lane = cr_lane(), per = (nbk + 31) / 32;
+    const int hi = (int)nbk - (int)(lane * per), lo = hi - (int)per;
+    unsigned long long c = 0;
+    for (int b = hi - 1; b >= lo && b >= 0; --b) c += hist[b];
+    unsigned long long inc = c;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        const unsigned long long y = __shfl_up_sync(0xffffffffu, inc, o);
+        if (lane >= (uint32_t)o) inc += y;
+    }
+    const bool here = inc >= want && inc - c < want;
+    if (here) {
+        unsigned long long run = inc - c;  // counted in buckets above this lane's chunk
+        for (int b = hi - 1; b >= lo && b >= 0; --b) {
+            if (run + hist[b] >= want) {
+                res[0] = (uint32_t)b;
+                res[1] = (uint32_t)run;
+                break;
+            }
+            run += hist[b];
+        }
+    }
+}
+
+__global__ void __launch_bounds__(kSmallBlock) k_plan_topk(cr_plan_info_dev *info, unsigned long long n, int cbits,
+                                                           unsigned long long cmax, unsigned long long *kA,
+                                                           uint32_t *vA, unsigned long long *kB, uint32_t *vB,
+                                                           unsigned long long *__restrict__ ukey,
+                                                           unsigned long long *__restrict__ ucnt, uint32_t *s32A,
+                                                           uint32_t *s32B, uint32_t *o32A, uint32_t *o32B,
+                                                           uint32_t *__restrict__ order)
+{
+    __shared__ small_sort_smem sm;
+    __shared__ uint32_t res[4];
+    __shared__ uint32_t wtot[2][kSmallWarps];
+    const uint32_t U = (uint32_t)info->U;
+    const uint32_t tid = threadIdx.x, lane = cr_lane(), warp = tid >> 5, lt = (1u << lane) - 1u;
+    if (U <= cmax) {  // every key is a candidate
+        small_sort(sm, U, n, cbits, kA, vA, kB, vB, ukey, ucnt, s32A, s32B, o32A, o32B, order);
+        if (tid == 0) info->S = U;
+        return;
+    }
+    uint32_t *h1 = &sm.hist[0][0], *h2 = h1 + 1024;
+    const int nb = 64 - __clzll(n);  // counts are <= n < 2^nb
+    const int s1 = nb > 10 ? nb - 10 : 0;
+    const uint32_t nb1 = 1u << (nb - s1), nb2 = 1u << s1;
+    for (uint32_t x = tid; x < 2048; x += kSmallBlock) h1[x] = 0;
+    __syncthreads();
+    const uint32_t Ur = (U + kSmallBlock - 1) / kSmallBlock * kSmallBlock;
+    for (uint32_t u = tid; u < Ur; u += kSmallBlock) {  // level 1: high bits of the count
+        const uint32_t b = u < U ? (vA[u] >> s1) : 0xffffffffu;
+        const uint32_t peers = __match_any_sync(0xffffffffu, b);
+        if (b != 0xffffffffu && (peers & lt) == 0) atomicAdd(&h1[b], (uint32_t)__popc(peers));
+    }
+    __syncthreads();
+    if (warp == 0) select_from_top(h1, nb1, cmax, res);
+    __syncthreads();
+    const uint32_t b1 = res[0], above1 = res[1];
+    for (uint32_t u = tid; u < Ur; u += kSmallBlock) {  // level 2: low bits inside bucket b1
+        const uint32_t v = u < U ? vA[u] : 0u;
+        const uint32_t b = (u < U && (v >> s1) == b1) ? (v & (nb2 - 1u)) : 0xffffffffu;
+        const uint32_t peers = __match_any_sync(0xffffffffu, b);
+        if (b != 0xffffffffu && (peers & lt) == 0) atomicAdd(&h2[b], (uint32_t)__popc(peers));
+    }
+    __syncthreads();
+    if (warp == 0) select_from_top(h2, nb2, cmax - above1, res + 2);
+    __syncthreads();
+    const uint32_t thr = (b1 << s1) | res[2];
+    const uint32_t S = above1 + res[3] + h2[res[2]];
+    // stable partition: candidates to (kB, vB)[0..S), the rest to ukey/ucnt[S..U)
+    uint32_t run_c = 0, run_o = 0;
+    for (uint32_t base = 0; base < U; base += kSmallBlock) {
+        const uint32_t u = base + tid;
+        const bool valid = u < U;
+        const unsigned long long key = valid ? kA[u] : 0ull;
+        const uint32_t cnt = valid ? vA[u] : 0u;
+        const bool cand = valid && cnt >= thr;
+        const uint32_t bc = __ballot_sync(0xffffffffu, cand), bo = __ballot_sync(0xffffffffu, valid && !cand);
+        if (lane == 0) {
+            wtot[0][warp] = __popc(bc);
+            wtot[1][warp] = __popc(bo);
+        }
+        __syncthreads();
+        uint32_t pc = 0, po = 0, tc = 0, to = 0;
+        for (uint32_t w = 0; w < kSmallWarps; ++w) {
+            const uint32_t a = wtot[0][w], o = wtot[1][w];
+            if (w < warp) {
+                pc += a;
+                po += o;
+            }
+            tc += a;
+            to += o;
+        }
+        if (cand) {
+            const uint32_t pos = run_c + pc + __popc(bc & lt);
+            kB[pos] = key;
+            vB[pos] = cnt;
+        } else if (valid) {
+            const uint32_t pos = S + run_o + po + __popc(bo & lt);
+            ukey[pos] = key;
+            ucnt[pos] = cnt;
+        }
+        run_c += tc;
+        run_o += to;
+        __syncthreads();
+    }
+    small_sort(sm, S, n, cbits, kB, vB, kA, vA, ukey, ucnt, s32A, s32B, o32A, o32B, order);
+    if (tid == 0) info->S = S;
+}
 // Intervals of up to this many requests sort their histogram in one CTA (one
 // launch, one SM, so the planner barely touches the SMs the overlapped main
 // stream uses); larger ones in device-wide radix passes.
@@ -296,10 +427,11 @@ __global__ void k_plan_sorted_keys(const cr_plan_info_dev *info, unsigned long l
     }
 }
 
-__global__ void k_plan_copy_order(const cr_plan_info_dev *info, const uint32_t *__restrict__ src,
+__global__ void k_plan_copy_order(cr_plan_info_dev *info, const uint32_t *__restrict__ src,
                                   uint32_t *__restrict__ order)
 {
     const unsigned long long U = info->U;
+    if (blockIdx.x == 0 && threadIdx.x == 0) info->S = U;  // every key ordered
     for (uint64_t u = (uint64_t)blockIdx.x * blockDim.x + threadIdx.x; u < U; u += (uint64_t)gridDim.x * blockDim.x)
         order[u] = src[u];
 }
@@ -319,8 +451,8 @@ __global__ void k_plan_kb(const uint32_t *__restrict__ order, const unsigned lon
                           uint64_t n, const cr_plan_info_dev *info, unsigned long long num, unsigned long long den,
                           uint32_t R, int norepl, unsigned long long *__restrict__ kk)
 {
-    const unsigned long long U = info->U;
-    for (uint64_t a = (uint64_t)blockIdx.x * blockDim.x + threadIdx.x; a < U; a += (uint64_t)gridDim.x * blockDim.x)
+    const unsigned long long S = info->S;
+    for (uint64_t a = (uint64_t)blockIdx.x * blockDim.x + threadIdx.x; a < S; a += (uint64_t)gridDim.x * blockDim.x)
         kk[a] = norepl ? 1ull : eq1_kb(ucnt[order[a]], num, den, R);
 }
 
@@ -328,9 +460,9 @@ __global__ void k_plan_kb(const uint32_t *__restrict__ order, const unsigned lon
 __global__ void k_plan_admit(const unsigned long long *__restrict__ kscan, cr_plan_info_dev *info,
                              unsigned long long C)
 {
-    const unsigned long long U = info->U;
-    for (uint64_t a = (uint64_t)blockIdx.x * blockDim.x + threadIdx.x; a < U; a += (uint64_t)gridDim.x * blockDim.x) {
-        if (kscan[a] <= C && (a + 1 == U || kscan[a + 1] > C)) {
+    const unsigned long long S = info->S;
+    for (uint64_t a = (uint64_t)blockIdx.x * blockDim.x + threadIdx.x; a < S; a += (uint64_t)gridDim.x * blockDim.x) {
+        if (kscan[a] <= C && (a + 1 == S || kscan[a + 1] > C)) {
             info->n_adm = a + 1;
             info->sum_k = kscan[a];
         }
@@ -343,12 +475,12 @@ __global__ void k_plan_fill(const uint32_t *__restrict__ order, const unsigned l
                             unsigned long long *__restrict__ adm_cnt, uint32_t *__restrict__ adm_k,
                             uint32_t *__restrict__ koff)
 {
-    const unsigned long long U = info->U, na = info->n_adm;
-    unsigned long long cold = 0;
+    const unsigned long long na = info->n_adm;
+    unsigned long long lam = 0;
     uint32_t kmax = 0;
-    for (uint64_t a = (uint64_t)blockIdx.x * blockDim.x + threadIdx.x; a < U; a += (uint64_t)gridDim.x * blockDim.x) {
+    for (uint64_t a = (uint64_t)blockIdx.x * blockDim.x + threadIdx.x; a < na; a += (uint64_t)gridDim.x * blockDim.x) {
         uint32_t u = order[a];
-        if (a < na) {
+        {
             uint32_t k = (uint32_t)(kscan[a] - (a ? kscan[a - 1] : 0ull));
             adm_key[a] = ukey[u];
             adm_cnt[a] = ucnt[u];
@@ -356,23 +488,25 @@ __global__ void k_plan_fill(const uint32_t *__restrict__ order, const unsigned l
             koff[a] = (uint32_t)(kscan[a] - k);
             kmax = k > kmax ? k : kmax;
             if (a + 1 == na) koff[na] = (uint32_t)kscan[a];
-        } else {
-            cold += ucnt[u];
+            lam += ucnt[u];
         }
     }
-    cold = cr_warp_sum_u64(cold);
+    lam = cr_warp_sum_u64(lam);
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) kmax = max(kmax, __shfl_xor_sync(0xffffffffu, kmax, o));
     if (cr_lane() == 0) {
-        if (cold) atomicAdd(&info->cold, cold);
+        if (lam) atomicAdd(&info->adm_lam, lam);
         if (kmax) atomicMax(&info->max_k, (unsigned long long)kmax);
     }
 }
 
-__global__ void k_plan_init_load(const cr_plan_info_dev *info, const unsigned long long *__restrict__ init_load,
+// Cold tail: every request of a key that was not admitted (n - admitted).
+__global__ void k_plan_init_load(cr_plan_info_dev *info, const unsigned long long *__restrict__ init_load,
                                  uint32_t R, unsigned long long *__restrict__ load, uint32_t *status)
 {
-    const unsigned long long share = info->cold / R;
+    const unsigned long long cold = info->n - info->adm_lam;
+    if (blockIdx.x == 0 && threadIdx.x == 0) info->cold = cold;
+    const unsigned long long share = cold / R;
     for (uint32_t r = blockIdx.x * blockDim.x + threadIdx.x; r < R; r += gridDim.x * blockDim.x) {
         unsigned long long v = init_load ? init_load[r] : share;
         if (v >= kLoadLimit) atomicOr(status, CR_FLAG_OVERFLOW);
@@ -1059,10 +1193,15 @@ extern "C" int cr_build_plans(cr_ctx *ctx, const uint64_t *d_key, uint64_t n, co
         uint32_t *s32A = (uint32_t *)ptk, *s32B = s32A + n, *o32B = (uint32_t *)ptc;
         uint32_t *ord = (uint32_t *)po;
         if (n <= kPlanSortOneCta) {
-            CR_LAUNCH(ctx, k_plan_sort, 1, kSmallBlock, 0, (const cr_plan_info_dev *)p0->d_info,
-                      (unsigned long long)n, bits_for(n), (unsigned long long *)pk0, (uint32_t *)pv0,
-                      (unsigned long long *)pk1, (uint32_t *)pv1, p0->d_ukey, p0->d_ucnt, s32A, s32B, ord + n, o32B,
-                      ord, ~0ull);
+            // admission candidates only: the largest slot budget of the build bounds how far it reaches
+            unsigned long long cmax = 0;
+            for (uint32_t j = 0; j < n_plans; ++j) {
+                const unsigned long long c = (unsigned long long)params[j].R * params[j].W;
+                cmax = c > cmax ? c : cmax;
+            }
+            CR_LAUNCH(ctx, k_plan_topk, 1, kSmallBlock, 0, p0->d_info, (unsigned long long)n, bits_for(n), cmax,
+                      (unsigned long long *)pk0, (uint32_t *)pv0, (unsigned long long *)pk1, (uint32_t *)pv1,
+                      p0->d_ukey, p0->d_ucnt, s32A, s32B, ord + n, o32B, ord);
         } else {
             // the same two sorts in device-wide passes, the key count read on the device
             const unsigned long long *dU = &p0->d_info->U;
@@ -1074,7 +1213,7 @@ extern "C" int cr_build_plans(cr_ctx *ctx, const uint64_t *d_key, uint64_t n, co
                       (const uint32_t *)(in1 ? pv1 : pv0), p0->d_ukey, p0->d_ucnt, s32A);
             uint32_t *o32A = (uint32_t *)pv0;  // free again after the key sort's results were copied out
             CR_TRY(cr_radix_pairs_u32_dev(ctx, s32A, o32A, s32B, o32B, n, dU, 0ull, bits_for(n), 1, &in1));
-            CR_LAUNCH(ctx, k_plan_copy_order, grid_n, 256, 0, (const cr_plan_info_dev *)p0->d_info,
+            CR_LAUNCH(ctx, k_plan_copy_order, grid_n, 256, 0, p0->d_info,
                       (const uint32_t *)(in1 ? o32B : o32A), ord);
         }
         order = ord;
@@ -1122,8 +1261,8 @@ extern "C" int cr_build_plans(cr_ctx *ctx, const uint64_t *d_key, uint64_t n, co
                                          cudaMemcpyDeviceToDevice, ctx->stream));
             CR_CUDA(ctx, cudaMemcpyAsync(p->d_ucnt, p0->d_ucnt, n * sizeof(unsigned long long),
                                          cudaMemcpyDeviceToDevice, ctx->stream));
-            CR_CUDA(ctx, cudaMemcpyAsync(&p->d_info->U, &p0->d_info->U, sizeof(unsigned long long),
-                                         cudaMemcpyDeviceToDevice, ctx->stream));
+            CR_CUDA(ctx, cudaMemcpyAsync(&p->d_info->U, &p0->d_info->U, 2 * sizeof(unsigned long long),
+                                         cudaMemcpyDeviceToDevice, ctx->stream));  // U and S
         }
         CR_CUDA(ctx, cudaMemsetAsync(p->d_table, 0xff, p->table_slots * sizeof(cr_table_slot), ctx->stream));
         if (n > 0) {
@@ -1140,7 +1279,7 @@ extern "C" int cr_build_plans(cr_ctx *ctx, const uint64_t *d_key, uint64_t n, co
                       (const unsigned long long *)p->d_ucnt, (const unsigned long long *)kk, p->d_info,
                       p->d_adm_key, p->d_adm_cnt, p->d_adm_k, p->d_koff);
         }
-        CR_LAUNCH(ctx, k_plan_init_load, cr_blocks(pp.R, 256, gcap), 256, 0, (const cr_plan_info_dev *)p->d_info,
+        CR_LAUNCH(ctx, k_plan_init_load, cr_blocks(pp.R, 256, gcap), 256, 0, p->d_info,
                   (const unsigned long long *)pp.d_init_load, pp.R, p->d_load, ctx->d_status);
         if (n > 0) {
             if (pp.variant == CR_VARIANT_RANDOM) {
@@ -1213,6 +1352,13 @@ extern "C" int cr_plan_get_info(cr_ctx *ctx, const cr_plan *p, cr_plan_info *out
     return CR_OK;
 }
 
+__global__ void k_gather_u64(const unsigned long long *__restrict__ src, const uint32_t *__restrict__ idx,
+                             unsigned long long n, unsigned long long *__restrict__ out)
+{
+    for (uint64_t i = (uint64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (uint64_t)gridDim.x * blockDim.x)
+        out[i] = src[idx[i]];
+}
+
 extern "C" int cr_plan_export(cr_ctx *ctx, const cr_plan *p, uint64_t *ukey, uint64_t *ucnt, uint64_t *adm_key,
                               uint64_t *adm_cnt, uint32_t *adm_k, uint32_t *koff, uint16_t *members,
                               uint64_t *jobs, uint64_t *load)
@@ -1220,8 +1366,24 @@ extern "C" int cr_plan_export(cr_ctx *ctx, const cr_plan *p, uint64_t *ukey, uin
     cr_plan_info info;
     CR_TRY(cr_plan_get_info(ctx, p, &info));
     cudaStream_t s = ctx->stream;
-    if (ukey && info.U) CR_CUDA(ctx, cudaMemcpyAsync(ukey, p->d_ukey, info.U * 8, cudaMemcpyDeviceToHost, s));
-    if (ucnt && info.U) CR_CUDA(ctx, cudaMemcpyAsync(ucnt, p->d_ucnt, info.U * 8, cudaMemcpyDeviceToHost, s));
+    cr_plan_info_dev d;
+    CR_CUDA(ctx, cudaMemcpyAsync(&d, p->d_info, sizeof(d), cudaMemcpyDeviceToHost, s));
+    CR_TRY(cr_sync(ctx));
+    const unsigned long long *sk = (const unsigned long long *)p->d_ukey, *sc = (const unsigned long long *)p->d_ucnt;
+    if ((ukey || ucnt) && d.U && d.S < d.U) {
+        // only the admission candidates are in key order: sort the whole histogram by key
+        const unsigned long long *ks;
+        const uint32_t *pos;
+        CR_TRY(cr_radix_sort_u64(ctx, (const unsigned long long *)p->d_ukey, nullptr, d.U, 64, &ks, &pos));
+        void *pc;
+        CR_TRY(cr_scratch(ctx, SCR_PLAN_A, d.U * sizeof(unsigned long long), &pc));
+        CR_LAUNCH(ctx, k_gather_u64, cr_blocks(d.U, 256, (unsigned int)ctx->num_sms * 8u), 256, 0,
+                  (const unsigned long long *)p->d_ucnt, pos, (unsigned long long)d.U, (unsigned long long *)pc);
+        sk = ks;
+        sc = (const unsigned long long *)pc;
+    }
+    if (ukey && info.U) CR_CUDA(ctx, cudaMemcpyAsync(ukey, sk, info.U * 8, cudaMemcpyDeviceToHost, s));
+    if (ucnt && info.U) CR_CUDA(ctx, cudaMemcpyAsync(ucnt, sc, info.U * 8, cudaMemcpyDeviceToHost, s));
     if (adm_key && info.n_adm)
         CR_CUDA(ctx, cudaMemcpyAsync(adm_key, p->d_adm_key, info.n_adm * 8, cudaMemcpyDeviceToHost, s));
     if (adm_cnt && info.n_adm)
@@ -1324,7 +1486,7 @@ extern "C" int cr_key_histogram_noalloc(const uint64_t *d_key, uint64_t n, uint6
         uint32_t *s32A = (uint32_t *)tkey, *s32B = s32A + n;
         k_plan_sort<<<1, kSmallBlock, 0, s>>>(info, (unsigned long long)n, bits_for(n), kA, vA, kB, vB,
                                               (unsigned long long *)d_ukey, (unsigned long long *)d_ucnt, s32A,
-                                              s32B, ord + n, tcnt, ord, ~0ull);
+                                              s32B, ord + n, tcnt, ord);
     }
     k_copy_u<<<1, 1, 0, s>>>(info, (unsigned long long *)d_U);
     cudaError_t e = cudaGetLastError();

@@ -14,11 +14,15 @@ One control interval t:
 With ``overlap=True`` the planner runs on its own high-priority stream and
 library context, ordered by CUDA events: plans(t+1) need only interval t's
 keys, so they are built on a few SMs while interval t is routed and replayed
-and interval t+1 is hashed on the main stream.  (The driver can also put
+and interval t+1 is hashed on the main stream.  The replay also has a stream
+and context of its own: replay(t) needs only interval t's destinations, so it
+runs while interval t+1 is hashed and routed.  (The driver can also put
 hashing on a stream of its own; that is off because the hash kernel's CTAs
 occupy every SM and would delay the single-SM routing CTAs instead of sharing
-the machine with them.)  Keys are triple-buffered and plans double-buffered; a
-buffer is reused only after events show its last reader has finished.
+the machine with them.)  Keys are triple-buffered, plans and destinations
+double-buffered; a buffer is reused only after events show its last reader has
+finished.  ``inputs_free`` is the event after which the last interval's input
+tensors are no longer read.
 """
 from __future__ import annotations
 
@@ -65,14 +69,19 @@ class Pipeline:
             self.hstream, self.hctx = self.mstream, ctx
             self.pstream = torch.cuda.Stream(dev, priority=hi)
             self.pctx = Context(ctx.device, self.pstream)
+            self.ystream = torch.cuda.Stream(dev)
+            self.yctx = Context(ctx.device, self.ystream)
         else:
-            self.hstream = self.pstream = self.mstream
-            self.hctx = self.pctx = ctx
+            self.hstream = self.pstream = self.ystream = self.mstream
+            self.hctx = self.pctx = self.yctx = ctx
         self.plans = [[Plan(self.pctx) for _ in self.plan_keys] for _ in range(2)]
         self.replay = Replay(ctx, len(self.replicas), R, self.caps)
         self.ctr = torch.zeros((len(self.replicas), len(self.caps), R, 5), dtype=torch.int64, device=dev)
         self.load = torch.zeros((len(self.replicas), R), dtype=torch.int64, device=dev)
-        self._dest = None
+        self._dests = [None, None]   # destinations, double-buffered when the replay lags
+        self._dest_free = [None, None]  # event: the replay that read this buffer has finished
+        self._dbuf = 0
+        self.inputs_free = None
         self._keys = [None] * NKEYS
         self._released = [[] for _ in range(NKEYS)]  # events after which a keys buffer may be rewritten
         self._kidx = 0
@@ -89,16 +98,19 @@ class Pipeline:
     @property
     def contexts(self):
         out = []
-        for c in (self.ctx, self.hctx, self.pctx):
+        for c in (self.ctx, self.hctx, self.pctx, self.yctx):
             if all(c is not o for o in out):
                 out.append(c)
         return out
 
     def _alloc(self, n: int):
         import torch
-        if self._dest is None or self._dest.shape[1] < n:
+        if self._dests[0] is None or self._dests[0].shape[1] < n:
             self.sync()
-            self._dest = torch.empty((len(self.replicas), n), dtype=torch.int16, device=self.dev)
+            nd = 2 if self.overlap else 1
+            self._dests = [torch.empty((len(self.replicas), n), dtype=torch.int16, device=self.dev)
+                           for _ in range(nd)] + [None] * (2 - nd)
+            self._dest_free = [None, None]
             self._keys = [torch.empty(n, dtype=torch.int64, device=self.dev) for _ in range(NKEYS)]
             self._released = [[] for _ in range(NKEYS)]
 
@@ -117,6 +129,7 @@ class Pipeline:
             start.record(self.mstream)
             self.hstream.wait_event(start)
             self.pstream.wait_event(start)
+            self.ystream.wait_event(start)
 
     def _event(self, stream, timing=False):
         import torch
@@ -201,18 +214,28 @@ class Pipeline:
             marks[1].record(self.mstream)
             marks[2].record(self.mstream)
         self.load.zero_()
-        dest = self._dest[:, :n] if n == self._dest.shape[1] else self._dest.view(-1)[:len(self.replicas) * n].view(
-            len(self.replicas), n)
+        db = self._dbuf
+        if self.overlap:
+            self._dbuf ^= 1
+            if self._dest_free[db] is not None:
+                self.mstream.wait_event(self._dest_free[db])
+        D = self._dests[db]
+        dest = D[:, :n] if n == D.shape[1] else D.view(-1)[:len(self.replicas) * n].view(len(self.replicas), n)
         plans = [self.plans[cur][i] if i is not None else None for i in self.rep_plan]
         route_batch(self.ctx, plans, self.policies, self.seeds, self.R, keys, g0, self.B, self.load, dest)
         if mark:
             marks[3].record(self.mstream)
-        shadow_replay(self.ctx, self.replay, keys, plen, slen, dest, self.ctr)
+        if self.overlap:
+            self.ystream.wait_event(self._event(self.mstream))
+        shadow_replay(self.yctx, self.replay, keys, plen, slen, dest, self.ctr)
+        replayed = self._event(self.ystream)
         if mark:
-            marks[4].record(self.mstream)
+            marks[4].record(self.ystream)
+        self.inputs_free = replayed
         # keys buffer kb is free once this interval's replay and the next plans have read it
         if self.overlap:
-            self._released[kb].append(self._event(self.mstream))
+            self._dest_free[db] = replayed
+            self._released[kb].append(replayed)
             if plan_reader is not None:
                 self._released[kb].append(plan_reader)
         self.prev_keys = keys
@@ -229,6 +252,7 @@ class Pipeline:
         if self.overlap:
             self.mstream.wait_event(self._event(self.hstream))
             self.mstream.wait_event(self._event(self.pstream))
+            self.mstream.wait_event(self._event(self.ystream))
 
     def sync(self):
         for c in self.contexts:
