@@ -92,6 +92,8 @@ class Pipeline:
         self._next_built = False     # the next interval's plans are already enqueued
         self.plan_marks = []         # (start, end) events of every plan build, when marked
         self.hash_marks = []         # (start, end) events of every hash, when marked
+        self.route_marks = []        # (start, end) events of every route call, after its waits
+        self.replay_marks = []       # (start, end) events of every replay call, after its waits
         if max_n:
             self._alloc(max_n)
 
@@ -124,6 +126,8 @@ class Pipeline:
         self._next_built = False
         self.plan_marks = []
         self.hash_marks = []
+        self.route_marks = []
+        self.replay_marks = []
         if self.overlap:
             start = torch.cuda.Event()
             start.record(self.mstream)
@@ -222,15 +226,19 @@ class Pipeline:
         D = self._dests[db]
         dest = D[:, :n] if n == D.shape[1] else D.view(-1)[:len(self.replicas) * n].view(len(self.replicas), n)
         plans = [self.plans[cur][i] if i is not None else None for i in self.rep_plan]
+        r0 = self._event(self.mstream, True) if mark else None
         route_batch(self.ctx, plans, self.policies, self.seeds, self.R, keys, g0, self.B, self.load, dest)
         if mark:
             marks[3].record(self.mstream)
+            self.route_marks.append((r0, marks[3]))
         if self.overlap:
             self.ystream.wait_event(self._event(self.mstream))
+        y0 = self._event(self.ystream, True) if mark else None
         shadow_replay(self.yctx, self.replay, keys, plen, slen, dest, self.ctr)
-        replayed = self._event(self.ystream)
+        replayed = self._event(self.ystream, mark)
         if mark:
             marks[4].record(self.ystream)
+            self.replay_marks.append((y0, replayed))
         self.inputs_free = replayed
         # keys buffer kb is free once this interval's replay and the next plans have read it
         if self.overlap:
