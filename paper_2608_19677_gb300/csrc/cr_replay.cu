@@ -3,14 +3,14 @@
 //   partition  one stable counting sort per replica by destination: each
 //              (replica, destination) stream's (key, prefix, suffix) records
 //              in arrival order
-//   replay     one warp per stream; the stream's LRU at the LARGEST capacity
-//              lives in shared memory (key + access stamp per entry, spread
-//              over the lanes).  A hit's depth (1 + entries touched after it)
-//              decides the hit at every smaller capacity at once, because LRU
-//              caches are nested (Mattson et al. 1970): the cache of capacity c
-//              is the c most recent entries of any larger one.
-//   state      kept between calls as keys in recency order (most recent first);
-//              stamps are re-derived from that order at the start of a call.
+//   replay     one warp per (stream, chunk); the stream's LRU at the LARGEST
+//              capacity lives in shared memory as keys in recency order with
+//              a hash index, and 32 requests are simulated per step, one per
+//              lane.  A request's depth (its LRU stack distance) decides the
+//              hit at every smaller capacity at once, because LRU caches are
+//              nested (Mattson et al. 1970): the cache of capacity c is the c
+//              most recent entries of any larger one.
+//   state      kept between calls as keys in recency order (most recent first).
 #include <stdlib.h>
 #include <string.h>
 
@@ -154,233 +154,7 @@ struct replay_state {
     uint32_t *fill_out;
 };
 
-// One warp per (stream, chunk).  The LRU state at the chunk's first request is
-// rebuilt by walking the stream backwards (and then the state carried in from
-// the previous call) collecting distinct keys, most recent first, until cmax
-// are found: those are exactly the resident entries of an LRU of capacity
-// cmax at that point.  The chunk is then simulated forwards.
-template <int E, int NC>  // NC: capacities counted (a compile-time bound on caps.n_caps)
-__global__ void __launch_bounds__(E == 1 ? 256 : 128, E == 1 ? 4 : 1)
-k_lru_chunks(const replay_caps caps, uint32_t cmax, uint32_t R, uint32_t ns, uint32_t CL,
-             const uint32_t *__restrict__ start, const uint32_t *__restrict__ coff, const uint32_t *__restrict__ total,
-             const rec16 *__restrict__ rec, const replay_state st, unsigned long long *__restrict__ ctr)
-{
-    extern __shared__ unsigned long long sm[];
-    const uint32_t lane = cr_lane(), warp = threadIdx.x >> 5, wpb = blockDim.x >> 5;
-    const uint32_t slots = 32u * E;
-    unsigned long long *sk = sm + (size_t)warp * slots;
-    uint32_t *ss = reinterpret_cast<uint32_t *>(sm + (size_t)wpb * slots) + (size_t)warp * slots;
-    const uint32_t w = blockIdx.x * wpb + warp;
-    if (w >= *total) return;
-    // stream of this work item: the last s with coff[s] <= w
-    uint32_t lo = 0, hi = ns;
-    while (hi - lo > 1) {
-        uint32_t mid = (lo + hi) >> 1;
-        if (coff[mid] <= w)
-            lo = mid;
-        else
-            hi = mid;
-    }
-    const uint32_t s = lo, ci = w - coff[s];
-    const uint32_t b = start[s], e = start[s + 1];
-    const uint32_t p0 = b + ci * CL;
-    const uint32_t p1 = (e - p0) < CL ? e : p0 + CL;
-    const uint32_t rep = s / R, r = s % R;
-    const uint32_t fill_in = st.fill_in[s];
-    const unsigned long long *kin = st.keys_in + (unsigned long long)s * cmax;
-    const uint32_t lt = (1u << lane) - 1u;
-
-    if (b == e) {  // nothing routed here: carry the state over unchanged
-        unsigned long long *kout = st.keys_out + (unsigned long long)s * cmax;
-        for (uint32_t q = lane; q < fill_in; q += 32) kout[q] = kin[q];
-        if (lane == 0) st.fill_out[s] = fill_in;
-        return;
-    }
-
-    // ---- state at p0 -------------------------------------------------------
-    uint32_t fill = 0;
-    if (ci == 0) {
-        for (uint32_t q = lane; q < fill_in; q += 32) sk[q] = kin[q];
-        fill = fill_in;
-    } else {
-        const uint32_t back = p0 - b;            // stream positions before the chunk
-        const uint32_t vtot = back + fill_in;    // then the carried-in state
-        for (uint32_t v0 = 0; v0 < vtot && fill < cmax; v0 += 32) {
-            const uint32_t v = v0 + lane;
-            const bool valid = v < vtot;
-            unsigned long long key = 0;
-            if (valid) key = v < back ? rec[p0 - 1 - v].key : kin[v - back];
-            const uint32_t peers = __match_any_sync(0xffffffffu, key);
-            bool fresh = valid && (peers & lt) == 0;
-            for (uint32_t q = 0; q < fill; ++q)
-                if (sk[q] == key) fresh = false;
-            const uint32_t bal = __ballot_sync(0xffffffffu, fresh);
-            const uint32_t rank = __popc(bal & lt);
-            __syncwarp();
-            if (fresh && fill + rank < cmax) sk[fill + rank] = key;
-            fill = min(cmax, fill + (uint32_t)__popc(bal));
-            __syncwarp();
-        }
-    }
-    for (uint32_t q = lane; q < fill; q += 32) ss[q] = fill - q;
-    __syncwarp();
-    uint32_t clock = fill;
-
-    // register copy of the state when it fits one entry per lane
-    unsigned long long ek = 0;
-    uint32_t es = 0;
-    if (E == 1 && lane < fill) {
-        ek = sk[lane];
-        es = ss[lane];
-    }
-
-    unsigned long long my_req = 0, my_prompt = 0;
-    unsigned long long my_hit[NC], my_tok[NC];
-#pragma unroll
-    for (int c = 0; c < NC; ++c) my_hit[c] = my_tok[c] = 0;
-
-    for (uint32_t t0 = p0; t0 < p1; t0 += 32) {
-        rec16 mine_rec = {0ull, 0u, 0u};
-        if (t0 + lane < p1) {
-            mine_rec = rec[t0 + lane];
-            my_req += 1;
-            my_prompt += (unsigned long long)mine_rec.P + mine_rec.S;
-        }
-        const uint32_t cnt = (p1 - t0) < 32u ? (p1 - t0) : 32u;
-        uint32_t my_depth = 0xffffffffu;  // lanes without a request never count a hit
-        for (uint32_t j = 0; j < cnt; ++j) {
-            const unsigned long long key = __shfl_sync(0xffffffffu, mine_rec.key, j);
-            ++clock;
-            uint32_t depth = 0xffffffffu;
-            if (E == 1) {
-                const bool have = lane < fill;
-                const uint32_t hb = __ballot_sync(0xffffffffu, have && ek == key);
-                if (hb) {
-                    const uint32_t hl = __ffs(hb) - 1;
-                    const uint32_t s_hit = __shfl_sync(0xffffffffu, es, hl);
-                    depth = 1u + __popc(__ballot_sync(0xffffffffu, have && es > s_hit));
-                    if (lane == hl) es = clock;
-                } else if (fill < cmax) {
-                    if (lane == fill) {
-                        ek = key;
-                        es = clock;
-                    }
-                    ++fill;
-                } else {
-                    const uint32_t mn = __reduce_min_sync(0xffffffffu, have ? es : 0xffffffffu);
-                    const uint32_t vl = __ffs(__ballot_sync(0xffffffffu, have && es == mn)) - 1;
-                    if (lane == vl) {
-                        ek = key;
-                        es = clock;
-                    }
-                }
-            } else {
-                int mine = -1;
-#pragma unroll
-                for (int x = 0; x < E; ++x) {
-                    const uint32_t idx = (uint32_t)x * 32u + lane;
-                    if (idx < fill && sk[idx] == key) mine = (int)idx;
-                }
-                const uint32_t hb = __ballot_sync(0xffffffffu, mine >= 0);
-                if (hb) {
-                    const uint32_t hl = __ffs(hb) - 1;
-                    const uint32_t hs = (uint32_t)__shfl_sync(0xffffffffu, mine, hl);
-                    const uint32_t s_hit = ss[hs];
-                    uint32_t newer = 0;
-#pragma unroll
-                    for (int x = 0; x < E; ++x) {
-                        const uint32_t idx = (uint32_t)x * 32u + lane;
-                        if (idx < fill && ss[idx] > s_hit) ++newer;
-                    }
-                    depth = 1u + __reduce_add_sync(0xffffffffu, newer);
-                    __syncwarp();
-                    if (lane == hl) ss[hs] = clock;
-                } else if (fill < cmax) {
-                    if (lane == 0) {
-                        sk[fill] = key;
-                        ss[fill] = clock;
-                    }
-                    ++fill;
-                } else {
-                    uint32_t lmin = 0xffffffffu, lidx = 0;
-#pragma unroll
-                    for (int x = 0; x < E; ++x) {
-                        const uint32_t idx = (uint32_t)x * 32u + lane;
-                        if (idx < fill && ss[idx] < lmin) {
-                            lmin = ss[idx];
-                            lidx = idx;
-                        }
-                    }
-                    const uint32_t wmin = __reduce_min_sync(0xffffffffu, lmin);
-                    const uint32_t vl = __ffs(__ballot_sync(0xffffffffu, lmin == wmin)) - 1;
-                    const uint32_t vidx = __shfl_sync(0xffffffffu, lidx, vl);
-                    __syncwarp();
-                    if (lane == 0) {
-                        sk[vidx] = key;
-                        ss[vidx] = clock;
-                    }
-                }
-                __syncwarp();
-            }
-            // the lane that loaded request j keeps its depth
-            if (lane == j) my_depth = depth;
-        }
-        // counters of the group, each lane for its own request
-#pragma unroll
-        for (int c = 0; c < NC; ++c) {
-            if (c < (int)caps.n_caps && my_depth <= caps.cap[c]) {
-                my_hit[c] += 1;
-                my_tok[c] += mine_rec.P;
-            }
-        }
-    }
-
-    // ---- counters -------------------------------------------------------------
-    my_req = cr_warp_sum_u64(my_req);
-    my_prompt = cr_warp_sum_u64(my_prompt);
-#pragma unroll
-    for (int c = 0; c < NC; ++c) {
-        if (c < (int)caps.n_caps) {
-            const unsigned long long h = cr_warp_sum_u64(my_hit[c]);
-            const unsigned long long tk = cr_warp_sum_u64(my_tok[c]);
-            if (lane == 0) {
-                unsigned long long *C = ctr + (((unsigned long long)rep * caps.n_caps + c) * R + r) * CR_CTR_FIELDS;
-                atomicAdd(&C[0], my_req);
-                if (h) atomicAdd(&C[1], h);
-                if (tk) atomicAdd(&C[2], tk);
-                atomicAdd(&C[3], my_prompt);
-                atomicAdd(&C[4], my_prompt - tk);
-            }
-        }
-    }
-
-    // ---- the stream's last chunk hands the state to the next call ---------------
-    if (p1 == e) {
-        unsigned long long *kout = st.keys_out + (unsigned long long)s * cmax;
-        if (E == 1) {
-            uint32_t rank = 0;
-            for (uint32_t q = 0; q < 32; ++q) {
-                const uint32_t sq = __shfl_sync(0xffffffffu, es, q);
-                if (q < fill && sq > es) ++rank;
-            }
-            if (lane < fill) kout[rank] = ek;
-        } else {
-#pragma unroll
-            for (int x = 0; x < E; ++x) {
-                const uint32_t idx = (uint32_t)x * 32u + lane;
-                if (idx < fill) {
-                    const uint32_t my = ss[idx];
-                    uint32_t rank = 0;
-                    for (uint32_t f = 0; f < fill; ++f) rank += (ss[f] > my) ? 1u : 0u;
-                    kout[rank] = sk[idx];
-                }
-            }
-        }
-        if (lane == 0) st.fill_out[s] = fill;
-    }
-}
-
-// ---- capacities above 32: batched stack distances ---------------------------
+// ---- replay: batched stack distances ------------------------------------------
 // One warp per (stream, chunk) holds the LRU of the largest capacity as keys in
 // recency order, K[0] most recent, in shared memory, with an open-addressing
 // index key -> position (u16, position + 1, 0 = empty) rebuilt after every
@@ -683,37 +457,6 @@ k_lru_batch(const replay_caps caps, uint32_t cmax, uint32_t R, uint32_t ns, uint
     }
 }
 
-template <int E, int NC>
-int launch_replay_nc(cr_ctx *ctx, cr_replay *rp, const replay_caps &caps, uint32_t CL, const uint32_t *start,
-                     const uint32_t *coff, const uint32_t *total, uint64_t m, const rec16 *rec, uint64_t *d_ctr)
-{
-    const uint32_t wpb = E == 1 ? 8 : 4;
-    const size_t smem = (size_t)wpb * 32 * E * (sizeof(unsigned long long) + sizeof(uint32_t));
-    if (smem > 48 * 1024)
-        CR_CUDA(ctx, cudaFuncSetAttribute(k_lru_chunks<E, NC>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                          (int)smem));
-    const uint32_t ns = rp->n_rep * rp->R;
-    const uint64_t items = (uint64_t)ns + (m + CL - 1) / CL;  // upper bound on work items
-    replay_state st;
-    st.keys_in = rp->d_keys[rp->cur];
-    st.fill_in = rp->d_fill[rp->cur];
-    st.keys_out = rp->d_keys[rp->cur ^ 1];
-    st.fill_out = rp->d_fill[rp->cur ^ 1];
-    CR_LAUNCH(ctx, (k_lru_chunks<E, NC>), (unsigned int)((items + wpb - 1) / wpb), wpb * 32, smem, caps, rp->cmax,
-              rp->R, ns, CL, start, coff, total, rec, st, (unsigned long long *)d_ctr);
-    rp->cur ^= 1;
-    return CR_OK;
-}
-
-template <int E>
-int launch_replay(cr_ctx *ctx, cr_replay *rp, const replay_caps &caps, uint32_t CL, const uint32_t *start,
-                  const uint32_t *coff, const uint32_t *total, uint64_t m, const rec16 *rec, uint64_t *d_ctr)
-{
-    if (caps.n_caps == 1) return launch_replay_nc<E, 1>(ctx, rp, caps, CL, start, coff, total, m, rec, d_ctr);
-    if (caps.n_caps <= 3) return launch_replay_nc<E, 3>(ctx, rp, caps, CL, start, coff, total, m, rec, d_ctr);
-    return launch_replay_nc<E, CR_MAX_CAPS>(ctx, rp, caps, CL, start, coff, total, m, rec, d_ctr);
-}
-
 template <int NC>
 int launch_batch_nc(cr_ctx *ctx, cr_replay *rp, const replay_caps &caps, uint32_t CL, const uint32_t *start,
                     const uint32_t *coff, const uint32_t *total, uint64_t m, const rec16 *rec, uint64_t *d_ctr)
@@ -860,10 +603,7 @@ extern "C" int cr_shadow_replay(cr_ctx *ctx, cr_replay *rp, const uint64_t *d_ke
     const uint32_t CL = rp->cmax * 16u > 256u ? rp->cmax * 16u : 256u;
     CR_LAUNCH(ctx, k_chunk_counts, cr_blocks(ns, 256, gcap), 256, 0, (const uint32_t *)start, ns, CL, coff);
     CR_TRY(cr_scan_u32(ctx, coff, coff, ns, total));
-    const uint32_t E = (rp->cmax + 31) / 32;
-    // capacities up to 32: one entry per lane in registers; above: batched stack distances
-    if (E > 1) return launch_batch(ctx, rp, caps, CL, start, coff, total, m, rec, d_ctr);
-    return launch_replay<1>(ctx, rp, caps, CL, start, coff, total, m, rec, d_ctr);
+    return launch_batch(ctx, rp, caps, CL, start, coff, total, m, rec, d_ctr);
 }
 
 extern "C" int cr_replay_export_state(cr_ctx *ctx, const cr_replay *rp, uint32_t rep, uint32_t r,
