@@ -136,6 +136,48 @@ def test_plan_parity(P, ctx, seed):
         _cmp_plan(got, O.build_plan(keys, R, W, num, den, variant=v, seed=seed, epoch=3))
 
 
+def _keys_with_counts(rng, counts):
+    ks = np.unique(rng.integers(0, 2**64 - 1, size=len(counts) + 64, dtype=np.uint64))[:len(counts)]
+    rng.shuffle(ks)
+    keys = np.repeat(ks, np.asarray(counts, np.int64))
+    rng.shuffle(keys)
+    return keys
+
+
+@pytest.mark.parametrize("case", ["ties_at_threshold", "U_eq_C", "U_eq_C_minus_1", "U_eq_C_plus_1",
+                                  "wide_counts", "single_key", "all_equal"])
+def test_plan_admission_candidates(P, ctx, case):
+    # the planner sorts only keys whose count reaches the C-th largest (C = R*W);
+    # these traces put that threshold on its edge cases
+    rng = np.random.default_rng(len(case))
+    R, W = 8, 5                      # C = 40
+    if case == "ties_at_threshold":  # 30 distinct counts above, 500 keys tied at the 40th count
+        counts = list(range(100, 130)) + [7] * 500 + [3] * 200
+    elif case == "U_eq_C":
+        counts = list(rng.integers(1, 50, size=40))
+    elif case == "U_eq_C_minus_1":
+        counts = list(rng.integers(1, 50, size=39))
+    elif case == "U_eq_C_plus_1":
+        counts = list(rng.integers(1, 50, size=41))
+    elif case == "wide_counts":      # counts over 17 bits: both select levels matter
+        counts = list(rng.integers(1, 120000, size=60)) + list(rng.integers(1, 40, size=3000))
+    elif case == "single_key":
+        R, W = 1, 1
+        counts = [12345]
+    else:                            # every key ties
+        counts = [5] * 2000
+    keys = _keys_with_counts(rng, counts)
+    n = keys.size
+    params = [P.plan_params(R, W, 5 * n, 4 * R, v, seed=2, epoch=4) for v in ("LPT", "RANDOM", "NOREPL")]
+    plans = [P.Plan(ctx) for _ in params]
+    P.build_plans(ctx, d_u64(keys), params, plans)
+    uk, uc = O.histogram(keys)
+    for pl, v in zip(plans, ("LPT", "RANDOM", "NOREPL")):
+        got = pl.export()
+        assert (got["ukey"] == uk).all() and (got["ucnt"] == uc).all()
+        _cmp_plan(got, O.build_plan(keys, R, W, 5 * n, 4 * R, variant=v, seed=2, epoch=4))
+
+
 @pytest.mark.parametrize("R,nkeys,total", [(30, 150000, 400000), (1024, 300000, 1200000)])
 def test_plan_parity_large_histogram(P, ctx, R, nkeys, total):
     # histograms far above the one-CTA sort size (device-wide radix passes)
