@@ -157,8 +157,10 @@ struct replay_state {
 // ---- replay: batched stack distances ------------------------------------------
 // One warp per (stream, chunk) holds the LRU of the largest capacity as keys in
 // recency order, K[0] most recent, in shared memory, with an open-addressing
-// index key -> position (u16, position + 1, 0 = empty) rebuilt after every
-// batch.  A batch is 32 consecutive requests, one per lane.  The depth of
+// index key -> physical slot (u16, slot + 1, 0 = empty, tombstones for evicted
+// keys, rebuilt when a quarter of it is tombstones).  The keys form a ring:
+// recency position q (0 = most recent) is slot (H + q) mod cmax.  A batch is
+// 32 consecutive requests, one per lane.  The depth of
 // request i (its LRU stack distance, Mattson et al. 1970) follows from the
 // state before the batch and the batch itself:
 //   - key seen earlier in the batch, last at lane j: 1 + the number of
@@ -168,14 +170,16 @@ struct replay_state {
 //   - absent before the batch: a miss at every capacity.
 // A request hits capacity c iff its depth <= c.  The state after the batch is
 // the batch's distinct keys by last access (latest first) followed by the
-// untouched old keys in their old order, cut at cmax.
+// untouched old keys in their old order, cut at cmax.  Old keys below the
+// deepest one the batch touched move (in place); those beyond it all shift by
+// the same amount, which moving the head H does, so they stay where they are.
 constexpr uint32_t kNone = 0xffffffffu;
 constexpr uint16_t kTomb = 0xffffu;  // index slot whose key was evicted
 
 struct lru_index {
-    unsigned long long *K;  // [cmax] keys, recency order
-    uint16_t *TS;           // [cmax] index slot of the key at each position
-    uint16_t *tab;          // [tsz] position + 1; 0 = empty, kTomb = evicted
+    unsigned long long *K;  // [cmax] keys: a ring, recency position q at slot (H + q) mod cmax
+    uint16_t *TS;           // [cmax] index slot of the key in each ring slot
+    uint16_t *tab;          // [tsz] ring slot + 1; 0 = empty, kTomb = evicted
     uint32_t *bm;           // [32] bitmap of old positions touched by the batch
     uint32_t mask;
     int tbits;
@@ -183,7 +187,7 @@ struct lru_index {
 
 __device__ __forceinline__ uint32_t lru_home(unsigned long long key, int tbits) { return (uint32_t)(key >> (64 - tbits)); }
 
-// Position of `key` (kNone if absent); *slot gets its index slot.
+// Ring slot of `key` (kNone if absent); *slot gets its index slot.
 __device__ __forceinline__ uint32_t lru_lookup(const lru_index &X, unsigned long long key, uint32_t *slot)
 {
     uint32_t s = lru_home(key, X.tbits);
@@ -213,13 +217,24 @@ __device__ __forceinline__ uint32_t lru_insert(const lru_index &X, unsigned long
     }
 }
 
-// Index of K[0..fill) from scratch (warp-cooperative); clears every tombstone.
-__device__ __forceinline__ void lru_reindex(const lru_index &X, uint32_t fill, uint32_t lane)
+__device__ __forceinline__ uint32_t ring_slot(uint32_t H, uint32_t q, uint32_t cmax)
+{
+    const uint32_t x = H + q;  // H < cmax, q < 2 cmax
+    return x >= cmax ? (x - cmax >= cmax ? x - 2 * cmax : x - cmax) : x;
+}
+
+// Index of the fill keys from ring slot H on, from scratch (warp-cooperative);
+// clears every tombstone.
+__device__ __forceinline__ void lru_reindex(const lru_index &X, uint32_t H, uint32_t fill, uint32_t cmax,
+                                            uint32_t lane)
 {
     uint4 *t4 = reinterpret_cast<uint4 *>(X.tab);
     for (uint32_t x = lane; x < (X.mask + 1) / 8; x += 32) t4[x] = make_uint4(0, 0, 0, 0);
     __syncwarp();
-    for (uint32_t p = lane; p < fill; p += 32) X.TS[p] = (uint16_t)lru_insert(X, X.K[p], p);
+    for (uint32_t q = lane; q < fill; q += 32) {
+        const uint32_t ph = ring_slot(H, q, cmax);
+        X.TS[ph] = (uint16_t)lru_insert(X, X.K[ph], ph);
+    }
     __syncwarp();
 }
 
@@ -275,10 +290,10 @@ k_lru_batch(const replay_caps caps, uint32_t cmax, uint32_t R, uint32_t ns, uint
         for (uint32_t q = lane; q < fill_in; q += 32) X.K[q] = kin[q];
         fill = fill_in;
         __syncwarp();
-        lru_reindex(X, fill, lane);
+        lru_reindex(X, 0, fill, cmax, lane);
     } else {
         // walk backwards collecting distinct keys, most recent first
-        lru_reindex(X, 0, lane);
+        lru_reindex(X, 0, 0, cmax, lane);
         const uint32_t back = p0 - b;
         const uint32_t vtot = back + fill_in;
         for (uint32_t v0 = 0; v0 < vtot && fill < cmax; v0 += 32) {
@@ -308,6 +323,7 @@ k_lru_batch(const replay_caps caps, uint32_t cmax, uint32_t R, uint32_t ns, uint
     for (int c = 0; c < NC; ++c) my_hit[c] = my_tok[c] = 0;
     const uint32_t nwords = (cmax + 31) / 32;
     uint32_t tomb = 0;  // tombstones in the index
+    uint32_t H = 0;     // ring slot of recency position 0
 
     rec16 ahead = {0ull, 0u, 0u};  // the next batch's records, loaded one batch early
     if (p0 + lane < p1) ahead = rec[p0 + lane];
@@ -325,8 +341,11 @@ k_lru_batch(const replay_caps caps, uint32_t cmax, uint32_t R, uint32_t ns, uint
         const uint32_t below = grp & lt, above = grp & gt;
         const bool first = valid && below == 0;
         const uint32_t next = above ? (uint32_t)__ffs(above) - 1u : 32u;
-        uint32_t slot0 = kNone;
-        const uint32_t d0 = first ? lru_lookup(X, mine.key, &slot0) : kNone;
+        uint32_t slot0 = kNone, d0 = kNone;
+        if (first) {
+            const uint32_t ph = lru_lookup(X, mine.key, &slot0);
+            if (ph != kNone) d0 = ph >= H ? ph - H : ph + cmax - H;  // recency position
+        }
         // lanes that push request i deeper, for every lane at once, by comparing
         // bit-sliced values from the most significant bit down (per bit: lanes
         // still equal keep the ones with the same bit; a lane whose bit is 1
@@ -378,26 +397,41 @@ k_lru_batch(const replay_caps caps, uint32_t cmax, uint32_t R, uint32_t ns, uint
         }
         const uint32_t touched = __shfl_sync(0xffffffffu, pre, 31);
         pre -= (uint32_t)__popc(wv);  // exclusive
-        // untouched old keys move back (never forward): highest block first, in
-        // place; each rewrites its index slot, evicted ones leave a tombstone
+        // old keys up to the deepest touched one move back (never forward),
+        // highest block first, in place; each rewrites its index slot.  Those
+        // beyond it shift by delta = u - touched, done by moving the head.
+        const uint32_t pmax = __reduce_max_sync(0xffffffffu, d0 != kNone ? d0 + 1u : 0u);  // deepest + 1
+        const uint32_t delta = u - touched;
+        const uint32_t H2 = H >= delta % cmax ? H - delta % cmax : H + cmax - delta % cmax;
         uint32_t evicted = 0;
-        for (int tb = (int)((fill + 31) / 32) - 1; tb >= 0; --tb) {
+        for (int tb = (int)((pmax + 31) / 32) - 1; tb >= 0; --tb) {
             const uint32_t p = (uint32_t)tb * 32u + lane;
             const uint32_t wt = __shfl_sync(0xffffffffu, wv, tb), pt = __shfl_sync(0xffffffffu, pre, tb);
             unsigned long long v = 0;
             uint32_t np = kNone, ts = 0;
-            if (p < fill && !((wt >> lane) & 1u)) {
-                v = X.K[p];
-                ts = X.TS[p];
+            if (p < pmax && !((wt >> lane) & 1u)) {
+                const uint32_t ph = ring_slot(H, p, cmax);
+                v = X.K[ph];
+                ts = X.TS[ph];
                 np = p + u - (pt + (uint32_t)__popc(wt & lt));
             }
             __syncwarp();
             if (np < cmax) {
-                X.K[np] = v;
-                X.TS[np] = (uint16_t)ts;
-                X.tab[ts] = (uint16_t)(np + 1);
+                const uint32_t ph = ring_slot(H2, np, cmax);
+                X.K[ph] = v;
+                X.TS[ph] = (uint16_t)ts;
+                X.tab[ts] = (uint16_t)(ph + 1);
             } else if (np != kNone) {
                 X.tab[ts] = kTomb;
+                ++evicted;
+            }
+        }
+        // old keys beyond the deepest touched one that the shift pushes past cmax
+        {
+            const uint32_t from = max(pmax, cmax > delta ? cmax - delta : 0u);
+            const uint32_t p = from + lane;
+            if (p < fill) {  // at most delta <= 32 of them
+                X.tab[X.TS[ring_slot(H, p, cmax)]] = kTomb;
                 ++evicted;
             }
         }
@@ -410,23 +444,26 @@ k_lru_batch(const replay_caps caps, uint32_t cmax, uint32_t R, uint32_t ns, uint
         if (valid && above == 0) {
             if (kslot != kNone) {
                 if (rank < cmax) {
-                    X.K[rank] = mine.key;
-                    X.TS[rank] = (uint16_t)kslot;
-                    X.tab[kslot] = (uint16_t)(rank + 1);
+                    const uint32_t ph = ring_slot(H2, rank, cmax);
+                    X.K[ph] = mine.key;
+                    X.TS[ph] = (uint16_t)kslot;
+                    X.tab[kslot] = (uint16_t)(ph + 1);
                 } else {
                     X.tab[kslot] = kTomb;
                     ++evicted;
                 }
             } else if (rank < cmax) {
-                X.K[rank] = mine.key;
-                X.TS[rank] = (uint16_t)lru_insert(X, mine.key, rank);
+                const uint32_t ph = ring_slot(H2, rank, cmax);
+                X.K[ph] = mine.key;
+                X.TS[ph] = (uint16_t)lru_insert(X, mine.key, ph);
             }
         }
+        H = H2;
         fill = min(cmax, fill - touched + u);
         tomb += __reduce_add_sync(0xffffffffu, evicted);
         __syncwarp();
         if (4 * (fill + tomb) > 3 * (X.mask + 1)) {  // too many tombstones: index afresh
-            lru_reindex(X, fill, lane);
+            lru_reindex(X, H, fill, cmax, lane);
             tomb = 0;
         }
     }
@@ -452,7 +489,7 @@ k_lru_batch(const replay_caps caps, uint32_t cmax, uint32_t R, uint32_t ns, uint
     // ---- the stream's last chunk hands the state to the next call, most recent first
     if (p1 == e) {
         unsigned long long *kout = st.keys_out + (unsigned long long)s * cmax;
-        for (uint32_t q = lane; q < fill; q += 32) kout[q] = X.K[q];
+        for (uint32_t q = lane; q < fill; q += 32) kout[q] = X.K[ring_slot(H, q, cmax)];
         if (lane == 0) st.fill_out[s] = fill;
     }
 }
