@@ -500,6 +500,125 @@ __global__ void k_plan_fill(const uint32_t *__restrict__ order, const unsigned l
     }
 }
 
+// Admission for every plan of a build in one launch (intervals sorted by one
+// CTA, whose admission candidates are few): one 1024-thread CTA per plan clears
+// its table, runs Eq. 1 and the inclusive k-sum over the candidates tile by
+// tile (a block scan), admits the prefix that fits C (Algorithm 1 admission
+// step; it stops at the first tile with a key that does not fit), writes the
+// admitted arrays, the cold tail n - admitted requests and the initial loads.
+struct admit_job {
+    cr_plan_info_dev *info;
+    const unsigned long long *init_load;
+    unsigned long long *load, *adm_key, *adm_cnt;
+    uint32_t *adm_k, *koff;
+    uint4 *table;
+    unsigned long long table_slots, C, num, den;
+    uint32_t R;
+    int norepl;
+};
+
+struct admit_jobs {
+    admit_job j[16];
+};
+
+__device__ __forceinline__ unsigned long long warp_incl_scan_u64(unsigned long long x, uint32_t lane)
+{
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        const unsigned long long y = __shfl_up_sync(0xffffffffu, x, o);
+        if (lane >= (uint32_t)o) x += y;
+    }
+    return x;
+}
+
+__global__ void __launch_bounds__(kSmallBlock) k_plan_admit_cta(const __grid_constant__ admit_jobs jobs,
+                                                                const cr_plan_info_dev *info0,
+                                                                const uint32_t *__restrict__ order,
+                                                                const unsigned long long *__restrict__ ukey,
+                                                                const unsigned long long *__restrict__ ucnt,
+                                                                unsigned long long n, uint32_t *status)
+{
+    const admit_job J = jobs.j[blockIdx.x];
+    __shared__ unsigned long long wsum[kSmallWarps], wlam[kSmallWarps];
+    __shared__ uint32_t wkmax[kSmallWarps];
+    __shared__ unsigned long long s_cold;
+    const uint32_t tid = threadIdx.x, lane = cr_lane(), warp = tid >> 5;
+    for (unsigned long long x = tid; x < J.table_slots; x += kSmallBlock)
+        J.table[x] = make_uint4(0xffffffffu, 0xffffffffu, 0xffffffffu, 0xffffffffu);  // all slots empty
+    const unsigned long long S = info0->S;
+    unsigned long long carry = 0, n_adm = 0, lam = 0;
+    uint32_t kmax = 0;
+    for (unsigned long long base = 0; base < S; base += kSmallBlock) {
+        const unsigned long long a = base + tid;
+        const bool valid = a < S;
+        const uint32_t u = valid ? order[a] : 0u;
+        const unsigned long long cnt = valid ? ucnt[u] : 0ull;
+        const uint32_t k = !valid ? 0u : (J.norepl ? 1u : eq1_kb(cnt, J.num, J.den, J.R));
+        const unsigned long long x = warp_incl_scan_u64(k, lane);
+        if (lane == 31) wsum[warp] = x;
+        __syncthreads();
+        if (warp == 0) wsum[lane] = warp_incl_scan_u64(wsum[lane], lane);
+        __syncthreads();
+        const unsigned long long ks = carry + x + (warp ? wsum[warp - 1] : 0ull);
+        const bool adm = valid && ks <= J.C;  // ks grows with a: the admitted keys are a prefix
+        const unsigned long long nt = (unsigned long long)__syncthreads_count(adm);
+        if (adm) {
+            J.adm_key[a] = ukey[u];
+            J.adm_cnt[a] = cnt;
+            J.adm_k[a] = k;
+            J.koff[a] = (uint32_t)(ks - k);
+            lam += cnt;
+            kmax = k > kmax ? k : kmax;
+            if (a + 1 == base + nt) {  // the last admitted key so far
+                J.koff[a + 1] = (uint32_t)ks;
+                J.info->sum_k = ks;
+            }
+        }
+        n_adm += nt;
+        const unsigned long long tile = wsum[kSmallWarps - 1];
+        __syncthreads();
+        if (nt < (S - base < kSmallBlock ? S - base : (unsigned long long)kSmallBlock)) break;
+        carry += tile;
+    }
+    lam = cr_warp_sum_u64(lam);
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) kmax = max(kmax, __shfl_xor_sync(0xffffffffu, kmax, o));
+    if (lane == 0) {
+        wlam[warp] = lam;
+        wkmax[warp] = kmax;
+    }
+    __syncthreads();
+    if (tid == 0) {
+        unsigned long long L = 0;
+        uint32_t km = 0;
+        for (int w = 0; w < kSmallWarps; ++w) {
+            L += wlam[w];
+            km = wkmax[w] > km ? wkmax[w] : km;
+        }
+        cr_plan_info_dev *I = J.info;
+        I->n = n;
+        I->U = info0->U;
+        I->S = S;
+        I->special = info0->special;
+        I->n_adm = n_adm;
+        if (n_adm == 0) {
+            I->sum_k = 0;
+            J.koff[0] = 0;
+        }
+        I->max_k = km;
+        I->adm_lam = L;
+        I->cold = n - L;
+        s_cold = n - L;
+    }
+    __syncthreads();
+    const unsigned long long share = s_cold / J.R;
+    for (uint32_t r = tid; r < J.R; r += kSmallBlock) {
+        const unsigned long long v = J.init_load ? J.init_load[r] : share;
+        if (v >= kLoadLimit) atomicOr(status, CR_FLAG_OVERFLOW);
+        J.load[r] = v;
+    }
+}
+
 // Cold tail: every request of a key that was not admitted (n - admitted).
 __global__ void k_plan_init_load(cr_plan_info_dev *info, const unsigned long long *__restrict__ init_load,
                                  uint32_t R, unsigned long long *__restrict__ load, uint32_t *status)
@@ -1252,6 +1371,36 @@ extern "C" int cr_build_plans(cr_ctx *ctx, const uint64_t *d_key, uint64_t n, co
         lj_maxR = 0;
         return CR_OK;
     };
+    // small intervals: admission of every plan in one launch, one CTA per plan
+    const bool fused = n > 0 && n <= kPlanSortOneCta;
+    if (fused) {
+        for (uint32_t j0 = 0; j0 < n_plans; j0 += 16) {
+            admit_jobs aj;
+            const uint32_t nj = n_plans - j0 < 16 ? n_plans - j0 : 16;
+            for (uint32_t x = 0; x < nj; ++x) {
+                cr_plan *p = plans[j0 + x];
+                const cr_plan_params &pp = params[j0 + x];
+                admit_job &J = aj.j[x];
+                J.info = p->d_info;
+                J.init_load = (const unsigned long long *)pp.d_init_load;
+                J.load = p->d_load;
+                J.adm_key = p->d_adm_key;
+                J.adm_cnt = p->d_adm_cnt;
+                J.adm_k = p->d_adm_k;
+                J.koff = p->d_koff;
+                J.table = reinterpret_cast<uint4 *>(p->d_table);
+                J.table_slots = p->table_slots;
+                J.C = (unsigned long long)pp.R * pp.W;
+                J.num = pp.qcap_num;
+                J.den = pp.qcap_den;
+                J.R = pp.R;
+                J.norepl = pp.variant == CR_VARIANT_NOREPL ? 1 : 0;
+            }
+            CR_LAUNCH(ctx, k_plan_admit_cta, nj, kSmallBlock, 0, aj, (const cr_plan_info_dev *)p0->d_info, order,
+                      (const unsigned long long *)p0->d_ukey, (const unsigned long long *)p0->d_ucnt,
+                      (unsigned long long)n, ctx->d_status);
+        }
+    }
     for (uint32_t j = 0; j < n_plans; ++j) {
         cr_plan *p = plans[j];
         const cr_plan_params &pp = params[j];
@@ -1261,11 +1410,13 @@ extern "C" int cr_build_plans(cr_ctx *ctx, const uint64_t *d_key, uint64_t n, co
                                          cudaMemcpyDeviceToDevice, ctx->stream));
             CR_CUDA(ctx, cudaMemcpyAsync(p->d_ucnt, p0->d_ucnt, n * sizeof(unsigned long long),
                                          cudaMemcpyDeviceToDevice, ctx->stream));
-            CR_CUDA(ctx, cudaMemcpyAsync(&p->d_info->U, &p0->d_info->U, 2 * sizeof(unsigned long long),
-                                         cudaMemcpyDeviceToDevice, ctx->stream));  // U and S
+            if (!fused)
+                CR_CUDA(ctx, cudaMemcpyAsync(&p->d_info->U, &p0->d_info->U, 2 * sizeof(unsigned long long),
+                                             cudaMemcpyDeviceToDevice, ctx->stream));  // U and S
         }
-        CR_CUDA(ctx, cudaMemsetAsync(p->d_table, 0xff, p->table_slots * sizeof(cr_table_slot), ctx->stream));
-        if (n > 0) {
+        if (!fused)
+            CR_CUDA(ctx, cudaMemsetAsync(p->d_table, 0xff, p->table_slots * sizeof(cr_table_slot), ctx->stream));
+        if (n > 0 && !fused) {
             void *pk;
             CR_TRY(cr_scratch(ctx, SCR_PLAN_B, (n + 2) * sizeof(unsigned long long), &pk));
             unsigned long long *kk = (unsigned long long *)pk;
@@ -1279,8 +1430,9 @@ extern "C" int cr_build_plans(cr_ctx *ctx, const uint64_t *d_key, uint64_t n, co
                       (const unsigned long long *)p->d_ucnt, (const unsigned long long *)kk, p->d_info,
                       p->d_adm_key, p->d_adm_cnt, p->d_adm_k, p->d_koff);
         }
-        CR_LAUNCH(ctx, k_plan_init_load, cr_blocks(pp.R, 256, gcap), 256, 0, p->d_info,
-                  (const unsigned long long *)pp.d_init_load, pp.R, p->d_load, ctx->d_status);
+        if (!fused)
+            CR_LAUNCH(ctx, k_plan_init_load, cr_blocks(pp.R, 256, gcap), 256, 0, p->d_info,
+                      (const unsigned long long *)pp.d_init_load, pp.R, p->d_load, ctx->d_status);
         if (n > 0) {
             if (pp.variant == CR_VARIANT_RANDOM) {
                 size_t smem = (size_t)kRandWarps * pp.R * sizeof(uint16_t);
