@@ -513,6 +513,7 @@ struct admit_job {
     uint32_t *adm_k, *koff;
     uint4 *table;
     unsigned long long table_slots, C, num, den;
+    unsigned long long *ukey_out, *ucnt_out;  // copy of the histogram, or null
     uint32_t R;
     int norepl;
 };
@@ -545,6 +546,13 @@ __global__ void __launch_bounds__(kSmallBlock) k_plan_admit_cta(const __grid_con
     const uint32_t tid = threadIdx.x, lane = cr_lane(), warp = tid >> 5;
     for (unsigned long long x = tid; x < J.table_slots; x += kSmallBlock)
         J.table[x] = make_uint4(0xffffffffu, 0xffffffffu, 0xffffffffu, 0xffffffffu);  // all slots empty
+    if (J.ukey_out) {
+        const unsigned long long U = info0->U;
+        for (unsigned long long x = tid; x < U; x += kSmallBlock) {
+            J.ukey_out[x] = ukey[x];
+            J.ucnt_out[x] = ucnt[x];
+        }
+    }
     const unsigned long long S = info0->S;
     unsigned long long carry = 0, n_adm = 0, lam = 0;
     uint32_t kmax = 0;
@@ -746,7 +754,7 @@ __device__ __forceinline__ unsigned long long warp_bitonic_sort(unsigned long lo
     return x;
 }
 
-__global__ void __launch_bounds__(32) k_plan_lpt32(const cr_plan_info_dev *info,
+__device__ __forceinline__ void lpt32_body(const cr_plan_info_dev *info,
                                                    const unsigned long long *__restrict__ adm_cnt,
                                                    const uint32_t *__restrict__ adm_k,
                                                    const uint32_t *__restrict__ koff, uint32_t R,
@@ -800,6 +808,38 @@ __global__ void __launch_bounds__(32) k_plan_lpt32(const cr_plan_info_dev *info,
     }
     if (lane < R) load_g[key & 0xffffu] = key >> 16;
     if (__any_sync(0xffffffffu, overflow) && lane == 0) atomicOr(status, CR_FLAG_OVERFLOW);
+}
+
+__global__ void __launch_bounds__(32) k_plan_lpt32(const cr_plan_info_dev *info,
+                                                   const unsigned long long *__restrict__ adm_cnt,
+                                                   const uint32_t *__restrict__ adm_k,
+                                                   const uint32_t *__restrict__ koff, uint32_t R,
+                                                   unsigned long long *__restrict__ load_g,
+                                                   uint16_t *__restrict__ members,
+                                                   unsigned long long *__restrict__ jobs, uint32_t *status)
+{
+    lpt32_body(info, adm_cnt, adm_k, koff, R, load_g, members, jobs, status);
+}
+
+// Placement jobs of several plans in one launch (the block index picks the plan).
+struct place_job {
+    const cr_plan_info_dev *info;
+    const unsigned long long *adm_cnt;
+    const uint32_t *adm_k, *koff;
+    unsigned long long *load, *jobs;
+    uint16_t *members;
+    unsigned long long seed, epoch;
+    uint32_t R;
+};
+
+struct place_jobs {
+    place_job j[16];
+};
+
+__global__ void __launch_bounds__(32) k_plan_lpt32_multi(const __grid_constant__ place_jobs pj, uint32_t *status)
+{
+    const place_job &J = pj.j[blockIdx.x];
+    lpt32_body(J.info, J.adm_cnt, J.adm_k, J.koff, J.R, J.load, J.members, J.jobs, status);
 }
 
 // LPT for 32 < R <= 1024, all LPT plans of one build at once (one warp per
@@ -1075,7 +1115,7 @@ __global__ void __launch_bounds__(32) k_plan_lpt_reg(const __grid_constant__ lpt
 // Fisher-Yates shuffle of 0..R-1 held in shared memory.
 constexpr int kRandWarps = 4;
 
-__global__ void __launch_bounds__(kRandWarps * 32) k_plan_random(const cr_plan_info_dev *info,
+__device__ __forceinline__ void random_body(const cr_plan_info_dev *info,
                                                                  const unsigned long long *__restrict__ adm_cnt,
                                                                  const uint32_t *__restrict__ adm_k,
                                                                  const uint32_t *__restrict__ koff, uint32_t R,
@@ -1083,9 +1123,8 @@ __global__ void __launch_bounds__(kRandWarps * 32) k_plan_random(const cr_plan_i
                                                                  unsigned long long *__restrict__ load_g,
                                                                  uint16_t *__restrict__ members,
                                                                  unsigned long long *__restrict__ jobs,
-                                                                 uint32_t *status)
+                                                                 uint32_t *status, uint16_t *perm_all)
 {
-    extern __shared__ uint16_t perm_all[];
     const uint32_t lane = cr_lane(), warp = threadIdx.x >> 5;
     uint16_t *perm = perm_all + (size_t)warp * R;
     const unsigned long long na = info->n_adm;
@@ -1118,7 +1157,30 @@ __global__ void __launch_bounds__(kRandWarps * 32) k_plan_random(const cr_plan_i
     }
 }
 
-__global__ void k_table_insert(const cr_plan_info_dev *info, const unsigned long long *__restrict__ adm_key,
+__global__ void __launch_bounds__(kRandWarps * 32) k_plan_random(const cr_plan_info_dev *info,
+                                                                 const unsigned long long *__restrict__ adm_cnt,
+                                                                 const uint32_t *__restrict__ adm_k,
+                                                                 const uint32_t *__restrict__ koff, uint32_t R,
+                                                                 unsigned long long seed, unsigned long long epoch,
+                                                                 unsigned long long *__restrict__ load_g,
+                                                                 uint16_t *__restrict__ members,
+                                                                 unsigned long long *__restrict__ jobs,
+                                                                 uint32_t *status)
+{
+    extern __shared__ uint16_t perm_all[];
+    random_body(info, adm_cnt, adm_k, koff, R, seed, epoch, load_g, members, jobs, status, perm_all);
+}
+
+__global__ void __launch_bounds__(kRandWarps * 32) k_plan_random_multi(const __grid_constant__ place_jobs pj,
+                                                                       uint32_t *status)
+{
+    extern __shared__ uint16_t perm_all[];
+    const place_job &J = pj.j[blockIdx.y];
+    random_body(J.info, J.adm_cnt, J.adm_k, J.koff, J.R, J.seed, J.epoch, J.load, J.members, J.jobs, status,
+                perm_all);
+}
+
+__device__ __forceinline__ void table_body(const cr_plan_info_dev *info, const unsigned long long *__restrict__ adm_key,
                                const uint32_t *__restrict__ adm_k, const uint32_t *__restrict__ koff,
                                const uint16_t *__restrict__ members, cr_table_slot *__restrict__ table,
                                int bits)
@@ -1139,6 +1201,34 @@ __global__ void k_table_insert(const cr_plan_info_dev *info, const unsigned long
             s = (s + 1) & mask;  // the table has at least twice as many slots as keys
         }
     }
+}
+
+__global__ void k_table_insert(const cr_plan_info_dev *info, const unsigned long long *__restrict__ adm_key,
+                               const uint32_t *__restrict__ adm_k, const uint32_t *__restrict__ koff,
+                               const uint16_t *__restrict__ members, cr_table_slot *__restrict__ table,
+                               int bits)
+{
+    table_body(info, adm_key, adm_k, koff, members, table, bits);
+}
+
+struct table_job {
+    const cr_plan_info_dev *info;
+    const unsigned long long *adm_key;
+    const uint32_t *adm_k, *koff;
+    const uint16_t *members;
+    cr_table_slot *table;
+    int bits;
+};
+
+struct table_jobs {
+    table_job j[16];
+};
+
+// Tables of several plans in one launch (blockIdx.y picks the plan).
+__global__ void k_table_insert_multi(const __grid_constant__ table_jobs tj)
+{
+    const table_job &J = tj.j[blockIdx.y];
+    table_body(J.info, J.adm_key, J.adm_k, J.koff, J.members, J.table, J.bits);
 }
 
 template <typename T>
@@ -1280,7 +1370,8 @@ extern "C" int cr_build_plans(cr_ctx *ctx, const uint64_t *d_key, uint64_t n, co
         CR_TRY(plan_reserve(ctx, plans[j], n, params[j].R, params[j].W));
         plans[j]->n = n;
         plans[j]->built = 1;
-        CR_LAUNCH(ctx, k_plan_reset, 1, 1, 0, plans[j]->d_info, (unsigned long long)n);
+        if (j == 0 || n == 0 || n > kPlanSortOneCta)  // small intervals: the admission CTA writes every field
+            CR_LAUNCH(ctx, k_plan_reset, 1, 1, 0, plans[j]->d_info, (unsigned long long)n);
     }
     cr_plan *p0 = plans[0];
     const unsigned int gcap = (unsigned int)ctx->num_sms * 8u;
@@ -1343,6 +1434,8 @@ extern "C" int cr_build_plans(cr_ctx *ctx, const uint64_t *d_key, uint64_t n, co
     // warp per plan, followed by their tables.
     lpt_jobs lj;
     uint32_t n_lj = 0, lj_maxR = 0, deferred[16];
+    const bool fused = n > 0 && n <= kPlanSortOneCta;  // small intervals: batched launches throughout
+    const bool tables_later = fused;
     auto table_insert = [&](uint32_t j) -> int {
         cr_plan *p = plans[j];
         const uint64_t C = (uint64_t)params[j].R * params[j].W;
@@ -1366,13 +1459,13 @@ extern "C" int cr_build_plans(cr_ctx *ctx, const uint64_t *d_key, uint64_t n, co
             CR_LAUNCH(ctx, k_plan_lpt_reg<16>, n_lj, 32, 0, lj, ctx->d_status);
         else
             CR_LAUNCH(ctx, k_plan_lpt_reg<32>, n_lj, 32, 0, lj, ctx->d_status);
-        for (uint32_t x = 0; x < n_lj; ++x) CR_TRY(table_insert(deferred[x]));
+        if (!tables_later)
+            for (uint32_t x = 0; x < n_lj; ++x) CR_TRY(table_insert(deferred[x]));
         n_lj = 0;
         lj_maxR = 0;
         return CR_OK;
     };
     // small intervals: admission of every plan in one launch, one CTA per plan
-    const bool fused = n > 0 && n <= kPlanSortOneCta;
     if (fused) {
         for (uint32_t j0 = 0; j0 < n_plans; j0 += 16) {
             admit_jobs aj;
@@ -1395,11 +1488,106 @@ extern "C" int cr_build_plans(cr_ctx *ctx, const uint64_t *d_key, uint64_t n, co
                 J.den = pp.qcap_den;
                 J.R = pp.R;
                 J.norepl = pp.variant == CR_VARIANT_NOREPL ? 1 : 0;
+                J.ukey_out = j0 + x > 0 ? p->d_ukey : nullptr;  // every plan keeps the histogram
+                J.ucnt_out = j0 + x > 0 ? p->d_ucnt : nullptr;
             }
             CR_LAUNCH(ctx, k_plan_admit_cta, nj, kSmallBlock, 0, aj, (const cr_plan_info_dev *)p0->d_info, order,
                       (const unsigned long long *)p0->d_ukey, (const unsigned long long *)p0->d_ucnt,
                       (unsigned long long)n, ctx->d_status);
         }
+        // placements: random and single-warp LPT plans batched per launch
+        place_jobs rj, l32;
+        uint32_t nr = 0, n32 = 0, rmaxR = 0;
+        uint64_t radm = 0;
+        auto flush_random = [&]() -> int {
+            if (!nr) return CR_OK;
+            const size_t smem = (size_t)kRandWarps * rmaxR * sizeof(uint16_t);
+            if (smem > 48 * 1024)
+                CR_CUDA(ctx, cudaFuncSetAttribute(k_plan_random_multi, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                                  (int)smem));
+            CR_LAUNCH(ctx, k_plan_random_multi, dim3(cr_blocks(radm, kRandWarps, gcap), nr), kRandWarps * 32, smem,
+                      rj, ctx->d_status);
+            nr = 0;
+            rmaxR = 0;
+            radm = 0;
+            return CR_OK;
+        };
+        auto flush_l32 = [&]() -> int {
+            if (!n32) return CR_OK;
+            CR_LAUNCH(ctx, k_plan_lpt32_multi, n32, 32, 0, l32, ctx->d_status);
+            n32 = 0;
+            return CR_OK;
+        };
+        for (uint32_t j = 0; j < n_plans; ++j) {
+            cr_plan *p = plans[j];
+            const cr_plan_params &pp = params[j];
+            const uint64_t C = (uint64_t)pp.R * pp.W;
+            place_job J;
+            J.info = p->d_info;
+            J.adm_cnt = p->d_adm_cnt;
+            J.adm_k = p->d_adm_k;
+            J.koff = p->d_koff;
+            J.load = p->d_load;
+            J.jobs = p->d_jobs;
+            J.members = p->d_members;
+            J.seed = pp.seed;
+            J.epoch = pp.epoch;
+            J.R = pp.R;
+            if (pp.variant == CR_VARIANT_RANDOM) {
+                rj.j[nr++] = J;
+                rmaxR = pp.R > rmaxR ? pp.R : rmaxR;
+                radm = (n < C ? n : C) > radm ? (n < C ? n : C) : radm;
+                if (nr == 16) CR_TRY(flush_random());
+            } else if (pp.R <= 32) {
+                l32.j[n32++] = J;
+                if (n32 == 16) CR_TRY(flush_l32());
+            } else if (pp.R <= 1024) {
+                lpt_job &jb = lj.j[n_lj++];
+                jb.info = p->d_info;
+                jb.adm_cnt = p->d_adm_cnt;
+                jb.adm_k = p->d_adm_k;
+                jb.koff = p->d_koff;
+                jb.load = p->d_load;
+                jb.members = p->d_members;
+                jb.jobs = p->d_jobs;
+                jb.R = pp.R;
+                lj_maxR = pp.R > lj_maxR ? pp.R : lj_maxR;
+                deferred[n_lj - 1] = j;
+                if (n_lj == 16) CR_TRY(flush_lpt());
+            } else {
+                const size_t smem = (size_t)pp.R * (sizeof(unsigned long long) + 1) + 16;
+                if (smem > 48 * 1024)
+                    CR_CUDA(ctx, cudaFuncSetAttribute(k_plan_lpt, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                                      (int)smem));
+                CR_LAUNCH(ctx, k_plan_lpt, 1, 32, smem, (const cr_plan_info_dev *)p->d_info,
+                          (const unsigned long long *)p->d_adm_cnt, (const uint32_t *)p->d_adm_k,
+                          (const uint32_t *)p->d_koff, pp.R, p->d_load, p->d_members, p->d_jobs, ctx->d_status);
+            }
+        }
+        CR_TRY(flush_random());
+        CR_TRY(flush_l32());
+        CR_TRY(flush_lpt());
+        // tables of every plan, batched per launch
+        for (uint32_t j0 = 0; j0 < n_plans; j0 += 16) {
+            table_jobs tj;
+            const uint32_t nj = n_plans - j0 < 16 ? n_plans - j0 : 16;
+            uint64_t adm = 0;
+            for (uint32_t x = 0; x < nj; ++x) {
+                cr_plan *p = plans[j0 + x];
+                const uint64_t C = (uint64_t)params[j0 + x].R * params[j0 + x].W;
+                adm = (n < C ? n : C) > adm ? (n < C ? n : C) : adm;
+                table_job &T = tj.j[x];
+                T.info = p->d_info;
+                T.adm_key = p->d_adm_key;
+                T.adm_k = p->d_adm_k;
+                T.koff = p->d_koff;
+                T.members = p->d_members;
+                T.table = p->d_table;
+                T.bits = bits_for(p->table_slots - 1);
+            }
+            CR_LAUNCH(ctx, k_table_insert_multi, dim3(cr_blocks(adm, 256, gcap), nj), 256, 0, tj);
+        }
+        return CR_OK;
     }
     for (uint32_t j = 0; j < n_plans; ++j) {
         cr_plan *p = plans[j];
