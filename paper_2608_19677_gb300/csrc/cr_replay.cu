@@ -500,7 +500,7 @@ int launch_batch_nc(cr_ctx *ctx, cr_replay *rp, const replay_caps &caps, uint32_
 {
     const uint32_t cmax = rp->cmax;
     int tbits = 6;
-    while ((1u << tbits) < 2 * cmax) ++tbits;
+    while ((1u << tbits) < 4 * cmax) ++tbits;  // index at most a quarter full of live keys
     const size_t per_warp = ((size_t)(1u << tbits) * 2 + 128 + (size_t)cmax * 10 + 15) & ~(size_t)15;
     // warps per block: the most warps per SM that shared memory allows
     const size_t sm_bytes = 227 * 1024;
