@@ -1017,6 +1017,11 @@ __device__ __forceinline__ bool lpt_equal_run(unsigned long long (&v)[NE], uint3
     return true;
 }
 
+// LPT for R <= 32 uses the sorted-lane kernel (fastest per key) unless the slot
+// budget admits this many keys or more: long admission lists reach the long
+// runs of equal counts in the tail, which the register kernel places at once.
+constexpr uint64_t kLptRunsFrom = 512;
+
 template <int NE>
 __global__ void __launch_bounds__(32) k_plan_lpt_reg(const __grid_constant__ lpt_jobs jobs_in, uint32_t *status)
 {
@@ -1449,7 +1454,9 @@ extern "C" int cr_build_plans(cr_ctx *ctx, const uint64_t *d_key, uint64_t n, co
     auto flush_lpt = [&]() -> int {
         if (!n_lj) return CR_OK;
         const uint32_t ne = (lj_maxR + 31) / 32;
-        if (ne <= 2)
+        if (ne <= 1)
+            CR_LAUNCH(ctx, k_plan_lpt_reg<1>, n_lj, 32, 0, lj, ctx->d_status);
+        else if (ne <= 2)
             CR_LAUNCH(ctx, k_plan_lpt_reg<2>, n_lj, 32, 0, lj, ctx->d_status);
         else if (ne <= 4)
             CR_LAUNCH(ctx, k_plan_lpt_reg<4>, n_lj, 32, 0, lj, ctx->d_status);
@@ -1538,7 +1545,7 @@ extern "C" int cr_build_plans(cr_ctx *ctx, const uint64_t *d_key, uint64_t n, co
                 rmaxR = pp.R > rmaxR ? pp.R : rmaxR;
                 radm = (n < C ? n : C) > radm ? (n < C ? n : C) : radm;
                 if (nr == 16) CR_TRY(flush_random());
-            } else if (pp.R <= 32) {
+            } else if (pp.R <= 32 && C < kLptRunsFrom) {
                 l32.j[n32++] = J;
                 if (n32 == 16) CR_TRY(flush_l32());
             } else if (pp.R <= 1024) {
@@ -1638,7 +1645,7 @@ extern "C" int cr_build_plans(cr_ctx *ctx, const uint64_t *d_key, uint64_t n, co
                 if (smem > 48 * 1024)
                     CR_CUDA(ctx, cudaFuncSetAttribute(k_plan_lpt, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                                       (int)smem));
-                if (pp.R <= 32)
+                if (pp.R <= 32 && C < kLptRunsFrom)
                     CR_LAUNCH(ctx, k_plan_lpt32, 1, 32, 0, (const cr_plan_info_dev *)p->d_info,
                               (const unsigned long long *)p->d_adm_cnt, (const uint32_t *)p->d_adm_k,
                               (const uint32_t *)p->d_koff, pp.R, p->d_load, p->d_members, p->d_jobs,
