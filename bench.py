@@ -551,7 +551,7 @@ def e2e(args, ctx, pipe, inputs, dev, stream, n_step, world):
         host.append((t, h, g0, n))
         h2d += sum(x.numel() * x.element_size() for x in h)
     max_tok = max(x[1][0].numel() for x in host)
-    NB = 3  # input buffers: the replay, their last reader, runs up to an interval behind the copies
+    NB = 4  # input buffers: the replay, their last reader, runs intervals behind the copies
     max_n = max(x[3] for x in host)
     bufs = [(torch.empty(max_tok, dtype=torch.int32, device=dev), torch.empty(max_n, dtype=torch.int64, device=dev),
              torch.empty(max_n, dtype=torch.int32, device=dev), torch.empty(max_n, dtype=torch.int32, device=dev))
@@ -596,7 +596,7 @@ def e2e(args, ctx, pipe, inputs, dev, stream, n_step, world):
     ms = e0.elapsed_time(e1) / args.e2e_steps
     return {"value": n_step * world / (ms / 1e3), "unit": UNIT, "h2d_bytes_per_step": h2d,
             "d2h_bytes_per_step": d2h, "ms_per_step": ms,
-            "note": "pinned host -> HBM copies on a second stream overlapped with compute (three buffers)"}
+            "note": "pinned host -> HBM copies on a second stream overlapped with compute (four buffers)"}
 
 
 if __name__ == "__main__":
