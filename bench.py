@@ -33,7 +33,7 @@ METRIC = "requests/s routed+shadow-replayed on 1 GB300 (and % HBM roofline); pla
 UNIT = "requests/s"
 
 
-def parse_args():
+def parse_args(argv=None):
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
     ap.add_argument("--steps", type=int, default=20)
@@ -50,7 +50,7 @@ def parse_args():
                          "(automatic when the arenas do not fit in HBM)")
     ap.add_argument("--intervals", type=int, default=0,
                     help="profiling aid: run only the first N intervals (the JSON line says so)")
-    return ap.parse_args()
+    return ap.parse_args(argv)
 
 
 def workload_config(cfg, B):
@@ -209,6 +209,30 @@ def run_reference(args):
     print(json.dumps(line), flush=True)
 
 
+# ----------------------------------------------------------- multi-rank ---
+# One process per GPU, each running an independent replica of the workload
+# (the path has no exchange step, so ranks share nothing but the timing).
+def replica_cfg(cfg, rank: int, world: int):
+    """The workload of one rank: the same configuration with its own trace seed."""
+    import dataclasses
+    return dataclasses.replace(cfg, trace_seed=cfg.trace_seed + rank) if world > 1 else cfg
+
+
+def max_over_ranks(x: float, world: int, device) -> float:
+    """The slowest rank's value (the job ends when the last rank does)."""
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([x], dtype=torch.float64, device=device)
+    if world > 1:
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_throughput(units_per_rank: int, world: int, ms_max: float) -> float:
+    """Units of all ranks per second of the slowest rank's time."""
+    return units_per_rank * world / (ms_max / 1e3)
+
+
 # ----------------------------------------------------------------- ours ---
 def main():
     args = parse_args()
@@ -238,9 +262,7 @@ def main():
     from paper_2608_19677_gb300.pipeline import Pipeline
 
     cfg = tg.CONFIGS[args.config]
-    if world > 1:  # independent replica per rank
-        import dataclasses
-        cfg = dataclasses.replace(cfg, trace_seed=cfg.trace_seed + rank)
+    cfg = replica_cfg(cfg, rank, world)  # independent replica per rank
     trace = tg.Trace(cfg)
     dev = torch.device("cuda", local)
     stream = torch.cuda.current_stream(dev)
@@ -334,11 +356,8 @@ def main():
     ctx.sync()
     ms_total = ev0.elapsed_time(ev1)
     ms = ms_total / args.steps
-    t_max = torch.tensor([ms], dtype=torch.float64, device=dev)
-    if world > 1:
-        dist.all_reduce(t_max, op=dist.ReduceOp.MAX)
-    ms_max = float(t_max.item())
-    value = n_step * world / (ms_max / 1e3)
+    ms_max = max_over_ranks(ms, world, dev)
+    value = job_throughput(n_step, world, ms_max)
 
     # per-stage summaries (hash and plan builds are timed on their own streams)
     hash_ms = np.array([[a.elapsed_time(b) for a, b in hm] for hm in hash_marks])
@@ -473,10 +492,7 @@ def run_keys_mode(args, cfg, trace, dev, stream, world, rank, barrier):
     clk = clocks.stop()
     pipe.sync()
     ms = ev0.elapsed_time(ev1) / args.steps
-    t_max = torch.tensor([ms], dtype=torch.float64, device=dev)
-    if world > 1:
-        dist.all_reduce(t_max, op=dist.ReduceOp.MAX)
-    ms_max = float(t_max.item())
+    ms_max = max_over_ranks(ms, world, dev)
     stage = np.zeros((args.steps, cfg.n_intervals, 4))
     for k in range(args.steps):
         for t in range(cfg.n_intervals):
@@ -506,7 +522,7 @@ def run_keys_mode(args, cfg, trace, dev, stream, world, rank, barrier):
     rr_rps = n_step / (ms_max / 1e3)
     rr_gbs = rr_bytes * rr_rps / 1e9
     line = {
-        "metric": METRIC, "value": n_step * world / (ms_max / 1e3), "unit": UNIT, "n_gpus": world,
+        "metric": METRIC, "value": job_throughput(n_step, world, ms_max), "unit": UNIT, "n_gpus": world,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_max, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "u64", "data": "synthetic",
         "config": dict(workload_config(cfg, args.batch),
@@ -593,8 +609,8 @@ def e2e(args, ctx, pipe, inputs, dev, stream, n_step, world):
         step()
     e1.record(stream)
     torch.cuda.synchronize()
-    ms = e0.elapsed_time(e1) / args.e2e_steps
-    return {"value": n_step * world / (ms / 1e3), "unit": UNIT, "h2d_bytes_per_step": h2d,
+    ms = max_over_ranks(e0.elapsed_time(e1) / args.e2e_steps, world, dev)
+    return {"value": job_throughput(n_step, world, ms), "unit": UNIT, "h2d_bytes_per_step": h2d,
             "d2h_bytes_per_step": d2h, "ms_per_step": ms,
             "note": "pinned host -> HBM copies on a second stream overlapped with compute (four buffers)"}
 
