@@ -1,14 +1,20 @@
 // a2..a6: per-interval plan construction (Eq. 1 and Algorithm 1).
 //
-//   histogram   radix sort of the interval's keys, run-length encoding -> (b, lambda_b)
-//   order       stable radix sort of (n - lambda_b): lambda descending, key ascending
-//   per plan    k_b (Eq. 1), inclusive scan of k_b, admission cut, admitted arrays,
-//               cold-tail total, placement (LPT: one warp, sequential over admitted
-//               keys, warp argmin over cached per-lane minima; RANDOM: one warp per
-//               key, Fisher-Yates steps in shared memory), then the device hash
-//               table b -> (offset, k_b, first member) used by dispatch.
-// No host synchronisation: sizes known only on the device (U, n_adm) are read
-// by the kernels, and grids are sized from host-side upper bounds.
+//   histogram   warp-aggregated counts in an L2-resident open-addressing table,
+//               occupied slots compacted to (b, lambda_b)
+//   order       (lambda desc, key asc): for intervals of up to 524,288 requests
+//               one CTA sorts only the admission candidates (the keys whose count
+//               reaches the C-th largest, C = R*W); above, device-wide radix
+//               passes sort every key
+//   per plan    k_b (Eq. 1), inclusive scan of k_b, admission cut, admitted
+//               arrays, cold-tail total and initial loads (small intervals: every
+//               plan in one launch, one CTA each), placement (LPT: one warp per
+//               plan, warp argmin over per-lane minima, runs of equal-count
+//               single-copy keys placed at once; RANDOM: one warp per key,
+//               Fisher-Yates steps in shared memory), then the device hash table
+//               b -> (offset, k_b, first member) used by dispatch.
+// No host synchronisation: sizes known only on the device (U, S, n_adm) are
+// read by the kernels, and grids are sized from host-side upper bounds.
 #include <stdlib.h>
 #include <string.h>
 
@@ -1596,6 +1602,7 @@ extern "C" int cr_build_plans(cr_ctx *ctx, const uint64_t *d_key, uint64_t n, co
         }
         return CR_OK;
     }
+    // large intervals (and empty ones): plan by plan
     for (uint32_t j = 0; j < n_plans; ++j) {
         cr_plan *p = plans[j];
         const cr_plan_params &pp = params[j];
@@ -1605,13 +1612,11 @@ extern "C" int cr_build_plans(cr_ctx *ctx, const uint64_t *d_key, uint64_t n, co
                                          cudaMemcpyDeviceToDevice, ctx->stream));
             CR_CUDA(ctx, cudaMemcpyAsync(p->d_ucnt, p0->d_ucnt, n * sizeof(unsigned long long),
                                          cudaMemcpyDeviceToDevice, ctx->stream));
-            if (!fused)
-                CR_CUDA(ctx, cudaMemcpyAsync(&p->d_info->U, &p0->d_info->U, 2 * sizeof(unsigned long long),
-                                             cudaMemcpyDeviceToDevice, ctx->stream));  // U and S
+            CR_CUDA(ctx, cudaMemcpyAsync(&p->d_info->U, &p0->d_info->U, 2 * sizeof(unsigned long long),
+                                         cudaMemcpyDeviceToDevice, ctx->stream));  // U and S
         }
-        if (!fused)
-            CR_CUDA(ctx, cudaMemsetAsync(p->d_table, 0xff, p->table_slots * sizeof(cr_table_slot), ctx->stream));
-        if (n > 0 && !fused) {
+        CR_CUDA(ctx, cudaMemsetAsync(p->d_table, 0xff, p->table_slots * sizeof(cr_table_slot), ctx->stream));
+        if (n > 0) {
             void *pk;
             CR_TRY(cr_scratch(ctx, SCR_PLAN_B, (n + 2) * sizeof(unsigned long long), &pk));
             unsigned long long *kk = (unsigned long long *)pk;
@@ -1625,9 +1630,8 @@ extern "C" int cr_build_plans(cr_ctx *ctx, const uint64_t *d_key, uint64_t n, co
                       (const unsigned long long *)p->d_ucnt, (const unsigned long long *)kk, p->d_info,
                       p->d_adm_key, p->d_adm_cnt, p->d_adm_k, p->d_koff);
         }
-        if (!fused)
-            CR_LAUNCH(ctx, k_plan_init_load, cr_blocks(pp.R, 256, gcap), 256, 0, p->d_info,
-                      (const unsigned long long *)pp.d_init_load, pp.R, p->d_load, ctx->d_status);
+        CR_LAUNCH(ctx, k_plan_init_load, cr_blocks(pp.R, 256, gcap), 256, 0, p->d_info,
+                  (const unsigned long long *)pp.d_init_load, pp.R, p->d_load, ctx->d_status);
         if (n > 0) {
             if (pp.variant == CR_VARIANT_RANDOM) {
                 size_t smem = (size_t)kRandWarps * pp.R * sizeof(uint16_t);
