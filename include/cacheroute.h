@@ -14,6 +14,7 @@
  *   cr_hash_prefixes  request prefix span -> 64-bit routing key b
  *   cr_build_plan     keys of one interval -> lambda_b, k_b, admission, LPT, table
  *   cr_route_batch    keys -> one destination per (request, replica)
+ *   cr_ring_create    consistent-hashing ring of the bounded-load comparison policy
  *   cr_shadow_replay  routed requests -> per-destination LRU hits and load
  *
  * Conventions shared by every call:
@@ -63,6 +64,7 @@ extern "C" {
 #define CR_POLICY_P2C 3        /* power-of-two choices over all R ("Flat-LB")   */
 #define CR_POLICY_RR 4         /* round robin over the global request index      */
 #define CR_POLICY_HASH 5       /* sticky: jump consistent hash of the key        */
+#define CR_POLICY_CHWBL 6      /* consistent hashing with bounded loads, eps 1/4 */
 
 /* ---- plan variants (cr_plan_params.variant) ------------------------------- */
 #define CR_VARIANT_LPT 0    /* Algorithm 1 as printed                            */
@@ -74,11 +76,13 @@ extern "C" {
 #define CR_MAX_CAP 1024       /* LRU capacity (prefix entries) per simulator     */
 #define CR_MAX_CAPS 8         /* capacities replayed together                    */
 #define CR_MAX_REPLICAS 256   /* (policy, seed) replicas per route/replay call   */
+#define CR_MAX_VNODES 1024    /* ring points per destination (cr_ring_create)    */
 #define CR_CTR_FIELDS 5       /* requests, hits, hit tokens, prompt, prefill     */
 
 typedef struct cr_ctx cr_ctx;
 typedef struct cr_plan cr_plan;
 typedef struct cr_replay cr_replay;
+typedef struct cr_ring cr_ring;
 
 /* ==== context ============================================================ */
 
@@ -204,18 +208,38 @@ CR_API int cr_plan_export(cr_ctx *ctx, const cr_plan *plan, uint64_t *ukey, uint
 
 /* ==== a7: batched dispatch ========================================== */
 
+/*
+ * Ring of the bounded-load comparison policy (CHWBL, sec. 4; epsilon = 0.25;
+ * consistent hashing with bounded loads, Mirrokni, Thorup and Zadimoghaddam,
+ * SODA 2018).  The paper fixes epsilon only; the ring is this library's
+ * reading: destination d owns `vnodes` points, point (d, v) being output
+ * number k = d*vnodes + v of SplitMix64 from state `seed`, that is
+ * fmix64(seed + (k + 1) * 0x9e3779b97f4a7c15) mod 2^64, and the ring lists
+ * the R*vnodes points in ascending (point, d) order.
+ * cr_ring_create builds it on the device (enqueued on the context's stream;
+ * R in 1..CR_MAX_R, vnodes in 1..CR_MAX_VNODES).  Errors: CR_EINVAL,
+ * CR_ENOMEM, CR_ECUDA.  The ring is read-only afterwards and may be shared
+ * by any number of replicas and calls. */
+CR_API int cr_ring_create(cr_ctx *ctx, uint32_t R, uint32_t vnodes, uint64_t seed, cr_ring **out);
+/* Destroy (waits for the context's stream).  NULL is accepted. */
+CR_API int cr_ring_destroy(cr_ctx *ctx, cr_ring *ring);
+/* Blocking: copy the ring to host arrays point[R*vnodes] (ascending) and
+ * owner[R*vnodes]. */
+CR_API int cr_ring_export(cr_ctx *ctx, const cr_ring *ring, uint64_t *point, uint16_t *owner);
+
 typedef struct {
-    uint32_t policy;  /* CR_POLICY_* */
-    uint32_t reserved;/* must be 0 */
-    uint64_t seed;    /* RNG / offset / hash seed of this replica */
+    uint32_t policy;      /* CR_POLICY_* */
+    uint32_t reserved;    /* must be 0 */
+    uint64_t seed;        /* RNG / offset / hash seed of this replica */
+    const cr_ring *ring;  /* CR_POLICY_CHWBL: its ring (R destinations); else ignored */
 } cr_replica;
 
 /*
  * Route requests d_key[n] (device, arrival order, global request indices
  * first_req_index .. first_req_index+n-1) for n_rep replicas at once.
  *   plans[i]  plan used by replica i (CACHEROUTE, CR_NOLPT, CR_NOREPL), or
- *             NULL for P2C, RR and HASH.  Plans may be shared; plan R must
- *             equal R.
+ *             NULL for P2C, RR, HASH and CHWBL.  Plans may be shared; plan R
+ *             must equal R.
  *   reps[i]   policy and seed (host array)
  *   batch_B   requests are taken in batches of batch_B (>= 1); every request
  *             of a batch sees the load vector as it stood when the batch
@@ -231,8 +255,19 @@ typedef struct {
  *     d1 = floor(u0 R / 2^64), d2 = (d1 + 1 + floor(u1 (R-1) / 2^64)) mod R;
  *     pick d1 if load[d1] <= load[d2], else d2.
  *   RR: (g + seed) mod R.     HASH: jump_hash(fmix64(b ^ seed), R).
+ *   CHWBL: with m = the sum of the load vector the request sees, every
+ *     destination may hold cap = ceil(5 (m + 1) / (4 R)) requests; starting
+ *     at the first ring point >= fmix64(b ^ seed) (wrapping to the first
+ *     point), walk the ring and take the first owner whose load is < cap.
+ *     The least-loaded destination is always below cap, so the walk ends.
+ * Batches of at most 32 requests are resolved by one warp per replica that
+ * takes 32 // batch_B whole batches per step; longer batches by one CTA per
+ * replica.  Both give the sequential result defined above.
  * Errors: CR_EINVAL (R == 0 or > CR_MAX_R, n_rep > CR_MAX_REPLICAS, missing
- * or mismatched plan, batch_B == 0, n >= 2^40). */
+ * or mismatched plan or ring, batch_B == 0, n >= 2^40).  A load sum that
+ * has wrapped past 2^64 can leave no destination below cap: the request then
+ * takes the owner of its first ring point and the next blocking call
+ * reports CR_EOVERFLOW. */
 CR_API int cr_route_batch(cr_ctx *ctx, const cr_plan *const *plans, const cr_replica *reps,
                    uint32_t n_rep, uint32_t R, const uint64_t *d_key, uint64_t n,
                    uint64_t first_req_index, uint32_t batch_B, uint64_t *d_load,

@@ -39,7 +39,7 @@ _LIB = os.path.join(_HERE, "libcr_oracle.so")
 
 CTR_FIELDS = ("requests", "hits", "hit_tokens", "prompt_tokens", "prefill_tokens")
 VARIANT = {"LPT": 0, "RANDOM": 1, "NOREPL": 2}
-POLICY = {"CR": 0, "CR_NOLPT": 1, "CR_NOREPL": 2, "P2C": 3, "RR": 4, "HASH": 5}
+POLICY = {"CR": 0, "CR_NOLPT": 1, "CR_NOREPL": 2, "P2C": 3, "RR": 4, "HASH": 5, "CHWBL": 6}
 
 
 def build(force: bool = False) -> str:
@@ -75,8 +75,12 @@ def lib():
         _lib.orc_jump_hash.restype = C.c_uint32
         _lib.orc_jump_hash.argtypes = [C.c_uint64, C.c_uint32]
         _lib.orc_route.restype = C.c_int
-        _lib.orc_route.argtypes = [C.c_void_p, u32p, u64p, C.c_uint32, C.c_uint32, u64p,
+        _lib.orc_route.argtypes = [C.c_void_p, C.c_void_p, u32p, u64p, C.c_uint32, C.c_uint32, u64p,
                                    C.c_uint64, C.c_uint64, C.c_uint32, u64p, u16p]
+        _lib.orc_ring_create.restype = C.c_void_p
+        _lib.orc_ring_create.argtypes = [C.c_uint32, C.c_uint32, C.c_uint64]
+        _lib.orc_ring_free.argtypes = [C.c_void_p]
+        _lib.orc_ring_export.argtypes = [C.c_void_p, u64p, u16p]
         _lib.orc_replay_create.restype = C.c_void_p
         _lib.orc_replay_create.argtypes = [C.c_uint32, C.c_uint32, u32p, C.c_uint32]
         _lib.orc_replay_free.argtypes = [C.c_void_p]
@@ -228,8 +232,32 @@ def build_plan(keys, R: int, W: int, qcap_num: int, qcap_den: int, variant="LPT"
 
 
 # -- a7 ----------------------------------------------------------------------
+class Ring:
+    """Consistent-hashing ring of the bounded-load policy: R destinations x V points."""
+
+    def __init__(self, R: int, V: int, seed: int):
+        self.R, self.V, self.seed = R, V, seed & ((1 << 64) - 1)
+        self._h = lib().orc_ring_create(R, V, self.seed)
+        if not self._h:
+            raise ValueError("orc_ring_create: invalid arguments")
+
+    def __del__(self):
+        if getattr(self, "_h", None):
+            lib().orc_ring_free(self._h)
+            self._h = None
+
+    def export(self):
+        """(point uint64 [R*V] ascending, owner uint16 [R*V])."""
+        M = self.R * self.V
+        pt = np.zeros(M, np.uint64)
+        ow = np.zeros(M, np.uint16)
+        lib().orc_ring_export(self._h, _p(pt, C.c_uint64), _p(ow, C.c_uint16))
+        return pt, ow
+
+
 def route(plans: Sequence[Optional[Plan]], policies: Sequence, seeds: Sequence[int], R: int,
-          keys, g0: int, B: int, load: Optional[np.ndarray] = None):
+          keys, g0: int, B: int, load: Optional[np.ndarray] = None,
+          rings: Optional[Sequence[Optional[Ring]]] = None):
     """Returns (dest uint16 [n_rep, n], load uint64 [n_rep, R])."""
     n_rep = len(policies)
     k = _c(keys, np.uint64)
@@ -241,8 +269,10 @@ def route(plans: Sequence[Optional[Plan]], policies: Sequence, seeds: Sequence[i
     structs = [pl._struct() if pl is not None else None for pl in plans]
     ptrs = (C.c_void_p * n_rep)(*[C.cast(C.pointer(s), C.c_void_p) if s is not None else None
                                   for s in structs])
+    rg = rings if rings is not None else [None] * n_rep
+    rptrs = (C.c_void_p * n_rep)(*[r._h if r is not None else None for r in rg])
     kk = k if n else np.zeros(1, np.uint64)
-    rc = lib().orc_route(ptrs, _p(pol, C.c_uint32), _p(sd, C.c_uint64), n_rep, R,
+    rc = lib().orc_route(ptrs, rptrs, _p(pol, C.c_uint32), _p(sd, C.c_uint64), n_rep, R,
                          _p(kk, C.c_uint64), n, g0, B, _p(ld, C.c_uint64),
                          _p(dest, C.c_uint16))
     if rc != 0:

@@ -25,8 +25,10 @@
  *       Algorithm 1 placement loop).
  *   orc_route ........................ dispatch (Fig. 1; sec. 3.1: least-loaded
  *       member of T(b), otherwise power-of-two choices over the fleet) and the
- *       comparison policies of sec. 4 (Flat-LB, sticky hashing) plus
- *       round-robin.
+ *       comparison policies of sec. 4 (Flat-LB, sticky hashing, consistent
+ *       hashing with bounded loads at epsilon = 0.25) plus round-robin.
+ *   orc_ring_* ....................... the consistent-hashing ring of that
+ *       bounded-load policy (the ring layout is this library's reading).
  *   orc_replay_* ..................... shadow replay of each destination's
  *       prefix cache as a whole-prefix LRU (deployment gate of sec. 3.2 and 5.3; the paper
  *       replays on hardware, the LRU model is this library's reading).
@@ -157,7 +159,7 @@ uint64_t orc_histogram(const uint64_t *key, uint64_t n, uint64_t *ukey, uint64_t
 /* ---------------------------------------------------------------------- */
 
 enum { ORC_VARIANT_LPT = 0, ORC_VARIANT_RANDOM = 1, ORC_VARIANT_NOREPL = 2 };
-enum { ORC_CR = 0, ORC_CR_NOLPT = 1, ORC_CR_NOREPL = 2, ORC_P2C = 3, ORC_RR = 4, ORC_HASH = 5 };
+enum { ORC_CR = 0, ORC_CR_NOLPT = 1, ORC_CR_NOREPL = 2, ORC_P2C = 3, ORC_RR = 4, ORC_HASH = 5, ORC_CHWBL = 6 };
 
 typedef struct {
     uint32_t R, W;
@@ -365,15 +367,118 @@ static uint32_t p2c(uint64_t seed, uint32_t policy, uint64_t g, uint32_t R, cons
 }
 
 /*
+ * Consistent-hashing ring for bounded-load dispatch (the CHWBL comparison
+ * policy of sec. 4, epsilon = 0.25; Mirrokni, Thorup and Zadimoghaddam, SODA
+ * 2018).  The paper fixes only epsilon; the ring is this library's reading:
+ * destination d owns V points, point (d, v) being output number d*V + v of
+ * SplitMix64 started from state `seed` (output k = fmix64(seed + (k+1)*gamma)),
+ * and the ring lists all R*V points in ascending (point, destination) order.
+ */
+typedef struct {
+    uint32_t R, V;
+    uint64_t M;       /* R * V */
+    uint64_t *point;  /* ascending */
+    uint16_t *owner;
+} orc_ring;
+
+typedef struct {
+    uint64_t point;
+    uint32_t owner;
+} ring_ent;
+
+static int cmp_ring_ent(const void *a, const void *b)
+{
+    const ring_ent *x = (const ring_ent *)a, *y = (const ring_ent *)b;
+    if (x->point != y->point)
+        return x->point < y->point ? -1 : 1;
+    return (x->owner > y->owner) - (x->owner < y->owner);
+}
+
+orc_ring *orc_ring_create(uint32_t R, uint32_t V, uint64_t seed)
+{
+    if (R == 0 || R > 65535 || V == 0)
+        return NULL;
+    uint64_t M = (uint64_t)R * V;
+    ring_ent *e = (ring_ent *)malloc(M * sizeof(ring_ent));
+    orc_ring *g = (orc_ring *)calloc(1, sizeof(orc_ring));
+    if (!e || !g) {
+        free(e);
+        free(g);
+        return NULL;
+    }
+    for (uint32_t d = 0; d < R; ++d)
+        for (uint32_t v = 0; v < V; ++v) {
+            uint64_t k = (uint64_t)d * V + v;
+            e[k].point = orc_fmix64(seed + (k + 1) * ORC_GAMMA);
+            e[k].owner = d;
+        }
+    qsort(e, M, sizeof(ring_ent), cmp_ring_ent);
+    g->R = R;
+    g->V = V;
+    g->M = M;
+    g->point = (uint64_t *)malloc(M * sizeof(uint64_t));
+    g->owner = (uint16_t *)malloc(M * sizeof(uint16_t));
+    for (uint64_t j = 0; j < M; ++j) {
+        g->point[j] = e[j].point;
+        g->owner[j] = (uint16_t)e[j].owner;
+    }
+    free(e);
+    return g;
+}
+
+void orc_ring_free(orc_ring *g)
+{
+    if (!g)
+        return;
+    free(g->point);
+    free(g->owner);
+    free(g);
+}
+
+void orc_ring_export(const orc_ring *g, uint64_t *point, uint16_t *owner)
+{
+    memcpy(point, g->point, g->M * sizeof(uint64_t));
+    memcpy(owner, g->owner, g->M * sizeof(uint16_t));
+}
+
+/* Bounded-load choice for one request.  Every destination may hold at most
+ * cap = ceil((1 + 1/4) (m + 1) / R) requests, m being the requests in the
+ * load vector; the request goes to the first destination, walking the ring
+ * clockwise from its key's position h (the first point >= h, wrapping to the
+ * start), whose load is below cap.  The least-loaded destination holds at most
+ * m / R < cap, so the walk always ends.  Returns R on an exhausted walk. */
+static uint32_t chwbl(const orc_ring *g, uint64_t h, uint32_t R, const uint64_t *snap, uint64_t m)
+{
+    uint64_t cap = (5 * (m + 1) + 4 * (uint64_t)R - 1) / (4 * (uint64_t)R);
+    uint64_t lo = 0, hi = g->M;
+    while (lo < hi) {
+        uint64_t mid = lo + (hi - lo) / 2;
+        if (g->point[mid] < h)
+            lo = mid + 1;
+        else
+            hi = mid;
+    }
+    uint64_t j = lo == g->M ? 0 : lo;
+    for (uint64_t t = 0; t < g->M; ++t) {
+        uint32_t d = g->owner[j];
+        if (snap[d] < cap)
+            return d;
+        j = j + 1 == g->M ? 0 : j + 1;
+    }
+    return R;
+}
+
+/*
  * Route n requests (arrival order, global indices g0..g0+n-1) for n_rep replicas.
  * Requests are taken in batches of B; every request of a batch sees the load
  * vector as it stood when the batch began, and the batch's counts are added
  * after it.  load is [n_rep][R] (in/out), dest is [n_rep][n].
- * plans[i] may be NULL for P2C, RR and HASH.
+ * plans[i] may be NULL for P2C, RR, HASH and CHWBL; rings[i] (R destinations)
+ * is needed by CHWBL only.  The key's ring position is fmix64(key ^ seed).
  */
-int orc_route(const orc_plan *const *plans, const uint32_t *policy, const uint64_t *seed,
-              uint32_t n_rep, uint32_t R, const uint64_t *key, uint64_t n, uint64_t g0,
-              uint32_t B, uint64_t *load, uint16_t *dest)
+int orc_route(const orc_plan *const *plans, const orc_ring *const *rings, const uint32_t *policy,
+              const uint64_t *seed, uint32_t n_rep, uint32_t R, const uint64_t *key, uint64_t n,
+              uint64_t g0, uint32_t B, uint64_t *load, uint16_t *dest)
 {
     if (R == 0 || R > 65535 || B == 0)
         return ORC_EINVAL;
@@ -381,7 +486,9 @@ int orc_route(const orc_plan *const *plans, const uint32_t *policy, const uint64
     for (uint32_t rp = 0; rp < n_rep; ++rp) {
         uint32_t pol = policy[rp];
         const orc_plan *pl = plans ? plans[rp] : NULL;
-        if (pol > ORC_HASH || (pol <= ORC_CR_NOREPL && !pl)) {
+        const orc_ring *rg = rings ? rings[rp] : NULL;
+        if (pol > ORC_CHWBL || (pol <= ORC_CR_NOREPL && !pl) ||
+            (pol == ORC_CHWBL && (!rg || rg->R != R))) {
             free(snap);
             return ORC_EINVAL;
         }
@@ -401,6 +508,9 @@ int orc_route(const orc_plan *const *plans, const uint32_t *policy, const uint64
         for (uint64_t b0 = 0; b0 < n; b0 += B) {
             uint64_t b1 = b0 + B < n ? b0 + B : n;
             memcpy(snap, L, R * sizeof(uint64_t));
+            uint64_t m = 0;
+            for (uint32_t r = 0; r < R; ++r)
+                m += snap[r];
             for (uint64_t i = b0; i < b1; ++i) {
                 uint64_t g = g0 + i;
                 uint32_t d;
@@ -410,6 +520,13 @@ int orc_route(const orc_plan *const *plans, const uint32_t *policy, const uint64
                     d = orc_jump_hash(orc_fmix64(key[i] ^ seed[rp]), R);
                 } else if (pol == ORC_P2C) {
                     d = p2c(seed[rp], pol, g, R, snap);
+                } else if (pol == ORC_CHWBL) {
+                    d = chwbl(rg, orc_fmix64(key[i] ^ seed[rp]), R, snap, m);
+                    if (d >= R) {
+                        free(tab);
+                        free(snap);
+                        return ORC_EINVAL;
+                    }
                 } else {
                     int64_t e = lookup(tab, nt, key[i]);
                     if (e >= 0) {

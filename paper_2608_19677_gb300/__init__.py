@@ -10,6 +10,7 @@ fails loudly otherwise.
   hash_prefixes   request prefix spans -> routing keys          (cr_hash_prefixes)
   build_plans     one interval's keys -> plans (Eq. 1, Alg. 1)  (cr_build_plans)
   route_batch     keys -> destination per (request, replica)    (cr_route_batch)
+  Ring            ring of the bounded-load policy               (cr_ring_create)
   shadow_replay   routed requests -> LRU hit / load counters    (cr_shadow_replay)
 """
 from __future__ import annotations
@@ -26,15 +27,16 @@ LIB_PATH = os.path.join(_HERE, "libcacheroute.so")
 CR_OK, CR_EINVAL, CR_ENOMEM, CR_ECUDA, CR_ETIMEOUT, CR_EOVERFLOW = range(6)
 STATUS_NAMES = {0: "CR_OK", 1: "CR_EINVAL", 2: "CR_ENOMEM", 3: "CR_ECUDA", 4: "CR_ETIMEOUT",
                 5: "CR_EOVERFLOW"}
-POLICY = {"CR": 0, "CR_NOLPT": 1, "CR_NOREPL": 2, "P2C": 3, "RR": 4, "HASH": 5}
+POLICY = {"CR": 0, "CR_NOLPT": 1, "CR_NOREPL": 2, "P2C": 3, "RR": 4, "HASH": 5, "CHWBL": 6}
 VARIANT = {"LPT": 0, "RANDOM": 1, "NOREPL": 2}
-MAX_R, MAX_CAP, MAX_CAPS, MAX_REPLICAS, CTR_FIELDS = 8192, 1024, 8, 256, 5
+MAX_R, MAX_CAP, MAX_CAPS, MAX_REPLICAS, CTR_FIELDS, MAX_VNODES = 8192, 1024, 8, 256, 5, 1024
 
 # every symbol the header declares (checked by the CPU test suite)
 EXPORTS = ("cr_create", "cr_destroy", "cr_set_stream", "cr_sync", "cr_last_error", "cr_launch_count",
            "cr_hash_prefixes", "cr_plan_create", "cr_plan_destroy", "cr_build_plans", "cr_build_plan",
            "cr_plan_get_info", "cr_plan_export", "cr_route_batch", "cr_replay_create", "cr_replay_reset",
-           "cr_replay_destroy", "cr_shadow_replay", "cr_replay_export_state", "cr_key_histogram_noalloc")
+           "cr_replay_destroy", "cr_shadow_replay", "cr_replay_export_state", "cr_key_histogram_noalloc",
+           "cr_ring_create", "cr_ring_destroy", "cr_ring_export")
 CR_NOALLOC_MAX_KEYS = 65536
 
 
@@ -56,7 +58,7 @@ class PlanInfo(C.Structure):
 
 
 class Replica(C.Structure):
-    _fields_ = [("policy", C.c_uint32), ("reserved", C.c_uint32), ("seed", C.c_uint64)]
+    _fields_ = [("policy", C.c_uint32), ("reserved", C.c_uint32), ("seed", C.c_uint64), ("ring", C.c_void_p)]
 
 
 _lib = None
@@ -99,6 +101,9 @@ def lib() -> C.CDLL:
         "cr_shadow_replay": ([vp, vp, vp, vp, vp, vp, u64, vp], i32),
         "cr_replay_export_state": ([vp, vp, u32, u32, vp, C.POINTER(C.c_uint32)], i32),
         "cr_key_histogram_noalloc": ([vp, u64, vp, vp, vp, vp], i32),
+        "cr_ring_create": ([vp, u32, u32, u64, C.POINTER(vp)], i32),
+        "cr_ring_destroy": ([vp, vp], i32),
+        "cr_ring_export": ([vp, vp, vp, vp], i32),
     }
     for name, (args, res) in sig.items():
         f = getattr(L, name)
@@ -253,9 +258,45 @@ def build_plan(ctx: Context, keys, params: PlanParams, plan: Optional[Plan] = No
     return plan
 
 
+class Ring:
+    """Consistent-hashing ring of the bounded-load policy (R destinations x vnodes points), on the device."""
+
+    def __init__(self, ctx: Context, R: int, vnodes: int, seed: int):
+        self.ctx, self.R, self.vnodes, self.seed = ctx, R, vnodes, seed & ((1 << 64) - 1)
+        h = C.c_void_p()
+        ctx.check(lib().cr_ring_create(ctx.handle, R, vnodes, self.seed, C.byref(h)), "cr_ring_create")
+        self._h = h
+
+    @property
+    def handle(self):
+        return self._h
+
+    def export(self):
+        """(point uint64 [R*vnodes] ascending, owner uint16 [R*vnodes]) on the host."""
+        M = self.R * self.vnodes
+        pt = np.zeros(M, np.uint64)
+        ow = np.zeros(M, np.uint16)
+        self.ctx.check(lib().cr_ring_export(self.ctx.handle, self._h, _np_ptr(pt), _np_ptr(ow)), "cr_ring_export")
+        return pt, ow
+
+    def close(self):
+        if getattr(self, "_h", None):
+            lib().cr_ring_destroy(self.ctx.handle, self._h)
+            self._h = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+
 def route_batch(ctx: Context, plans: Sequence[Optional[Plan]], policies: Sequence, seeds: Sequence[int],
-                R: int, keys, first_req_index: int, batch_B: int, load, dest=None):
-    """Destinations (uint16 values in an int16 tensor [n_rep, n]); ``load`` [n_rep, R] is updated in place."""
+                R: int, keys, first_req_index: int, batch_B: int, load, dest=None,
+                rings: Optional[Sequence[Optional[Ring]]] = None):
+    """Destinations (uint16 values in an int16 tensor [n_rep, n]); ``load`` [n_rep, R] is updated in place.
+
+    ``rings[i]`` is the ring of replica i when its policy is CHWBL."""
     import torch
     n_rep = len(policies)
     n = int(keys.shape[0])
@@ -264,8 +305,10 @@ def route_batch(ctx: Context, plans: Sequence[Optional[Plan]], policies: Sequenc
     if dest is None:
         dest = torch.empty((n_rep, n), dtype=torch.int16, device=keys.device)
     _need_cuda("dest", dest, torch.int16)
+    rg = list(rings) if rings is not None else [None] * n_rep
     reps = (Replica * n_rep)(*[Replica(POLICY[p] if isinstance(p, str) else int(p), 0,
-                                       int(s) & ((1 << 64) - 1)) for p, s in zip(policies, seeds)])
+                                       int(s) & ((1 << 64) - 1), (g.handle.value if g is not None else None))
+                               for p, s, g in zip(policies, seeds, rg)])
     hs = (C.c_void_p * n_rep)(*[(p.handle if p is not None else None) for p in plans])
     ctx.check(lib().cr_route_batch(ctx.handle, hs, reps, n_rep, R, _ptr(keys), n, first_req_index, batch_B,
                                    _ptr(load), _ptr(dest)), "cr_route_batch")

@@ -75,6 +75,16 @@ struct cr_plan {
     int built;
 };
 
+// Ring of the bounded-load policy: R*V points ascending, their owners, and a
+// directory dir[t] = first ring index whose point is >= t << (64 - dbits).
+struct cr_ring {
+    uint32_t R, V, dbits;
+    uint64_t M;
+    unsigned long long *d_point;
+    uint16_t *d_owner;
+    uint32_t *d_dir;
+};
+
 struct cr_replay {
     uint32_t n_rep, R, n_caps, cmax;
     uint32_t caps[CR_MAX_CAPS];

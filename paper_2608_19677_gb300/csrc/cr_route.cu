@@ -1,14 +1,32 @@
-// a7: batched dispatch (cr_route_batch).
+// a7: batched dispatch (cr_route_batch) and the ring of the bounded-load
+// comparison policy (cr_ring_*).
 //
 // Two passes.  k_route_cand runs over every (replica, request) pair at once and
 // does all the work that does not depend on the live load: the table probe,
-// the Philox draws of power-of-two choices, round robin and the jump hash.
-// Round-robin and hash replicas are then finished (their loads are counted by
-// k_route_count); every other replica leaves one packed candidate per request.
-// k_route_resolve then walks each load-dependent replica's requests in arrival
-// order, batch by batch, on one CTA that holds the replica's live load in
-// shared memory: a decision is one or two shared-memory reads, the batch's
-// counts accumulate in a second shared vector and are merged at the boundary.
+// the Philox draws of power-of-two choices, the ring position of consistent
+// hashing with bounded loads, round robin and the jump hash.  Round-robin and
+// hash replicas are then finished (their loads are counted by k_route_count);
+// every other replica leaves one packed candidate per request.  The
+// load-dependent pass then walks each replica's requests in arrival order:
+//   - batches longer than a warp: k_route_resolve, one CTA per replica that
+//     holds the live load in shared memory; a batch is resolved by all its
+//     threads against the batch-start loads, the batch's counts accumulate in
+//     a second shared vector and are merged at the boundary;
+//   - batches of at most 32 requests (batch_B = 1 is exact sequential
+//     dispatch): k_route_resolve_warp, one warp per replica taking
+//     S = floor(32 / B) * B requests (whole batches) per step.  Inside a step a
+//     request's decision depends on the destinations of the earlier batches of
+//     the step; the warp finds them by fixed-point iteration: every lane
+//     decides from the step-start loads plus the lanes of earlier batches that
+//     currently sit on each candidate (a per-destination lane bitmask in
+//     shared memory), until no lane changes.  After iteration t the first t
+//     batches are final, so at most S iterations are needed and typically two
+//     or three; the result is the sequential one.
+#include <stdlib.h>
+#include <string.h>
+
+#include <algorithm>
+
 #include "cr_device.cuh"
 #include "cr_internal.cuh"
 
@@ -16,6 +34,7 @@ namespace {
 
 constexpr int kRouteBlock = 1024;
 constexpr uint32_t kEmpty = 0xffffffffu;
+constexpr size_t kSmemBudget = 200 * 1024;  // dynamic shared memory a resolve CTA may take
 
 struct route_desc {
     uint32_t policy;
@@ -23,6 +42,12 @@ struct route_desc {
     unsigned long long seed;
     const cr_table_slot *table;
     const uint16_t *members;
+    const unsigned long long *n_members;  // device: the plan's sum of k_b
+    const unsigned long long *rpoint; // ring (CHWBL)
+    const uint16_t *rowner;
+    const uint32_t *rdir;
+    uint32_t rM;                      // ring points
+    int32_t rdbits;                   // log2 directory entries
 };
 
 struct route_args {
@@ -34,7 +59,9 @@ struct route_args {
 //   kind 0 FIXED  bits 0..15  destination (RR, HASH, and keys with k_b = 1)
 //   kind 1 PAIR   bits 0..12  d1, bits 13..25 d2 (power-of-two choices; R <= 8192)
 //   kind 2 SET    bits 0..29  table slot of a key with k_b > 1
-constexpr uint32_t kFixed = 0u << 30, kPair = 1u << 30, kSet = 2u << 30, kKindMask = 3u << 30;
+//   kind 3 RING   bits 0..29  first ring index at or after the key's position
+constexpr uint32_t kFixed = 0u << 30, kPair = 1u << 30, kSet = 2u << 30, kRing = 3u << 30,
+                   kKindMask = 3u << 30, kLow30 = 0x3fffffffu;
 
 __device__ __forceinline__ uint32_t p2c_pair(unsigned long long seed, uint32_t policy, unsigned long long g,
                                              uint32_t R)
@@ -43,6 +70,21 @@ __device__ __forceinline__ uint32_t p2c_pair(unsigned long long seed, uint32_t p
     uint32_t d1 = cr_scale(u.x, R);
     uint32_t d2 = (uint32_t)((d1 + 1ull + cr_scale(u.y, (unsigned long long)(R - 1))) % R);
     return kPair | d1 | (d2 << 13);
+}
+
+// First ring index whose point is >= h, wrapping to 0 past the last point.
+__device__ __forceinline__ uint32_t ring_start(const route_desc &rd, unsigned long long h)
+{
+    uint32_t j = rd.rdir[h >> (64 - rd.rdbits)];
+    while (j < rd.rM && rd.rpoint[j] < h) ++j;
+    return j == rd.rM ? 0u : j;
+}
+
+// ceil(5 (m + 1) / (4 R)): the per-destination bound at epsilon = 1/4.
+__device__ __forceinline__ unsigned long long chwbl_cap(unsigned long long m, uint32_t R)
+{
+    const unsigned long long den = 4ull * R;
+    return (5ull * (m + 1ull) + den - 1ull) / den;
 }
 
 // Everything that does not depend on the live load, for every (replica, request).
@@ -68,6 +110,9 @@ __global__ void __launch_bounds__(256) k_route_cand(const __grid_constant__ rout
             break;
         case CR_POLICY_P2C:
             cand[j] = p2c_pair(rd.seed, rd.policy, g, R);
+            break;
+        case CR_POLICY_CHWBL:
+            cand[j] = kRing | ring_start(rd, cr_fmix64(keys[i] ^ rd.seed));
             break;
         default: {
             const unsigned long long key = keys[i];
@@ -106,8 +151,72 @@ __global__ void __launch_bounds__(256) k_route_count(const uint16_t *__restrict_
         if (hist[r]) atomicAdd(&L[r], (unsigned long long)hist[r]);
 }
 
+// Walk the ring from index j for the first owner whose load is below cap.
+// The least-loaded destination always is, so the walk ends within M steps
+// unless the load sum has wrapped; then the first owner is taken and the
+// overflow flag raised.
+template <typename LoadOf>
+__device__ __forceinline__ uint32_t ring_walk(const route_desc &rd, uint32_t j, unsigned long long cap,
+                                              LoadOf load_of, uint32_t *status)
+{
+    const uint32_t j0 = j;
+    for (uint32_t t = 0; t < rd.rM; ++t) {
+        const uint32_t d = rd.rowner[j];
+        if (load_of(d) < cap) return d;
+        j = (j + 1 == rd.rM) ? 0u : j + 1;
+    }
+    atomicOr(status, CR_FLAG_OVERFLOW);
+    return rd.rowner[j0];
+}
+
+// Least-loaded member of T(b) = mem[off .. off + k), first member m0 given;
+// ties keep the earlier member.  Members are read four at a time.
+template <typename LoadOf>
+__device__ __forceinline__ uint32_t set_min(const uint16_t *mem, uint32_t off, uint32_t k, uint32_t m0,
+                                            LoadOf load_of)
+{
+    uint32_t best = m0;
+    unsigned long long bl = load_of(best);
+    uint32_t m = 1;
+    for (; m + 4 <= k; m += 4) {
+        uint32_t d[4];
+        unsigned long long l[4];
+#pragma unroll
+        for (int u = 0; u < 4; ++u) d[u] = mem[off + m + u];
+#pragma unroll
+        for (int u = 0; u < 4; ++u) l[u] = load_of(d[u]);
+#pragma unroll
+        for (int u = 0; u < 4; ++u)
+            if (l[u] < bl) {
+                bl = l[u];
+                best = d[u];
+            }
+    }
+    for (; m < k; ++m) {
+        const uint32_t d = mem[off + m];
+        const unsigned long long l = load_of(d);
+        if (l < bl) {
+            bl = l;
+            best = d;
+        }
+    }
+    return best;
+}
+
+// Copy a replica's member lists into shared memory when they fit (cap
+// entries); returns the array the decisions read.
+__device__ __forceinline__ const uint16_t *stage_members(const route_desc &rd, uint16_t *sm, unsigned long long cap)
+{
+    if (cap == 0 || rd.n_members == nullptr) return rd.members;
+    const unsigned long long nk = *rd.n_members;
+    if (nk > cap) return rd.members;
+    for (unsigned long long x = threadIdx.x; x < nk; x += blockDim.x) sm[x] = rd.members[x];
+    return sm;
+}
+
 // Sequential part: one CTA per load-dependent replica walks the batches.
-__device__ __forceinline__ uint32_t resolve(uint32_t c, const route_desc &rd, const unsigned long long *L)
+__device__ __forceinline__ uint32_t resolve(uint32_t c, const route_desc &rd, const uint16_t *mem,
+                                            const unsigned long long *L, unsigned long long cap, uint32_t *status)
 {
     const uint32_t kind = c & kKindMask;
     if (kind == kFixed) return c & 0xffffu;
@@ -115,18 +224,10 @@ __device__ __forceinline__ uint32_t resolve(uint32_t c, const route_desc &rd, co
         const uint32_t d1 = c & 0x1fffu, d2 = (c >> 13) & 0x1fffu;
         return L[d1] <= L[d2] ? d1 : d2;
     }
-    const cr_table_slot slot = rd.table[c & 0x3fffffffu];
-    uint32_t best = slot.m0;
-    unsigned long long bl = L[best];
-    for (uint32_t m = 1; m < slot.k; ++m) {
-        const uint32_t d = rd.members[slot.koff + m];
-        const unsigned long long l = L[d];
-        if (l < bl) {  // ties keep the earlier member
-            bl = l;
-            best = d;
-        }
-    }
-    return best;
+    auto load_of = [&](uint32_t d) { return L[d]; };
+    if (kind == kRing) return ring_walk(rd, c & kLow30, cap, load_of, status);
+    const cr_table_slot slot = rd.table[c & kLow30];
+    return set_min(mem, slot.koff, slot.k, slot.m0, load_of);
 }
 
 // Candidates are staged in shared memory a whole chunk (a multiple of the
@@ -135,16 +236,32 @@ __device__ __forceinline__ uint32_t resolve(uint32_t c, const route_desc &rd, co
 constexpr uint32_t kStage = 16384;
 constexpr int kStageRegs = kStage / kRouteBlock;  // 16
 
+// Sum of a replica's load vector on entry (the m of the bounded-load rule).
+__device__ __forceinline__ unsigned long long block_load_sum(const unsigned long long *L, uint32_t R)
+{
+    __shared__ unsigned long long s_tot;
+    if (threadIdx.x == 0) s_tot = 0;
+    __syncthreads();
+    unsigned long long t = 0;
+    for (uint32_t r = threadIdx.x; r < R; r += blockDim.x) t += L[r];
+    for (int o = 16; o > 0; o >>= 1) t += __shfl_xor_sync(0xffffffffu, t, o);
+    if ((threadIdx.x & 31) == 0 && t) atomicAdd(&s_tot, t);
+    __syncthreads();
+    return s_tot;
+}
+
 __global__ void __launch_bounds__(kRouteBlock) k_route_resolve(const __grid_constant__ route_args args,
                                                                const uint32_t *__restrict__ cand,
                                                                unsigned long long n, uint32_t B, uint32_t CH,
                                                                uint32_t R, unsigned long long *__restrict__ load,
-                                                               uint16_t *__restrict__ dest)
+                                                               uint16_t *__restrict__ dest, uint32_t *status,
+                                                               unsigned long long MC)
 {
     extern __shared__ unsigned long long sh[];
     unsigned long long *L = sh;                              // [R] live load
     uint32_t *delta = reinterpret_cast<uint32_t *>(sh + R);  // [R] this batch
     uint32_t *cbuf = delta + R;                              // [2][CH] staged candidates
+    uint16_t *smem_members = reinterpret_cast<uint16_t *>(cbuf + 2 * (size_t)CH);  // [MC]
     const uint32_t rep = args.dep[blockIdx.x];
     const route_desc rd = args.d[rep];
     unsigned long long *Lg = load + (unsigned long long)rep * R;
@@ -155,13 +272,15 @@ __global__ void __launch_bounds__(kRouteBlock) k_route_resolve(const __grid_cons
         L[r] = Lg[r];
         delta[r] = 0;
     }
+    const uint16_t *mem = stage_members(rd, smem_members, MC);
+    const unsigned long long tot0 = block_load_sum(L, R);  // also orders the copies above
     if (CH == 0) {
         // batches longer than the stage: candidates straight from global memory
-        __syncthreads();
         for (unsigned long long b0 = 0; b0 < n; b0 += B) {
             const unsigned long long b1 = (b0 + B < n) ? b0 + B : n;
+            const unsigned long long cap = chwbl_cap(tot0 + b0, R);
             for (unsigned long long i = b0 + tid; i < b1; i += blockDim.x) {
-                const uint32_t d = resolve(Cd[i], rd, L);
+                const uint32_t d = resolve(Cd[i], rd, mem, L, cap, status);
                 D[i] = (uint16_t)d;
                 atomicAdd(&delta[d], 1u);
             }
@@ -190,8 +309,9 @@ __global__ void __launch_bounds__(kRouteBlock) k_route_resolve(const __grid_cons
         const uint32_t *cb = cbuf + (size_t)cur * CH;
         for (unsigned long long b0 = c0; b0 < c1; b0 += B) {
             const unsigned long long b1 = (b0 + B < c1) ? b0 + B : c1;
+            const unsigned long long cap = chwbl_cap(tot0 + b0, R);
             for (unsigned long long i = b0 + tid; i < b1; i += blockDim.x) {
-                const uint32_t d = resolve(cb[i - c0], rd, L);
+                const uint32_t d = resolve(cb[i - c0], rd, mem, L, cap, status);
                 D[i] = (uint16_t)d;
                 atomicAdd(&delta[d], 1u);
             }
@@ -212,7 +332,256 @@ __global__ void __launch_bounds__(kRouteBlock) k_route_resolve(const __grid_cons
     for (uint32_t r = tid; r < R; r += blockDim.x) Lg[r] = L[r];
 }
 
+// ---- batches of at most one warp: one warp per replica ----------------------
+
+constexpr int kWarpChunk = 8;  // steps whose candidates are fetched one chunk ahead
+
+// A candidate with its table slot or first ring owner already fetched.
+struct prep_cand {
+    uint32_t kind;
+    uint32_t a;  // FIXED: destination; PAIR: d1; SET: first member; RING: owner of the first point
+    uint32_t b;  // PAIR: d2; SET: member offset; RING: first ring index
+    uint32_t k;  // SET: members
+};
+
+__device__ __forceinline__ prep_cand prepare(uint32_t c, const route_desc &rd)
+{
+    prep_cand p;
+    p.kind = c & kKindMask;
+    p.a = c & 0xffffu;
+    p.b = 0;
+    p.k = 1;
+    if (p.kind == kPair) {
+        p.a = c & 0x1fffu;
+        p.b = (c >> 13) & 0x1fffu;
+    } else if (p.kind == kSet) {
+        const cr_table_slot slot = rd.table[c & kLow30];
+        p.a = slot.m0;
+        p.b = slot.koff;
+        p.k = slot.k;
+    } else if (p.kind == kRing) {
+        p.b = c & kLow30;
+        p.a = rd.rowner[p.b];
+    }
+    return p;
+}
+
+// The decision of one request that sees load L[d] plus the lanes of `earlier`
+// currently placed on d.
+__device__ __forceinline__ uint32_t decide(const prep_cand &p, const route_desc &rd, const uint16_t *mem,
+                                           const unsigned long long *L, const uint32_t *mask, uint32_t earlier,
+                                           unsigned long long cap, uint32_t *status)
+{
+    auto seen = [&](uint32_t d) { return L[d] + (unsigned long long)__popc(mask[d] & earlier); };
+    if (p.kind == kFixed) return p.a;
+    if (p.kind == kPair) return seen(p.a) <= seen(p.b) ? p.a : p.b;
+    if (p.kind == kRing) return seen(p.a) < cap ? p.a : ring_walk(rd, p.b, cap, seen, status);
+    return set_min(mem, p.b, p.k, p.a, seen);
+}
+
+__global__ void __launch_bounds__(32) k_route_resolve_warp(const __grid_constant__ route_args args,
+                                                           const uint32_t *__restrict__ cand, unsigned long long n,
+                                                           uint32_t B, uint32_t R,
+                                                           unsigned long long *__restrict__ load,
+                                                           uint16_t *__restrict__ dest, uint32_t *status,
+                                                           unsigned long long MC)
+{
+    extern __shared__ unsigned long long sh[];
+    unsigned long long *L = sh;                             // [R] load at the start of the step
+    uint32_t *mask = reinterpret_cast<uint32_t *>(sh + R);  // [R] lanes of the step on each destination
+    uint16_t *smem_members = reinterpret_cast<uint16_t *>(mask + R);  // [MC]
+    const uint32_t rep = args.dep[blockIdx.x];
+    const route_desc &rd = args.d[rep];
+    unsigned long long *Lg = load + (unsigned long long)rep * R;
+    const uint32_t *Cd = cand + (unsigned long long)rep * n;
+    uint16_t *D = dest + (unsigned long long)rep * n;
+    const uint32_t lane = threadIdx.x;
+    unsigned long long tot = 0;
+    for (uint32_t r = lane; r < R; r += 32) {
+        const unsigned long long v = Lg[r];
+        L[r] = v;
+        mask[r] = 0;
+        tot += v;
+    }
+    for (int o = 16; o > 0; o >>= 1) tot += __shfl_xor_sync(0xffffffffu, tot, o);
+    const uint16_t *mem = stage_members(rd, smem_members, MC);
+    __syncwarp();
+    const uint32_t S = (32u / B) * B;               // requests per step: whole batches
+    const uint32_t bstart = (lane / B) * B;         // first lane of this lane's batch
+    const uint32_t earlier = (1u << bstart) - 1u;   // lanes of the earlier batches of the step
+    const uint32_t bit = 1u << lane;
+    const bool several = S > B;
+    const unsigned long long CHR = (unsigned long long)S * kWarpChunk;
+    uint32_t cn[kWarpChunk];
+#pragma unroll
+    for (int q = 0; q < kWarpChunk; ++q) {
+        const unsigned long long i = (unsigned long long)q * S + lane;
+        cn[q] = (lane < S && i < n) ? Cd[i] : 0u;  // 0 = FIXED 0: inactive lanes read nothing
+    }
+    for (unsigned long long c0 = 0; c0 < n; c0 += CHR) {
+        prep_cand p[kWarpChunk];
+#pragma unroll
+        for (int q = 0; q < kWarpChunk; ++q) p[q] = prepare(cn[q], rd);
+#pragma unroll
+        for (int q = 0; q < kWarpChunk; ++q) {
+            const unsigned long long i = c0 + CHR + (unsigned long long)q * S + lane;
+            cn[q] = (lane < S && i < n) ? Cd[i] : 0u;
+        }
+#pragma unroll
+        for (int q = 0; q < kWarpChunk; ++q) {
+            const unsigned long long s0 = c0 + (unsigned long long)q * S;
+            if (s0 >= n) break;  // uniform over the warp
+            const unsigned long long i = s0 + lane;
+            const bool active = lane < S && i < n;
+            const unsigned long long cap = chwbl_cap(tot + bstart, R);
+            uint32_t d = decide(p[q], rd, mem, L, mask, 0u, cap, status);
+            if (active) atomicOr(&mask[d], bit);
+            __syncwarp();
+            if (several) {
+                // fixed point: after iteration t the first t batches of the step are final
+                for (uint32_t it = 0;; ++it) {
+                    const uint32_t nd = active ? decide(p[q], rd, mem, L, mask, earlier, cap, status) : d;
+                    const uint32_t moved = __ballot_sync(0xffffffffu, nd != d);
+                    if (!moved) break;
+                    if (it >= S) {  // unreachable: S iterations always settle the step
+                        if (lane == 0) atomicOr(status, CR_FLAG_TIMEOUT);
+                        break;
+                    }
+                    if (nd != d) {
+                        atomicAnd(&mask[d], ~bit);
+                        atomicOr(&mask[nd], bit);
+                        d = nd;
+                    }
+                    __syncwarp();
+                }
+            }
+            if (active) {
+                const uint32_t mk = mask[d];
+                if ((mk & (0u - mk)) == bit) L[d] += (unsigned long long)__popc(mk);  // lowest lane adds
+                D[i] = (uint16_t)d;
+            }
+            __syncwarp();
+            if (active) mask[d] = 0;
+            __syncwarp();
+            const unsigned long long left = n - s0;
+            tot += left < S ? left : S;
+        }
+    }
+    for (uint32_t r = lane; r < R; r += 32) Lg[r] = L[r];
+}
+
+// ---- ring construction ------------------------------------------------------
+
+__global__ void __launch_bounds__(256) k_ring_points(unsigned long long seed, unsigned long long M,
+                                                     unsigned long long *__restrict__ pt)
+{
+    for (unsigned long long k = (unsigned long long)blockIdx.x * blockDim.x + threadIdx.x; k < M;
+         k += (unsigned long long)gridDim.x * blockDim.x)
+        pt[k] = cr_fmix64(seed + (k + 1ull) * CR_GAMMA);  // SplitMix64 output k
+}
+
+// Sorted points (stable: equal points keep ascending owner) -> point and owner arrays.
+__global__ void __launch_bounds__(256) k_ring_finish(const unsigned long long *__restrict__ ks,
+                                                     const uint32_t *__restrict__ pos, unsigned long long M,
+                                                     uint32_t V, unsigned long long *__restrict__ pt,
+                                                     uint16_t *__restrict__ ow)
+{
+    for (unsigned long long j = (unsigned long long)blockIdx.x * blockDim.x + threadIdx.x; j < M;
+         j += (unsigned long long)gridDim.x * blockDim.x) {
+        pt[j] = ks[j];
+        ow[j] = (uint16_t)(pos[j] / V);
+    }
+}
+
+// dir[t] = first ring index whose point is >= t << (64 - dbits) (M if none).
+__global__ void __launch_bounds__(256) k_ring_dir(const unsigned long long *__restrict__ pt, unsigned long long M,
+                                                  int dbits, uint32_t *__restrict__ dir)
+{
+    const unsigned long long nd = 1ull << dbits;
+    for (unsigned long long t = (unsigned long long)blockIdx.x * blockDim.x + threadIdx.x; t < nd;
+         t += (unsigned long long)gridDim.x * blockDim.x) {
+        const unsigned long long h = t << (64 - dbits);
+        unsigned long long lo = 0, hi = M;
+        while (lo < hi) {
+            const unsigned long long mid = (lo + hi) >> 1;
+            if (pt[mid] < h)
+                lo = mid + 1;
+            else
+                hi = mid;
+        }
+        dir[t] = (uint32_t)lo;
+    }
+}
+
 }  // namespace
+
+static int ring_fill(cr_ctx *ctx, cr_ring *g, uint64_t seed)
+{
+    const unsigned int gcap = (unsigned int)ctx->num_sms * 8u;
+    const unsigned long long M = g->M;
+    const unsigned long long *ks = nullptr;
+    const uint32_t *pos = nullptr;
+    CR_LAUNCH(ctx, k_ring_points, cr_blocks(M, 256, gcap), 256, 0, (unsigned long long)seed, M, g->d_point);
+    CR_TRY(cr_radix_sort_u64(ctx, g->d_point, nullptr, M, 64, &ks, &pos));
+    CR_LAUNCH(ctx, k_ring_finish, cr_blocks(M, 256, gcap), 256, 0, ks, pos, M, g->V, g->d_point, g->d_owner);
+    CR_LAUNCH(ctx, k_ring_dir, cr_blocks(1ull << g->dbits, 256, gcap), 256, 0, (const unsigned long long *)g->d_point,
+              M, (int)g->dbits, g->d_dir);
+    return CR_OK;
+}
+
+extern "C" int cr_ring_create(cr_ctx *ctx, uint32_t R, uint32_t vnodes, uint64_t seed, cr_ring **out)
+{
+    if (!ctx || !out) return CR_EINVAL;
+    *out = nullptr;
+    if (R == 0 || R > CR_MAX_R) return cr_fail(ctx, CR_EINVAL, "cr_ring_create: R=%u outside 1..%u", R, CR_MAX_R);
+    if (vnodes == 0 || vnodes > CR_MAX_VNODES)
+        return cr_fail(ctx, CR_EINVAL, "cr_ring_create: vnodes=%u outside 1..%u", vnodes, CR_MAX_VNODES);
+    const uint64_t M = (uint64_t)R * vnodes;
+    int dbits = 1;
+    while ((1ull << dbits) < M) ++dbits;
+    cr_ring *g = (cr_ring *)calloc(1, sizeof(cr_ring));
+    if (!g) return cr_fail(ctx, CR_ENOMEM, "cr_ring_create: host allocation failed");
+    g->R = R;
+    g->V = vnodes;
+    g->M = M;
+    g->dbits = (uint32_t)dbits;
+    if (cudaMalloc(&g->d_point, M * sizeof(unsigned long long)) != cudaSuccess ||
+        cudaMalloc(&g->d_owner, M * sizeof(uint16_t)) != cudaSuccess ||
+        cudaMalloc(&g->d_dir, (1ull << dbits) * sizeof(uint32_t)) != cudaSuccess) {
+        cudaGetLastError();
+        cr_ring_destroy(ctx, g);
+        return cr_fail(ctx, CR_ENOMEM, "cr_ring_create: device allocation of %llu points failed",
+                       (unsigned long long)M);
+    }
+    const int st = ring_fill(ctx, g, seed);
+    if (st != CR_OK) {
+        cr_ring_destroy(ctx, g);
+        return st;
+    }
+    *out = g;
+    return CR_OK;
+}
+
+extern "C" int cr_ring_destroy(cr_ctx *ctx, cr_ring *g)
+{
+    if (!g) return CR_OK;
+    if (ctx) cudaStreamSynchronize(ctx->stream);
+    if (g->d_point) cudaFree(g->d_point);
+    if (g->d_owner) cudaFree(g->d_owner);
+    if (g->d_dir) cudaFree(g->d_dir);
+    free(g);
+    return CR_OK;
+}
+
+extern "C" int cr_ring_export(cr_ctx *ctx, const cr_ring *g, uint64_t *point, uint16_t *owner)
+{
+    if (!ctx || !g) return CR_EINVAL;
+    if (point)
+        CR_CUDA(ctx, cudaMemcpyAsync(point, g->d_point, g->M * sizeof(uint64_t), cudaMemcpyDeviceToHost, ctx->stream));
+    if (owner)
+        CR_CUDA(ctx, cudaMemcpyAsync(owner, g->d_owner, g->M * sizeof(uint16_t), cudaMemcpyDeviceToHost, ctx->stream));
+    return cr_sync(ctx);
+}
 
 extern "C" int cr_route_batch(cr_ctx *ctx, const cr_plan *const *plans, const cr_replica *reps, uint32_t n_rep,
                               uint32_t R, const uint64_t *d_key, uint64_t n, uint64_t first_req_index,
@@ -227,14 +596,13 @@ extern "C" int cr_route_batch(cr_ctx *ctx, const cr_plan *const *plans, const cr
     if (!d_load) return cr_fail(ctx, CR_EINVAL, "cr_route_batch: d_load is NULL");
     if (n > 0 && (!d_key || !d_dest)) return cr_fail(ctx, CR_EINVAL, "cr_route_batch: NULL key or dest");
     route_args args;
+    memset(&args, 0, sizeof(args));
+    uint64_t mc = 0;  // largest member list of a plan replica
     for (uint32_t i = 0; i < n_rep; ++i) {
         route_desc &d = args.d[i];
         d.policy = reps[i].policy;
         d.seed = reps[i].seed;
-        d.tbits = 0;
-        d.table = nullptr;
-        d.members = nullptr;
-        if (reps[i].policy > CR_POLICY_HASH || reps[i].reserved != 0)
+        if (reps[i].policy > CR_POLICY_CHWBL || reps[i].reserved != 0)
             return cr_fail(ctx, CR_EINVAL, "cr_route_batch: replica %u has policy %u", i, reps[i].policy);
         if (reps[i].policy <= CR_POLICY_CR_NOREPL) {
             const cr_plan *p = plans ? plans[i] : nullptr;
@@ -244,15 +612,25 @@ extern "C" int cr_route_batch(cr_ctx *ctx, const cr_plan *const *plans, const cr
                 return cr_fail(ctx, CR_EINVAL, "cr_route_batch: replica %u plan has R=%u, call has R=%u", i, p->R, R);
             int bits = 0;
             while ((1ull << bits) < p->table_slots) ++bits;
+            if (bits > 30) return cr_fail(ctx, CR_EINVAL, "cr_route_batch: plan table too large");
             d.tbits = bits;
             d.table = p->d_table;
             d.members = p->d_members;
+            d.n_members = &p->d_info->sum_k;
+            mc = std::max<uint64_t>(mc, (uint64_t)p->R * p->W);  // sum of k_b <= C = R W
+        } else if (reps[i].policy == CR_POLICY_CHWBL) {
+            const cr_ring *g = reps[i].ring;
+            if (!g) return cr_fail(ctx, CR_EINVAL, "cr_route_batch: replica %u needs a ring", i);
+            if (g->R != R)
+                return cr_fail(ctx, CR_EINVAL, "cr_route_batch: replica %u ring has R=%u, call has R=%u", i, g->R, R);
+            d.rpoint = g->d_point;
+            d.rowner = g->d_owner;
+            d.rdir = g->d_dir;
+            d.rM = (uint32_t)g->M;
+            d.rdbits = (int32_t)g->dbits;
         }
     }
     if (n == 0) return CR_OK;
-    for (uint32_t i = 0; i < n_rep; ++i)
-        if (args.d[i].policy <= CR_POLICY_CR_NOREPL && args.d[i].tbits > 30)
-            return cr_fail(ctx, CR_EINVAL, "cr_route_batch: plan table too large");
     // replicas whose choices depend on the live load
     uint32_t n_dep = 0;
     for (uint32_t i = 0; i < n_rep; ++i)
@@ -274,15 +652,29 @@ extern "C" int cr_route_batch(cr_ctx *ctx, const cr_plan *const *plans, const cr
                   (unsigned long long)n, R, (unsigned long long *)d_load + (uint64_t)i * R);
         i = j;
     }
-    if (n_dep) {
-        // staging chunk: a whole number of batches, at most kStage requests
-        const uint32_t CH = batch_B <= kStage ? (kStage / batch_B) * batch_B : 0u;  // 0: no staging
-        size_t smem = (size_t)R * (sizeof(unsigned long long) + sizeof(uint32_t)) + 2ull * CH * sizeof(uint32_t);
+    if (!n_dep) return CR_OK;
+    // member lists go to shared memory when they fit beside the loads
+    auto with_members = [&](size_t base, uint64_t *MC) {
+        *MC = (mc && base + mc * sizeof(uint16_t) <= kSmemBudget) ? mc : 0;
+        return base + *MC * sizeof(uint16_t);
+    };
+    uint64_t MC;
+    if (batch_B <= 32) {
+        const size_t smem = with_members((size_t)R * (sizeof(unsigned long long) + sizeof(uint32_t)), &MC);
         if (smem > 48 * 1024)
-            CR_CUDA(ctx, cudaFuncSetAttribute(k_route_resolve, cudaFuncAttributeMaxDynamicSharedMemorySize,
+            CR_CUDA(ctx, cudaFuncSetAttribute(k_route_resolve_warp, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                               (int)smem));
-        CR_LAUNCH(ctx, k_route_resolve, n_dep, kRouteBlock, smem, args, (const uint32_t *)cand,
-                  (unsigned long long)n, batch_B, CH, R, (unsigned long long *)d_load, d_dest);
+        CR_LAUNCH(ctx, k_route_resolve_warp, n_dep, 32, smem, args, (const uint32_t *)cand, (unsigned long long)n,
+                  batch_B, R, (unsigned long long *)d_load, d_dest, ctx->d_status, (unsigned long long)MC);
+        return CR_OK;
     }
+    // staging chunk: a whole number of batches, at most kStage requests
+    const uint32_t CH = batch_B <= kStage ? (kStage / batch_B) * batch_B : 0u;  // 0: no staging
+    const size_t smem = with_members(
+        (size_t)R * (sizeof(unsigned long long) + sizeof(uint32_t)) + 2ull * CH * sizeof(uint32_t), &MC);
+    if (smem > 48 * 1024)
+        CR_CUDA(ctx, cudaFuncSetAttribute(k_route_resolve, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
+    CR_LAUNCH(ctx, k_route_resolve, n_dep, kRouteBlock, smem, args, (const uint32_t *)cand, (unsigned long long)n,
+              batch_B, CH, R, (unsigned long long *)d_load, d_dest, ctx->d_status, (unsigned long long)MC);
     return CR_OK;
 }

@@ -262,13 +262,18 @@ def test_plan_bad_params(P, ctx):
 
 # ------------------------------------------------------------------ a7 route ---
 @pytest.mark.parametrize("R,B", [(1, 1), (3, 1), (7, 33), (30, 1024), (64, 5000), (1024, 256), (30, 20000),
-                                 (5, 16384), (9, 16385)])
+                                 (5, 16384), (9, 16385), (1024, 1), (64, 2), (30, 3), (7, 31), (1024, 32),
+                                 (257, 5), (8192, 1), (8192, 7), (8192, 64)])
 def test_route_parity(P, ctx, R, B):
+    # batches of <= 32 requests take the one-warp-per-replica kernel, longer ones the CTA kernel
     rng = np.random.default_rng(R * 7 + B)
     keys = _rates_keys(rng, 3000, 40000)
     n = keys.size
-    pols = ["CR", "CR_NOLPT", "CR_NOREPL", "P2C", "RR", "HASH", "CR", "P2C"]
-    seeds = [0, 1, 0, 2, 3, 4, 9, 2**63 + 5]
+    pols = ["CR", "CR_NOLPT", "CR_NOREPL", "P2C", "RR", "HASH", "CR", "P2C", "CHWBL", "CHWBL"]
+    seeds = [0, 1, 0, 2, 3, 4, 9, 2**63 + 5, 11, 2**64 - 1]
+    ring_args = {8: (64, 5), 9: (1, 2**63 + 1)}  # replica -> (vnodes, ring seed)
+    orings = [O.Ring(R, *ring_args[i]) if i in ring_args else None for i in range(len(pols))]
+    drings = [P.Ring(ctx, R, *ring_args[i]) if i in ring_args else None for i in range(len(pols))]
     num, den = n, 6 * R            # tight: replicated keys
     W = 4
     oplans = {v: O.build_plan(keys, R, W, num, den, variant=v, seed=s, epoch=1)
@@ -279,9 +284,79 @@ def test_route_parity(P, ctx, R, B):
     vmap = {"CR": "LPT", "CR_NOLPT": "RANDOM", "CR_NOREPL": "NOREPL"}
     init = rng.integers(0, 50, size=(len(pols), R)).astype(np.uint64)
     ref_dest, ref_load = O.route([oplans.get(vmap.get(p)) for p in pols], pols, seeds, R, keys, 777, B,
-                                 load=init)
+                                 load=init, rings=orings)
     load = d_u64(init.reshape(-1)).view(len(pols), R).contiguous()
-    dest = P.route_batch(ctx, [dplans.get(vmap.get(p)) for p in pols], pols, seeds, R, d_u64(keys), 777, B, load)
+    dest = P.route_batch(ctx, [dplans.get(vmap.get(p)) for p in pols], pols, seeds, R, d_u64(keys), 777, B, load,
+                         rings=drings)
+    ctx.sync()
+    for i, p in enumerate(pols):
+        assert (h_u16(dest[i]) == ref_dest[i]).all(), (i, p)
+    assert (h_u64(load) == ref_load).all()
+
+
+@pytest.mark.parametrize("R,V,seed", [(1, 1, 0), (3, 1, 0), (7, 5, 123), (1024, 64, 9), (8192, 16, 2**64 - 1),
+                                      (5, 1024, 77)])
+def test_ring_parity(P, ctx, R, V, seed):
+    pt, ow = P.Ring(ctx, R, V, seed).export()
+    opt, oow = O.Ring(R, V, seed).export()
+    assert (pt == opt).all() and (ow == oow).all()
+
+
+def _inv_mix(z):
+    m64 = (1 << 64) - 1
+
+    def unxs(y, s):
+        x = y
+        for _ in range(64 // s + 1):
+            x = y ^ (x >> s)
+        return x & m64
+    z = unxs(z, 31)
+    z = (z * pow(0x94D049BB133111EB, -1, 1 << 64)) & m64
+    z = unxs(z, 27)
+    z = (z * pow(0xBF58476D1CE4E5B9, -1, 1 << 64)) & m64
+    return unxs(z, 30)
+
+
+@pytest.mark.parametrize("R,V,B", [(2, 1, 1), (13, 3, 1), (13, 3, 4), (600, 8, 1), (600, 8, 1000)])
+def test_route_chwbl_ring_edges(P, ctx, R, V, B):
+    # keys exactly on ring points, one past a point, past the last point (wrap), on a
+    # half-saturated fleet, so walks run past destinations at their bound
+    rng = np.random.default_rng(R + B)
+    rs, ks = 2**62 + R, 12345
+    opt, _ = O.Ring(R, V, rs).export()
+    edge = []
+    for p in [int(x) for x in opt[:4]] + [int(x) for x in opt[-4:]]:
+        edge += [_inv_mix(p) ^ ks, _inv_mix((p + 1) % 2**64) ^ ks]
+    edge += [_inv_mix(2**64 - 1) ^ ks, _inv_mix(0) ^ ks]
+    hot = rng.integers(0, 2**63, 8, dtype=np.int64).astype(np.uint64)
+    keys = np.concatenate([np.array(edge, np.uint64), hot[rng.integers(0, 8, 5000)],
+                           rng.integers(0, 2**63, 3000, dtype=np.int64).astype(np.uint64)])
+    rng.shuffle(keys)
+    init = np.zeros((1, R), np.uint64)
+    init[0, : R // 2] = rng.integers(0, 30, R // 2).astype(np.uint64) + np.uint64(keys.size // R)
+    ref_dest, ref_load = O.route([None], ["CHWBL"], [ks], R, keys, 5, B, load=init, rings=[O.Ring(R, V, rs)])
+    load = d_u64(init.reshape(-1)).view(1, R).contiguous()
+    dest = P.route_batch(ctx, [None], ["CHWBL"], [ks], R, d_u64(keys), 5, B, load, rings=[P.Ring(ctx, R, V, rs)])
+    ctx.sync()
+    assert (h_u16(dest) == ref_dest).all()
+    assert (h_u64(load) == ref_load).all()
+
+
+@pytest.mark.parametrize("B", [1, 2, 3, 16, 32])
+def test_route_small_batches_one_hot_key(P, ctx, B):
+    # every request carries the same replicated key: every lane of a warp step competes
+    # for the same members, the slowest case of the fixed-point resolution
+    R, W = 64, 2
+    keys = np.concatenate([np.full(20000, 0xDEADBEEF, np.uint64), np.arange(1, 2001, dtype=np.uint64)])
+    num, den = 1, 1  # q_cap = 1: k_b = min(R, lambda) -> all R destinations
+    opl = O.build_plan(keys, R, W, num, den)
+    dpl = P.build_plan(ctx, d_u64(keys), P.plan_params(R, W, num, den))
+    pols, seeds = ["CR", "P2C", "CHWBL"], [0, 1, 2]
+    ref_dest, ref_load = O.route([opl, None, None], pols, seeds, R, keys, 0, B,
+                                 rings=[None, None, O.Ring(R, 4, 3)])
+    load = torch.zeros((3, R), dtype=torch.int64, device=DEV)
+    dest = P.route_batch(ctx, [dpl, None, None], pols, seeds, R, d_u64(keys), 0, B, load,
+                         rings=[None, None, P.Ring(ctx, R, 4, 3)])
     ctx.sync()
     assert (h_u16(dest) == ref_dest).all()
     assert (h_u64(load) == ref_load).all()
@@ -296,6 +371,14 @@ def test_route_rejects_bad_args(P, ctx):
         P.route_batch(ctx, [None], ["P2C"], [0], 4, keys, 0, 0, load)       # B = 0
     with pytest.raises(P.CacheRouteError):
         P.route_batch(ctx, [None], ["P2C"], [0], 0, keys, 0, 4, load)       # R = 0
+    with pytest.raises(P.CacheRouteError):
+        P.route_batch(ctx, [None], ["CHWBL"], [0], 4, keys, 0, 1, load)     # ring missing
+    with pytest.raises(P.CacheRouteError):
+        P.route_batch(ctx, [None], ["CHWBL"], [0], 4, keys, 0, 1, load, rings=[P.Ring(ctx, 5, 2, 0)])  # R differs
+    with pytest.raises(P.CacheRouteError):
+        P.Ring(ctx, 4, 0, 0)                                                # no points
+    with pytest.raises(P.CacheRouteError):
+        P.Ring(ctx, 4, P.MAX_VNODES + 1, 0)
 
 
 # ------------------------------------------------------------------ a8, a9 ---
