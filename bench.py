@@ -41,6 +41,9 @@ def parse_args(argv=None):
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--config", default="70b")
     ap.add_argument("--batch", type=int, default=1024)
+    ap.add_argument("--policies", default="",
+                    help="comma-separated dispatch policies replacing the configuration's (same seeds), "
+                         "e.g. CR,P2C,RR,HASH,CHWBL")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-overlap", action="store_true", help="build plans in line instead of on a second stream")
@@ -51,6 +54,15 @@ def parse_args(argv=None):
     ap.add_argument("--intervals", type=int, default=0,
                     help="profiling aid: run only the first N intervals (the JSON line says so)")
     return ap.parse_args(argv)
+
+
+def with_policies(cfg, args):
+    """The configuration with --policies applied (unchanged without it)."""
+    if not getattr(args, "policies", ""):
+        return cfg
+    import dataclasses
+    pols = [p.strip() for p in args.policies.split(",") if p.strip()]
+    return dataclasses.replace(cfg, policies=pols, name=f"{cfg.name} [{','.join(pols)}]")
 
 
 def workload_config(cfg, B):
@@ -152,6 +164,7 @@ def oracle_sample(trace, n_intervals: int = 1, B: int = 1024):
     pols = [p for p, _ in reps]
     seeds = [s for _, s in reps]
     rp = O.Replay(len(reps), cfg.R, cfg.caps)
+    rings = OP.rings_for(cfg)
     prev = None
     busy = 0.0
     reqs = 0
@@ -161,7 +174,7 @@ def oracle_sample(trace, n_intervals: int = 1, B: int = 1024):
         t0 = time.perf_counter()
         keys = O.hash_prefixes(tok, off, iv.plen)
         per_rep, _ = OP.plans_for_interval(trace, keys if prev is None else prev, t)
-        dest, _ = O.route(per_rep, pols, seeds, cfg.R, keys, iv.g0, B)
+        dest, _ = O.route(per_rep, pols, seeds, cfg.R, keys, iv.g0, B, rings=rings)
         rp.step(keys, iv.plen, iv.slen, dest)
         busy += time.perf_counter() - t0
         reqs += iv.n
@@ -174,7 +187,7 @@ def run_reference(args):
     if rank != 0:
         return
     import tracegen as tg
-    cfg = tg.CONFIGS[args.config]
+    cfg = with_policies(tg.CONFIGS[args.config], args)
     trace = tg.Trace(cfg)
     import oracle as O
     import oracle.pipeline as OP
@@ -183,12 +196,13 @@ def run_reference(args):
     reps = cfg.replicas
     pols = [p for p, _ in reps]
     seeds = [s for _, s in reps]
+    rings = OP.rings_for(cfg)
 
     def step():
         rp = O.Replay(len(reps), cfg.R, cfg.caps)
         keys = O.hash_prefixes(tok, off, iv.plen)
         per_rep, _ = OP.plans_for_interval(trace, keys, 0)
-        dest, _ = O.route(per_rep, pols, seeds, cfg.R, keys, iv.g0, args.batch)
+        dest, _ = O.route(per_rep, pols, seeds, cfg.R, keys, iv.g0, args.batch, rings=rings)
         rp.step(keys, iv.plen, iv.slen, dest)
 
     for _ in range(args.warmup):
@@ -261,7 +275,7 @@ def main():
     import tracegen as tg
     from paper_2608_19677_gb300.pipeline import Pipeline
 
-    cfg = tg.CONFIGS[args.config]
+    cfg = with_policies(tg.CONFIGS[args.config], args)
     cfg = replica_cfg(cfg, rank, world)  # independent replica per rank
     trace = tg.Trace(cfg)
     dev = torch.device("cuda", local)
@@ -300,7 +314,7 @@ def main():
 
     ctx = P.Context(local, stream)
     pipe = Pipeline(ctx, cfg.R, cfg.W, cfg.caps, cfg.replicas, trace.qcap, batch_B=args.batch, max_n=max_n,
-                    overlap=not args.no_overlap)
+                    overlap=not args.no_overlap, vnodes=cfg.vnodes)
     marks = [[[torch.cuda.Event(enable_timing=True) for _ in range(5)] for _ in range(cfg.n_intervals)]
              for _ in range(max(args.steps, 1))]
 
@@ -453,7 +467,7 @@ def run_keys_mode(args, cfg, trace, dev, stream, world, rank, barrier):
     torch.cuda.empty_cache()  # the arenas are gone: only keys and lengths stay on the device
     n_step = sum(ns)
     pipe = Pipeline(ctx, cfg.R, cfg.W, cfg.caps, cfg.replicas, trace.qcap, batch_B=args.batch, max_n=max(ns),
-                    overlap=not args.no_overlap)
+                    overlap=not args.no_overlap, vnodes=cfg.vnodes)
     marks = [[[torch.cuda.Event(enable_timing=True) for _ in range(5)] for _ in range(cfg.n_intervals)]
              for _ in range(max(args.steps, 1))]
     plan_marks = [[] for _ in range(max(args.steps, 1))]

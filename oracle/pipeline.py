@@ -20,7 +20,7 @@ from typing import Iterable, Optional
 import numpy as np
 
 import tracegen as tg
-from . import Replay, build_plan, hash_prefixes, route
+from . import Replay, Ring, build_plan, hash_prefixes, route
 
 VARIANT_OF = {"CR": "LPT", "CR_NOLPT": "RANDOM", "CR_NOREPL": "NOREPL"}
 
@@ -43,6 +43,11 @@ def plans_for_interval(trace: tg.Trace, plan_keys: np.ndarray, t: int):
     return per_rep, built
 
 
+def rings_for(cfg):
+    """Ring of every bounded-load (CHWBL) replica, seeded by the replica's seed; None elsewhere."""
+    return [Ring(cfg.R, cfg.vnodes, seed) if pol == "CHWBL" else None for pol, seed in cfg.replicas]
+
+
 def run_trace(trace: tg.Trace, intervals: Optional[Iterable[int]] = None, align: int = 4,
               B: int = 1024, salt: int = 0, keep: bool = False, time_budget_s: Optional[float] = None):
     """Run the protocol; returns a dict with the counters (and per-interval data if keep)."""
@@ -51,6 +56,7 @@ def run_trace(trace: tg.Trace, intervals: Optional[Iterable[int]] = None, align:
     pols = [p for p, _ in reps]
     seeds = [s for _, s in reps]
     rp = Replay(len(reps), cfg.R, cfg.caps)
+    rings = rings_for(cfg)
     prev = None
     out = {"intervals": [], "keys": [], "plans": [], "dest": [], "load": [], "requests": 0}
     t_start = time.perf_counter()
@@ -59,7 +65,7 @@ def run_trace(trace: tg.Trace, intervals: Optional[Iterable[int]] = None, align:
         tok, off = tg.arena_host(trace, iv, align)
         keys = hash_prefixes(tok, off, iv.plen, salt)
         per_rep, built = plans_for_interval(trace, keys if prev is None else prev, t)
-        dest, load = route(per_rep, pols, seeds, cfg.R, keys, iv.g0, B)
+        dest, load = route(per_rep, pols, seeds, cfg.R, keys, iv.g0, B, rings=rings)
         rp.step(keys, iv.plen, iv.slen, dest)
         prev = keys
         out["intervals"].append(t)

@@ -7,7 +7,8 @@ One control interval t:
      request count, one plan per variant in use (LPT for CacheRoute, RANDOM
      seeded per replica for CacheRoute without LPT, NOREPL for single-copy
      CacheRoute), epoch = t;
-  3. cr_route_batch: every (policy, seed) replica, loads starting at zero;
+  3. cr_route_batch: every (policy, seed) replica, loads starting at zero
+     (bounded-load replicas use a ring built once, seeded by the replica);
   4. cr_shadow_replay: LRU simulators whose state and counters persist over
      intervals.
 
@@ -28,7 +29,7 @@ from __future__ import annotations
 
 from typing import Callable, List, Optional, Sequence, Tuple
 
-from . import (Context, Plan, Replay, build_plans, hash_prefixes, plan_params, route_batch,
+from . import (Context, Plan, Replay, Ring, build_plans, hash_prefixes, plan_params, route_batch,
                shadow_replay)
 
 VARIANT_OF = {"CR": "LPT", "CR_NOLPT": "RANDOM", "CR_NOREPL": "NOREPL"}
@@ -38,7 +39,8 @@ NKEYS = 3
 class Pipeline:
     def __init__(self, ctx: Context, R: int, W: int, caps: Sequence[int],
                  replicas: Sequence[Tuple[str, int]], qcap: Callable[[int], Tuple[int, int]],
-                 batch_B: int = 1024, salt: int = 0, max_n: int = 0, overlap: bool = False):
+                 batch_B: int = 1024, salt: int = 0, max_n: int = 0, overlap: bool = False,
+                 vnodes: int = 64):
         import torch
         self.ctx, self.R, self.W, self.caps = ctx, R, W, list(caps)
         self.replicas = list(replicas)
@@ -76,6 +78,8 @@ class Pipeline:
             self.hctx = self.pctx = self.yctx = ctx
         self.plans = [[Plan(self.pctx) for _ in self.plan_keys] for _ in range(2)]
         self.replay = Replay(ctx, len(self.replicas), R, self.caps)
+        # ring of every bounded-load replica, seeded by the replica's seed (built once)
+        self.rings = [Ring(ctx, R, vnodes, s) if p == "CHWBL" else None for p, s in self.replicas]
         self.ctr = torch.zeros((len(self.replicas), len(self.caps), R, 5), dtype=torch.int64, device=dev)
         self.load = torch.zeros((len(self.replicas), R), dtype=torch.int64, device=dev)
         self._dests = [None, None]   # destinations, double-buffered when the replay lags
@@ -227,7 +231,8 @@ class Pipeline:
         dest = D[:, :n] if n == D.shape[1] else D.view(-1)[:len(self.replicas) * n].view(len(self.replicas), n)
         plans = [self.plans[cur][i] if i is not None else None for i in self.rep_plan]
         r0 = self._event(self.mstream, True) if mark else None
-        route_batch(self.ctx, plans, self.policies, self.seeds, self.R, keys, g0, self.B, self.load, dest)
+        route_batch(self.ctx, plans, self.policies, self.seeds, self.R, keys, g0, self.B, self.load, dest,
+                    rings=self.rings)
         if mark:
             marks[3].record(self.mstream)
             self.route_marks.append((r0, marks[3]))

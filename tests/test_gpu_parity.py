@@ -458,3 +458,25 @@ def test_pipeline_parity(P, ctx, name, n, nint, overlap):
                 assert got["n_adm"] == opl.n_adm and (got["members"] == opl.members).all()
         pipe.sync()
         assert (h_u64(pipe.ctr) == ref["ctr"]).all()
+
+
+@pytest.mark.parametrize("B", [1, 7, 1024])
+def test_pipeline_parity_bounded_load_and_small_batches(P, ctx, B):
+    # the 70B shape with the bounded-load comparison policy added, routed in
+    # batches of 1 (exact sequential), 7 and 1024 requests
+    import dataclasses
+    from paper_2608_19677_gb300.pipeline import Pipeline
+    cfg = dataclasses.replace(tg.CONFIGS["70b"].scaled(20000, 2), policies=["CR", "P2C", "HASH", "CHWBL"],
+                              seeds=[0, 3])
+    tr = tg.Trace(cfg)
+    ref = OP.run_trace(tr, B=B, keep=True)
+    pipe = Pipeline(ctx, cfg.R, cfg.W, cfg.caps, cfg.replicas, tr.qcap, batch_B=B, overlap=True,
+                    vnodes=cfg.vnodes)
+    for t in range(cfg.n_intervals):
+        iv = tr.interval(t)
+        tok, off = tg.arena_host(tr, iv, 4)
+        pipe.interval(t, torch.from_numpy(tok).to(DEV), d_u64(off), d_u32(iv.plen), d_u32(iv.slen), iv.g0,
+                      plan_next=t + 1 < cfg.n_intervals)
+        assert (h_u16(pipe.last_dest) == ref["dest"][t]).all()
+    pipe.sync()
+    assert (h_u64(pipe.ctr) == ref["ctr"]).all()

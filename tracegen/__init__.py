@@ -73,6 +73,7 @@ class TraceConfig:
     whales: Optional[Sequence[int]] = None  # multipliers of injected whale keys
     whale_share: float = 0.25
     burst: Optional[Tuple[float, float, float]] = None  # (factor, burst_len_s, period_s)
+    vnodes: int = 64            # ring points per destination of bounded-load (CHWBL) replicas
 
     @property
     def replicas(self) -> List[Tuple[str, int]]:
