@@ -65,6 +65,14 @@ def with_policies(cfg, args):
     return dataclasses.replace(cfg, policies=pols, name=f"{cfg.name} [{','.join(pols)}]")
 
 
+def plan_stats(plan_ms):
+    """Median and max plan-build time per interval; empty when no replica uses a plan."""
+    if plan_ms.size == 0:
+        return {"median": None, "max": None, "builds_per_step": 0}
+    return {"median": float(np.median(plan_ms)), "max": float(plan_ms.max()),
+            "builds_per_step": int(plan_ms.shape[1])}
+
+
 def workload_config(cfg, B):
     return {
         "workload": (f"{cfg.name}: {cfg.R} destinations, {cfg.total_keys} keys Zipf s={cfg.zipf_s}"
@@ -404,11 +412,10 @@ def main():
         "stages_ms_per_step": {"hash": float(hash_ms.sum(1).mean()),
                                "main_wait_for_keys_and_plans": float(plan_wait_ms.sum(1).mean()),
                                "route": float(route_ms.sum(1).mean()), "replay": float(replay_ms.sum(1).mean())},
-        "plan_build_ms": {"median": float(np.median(plan_ms)), "max": float(plan_ms.max()),
-                          "builds_per_step": int(plan_ms.shape[1]),
-                          "per": "interval (histogram + admission + placement + table for all plan variants), "
-                                 + ("on its own stream, overlapped with hash/route/replay" if pipe.overlap
-                                    else "in line on the main stream")},
+        "plan_build_ms": dict(plan_stats(plan_ms),
+                              per="interval (histogram + admission + placement + table for all plan variants), "
+                                  + ("on its own stream, overlapped with hash/route/replay" if pipe.overlap
+                                     else "in line on the main stream")),
         "streams": ("hash (low priority) / planner (high priority) / route+replay: overlapped"
                     if pipe.overlap else "one stream"),
         "route_replay_requests_per_s": n_step / (rr_ms / 1e3),
@@ -554,8 +561,7 @@ def run_keys_mode(args, cfg, trace, dev, stream, world, rank, barrier):
                          "algorithmic_bytes_per_request": rr_bytes,
                          "achieved_GBps": rr_gbs, "hbm_frac": rr_gbs / hbm_peak},
         "hash_ms_per_pass": float(hms.sum()),
-        "plan_build_ms": {"median": float(np.median(plan_ms)), "max": float(plan_ms.max()),
-                          "builds_per_step": int(plan_ms.shape[1])},
+        "plan_build_ms": plan_stats(plan_ms),
         "main_wait_for_plans_ms_per_step": float((stage[:, :, 0] + stage[:, :, 1]).sum(1).mean()),
         "gpu_launches": int(n_launch), "clocks": clk,
     }

@@ -156,17 +156,17 @@ __global__ void __launch_bounds__(256) k_route_count(const uint16_t *__restrict_
 // unless the load sum has wrapped; then the first owner is taken and the
 // overflow flag raised.
 template <typename LoadOf>
-__device__ __forceinline__ uint32_t ring_walk(const route_desc &rd, uint32_t j, unsigned long long cap,
-                                              LoadOf load_of, uint32_t *status)
+__device__ __forceinline__ uint32_t ring_walk(const route_desc &rd, const uint16_t *own, uint32_t j,
+                                              unsigned long long cap, LoadOf load_of, uint32_t *status)
 {
     const uint32_t j0 = j;
     for (uint32_t t = 0; t < rd.rM; ++t) {
-        const uint32_t d = rd.rowner[j];
+        const uint32_t d = own[j];
         if (load_of(d) < cap) return d;
         j = (j + 1 == rd.rM) ? 0u : j + 1;
     }
     atomicOr(status, CR_FLAG_OVERFLOW);
-    return rd.rowner[j0];
+    return own[j0];
 }
 
 // Least-loaded member of T(b) = mem[off .. off + k), first member m0 given;
@@ -203,14 +203,16 @@ __device__ __forceinline__ uint32_t set_min(const uint16_t *mem, uint32_t off, u
     return best;
 }
 
-// Copy a replica's member lists into shared memory when they fit (cap
-// entries); returns the array the decisions read.
-__device__ __forceinline__ const uint16_t *stage_members(const route_desc &rd, uint16_t *sm, unsigned long long cap)
+// Copy a replica's u16 side array -- a plan's member lists, or a ring's
+// owners -- into shared memory when it fits (cap entries); returns the array
+// the decisions read.
+__device__ __forceinline__ const uint16_t *stage_aux(const route_desc &rd, uint16_t *sm, unsigned long long cap)
 {
-    if (cap == 0 || rd.n_members == nullptr) return rd.members;
-    const unsigned long long nk = *rd.n_members;
-    if (nk > cap) return rd.members;
-    for (unsigned long long x = threadIdx.x; x < nk; x += blockDim.x) sm[x] = rd.members[x];
+    const uint16_t *src = rd.policy == CR_POLICY_CHWBL ? rd.rowner : rd.members;
+    if (cap == 0 || src == nullptr) return src;
+    const unsigned long long nk = rd.policy == CR_POLICY_CHWBL ? rd.rM : (rd.n_members ? *rd.n_members : cap + 1);
+    if (nk > cap) return src;
+    for (unsigned long long x = threadIdx.x; x < nk; x += blockDim.x) sm[x] = src[x];
     return sm;
 }
 
@@ -225,7 +227,7 @@ __device__ __forceinline__ uint32_t resolve(uint32_t c, const route_desc &rd, co
         return L[d1] <= L[d2] ? d1 : d2;
     }
     auto load_of = [&](uint32_t d) { return L[d]; };
-    if (kind == kRing) return ring_walk(rd, c & kLow30, cap, load_of, status);
+    if (kind == kRing) return ring_walk(rd, mem, c & kLow30, cap, load_of, status);
     const cr_table_slot slot = rd.table[c & kLow30];
     return set_min(mem, slot.koff, slot.k, slot.m0, load_of);
 }
@@ -250,7 +252,7 @@ __device__ __forceinline__ unsigned long long block_load_sum(const unsigned long
     return s_tot;
 }
 
-__global__ void __launch_bounds__(kRouteBlock) k_route_resolve(const __grid_constant__ route_args args,
+__global__ void __launch_bounds__(kRouteBlock, 1) k_route_resolve(const __grid_constant__ route_args args,
                                                                const uint32_t *__restrict__ cand,
                                                                unsigned long long n, uint32_t B, uint32_t CH,
                                                                uint32_t R, unsigned long long *__restrict__ load,
@@ -261,7 +263,7 @@ __global__ void __launch_bounds__(kRouteBlock) k_route_resolve(const __grid_cons
     unsigned long long *L = sh;                              // [R] live load
     uint32_t *delta = reinterpret_cast<uint32_t *>(sh + R);  // [R] this batch
     uint32_t *cbuf = delta + R;                              // [2][CH] staged candidates
-    uint16_t *smem_members = reinterpret_cast<uint16_t *>(cbuf + 2 * (size_t)CH);  // [MC]
+    uint16_t *smem_aux = reinterpret_cast<uint16_t *>(cbuf + 2 * (size_t)CH);  // [MC] members or ring owners
     const uint32_t rep = args.dep[blockIdx.x];
     const route_desc rd = args.d[rep];
     unsigned long long *Lg = load + (unsigned long long)rep * R;
@@ -272,7 +274,7 @@ __global__ void __launch_bounds__(kRouteBlock) k_route_resolve(const __grid_cons
         L[r] = Lg[r];
         delta[r] = 0;
     }
-    const uint16_t *mem = stage_members(rd, smem_members, MC);
+    const uint16_t *mem = stage_aux(rd, smem_aux, MC);
     const unsigned long long tot0 = block_load_sum(L, R);  // also orders the copies above
     if (CH == 0) {
         // batches longer than the stage: candidates straight from global memory
@@ -344,7 +346,7 @@ struct prep_cand {
     uint32_t k;  // SET: members
 };
 
-__device__ __forceinline__ prep_cand prepare(uint32_t c, const route_desc &rd)
+__device__ __forceinline__ prep_cand prepare(uint32_t c, const route_desc &rd, const uint16_t *own)
 {
     prep_cand p;
     p.kind = c & kKindMask;
@@ -361,7 +363,7 @@ __device__ __forceinline__ prep_cand prepare(uint32_t c, const route_desc &rd)
         p.k = slot.k;
     } else if (p.kind == kRing) {
         p.b = c & kLow30;
-        p.a = rd.rowner[p.b];
+        p.a = own[p.b];
     }
     return p;
 }
@@ -375,7 +377,7 @@ __device__ __forceinline__ uint32_t decide(const prep_cand &p, const route_desc 
     auto seen = [&](uint32_t d) { return L[d] + (unsigned long long)__popc(mask[d] & earlier); };
     if (p.kind == kFixed) return p.a;
     if (p.kind == kPair) return seen(p.a) <= seen(p.b) ? p.a : p.b;
-    if (p.kind == kRing) return seen(p.a) < cap ? p.a : ring_walk(rd, p.b, cap, seen, status);
+    if (p.kind == kRing) return seen(p.a) < cap ? p.a : ring_walk(rd, mem, p.b, cap, seen, status);
     return set_min(mem, p.b, p.k, p.a, seen);
 }
 
@@ -387,9 +389,10 @@ __global__ void __launch_bounds__(32) k_route_resolve_warp(const __grid_constant
                                                            unsigned long long MC)
 {
     extern __shared__ unsigned long long sh[];
-    unsigned long long *L = sh;                             // [R] load at the start of the step
-    uint32_t *mask = reinterpret_cast<uint32_t *>(sh + R);  // [R] lanes of the step on each destination
-    uint16_t *smem_members = reinterpret_cast<uint16_t *>(mask + R);  // [MC]
+    prep_cand *ps = reinterpret_cast<prep_cand *>(sh);      // [kWarpChunk][32] prepared candidates
+    unsigned long long *L = sh + kWarpChunk * 32 * sizeof(prep_cand) / sizeof(unsigned long long);  // [R]
+    uint32_t *mask = reinterpret_cast<uint32_t *>(L + R);   // [R] lanes of the step on each destination
+    uint16_t *smem_aux = reinterpret_cast<uint16_t *>(mask + R);  // [MC] members or ring owners
     const uint32_t rep = args.dep[blockIdx.x];
     const route_desc &rd = args.d[rep];
     unsigned long long *Lg = load + (unsigned long long)rep * R;
@@ -404,13 +407,14 @@ __global__ void __launch_bounds__(32) k_route_resolve_warp(const __grid_constant
         tot += v;
     }
     for (int o = 16; o > 0; o >>= 1) tot += __shfl_xor_sync(0xffffffffu, tot, o);
-    const uint16_t *mem = stage_members(rd, smem_members, MC);
+    const uint16_t *mem = stage_aux(rd, smem_aux, MC);
     __syncwarp();
     const uint32_t S = (32u / B) * B;               // requests per step: whole batches
     const uint32_t bstart = (lane / B) * B;         // first lane of this lane's batch
     const uint32_t earlier = (1u << bstart) - 1u;   // lanes of the earlier batches of the step
     const uint32_t bit = 1u << lane;
     const bool several = S > B;
+    const bool ring = rd.policy == CR_POLICY_CHWBL;  // only its decisions read the cap
     const unsigned long long CHR = (unsigned long long)S * kWarpChunk;
     uint32_t cn[kWarpChunk];
 #pragma unroll
@@ -419,28 +423,29 @@ __global__ void __launch_bounds__(32) k_route_resolve_warp(const __grid_constant
         cn[q] = (lane < S && i < n) ? Cd[i] : 0u;  // 0 = FIXED 0: inactive lanes read nothing
     }
     for (unsigned long long c0 = 0; c0 < n; c0 += CHR) {
-        prep_cand p[kWarpChunk];
+        // each lane prepares (and later reads) only its own entries: no barrier needed
 #pragma unroll
-        for (int q = 0; q < kWarpChunk; ++q) p[q] = prepare(cn[q], rd);
+        for (int q = 0; q < kWarpChunk; ++q) ps[q * 32 + lane] = prepare(cn[q], rd, mem);
 #pragma unroll
         for (int q = 0; q < kWarpChunk; ++q) {
             const unsigned long long i = c0 + CHR + (unsigned long long)q * S + lane;
             cn[q] = (lane < S && i < n) ? Cd[i] : 0u;
         }
-#pragma unroll
+#pragma unroll 1
         for (int q = 0; q < kWarpChunk; ++q) {
             const unsigned long long s0 = c0 + (unsigned long long)q * S;
             if (s0 >= n) break;  // uniform over the warp
             const unsigned long long i = s0 + lane;
             const bool active = lane < S && i < n;
-            const unsigned long long cap = chwbl_cap(tot + bstart, R);
-            uint32_t d = decide(p[q], rd, mem, L, mask, 0u, cap, status);
+            const unsigned long long cap = ring ? chwbl_cap(tot + bstart, R) : 0ull;
+            const prep_cand pq = ps[q * 32 + lane];
+            uint32_t d = decide(pq, rd, mem, L, mask, 0u, cap, status);
             if (active) atomicOr(&mask[d], bit);
             __syncwarp();
             if (several) {
                 // fixed point: after iteration t the first t batches of the step are final
                 for (uint32_t it = 0;; ++it) {
-                    const uint32_t nd = active ? decide(p[q], rd, mem, L, mask, earlier, cap, status) : d;
+                    const uint32_t nd = active ? decide(pq, rd, mem, L, mask, earlier, cap, status) : d;
                     const uint32_t moved = __ballot_sync(0xffffffffu, nd != d);
                     if (!moved) break;
                     if (it >= S) {  // unreachable: S iterations always settle the step
@@ -597,7 +602,7 @@ extern "C" int cr_route_batch(cr_ctx *ctx, const cr_plan *const *plans, const cr
     if (n > 0 && (!d_key || !d_dest)) return cr_fail(ctx, CR_EINVAL, "cr_route_batch: NULL key or dest");
     route_args args;
     memset(&args, 0, sizeof(args));
-    uint64_t mc = 0;  // largest member list of a plan replica
+    uint64_t mc = 0;  // largest u16 side array: a plan's member lists or a ring's owners
     for (uint32_t i = 0; i < n_rep; ++i) {
         route_desc &d = args.d[i];
         d.policy = reps[i].policy;
@@ -628,6 +633,7 @@ extern "C" int cr_route_batch(cr_ctx *ctx, const cr_plan *const *plans, const cr
             d.rdir = g->d_dir;
             d.rM = (uint32_t)g->M;
             d.rdbits = (int32_t)g->dbits;
+            mc = std::max<uint64_t>(mc, g->M);
         }
     }
     if (n == 0) return CR_OK;
@@ -653,14 +659,15 @@ extern "C" int cr_route_batch(cr_ctx *ctx, const cr_plan *const *plans, const cr
         i = j;
     }
     if (!n_dep) return CR_OK;
-    // member lists go to shared memory when they fit beside the loads
+    // member lists and ring owners go to shared memory when they fit beside the loads
     auto with_members = [&](size_t base, uint64_t *MC) {
         *MC = (mc && base + mc * sizeof(uint16_t) <= kSmemBudget) ? mc : 0;
         return base + *MC * sizeof(uint16_t);
     };
     uint64_t MC;
     if (batch_B <= 32) {
-        const size_t smem = with_members((size_t)R * (sizeof(unsigned long long) + sizeof(uint32_t)), &MC);
+        const size_t smem = with_members(kWarpChunk * 32 * sizeof(prep_cand) +
+                                             (size_t)R * (sizeof(unsigned long long) + sizeof(uint32_t)), &MC);
         if (smem > 48 * 1024)
             CR_CUDA(ctx, cudaFuncSetAttribute(k_route_resolve_warp, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                               (int)smem));

@@ -59,3 +59,12 @@ def test_reference_arm_runs_on_rank_zero_only(monkeypatch, capsys):
     monkeypatch.setenv("RANK", "1")
     bench.run_reference(bench.parse_args(["--impl", "reference", "--steps", "1", "--warmup", "0"]))
     assert capsys.readouterr().out == ""                     # other ranks exit without work
+
+
+def test_plan_stats_without_plans():
+    # replica sets with no plan-based policy (e.g. --policies P2C) build no plans
+    import numpy as np
+    import bench
+    assert bench.plan_stats(np.zeros((3, 0))) == {"median": None, "max": None, "builds_per_step": 0}
+    st = bench.plan_stats(np.array([[1.0, 3.0], [2.0, 5.0]]))
+    assert st == {"median": 2.5, "max": 5.0, "builds_per_step": 2}
