@@ -15,6 +15,7 @@
  *   cr_build_plan     keys of one interval -> lambda_b, k_b, admission, LPT, table
  *   cr_route_batch    keys -> one destination per (request, replica)
  *   cr_ring_create    consistent-hashing ring of the bounded-load comparison policy
+ *   cr_plan_diff      cache and count churn between two plans (replanning under drift)
  *   cr_shadow_replay  routed requests -> per-destination LRU hits and load
  *
  * Conventions shared by every call:
@@ -205,6 +206,36 @@ CR_API int cr_plan_get_info(cr_ctx *ctx, const cr_plan *plan, cr_plan_info *out)
 CR_API int cr_plan_export(cr_ctx *ctx, const cr_plan *plan, uint64_t *ukey, uint64_t *ucnt,
                    uint64_t *adm_key, uint64_t *adm_cnt, uint32_t *adm_k, uint32_t *koff,
                    uint16_t *members, uint64_t *jobs, uint64_t *load);
+
+/* ==== f2: plan difference (replanning under drift) ===================== */
+
+/* Integer counts describing how plan b differs from plan a (supplement
+ * "Replanning Under Drift", replan table; sec. 5 "Rate drift and remapping").
+ * The assignment set of a plan is its set of (key, destination) pairs.
+ *   cache churn = 1 - pairs_common / (pairs_a + pairs_b - pairs_common)
+ *   count churn = hist_kb_changed / hist_keys
+ * Count churn is taken over every key of either plan's histogram with k_b
+ * from Eq. 1 of that plan's rate and q_cap (single-copy plans: 1); a key
+ * missing from one histogram has lambda = 0 there, so k_b = 1.  The adm_*
+ * counts restrict the comparison to admitted keys (k = 0 and an empty set for
+ * a key a plan did not admit). */
+typedef struct {
+    uint64_t keys_a, keys_b;       /* admitted keys of each plan */
+    uint64_t keys_common;          /* keys admitted by both */
+    uint64_t pairs_a, pairs_b;     /* (key, destination) pairs = sum of k_b over admitted keys */
+    uint64_t pairs_common;         /* pairs in both tables */
+    uint64_t adm_k_changed;        /* keys admitted by either plan whose k in T differs */
+    uint64_t adm_set_changed;      /* keys admitted by either plan whose destination set differs */
+    uint64_t hist_keys;            /* keys in either plan's histogram */
+    uint64_t hist_kb_changed;      /* of those, keys whose Eq. 1 k_b differs */
+} cr_plan_diff_counts;
+
+/* Blocking: compare two built plans with the same R (device kernels: one warp
+ * per admitted key, member sets compared through per-warp bitmaps of R bits;
+ * histograms through per-plan hash tables in context scratch, 32 bytes per
+ * request of the larger build); *out receives the counts.  Errors: CR_EINVAL
+ * (plan not built, R differs), CR_ENOMEM, CR_ECUDA. */
+CR_API int cr_plan_diff(cr_ctx *ctx, const cr_plan *a, const cr_plan *b, cr_plan_diff_counts *out);
 
 /* ==== a7: batched dispatch ========================================== */
 

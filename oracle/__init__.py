@@ -23,6 +23,13 @@ Parity status per function (what pins it; see tests/test_oracle_*.py):
   shadow_replay ........... hand trace, infinite-capacity closed form,
                             capacity-1 rule, brute-force stack distances
                             (Mattson inclusion).
+  Ring / route CHWBL ...... published SplitMix64 outputs, brute-force
+                            clockwise-distance walk, exact inverse-mixer edge
+                            keys, the sequential load bound, plain consistent
+                            hashing when unsaturated.
+  plan_diff / churn ....... hand-built plans, Jaccard of key x destination
+                            incidence matrices, identity and symmetry, the
+                            all-move / no-count-change case.
 """
 from __future__ import annotations
 
@@ -176,6 +183,11 @@ class Plan:
         self.adm_key, self.adm_cnt, self.adm_k = adm_key, adm_cnt, adm_k
         self.koff, self.members, self.jobs, self.load = koff, members, jobs, load
         self._keep = None
+        # set by build_plan: the interval's histogram and the plan's Eq. 1 inputs
+        self.hist_key = np.zeros(0, np.uint64)
+        self.hist_cnt = np.zeros(0, np.uint64)
+        self.qcap = (1, 1)
+        self.variant = "LPT"
 
     def table(self):
         """{key: [members...]} for every admitted key."""
@@ -226,9 +238,58 @@ def build_plan(keys, R: int, W: int, qcap_num: int, qcap_den: int, variant="LPT"
     if rc != 0:
         raise ValueError(f"orc_build_plan: status {rc}")
     na, sk = int(pl.n_adm), int(pl.sum_k)
-    return Plan(R, W, int(pl.U), na, sk, int(pl.cold), adm_key[:na].copy(), adm_cnt[:na].copy(),
-                adm_k[:na].copy(), koff[:na + 1].copy(), members[:sk].copy(), jobs[:sk].copy(),
-                load.copy())
+    out = Plan(R, W, int(pl.U), na, sk, int(pl.cold), adm_key[:na].copy(), adm_cnt[:na].copy(),
+               adm_k[:na].copy(), koff[:na + 1].copy(), members[:sk].copy(), jobs[:sk].copy(),
+               load.copy())
+    out.hist_key, out.hist_cnt = histogram(k)
+    out.qcap = (qcap_num, qcap_den)
+    out.variant = variant if isinstance(variant, str) else {v: s for s, v in VARIANT.items()}[variant]
+    return out
+
+
+# -- f2: replanning under drift ----------------------------------------------
+DIFF_FIELDS = ("keys_a", "keys_b", "keys_common", "pairs_a", "pairs_b", "pairs_common",
+               "adm_k_changed", "adm_set_changed", "hist_keys", "hist_kb_changed")
+
+
+def plan_kb(plan: Plan, lam: int) -> int:
+    """k_b of a key with lambda requests under the plan's q_cap (Eq. 1); 1 for single-copy plans."""
+    if plan.variant == "NOREPL":
+        return 1
+    return kb(lam, plan.qcap[0], plan.qcap[1], plan.R)
+
+
+def plan_diff(a: Plan, b: Plan) -> dict:
+    """Difference of two consecutive plans (supplement "Replanning Under Drift",
+    replan table).  The assignment set of a plan is its set of (key, destination)
+    pairs.  Count churn is over every key of either histogram, with k_b from Eq. 1
+    of each plan's own rate (a key absent from a histogram has lambda = 0, k_b = 1);
+    the adm_* counts compare admitted keys only (k = 0, empty set when not
+    admitted).  Returns integer counts; ``churn`` turns them into the two ratios."""
+    ta, tb = a.table(), b.table()
+    pa = {(key, d) for key, ms in ta.items() for d in ms}
+    pb = {(key, d) for key, ms in tb.items() for d in ms}
+    adm = set(ta) | set(tb)
+    ha = dict(zip(a.hist_key.tolist(), a.hist_cnt.tolist()))
+    hb = dict(zip(b.hist_key.tolist(), b.hist_cnt.tolist()))
+    hk = set(ha) | set(hb)
+    return dict(
+        keys_a=len(ta), keys_b=len(tb), keys_common=len(set(ta) & set(tb)),
+        pairs_a=len(pa), pairs_b=len(pb), pairs_common=len(pa & pb),
+        adm_k_changed=sum(1 for key in adm if len(ta.get(key, [])) != len(tb.get(key, []))),
+        adm_set_changed=sum(1 for key in adm if set(ta.get(key, [])) != set(tb.get(key, []))),
+        hist_keys=len(hk),
+        hist_kb_changed=sum(1 for key in hk if plan_kb(a, ha.get(key, 0)) != plan_kb(b, hb.get(key, 0))))
+
+
+def churn(diff: dict):
+    """(cache churn, count churn) as exact fractions: cache churn = 1 - Jaccard of the two
+    assignment sets; count churn = share of the keys of either histogram whose k_b changed."""
+    from fractions import Fraction
+    union_pairs = diff["pairs_a"] + diff["pairs_b"] - diff["pairs_common"]
+    cache = 1 - Fraction(diff["pairs_common"], union_pairs) if union_pairs else Fraction(0)
+    count = Fraction(diff["hist_kb_changed"], diff["hist_keys"]) if diff["hist_keys"] else Fraction(0)
+    return cache, count
 
 
 # -- a7 ----------------------------------------------------------------------

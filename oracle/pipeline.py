@@ -3,7 +3,9 @@
 One control interval t of a trace:
   1. hash every request's prefix span into its routing key;
   2. build the plan from the PREVIOUS interval's keys (interval 0, which has no
-     predecessor, plans from its own keys); q_cap = 1.25 x the mean
+     predecessor, plans from its own keys; with ``fresh`` every interval plans
+     from its own keys: the fresh plan of the stale-vs-fresh comparison in the
+     supplement "Replanning Under Drift"); q_cap = 1.25 x the mean
      destination load of the planning interval (or N/208 for the whale study);
      one plan per variant: LPT for CacheRoute, RANDOM (seeded) for CacheRoute
      without LPT, NOREPL for single-copy CacheRoute; epoch = t;
@@ -49,7 +51,8 @@ def rings_for(cfg):
 
 
 def run_trace(trace: tg.Trace, intervals: Optional[Iterable[int]] = None, align: int = 4,
-              B: int = 1024, salt: int = 0, keep: bool = False, time_budget_s: Optional[float] = None):
+              B: int = 1024, salt: int = 0, keep: bool = False, time_budget_s: Optional[float] = None,
+              fresh: bool = False):
     """Run the protocol; returns a dict with the counters (and per-interval data if keep)."""
     cfg = trace.cfg
     reps = cfg.replicas
@@ -64,7 +67,7 @@ def run_trace(trace: tg.Trace, intervals: Optional[Iterable[int]] = None, align:
         iv = trace.interval(t)
         tok, off = tg.arena_host(trace, iv, align)
         keys = hash_prefixes(tok, off, iv.plen, salt)
-        per_rep, built = plans_for_interval(trace, keys if prev is None else prev, t)
+        per_rep, built = plans_for_interval(trace, keys if (prev is None or fresh) else prev, t)
         dest, load = route(per_rep, pols, seeds, cfg.R, keys, iv.g0, B, rings=rings)
         rp.step(keys, iv.plen, iv.slen, dest)
         prev = keys

@@ -11,6 +11,7 @@ fails loudly otherwise.
   build_plans     one interval's keys -> plans (Eq. 1, Alg. 1)  (cr_build_plans)
   route_batch     keys -> destination per (request, replica)    (cr_route_batch)
   Ring            ring of the bounded-load policy               (cr_ring_create)
+  plan_diff       churn between two plans                       (cr_plan_diff)
   shadow_replay   routed requests -> LRU hit / load counters    (cr_shadow_replay)
 """
 from __future__ import annotations
@@ -36,7 +37,7 @@ EXPORTS = ("cr_create", "cr_destroy", "cr_set_stream", "cr_sync", "cr_last_error
            "cr_hash_prefixes", "cr_plan_create", "cr_plan_destroy", "cr_build_plans", "cr_build_plan",
            "cr_plan_get_info", "cr_plan_export", "cr_route_batch", "cr_replay_create", "cr_replay_reset",
            "cr_replay_destroy", "cr_shadow_replay", "cr_replay_export_state", "cr_key_histogram_noalloc",
-           "cr_ring_create", "cr_ring_destroy", "cr_ring_export")
+           "cr_ring_create", "cr_ring_destroy", "cr_ring_export", "cr_plan_diff")
 CR_NOALLOC_MAX_KEYS = 65536
 
 
@@ -55,6 +56,12 @@ class PlanParams(C.Structure):
 class PlanInfo(C.Structure):
     _fields_ = [("n", C.c_uint64), ("U", C.c_uint64), ("n_adm", C.c_uint64), ("sum_k", C.c_uint64),
                 ("cold", C.c_uint64), ("max_k", C.c_uint64), ("R", C.c_uint32), ("W", C.c_uint32)]
+
+
+class PlanDiff(C.Structure):
+    _fields_ = [(f, C.c_uint64) for f in ("keys_a", "keys_b", "keys_common", "pairs_a", "pairs_b",
+                                          "pairs_common", "adm_k_changed", "adm_set_changed", "hist_keys",
+                                          "hist_kb_changed")]
 
 
 class Replica(C.Structure):
@@ -104,6 +111,7 @@ def lib() -> C.CDLL:
         "cr_ring_create": ([vp, u32, u32, u64, C.POINTER(vp)], i32),
         "cr_ring_destroy": ([vp, vp], i32),
         "cr_ring_export": ([vp, vp, vp, vp], i32),
+        "cr_plan_diff": ([vp, vp, vp, C.POINTER(PlanDiff)], i32),
     }
     for name, (args, res) in sig.items():
         f = getattr(L, name)
@@ -256,6 +264,21 @@ def build_plan(ctx: Context, keys, params: PlanParams, plan: Optional[Plan] = No
     plan = plan or Plan(ctx)
     build_plans(ctx, keys, [params], [plan])
     return plan
+
+
+def plan_diff(ctx: Context, a: Plan, b: Plan) -> dict:
+    """Counts of how plan b differs from plan a (blocking); see ``churn``."""
+    out = PlanDiff()
+    ctx.check(lib().cr_plan_diff(ctx.handle, a.handle, b.handle, C.byref(out)), "cr_plan_diff")
+    return {f: int(getattr(out, f)) for f, _ in PlanDiff._fields_}
+
+
+def churn(diff: dict):
+    """(cache churn, count churn) as floats: 1 - Jaccard of the assignment sets, and the share of
+    the keys of either histogram whose Eq. 1 k_b changed."""
+    up = diff["pairs_a"] + diff["pairs_b"] - diff["pairs_common"]
+    return (1.0 - diff["pairs_common"] / up if up else 0.0,
+            diff["hist_kb_changed"] / diff["hist_keys"] if diff["hist_keys"] else 0.0)
 
 
 class Ring:

@@ -29,6 +29,7 @@ enum cr_scratch_slot {
     SCR_REPLAY_REC,    // gathered (key, prefix, suffix) records in stream order
     SCR_REPLAY_CHUNK,  // per-stream chunk counts -> offsets, and their total
     SCR_ROUTE_DESC,    // per-replica route descriptors
+    SCR_DIFF,          // plan-difference counters
     SCR_NUM
 };
 
@@ -72,6 +73,8 @@ struct cr_plan {
     unsigned long long *d_jobs, *d_load;
     cr_table_slot *d_table;
     cr_plan_info_dev *d_info;
+    uint64_t qnum, qden;             // q_cap = qnum / qden of the last build
+    uint32_t variant;                // CR_VARIANT_* of the last build
     int built;
 };
 

@@ -1380,6 +1380,9 @@ extern "C" int cr_build_plans(cr_ctx *ctx, const uint64_t *d_key, uint64_t n, co
     for (uint32_t j = 0; j < n_plans; ++j) {
         CR_TRY(plan_reserve(ctx, plans[j], n, params[j].R, params[j].W));
         plans[j]->n = n;
+        plans[j]->qnum = params[j].qcap_num;
+        plans[j]->qden = params[j].qcap_den;
+        plans[j]->variant = params[j].variant;
         plans[j]->built = 1;
         if (j == 0 || n == 0 || n > kPlanSortOneCta)  // small intervals: the admission CTA writes every field
             CR_LAUNCH(ctx, k_plan_reset, 1, 1, 0, plans[j]->d_info, (unsigned long long)n);

@@ -3,7 +3,9 @@
 One control interval t:
   1. cr_hash_prefixes: routing key of every request;
   2. cr_build_plans: plans from the PREVIOUS interval's keys (the first
-     interval plans from its own keys), q_cap from the planning interval's
+     interval plans from its own keys; with ``fresh`` every interval plans
+     from its own keys, as in the paper's stale-vs-fresh replanning
+     comparison), q_cap from the planning interval's
      request count, one plan per variant in use (LPT for CacheRoute, RANDOM
      seeded per replica for CacheRoute without LPT, NOREPL for single-copy
      CacheRoute), epoch = t;
@@ -40,11 +42,12 @@ class Pipeline:
     def __init__(self, ctx: Context, R: int, W: int, caps: Sequence[int],
                  replicas: Sequence[Tuple[str, int]], qcap: Callable[[int], Tuple[int, int]],
                  batch_B: int = 1024, salt: int = 0, max_n: int = 0, overlap: bool = False,
-                 vnodes: int = 64):
+                 vnodes: int = 64, fresh: bool = False):
         import torch
         self.ctx, self.R, self.W, self.caps = ctx, R, W, list(caps)
         self.replicas = list(replicas)
         self.qcap, self.B, self.salt = qcap, batch_B, salt
+        self.fresh = fresh  # plans from each interval's own keys instead of the previous interval's
         self.policies = [p for p, _ in self.replicas]
         self.seeds = [s for _, s in self.replicas]
         dev = torch.device("cuda", ctx.device)
@@ -197,7 +200,11 @@ class Pipeline:
         # ---- plans ----------------------------------------------------------------
         cur = self._pbuf
         plan_reader = None
-        if self.plan_keys:
+        if self.plan_keys and self.fresh:
+            # a freshly computed plan: this interval's own keys (replanning study)
+            plan_reader = self._build(cur, keys, t, hashed, mark)
+            self._next_built = False
+        elif self.plan_keys:
             if not self._next_built:
                 # nothing planned ahead: plan this interval from the previous keys (or its own)
                 if self.prev_keys is None:

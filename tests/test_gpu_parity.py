@@ -480,3 +480,75 @@ def test_pipeline_parity_bounded_load_and_small_batches(P, ctx, B):
         assert (h_u16(pipe.last_dest) == ref["dest"][t]).all()
     pipe.sync()
     assert (h_u64(pipe.ctr) == ref["ctr"]).all()
+
+
+# ------------------------------------------------------------------ f2 replanning ---
+def _diff_case(P, ctx, keys_a, keys_b, R, W, num_den_a, num_den_b, var_a="LPT", var_b="LPT"):
+    oa = O.build_plan(keys_a, R, W, *num_den_a, variant=var_a, seed=1, epoch=0)
+    ob = O.build_plan(keys_b, R, W, *num_den_b, variant=var_b, seed=2, epoch=1)
+    da = P.build_plan(ctx, d_u64(keys_a), P.plan_params(R, W, *num_den_a, var_a, seed=1, epoch=0))
+    db = P.build_plan(ctx, d_u64(keys_b), P.plan_params(R, W, *num_den_b, var_b, seed=2, epoch=1))
+    got = P.plan_diff(ctx, da, db)
+    want = O.plan_diff(oa, ob)
+    assert got == want
+    assert P.plan_diff(ctx, db, da) == O.plan_diff(ob, oa)
+    assert P.plan_diff(ctx, da, da) == O.plan_diff(oa, oa)
+    return got
+
+
+@pytest.mark.parametrize("t", range(5))
+def test_plan_diff_drift_transitions(P, ctx, t):
+    # consecutive fresh LPT plans of the drift trace (70B shape, lognormal rate walk)
+    cfg = tg.CONFIGS["drift"]
+    tr = tg.Trace(cfg)
+    ka = O.hash_prefixes(*tg.arena_host(tr, tr.interval(t), 4), tr.interval(t).plen)
+    kb = O.hash_prefixes(*tg.arena_host(tr, tr.interval(t + 1), 4), tr.interval(t + 1).plen)
+    d = _diff_case(P, ctx, ka, kb, cfg.R, cfg.W, tr.qcap(ka.size), tr.qcap(kb.size))
+    cache, count = O.churn(d)
+    assert 0 < cache <= 1 and 0 <= count < 1
+
+
+@pytest.mark.parametrize("R,W,spread", [(1, 4, 50), (7, 3, 400), (64, 8, 3000), (1024, 16, 20000),
+                                        (8192, 2, 30000)])
+def test_plan_diff_shapes(P, ctx, R, W, spread):
+    rng = np.random.default_rng(R)
+    ka = _rates_keys(rng, spread, 60000)
+    kb = np.concatenate([ka[: ka.size // 2], _rates_keys(rng, spread, 30000)])  # half the traffic changes
+    n = ka.size
+    _diff_case(P, ctx, ka, kb, R, W, (n, 4 * R), (n, 3 * R), "LPT", "RANDOM")  # replicated keys, k_b up to R
+
+
+def test_plan_diff_empty_and_errors(P, ctx):
+    keys = np.arange(1, 500, dtype=np.uint64) * np.uint64(7919)
+    e = np.zeros(0, np.uint64)
+    _diff_case(P, ctx, e, keys, 16, 4, (1, 1), (keys.size, 64))
+    _diff_case(P, ctx, e, e, 16, 4, (1, 1), (1, 1))
+    a = P.build_plan(ctx, d_u64(keys), P.plan_params(16, 4, keys.size, 64))
+    b = P.build_plan(ctx, d_u64(keys), P.plan_params(17, 4, keys.size, 64))
+    with pytest.raises(P.CacheRouteError):
+        P.plan_diff(ctx, a, b)                                              # R differs
+    with pytest.raises(P.CacheRouteError):
+        P.plan_diff(ctx, a, P.Plan(ctx))                                    # not built
+
+
+@pytest.mark.parametrize("fresh", [True, False])
+def test_pipeline_parity_drift_fresh_and_stale(P, ctx, fresh):
+    # the replanning comparison: every interval routed with a plan from its own keys
+    # (fresh) or from the previous interval's (stale), replayed through persistent LRUs
+    from paper_2608_19677_gb300.pipeline import Pipeline
+    cfg = tg.CONFIGS["drift"].scaled(60000, 6)
+    tr = tg.Trace(cfg)
+    ref = OP.run_trace(tr, B=1024, keep=True, fresh=fresh)
+    pipe = Pipeline(ctx, cfg.R, cfg.W, cfg.caps, cfg.replicas, tr.qcap, batch_B=1024, overlap=True, fresh=fresh)
+    for t in range(cfg.n_intervals):
+        iv = tr.interval(t)
+        tok, off = tg.arena_host(tr, iv, 4)
+        pipe.interval(t, torch.from_numpy(tok).to(DEV), d_u64(off), d_u32(iv.plen), d_u32(iv.slen), iv.g0,
+                      plan_next=t + 1 < cfg.n_intervals)
+        assert (h_u16(pipe.last_dest) == ref["dest"][t]).all()
+        for (v, s), pl in zip(pipe.plan_keys, pipe.last_plans):
+            got = pl.export()
+            opl = ref["plans"][t][(v, s)]
+            assert got["n_adm"] == opl.n_adm and (got["members"] == opl.members).all()
+    pipe.sync()
+    assert (h_u64(pipe.ctr) == ref["ctr"]).all()

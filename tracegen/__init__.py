@@ -10,7 +10,10 @@ exactly the arrays produced here.
 Workload shapes follow the paper's description of its traffic (section 2.1 and
 the workload table in the supplement: skewed per-key rates, a stable per-key
 context that recurs, Poisson or bursty arrivals) at the sizes of the five
-synthetic configurations listed in ``CONFIGS``.  The paper's de-identified
+synthetic configurations listed in ``CONFIGS``, plus a drift configuration
+for the replanning study (sec. 5 "Rate drift and remapping", supplement
+"Replanning Under Drift": the 70B-shaped key rates evolve for six intervals by
+a lognormal random walk with sigma = 0.3 per step).  The paper's de-identified
 telemetry is not available; these seeded traces stand in for it.
 
 Token values come from a counter-based integer map (``token_values``) over
@@ -31,7 +34,7 @@ VOCAB = 128256
 M31 = (1 << 31) - 1
 
 # Policy names (the numeric ids are fixed by the library's public header).
-POLICY_IDS = {"CR": 0, "CR_NOLPT": 1, "CR_NOREPL": 2, "P2C": 3, "RR": 4, "HASH": 5}
+POLICY_IDS = {"CR": 0, "CR_NOLPT": 1, "CR_NOREPL": 2, "P2C": 3, "RR": 4, "HASH": 5, "CHWBL": 6}
 SIX_POLICIES = ["CR", "CR_NOLPT", "CR_NOREPL", "P2C", "RR", "HASH"]
 
 
@@ -74,6 +77,7 @@ class TraceConfig:
     whale_share: float = 0.25
     burst: Optional[Tuple[float, float, float]] = None  # (factor, burst_len_s, period_s)
     vnodes: int = 64            # ring points per destination of bounded-load (CHWBL) replicas
+    drift: Optional[float] = None  # sigma of a per-interval lognormal random walk of every key's rate
 
     @property
     def replicas(self) -> List[Tuple[str, int]]:
@@ -108,6 +112,10 @@ CONFIGS: Dict[str, TraceConfig] = {
         name="burst", R=64, n_keys=100_000, zipf_s=0.9, n_requests=16_000_000, n_intervals=120,
         interval_s=5.0, plen=("lognormal", 4096, 0.5, 32768), W=128, caps=[128],
         policies=SIX_POLICIES, seeds=[0, 1, 2, 3, 4], burst=(5.0, 2.0, 30.0)),
+    "drift": TraceConfig(
+        name="drift", R=30, n_keys=20_000, zipf_s=1.0, n_requests=1_000_000, n_intervals=6,
+        interval_s=10.0, plen=("lognormal", 2048, 0.5, 16384), W=12, caps=[12],
+        policies=["CR", "P2C"], seeds=[0, 1, 2, 3, 4], hot_cap=1.0 / 30, drift=0.3),
     "large": TraceConfig(
         name="large", R=1024, n_keys=1_000_000, zipf_s=0.8, n_requests=64_000_000,
         n_intervals=60, interval_s=10.0, plen=("lognormal", 2048, 0.5, 32768), W=256,
@@ -159,6 +167,7 @@ class Trace:
         self.g0 = np.concatenate([[0], np.cumsum(self.counts)[:-1]]).astype(np.int64)
         self._cdf = np.cumsum(self.key_p)
         self._cdf[-1] = 1.0
+        self._drift_cdf = {}
 
     # -- key popularity -------------------------------------------------
     def _key_shares(self) -> np.ndarray:
@@ -204,12 +213,35 @@ class Trace:
         per_int = int(round(c.interval_s))
         return per_sec.reshape(c.n_intervals, per_int).sum(axis=1).astype(np.int64)
 
+    # -- rate drift ---------------------------------------------------------
+    def shares(self, t: int) -> np.ndarray:
+        """Key shares of interval t.  With drift sigma, every key's log-rate takes an
+        independent N(0, sigma^2) step per interval from the primary shares (interval 0),
+        and the shares are renormalised (lognormal random walk of the rates)."""
+        c = self.cfg
+        if not c.drift or t == 0:
+            return self.key_p
+        walk = np.zeros(c.total_keys)
+        for s in range(1, t + 1):
+            walk += c.drift * _rng(c.trace_seed, 0x44524654, s).standard_normal(c.total_keys)  # "DRFT"
+        p = self.key_p * np.exp(walk)
+        return p / p.sum()
+
+    def _cdf_at(self, t: int) -> np.ndarray:
+        if not self.cfg.drift or t == 0:
+            return self._cdf
+        if t not in self._drift_cdf:
+            cdf = np.cumsum(self.shares(t))
+            cdf[-1] = 1.0
+            self._drift_cdf[t] = cdf
+        return self._drift_cdf[t]
+
     def interval(self, t: int) -> Interval:
         c = self.cfg
         n = int(self.counts[t])
         rng = _rng(c.trace_seed, 0x4B455953, t)  # "KEYS"
         u = rng.random(n)
-        kid = np.searchsorted(self._cdf, u, side="right").astype(np.int64)
+        kid = np.searchsorted(self._cdf_at(t), u, side="right").astype(np.int64)
         np.minimum(kid, c.total_keys - 1, out=kid)
         plen = self.key_plen[kid]
         slen = np.full(n, c.suffix, dtype=np.uint32)
