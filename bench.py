@@ -41,6 +41,9 @@ def parse_args(argv=None):
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--config", default="70b")
     ap.add_argument("--batch", type=int, default=1024)
+    ap.add_argument("--fresh-plans", action="store_true",
+                    help="plan every interval from its own keys (the fresh plan of the replanning study) "
+                         "instead of from the previous interval's")
     ap.add_argument("--policies", default="",
                     help="comma-separated dispatch policies replacing the configuration's (same seeds), "
                          "e.g. CR,P2C,RR,HASH,CHWBL")
@@ -73,7 +76,7 @@ def plan_stats(plan_ms):
             "builds_per_step": int(plan_ms.shape[1])}
 
 
-def workload_config(cfg, B):
+def workload_config(cfg, B, fresh=False):
     return {
         "workload": (f"{cfg.name}: {cfg.R} destinations, {cfg.total_keys} keys Zipf s={cfg.zipf_s}"
                      f"{' (hottest capped)' if cfg.hot_cap else ''}, {cfg.n_requests} requests over "
@@ -87,6 +90,8 @@ def workload_config(cfg, B):
         "lru_caps": cfg.caps,
         "slots_per_destination": cfg.W,
         "batch_B": B,
+        "plans_from": "each interval's own keys (fresh)" if fresh else "the previous interval's keys",
+        "rate_drift_sigma": cfg.drift,
         "trace_seed": cfg.trace_seed,
         "l2": "inputs larger than L2 (token arenas of all intervals resident in HBM)",
     }
@@ -225,7 +230,7 @@ def run_reference(args):
     line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": dt * 1e3, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "u64", "data": "synthetic",
-            "config": workload_config(cfg, args.batch),
+            "config": workload_config(cfg, args.batch, args.fresh_plans),
             "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "kind": "oracle", "sample": sample},
             "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     print(json.dumps(line), flush=True)
@@ -322,7 +327,7 @@ def main():
 
     ctx = P.Context(local, stream)
     pipe = Pipeline(ctx, cfg.R, cfg.W, cfg.caps, cfg.replicas, trace.qcap, batch_B=args.batch, max_n=max_n,
-                    overlap=not args.no_overlap, vnodes=cfg.vnodes)
+                    overlap=not args.no_overlap, vnodes=cfg.vnodes, fresh=args.fresh_plans)
     marks = [[[torch.cuda.Event(enable_timing=True) for _ in range(5)] for _ in range(cfg.n_intervals)]
              for _ in range(max(args.steps, 1))]
 
@@ -407,7 +412,7 @@ def main():
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": ms_max, "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "u64", "data": "synthetic",
-        "config": workload_config(cfg, args.batch),
+        "config": workload_config(cfg, args.batch, args.fresh_plans),
         "roofline": roofline,
         "stages_ms_per_step": {"hash": float(hash_ms.sum(1).mean()),
                                "main_wait_for_keys_and_plans": float(plan_wait_ms.sum(1).mean()),
@@ -425,6 +430,9 @@ def main():
         "clocks": clk,
     }
 
+    # ---- replanning under drift (untimed study) ----------------------------
+    if cfg.drift:
+        line["replan"] = replan_study(args, ctx, cfg, trace, inputs, dev, stream, max_n)
     # ---- end to end through the public API with pinned host buffers -------
     if not args.no_e2e:
         line["e2e"] = e2e(args, ctx, pipe, inputs, dev, stream, n_step, world)
@@ -439,6 +447,71 @@ def main():
         print(json.dumps(line), flush=True)
     if world > 1:
         dist.destroy_process_group()
+
+
+def replan_study(args, ctx, cfg, trace, inputs, dev, stream, max_n):
+    """Replanning under drift, after the timed region (supplement "Replanning Under Drift"):
+    cache and count churn between the fresh LPT plans of consecutive intervals (cr_plan_diff,
+    timed with CUDA events), and per-interval LRU hit rates when every interval is routed with a
+    stale plan (previous interval's keys) or a fresh one (its own keys)."""
+    import torch
+    import paper_2608_19677_gb300 as P
+    from paper_2608_19677_gb300.pipeline import Pipeline
+    keys = []
+    for (t, tok, off, plen, slen, g0, n) in inputs:
+        k = torch.empty(n, dtype=torch.int64, device=dev)
+        P.hash_prefixes(ctx, tok, off, plen, 0, out=k)
+        keys.append(k)
+    plans = []
+    for t, k in enumerate(keys):
+        num, den = trace.qcap(int(k.shape[0]))
+        plans.append(P.build_plan(ctx, k, P.plan_params(cfg.R, cfg.W, num, den, "LPT", epoch=t)))
+    ctx.sync()
+    transitions, diff_ms = [], []
+    for t in range(len(plans) - 1):
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        d = P.plan_diff(ctx, plans[t], plans[t + 1])  # blocking
+        e1.record(stream)
+        e1.synchronize()
+        diff_ms.append(e0.elapsed_time(e1))
+        cache, count = P.churn(d)
+        transitions.append(dict(transition=f"{t}->{t + 1}", cache_churn=cache, count_churn=count, **d))
+    pols = sorted(set(cfg.policies), key=cfg.policies.index)
+    rows = {p: [i for i, (q, _) in enumerate(cfg.replicas) if q == p] for p in pols}
+
+    def hit_rates(fresh):
+        pipe = Pipeline(ctx, cfg.R, cfg.W, cfg.caps, cfg.replicas, trace.qcap, batch_B=args.batch, max_n=max_n,
+                        overlap=not args.no_overlap, vnodes=cfg.vnodes, fresh=fresh)
+        pipe.reset()
+        prev = torch.zeros_like(pipe.ctr)
+        out = {p: [] for p in pols}
+        for i, (t, tok, off, plen, slen, g0, n) in enumerate(inputs):
+            pipe.interval(t, None, off, plen, slen, g0, plan_next=i + 1 < len(inputs), keys=keys[i])
+            pipe.finish()
+            pipe.sync()
+            cur = pipe.ctr.clone()
+            dt = (cur - prev)[:, 0]  # first LRU capacity
+            prev = cur
+            for p in pols:
+                req = int(dt[rows[p], :, 0].sum())
+                out[p].append(int(dt[rows[p], :, 1].sum()) / req if req else 0.0)
+        return out
+
+    stale, fresh = hit_rates(False), hit_rates(True)
+    return {
+        "sigma": cfg.drift,
+        "transitions": transitions,
+        "plan_diff_ms": {"median": float(np.median(diff_ms)), "max": float(np.max(diff_ms)),
+                         "per": "cr_plan_diff call (blocking: kernels + counter read-back)"},
+        "hit_rate_per_interval": {"stale_plan": stale, "fresh_plan": fresh,
+                                  "lru_capacity": cfg.caps[0]},
+        "kv_loss_points_of_stale": {p: [100.0 * (fresh[p][t] - stale[p][t]) for t in range(1, len(inputs))]
+                                    for p in pols},
+        "note": "fresh = plan from the interval's own keys; stale = plan from the previous interval's keys "
+                "(the pipeline's default); LRU state carries over intervals, so a fresh plan's hit rate "
+                "includes its rewarming misses",
+    }
 
 
 def run_keys_mode(args, cfg, trace, dev, stream, world, rank, barrier):
@@ -474,7 +547,7 @@ def run_keys_mode(args, cfg, trace, dev, stream, world, rank, barrier):
     torch.cuda.empty_cache()  # the arenas are gone: only keys and lengths stay on the device
     n_step = sum(ns)
     pipe = Pipeline(ctx, cfg.R, cfg.W, cfg.caps, cfg.replicas, trace.qcap, batch_B=args.batch, max_n=max(ns),
-                    overlap=not args.no_overlap, vnodes=cfg.vnodes)
+                    overlap=not args.no_overlap, vnodes=cfg.vnodes, fresh=args.fresh_plans)
     marks = [[[torch.cuda.Event(enable_timing=True) for _ in range(5)] for _ in range(cfg.n_intervals)]
              for _ in range(max(args.steps, 1))]
     plan_marks = [[] for _ in range(max(args.steps, 1))]
@@ -546,7 +619,7 @@ def run_keys_mode(args, cfg, trace, dev, stream, world, rank, barrier):
         "metric": METRIC, "value": job_throughput(n_step, world, ms_max), "unit": UNIT, "n_gpus": world,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_max, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "u64", "data": "synthetic",
-        "config": dict(workload_config(cfg, args.batch),
+        "config": dict(workload_config(cfg, args.batch, args.fresh_plans),
                        step="plans + route + replay over resident keys (the token arenas of all intervals do "
                             "not fit in HBM: each interval's arena was generated and hashed one at a time, each "
                             "hash launch timed alone)",
