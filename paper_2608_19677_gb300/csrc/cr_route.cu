@@ -36,19 +36,27 @@ constexpr int kRouteBlock = 1024;
 constexpr uint32_t kEmpty = 0xffffffffu;
 constexpr size_t kSmemBudget = 200 * 1024;  // dynamic shared memory a resolve CTA may take
 
+// 48 bytes: a replica uses either a plan (CACHEROUTE-type) or a ring (CHWBL).
 struct route_desc {
     uint32_t policy;
     int32_t tbits;                    // log2 table slots (plan policies)
     unsigned long long seed;
-    const cr_table_slot *table;
-    const uint16_t *members;
-    const unsigned long long *n_members;  // device: the plan's sum of k_b
-    const unsigned long long *rpoint; // ring (CHWBL)
-    const uint16_t *rowner;
-    const uint32_t *rdir;
+    union {
+        const cr_table_slot *table;      // plan
+        const unsigned long long *rpoint;  // ring points
+    };
+    union {
+        const uint16_t *members;         // plan: member lists
+        const uint16_t *rowner;          // ring: owner of each point
+    };
+    union {
+        const unsigned long long *n_members;  // plan, device: the sum of k_b
+        const uint32_t *rdir;                 // ring: start directory
+    };
     uint32_t rM;                      // ring points
     int32_t rdbits;                   // log2 directory entries
 };
+static_assert(sizeof(route_desc) == 48, "route_desc layout");
 
 struct route_args {
     route_desc d[CR_MAX_REPLICAS];
@@ -217,17 +225,23 @@ __device__ __forceinline__ const uint16_t *stage_aux(const route_desc &rd, uint1
 }
 
 // Sequential part: one CTA per load-dependent replica walks the batches.
+// One decision against the batch-start loads.  A bounded-load replica's
+// candidates are all RING; every other replica's are FIXED, PAIR or SET, so
+// the two cases are compiled apart.  m: requests in the load vector the batch
+// sees (the bounded-load rule's m).
+template <bool RING>
 __device__ __forceinline__ uint32_t resolve(uint32_t c, const route_desc &rd, const uint16_t *mem,
-                                            const unsigned long long *L, unsigned long long cap, uint32_t *status)
+                                            const unsigned long long *L, unsigned long long m, uint32_t R,
+                                            uint32_t *status)
 {
+    auto load_of = [&](uint32_t d) { return L[d]; };
+    if (RING) return ring_walk(rd, mem, c & kLow30, chwbl_cap(m, R), load_of, status);
     const uint32_t kind = c & kKindMask;
     if (kind == kFixed) return c & 0xffffu;
     if (kind == kPair) {
         const uint32_t d1 = c & 0x1fffu, d2 = (c >> 13) & 0x1fffu;
         return L[d1] <= L[d2] ? d1 : d2;
     }
-    auto load_of = [&](uint32_t d) { return L[d]; };
-    if (kind == kRing) return ring_walk(rd, mem, c & kLow30, cap, load_of, status);
     const cr_table_slot slot = rd.table[c & kLow30];
     return set_min(mem, slot.koff, slot.k, slot.m0, load_of);
 }
@@ -252,37 +266,20 @@ __device__ __forceinline__ unsigned long long block_load_sum(const unsigned long
     return s_tot;
 }
 
-__global__ void __launch_bounds__(kRouteBlock, 1) k_route_resolve(const __grid_constant__ route_args args,
-                                                               const uint32_t *__restrict__ cand,
-                                                               unsigned long long n, uint32_t B, uint32_t CH,
-                                                               uint32_t R, unsigned long long *__restrict__ load,
-                                                               uint16_t *__restrict__ dest, uint32_t *status,
-                                                               unsigned long long MC)
+// The batch loop of one replica (L already holds its loads; ends with a barrier).
+template <bool RING>
+__device__ __forceinline__ void resolve_batches(const route_desc &rd, const uint16_t *mem, unsigned long long *L,
+                                                uint32_t *delta, uint32_t *cbuf, const uint32_t *__restrict__ Cd,
+                                                uint16_t *__restrict__ D, unsigned long long n, uint32_t B,
+                                                uint32_t CH, uint32_t R, unsigned long long tot0, uint32_t *status)
 {
-    extern __shared__ unsigned long long sh[];
-    unsigned long long *L = sh;                              // [R] live load
-    uint32_t *delta = reinterpret_cast<uint32_t *>(sh + R);  // [R] this batch
-    uint32_t *cbuf = delta + R;                              // [2][CH] staged candidates
-    uint16_t *smem_aux = reinterpret_cast<uint16_t *>(cbuf + 2 * (size_t)CH);  // [MC] members or ring owners
-    const uint32_t rep = args.dep[blockIdx.x];
-    const route_desc rd = args.d[rep];
-    unsigned long long *Lg = load + (unsigned long long)rep * R;
-    const uint32_t *Cd = cand + (unsigned long long)rep * n;
-    uint16_t *D = dest + (unsigned long long)rep * n;
     const uint32_t tid = threadIdx.x;
-    for (uint32_t r = tid; r < R; r += blockDim.x) {
-        L[r] = Lg[r];
-        delta[r] = 0;
-    }
-    const uint16_t *mem = stage_aux(rd, smem_aux, MC);
-    const unsigned long long tot0 = block_load_sum(L, R);  // also orders the copies above
     if (CH == 0) {
         // batches longer than the stage: candidates straight from global memory
         for (unsigned long long b0 = 0; b0 < n; b0 += B) {
             const unsigned long long b1 = (b0 + B < n) ? b0 + B : n;
-            const unsigned long long cap = chwbl_cap(tot0 + b0, R);
             for (unsigned long long i = b0 + tid; i < b1; i += blockDim.x) {
-                const uint32_t d = resolve(Cd[i], rd, mem, L, cap, status);
+                const uint32_t d = resolve<RING>(Cd[i], rd, mem, L, tot0 + b0, R, status);
                 D[i] = (uint16_t)d;
                 atomicAdd(&delta[d], 1u);
             }
@@ -293,7 +290,6 @@ __global__ void __launch_bounds__(kRouteBlock, 1) k_route_resolve(const __grid_c
             }
             __syncthreads();
         }
-        for (uint32_t r = tid; r < R; r += blockDim.x) Lg[r] = L[r];
         return;
     }
     for (uint32_t x = tid; x < CH && x < n; x += blockDim.x) cbuf[x] = Cd[x];
@@ -311,9 +307,8 @@ __global__ void __launch_bounds__(kRouteBlock, 1) k_route_resolve(const __grid_c
         const uint32_t *cb = cbuf + (size_t)cur * CH;
         for (unsigned long long b0 = c0; b0 < c1; b0 += B) {
             const unsigned long long b1 = (b0 + B < c1) ? b0 + B : c1;
-            const unsigned long long cap = chwbl_cap(tot0 + b0, R);
             for (unsigned long long i = b0 + tid; i < b1; i += blockDim.x) {
-                const uint32_t d = resolve(cb[i - c0], rd, mem, L, cap, status);
+                const uint32_t d = resolve<RING>(cb[i - c0], rd, mem, L, tot0 + b0, R, status);
                 D[i] = (uint16_t)d;
                 atomicAdd(&delta[d], 1u);
             }
@@ -331,7 +326,38 @@ __global__ void __launch_bounds__(kRouteBlock, 1) k_route_resolve(const __grid_c
         __syncthreads();
         cur ^= 1;
     }
-    for (uint32_t r = tid; r < R; r += blockDim.x) Lg[r] = L[r];
+}
+
+__global__ void __launch_bounds__(kRouteBlock) k_route_resolve(const __grid_constant__ route_args args,
+                                                               const uint32_t *__restrict__ cand,
+                                                               unsigned long long n, uint32_t B, uint32_t CH,
+                                                               uint32_t R, unsigned long long *__restrict__ load,
+                                                               uint16_t *__restrict__ dest, uint32_t *status,
+                                                               unsigned long long MC)
+{
+    extern __shared__ unsigned long long sh[];
+    unsigned long long *L = sh;                              // [R] live load
+    uint32_t *delta = reinterpret_cast<uint32_t *>(sh + R);  // [R] this batch
+    uint32_t *cbuf = delta + R;                              // [2][CH] staged candidates
+    uint16_t *smem_aux = reinterpret_cast<uint16_t *>(cbuf + 2 * (size_t)CH);  // [MC] members or ring owners
+    const uint32_t rep = args.dep[blockIdx.x];
+    const route_desc rd = args.d[rep];
+    unsigned long long *Lg = load + (unsigned long long)rep * R;
+    const uint32_t *Cd = cand + (unsigned long long)rep * n;
+    uint16_t *D = dest + (unsigned long long)rep * n;
+    for (uint32_t r = threadIdx.x; r < R; r += blockDim.x) {
+        L[r] = Lg[r];
+        delta[r] = 0;
+    }
+    const uint16_t *mem = stage_aux(rd, smem_aux, MC);
+    if (rd.policy == CR_POLICY_CHWBL) {  // uniform over the block
+        const unsigned long long tot0 = block_load_sum(L, R);
+        resolve_batches<true>(rd, mem, L, delta, cbuf, Cd, D, n, B, CH, R, tot0, status);
+    } else {
+        __syncthreads();  // orders the copies above
+        resolve_batches<false>(rd, mem, L, delta, cbuf, Cd, D, n, B, CH, R, 0ull, status);
+    }
+    for (uint32_t r = threadIdx.x; r < R; r += blockDim.x) Lg[r] = L[r];
 }
 
 // ---- batches of at most one warp: one warp per replica ----------------------
