@@ -44,6 +44,8 @@ def parse_args(argv=None):
     ap.add_argument("--fresh-plans", action="store_true",
                     help="plan every interval from its own keys (the fresh plan of the replanning study) "
                          "instead of from the previous interval's")
+    ap.add_argument("--token-lru", action="store_true",
+                    help="replay with token-weighted LRU capacities (byte-aware variant)")
     ap.add_argument("--policies", default="",
                     help="comma-separated dispatch policies replacing the configuration's (same seeds), "
                          "e.g. CR,P2C,RR,HASH,CHWBL")
@@ -60,7 +62,9 @@ def parse_args(argv=None):
 
 
 def with_policies(cfg, args):
-    """The configuration with --policies applied (unchanged without it)."""
+    """The configuration with --policies and --token-lru applied (unchanged without them)."""
+    if getattr(args, "token_lru", False):
+        cfg = cfg.token_lru()
     if not getattr(args, "policies", ""):
         return cfg
     import dataclasses
@@ -88,6 +92,7 @@ def workload_config(cfg, B, fresh=False):
         "replicas": len(cfg.replicas),
         "policies": cfg.policies,
         "lru_caps": cfg.caps,
+        "lru_capacity_unit": "prefix tokens" if cfg.lru_tokens else "prefixes",
         "slots_per_destination": cfg.W,
         "batch_B": B,
         "plans_from": "each interval's own keys (fresh)" if fresh else "the previous interval's keys",
@@ -176,7 +181,7 @@ def oracle_sample(trace, n_intervals: int = 1, B: int = 1024):
     reps = cfg.replicas
     pols = [p for p, _ in reps]
     seeds = [s for _, s in reps]
-    rp = O.Replay(len(reps), cfg.R, cfg.caps)
+    rp = O.Replay(len(reps), cfg.R, cfg.caps, tokens=cfg.lru_tokens)
     rings = OP.rings_for(cfg)
     prev = None
     busy = 0.0
@@ -212,7 +217,7 @@ def run_reference(args):
     rings = OP.rings_for(cfg)
 
     def step():
-        rp = O.Replay(len(reps), cfg.R, cfg.caps)
+        rp = O.Replay(len(reps), cfg.R, cfg.caps, tokens=cfg.lru_tokens)
         keys = O.hash_prefixes(tok, off, iv.plen)
         per_rep, _ = OP.plans_for_interval(trace, keys, 0)
         dest, _ = O.route(per_rep, pols, seeds, cfg.R, keys, iv.g0, args.batch, rings=rings)
@@ -327,7 +332,8 @@ def main():
 
     ctx = P.Context(local, stream)
     pipe = Pipeline(ctx, cfg.R, cfg.W, cfg.caps, cfg.replicas, trace.qcap, batch_B=args.batch, max_n=max_n,
-                    overlap=not args.no_overlap, vnodes=cfg.vnodes, fresh=args.fresh_plans)
+                    overlap=not args.no_overlap, vnodes=cfg.vnodes, fresh=args.fresh_plans,
+                    lru_tokens=cfg.lru_tokens)
     marks = [[[torch.cuda.Event(enable_timing=True) for _ in range(5)] for _ in range(cfg.n_intervals)]
              for _ in range(max(args.steps, 1))]
 
@@ -482,7 +488,8 @@ def replan_study(args, ctx, cfg, trace, inputs, dev, stream, max_n):
 
     def hit_rates(fresh):
         pipe = Pipeline(ctx, cfg.R, cfg.W, cfg.caps, cfg.replicas, trace.qcap, batch_B=args.batch, max_n=max_n,
-                        overlap=not args.no_overlap, vnodes=cfg.vnodes, fresh=fresh)
+                        overlap=not args.no_overlap, vnodes=cfg.vnodes, fresh=fresh,
+                        lru_tokens=cfg.lru_tokens)
         pipe.reset()
         prev = torch.zeros_like(pipe.ctr)
         out = {p: [] for p in pols}
@@ -547,7 +554,8 @@ def run_keys_mode(args, cfg, trace, dev, stream, world, rank, barrier):
     torch.cuda.empty_cache()  # the arenas are gone: only keys and lengths stay on the device
     n_step = sum(ns)
     pipe = Pipeline(ctx, cfg.R, cfg.W, cfg.caps, cfg.replicas, trace.qcap, batch_B=args.batch, max_n=max(ns),
-                    overlap=not args.no_overlap, vnodes=cfg.vnodes, fresh=args.fresh_plans)
+                    overlap=not args.no_overlap, vnodes=cfg.vnodes, fresh=args.fresh_plans,
+                    lru_tokens=cfg.lru_tokens)
     marks = [[[torch.cuda.Event(enable_timing=True) for _ in range(5)] for _ in range(cfg.n_intervals)]
              for _ in range(max(args.steps, 1))]
     plan_marks = [[] for _ in range(max(args.steps, 1))]

@@ -311,6 +311,21 @@ CR_API int cr_route_batch(cr_ctx *ctx, const cr_plan *const *plans, const cr_rep
  * Every simulator starts empty.  Errors: CR_EINVAL, CR_ENOMEM. */
 CR_API int cr_replay_create(cr_ctx *ctx, uint32_t n_rep, uint32_t R, const uint32_t *caps,
                      uint32_t n_caps, cr_replay **out);
+/* Byte-aware variant (token-weighted capacity; the paper's byte budgets of
+ * sec. 3.1 and 6, and the 70B configuration's 24k-token slot budget read as
+ * tokens): every simulator holds whole prefixes, most recent first, while their
+ * prefix tokens sum to at most its capacity (token_caps[], 1 .. 2^32-1) and
+ * there are at most CR_MAX_CAP of them; an access moves or inserts its key at
+ * the front, then the least recent prefixes are evicted until both limits
+ * hold.  A key must have the same prefix length at every access (the longest
+ * recent run of prefixes that fits is then what every capacity holds, and one
+ * list decides all capacities); a key that comes back with another length
+ * makes the next blocking call return CR_EINVAL, and the counters of that call
+ * are not meaningful.  cr_shadow_replay, cr_replay_reset, cr_replay_destroy
+ * and cr_replay_export_state work on it unchanged.  Errors: CR_EINVAL,
+ * CR_ENOMEM. */
+CR_API int cr_replay_create_tokens(cr_ctx *ctx, uint32_t n_rep, uint32_t R, const uint32_t *token_caps,
+                                   uint32_t n_caps, cr_replay **out);
 /* Empty every simulator (enqueued on the stream). */
 CR_API int cr_replay_reset(cr_ctx *ctx, cr_replay *rp);
 /* Destroy (waits for the stream).  NULL is accepted. */

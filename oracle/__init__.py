@@ -90,6 +90,8 @@ def lib():
         _lib.orc_ring_export.argtypes = [C.c_void_p, u64p, u16p]
         _lib.orc_replay_create.restype = C.c_void_p
         _lib.orc_replay_create.argtypes = [C.c_uint32, C.c_uint32, u32p, C.c_uint32]
+        _lib.orc_replay_create_tokens.restype = C.c_void_p
+        _lib.orc_replay_create_tokens.argtypes = [C.c_uint32, C.c_uint32, u32p, C.c_uint32]
         _lib.orc_replay_free.argtypes = [C.c_void_p]
         _lib.orc_shadow_replay.restype = C.c_int
         _lib.orc_shadow_replay.argtypes = [C.c_void_p, u64p, u32p, u32p, u16p, C.c_uint64, u64p]
@@ -342,13 +344,18 @@ def route(plans: Sequence[Optional[Plan]], policies: Sequence, seeds: Sequence[i
 
 
 # -- a8, a9 --------------------------------------------------------------------
-class Replay:
-    """Whole-prefix LRU per (replica, capacity, destination); state persists across calls."""
+TOKEN_LRU_MAX_ENTRIES = 1024
 
-    def __init__(self, n_rep: int, R: int, caps: Sequence[int]):
-        self.n_rep, self.R, self.caps = n_rep, R, list(caps)
+
+class Replay:
+    """Whole-prefix LRU per (replica, capacity, destination); state persists across calls.
+    With ``tokens`` the capacities count prefix tokens (byte-aware variant) instead of prefixes."""
+
+    def __init__(self, n_rep: int, R: int, caps: Sequence[int], tokens: bool = False):
+        self.n_rep, self.R, self.caps, self.tokens = n_rep, R, list(caps), tokens
         cp = _c(caps, np.uint32)
-        self._h = lib().orc_replay_create(n_rep, R, _p(cp, C.c_uint32), len(caps))
+        make = lib().orc_replay_create_tokens if tokens else lib().orc_replay_create
+        self._h = make(n_rep, R, _p(cp, C.c_uint32), len(caps))
         if not self._h:
             raise ValueError("orc_replay_create: invalid arguments")
         self.ctr = np.zeros((n_rep, len(caps), R, 5), np.uint64)
@@ -374,6 +381,6 @@ class Replay:
         return self.ctr
 
     def state(self, rep: int, cap_idx: int, r: int) -> np.ndarray:
-        out = np.zeros(self.caps[cap_idx], np.uint64)
+        out = np.zeros(TOKEN_LRU_MAX_ENTRIES if self.tokens else self.caps[cap_idx], np.uint64)
         f = lib().orc_replay_state(self._h, rep, cap_idx, r, _p(out, C.c_uint64))
         return out[:f].copy()

@@ -557,11 +557,36 @@ int orc_route(const orc_plan *const *plans, const orc_ring *const *rings, const 
 typedef struct {
     uint32_t n_rep, R, n_caps;
     uint32_t *caps;
+    uint32_t tokens;  /* 0: capacities in prefixes; 1: in prefix tokens */
     uint32_t *fill;   /* [n_rep][n_caps][R] */
     uint64_t **list;  /* [n_rep][n_caps][R] -> keys, most recent first */
+    uint32_t **size;  /* token mode: prefix tokens of each listed key */
+    uint64_t *total;  /* token mode: tokens held by each simulator */
 } orc_replay;
 
+/* A token-weighted simulator also holds at most this many prefixes. */
+#define ORC_TOKEN_LRU_MAX_ENTRIES 1024
+
+static orc_replay *replay_new(uint32_t n_rep, uint32_t R, const uint32_t *caps, uint32_t n_caps,
+                              uint32_t tokens);
+
 orc_replay *orc_replay_create(uint32_t n_rep, uint32_t R, const uint32_t *caps, uint32_t n_caps)
+{
+    return replay_new(n_rep, R, caps, n_caps, 0);
+}
+
+/* Token-weighted variant (byte-aware capacity): a simulator holds whole
+ * prefixes, most recent first, while their prefix tokens sum to at most its
+ * capacity (and at most ORC_TOKEN_LRU_MAX_ENTRIES prefixes); an access moves
+ * or inserts its key at the front with the request's prefix length, then the
+ * least recent prefixes are evicted until both limits hold. */
+orc_replay *orc_replay_create_tokens(uint32_t n_rep, uint32_t R, const uint32_t *caps, uint32_t n_caps)
+{
+    return replay_new(n_rep, R, caps, n_caps, 1);
+}
+
+static orc_replay *replay_new(uint32_t n_rep, uint32_t R, const uint32_t *caps, uint32_t n_caps,
+                              uint32_t tokens)
 {
     if (n_rep == 0 || R == 0 || n_caps == 0)
         return NULL;
@@ -574,12 +599,19 @@ orc_replay *orc_replay_create(uint32_t n_rep, uint32_t R, const uint32_t *caps, 
     s->n_caps = n_caps;
     s->caps = (uint32_t *)malloc(n_caps * sizeof(uint32_t));
     memcpy(s->caps, caps, n_caps * sizeof(uint32_t));
+    s->tokens = tokens;
     uint64_t nsim = (uint64_t)n_rep * n_caps * R;
     s->fill = (uint32_t *)calloc(nsim, sizeof(uint32_t));
     s->list = (uint64_t **)calloc(nsim, sizeof(uint64_t *));
+    if (tokens) {
+        s->size = (uint32_t **)calloc(nsim, sizeof(uint32_t *));
+        s->total = (uint64_t *)calloc(nsim, sizeof(uint64_t));
+    }
     for (uint64_t i = 0; i < nsim; ++i) {
-        uint32_t c = caps[(i / R) % n_caps];
+        uint32_t c = tokens ? ORC_TOKEN_LRU_MAX_ENTRIES : caps[(i / R) % n_caps];
         s->list[i] = (uint64_t *)malloc((uint64_t)c * sizeof(uint64_t));
+        if (tokens)
+            s->size[i] = (uint32_t *)malloc((uint64_t)c * sizeof(uint32_t));
     }
     return s;
 }
@@ -589,9 +621,14 @@ void orc_replay_free(orc_replay *s)
     if (!s)
         return;
     uint64_t nsim = (uint64_t)s->n_rep * s->n_caps * s->R;
-    for (uint64_t i = 0; i < nsim; ++i)
+    for (uint64_t i = 0; i < nsim; ++i) {
         free(s->list[i]);
+        if (s->tokens)
+            free(s->size[i]);
+    }
     free(s->list);
+    free(s->size);
+    free(s->total);
     free(s->fill);
     free(s->caps);
     free(s);
@@ -624,6 +661,38 @@ int orc_shadow_replay(orc_replay *s, const uint64_t *key, const uint32_t *plen,
                     }
                 C[CTR_REQ] += 1;
                 C[CTR_PROMPT] += (uint64_t)plen[i] + slen[i];
+                if (s->tokens) {
+                    uint32_t *sz = s->size[sim];
+                    uint64_t T = s->total[sim];
+                    if (at < f) {
+                        C[CTR_HIT] += 1;
+                        C[CTR_HIT_TOK] += plen[i];
+                        C[CTR_PREFILL] += slen[i];
+                        T -= sz[at];
+                    } else {
+                        C[CTR_PREFILL] += (uint64_t)plen[i] + slen[i];
+                        if (f == ORC_TOKEN_LRU_MAX_ENTRIES) {
+                            /* a full list: the least recent prefix makes room (the
+                             * entry limit would evict it after the insertion) */
+                            T -= sz[f - 1];
+                            f -= 1;
+                        }
+                        at = f;
+                        f += 1;
+                    }
+                    memmove(lst + 1, lst, (uint64_t)at * sizeof(uint64_t));
+                    memmove(sz + 1, sz, (uint64_t)at * sizeof(uint32_t));
+                    lst[0] = key[i];
+                    sz[0] = plen[i];
+                    T += plen[i];
+                    while (f > 0 && T > cap) { /* least recent first */
+                        T -= sz[f - 1];
+                        f -= 1;
+                    }
+                    s->fill[sim] = f;
+                    s->total[sim] = T;
+                    continue;
+                }
                 if (at < f) {
                     /* hit: move to the most-recent position */
                     memmove(lst + 1, lst, (uint64_t)at * sizeof(uint64_t));

@@ -58,7 +58,7 @@ def run_trace(trace: tg.Trace, intervals: Optional[Iterable[int]] = None, align:
     reps = cfg.replicas
     pols = [p for p, _ in reps]
     seeds = [s for _, s in reps]
-    rp = Replay(len(reps), cfg.R, cfg.caps)
+    rp = Replay(len(reps), cfg.R, cfg.caps, tokens=cfg.lru_tokens)
     rings = rings_for(cfg)
     prev = None
     out = {"intervals": [], "keys": [], "plans": [], "dest": [], "load": [], "requests": 0}

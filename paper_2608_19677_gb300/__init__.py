@@ -37,7 +37,8 @@ EXPORTS = ("cr_create", "cr_destroy", "cr_set_stream", "cr_sync", "cr_last_error
            "cr_hash_prefixes", "cr_plan_create", "cr_plan_destroy", "cr_build_plans", "cr_build_plan",
            "cr_plan_get_info", "cr_plan_export", "cr_route_batch", "cr_replay_create", "cr_replay_reset",
            "cr_replay_destroy", "cr_shadow_replay", "cr_replay_export_state", "cr_key_histogram_noalloc",
-           "cr_ring_create", "cr_ring_destroy", "cr_ring_export", "cr_plan_diff")
+           "cr_ring_create", "cr_ring_destroy", "cr_ring_export", "cr_plan_diff",
+           "cr_replay_create_tokens")
 CR_NOALLOC_MAX_KEYS = 65536
 
 
@@ -103,6 +104,7 @@ def lib() -> C.CDLL:
         "cr_plan_export": ([vp, vp] + [vp] * 9, i32),
         "cr_route_batch": ([vp, C.POINTER(vp), C.POINTER(Replica), u32, u32, vp, u64, u64, u32, vp, vp], i32),
         "cr_replay_create": ([vp, u32, u32, C.POINTER(C.c_uint32), u32, C.POINTER(vp)], i32),
+        "cr_replay_create_tokens": ([vp, u32, u32, C.POINTER(C.c_uint32), u32, C.POINTER(vp)], i32),
         "cr_replay_reset": ([vp, vp], i32),
         "cr_replay_destroy": ([vp, vp], i32),
         "cr_shadow_replay": ([vp, vp, vp, vp, vp, vp, u64, vp], i32),
@@ -339,13 +341,16 @@ def route_batch(ctx: Context, plans: Sequence[Optional[Plan]], policies: Sequenc
 
 
 class Replay:
-    """Library-owned LRU state for n_rep x R destinations x len(caps) capacities."""
+    """Library-owned LRU state for n_rep x R destinations x len(caps) capacities.
 
-    def __init__(self, ctx: Context, n_rep: int, R: int, caps: Sequence[int]):
-        self.ctx, self.n_rep, self.R, self.caps = ctx, n_rep, R, list(caps)
+    ``tokens``: capacities count prefix tokens (byte-aware variant, cr_replay_create_tokens)."""
+
+    def __init__(self, ctx: Context, n_rep: int, R: int, caps: Sequence[int], tokens: bool = False):
+        self.ctx, self.n_rep, self.R, self.caps, self.tokens = ctx, n_rep, R, list(caps), tokens
         cp = (C.c_uint32 * len(caps))(*caps)
         h = C.c_void_p()
-        ctx.check(lib().cr_replay_create(ctx.handle, n_rep, R, cp, len(caps), C.byref(h)), "cr_replay_create")
+        name = "cr_replay_create_tokens" if tokens else "cr_replay_create"
+        ctx.check(getattr(lib(), name)(ctx.handle, n_rep, R, cp, len(caps), C.byref(h)), name)
         self._h = h
 
     @property

@@ -12,6 +12,7 @@
 #define CR_FLAG_OVERFLOW 1u  // a load reached 2^47, or a stamp counter overflowed
 #define CR_FLAG_BADDEST 2u   // a destination index >= R reached the replay
 #define CR_FLAG_TIMEOUT 4u   // a bounded wait gave up
+#define CR_FLAG_BADSIZE 8u   // token-weighted replay: a key came back with another prefix length
 
 // ---- scratch slots owned by the context ------------------------------------
 enum cr_scratch_slot {
@@ -89,7 +90,9 @@ struct cr_ring {
 };
 
 struct cr_replay {
-    uint32_t n_rep, R, n_caps, cmax;
+    uint32_t n_rep, R, n_caps, cmax;  // cmax: largest capacity, or CR_MAX_CAP entries in token mode
+    int tokens;                       // capacities in prefix tokens (one state buffer, d_size used)
+    uint32_t *d_size;                // token mode: [stream][cmax] prefix tokens of each listed key
     uint32_t caps[CR_MAX_CAPS];
     uint64_t n_streams;              // n_rep * R
     unsigned long long *d_keys[2];   // [stream][cmax], most recent first; double-buffered

@@ -537,6 +537,146 @@ int launch_batch(cr_ctx *ctx, cr_replay *rp, const replay_caps &caps, uint32_t C
     return launch_batch_nc<CR_MAX_CAPS>(ctx, rp, caps, CL, start, coff, total, m, rec, d_ctr);
 }
 
+// ---- token-weighted variant ---------------------------------------------------
+// Capacities count prefix tokens.  With one prefix length per key, the cache
+// of capacity c holds the longest run of most recent prefixes whose tokens fit
+// in c (evictions always take the least recent), so one list at the largest
+// capacity decides every capacity: a request hits at c iff its key is listed
+// and the tokens from the front of the list through the key are <= c.  One
+// warp per (replica, destination) stream walks the stream's requests in
+// order; the list (key, tokens) lives in shared memory, scanned 32 entries at
+// a time with a ballot for the key and a warp scan of the tokens; records are
+// fetched 32 ahead, one per lane, and broadcast by shuffles.
+constexpr int kTokWarps = 4;
+constexpr uint32_t kTokMax = CR_MAX_CAP;  // prefixes per list
+
+__global__ void __launch_bounds__(kTokWarps * 32) k_lru_tokens(const __grid_constant__ replay_caps caps, uint32_t ns,
+                                                               uint32_t R, const uint32_t *__restrict__ start,
+                                                               const rec16 *__restrict__ rec,
+                                                               unsigned long long *__restrict__ keys_state,
+                                                               uint32_t *__restrict__ size_state,
+                                                               uint32_t *__restrict__ fill_state,
+                                                               unsigned long long *__restrict__ ctr, uint32_t *status)
+{
+    extern __shared__ unsigned long long tok_sh[];
+    const uint32_t lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+    const uint32_t s = blockIdx.x * kTokWarps + w;
+    if (s >= ns) return;  // whole warps only; the kernel has no block-wide barrier
+    unsigned long long *K = tok_sh + (size_t)w * kTokMax;
+    uint32_t *Z = reinterpret_cast<uint32_t *>(tok_sh + (size_t)kTokWarps * kTokMax) + (size_t)w * kTokMax;
+    uint32_t capmax = 0;
+    for (uint32_t c = 0; c < caps.n_caps; ++c) capmax = caps.cap[c] > capmax ? caps.cap[c] : capmax;
+    const uint32_t mycap = lane < caps.n_caps ? caps.cap[lane] : 0u;
+    // state
+    uint32_t f = fill_state[s];
+    unsigned long long T = 0;
+    for (uint32_t j = lane; j < f; j += 32) {
+        K[j] = keys_state[(size_t)s * kTokMax + j];
+        const uint32_t z = size_state[(size_t)s * kTokMax + j];
+        Z[j] = z;
+        T += z;
+    }
+    for (int o = 16; o > 0; o >>= 1) T += __shfl_xor_sync(0xffffffffu, T, o);
+    __syncwarp();
+    unsigned long long c_req = 0, c_hit = 0, c_hit_tok = 0, c_prompt = 0, c_prefill = 0;  // lane = capacity
+    const uint32_t i0 = start[s], i1 = start[s + 1];
+    rec16 nx = {0ull, 0u, 0u};
+    if (i0 + lane < i1) nx = rec[i0 + lane];
+    for (uint32_t b0 = i0; b0 < i1; b0 += 32) {
+        const rec16 cur = nx;
+        if (b0 + 32 + lane < i1) nx = rec[b0 + 32 + lane];  // next 32 records in flight
+        const uint32_t nb = i1 - b0 < 32 ? i1 - b0 : 32;
+        for (uint32_t q = 0; q < nb; ++q) {
+            const unsigned long long x = __shfl_sync(0xffffffffu, cur.key, q);
+            const uint32_t P = __shfl_sync(0xffffffffu, cur.P, q);
+            const uint32_t S = __shfl_sync(0xffffffffu, cur.S, q);
+            // find x and the tokens from the front through it
+            uint32_t pos = f, zx = 0;
+            unsigned long long upto = 0, acc = 0;
+            for (uint32_t c0 = 0; c0 < f; c0 += 32) {
+                const uint32_t j = c0 + lane;
+                const bool v = j < f;
+                const uint32_t z = v ? Z[j] : 0u;
+                const unsigned match = __ballot_sync(0xffffffffu, v && K[j] == x);
+                unsigned long long incl = z;  // inclusive scan of the chunk's tokens
+                for (int o = 1; o < 32; o <<= 1) {
+                    const unsigned long long y = __shfl_up_sync(0xffffffffu, incl, o);
+                    if (lane >= (uint32_t)o) incl += y;
+                }
+                if (match) {
+                    const uint32_t l = __ffs(match) - 1;
+                    pos = c0 + l;
+                    zx = __shfl_sync(0xffffffffu, z, l);
+                    upto = acc + __shfl_sync(0xffffffffu, incl, l);
+                    break;
+                }
+                acc += __shfl_sync(0xffffffffu, incl, 31);
+            }
+            const bool found = pos < f;
+            if (found && zx != P && lane == 0) atomicOr(status, CR_FLAG_BADSIZE);
+            if (lane < caps.n_caps) {
+                const bool hit = found && upto <= mycap;
+                c_req += 1;
+                c_prompt += (unsigned long long)P + S;
+                if (hit) {
+                    c_hit += 1;
+                    c_hit_tok += P;
+                    c_prefill += S;
+                } else {
+                    c_prefill += (unsigned long long)P + S;
+                }
+            }
+            // move or insert x at the front
+            if (found) {
+                T -= zx;
+            } else {
+                if (f == kTokMax) {  // the least recent prefix makes room
+                    T -= Z[f - 1];
+                    --f;
+                }
+                pos = f;
+                ++f;
+            }
+            for (int c0 = (int)((pos + 31) / 32) * 32 - 32; c0 >= 0; c0 -= 32) {  // shift [0, pos) down by one
+                const uint32_t j = (uint32_t)c0 + lane;
+                const bool m = j < pos;
+                const unsigned long long k = m ? K[j] : 0ull;
+                const uint32_t z = m ? Z[j] : 0u;
+                __syncwarp();
+                if (m) {
+                    K[j + 1] = k;
+                    Z[j + 1] = z;
+                }
+                __syncwarp();
+            }
+            if (lane == 0) {
+                K[0] = x;
+                Z[0] = P;
+            }
+            T += P;
+            __syncwarp();
+            while (f > 0 && T > capmax) {  // evict the least recent until the tokens fit
+                T -= Z[f - 1];
+                --f;
+            }
+        }
+    }
+    for (uint32_t j = lane; j < f; j += 32) {
+        keys_state[(size_t)s * kTokMax + j] = K[j];
+        size_state[(size_t)s * kTokMax + j] = Z[j];
+    }
+    if (lane == 0) fill_state[s] = f;
+    if (lane < caps.n_caps) {
+        const uint32_t rep = s / R, r = s - rep * R;
+        unsigned long long *C = ctr + (((unsigned long long)rep * caps.n_caps + lane) * R + r) * CR_CTR_FIELDS;
+        C[0] += c_req;
+        C[1] += c_hit;
+        C[2] += c_hit_tok;
+        C[3] += c_prompt;
+        C[4] += c_prefill;
+    }
+}
+
 }  // namespace
 
 extern "C" int cr_replay_create(cr_ctx *ctx, uint32_t n_rep, uint32_t R, const uint32_t *caps, uint32_t n_caps,
@@ -577,11 +717,43 @@ extern "C" int cr_replay_create(cr_ctx *ctx, uint32_t n_rep, uint32_t R, const u
     return cr_replay_reset(ctx, rp);
 }
 
+extern "C" int cr_replay_create_tokens(cr_ctx *ctx, uint32_t n_rep, uint32_t R, const uint32_t *token_caps,
+                                       uint32_t n_caps, cr_replay **out)
+{
+    if (!ctx || !out || !token_caps) return CR_EINVAL;
+    *out = nullptr;
+    if (n_rep == 0 || n_rep > CR_MAX_REPLICAS) return cr_fail(ctx, CR_EINVAL, "replay: n_rep=%u", n_rep);
+    if (R == 0 || R > CR_MAX_R) return cr_fail(ctx, CR_EINVAL, "replay: R=%u", R);
+    if (n_caps == 0 || n_caps > CR_MAX_CAPS) return cr_fail(ctx, CR_EINVAL, "replay: n_caps=%u", n_caps);
+    for (uint32_t c = 0; c < n_caps; ++c)
+        if (token_caps[c] == 0) return cr_fail(ctx, CR_EINVAL, "replay: token capacity 0");
+    if ((uint64_t)n_rep * R >= (1ull << 31)) return cr_fail(ctx, CR_EINVAL, "replay: too many streams");
+    cr_replay *rp = (cr_replay *)calloc(1, sizeof(cr_replay));
+    if (!rp) return cr_fail(ctx, CR_ENOMEM, "replay: host allocation failed");
+    rp->n_rep = n_rep;
+    rp->R = R;
+    rp->n_caps = n_caps;
+    rp->cmax = kTokMax;
+    rp->tokens = 1;
+    memcpy(rp->caps, token_caps, n_caps * sizeof(uint32_t));
+    rp->n_streams = (uint64_t)n_rep * R;
+    if (cudaMalloc(&rp->d_keys[0], rp->n_streams * kTokMax * sizeof(unsigned long long)) != cudaSuccess ||
+        cudaMalloc(&rp->d_size, rp->n_streams * kTokMax * sizeof(uint32_t)) != cudaSuccess ||
+        cudaMalloc(&rp->d_fill[0], rp->n_streams * sizeof(uint32_t)) != cudaSuccess) {
+        cudaGetLastError();
+        cr_replay_destroy(ctx, rp);
+        return cr_fail(ctx, CR_ENOMEM, "replay: cannot allocate state");
+    }
+    *out = rp;
+    return cr_replay_reset(ctx, rp);
+}
+
 extern "C" int cr_replay_reset(cr_ctx *ctx, cr_replay *rp)
 {
     if (!ctx || !rp) return CR_EINVAL;
     for (int b = 0; b < 2; ++b)
-        CR_CUDA(ctx, cudaMemsetAsync(rp->d_fill[b], 0, rp->n_streams * sizeof(uint32_t), ctx->stream));
+        if (rp->d_fill[b])
+            CR_CUDA(ctx, cudaMemsetAsync(rp->d_fill[b], 0, rp->n_streams * sizeof(uint32_t), ctx->stream));
     return CR_OK;
 }
 
@@ -590,9 +762,10 @@ extern "C" int cr_replay_destroy(cr_ctx *ctx, cr_replay *rp)
     if (!rp) return CR_OK;
     if (ctx) cudaStreamSynchronize(ctx->stream);
     for (int b = 0; b < 2; ++b) {
-        cudaFree(rp->d_keys[b]);
-        cudaFree(rp->d_fill[b]);
+        if (rp->d_keys[b]) cudaFree(rp->d_keys[b]);
+        if (rp->d_fill[b]) cudaFree(rp->d_fill[b]);
     }
+    if (rp->d_size) cudaFree(rp->d_size);
     free(rp);
     return CR_OK;
 }
@@ -636,6 +809,16 @@ extern "C" int cr_shadow_replay(cr_ctx *ctx, cr_replay *rp, const uint64_t *d_ke
     replay_caps caps;
     caps.n_caps = rp->n_caps;
     for (uint32_t c = 0; c < CR_MAX_CAPS; ++c) caps.cap[c] = c < rp->n_caps ? rp->caps[c] : 0;
+    if (rp->tokens) {
+        // token-weighted: one warp per stream, its list in shared memory, state updated in place
+        const size_t tsmem = (size_t)kTokWarps * kTokMax * (sizeof(unsigned long long) + sizeof(uint32_t));
+        if (tsmem > 48 * 1024)
+            CR_CUDA(ctx, cudaFuncSetAttribute(k_lru_tokens, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)tsmem));
+        CR_LAUNCH(ctx, k_lru_tokens, (ns + kTokWarps - 1) / kTokWarps, kTokWarps * 32, tsmem, caps, ns, R,
+                  (const uint32_t *)start, (const rec16 *)rec, (unsigned long long *)rp->d_keys[0], rp->d_size,
+                  rp->d_fill[0], (unsigned long long *)d_ctr, ctx->d_status);
+        return CR_OK;
+    }
     // chunk length: long enough that rebuilding an LRU state of cmax entries is amortised
     const uint32_t CL = rp->cmax * 16u > 256u ? rp->cmax * 16u : 256u;
     CR_LAUNCH(ctx, k_chunk_counts, cr_blocks(ns, 256, gcap), 256, 0, (const uint32_t *)start, ns, CL, coff);

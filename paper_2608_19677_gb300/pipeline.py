@@ -12,7 +12,7 @@ One control interval t:
   3. cr_route_batch: every (policy, seed) replica, loads starting at zero
      (bounded-load replicas use a ring built once, seeded by the replica);
   4. cr_shadow_replay: LRU simulators whose state and counters persist over
-     intervals.
+     intervals (capacities in prefixes, or with ``lru_tokens`` in prefix tokens).
 
 With ``overlap=True`` the planner runs on its own high-priority stream and
 library context, ordered by CUDA events: plans(t+1) need only interval t's
@@ -42,7 +42,7 @@ class Pipeline:
     def __init__(self, ctx: Context, R: int, W: int, caps: Sequence[int],
                  replicas: Sequence[Tuple[str, int]], qcap: Callable[[int], Tuple[int, int]],
                  batch_B: int = 1024, salt: int = 0, max_n: int = 0, overlap: bool = False,
-                 vnodes: int = 64, fresh: bool = False):
+                 vnodes: int = 64, fresh: bool = False, lru_tokens: bool = False):
         import torch
         self.ctx, self.R, self.W, self.caps = ctx, R, W, list(caps)
         self.replicas = list(replicas)
@@ -80,7 +80,7 @@ class Pipeline:
             self.hstream = self.pstream = self.ystream = self.mstream
             self.hctx = self.pctx = self.yctx = ctx
         self.plans = [[Plan(self.pctx) for _ in self.plan_keys] for _ in range(2)]
-        self.replay = Replay(ctx, len(self.replicas), R, self.caps)
+        self.replay = Replay(ctx, len(self.replicas), R, self.caps, tokens=lru_tokens)
         # ring of every bounded-load replica, seeded by the replica's seed (built once)
         self.rings = [Ring(ctx, R, vnodes, s) if p == "CHWBL" else None for p, s in self.replicas]
         self.ctr = torch.zeros((len(self.replicas), len(self.caps), R, 5), dtype=torch.int64, device=dev)

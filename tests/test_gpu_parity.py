@@ -552,3 +552,75 @@ def test_pipeline_parity_drift_fresh_and_stale(P, ctx, fresh):
             assert got["n_adm"] == opl.n_adm and (got["members"] == opl.members).all()
     pipe.sync()
     assert (h_u64(pipe.ctr) == ref["ctr"]).all()
+
+
+# ------------------------------------------------------------------ f3 token-weighted replay ---
+def _fixed_len_stream(rng, n, nkeys, lo=16, hi=5000, spread=1.2):
+    keys = _rates_keys(rng, nkeys, n, skew=spread)[:n]
+    uk, inv = np.unique(keys, return_inverse=True)
+    size_of = rng.integers(lo, hi, size=uk.size).astype(np.uint32)  # one prefix length per key
+    return keys, size_of[inv]
+
+
+@pytest.mark.parametrize("caps,lo,hi", [([24576], 16, 5000), ([1, 100, 3000], 16, 5000),
+                                        ([4096, 65536, 2 ** 32 - 1], 16, 200),   # 1024-prefix bound
+                                        ([5000, 10 ** 6], 1, 3)])
+def test_token_replay_parity(P, ctx, caps, lo, hi):
+    rng = np.random.default_rng(sum(caps) % 1000 + lo)
+    n_rep, R, n = 3, 7, 24000
+    keys, plen = _fixed_len_stream(rng, n, int(rng.integers(50, 3000)), lo, hi)
+    n = keys.size
+    slen = rng.integers(0, 200, size=n).astype(np.uint32)
+    dest = tg.random_dest(n_rep, n, R, 5)
+    orp = O.Replay(n_rep, R, caps, tokens=True)
+    rp = P.Replay(ctx, n_rep, R, caps, tokens=True)
+    ctr = torch.zeros((n_rep, len(caps), R, 5), dtype=torch.int64, device=DEV)
+    dk, dp, ds, dd = d_u64(keys), d_u32(plen), d_u32(slen), d_u16(dest)
+    cut = n // 3
+    for a, b in ((0, cut), (cut, n)):  # state persists across calls
+        orp.step(keys[a:b], plen[a:b], slen[a:b], dest[:, a:b])
+        P.shadow_replay(ctx, rp, dk[a:b].contiguous(), dp[a:b].contiguous(), ds[a:b].contiguous(),
+                        dd[:, a:b].contiguous(), ctr)
+        ctx.sync()
+        assert (h_u64(ctr) == orp.ctr).all()
+    ci = caps.index(max(caps))
+    for rep in range(n_rep):
+        for r in range(R):
+            assert (rp.state(rep, r) == orp.state(rep, ci, r)).all()
+
+
+def test_token_replay_changed_length_is_reported(P, ctx):
+    rp = P.Replay(ctx, 1, 2, [10000], tokens=True)
+    keys = d_u64(np.array([5, 6, 5], np.uint64))
+    plen = d_u32(np.array([100, 200, 150], np.uint32))  # key 5 comes back with another length
+    slen = d_u32(np.zeros(3, np.uint32))
+    dest = d_u16(np.zeros((1, 3), np.uint16))
+    ctr = torch.zeros((1, 1, 2, 5), dtype=torch.int64, device=DEV)
+    P.shadow_replay(ctx, rp, keys, plen, slen, dest, ctr)
+    with pytest.raises(P.CacheRouteError):
+        ctx.sync()
+    rp.reset()
+    P.shadow_replay(ctx, rp, keys[:2].contiguous(), plen[:2].contiguous(), slen[:2].contiguous(),
+                    dest[:, :2].contiguous(), ctr)
+    ctx.sync()
+    assert rp.state(0, 0).tolist() == [6, 5]
+
+
+@pytest.mark.parametrize("name,n,nint", [("70b", 40000, 3), ("large", 100000, 2)])
+def test_pipeline_parity_token_lru(P, ctx, name, n, nint):
+    from paper_2608_19677_gb300.pipeline import Pipeline
+    cfg = tg.CONFIGS[name].scaled(n, nint).token_lru()
+    if name == "large":  # fewer replicas keep the oracle quick; R, caps and the 1024-prefix bound stay
+        import dataclasses
+        cfg = dataclasses.replace(cfg, seeds=[0, 1])
+    tr = tg.Trace(cfg)
+    ref = OP.run_trace(tr, B=1024, keep=True)
+    pipe = Pipeline(ctx, cfg.R, cfg.W, cfg.caps, cfg.replicas, tr.qcap, batch_B=1024, overlap=True,
+                    lru_tokens=True)
+    for t in range(cfg.n_intervals):
+        iv = tr.interval(t)
+        tok, off = tg.arena_host(tr, iv, 4)
+        pipe.interval(t, torch.from_numpy(tok).to(DEV), d_u64(off), d_u32(iv.plen), d_u32(iv.slen), iv.g0,
+                      plan_next=t + 1 < cfg.n_intervals)
+    pipe.sync()
+    assert (h_u64(pipe.ctr) == ref["ctr"]).all()

@@ -78,6 +78,8 @@ class TraceConfig:
     burst: Optional[Tuple[float, float, float]] = None  # (factor, burst_len_s, period_s)
     vnodes: int = 64            # ring points per destination of bounded-load (CHWBL) replicas
     drift: Optional[float] = None  # sigma of a per-interval lognormal random walk of every key's rate
+    token_caps: Optional[List[int]] = None  # LRU capacities in prefix tokens for the byte-aware replay
+    lru_tokens: bool = False    # replay capacities (caps) count prefix tokens instead of prefixes
 
     @property
     def replicas(self) -> List[Tuple[str, int]]:
@@ -86,6 +88,19 @@ class TraceConfig:
     @property
     def total_keys(self) -> int:
         return self.n_keys + (len(self.whales) if self.whales else 0)
+
+    def token_lru(self) -> "TraceConfig":
+        """The same workload replayed with token-weighted LRU capacities: ``token_caps``, or
+        each prefix-count capacity times the typical prefix length."""
+        if self.lru_tokens:
+            return self
+        if self.token_caps:
+            caps = list(self.token_caps)
+        else:
+            kind = self.plen[0]
+            typical = self.plen[1] if kind in ("fixed", "lognormal") else (self.plen[1] + self.plen[2]) // 2
+            caps = [c * typical for c in self.caps]
+        return dataclasses.replace(self, caps=caps, lru_tokens=True, name=f"{self.name} [token LRU]")
 
     def scaled(self, n_requests: int, n_intervals: Optional[int] = None, name: Optional[str] = None):
         """Same shape, fewer requests (for sampled or quick runs)."""
@@ -102,7 +117,7 @@ CONFIGS: Dict[str, TraceConfig] = {
     "70b": TraceConfig(
         name="70b", R=30, n_keys=20_000, zipf_s=1.0, n_requests=2_000_000, n_intervals=12,
         interval_s=10.0, plen=("lognormal", 2048, 0.5, 16384), W=12, caps=[12],
-        policies=["CR", "P2C", "RR", "HASH"], seeds=[0, 1, 2, 3, 4], hot_cap=1.0 / 30),
+        policies=["CR", "P2C", "RR", "HASH"], seeds=[0, 1, 2, 3, 4], hot_cap=1.0 / 30, token_caps=[24576]),
     "8b": TraceConfig(
         name="8b", R=16, n_keys=5_000, zipf_s=1.1, n_requests=4_000_000, n_intervals=800,
         interval_s=10.0, plen=("uniform", 1024, 4096), W=64, caps=[64],
