@@ -314,7 +314,7 @@ CR_API int cr_replay_create(cr_ctx *ctx, uint32_t n_rep, uint32_t R, const uint3
 /* Byte-aware variant (token-weighted capacity; the paper's byte budgets of
  * sec. 3.1 and 6, and the 70B configuration's 24k-token slot budget read as
  * tokens): every simulator holds whole prefixes, most recent first, while their
- * prefix tokens sum to at most its capacity (token_caps[], 1 .. 2^32-1) and
+ * prefix tokens sum to at most its capacity (token_caps[], 1 .. 2^31) and
  * there are at most CR_MAX_CAP of them; an access moves or inserts its key at
  * the front, then the least recent prefixes are evicted until both limits
  * hold.  A key must have the same prefix length at every access (the longest

@@ -92,7 +92,7 @@ struct cr_ring {
 struct cr_replay {
     uint32_t n_rep, R, n_caps, cmax;  // cmax: largest capacity, or CR_MAX_CAP entries in token mode
     int tokens;                       // capacities in prefix tokens (one state buffer, d_size used)
-    uint32_t *d_size;                // token mode: [stream][cmax] prefix tokens of each listed key
+    uint32_t *d_size;                // token mode: [stream][cmax] tokens of the listed keys up to each one
     uint32_t caps[CR_MAX_CAPS];
     uint64_t n_streams;              // n_rep * R
     unsigned long long *d_keys[2];   // [stream][cmax], most recent first; double-buffered

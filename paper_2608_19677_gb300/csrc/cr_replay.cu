@@ -544,17 +544,28 @@ int launch_batch(cr_ctx *ctx, cr_replay *rp, const replay_caps &caps, uint32_t C
 // capacity decides every capacity: a request hits at c iff its key is listed
 // and the tokens from the front of the list through the key are <= c.  One
 // warp per (replica, destination) stream walks the stream's requests in
-// order; the list (key, tokens) lives in shared memory, scanned 32 entries at
-// a time with a ballot for the key and a warp scan of the tokens; records are
-// fetched 32 ahead, one per lane, and broadcast by shuffles.
+// order.  The list holds keys and CUMULATIVE tokens (entry j: the tokens of
+// entries 0..j), so a lookup is a ballot plus one read, moving a key to the
+// front adds its length to the entries it passes, and eviction is a ballot on
+// the tail.  A list of at most 32 prefixes lives in registers (lane j holds
+// entry j; the move is a shuffle-up); a longer one lives in shared memory and
+// is scanned 32 entries at a time.  Only hits and hit tokens depend on the
+// capacity; request and prompt totals are summed once per 32 records.
 constexpr int kTokWarps = 4;
 constexpr uint32_t kTokMax = CR_MAX_CAP;  // prefixes per list
+
+__device__ __forceinline__ uint32_t sat_add(uint32_t a, uint32_t b)
+{
+    // a sum past 2^32 - 1 is above every capacity (<= 2^31) and is evicted anyway
+    const unsigned long long v = (unsigned long long)a + b;
+    return v > 0xffffffffull ? 0xffffffffu : (uint32_t)v;
+}
 
 __global__ void __launch_bounds__(kTokWarps * 32) k_lru_tokens(const __grid_constant__ replay_caps caps, uint32_t ns,
                                                                uint32_t R, const uint32_t *__restrict__ start,
                                                                const rec16 *__restrict__ rec,
                                                                unsigned long long *__restrict__ keys_state,
-                                                               uint32_t *__restrict__ size_state,
+                                                               uint32_t *__restrict__ cum_state,
                                                                uint32_t *__restrict__ fill_state,
                                                                unsigned long long *__restrict__ ctr, uint32_t *status)
 {
@@ -563,22 +574,27 @@ __global__ void __launch_bounds__(kTokWarps * 32) k_lru_tokens(const __grid_cons
     const uint32_t s = blockIdx.x * kTokWarps + w;
     if (s >= ns) return;  // whole warps only; the kernel has no block-wide barrier
     unsigned long long *K = tok_sh + (size_t)w * kTokMax;
-    uint32_t *Z = reinterpret_cast<uint32_t *>(tok_sh + (size_t)kTokWarps * kTokMax) + (size_t)w * kTokMax;
+    uint32_t *Cm = reinterpret_cast<uint32_t *>(tok_sh + (size_t)kTokWarps * kTokMax) + (size_t)w * kTokMax;
     uint32_t capmax = 0;
     for (uint32_t c = 0; c < caps.n_caps; ++c) capmax = caps.cap[c] > capmax ? caps.cap[c] : capmax;
     const uint32_t mycap = lane < caps.n_caps ? caps.cap[lane] : 0u;
-    // state
     uint32_t f = fill_state[s];
-    unsigned long long T = 0;
-    for (uint32_t j = lane; j < f; j += 32) {
-        K[j] = keys_state[(size_t)s * kTokMax + j];
-        const uint32_t z = size_state[(size_t)s * kTokMax + j];
-        Z[j] = z;
-        T += z;
+    unsigned long long kr = 0;  // register list: entry `lane`
+    uint32_t cr = 0;
+    bool inreg = f <= 32;
+    if (inreg) {
+        if (lane < f) {
+            kr = keys_state[(size_t)s * kTokMax + lane];
+            cr = cum_state[(size_t)s * kTokMax + lane];
+        }
+    } else {
+        for (uint32_t j = lane; j < f; j += 32) {
+            K[j] = keys_state[(size_t)s * kTokMax + j];
+            Cm[j] = cum_state[(size_t)s * kTokMax + j];
+        }
     }
-    for (int o = 16; o > 0; o >>= 1) T += __shfl_xor_sync(0xffffffffu, T, o);
     __syncwarp();
-    unsigned long long c_req = 0, c_hit = 0, c_hit_tok = 0, c_prompt = 0, c_prefill = 0;  // lane = capacity
+    unsigned long long c_hit = 0, c_hit_tok = 0, c_prompt = 0;  // lane = capacity (prompt: every lane)
     const uint32_t i0 = start[s], i1 = start[s + 1];
     rec16 nx = {0ull, 0u, 0u};
     if (i0 + lane < i1) nx = rec[i0 + lane];
@@ -586,94 +602,132 @@ __global__ void __launch_bounds__(kTokWarps * 32) k_lru_tokens(const __grid_cons
         const rec16 cur = nx;
         if (b0 + 32 + lane < i1) nx = rec[b0 + 32 + lane];  // next 32 records in flight
         const uint32_t nb = i1 - b0 < 32 ? i1 - b0 : 32;
+        if (lane < nb) c_prompt += (unsigned long long)cur.P + cur.S;
         for (uint32_t q = 0; q < nb; ++q) {
             const unsigned long long x = __shfl_sync(0xffffffffu, cur.key, q);
             const uint32_t P = __shfl_sync(0xffffffffu, cur.P, q);
-            const uint32_t S = __shfl_sync(0xffffffffu, cur.S, q);
-            // find x and the tokens from the front through it
-            uint32_t pos = f, zx = 0;
-            unsigned long long upto = 0, acc = 0;
-            for (uint32_t c0 = 0; c0 < f; c0 += 32) {
-                const uint32_t j = c0 + lane;
-                const bool v = j < f;
-                const uint32_t z = v ? Z[j] : 0u;
-                const unsigned match = __ballot_sync(0xffffffffu, v && K[j] == x);
-                unsigned long long incl = z;  // inclusive scan of the chunk's tokens
-                for (int o = 1; o < 32; o <<= 1) {
-                    const unsigned long long y = __shfl_up_sync(0xffffffffu, incl, o);
-                    if (lane >= (uint32_t)o) incl += y;
+            bool found;
+            uint32_t upto = 0, zx = 0;
+            if (inreg) {
+                // ---- list in registers (f <= 32) ----
+                const unsigned match = __ballot_sync(0xffffffffu, lane < f && kr == x);
+                found = match != 0;
+                const uint32_t pos = found ? __ffs(match) - 1 : f;
+                const uint32_t cprev = __shfl_sync(0xffffffffu, cr, pos == 0 ? 0 : pos - 1);
+                if (found) {
+                    upto = __shfl_sync(0xffffffffu, cr, pos);
+                    zx = upto - (pos ? cprev : 0u);
                 }
-                if (match) {
-                    const uint32_t l = __ffs(match) - 1;
-                    pos = c0 + l;
-                    zx = __shfl_sync(0xffffffffu, z, l);
-                    upto = acc + __shfl_sync(0xffffffffu, incl, l);
-                    break;
+                // entries [0, pos) move down one place and now follow x
+                const unsigned long long kup = __shfl_up_sync(0xffffffffu, kr, 1);
+                const uint32_t cup = __shfl_up_sync(0xffffffffu, cr, 1);
+                const unsigned long long k31 = __shfl_sync(0xffffffffu, kr, 31);
+                const uint32_t c31 = __shfl_sync(0xffffffffu, cr, 31);
+                if (lane == 0) {
+                    kr = x;
+                    cr = P;
+                } else if (lane <= pos) {
+                    kr = kup;
+                    cr = sat_add(cup, P);
                 }
-                acc += __shfl_sync(0xffffffffu, incl, 31);
-            }
-            const bool found = pos < f;
-            if (found && zx != P && lane == 0) atomicOr(status, CR_FLAG_BADSIZE);
-            if (lane < caps.n_caps) {
-                const bool hit = found && upto <= mycap;
-                c_req += 1;
-                c_prompt += (unsigned long long)P + S;
-                if (hit) {
-                    c_hit += 1;
-                    c_hit_tok += P;
-                    c_prefill += S;
-                } else {
-                    c_prefill += (unsigned long long)P + S;
+                if (!found) ++f;  // f may reach 33: entry 32 is the old entry 31
+                const unsigned over = __ballot_sync(0xffffffffu, lane < f && cr > capmax);
+                if (over) {
+                    f = __ffs(over) - 1;  // the 33rd entry, if any, lies beyond and goes too
+                } else if (f == 33) {
+                    const uint32_t c32 = sat_add(c31, P);
+                    if (c32 > capmax) {
+                        f = 32;
+                    } else {  // the list outgrows the registers
+                        K[lane] = kr;
+                        Cm[lane] = cr;
+                        if (lane == 0) {
+                            K[32] = k31;
+                            Cm[32] = c32;
+                        }
+                        __syncwarp();
+                        inreg = false;
+                    }
                 }
-            }
-            // move or insert x at the front
-            if (found) {
-                T -= zx;
             } else {
-                if (f == kTokMax) {  // the least recent prefix makes room
-                    T -= Z[f - 1];
-                    --f;
+                // ---- list in shared memory (f > 32) ----
+                uint32_t pos = f;
+                for (uint32_t c0 = 0; c0 < f; c0 += 32) {
+                    const uint32_t j = c0 + lane;
+                    const unsigned match = __ballot_sync(0xffffffffu, j < f && K[j] == x);
+                    if (match) {
+                        pos = c0 + __ffs(match) - 1;
+                        break;
+                    }
                 }
-                pos = f;
-                ++f;
-            }
-            for (int c0 = (int)((pos + 31) / 32) * 32 - 32; c0 >= 0; c0 -= 32) {  // shift [0, pos) down by one
-                const uint32_t j = (uint32_t)c0 + lane;
-                const bool m = j < pos;
-                const unsigned long long k = m ? K[j] : 0ull;
-                const uint32_t z = m ? Z[j] : 0u;
+                found = pos < f;
+                if (found) {
+                    upto = Cm[pos];
+                    zx = upto - (pos ? Cm[pos - 1] : 0u);
+                } else {
+                    if (f == kTokMax) --f;  // the least recent prefix makes room
+                    pos = f;
+                    ++f;
+                }
+                for (int c0 = (int)((pos + 31) / 32) * 32 - 32; c0 >= 0; c0 -= 32) {  // [0, pos) down one
+                    const uint32_t j = (uint32_t)c0 + lane;
+                    const bool m = j < pos;
+                    const unsigned long long k = m ? K[j] : 0ull;
+                    const uint32_t cm = m ? Cm[j] : 0u;
+                    __syncwarp();
+                    if (m) {
+                        K[j + 1] = k;
+                        Cm[j + 1] = sat_add(cm, P);
+                    }
+                    __syncwarp();
+                }
+                if (lane == 0) {
+                    K[0] = x;
+                    Cm[0] = P;
+                }
                 __syncwarp();
-                if (m) {
-                    K[j + 1] = k;
-                    Z[j + 1] = z;
+                // the entries whose sums exceed the largest capacity form a suffix
+                for (int c0 = (int)((f + 31) / 32) * 32 - 32; c0 >= 0; c0 -= 32) {
+                    const uint32_t j = (uint32_t)c0 + lane;
+                    const unsigned over = __ballot_sync(0xffffffffu, j < f && Cm[j] > capmax);
+                    if (!over) break;
+                    f = (uint32_t)c0 + __ffs(over) - 1;
+                }
+                if (f <= 32) {  // back to registers
+                    kr = lane < f ? K[lane] : 0ull;
+                    cr = lane < f ? Cm[lane] : 0u;
+                    inreg = true;
                 }
                 __syncwarp();
             }
-            if (lane == 0) {
-                K[0] = x;
-                Z[0] = P;
-            }
-            T += P;
-            __syncwarp();
-            while (f > 0 && T > capmax) {  // evict the least recent until the tokens fit
-                T -= Z[f - 1];
-                --f;
+            if (found && zx != P && lane == 0) atomicOr(status, CR_FLAG_BADSIZE);
+            if (found && upto <= mycap) {  // lanes past n_caps have mycap 0 < upto
+                c_hit += 1;
+                c_hit_tok += P;
             }
         }
     }
-    for (uint32_t j = lane; j < f; j += 32) {
-        keys_state[(size_t)s * kTokMax + j] = K[j];
-        size_state[(size_t)s * kTokMax + j] = Z[j];
+    if (inreg) {
+        if (lane < f) {
+            keys_state[(size_t)s * kTokMax + lane] = kr;
+            cum_state[(size_t)s * kTokMax + lane] = cr;
+        }
+    } else {
+        for (uint32_t j = lane; j < f; j += 32) {
+            keys_state[(size_t)s * kTokMax + j] = K[j];
+            cum_state[(size_t)s * kTokMax + j] = Cm[j];
+        }
     }
     if (lane == 0) fill_state[s] = f;
+    for (int o = 16; o > 0; o >>= 1) c_prompt += __shfl_xor_sync(0xffffffffu, c_prompt, o);
     if (lane < caps.n_caps) {
         const uint32_t rep = s / R, r = s - rep * R;
         unsigned long long *C = ctr + (((unsigned long long)rep * caps.n_caps + lane) * R + r) * CR_CTR_FIELDS;
-        C[0] += c_req;
+        C[0] += i1 - i0;
         C[1] += c_hit;
         C[2] += c_hit_tok;
         C[3] += c_prompt;
-        C[4] += c_prefill;
+        C[4] += c_prompt - c_hit_tok;
     }
 }
 
@@ -726,7 +780,8 @@ extern "C" int cr_replay_create_tokens(cr_ctx *ctx, uint32_t n_rep, uint32_t R, 
     if (R == 0 || R > CR_MAX_R) return cr_fail(ctx, CR_EINVAL, "replay: R=%u", R);
     if (n_caps == 0 || n_caps > CR_MAX_CAPS) return cr_fail(ctx, CR_EINVAL, "replay: n_caps=%u", n_caps);
     for (uint32_t c = 0; c < n_caps; ++c)
-        if (token_caps[c] == 0) return cr_fail(ctx, CR_EINVAL, "replay: token capacity 0");
+        if (token_caps[c] == 0 || token_caps[c] > (1u << 31))
+            return cr_fail(ctx, CR_EINVAL, "replay: token capacity %u outside 1..2^31", token_caps[c]);
     if ((uint64_t)n_rep * R >= (1ull << 31)) return cr_fail(ctx, CR_EINVAL, "replay: too many streams");
     cr_replay *rp = (cr_replay *)calloc(1, sizeof(cr_replay));
     if (!rp) return cr_fail(ctx, CR_ENOMEM, "replay: host allocation failed");

@@ -563,7 +563,7 @@ def _fixed_len_stream(rng, n, nkeys, lo=16, hi=5000, spread=1.2):
 
 
 @pytest.mark.parametrize("caps,lo,hi", [([24576], 16, 5000), ([1, 100, 3000], 16, 5000),
-                                        ([4096, 65536, 2 ** 32 - 1], 16, 200),   # 1024-prefix bound
+                                        ([4096, 65536, 2 ** 31], 16, 200),       # 1024-prefix bound
                                         ([5000, 10 ** 6], 1, 3)])
 def test_token_replay_parity(P, ctx, caps, lo, hi):
     rng = np.random.default_rng(sum(caps) % 1000 + lo)
@@ -587,6 +587,26 @@ def test_token_replay_parity(P, ctx, caps, lo, hi):
     for rep in range(n_rep):
         for r in range(R):
             assert (rp.state(rep, r) == orp.state(rep, ci, r)).all()
+
+
+def test_token_replay_saturating_sums(P, ctx):
+    # prefixes near 2^31 tokens: sums past 2^32 saturate and are evicted like any over-capacity run
+    caps = [2 ** 31, 2 ** 30]
+    keys = np.array([1, 2, 1, 3, 4, 3, 2, 1, 1, 3, 4], np.uint64)
+    size = {1: 2 ** 30, 2: 2 ** 31 - 5, 3: 2 ** 31, 4: 2 ** 32 - 1}  # 3 then 4: 3's sum passes 2^32
+    plen = np.array([size[int(k)] for k in keys], np.uint32)
+    slen = np.zeros(keys.size, np.uint32)
+    dest = np.zeros((1, keys.size), np.uint16)
+    orp = O.Replay(1, 1, caps, tokens=True)
+    orp.step(keys, plen, slen, dest)
+    rp = P.Replay(ctx, 1, 1, caps, tokens=True)
+    ctr = torch.zeros((1, 2, 1, 5), dtype=torch.int64, device=DEV)
+    P.shadow_replay(ctx, rp, d_u64(keys), d_u32(plen), d_u32(slen), d_u16(dest), ctr)
+    ctx.sync()
+    assert (h_u64(ctr) == orp.ctr).all()
+    assert (rp.state(0, 0) == orp.state(0, 0, 0)).all()
+    with pytest.raises(P.CacheRouteError):
+        P.Replay(ctx, 1, 1, [2 ** 31 + 1], tokens=True)
 
 
 def test_token_replay_changed_length_is_reported(P, ctx):
