@@ -44,6 +44,8 @@ def parse_args(argv=None):
     ap.add_argument("--fresh-plans", action="store_true",
                     help="plan every interval from its own keys (the fresh plan of the replanning study) "
                          "instead of from the previous interval's")
+    ap.add_argument("--trace-seed", type=int, default=None,
+                    help="seed of the trace realisation (default: the configuration's); ranks add their rank")
     ap.add_argument("--token-lru", action="store_true",
                     help="replay with token-weighted LRU capacities (byte-aware variant)")
     ap.add_argument("--policies", default="",
@@ -65,6 +67,9 @@ def with_policies(cfg, args):
     """The configuration with --policies and --token-lru applied (unchanged without them)."""
     if getattr(args, "token_lru", False):
         cfg = cfg.token_lru()
+    if getattr(args, "trace_seed", None) is not None:
+        import dataclasses
+        cfg = dataclasses.replace(cfg, trace_seed=args.trace_seed)
     if not getattr(args, "policies", ""):
         return cfg
     import dataclasses

@@ -433,7 +433,7 @@ def test_replay_reset_and_bad_dest(P, ctx):
 # ------------------------------------------------------------------ pipeline ---
 @pytest.mark.parametrize("overlap", [False, True])
 @pytest.mark.parametrize("name,n,nint", [("tiny", 20000, 1), ("70b", 30000, 3), ("8b", 6000, 4),
-                                          ("burst", 30000, 2)])
+                                          ("burst", 30000, 2), ("70b-gamma", 30000, 3)])
 def test_pipeline_parity(P, ctx, name, n, nint, overlap):
     from paper_2608_19677_gb300.pipeline import Pipeline
     cfg = tg.CONFIGS[name]

@@ -147,3 +147,17 @@ def test_drift_generator_is_a_lognormal_walk():
         assert abs(np.mean(step ** 3)) < 0.01 * cfg.drift ** 3 * 10  # symmetric
         prev = cur
     assert all(abs(tr.shares(t).sum() - 1) < 1e-12 for t in range(cfg.n_intervals))
+
+
+def test_gamma_arrivals_have_the_configured_cv():
+    cfg = tg.CONFIGS["70b-gamma"]
+    tr = tg.Trace(cfg)
+    t = tr.arrival_times()
+    gaps = np.diff(t)
+    assert abs(gaps.std() / gaps.mean() - cfg.arrival_cv) < 0.02
+    assert t[0] >= 0 and t[-1] < cfg.n_intervals * cfg.interval_s
+    assert tr.counts.sum() == cfg.n_requests
+    assert np.array_equal(tr.counts, np.histogram(t, bins=cfg.n_intervals,
+                                                  range=(0, cfg.n_intervals * cfg.interval_s))[0])
+    # the Poisson configuration is unchanged by the option
+    assert tg.CONFIGS["70b"].arrival_cv is None

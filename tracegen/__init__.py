@@ -13,7 +13,9 @@ context that recurs, Poisson or bursty arrivals) at the sizes of the five
 synthetic configurations listed in ``CONFIGS``, plus a drift configuration
 for the replanning study (sec. 5 "Rate drift and remapping", supplement
 "Replanning Under Drift": the 70B-shaped key rates evolve for six intervals by
-a lognormal random walk with sigma = 0.3 per step).  The paper's de-identified
+a lognormal random walk with sigma = 0.3 per step), and a 70B variant whose
+arrivals are a Gamma renewal process with inter-arrival CV 1.9 (sec. 5
+"Arrival burstiness").  The paper's de-identified
 telemetry is not available; these seeded traces stand in for it.
 
 Token values come from a counter-based integer map (``token_values``) over
@@ -80,6 +82,7 @@ class TraceConfig:
     drift: Optional[float] = None  # sigma of a per-interval lognormal random walk of every key's rate
     token_caps: Optional[List[int]] = None  # LRU capacities in prefix tokens for the byte-aware replay
     lru_tokens: bool = False    # replay capacities (caps) count prefix tokens instead of prefixes
+    arrival_cv: Optional[float] = None  # Gamma renewal arrivals with this inter-arrival CV (else Poisson)
 
     @property
     def replicas(self) -> List[Tuple[str, int]]:
@@ -131,6 +134,11 @@ CONFIGS: Dict[str, TraceConfig] = {
         name="drift", R=30, n_keys=20_000, zipf_s=1.0, n_requests=1_000_000, n_intervals=6,
         interval_s=10.0, plen=("lognormal", 2048, 0.5, 16384), W=12, caps=[12],
         policies=["CR", "P2C"], seeds=[0, 1, 2, 3, 4], hot_cap=1.0 / 30, drift=0.3),
+    "70b-gamma": TraceConfig(
+        name="70b-gamma", R=30, n_keys=20_000, zipf_s=1.0, n_requests=2_000_000, n_intervals=12,
+        interval_s=10.0, plen=("lognormal", 2048, 0.5, 16384), W=12, caps=[12],
+        policies=["CR", "P2C", "RR", "HASH"], seeds=[0, 1, 2, 3, 4], hot_cap=1.0 / 30, token_caps=[24576],
+        arrival_cv=1.9),
     "large": TraceConfig(
         name="large", R=1024, n_keys=1_000_000, zipf_s=0.8, n_requests=64_000_000,
         n_intervals=60, interval_s=10.0, plen=("lognormal", 2048, 0.5, 32768), W=256,
@@ -218,6 +226,10 @@ class Trace:
         c = self.cfg
         rng = _rng(c.trace_seed, 0x41525256)  # "ARRV"
         secs = int(round(c.n_intervals * c.interval_s))
+        if c.arrival_cv:
+            t = self.arrival_times()
+            idx = np.minimum((t // c.interval_s).astype(np.int64), c.n_intervals - 1)
+            return np.bincount(idx, minlength=c.n_intervals).astype(np.int64)
         if c.burst is None:
             w = np.ones(c.n_intervals)
             return rng.multinomial(c.n_requests, w / w.sum()).astype(np.int64)
@@ -250,6 +262,17 @@ class Trace:
             cdf[-1] = 1.0
             self._drift_cdf[t] = cdf
         return self._drift_cdf[t]
+
+    def arrival_times(self) -> np.ndarray:
+        """Gamma renewal arrivals (configurations with ``arrival_cv``): n gaps of shape
+        1/CV^2 (so the gaps' coefficient of variation is arrival_cv), rescaled so the n
+        arrivals span the trace; seconds from the trace start."""
+        c = self.cfg
+        rng = _rng(c.trace_seed, 0x47414D41)  # "GAMA"
+        gaps = rng.gamma(1.0 / c.arrival_cv ** 2, 1.0, size=c.n_requests)
+        t = np.cumsum(gaps)
+        t *= (c.n_intervals * c.interval_s) / (t[-1] * (1.0 + 1e-12))
+        return t
 
     def interval(self, t: int) -> Interval:
         c = self.cfg
