@@ -11,6 +11,8 @@
 //              nested (Mattson et al. 1970): the cache of capacity c is the c
 //              most recent entries of any larger one.
 //   state      kept between calls as keys in recency order (most recent first).
+//   tokens     the byte-aware variant (cr_replay_create_tokens): capacities in
+//              prefix tokens, one warp walking each stream (k_lru_tokens).
 #include <stdlib.h>
 #include <string.h>
 

@@ -224,7 +224,6 @@ __device__ __forceinline__ const uint16_t *stage_aux(const route_desc &rd, uint1
     return sm;
 }
 
-// Sequential part: one CTA per load-dependent replica walks the batches.
 // One decision against the batch-start loads.  A bounded-load replica's
 // candidates are all RING; every other replica's are FIXED, PAIR or SET, so
 // the two cases are compiled apart.  m: requests in the load vector the batch
