@@ -41,6 +41,9 @@ def parse_args(argv=None):
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--config", default="70b")
     ap.add_argument("--batch", type=int, default=1024)
+    ap.add_argument("--graph", action="store_true",
+                    help="capture the whole step (every interval) once as a CUDA graph and replay it; stage "
+                         "times and the roofline then come from one ordinary step after the timed region")
     ap.add_argument("--fresh-plans", action="store_true",
                     help="plan every interval from its own keys (the fresh plan of the replanning study) "
                          "instead of from the previous interval's")
@@ -302,6 +305,8 @@ def main():
     cfg = replica_cfg(cfg, rank, world)  # independent replica per rank
     trace = tg.Trace(cfg)
     dev = torch.device("cuda", local)
+    if args.graph:  # graphs are captured on a stream of their own; torch's ops follow it
+        torch.cuda.set_stream(torch.cuda.Stream(dev))
     stream = torch.cuda.current_stream(dev)
 
     if args.intervals:
@@ -368,6 +373,18 @@ def main():
     ctx.sync()
     torch.cuda.synchronize()
 
+    # ---- optional CUDA graph of the whole step ---------------------------------
+    graph, graph_launches = None, 0
+    if args.graph:
+        pipe.quiesce()
+        graph = torch.cuda.CUDAGraph()
+        lc0 = launches()
+        with torch.cuda.graph(graph, stream=stream):
+            step()
+        graph_launches = launches() - lc0  # library launches in one replay
+        graph.replay()
+        torch.cuda.synchronize()
+
     # ---- timed region: K steps, stage events on the launching stream -------
     clocks = ClockSampler(local)
     clocks.start()
@@ -379,18 +396,29 @@ def main():
     ev1 = torch.cuda.Event(enable_timing=True)
     ev0.record(stream)
     for k in range(args.steps):
-        step(k)
+        if graph is not None:
+            graph.replay()
+        else:
+            step(k)
     ev1.record(stream)
     torch.cuda.synchronize()
     barrier()
-    n_launch = launches() - l0
-    stage_ms = np.zeros((args.steps, cfg.n_intervals, 4))
-    for k in range(args.steps):
+    n_launch = graph_launches * args.steps if graph is not None else launches() - l0
+    clk = clocks.stop()
+    if graph is not None:
+        # per-stage times and the hash roofline from one ordinary step after the timed region
+        pipe.quiesce()
+        step(0)
+        torch.cuda.synchronize()
+    marked = [0] if graph is not None else list(range(args.steps))
+    stage_ms = np.zeros((len(marked), cfg.n_intervals, 4))
+    for j, k in enumerate(marked):
         for i in range(cfg.n_intervals):
             m = marks[k][i]
             for s in range(4):
-                stage_ms[k, i, s] = m[s].elapsed_time(m[s + 1])
-    clk = clocks.stop()
+                stage_ms[j, i, s] = m[s].elapsed_time(m[s + 1])
+    hash_marks, plan_marks = [hash_marks[k] for k in marked], [plan_marks[k] for k in marked]
+    route_marks, replay_marks = [route_marks[k] for k in marked], [replay_marks[k] for k in marked]
     ctx.sync()
     ms_total = ev0.elapsed_time(ev1)
     ms = ms_total / args.steps
@@ -440,6 +468,10 @@ def main():
         "gpu_launches": int(n_launch),
         "clocks": clk,
     }
+    if graph is not None:
+        line["cuda_graph"] = ("the timed steps replay one CUDA graph of the whole step; stage times, plan-build "
+                              "times and the roofline come from one ordinary step after the timed region")
+        pipe.quiesce()
 
     # ---- replanning under drift (untimed study) ----------------------------
     if cfg.drift:
@@ -581,6 +613,16 @@ def run_keys_mode(args, cfg, trace, dev, stream, world, rank, barrier):
     for _ in range(max(args.warmup, 0)):
         step()
     pipe.sync()
+    graph, graph_launches = None, 0
+    if args.graph:
+        pipe.quiesce()
+        graph = torch.cuda.CUDAGraph()
+        lc0 = pipe.launches
+        with torch.cuda.graph(graph, stream=stream):
+            step()
+        graph_launches = pipe.launches - lc0
+        graph.replay()
+        torch.cuda.synchronize()
     clocks = ClockSampler(dev.index or 0)
     clocks.start()
     time.sleep(0.3)
@@ -591,21 +633,30 @@ def run_keys_mode(args, cfg, trace, dev, stream, world, rank, barrier):
     ev1 = torch.cuda.Event(enable_timing=True)
     ev0.record(stream)
     for k in range(args.steps):
-        step(k)
+        if graph is not None:
+            graph.replay()
+        else:
+            step(k)
     ev1.record(stream)
     torch.cuda.synchronize()
     barrier()
-    n_launch = pipe.launches - l0
+    n_launch = graph_launches * args.steps if graph is not None else pipe.launches - l0
     clk = clocks.stop()
+    if graph is not None:  # stage and plan times from one ordinary step after the timed region
+        pipe.quiesce()
+        step(0)
     pipe.sync()
     ms = ev0.elapsed_time(ev1) / args.steps
     ms_max = max_over_ranks(ms, world, dev)
-    stage = np.zeros((args.steps, cfg.n_intervals, 4))
-    for k in range(args.steps):
+    marked = [0] if graph is not None else list(range(args.steps))
+    plan_marks = [plan_marks[k] for k in marked]
+    route_marks, replay_marks = [route_marks[k] for k in marked], [replay_marks[k] for k in marked]
+    stage = np.zeros((len(marked), cfg.n_intervals, 4))
+    for j, k in enumerate(marked):
         for t in range(cfg.n_intervals):
             m = marks[k][t]
             for s_ in range(4):
-                stage[k, t, s_] = m[s_].elapsed_time(m[s_ + 1])
+                stage[j, t, s_] = m[s_].elapsed_time(m[s_ + 1])
     plan_ms = np.array([[a.elapsed_time(b) for a, b in pm] for pm in plan_marks])
     # route and replay calls timed on their own streams, after their waits
     route_ms = float(np.array([[a.elapsed_time(b) for a, b in rm] for rm in route_marks]).sum(1).mean())
@@ -651,6 +702,9 @@ def run_keys_mode(args, cfg, trace, dev, stream, world, rank, barrier):
         "main_wait_for_plans_ms_per_step": float((stage[:, :, 0] + stage[:, :, 1]).sum(1).mean()),
         "gpu_launches": int(n_launch), "clocks": clk,
     }
+    if graph is not None:
+        line["cuda_graph"] = ("the timed steps replay one CUDA graph of the whole step; stage, route, replay "
+                              "and plan-build times come from one ordinary step after the timed region")
     if rank == 0:
         print(json.dumps(line), flush=True)
     if world > 1:

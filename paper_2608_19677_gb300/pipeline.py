@@ -267,6 +267,16 @@ class Pipeline:
             self._pbuf = cur ^ 1
         return keys
 
+    def quiesce(self):
+        """Wait for all enqueued work and forget the events that ordered it, so the next
+        interval waits on nothing recorded before (e.g. before capturing a CUDA graph)."""
+        self.sync()
+        self._released = [[] for _ in range(NKEYS)]
+        self._dest_free = [None, None]
+        self._ready = [None, None]
+        self._next_built = False
+        self.inputs_free = None
+
     def finish(self):
         """Make the main stream wait for every other stream's enqueued work."""
         if self.overlap:

@@ -644,3 +644,43 @@ def test_pipeline_parity_token_lru(P, ctx, name, n, nint):
                       plan_next=t + 1 < cfg.n_intervals)
     pipe.sync()
     assert (h_u64(pipe.ctr) == ref["ctr"]).all()
+
+
+@pytest.mark.parametrize("name,n,nint", [("8b", 6000, 5), ("70b", 30000, 3)])
+def test_pipeline_cuda_graph_replay(P, ctx, name, n, nint):
+    # a whole step captured once as a CUDA graph (planner and replay streams joined through
+    # events) gives the counters of the ordinary step, replay after replay
+    from paper_2608_19677_gb300.pipeline import Pipeline
+    cfg = tg.CONFIGS[name].scaled(n, nint)
+    tr = tg.Trace(cfg)
+    ref = OP.run_trace(tr, B=1024)
+    s = torch.cuda.Stream(DEV)
+    with torch.cuda.stream(s):
+        gctx = P.Context(0, s)
+        ins = []
+        for t in range(cfg.n_intervals):
+            iv = tr.interval(t)
+            tok, off = tg.arena_host(tr, iv, 4)
+            ins.append((t, torch.from_numpy(tok).to(DEV), d_u64(off), d_u32(iv.plen), d_u32(iv.slen), iv.g0))
+        pipe = Pipeline(gctx, cfg.R, cfg.W, cfg.caps, cfg.replicas, tr.qcap, batch_B=1024, overlap=True,
+                        max_n=max(int(x[2].shape[0]) for x in ins))
+
+        def step():
+            pipe.reset()
+            for i, (t, tok, off, pl, sl, g0) in enumerate(ins):
+                pipe.interval(t, tok, off, pl, sl, g0, plan_next=i + 1 < len(ins))
+            pipe.finish()
+
+        step()
+        torch.cuda.synchronize()
+        assert (h_u64(pipe.ctr) == ref["ctr"]).all()
+        pipe.quiesce()
+        graph = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(graph, stream=s):
+            step()
+        for _ in range(2):
+            pipe.ctr.fill_(-1)
+            graph.replay()
+            torch.cuda.synchronize()
+            assert (h_u64(pipe.ctr) == ref["ctr"]).all()
+    gctx.sync()
