@@ -187,7 +187,7 @@ def oracle_sample(trace, n_intervals: int = 1, B: int = 1024):
     import tracegen as tg
     cfg = trace.cfg
     reps = cfg.replicas
-    pols = [p for p, _ in reps]
+    pols = [OP.ROUTE_AS.get(p, p) for p, _ in reps]
     seeds = [s for _, s in reps]
     rp = O.Replay(len(reps), cfg.R, cfg.caps, tokens=cfg.lru_tokens)
     rings = OP.rings_for(cfg)
@@ -220,7 +220,7 @@ def run_reference(args):
     iv = trace.interval(0)
     tok, off = tg.arena_host(trace, iv, 4)
     reps = cfg.replicas
-    pols = [p for p, _ in reps]
+    pols = [OP.ROUTE_AS.get(p, p) for p, _ in reps]
     seeds = [s for _, s in reps]
     rings = OP.rings_for(cfg)
 

@@ -71,6 +71,8 @@ extern "C" {
 #define CR_VARIANT_LPT 0    /* Algorithm 1 as printed                            */
 #define CR_VARIANT_RANDOM 1 /* Eq. 1 replica counts, random distinct placement  */
 #define CR_VARIANT_NOREPL 2 /* k_b = 1 for every key, LPT placement              */
+#define CR_VARIANT_SLOTCAP 3 /* LPT with at most W replicas per destination; a key
+                                gets min(k_b, destinations with a free slot)       */
 
 /* ---- limits --------------------------------------------------------------- */
 #define CR_MAX_R 8192         /* destinations per plan / route call              */

@@ -45,7 +45,7 @@ _SRC = os.path.join(_HERE, "cr_oracle.c")
 _LIB = os.path.join(_HERE, "libcr_oracle.so")
 
 CTR_FIELDS = ("requests", "hits", "hit_tokens", "prompt_tokens", "prefill_tokens")
-VARIANT = {"LPT": 0, "RANDOM": 1, "NOREPL": 2}
+VARIANT = {"LPT": 0, "RANDOM": 1, "NOREPL": 2, "SLOTCAP": 3}
 POLICY = {"CR": 0, "CR_NOLPT": 1, "CR_NOREPL": 2, "P2C": 3, "RR": 4, "HASH": 5, "CHWBL": 6}
 
 

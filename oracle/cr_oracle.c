@@ -158,7 +158,7 @@ uint64_t orc_histogram(const uint64_t *key, uint64_t n, uint64_t *ukey, uint64_t
 /* a3..a6: the plan (Eq. 1 and Algorithm 1)                                */
 /* ---------------------------------------------------------------------- */
 
-enum { ORC_VARIANT_LPT = 0, ORC_VARIANT_RANDOM = 1, ORC_VARIANT_NOREPL = 2 };
+enum { ORC_VARIANT_LPT = 0, ORC_VARIANT_RANDOM = 1, ORC_VARIANT_NOREPL = 2, ORC_VARIANT_SLOTCAP = 3 };
 enum { ORC_CR = 0, ORC_CR_NOLPT = 1, ORC_CR_NOREPL = 2, ORC_P2C = 3, ORC_RR = 4, ORC_HASH = 5, ORC_CHWBL = 6 };
 
 typedef struct {
@@ -209,7 +209,7 @@ uint32_t orc_kb(uint64_t lambda, uint64_t num, uint64_t den, uint32_t R)
 int orc_build_plan(const uint64_t *key, uint64_t n, const orc_plan_params *p, orc_plan *out)
 {
     if (!p || !out || p->R == 0 || p->R > 65535 || p->W == 0 || p->qcap_num == 0 ||
-        p->qcap_den == 0 || p->qcap_den >= (1ULL << 32) || n >= (1ULL << 32) || p->variant > 2)
+        p->qcap_den == 0 || p->qcap_den >= (1ULL << 32) || n >= (1ULL << 32) || p->variant > 3)
         return ORC_EINVAL;
     const uint32_t R = p->R;
     const uint64_t C = (uint64_t)R * p->W;
@@ -248,8 +248,15 @@ int orc_build_plan(const uint64_t *key, uint64_t n, const orc_plan_params *p, or
     for (uint32_t r = 0; r < R; ++r)
         out->load[r] = p->init_load ? p->init_load[r] : cold / R;
 
-    /* placement, in admission (decreasing-rate) order */
+    /* placement, in admission (decreasing-rate) order.  Slot-capped variant
+     * (per-destination byte budget, this library's reading): a destination
+     * holds at most W replicas; a key goes to the k smallest (L[r], r) among
+     * destinations with a free slot, k = min(k_b, such destinations), so it
+     * may get fewer replicas than Eq. 1 asks, or none (then T has no entry
+     * for it and it is routed like a key that was not admitted). */
     uint8_t *taken = (uint8_t *)calloc(R, 1);
+    uint32_t *slots = (uint32_t *)calloc(R, sizeof(uint32_t));
+    uint64_t placed = 0;
     uint32_t *chosen = (uint32_t *)malloc(R * sizeof(uint32_t));
     uint32_t *perm = (uint32_t *)malloc(R * sizeof(uint32_t));
     uint32_t pos = 0;
@@ -257,6 +264,16 @@ int orc_build_plan(const uint64_t *key, uint64_t n, const orc_plan_params *p, or
         uint32_t k = out->adm_k[a];
         uint64_t lam = out->adm_cnt[a];
         out->koff[a] = pos;
+        if (p->variant == ORC_VARIANT_SLOTCAP) {
+            uint32_t free_dest = 0;
+            for (uint32_t r = 0; r < R; ++r)
+                free_dest += slots[r] < p->W;
+            if (k > free_dest)
+                k = free_dest;
+            out->adm_k[a] = k;
+            if (k == 0)
+                continue;
+        }
         if (p->variant == ORC_VARIANT_RANDOM) {
             /* k distinct destinations in uniformly random order: the first k
              * steps of a Fisher-Yates shuffle of 0..R-1, step s swapping slot s
@@ -278,7 +295,7 @@ int orc_build_plan(const uint64_t *key, uint64_t n, const orc_plan_params *p, or
             for (uint32_t s = 0; s < k; ++s) {
                 int64_t best = -1;
                 for (uint32_t r = 0; r < R; ++r) {
-                    if (taken[r])
+                    if (taken[r] || (p->variant == ORC_VARIANT_SLOTCAP && slots[r] >= p->W))
                         continue;
                     if (best < 0 || out->load[r] < out->load[best])
                         best = r;
@@ -295,14 +312,17 @@ int orc_build_plan(const uint64_t *key, uint64_t n, const orc_plan_params *p, or
             out->jobs[pos + s] = job;
             out->load[chosen[s]] += job;
             taken[chosen[s]] = 0;
+            slots[chosen[s]] += 1;
         }
         pos += k;
+        placed += k;
     }
     out->koff[n_adm] = pos;
     out->U = U;
     out->n_adm = n_adm;
-    out->sum_k = sum;
+    out->sum_k = p->variant == ORC_VARIANT_SLOTCAP ? placed : sum;
     out->cold = cold;
+    free(slots);
     free(taken);
     free(chosen);
     free(perm);

@@ -24,7 +24,8 @@ import numpy as np
 import tracegen as tg
 from . import Replay, Ring, build_plan, hash_prefixes, route
 
-VARIANT_OF = {"CR": "LPT", "CR_NOLPT": "RANDOM", "CR_NOREPL": "NOREPL"}
+VARIANT_OF = {"CR": "LPT", "CR_NOLPT": "RANDOM", "CR_NOREPL": "NOREPL", "CR_SLOTCAP": "SLOTCAP"}
+ROUTE_AS = {"CR_SLOTCAP": "CR"}  # routed as CacheRoute on the slot-capped plan
 
 
 def plans_for_interval(trace: tg.Trace, plan_keys: np.ndarray, t: int):
@@ -56,7 +57,7 @@ def run_trace(trace: tg.Trace, intervals: Optional[Iterable[int]] = None, align:
     """Run the protocol; returns a dict with the counters (and per-interval data if keep)."""
     cfg = trace.cfg
     reps = cfg.replicas
-    pols = [p for p, _ in reps]
+    pols = [ROUTE_AS.get(p, p) for p, _ in reps]
     seeds = [s for _, s in reps]
     rp = Replay(len(reps), cfg.R, cfg.caps, tokens=cfg.lru_tokens)
     rings = rings_for(cfg)

@@ -29,7 +29,7 @@ CR_OK, CR_EINVAL, CR_ENOMEM, CR_ECUDA, CR_ETIMEOUT, CR_EOVERFLOW = range(6)
 STATUS_NAMES = {0: "CR_OK", 1: "CR_EINVAL", 2: "CR_ENOMEM", 3: "CR_ECUDA", 4: "CR_ETIMEOUT",
                 5: "CR_EOVERFLOW"}
 POLICY = {"CR": 0, "CR_NOLPT": 1, "CR_NOREPL": 2, "P2C": 3, "RR": 4, "HASH": 5, "CHWBL": 6}
-VARIANT = {"LPT": 0, "RANDOM": 1, "NOREPL": 2}
+VARIANT = {"LPT": 0, "RANDOM": 1, "NOREPL": 2, "SLOTCAP": 3}
 MAX_R, MAX_CAP, MAX_CAPS, MAX_REPLICAS, CTR_FIELDS, MAX_VNODES = 8192, 1024, 8, 256, 5, 1024
 
 # every symbol the header declares (checked by the CPU test suite)

@@ -739,6 +739,106 @@ __global__ void __launch_bounds__(32) k_plan_lpt(const cr_plan_info_dev *info,
     if (__any_sync(0xffffffffu, overflow) && lane == 0) atomicOr(status, CR_FLAG_OVERFLOW);
 }
 
+// Slot-capped LPT (per-destination budget of W replicas; this library's
+// reading of a byte-aware placement): as k_plan_lpt, but a destination that
+// holds W replicas is no longer eligible, and a key gets
+// k = min(k_b, destinations with a free slot) replicas (at least one: the
+// aggregate admission leaves a free slot for every admitted key).  Member
+// offsets are written compactly, adm_k receives the placed counts and
+// info->sum_k their sum.
+__device__ __forceinline__ unsigned long long lane_min_capped(const unsigned long long *L,
+                                                              const unsigned char *taken, const uint32_t *slots,
+                                                              uint32_t W, uint32_t R, uint32_t lane)
+{
+    unsigned long long m = ~0ull;
+    for (uint32_t r = lane; r < R; r += 32) {
+        if (taken[r] || slots[r] >= W) continue;
+        const unsigned long long v = (L[r] << 16) | r;
+        m = v < m ? v : m;
+    }
+    return m;
+}
+
+__global__ void __launch_bounds__(32) k_plan_lpt_capped(cr_plan_info_dev *info,
+                                                        const unsigned long long *__restrict__ adm_cnt,
+                                                        uint32_t *__restrict__ adm_k, uint32_t *__restrict__ koff,
+                                                        uint32_t R, uint32_t W, unsigned long long *__restrict__ load_g,
+                                                        uint16_t *__restrict__ members,
+                                                        unsigned long long *__restrict__ jobs, uint32_t *status)
+{
+    extern __shared__ unsigned long long smem_u64[];
+    unsigned long long *L = smem_u64;                                      // [R]
+    uint32_t *slots = reinterpret_cast<uint32_t *>(L + R);                 // [R] replicas held
+    unsigned char *taken = reinterpret_cast<unsigned char *>(slots + R);   // [R]
+    const uint32_t lane = cr_lane();
+    for (uint32_t r = lane; r < R; r += 32) {
+        L[r] = load_g[r];
+        slots[r] = 0;
+        taken[r] = 0;
+    }
+    __syncwarp();
+    unsigned long long m = lane_min_capped(L, taken, slots, W, R, lane);
+    const unsigned long long na = info->n_adm;
+    uint32_t free_dest = R;  // destinations with a free slot (uniform over the warp)
+    uint32_t pos = 0;        // compact member offset
+    bool overflow = false;
+    unsigned long long st_lam = 0;
+    uint32_t st_k = 0;
+    for (unsigned long long a = 0; a < na; ++a) {
+        const uint32_t slot = (uint32_t)(a & 31ull);
+        if (slot == 0) {
+            const unsigned long long ia = a + lane;
+            if (ia < na) {
+                st_lam = adm_cnt[ia];
+                st_k = adm_k[ia];
+            }
+        }
+        const uint32_t kb = __shfl_sync(0xffffffffu, st_k, slot);
+        const unsigned long long lam = __shfl_sync(0xffffffffu, st_lam, slot);
+        const uint32_t k = kb < free_dest ? kb : free_dest;
+        if (lane == 0) {
+            koff[a] = pos;
+            adm_k[a] = k;
+        }
+        if (k == 0) continue;
+        const unsigned long long q = lam / k, rem = lam % k;
+        bool took = false;
+        for (uint32_t s = 0; s < k; ++s) {
+            const unsigned long long best = warp_min_u64(m);
+            const uint32_t br = (uint32_t)(best & 0xffffu);
+            const unsigned long long job = q + (s < rem ? 1ull : 0ull);
+            if (lane == 0) {
+                members[pos + s] = (uint16_t)br;
+                jobs[pos + s] = job;
+            }
+            bool filled = false;
+            if ((br & 31u) == lane) {
+                if (k > 1) {
+                    taken[br] = 1;
+                    took = true;
+                }
+                const unsigned long long nl = L[br] + job;
+                if (nl >= kLoadLimit) overflow = true;
+                L[br] = nl;
+                filled = ++slots[br] == W;
+                m = lane_min_capped(L, taken, slots, W, R, lane);
+            }
+            free_dest -= __shfl_sync(0xffffffffu, filled ? 1u : 0u, br & 31u);
+        }
+        if (took) {  // release this key's destinations for the next key
+            for (uint32_t r = lane; r < R; r += 32) taken[r] = 0;
+            m = lane_min_capped(L, taken, slots, W, R, lane);
+        }
+        pos += k;
+    }
+    if (lane == 0) {
+        koff[na] = pos;
+        info->sum_k = pos;
+    }
+    for (uint32_t r = lane; r < R; r += 32) load_g[r] = L[r];
+    if (__any_sync(0xffffffffu, overflow) && lane == 0) atomicOr(status, CR_FLAG_OVERFLOW);
+}
+
 // LPT for R <= 32: lane i holds the i-th smallest packed key (L << 16 | r), so
 // T(b) for a key with k_b = k is lanes 0..k-1.  After a single-copy job the
 // grown key is re-inserted with one ballot and one shuffle; after a replicated
@@ -1199,6 +1299,7 @@ __device__ __forceinline__ void table_body(const cr_plan_info_dev *info, const u
     const unsigned long long na = info->n_adm;
     const unsigned long long mask = (1ull << bits) - 1ull;
     for (uint64_t a = (uint64_t)blockIdx.x * blockDim.x + threadIdx.x; a < na; a += (uint64_t)gridDim.x * blockDim.x) {
+        if (adm_k[a] == 0) continue;  // a key placed on no destination has no entry
         const unsigned long long key = adm_key[a];
         unsigned long long s = key >> (64 - bits);
         for (;;) {
@@ -1359,7 +1460,7 @@ static int check_params(cr_ctx *ctx, const cr_plan_params *pp)
     if ((uint64_t)pp->R * pp->W >= 0xffffffffull) return cr_fail(ctx, CR_EINVAL, "plan: C = R*W must be < 2^32-1");
     if (pp->qcap_num == 0 || pp->qcap_den == 0 || pp->qcap_den >= (1ull << 32))
         return cr_fail(ctx, CR_EINVAL, "plan: q_cap needs num >= 1 and 1 <= den < 2^32");
-    if (pp->variant > CR_VARIANT_NOREPL || pp->reserved != 0)
+    if (pp->variant > CR_VARIANT_SLOTCAP || pp->reserved != 0)
         return cr_fail(ctx, CR_EINVAL, "plan: bad variant %u or reserved field", pp->variant);
     return CR_OK;
 }
@@ -1549,7 +1650,14 @@ extern "C" int cr_build_plans(cr_ctx *ctx, const uint64_t *d_key, uint64_t n, co
             J.seed = pp.seed;
             J.epoch = pp.epoch;
             J.R = pp.R;
-            if (pp.variant == CR_VARIANT_RANDOM) {
+            if (pp.variant == CR_VARIANT_SLOTCAP) {
+                const size_t smem = (size_t)pp.R * (sizeof(unsigned long long) + sizeof(uint32_t) + 1) + 16;
+                if (smem > 48 * 1024)
+                    CR_CUDA(ctx, cudaFuncSetAttribute(k_plan_lpt_capped, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                                      (int)smem));
+                CR_LAUNCH(ctx, k_plan_lpt_capped, 1, 32, smem, p->d_info, (const unsigned long long *)p->d_adm_cnt,
+                          p->d_adm_k, p->d_koff, pp.R, pp.W, p->d_load, p->d_members, p->d_jobs, ctx->d_status);
+            } else if (pp.variant == CR_VARIANT_RANDOM) {
                 rj.j[nr++] = J;
                 rmaxR = pp.R > rmaxR ? pp.R : rmaxR;
                 radm = (n < C ? n : C) > radm ? (n < C ? n : C) : radm;
@@ -1636,7 +1744,14 @@ extern "C" int cr_build_plans(cr_ctx *ctx, const uint64_t *d_key, uint64_t n, co
         CR_LAUNCH(ctx, k_plan_init_load, cr_blocks(pp.R, 256, gcap), 256, 0, p->d_info,
                   (const unsigned long long *)pp.d_init_load, pp.R, p->d_load, ctx->d_status);
         if (n > 0) {
-            if (pp.variant == CR_VARIANT_RANDOM) {
+            if (pp.variant == CR_VARIANT_SLOTCAP) {
+                const size_t smem = (size_t)pp.R * (sizeof(unsigned long long) + sizeof(uint32_t) + 1) + 16;
+                if (smem > 48 * 1024)
+                    CR_CUDA(ctx, cudaFuncSetAttribute(k_plan_lpt_capped, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                                      (int)smem));
+                CR_LAUNCH(ctx, k_plan_lpt_capped, 1, 32, smem, p->d_info, (const unsigned long long *)p->d_adm_cnt,
+                          p->d_adm_k, p->d_koff, pp.R, pp.W, p->d_load, p->d_members, p->d_jobs, ctx->d_status);
+            } else if (pp.variant == CR_VARIANT_RANDOM) {
                 size_t smem = (size_t)kRandWarps * pp.R * sizeof(uint16_t);
                 if (smem > 48 * 1024)
                     CR_CUDA(ctx, cudaFuncSetAttribute(k_plan_random, cudaFuncAttributeMaxDynamicSharedMemorySize,

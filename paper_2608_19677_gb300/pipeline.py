@@ -34,7 +34,9 @@ from typing import Callable, List, Optional, Sequence, Tuple
 from . import (Context, Plan, Replay, Ring, build_plans, hash_prefixes, plan_params, route_batch,
                shadow_replay)
 
-VARIANT_OF = {"CR": "LPT", "CR_NOLPT": "RANDOM", "CR_NOREPL": "NOREPL"}
+VARIANT_OF = {"CR": "LPT", "CR_NOLPT": "RANDOM", "CR_NOREPL": "NOREPL", "CR_SLOTCAP": "SLOTCAP"}
+# CacheRoute on a slot-capped plan routes as CacheRoute (same fallback draws as CR, seed for seed)
+ROUTE_AS = {"CR_SLOTCAP": "CR"}
 NKEYS = 3
 
 
@@ -238,8 +240,8 @@ class Pipeline:
         dest = D[:, :n] if n == D.shape[1] else D.view(-1)[:len(self.replicas) * n].view(len(self.replicas), n)
         plans = [self.plans[cur][i] if i is not None else None for i in self.rep_plan]
         r0 = self._event(self.mstream, True) if mark else None
-        route_batch(self.ctx, plans, self.policies, self.seeds, self.R, keys, g0, self.B, self.load, dest,
-                    rings=self.rings)
+        route_batch(self.ctx, plans, [ROUTE_AS.get(p, p) for p in self.policies], self.seeds, self.R, keys, g0,
+                    self.B, self.load, dest, rings=self.rings)
         if mark:
             marks[3].record(self.mstream)
             self.route_marks.append((r0, marks[3]))

@@ -126,11 +126,12 @@ def test_plan_parity(P, ctx, seed):
     keys = _rates_keys(rng, nkeys, int(rng.integers(nkeys, 60000)))
     n = keys.size
     num, den = (5 * n, 4 * R) if seed % 2 == 0 else (n, 9 * R)
-    plans = [P.Plan(ctx) for _ in range(3)]
-    params = [P.plan_params(R, W, num, den, v, seed=seed, epoch=3) for v in ("LPT", "RANDOM", "NOREPL")]
+    variants = ("LPT", "RANDOM", "NOREPL", "SLOTCAP")
+    plans = [P.Plan(ctx) for _ in variants]
+    params = [P.plan_params(R, W, num, den, v, seed=seed, epoch=3) for v in variants]
     P.build_plans(ctx, d_u64(keys), params, plans)
     uk, uc = O.histogram(keys)
-    for pl, v in zip(plans, ("LPT", "RANDOM", "NOREPL")):
+    for pl, v in zip(plans, variants):
         got = pl.export()
         assert (got["ukey"] == uk).all() and (got["ucnt"] == uc).all()
         _cmp_plan(got, O.build_plan(keys, R, W, num, den, variant=v, seed=seed, epoch=3))
@@ -684,3 +685,42 @@ def test_pipeline_cuda_graph_replay(P, ctx, name, n, nint):
             torch.cuda.synchronize()
             assert (h_u64(pipe.ctr) == ref["ctr"]).all()
     gctx.sync()
+
+
+# ------------------------------------------------------------------ f3 slot-capped placement ---
+@pytest.mark.parametrize("R,W,nkeys,total,skew", [(2, 2, 4, 127, 0), (30, 3, 3000, 60000, 1),
+                                                  (300, 2, 20000, 700000, 1), (1024, 4, 60000, 300000, 0),
+                                                  (3000, 1, 5000, 40000, 1)])
+def test_plan_parity_slotcap(P, ctx, R, W, nkeys, total, skew):
+    # the capped LPT against the oracle, on the one-CTA build and on the device-wide build
+    # (700,000 requests), with and without a skewed starting load (which trims replica counts)
+    rng = np.random.default_rng(R + W)
+    keys = _rates_keys(rng, nkeys, total)
+    n = keys.size
+    init = None
+    if skew:
+        init = rng.integers(0, 50, R).astype(np.uint64)
+        init[: max(1, R // 4)] += np.uint64(10 ** 6)
+    for num, den in ((5 * n, 4 * R), (n, 20 * R)):
+        dl = d_u64(init) if init is not None else None
+        got = P.build_plan(ctx, d_u64(keys), P.plan_params(R, W, num, den, "SLOTCAP", init_load=dl)).export()
+        ref = O.build_plan(keys, R, W, num, den, variant="SLOTCAP", init_load=init)
+        _cmp_plan(got, ref)
+        assert np.bincount(got["members"].astype(np.int64), minlength=R).max() <= W
+
+
+def test_pipeline_parity_slotcap_policy(P, ctx):
+    import dataclasses
+    from paper_2608_19677_gb300.pipeline import Pipeline
+    cfg = dataclasses.replace(tg.CONFIGS["8b"].scaled(8000, 4), policies=["CR", "CR_SLOTCAP", "P2C"], seeds=[0, 1])
+    tr = tg.Trace(cfg)
+    ref = OP.run_trace(tr, B=1024, keep=True)
+    pipe = Pipeline(ctx, cfg.R, cfg.W, cfg.caps, cfg.replicas, tr.qcap, batch_B=1024, overlap=True)
+    for t in range(cfg.n_intervals):
+        iv = tr.interval(t)
+        tok, off = tg.arena_host(tr, iv, 4)
+        pipe.interval(t, torch.from_numpy(tok).to(DEV), d_u64(off), d_u32(iv.plen), d_u32(iv.slen), iv.g0,
+                      plan_next=t + 1 < cfg.n_intervals)
+        assert (h_u16(pipe.last_dest) == ref["dest"][t]).all()
+    pipe.sync()
+    assert (h_u64(pipe.ctr) == ref["ctr"]).all()
