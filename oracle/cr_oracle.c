@@ -22,7 +22,8 @@
  *   orc_build_plan ................... Eq. 1 (k_b), warm-set admission
  *       (sec. 3.1 "Warm-set admission", Algorithm 1 admission step), cold-tail
  *       initialisation and LPT placement (sec. 3.1 "Placement and dispatch",
- *       Algorithm 1 placement loop).
+ *       Algorithm 1 placement loop); random, single-copy and slot-capped
+ *       (per-destination budget, this library's reading) variants.
  *   orc_route ........................ dispatch (Fig. 1; sec. 3.1: least-loaded
  *       member of T(b), otherwise power-of-two choices over the fleet) and the
  *       comparison policies of sec. 4 (Flat-LB, sticky hashing, consistent
