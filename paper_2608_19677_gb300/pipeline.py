@@ -269,6 +269,15 @@ class Pipeline:
             self._pbuf = cur ^ 1
         return keys
 
+    def wait_last(self):
+        """Make torch's current stream wait for everything enqueued so far on the
+        pipeline's streams, so that ``last_dest`` and the counters can be read on it
+        whatever stream the caller uses; the host does not block."""
+        import torch
+        cur = torch.cuda.current_stream(self.dev)
+        for st in (self.mstream, self.pstream, self.ystream):
+            cur.wait_event(self._event(st))
+
     def quiesce(self):
         """Wait for all enqueued work and forget the events that ordered it, so the next
         interval waits on nothing recorded before (e.g. before capturing a CUDA graph)."""

@@ -63,6 +63,7 @@ def test_fullsize_two_intervals(P, name):
         slen = torch.from_numpy(iv.slen.view(np.int32)).to(DEV)
         keys = pipe.interval(t, tok, off, plen, slen, iv.g0, plan_next=t + 1 < nint)
         dkeys.append(keys.cpu().numpy().view(np.uint64).copy())
+        pipe.wait_last()
         dests.append(pipe.last_dest.cpu().numpy().view(np.uint16).copy())
         plans_used.append([pl.export() for pl in pipe.last_plans])
         del tok, off

@@ -451,6 +451,7 @@ def test_pipeline_parity(P, ctx, name, n, nint, overlap):
             keys = pipe.interval(t, torch.from_numpy(tok).to(DEV), d_u64(off), d_u32(iv.plen), d_u32(iv.slen),
                                  iv.g0, plan_next=t + 1 < cfg.n_intervals)
             assert (h_u64(keys) == ref["keys"][t]).all()
+            pipe.wait_last()
             assert (h_u16(pipe.last_dest) == ref["dest"][t]).all()
             # the plans the interval was routed with equal the oracle's
             for (v, s), pl in zip(pipe.plan_keys, pipe.last_plans):
@@ -478,6 +479,7 @@ def test_pipeline_parity_bounded_load_and_small_batches(P, ctx, B):
         tok, off = tg.arena_host(tr, iv, 4)
         pipe.interval(t, torch.from_numpy(tok).to(DEV), d_u64(off), d_u32(iv.plen), d_u32(iv.slen), iv.g0,
                       plan_next=t + 1 < cfg.n_intervals)
+        pipe.wait_last()
         assert (h_u16(pipe.last_dest) == ref["dest"][t]).all()
     pipe.sync()
     assert (h_u64(pipe.ctr) == ref["ctr"]).all()
@@ -546,6 +548,7 @@ def test_pipeline_parity_drift_fresh_and_stale(P, ctx, fresh):
         tok, off = tg.arena_host(tr, iv, 4)
         pipe.interval(t, torch.from_numpy(tok).to(DEV), d_u64(off), d_u32(iv.plen), d_u32(iv.slen), iv.g0,
                       plan_next=t + 1 < cfg.n_intervals)
+        pipe.wait_last()
         assert (h_u16(pipe.last_dest) == ref["dest"][t]).all()
         for (v, s), pl in zip(pipe.plan_keys, pipe.last_plans):
             got = pl.export()
@@ -721,6 +724,7 @@ def test_pipeline_parity_slotcap_policy(P, ctx):
         tok, off = tg.arena_host(tr, iv, 4)
         pipe.interval(t, torch.from_numpy(tok).to(DEV), d_u64(off), d_u32(iv.plen), d_u32(iv.slen), iv.g0,
                       plan_next=t + 1 < cfg.n_intervals)
+        pipe.wait_last()
         assert (h_u16(pipe.last_dest) == ref["dest"][t]).all()
     pipe.sync()
     assert (h_u64(pipe.ctr) == ref["ctr"]).all()
