@@ -235,8 +235,10 @@ typedef struct {
 /* Blocking: compare two built plans with the same R (device kernels: one warp
  * per admitted key, member sets compared through per-warp bitmaps of R bits;
  * histograms through per-plan hash tables in context scratch, 32 bytes per
- * request of the larger build); *out receives the counts.  Errors: CR_EINVAL
- * (plan not built, R differs), CR_ENOMEM, CR_ECUDA. */
+ * request of the larger build); *out receives the counts.  The kernels run on
+ * ctx's stream: plans built through another context must be complete first
+ * (e.g. cr_sync on that context).  Errors: CR_EINVAL (plan not built, R
+ * differs), CR_ENOMEM, CR_ECUDA. */
 CR_API int cr_plan_diff(cr_ctx *ctx, const cr_plan *a, const cr_plan *b, cr_plan_diff_counts *out);
 
 /* ==== a7: batched dispatch ========================================== */
