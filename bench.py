@@ -41,6 +41,9 @@ def parse_args(argv=None):
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--config", default="70b")
     ap.add_argument("--batch", type=int, default=1024)
+    ap.add_argument("--sm-split", type=int, default=0,
+                    help="run hashing and candidates on all but N SMs and the load-dependent route resolution on "
+                         "the other N (green contexts), so that it overlaps the next interval's hashing")
     ap.add_argument("--graph", action="store_true",
                     help="capture the whole step (every interval) once as a CUDA graph and replay it; stage "
                          "times and the roofline then come from one ordinary step after the timed region")
@@ -305,9 +308,14 @@ def main():
     cfg = replica_cfg(cfg, rank, world)  # independent replica per rank
     trace = tg.Trace(cfg)
     dev = torch.device("cuda", local)
-    if args.graph:  # graphs are captured on a stream of their own; torch's ops follow it
+    part = None
+    if args.sm_split:  # main stream on the large SM partition, route resolution on the small one
+        part = P.Partition(local, args.sm_split)
+        torch.cuda.set_stream(part.big)
+    elif args.graph:  # graphs are captured on a stream of their own; torch's ops follow it
         torch.cuda.set_stream(torch.cuda.Stream(dev))
     stream = torch.cuda.current_stream(dev)
+    resolve_stream = part.small if part is not None else None
 
     if args.intervals:
         import dataclasses
@@ -323,7 +331,7 @@ def main():
     tok_bytes = 4.0 * rec_tokens * float(sum(trace.counts[:cfg.n_intervals]))
     free, _total = torch.cuda.mem_get_info(dev)
     if args.keys_mode or tok_bytes > 0.6 * free:
-        return run_keys_mode(args, cfg, trace, dev, stream, world, rank, barrier)
+        return run_keys_mode(args, cfg, trace, dev, stream, world, rank, barrier, resolve_stream)
 
     # inputs resident in HBM (generated on the device, untimed)
     inputs = []
@@ -343,7 +351,7 @@ def main():
     ctx = P.Context(local, stream)
     pipe = Pipeline(ctx, cfg.R, cfg.W, cfg.caps, cfg.replicas, trace.qcap, batch_B=args.batch, max_n=max_n,
                     overlap=not args.no_overlap, vnodes=cfg.vnodes, fresh=args.fresh_plans,
-                    lru_tokens=cfg.lru_tokens)
+                    lru_tokens=cfg.lru_tokens, resolve_stream=resolve_stream)
     marks = [[[torch.cuda.Event(enable_timing=True) for _ in range(5)] for _ in range(cfg.n_intervals)]
              for _ in range(max(args.steps, 1))]
 
@@ -451,7 +459,7 @@ def main():
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": ms_max, "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "u64", "data": "synthetic",
-        "config": workload_config(cfg, args.batch, args.fresh_plans),
+        "config": dict(workload_config(cfg, args.batch, args.fresh_plans), sm_split=args.sm_split or None),
         "roofline": roofline,
         "stages_ms_per_step": {"hash": float(hash_ms.sum(1).mean()),
                                "main_wait_for_keys_and_plans": float(plan_wait_ms.sum(1).mean()),
@@ -558,7 +566,7 @@ def replan_study(args, ctx, cfg, trace, inputs, dev, stream, max_n):
     }
 
 
-def run_keys_mode(args, cfg, trace, dev, stream, world, rank, barrier):
+def run_keys_mode(args, cfg, trace, dev, stream, world, rank, barrier, resolve_stream=None):
     import torch
     import torch.distributed as dist
     import paper_2608_19677_gb300 as P
@@ -592,7 +600,7 @@ def run_keys_mode(args, cfg, trace, dev, stream, world, rank, barrier):
     n_step = sum(ns)
     pipe = Pipeline(ctx, cfg.R, cfg.W, cfg.caps, cfg.replicas, trace.qcap, batch_B=args.batch, max_n=max(ns),
                     overlap=not args.no_overlap, vnodes=cfg.vnodes, fresh=args.fresh_plans,
-                    lru_tokens=cfg.lru_tokens)
+                    lru_tokens=cfg.lru_tokens, resolve_stream=resolve_stream)
     marks = [[[torch.cuda.Event(enable_timing=True) for _ in range(5)] for _ in range(cfg.n_intervals)]
              for _ in range(max(args.steps, 1))]
     plan_marks = [[] for _ in range(max(args.steps, 1))]
@@ -683,7 +691,7 @@ def run_keys_mode(args, cfg, trace, dev, stream, world, rank, barrier):
         "metric": METRIC, "value": job_throughput(n_step, world, ms_max), "unit": UNIT, "n_gpus": world,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_max, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "u64", "data": "synthetic",
-        "config": dict(workload_config(cfg, args.batch, args.fresh_plans),
+        "config": dict(workload_config(cfg, args.batch, args.fresh_plans), sm_split=args.sm_split or None,
                        step="plans + route + replay over resident keys (the token arenas of all intervals do "
                             "not fit in HBM: each interval's arena was generated and hashed one at a time, each "
                             "hash launch timed alone)",

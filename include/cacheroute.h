@@ -86,6 +86,7 @@ typedef struct cr_ctx cr_ctx;
 typedef struct cr_plan cr_plan;
 typedef struct cr_replay cr_replay;
 typedef struct cr_ring cr_ring;
+typedef struct cr_partition cr_partition;
 
 /* ==== context ============================================================ */
 
@@ -100,6 +101,28 @@ CR_API int cr_destroy(cr_ctx *ctx);
 
 /* Switch the stream later calls enqueue on. */
 CR_API int cr_set_stream(cr_ctx *ctx, void *cuda_stream);
+
+/* Routing split over two streams: with a non-NULL stream, cr_route_batch runs
+ * the per-request candidates (and the load counts of RR / HASH replicas) on
+ * the context's stream and the load-dependent resolution on `cuda_stream`,
+ * ordered by an event; the resolution's end (on `cuda_stream`) then covers all
+ * of the call's writes to d_dest and d_load, and the next call's candidates
+ * wait for it.  Callers order later readers of d_dest / d_load after
+ * `cuda_stream`.  NULL restores single-stream routing.  Errors: CR_EINVAL,
+ * CR_ECUDA. */
+CR_API int cr_set_resolve_stream(cr_ctx *ctx, void *cuda_stream);
+
+/* Two CUDA streams whose kernels run on disjoint sets of SMs (green contexts):
+ * *small_stream on small_sms SMs, *big_stream on the rest (the driver may round
+ * the split to its SM granularity).  Kernels launched through the runtime API
+ * into either stream stay on its SMs; other streams may use every SM.  The
+ * streams live until cr_partition_destroy.  Errors: CR_EINVAL (bad device or
+ * small_sms not in 1 .. SMs - 1), CR_ECUDA (green contexts unavailable),
+ * CR_ENOMEM. */
+CR_API int cr_partition_create(int device, uint32_t small_sms, cr_partition **out, void **big_stream,
+                               void **small_stream);
+/* Waits for both streams, then destroys them and their green contexts.  NULL is accepted. */
+CR_API int cr_partition_destroy(cr_partition *p);
 
 /* Blocking: wait for the context's stream, then report any error a kernel
  * recorded since the last blocking call (CR_EOVERFLOW, CR_ETIMEOUT) and

@@ -38,7 +38,7 @@ EXPORTS = ("cr_create", "cr_destroy", "cr_set_stream", "cr_sync", "cr_last_error
            "cr_plan_get_info", "cr_plan_export", "cr_route_batch", "cr_replay_create", "cr_replay_reset",
            "cr_replay_destroy", "cr_shadow_replay", "cr_replay_export_state", "cr_key_histogram_noalloc",
            "cr_ring_create", "cr_ring_destroy", "cr_ring_export", "cr_plan_diff",
-           "cr_replay_create_tokens")
+           "cr_replay_create_tokens", "cr_set_resolve_stream", "cr_partition_create", "cr_partition_destroy")
 CR_NOALLOC_MAX_KEYS = 65536
 
 
@@ -114,6 +114,9 @@ def lib() -> C.CDLL:
         "cr_ring_destroy": ([vp, vp], i32),
         "cr_ring_export": ([vp, vp, vp, vp], i32),
         "cr_plan_diff": ([vp, vp, vp, C.POINTER(PlanDiff)], i32),
+        "cr_set_resolve_stream": ([vp, vp], i32),
+        "cr_partition_create": ([i32, u32, C.POINTER(vp), C.POINTER(vp), C.POINTER(vp)], i32),
+        "cr_partition_destroy": ([vp], i32),
     }
     for name, (args, res) in sig.items():
         f = getattr(L, name)
@@ -266,6 +269,39 @@ def build_plan(ctx: Context, keys, params: PlanParams, plan: Optional[Plan] = No
     plan = plan or Plan(ctx)
     build_plans(ctx, keys, [params], [plan])
     return plan
+
+
+def set_resolve_stream(ctx: Context, stream) -> None:
+    """Route with the load-dependent resolution on ``stream`` (a torch stream; None: the context's)."""
+    ctx.check(lib().cr_set_resolve_stream(ctx.handle, C.c_void_p(stream.cuda_stream) if stream is not None
+                                          else None), "cr_set_resolve_stream")
+
+
+class Partition:
+    """Two streams whose kernels run on disjoint SM sets (green contexts): ``big`` and ``small``
+    (torch external streams; ``small`` has ``small_sms`` SMs)."""
+
+    def __init__(self, device: int, small_sms: int):
+        import torch
+        h, b, sm = C.c_void_p(), C.c_void_p(), C.c_void_p()
+        st = lib().cr_partition_create(device, small_sms, C.byref(h), C.byref(b), C.byref(sm))
+        if st != CR_OK:
+            raise CacheRouteError(st, "cr_partition_create", lib().cr_last_error(None).decode())
+        self._h = h
+        dev = torch.device("cuda", device)
+        self.big = torch.cuda.ExternalStream(b.value, device=dev)
+        self.small = torch.cuda.ExternalStream(sm.value, device=dev)
+
+    def close(self):
+        if getattr(self, "_h", None):
+            lib().cr_partition_destroy(self._h)
+            self._h = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
 
 
 def plan_diff(ctx: Context, a: Plan, b: Plan) -> dict:

@@ -2,6 +2,8 @@
 #include <stdlib.h>
 #include <string.h>
 
+#include <cuda.h>
+
 #include "cr_internal.cuh"
 
 static char g_create_msg[320] = "no error";
@@ -84,6 +86,9 @@ extern "C" int cr_destroy(cr_ctx *ctx)
 {
     if (!ctx) return CR_OK;
     cudaStreamSynchronize(ctx->stream);
+    if (ctx->resolve_stream) cudaStreamSynchronize(ctx->resolve_stream);
+    if (ctx->ev_cand) cudaEventDestroy(ctx->ev_cand);
+    if (ctx->ev_resolve) cudaEventDestroy(ctx->ev_resolve);
     for (int i = 0; i < SCR_NUM; ++i)
         if (ctx->scratch[i]) cudaFree(ctx->scratch[i]);
     cudaFree(ctx->d_status);
@@ -95,6 +100,114 @@ extern "C" int cr_set_stream(cr_ctx *ctx, void *cuda_stream)
 {
     if (!ctx) return CR_EINVAL;
     ctx->stream = (cudaStream_t)cuda_stream;
+    return CR_OK;
+}
+
+extern "C" int cr_set_resolve_stream(cr_ctx *ctx, void *cuda_stream)
+{
+    if (!ctx) return CR_EINVAL;
+    if (cuda_stream && !ctx->ev_cand) {
+        CR_CUDA(ctx, cudaEventCreateWithFlags(&ctx->ev_cand, cudaEventDisableTiming));
+        CR_CUDA(ctx, cudaEventCreateWithFlags(&ctx->ev_resolve, cudaEventDisableTiming));
+    }
+    if (ctx->resolve_stream && ctx->resolve_stream != (cudaStream_t)cuda_stream)
+        CR_CUDA(ctx, cudaStreamSynchronize(ctx->resolve_stream));
+    ctx->resolve_stream = (cudaStream_t)cuda_stream;
+    ctx->resolve_recorded = 0;
+    return CR_OK;
+}
+
+// ---- SM partition (green contexts, reached through the runtime's driver entry points) ----
+struct cr_partition {
+    CUgreenCtx g[2];
+    CUstream s[2];
+};
+
+template <typename F>
+static int driver_fn(const char *name, F *fp)
+{
+    cudaDriverEntryPointQueryResult q;
+    void *p = nullptr;
+    if (cudaGetDriverEntryPointByVersion(name, &p, CUDART_VERSION, cudaEnableDefault, &q) != cudaSuccess ||
+        q != cudaDriverEntryPointSuccess || !p) {
+        cudaGetLastError();
+        return CR_ECUDA;
+    }
+    *fp = reinterpret_cast<F>(p);
+    return CR_OK;
+}
+
+extern "C" int cr_partition_create(int device, uint32_t small_sms, cr_partition **out, void **big_stream,
+                                   void **small_stream)
+{
+    if (!out || !big_stream || !small_stream) return cr_fail(NULL, CR_EINVAL, "cr_partition_create: NULL output");
+    *out = nullptr;
+    typedef CUresult (*fDeviceGet)(CUdevice *, int);
+    typedef CUresult (*fGetRes)(CUdevice, CUdevResource *, CUdevResourceType);
+    typedef CUresult (*fSplit)(CUdevResource *, unsigned int *, const CUdevResource *, CUdevResource *, unsigned int,
+                               unsigned int);
+    typedef CUresult (*fDesc)(CUdevResourceDesc *, CUdevResource *, unsigned int);
+    typedef CUresult (*fGreen)(CUgreenCtx *, CUdevResourceDesc, CUdevice, unsigned int);
+    typedef CUresult (*fStream)(CUstream *, CUgreenCtx, unsigned int, int);
+    fDeviceGet deviceGet;
+    fGetRes getRes;
+    fSplit split;
+    fDesc desc;
+    fGreen green;
+    fStream stream;
+    if (cudaSetDevice(device) != cudaSuccess || cudaFree(0) != cudaSuccess) {
+        cudaGetLastError();
+        return cr_fail(NULL, CR_EINVAL, "cr_partition_create: device %d not available", device);
+    }
+    if (driver_fn("cuDeviceGet", &deviceGet) || driver_fn("cuDeviceGetDevResource", &getRes) ||
+        driver_fn("cuDevSmResourceSplitByCount", &split) || driver_fn("cuDevResourceGenerateDesc", &desc) ||
+        driver_fn("cuGreenCtxCreate", &green) || driver_fn("cuGreenCtxStreamCreate", &stream))
+        return cr_fail(NULL, CR_ECUDA, "cr_partition_create: green contexts are not available from this driver");
+    CUdevice dev;
+    CUdevResource sm, part, rest;
+    if (deviceGet(&dev, device) != CUDA_SUCCESS || getRes(dev, &sm, CU_DEV_RESOURCE_TYPE_SM) != CUDA_SUCCESS)
+        return cr_fail(NULL, CR_ECUDA, "cr_partition_create: cannot read the SM resource");
+    if (small_sms == 0 || small_sms >= sm.sm.smCount)
+        return cr_fail(NULL, CR_EINVAL, "cr_partition_create: small_sms=%u outside 1..%u", small_sms,
+                       sm.sm.smCount - 1);
+    unsigned int nb = 1;
+    if (split(&part, &nb, &sm, &rest, 0, sm.sm.smCount - small_sms) != CUDA_SUCCESS || nb != 1 ||
+        rest.sm.smCount == 0)
+        return cr_fail(NULL, CR_ECUDA, "cr_partition_create: cannot split %u SMs", sm.sm.smCount);
+    cr_partition *pt = (cr_partition *)calloc(1, sizeof(cr_partition));
+    if (!pt) return cr_fail(NULL, CR_ENOMEM, "cr_partition_create: host allocation failed");
+    CUdevResource *res[2] = {&part, &rest};
+    for (int i = 0; i < 2; ++i) {
+        CUdevResourceDesc d;
+        if (desc(&d, res[i], 1) != CUDA_SUCCESS || green(&pt->g[i], d, dev, CU_GREEN_CTX_DEFAULT_STREAM) != CUDA_SUCCESS ||
+            stream(&pt->s[i], pt->g[i], CU_STREAM_NON_BLOCKING, 0) != CUDA_SUCCESS) {
+            cr_partition_destroy(pt);
+            return cr_fail(NULL, CR_ECUDA, "cr_partition_create: cannot create the green context");
+        }
+    }
+    *out = pt;
+    *big_stream = (void *)pt->s[0];
+    *small_stream = (void *)pt->s[1];
+    return CR_OK;
+}
+
+extern "C" int cr_partition_destroy(cr_partition *pt)
+{
+    if (!pt) return CR_OK;
+    typedef CUresult (*fStreamDestroy)(CUstream);
+    typedef CUresult (*fGreenDestroy)(CUgreenCtx);
+    fStreamDestroy sd = nullptr;
+    fGreenDestroy gd = nullptr;
+    driver_fn("cuStreamDestroy", &sd);
+    driver_fn("cuGreenCtxDestroy", &gd);
+    for (int i = 0; i < 2; ++i) {
+        if (pt->s[i] && sd) {
+            cudaStreamSynchronize((cudaStream_t)pt->s[i]);
+            sd(pt->s[i]);
+        }
+        if (pt->g[i] && gd) gd(pt->g[i]);
+    }
+    free(pt);
     return CR_OK;
 }
 

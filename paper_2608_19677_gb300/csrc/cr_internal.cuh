@@ -43,6 +43,11 @@ struct cr_ctx {
     void *scratch[SCR_NUM];
     size_t scratch_bytes[SCR_NUM];
     char msg[320];
+    // routing split over two streams (cr_set_resolve_stream): the load-dependent
+    // resolution runs on resolve_stream, after ev_cand; ev_resolve marks its end
+    cudaStream_t resolve_stream;     // NULL: everything on `stream`
+    cudaEvent_t ev_cand, ev_resolve;
+    int resolve_recorded;            // ev_resolve has been recorded at least once
 };
 
 // Plan: every array lives on the device; capacities are host-side upper bounds.
@@ -122,6 +127,14 @@ int cr_check_launch(cr_ctx *ctx, const char *what);
 #define CR_LAUNCH(ctx, kern, grid, block, smem, ...)                       \
     do {                                                                   \
         kern<<<(grid), (block), (smem), (ctx)->stream>>>(__VA_ARGS__);     \
+        (ctx)->launches++;                                                 \
+        CR_TRY(cr_check_launch((ctx), #kern));                             \
+    } while (0)
+
+// Launch on a given stream of the context (e.g. its resolve stream) and account for it.
+#define CR_LAUNCH_ON(ctx, st, kern, grid, block, smem, ...)                \
+    do {                                                                   \
+        kern<<<(grid), (block), (smem), (st)>>>(__VA_ARGS__);              \
         (ctx)->launches++;                                                 \
         CR_TRY(cr_check_launch((ctx), #kern));                             \
     } while (0)

@@ -613,6 +613,10 @@ extern "C" int cr_ring_export(cr_ctx *ctx, const cr_ring *g, uint64_t *point, ui
     return cr_sync(ctx);
 }
 
+static int launch_resolve(cr_ctx *ctx, cudaStream_t rs, const route_args &args, const uint32_t *cand, uint64_t n,
+                          uint32_t batch_B, uint32_t R, uint64_t mc, uint32_t n_dep, uint64_t *d_load,
+                          uint16_t *d_dest);
+
 extern "C" int cr_route_batch(cr_ctx *ctx, const cr_plan *const *plans, const cr_replica *reps, uint32_t n_rep,
                               uint32_t R, const uint64_t *d_key, uint64_t n, uint64_t first_req_index,
                               uint32_t batch_B, uint64_t *d_load, uint16_t *d_dest)
@@ -666,6 +670,10 @@ extern "C" int cr_route_batch(cr_ctx *ctx, const cr_plan *const *plans, const cr
     uint32_t n_dep = 0;
     for (uint32_t i = 0; i < n_rep; ++i)
         if (reps[i].policy != CR_POLICY_RR && reps[i].policy != CR_POLICY_HASH) args.dep[n_dep++] = i;
+    // split routing: the candidates scratch is free once the last resolution has read it
+    const cudaStream_t rs = ctx->resolve_stream ? ctx->resolve_stream : ctx->stream;
+    const bool split = rs != ctx->stream;
+    if (split && ctx->resolve_recorded) CR_CUDA(ctx, cudaStreamWaitEvent(ctx->stream, ctx->ev_resolve, 0));
     void *pc;
     CR_TRY(cr_scratch(ctx, SCR_ROUTE_DESC, (size_t)n * n_rep * sizeof(uint32_t), &pc));
     uint32_t *cand = (uint32_t *)pc;
@@ -683,7 +691,23 @@ extern "C" int cr_route_batch(cr_ctx *ctx, const cr_plan *const *plans, const cr
                   (unsigned long long)n, R, (unsigned long long *)d_load + (uint64_t)i * R);
         i = j;
     }
-    if (!n_dep) return CR_OK;
+    if (split) {  // the resolution (and the caller's later readers) follow everything above
+        CR_CUDA(ctx, cudaEventRecord(ctx->ev_cand, ctx->stream));
+        CR_CUDA(ctx, cudaStreamWaitEvent(rs, ctx->ev_cand, 0));
+    }
+    if (n_dep) CR_TRY(launch_resolve(ctx, rs, args, cand, n, batch_B, R, mc, n_dep, d_load, d_dest));
+    if (split) {
+        CR_CUDA(ctx, cudaEventRecord(ctx->ev_resolve, rs));
+        ctx->resolve_recorded = 1;
+    }
+    return CR_OK;
+}
+
+// The load-dependent resolution of every dependent replica, enqueued on stream rs.
+static int launch_resolve(cr_ctx *ctx, cudaStream_t rs, const route_args &args, const uint32_t *cand, uint64_t n,
+                          uint32_t batch_B, uint32_t R, uint64_t mc, uint32_t n_dep, uint64_t *d_load,
+                          uint16_t *d_dest)
+{
     // member lists and ring owners go to shared memory when they fit beside the loads
     auto with_members = [&](size_t base, uint64_t *MC) {
         *MC = (mc && base + mc * sizeof(uint16_t) <= kSmemBudget) ? mc : 0;
@@ -696,7 +720,7 @@ extern "C" int cr_route_batch(cr_ctx *ctx, const cr_plan *const *plans, const cr
         if (smem > 48 * 1024)
             CR_CUDA(ctx, cudaFuncSetAttribute(k_route_resolve_warp, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                               (int)smem));
-        CR_LAUNCH(ctx, k_route_resolve_warp, n_dep, 32, smem, args, (const uint32_t *)cand, (unsigned long long)n,
+        CR_LAUNCH_ON(ctx, rs, k_route_resolve_warp, n_dep, 32, smem, args, (const uint32_t *)cand, (unsigned long long)n,
                   batch_B, R, (unsigned long long *)d_load, d_dest, ctx->d_status, (unsigned long long)MC);
         return CR_OK;
     }
@@ -706,7 +730,7 @@ extern "C" int cr_route_batch(cr_ctx *ctx, const cr_plan *const *plans, const cr
         (size_t)R * (sizeof(unsigned long long) + sizeof(uint32_t)) + 2ull * CH * sizeof(uint32_t), &MC);
     if (smem > 48 * 1024)
         CR_CUDA(ctx, cudaFuncSetAttribute(k_route_resolve, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
-    CR_LAUNCH(ctx, k_route_resolve, n_dep, kRouteBlock, smem, args, (const uint32_t *)cand, (unsigned long long)n,
+    CR_LAUNCH_ON(ctx, rs, k_route_resolve, n_dep, kRouteBlock, smem, args, (const uint32_t *)cand, (unsigned long long)n,
               batch_B, CH, R, (unsigned long long *)d_load, d_dest, ctx->d_status, (unsigned long long)MC);
     return CR_OK;
 }

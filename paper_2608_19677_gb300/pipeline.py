@@ -32,7 +32,7 @@ from __future__ import annotations
 from typing import Callable, List, Optional, Sequence, Tuple
 
 from . import (Context, Plan, Replay, Ring, build_plans, hash_prefixes, plan_params, route_batch,
-               shadow_replay)
+               set_resolve_stream, shadow_replay)
 
 VARIANT_OF = {"CR": "LPT", "CR_NOLPT": "RANDOM", "CR_NOREPL": "NOREPL", "CR_SLOTCAP": "SLOTCAP"}
 # CacheRoute on a slot-capped plan routes as CacheRoute (same fallback draws as CR, seed for seed)
@@ -44,7 +44,7 @@ class Pipeline:
     def __init__(self, ctx: Context, R: int, W: int, caps: Sequence[int],
                  replicas: Sequence[Tuple[str, int]], qcap: Callable[[int], Tuple[int, int]],
                  batch_B: int = 1024, salt: int = 0, max_n: int = 0, overlap: bool = False,
-                 vnodes: int = 64, fresh: bool = False, lru_tokens: bool = False):
+                 vnodes: int = 64, fresh: bool = False, lru_tokens: bool = False, resolve_stream=None):
         import torch
         self.ctx, self.R, self.W, self.caps = ctx, R, W, list(caps)
         self.replicas = list(replicas)
@@ -81,6 +81,11 @@ class Pipeline:
         else:
             self.hstream = self.pstream = self.ystream = self.mstream
             self.hctx = self.pctx = self.yctx = ctx
+        # split routing: the load-dependent resolution on a stream of its own (e.g. a small SM
+        # partition), so that it overlaps the next interval's hashing on the main stream
+        self.xstream = resolve_stream if overlap else None
+        if self.xstream is not None:
+            set_resolve_stream(ctx, self.xstream)
         self.plans = [[Plan(self.pctx) for _ in self.plan_keys] for _ in range(2)]
         self.replay = Replay(ctx, len(self.replicas), R, self.caps, tokens=lru_tokens)
         # ring of every bounded-load replica, seeded by the replica's seed (built once)
@@ -97,6 +102,8 @@ class Pipeline:
         self.prev_keys = None
         self._prev_kb = None
         self._ready = [None, None]   # event: plans buffer b is built
+        self._plan_free = [None, None]  # event: the route that read plans buffer b has finished
+        self._routed_prev = None     # event: the last route call's end (split routing)
         self._pbuf = 0               # plans buffer used by the next interval
         self._next_built = False     # the next interval's plans are already enqueued
         self.plan_marks = []         # (start, end) events of every plan build, when marked
@@ -154,6 +161,8 @@ class Pipeline:
         """Enqueue the plans of one interval into plans buffer ``buf`` from ``keys``."""
         if self.overlap:
             self.pstream.wait_event(after)
+            if self._plan_free[buf] is not None:  # the route that last read this buffer
+                self.pstream.wait_event(self._plan_free[buf])
         ev0 = self._event(self.pstream, True) if mark else None
         num, den = self.qcap(int(keys.shape[0]))
         params = [plan_params(self.R, self.W, num, den, v, seed=s, epoch=epoch) for v, s in self.plan_keys]
@@ -177,6 +186,7 @@ class Pipeline:
         the interval's routing keys when they were computed beforehand (the
         token arena is then not read and may be None).
         """
+        import torch
         n = int(keys.shape[0]) if keys is not None else int(off.shape[0])
         mark = marks is not None
         if mark:
@@ -230,7 +240,10 @@ class Pipeline:
         if mark:
             marks[1].record(self.mstream)
             marks[2].record(self.mstream)
-        self.load.zero_()
+        if self.xstream is not None and self._routed_prev is not None:
+            self.mstream.wait_event(self._routed_prev)  # the last resolution wrote the loads
+        with torch.cuda.stream(self.mstream):
+            self.load.zero_()
         db = self._dbuf
         if self.overlap:
             self._dbuf ^= 1
@@ -242,11 +255,16 @@ class Pipeline:
         r0 = self._event(self.mstream, True) if mark else None
         route_batch(self.ctx, plans, [ROUTE_AS.get(p, p) for p in self.policies], self.seeds, self.R, keys, g0,
                     self.B, self.load, dest, rings=self.rings)
+        rstream = self.xstream if self.xstream is not None else self.mstream  # where the route call ends
         if mark:
-            marks[3].record(self.mstream)
+            marks[3].record(rstream)
             self.route_marks.append((r0, marks[3]))
         if self.overlap:
-            self.ystream.wait_event(self._event(self.mstream))
+            routed = self._event(rstream)
+            self.ystream.wait_event(routed)
+            if self.xstream is not None:
+                self._plan_free[cur] = routed
+                self._routed_prev = routed
         y0 = self._event(self.ystream, True) if mark else None
         shadow_replay(self.yctx, self.replay, keys, plen, slen, dest, self.ctr)
         replayed = self._event(self.ystream, mark)
@@ -275,7 +293,7 @@ class Pipeline:
         whatever stream the caller uses; the host does not block."""
         import torch
         cur = torch.cuda.current_stream(self.dev)
-        for st in (self.mstream, self.pstream, self.ystream):
+        for st in (self.mstream, self.pstream, self.ystream) + ((self.xstream,) if self.xstream is not None else ()):
             cur.wait_event(self._event(st))
 
     def quiesce(self):
@@ -285,6 +303,8 @@ class Pipeline:
         self._released = [[] for _ in range(NKEYS)]
         self._dest_free = [None, None]
         self._ready = [None, None]
+        self._plan_free = [None, None]
+        self._routed_prev = None
         self._next_built = False
         self.inputs_free = None
 
@@ -294,8 +314,12 @@ class Pipeline:
             self.mstream.wait_event(self._event(self.hstream))
             self.mstream.wait_event(self._event(self.pstream))
             self.mstream.wait_event(self._event(self.ystream))
+            if self.xstream is not None:
+                self.mstream.wait_event(self._event(self.xstream))
 
     def sync(self):
+        if self.xstream is not None:
+            self.xstream.synchronize()
         for c in self.contexts:
             c.sync()
 

@@ -728,3 +728,32 @@ def test_pipeline_parity_slotcap_policy(P, ctx):
         assert (h_u16(pipe.last_dest) == ref["dest"][t]).all()
     pipe.sync()
     assert (h_u64(pipe.ctr) == ref["ctr"]).all()
+
+
+def test_pipeline_split_routing_on_sm_partition(P, ctx):
+    # hashing and candidates on the large SM partition, the route resolution on the small one
+    # (green contexts): same destinations and counters as the oracle
+    from paper_2608_19677_gb300.pipeline import Pipeline
+    try:
+        part = P.Partition(0, 16)
+    except P.CacheRouteError as e:
+        pytest.skip(f"no SM partition on this driver: {e}")
+    cfg = tg.CONFIGS["70b"].scaled(40000, 4)
+    tr = tg.Trace(cfg)
+    ref = OP.run_trace(tr, B=1024, keep=True)
+    with torch.cuda.stream(part.big):
+        pctx = P.Context(0, part.big)
+        pipe = Pipeline(pctx, cfg.R, cfg.W, cfg.caps, cfg.replicas, tr.qcap, batch_B=1024, overlap=True,
+                        resolve_stream=part.small)
+        for t in range(cfg.n_intervals):
+            iv = tr.interval(t)
+            tok, off = tg.arena_host(tr, iv, 4)
+            pipe.interval(t, torch.from_numpy(tok).to(DEV), d_u64(off), d_u32(iv.plen), d_u32(iv.slen), iv.g0,
+                          plan_next=t + 1 < cfg.n_intervals)
+            pipe.wait_last()
+            assert (h_u16(pipe.last_dest) == ref["dest"][t]).all()
+        pipe.sync()
+        assert (h_u64(pipe.ctr) == ref["ctr"]).all()
+    del pipe  # contexts on the partition's streams go before the partition
+    pctx.close()
+    part.close()
