@@ -16,6 +16,8 @@
  *   cr_route_batch    keys -> one destination per (request, replica)
  *   cr_ring_create    consistent-hashing ring of the bounded-load comparison policy
  *   cr_plan_diff      cache and count churn between two plans (replanning under drift)
+ *   cr_partition_create, cr_set_resolve_stream
+ *                     routing split over two streams on disjoint SM sets
  *   cr_shadow_replay  routed requests -> per-destination LRU hits and load
  *
  * Conventions shared by every call:
