@@ -110,8 +110,9 @@ CR_API int cr_set_stream(cr_ctx *ctx, void *cuda_stream);
  * ordered by an event; the resolution's end (on `cuda_stream`) then covers all
  * of the call's writes to d_dest and d_load, and the next call's candidates
  * wait for it.  Callers order later readers of d_dest / d_load after
- * `cuda_stream`.  NULL restores single-stream routing.  Errors: CR_EINVAL,
- * CR_ECUDA. */
+ * `cuda_stream`.  NULL restores single-stream routing.  Setting the stream the
+ * context already has does nothing; switching waits for the old stream.
+ * Errors: CR_EINVAL, CR_ECUDA. */
 CR_API int cr_set_resolve_stream(cr_ctx *ctx, void *cuda_stream);
 
 /* Two CUDA streams whose kernels run on disjoint sets of SMs (green contexts):

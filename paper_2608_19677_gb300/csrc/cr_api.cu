@@ -110,10 +110,10 @@ extern "C" int cr_set_resolve_stream(cr_ctx *ctx, void *cuda_stream)
         CR_CUDA(ctx, cudaEventCreateWithFlags(&ctx->ev_cand, cudaEventDisableTiming));
         CR_CUDA(ctx, cudaEventCreateWithFlags(&ctx->ev_resolve, cudaEventDisableTiming));
     }
-    if (ctx->resolve_stream && ctx->resolve_stream != (cudaStream_t)cuda_stream)
-        CR_CUDA(ctx, cudaStreamSynchronize(ctx->resolve_stream));
+    if (ctx->resolve_stream == (cudaStream_t)cuda_stream) return CR_OK;  // unchanged: keep the ordering state
+    if (ctx->resolve_stream) CR_CUDA(ctx, cudaStreamSynchronize(ctx->resolve_stream));
     ctx->resolve_stream = (cudaStream_t)cuda_stream;
-    ctx->resolve_recorded = 0;
+    ctx->resolve_recorded = 0;  // the old stream's work is finished
     return CR_OK;
 }
 

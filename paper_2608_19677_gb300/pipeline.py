@@ -84,8 +84,6 @@ class Pipeline:
         # split routing: the load-dependent resolution on a stream of its own (e.g. a small SM
         # partition), so that it overlaps the next interval's hashing on the main stream
         self.xstream = resolve_stream if overlap else None
-        if self.xstream is not None:
-            set_resolve_stream(ctx, self.xstream)
         self.plans = [[Plan(self.pctx) for _ in self.plan_keys] for _ in range(2)]
         self.replay = Replay(ctx, len(self.replicas), R, self.caps, tokens=lru_tokens)
         # ring of every bounded-load replica, seeded by the replica's seed (built once)
@@ -253,6 +251,9 @@ class Pipeline:
         dest = D[:, :n] if n == D.shape[1] else D.view(-1)[:len(self.replicas) * n].view(len(self.replicas), n)
         plans = [self.plans[cur][i] if i is not None else None for i in self.rep_plan]
         r0 = self._event(self.mstream, True) if mark else None
+        # the split is a property of the library context, which other pipelines may share:
+        # set it for every call (the library synchronises only when it changes)
+        set_resolve_stream(self.ctx, self.xstream)
         route_batch(self.ctx, plans, [ROUTE_AS.get(p, p) for p in self.policies], self.seeds, self.R, keys, g0,
                     self.B, self.load, dest, rings=self.rings)
         rstream = self.xstream if self.xstream is not None else self.mstream  # where the route call ends
