@@ -57,6 +57,9 @@ def parse_args(argv=None):
     ap.add_argument("--policies", default="",
                     help="comma-separated dispatch policies replacing the configuration's (same seeds), "
                          "e.g. CR,P2C,RR,HASH,CHWBL")
+    ap.add_argument("--clocks-out", default="",
+                    help="keep the nvidia-smi clock samples of the timed region in this CSV file (default: a "
+                         "temporary file, removed after it is summarised)")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-overlap", action="store_true", help="build plans in line instead of on a second stream")
@@ -119,14 +122,21 @@ class ClockSampler:
               "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
               "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
 
-    def __init__(self, device_index: int):
+    def __init__(self, device_index: int, out_path: str = ""):
         self.dev = device_index
         self.proc = None
-        self.path = os.path.join(ROOT, "gpurun_out", f"clocks_rank{device_index}.csv")
+        self.keep = bool(out_path)  # a caller-chosen file is kept; a temporary one is removed
+        if out_path:
+            self.path = out_path
+        else:
+            import tempfile
+            fd, self.path = tempfile.mkstemp(prefix=f"cr_clocks_{device_index}_", suffix=".csv")
+            os.close(fd)
 
     def start(self):
         try:
-            os.makedirs(os.path.dirname(self.path), exist_ok=True)
+            if os.path.dirname(self.path):
+                os.makedirs(os.path.dirname(self.path), exist_ok=True)
             self.f = open(self.path, "w")
             self.proc = subprocess.Popen(["nvidia-smi", "-i", str(self.dev), f"--query-gpu={self.FIELDS}",
                                           "--format=csv,noheader,nounits", "-lms", "100"], stdout=self.f,
@@ -157,6 +167,11 @@ class ClockSampler:
             for nm, v in zip(names, parts[5:9]):
                 if v.lower() == "active":
                     reasons.add(nm)
+        if not self.keep:
+            try:
+                os.remove(self.path)
+            except OSError:
+                pass
         return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(mx) if mx else None,
                 "samples": len(sm), "reasons": sorted(reasons)}
 
@@ -276,6 +291,16 @@ def job_throughput(units_per_rank: int, world: int, ms_max: float) -> float:
     return units_per_rank * world / (ms_max / 1e3)
 
 
+def close_in_order(pipe, ctx, part):
+    """With an SM partition, free what uses its streams before the partition itself: the
+    pipeline (plans, replay, rings, its own contexts), then the context on the big stream."""
+    if part is None:
+        return
+    pipe.close()
+    ctx.close()
+    part.close()
+
+
 # ----------------------------------------------------------------- ours ---
 def main():
     args = parse_args()
@@ -309,6 +334,9 @@ def main():
     trace = tg.Trace(cfg)
     dev = torch.device("cuda", local)
     part = None
+    if args.sm_split and args.graph:
+        sys.exit("--sm-split and --graph cannot be combined (a graph capture would span the partition's "
+                 "streams and the resolve-stream switch)")
     if args.sm_split:  # main stream on the large SM partition, route resolution on the small one
         part = P.Partition(local, args.sm_split)
         torch.cuda.set_stream(part.big)
@@ -331,7 +359,7 @@ def main():
     tok_bytes = 4.0 * rec_tokens * float(sum(trace.counts[:cfg.n_intervals]))
     free, _total = torch.cuda.mem_get_info(dev)
     if args.keys_mode or tok_bytes > 0.6 * free:
-        return run_keys_mode(args, cfg, trace, dev, stream, world, rank, barrier, resolve_stream)
+        return run_keys_mode(args, cfg, trace, dev, stream, world, rank, barrier, resolve_stream, part)
 
     # inputs resident in HBM (generated on the device, untimed)
     inputs = []
@@ -394,7 +422,7 @@ def main():
         torch.cuda.synchronize()
 
     # ---- timed region: K steps, stage events on the launching stream -------
-    clocks = ClockSampler(local)
+    clocks = ClockSampler(local, args.clocks_out)
     clocks.start()
     time.sleep(0.3)
     barrier()
@@ -496,6 +524,7 @@ def main():
                                           f"single-threaded C oracle"}
     if rank == 0:
         print(json.dumps(line), flush=True)
+    close_in_order(pipe, ctx, part)
     if world > 1:
         dist.destroy_process_group()
 
@@ -566,7 +595,7 @@ def replan_study(args, ctx, cfg, trace, inputs, dev, stream, max_n):
     }
 
 
-def run_keys_mode(args, cfg, trace, dev, stream, world, rank, barrier, resolve_stream=None):
+def run_keys_mode(args, cfg, trace, dev, stream, world, rank, barrier, resolve_stream=None, part=None):
     import torch
     import torch.distributed as dist
     import paper_2608_19677_gb300 as P
@@ -631,7 +660,7 @@ def run_keys_mode(args, cfg, trace, dev, stream, world, rank, barrier, resolve_s
         graph_launches = pipe.launches - lc0
         graph.replay()
         torch.cuda.synchronize()
-    clocks = ClockSampler(dev.index or 0)
+    clocks = ClockSampler(dev.index or 0, args.clocks_out)
     clocks.start()
     time.sleep(0.3)
     barrier()
@@ -715,6 +744,7 @@ def run_keys_mode(args, cfg, trace, dev, stream, world, rank, barrier, resolve_s
                               "and plan-build times come from one ordinary step after the timed region")
     if rank == 0:
         print(json.dumps(line), flush=True)
+    close_in_order(pipe, ctx, part)
     if world > 1:
         dist.destroy_process_group()
 

@@ -112,6 +112,8 @@ CR_API int cr_set_stream(cr_ctx *ctx, void *cuda_stream);
  * wait for it.  Callers order later readers of d_dest / d_load after
  * `cuda_stream`.  NULL restores single-stream routing.  Setting the stream the
  * context already has does nothing; switching waits for the old stream.
+ * cr_sync also waits for the last resolution enqueued on `cuda_stream`, so an
+ * error it raised is reported by the first blocking call after it.
  * Errors: CR_EINVAL, CR_ECUDA. */
 CR_API int cr_set_resolve_stream(cr_ctx *ctx, void *cuda_stream);
 
@@ -121,15 +123,17 @@ CR_API int cr_set_resolve_stream(cr_ctx *ctx, void *cuda_stream);
  * into either stream stay on its SMs; other streams may use every SM.  The
  * streams live until cr_partition_destroy.  Errors: CR_EINVAL (bad device or
  * small_sms not in 1 .. SMs - 1), CR_ECUDA (green contexts unavailable),
- * CR_ENOMEM. */
+ * CR_ENOMEM.  The calling thread's current device is the same after the call
+ * as before it. */
 CR_API int cr_partition_create(int device, uint32_t small_sms, cr_partition **out, void **big_stream,
                                void **small_stream);
 /* Waits for both streams, then destroys them and their green contexts.  NULL is accepted. */
 CR_API int cr_partition_destroy(cr_partition *p);
 
-/* Blocking: wait for the context's stream, then report any error a kernel
- * recorded since the last blocking call (CR_EOVERFLOW, CR_ETIMEOUT) and
- * clear it. */
+/* Blocking: wait for the context's stream (and, when routing is split by
+ * cr_set_resolve_stream, for the last resolution enqueued on the resolve
+ * stream), then report any error a kernel recorded since the last blocking
+ * call (CR_EOVERFLOW, CR_ETIMEOUT, CR_EINVAL) and clear it. */
 CR_API int cr_sync(cr_ctx *ctx);
 
 /* Message for the last failing call on this context (static storage; never

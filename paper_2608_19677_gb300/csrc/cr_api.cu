@@ -137,18 +137,35 @@ static int driver_fn(const char *name, F *fp)
     return CR_OK;
 }
 
+typedef CUresult (*fDeviceGet)(CUdevice *, int);
+typedef CUresult (*fGetRes)(CUdevice, CUdevResource *, CUdevResourceType);
+typedef CUresult (*fSplit)(CUdevResource *, unsigned int *, const CUdevResource *, CUdevResource *, unsigned int,
+                           unsigned int);
+typedef CUresult (*fDesc)(CUdevResourceDesc *, CUdevResource *, unsigned int);
+typedef CUresult (*fGreen)(CUgreenCtx *, CUdevResourceDesc, CUdevice, unsigned int);
+typedef CUresult (*fStream)(CUstream *, CUgreenCtx, unsigned int, int);
+
+static int partition_create(int device, uint32_t small_sms, cr_partition **out, void **big_stream,
+                            void **small_stream);
+
 extern "C" int cr_partition_create(int device, uint32_t small_sms, cr_partition **out, void **big_stream,
                                    void **small_stream)
 {
     if (!out || !big_stream || !small_stream) return cr_fail(NULL, CR_EINVAL, "cr_partition_create: NULL output");
     *out = nullptr;
-    typedef CUresult (*fDeviceGet)(CUdevice *, int);
-    typedef CUresult (*fGetRes)(CUdevice, CUdevResource *, CUdevResourceType);
-    typedef CUresult (*fSplit)(CUdevResource *, unsigned int *, const CUdevResource *, CUdevResource *, unsigned int,
-                               unsigned int);
-    typedef CUresult (*fDesc)(CUdevResourceDesc *, CUdevResource *, unsigned int);
-    typedef CUresult (*fGreen)(CUgreenCtx *, CUdevResourceDesc, CUdevice, unsigned int);
-    typedef CUresult (*fStream)(CUstream *, CUgreenCtx, unsigned int, int);
+    int prev_dev = -1;
+    if (cudaGetDevice(&prev_dev) != cudaSuccess) {
+        cudaGetLastError();
+        prev_dev = -1;
+    }
+    const int st = partition_create(device, small_sms, out, big_stream, small_stream);
+    if (prev_dev >= 0) cudaSetDevice(prev_dev);  // the caller's current device is left as it was
+    return st;
+}
+
+static int partition_create(int device, uint32_t small_sms, cr_partition **out, void **big_stream,
+                            void **small_stream)
+{
     fDeviceGet deviceGet;
     fGetRes getRes;
     fSplit split;
@@ -215,6 +232,9 @@ extern "C" int cr_sync(cr_ctx *ctx)
 {
     if (!ctx) return CR_EINVAL;
     CR_CUDA(ctx, cudaStreamSynchronize(ctx->stream));
+    // a split route call's resolution raises its flags on the resolve stream:
+    // wait for it too, so that no flag is missed or reported against a later call
+    if (ctx->resolve_stream && ctx->resolve_recorded) CR_CUDA(ctx, cudaEventSynchronize(ctx->ev_resolve));
     uint32_t flags = 0;
     CR_CUDA(ctx, cudaMemcpy(&flags, ctx->d_status, sizeof(flags), cudaMemcpyDeviceToHost));
     if (flags) {

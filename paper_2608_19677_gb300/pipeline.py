@@ -318,6 +318,24 @@ class Pipeline:
             if self.xstream is not None:
                 self.mstream.wait_event(self._event(self.xstream))
 
+    def close(self):
+        """Free the pipeline's plans, replay state and rings, close the contexts it created,
+        and detach the caller's context from the resolve stream, in that order (so that a
+        stream the pipeline was given, e.g. of an SM partition, can be destroyed afterwards)."""
+        self.sync()
+        for buf in self.plans:
+            for pl in buf:
+                pl.close()
+        self.replay.close()
+        for g in self.rings:
+            if g is not None:
+                g.close()
+        if self.xstream is not None:
+            set_resolve_stream(self.ctx, None)
+        for c in self.contexts:
+            if c is not self.ctx:
+                c.close()
+
     def sync(self):
         if self.xstream is not None:
             self.xstream.synchronize()

@@ -57,6 +57,5 @@ def test_product_never_imports_the_oracle():
         for f in files:
             if f.endswith((".py", ".cu", ".cuh", ".h")):
                 txt = open(os.path.join(dirpath, f)).read()
-                assert "oracle" not in txt.replace("Oracle", "oracle").split("\n")[0] or True
                 assert not re.search(r"^\s*(import|from)\s+oracle\b", txt, flags=re.M), f
                 assert "cr_oracle" not in txt and "libcr_oracle" not in txt, f

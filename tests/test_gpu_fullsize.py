@@ -5,11 +5,14 @@ run through the device pipeline exactly as the benchmark runs them (planner
 on its own stream, batches of 1024).  The oracle then checks, at full size:
   - every request's routing key (the oracle hashes each distinct key's
     prefix once; requests that carry the same key share their prefix);
-  - the complete plan interval 1 was routed with (built from interval 0);
-  - the complete destinations of two sampled replicas in interval 1;
-  - the complete replay counters of one sampled replica after both intervals;
+  - the complete plans interval 1 was routed with (built from interval 0);
+  - the complete destinations, in both intervals, of every plan-based replica
+    (CacheRoute and its ablations: the method's own dispatch through the
+    device table) and of one power-of-two-choices replica;
+  - the complete replay counters of those replicas after both intervals;
 and every replica's counters satisfy request conservation, LRU inclusion
-across capacities and prefill = prompt - hit tokens.
+across capacities and prefill = prompt - hit tokens.  The oracle runs one
+replica per thread (each call is plain single-threaded C).
 """
 import numpy as np
 import pytest
@@ -87,25 +90,33 @@ def test_fullsize_two_intervals(P, name):
         assert (got["members"] == ref.members).all() and (got["jobs"] == ref.jobs).all()
         assert (got["load"] == ref.load).all()
 
-    # ---- complete destinations of two sampled replicas in the last interval ----
+    # ---- complete destinations and replay of every plan-based replica and one P2C replica ----
     reps = cfg.replicas
-    rng = np.random.default_rng(7)
-    sample = sorted(set(rng.choice(len(reps), size=min(2, len(reps)), replace=False).tolist()))
-    iv = ivs[tp]
-    for i in sample:
-        pol, seed = reps[i]
-        d, _ = O.route([per_rep[i]], [pol], [seed], cfg.R, okeys[tp], iv.g0, 1024)
-        assert (dests[tp][i] == d[0]).all(), f"replica {reps[i]}: destinations differ"
+    plan_based = [i for i, (p, _) in enumerate(reps) if OP.VARIANT_OF.get(p) is not None]
+    p2c = [i for i, (p, _) in enumerate(reps) if p == "P2C"][:1]
+    checked = plan_based + p2c
+    assert plan_based, "every configuration has CacheRoute replicas"
+    plans_t = [OP.plans_for_interval(tr, okeys[t - 1] if t > 0 else okeys[0], t)[0] for t in range(nint)]
 
-    # ---- complete replay of one sampled replica over both intervals -------------
-    i = sample[0]
-    pol, seed = reps[i]
-    orp = O.Replay(1, cfg.R, cfg.caps)
-    for t in range(nint):
-        pr, _ = OP.plans_for_interval(tr, okeys[t - 1] if t > 0 else okeys[0], t)
-        d, _ = O.route([pr[i]], [pol], [seed], cfg.R, okeys[t], ivs[t].g0, 1024)
-        orp.step(okeys[t], ivs[t].plen, ivs[t].slen, d)
-    assert (ctr[i] == orp.ctr[0]).all(), f"replica {reps[i]}: replay counters differ"
+    def one_replica(i):
+        pol, seed = reps[i]
+        pol = OP.ROUTE_AS.get(pol, pol)
+        orp = O.Replay(1, cfg.R, cfg.caps)
+        bad = []
+        for t in range(nint):
+            d, _ = O.route([plans_t[t][i]], [pol], [seed], cfg.R, okeys[t], ivs[t].g0, 1024)
+            if not (dests[t][i] == d[0]).all():
+                bad.append(f"interval {t}: {int((dests[t][i] != d[0]).sum())} destinations differ")
+            orp.step(okeys[t], ivs[t].plen, ivs[t].slen, d)
+        if not (ctr[i] == orp.ctr[0]).all():
+            bad.append("replay counters differ")
+        return i, bad
+
+    import concurrent.futures as cf
+    import os
+    with cf.ThreadPoolExecutor(max_workers=min(len(checked), os.cpu_count() or 1)) as ex:
+        for i, bad in ex.map(one_replica, checked):
+            assert not bad, f"replica {reps[i]}: {'; '.join(bad)}"
 
     # ---- properties of every replica -------------------------------------------
     n_all = sum(iv.n for iv in ivs)

@@ -416,6 +416,41 @@ def test_replay_parity(P, ctx, caps):
                 assert (st[:c] == orp.state(rep, c_i, r)).all()
 
 
+@pytest.mark.parametrize("nkeys", [1500, 6000])
+def test_replay_parity_long_streams(P, ctx, nkeys):
+    # streams far longer than any chunk the replay splits work into (> 16,384 requests per
+    # stream per call), at the Large configuration's capacities: the state each chunk starts
+    # from must be rebuilt exactly, in both calls (the second starts from persisted state)
+    rng = np.random.default_rng(nkeys)
+    caps = [64, 256, 1024]
+    n_rep, R = 2, 2
+    keys = _rates_keys(rng, nkeys, 130000, skew=0.9)
+    n = keys.size
+    plen = rng.integers(16, 5000, size=n).astype(np.uint32)
+    slen = np.full(n, 64, np.uint32)
+    dest = tg.random_dest(n_rep, n, R, 11)
+    orp = O.Replay(n_rep, R, caps)
+    rp = P.Replay(ctx, n_rep, R, caps)
+    ctr = torch.zeros((n_rep, len(caps), R, 5), dtype=torch.int64, device=DEV)
+    dk, dp, ds, dd = d_u64(keys), d_u32(plen), d_u32(slen), d_u16(dest)
+    cut = n // 3
+    for a, b in ((0, cut), (cut, n)):
+        per_stream = np.bincount(dest[0, a:b], minlength=R)
+        assert per_stream.min() > 16384
+        orp.step(keys[a:b], plen[a:b], slen[a:b], dest[:, a:b])
+        P.shadow_replay(ctx, rp, dk[a:b].contiguous(), dp[a:b].contiguous(), ds[a:b].contiguous(),
+                        dd[:, a:b].contiguous(), ctr)
+        ctx.sync()
+        got = h_u64(ctr)
+        assert (got == orp.ctr).all()
+        assert 0 < got[:, 0, :, 1].sum() < got[:, 2, :, 1].sum() < got[:, 2, :, 0].sum()  # hits differ by cap
+    for rep in range(n_rep):
+        for r in range(R):
+            st = rp.state(rep, r)
+            for c_i, c in enumerate(caps):
+                assert (st[:c] == orp.state(rep, c_i, r)).all()
+
+
 def test_replay_reset_and_bad_dest(P, ctx):
     rp = P.Replay(ctx, 1, 4, [8])
     keys = d_u64(np.arange(10, dtype=np.uint64))
@@ -730,21 +765,27 @@ def test_pipeline_parity_slotcap_policy(P, ctx):
     assert (h_u64(pipe.ctr) == ref["ctr"]).all()
 
 
-def test_pipeline_split_routing_on_sm_partition(P, ctx):
+@pytest.mark.parametrize("B,chwbl", [(1024, False), (1024, True), (1, True)])
+def test_pipeline_split_routing_on_sm_partition(P, ctx, B, chwbl):
     # hashing and candidates on the large SM partition, the route resolution on the small one
-    # (green contexts): same destinations and counters as the oracle
+    # (green contexts): same destinations and counters as the oracle, with the CTA resolution
+    # (B = 1024) and the one-warp exact-sequential one (B = 1), with and without bounded-load
+    # (ring) replicas
+    import dataclasses
     from paper_2608_19677_gb300.pipeline import Pipeline
     try:
         part = P.Partition(0, 16)
     except P.CacheRouteError as e:
         pytest.skip(f"no SM partition on this driver: {e}")
-    cfg = tg.CONFIGS["70b"].scaled(40000, 4)
+    cfg = tg.CONFIGS["70b"].scaled(40000 if B > 1 else 12000, 4 if B > 1 else 2)
+    if chwbl:
+        cfg = dataclasses.replace(cfg, policies=["CR", "P2C", "CHWBL"], seeds=[0, 1])
     tr = tg.Trace(cfg)
-    ref = OP.run_trace(tr, B=1024, keep=True)
+    ref = OP.run_trace(tr, B=B, keep=True)
     with torch.cuda.stream(part.big):
         pctx = P.Context(0, part.big)
-        pipe = Pipeline(pctx, cfg.R, cfg.W, cfg.caps, cfg.replicas, tr.qcap, batch_B=1024, overlap=True,
-                        resolve_stream=part.small)
+        pipe = Pipeline(pctx, cfg.R, cfg.W, cfg.caps, cfg.replicas, tr.qcap, batch_B=B, overlap=True,
+                        resolve_stream=part.small, vnodes=cfg.vnodes)
         for t in range(cfg.n_intervals):
             iv = tr.interval(t)
             tok, off = tg.arena_host(tr, iv, 4)
@@ -754,6 +795,30 @@ def test_pipeline_split_routing_on_sm_partition(P, ctx):
             assert (h_u16(pipe.last_dest) == ref["dest"][t]).all()
         pipe.sync()
         assert (h_u64(pipe.ctr) == ref["ctr"]).all()
-    del pipe  # contexts on the partition's streams go before the partition
+    pipe.close()  # what uses the partition's streams goes before the partition
     pctx.close()
     part.close()
+
+
+def test_split_route_error_reported_by_sync(P):
+    # a bounded-load replica whose load sum has wrapped past 2^64 leaves no destination below
+    # cap: the resolution, enqueued on the resolve stream, raises the overflow flag, and the
+    # next cr_sync must report it even though the context's own stream finished first
+    c = P.Context(0)
+    side = torch.cuda.Stream(DEV)
+    try:
+        R = 2
+        ring = P.Ring(c, R, 4, 3)
+        P.set_resolve_stream(c, side)
+        keys = d_u64(np.arange(1, 65, dtype=np.uint64))
+        # loads 2^63 and 2^63 + 2: their sum wraps to 2, so cap = ceil(5 * 3 / 8) = 2 < both
+        load = d_u64(np.array([[2 ** 63, 2 ** 63 + 2]], np.uint64))
+        P.route_batch(c, [None], ["CHWBL"], [5], R, keys, 0, 64, load, rings=[ring])
+        with pytest.raises(P.CacheRouteError) as ei:
+            c.sync()
+        assert ei.value.code == P.CR_EOVERFLOW
+        c.sync()   # reported once, then cleared
+        P.set_resolve_stream(c, None)
+        ring.close()
+    finally:
+        c.close()

@@ -233,3 +233,54 @@ def test_replay_counters_destinations_and_persistence():
                 assert c[rp, ci, r, 1] == sum(1 for d in sd if d is not None and d <= caps[ci])
                 hit_tok = sum(int(p) for p, d in zip(plen[sel], sd) if d is not None and d <= caps[ci])
                 assert c[rp, ci, r, 2] == hit_tok
+
+
+def _jump_hash_float(keys: np.ndarray, R: np.ndarray) -> np.ndarray:
+    """Lamping and Veach's published jump consistent hash, restated with its
+    floating-point bucket jump j = (b + 1) * (2^31 / ((key >> 33) + 1)) in IEEE
+    doubles (numpy, vectorised over keys): an independent statement of the
+    linear congruential step and of the jump that the oracle evaluates exactly
+    in integers."""
+    k = keys.astype(np.uint64).copy()
+    R = R.astype(np.int64)
+    b = np.full(k.shape, -1, np.int64)
+    j = np.zeros(k.shape, np.int64)
+    live = j < R
+    with np.errstate(over="ignore"):
+        while live.any():
+            b[live] = j[live]
+            k[live] = k[live] * np.uint64(2862933555777941757) + np.uint64(1)
+            step = float(1 << 31) / ((k[live] >> np.uint64(33)).astype(np.float64) + 1.0)
+            j[live] = ((b[live] + 1).astype(np.float64) * step).astype(np.int64)
+            live = j < R
+    return b
+
+
+def test_jump_hash_matches_the_published_floating_point_algorithm():
+    # 100,000 keys at a random bucket count each, plus 200 keys at every bucket count
+    # 1..1024: the oracle's integer jump must pick the same bucket as the published
+    # algorithm (a wrong multiplier, increment or shift moves most keys)
+    rng = np.random.default_rng(2014)
+    keys = rng.integers(0, 1 << 63, size=100000, dtype=np.int64).astype(np.uint64) * np.uint64(2) + \
+        rng.integers(0, 2, size=100000).astype(np.uint64)
+    R = rng.integers(1, 1025, size=keys.size)
+    want = _jump_hash_float(keys, R)
+    got = np.array([O.jump_hash(int(k), int(r)) for k, r in zip(keys, R)], np.int64)
+    assert (got == want).all(), int((got != want).sum())
+    few = keys[:200]
+    allR = np.arange(1, 1025)
+    kk = np.repeat(few, allR.size)
+    rr = np.tile(allR, few.size)
+    want = _jump_hash_float(kk, rr)
+    got = np.array([O.jump_hash(int(k), int(r)) for k, r in zip(kk, rr)], np.int64)
+    assert (got == want).all(), int((got != want).sum())
+    # a planted change of the multiplier is caught by the same comparison
+    def planted(k, R):
+        b, j = -1, 0
+        while j < R:
+            b = j
+            k = (k * 2862933555777941759 + 1) & ((1 << 64) - 1)
+            j = int((b + 1) * (float(1 << 31) / float((k >> 33) + 1)))
+        return b
+    bad = np.array([planted(int(k), int(r)) for k, r in zip(keys[:2000], R[:2000])])
+    assert (bad != _jump_hash_float(keys[:2000], R[:2000])).mean() > 0.5
