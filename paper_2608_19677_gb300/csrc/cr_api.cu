@@ -245,6 +245,9 @@ extern "C" int cr_sync(cr_ctx *ctx)
             return cr_fail(ctx, CR_EOVERFLOW, "a load or counter exceeded its documented range");
         if (flags & CR_FLAG_TIMEOUT)
             return cr_fail(ctx, CR_ETIMEOUT, "a bounded device-side wait gave up");
+        if (flags & CR_FLAG_INTERNAL)
+            return cr_fail(ctx, CR_ECUDA, "a kernel found its state inconsistent (results of that call are not "
+                                          "meaningful)");
         if (flags & CR_FLAG_BADSIZE)
             return cr_fail(ctx, CR_EINVAL,
                            "token-weighted replay: a key came back with another prefix length (counters of "

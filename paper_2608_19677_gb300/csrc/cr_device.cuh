@@ -47,17 +47,29 @@ __device__ __forceinline__ uint32_t cr_scale(unsigned long long u, unsigned long
 }
 
 // Jump consistent hash (Lamping and Veach 2014) with the jump evaluated exactly
-// in integers: j = floor((b + 1) * 2^31 / ((k >> 33) + 1)).
+// in integers: j = floor((b + 1) * 2^31 / d), d = (k >> 33) + 1 in [1, 2^31].
+// No 64-bit division: a single-precision estimate of the quotient (relative
+// error below 2^-21) settles j >= R whenever it exceeds R + 2; otherwise it is
+// at most R + 2 <= 8194, its error is below 0.01, and one integer step either
+// way (products below 2^46) gives the exact floor.
 __device__ __forceinline__ uint32_t cr_jump_hash(unsigned long long k, uint32_t R)
 {
-    long long b = -1;
-    unsigned long long j = 0;
+    uint32_t b = 0, j = 0;
     while (j < R) {
-        b = (long long)j;
+        b = j;
         k = k * 2862933555777941757ull + 1ull;
-        j = ((unsigned long long)(b + 1) << 31) / ((k >> 33) + 1ull);
+        const uint32_t d = (uint32_t)(k >> 33) + 1u;
+        const unsigned long long num = (unsigned long long)(b + 1u) << 31;
+        const float est = (float)(b + 1u) * (2147483648.0f / (float)d);
+        if (est > (float)R + 2.0f) break;  // the exact quotient is above R as well
+        uint32_t q = (uint32_t)est;
+        if ((unsigned long long)q * d > num)
+            --q;
+        else if ((unsigned long long)(q + 1u) * d <= num)
+            ++q;
+        j = q;
     }
-    return (uint32_t)b;
+    return b;
 }
 
 __device__ __forceinline__ unsigned long long cr_warp_sum_u64(unsigned long long v)

@@ -13,6 +13,7 @@
 #define CR_FLAG_BADDEST 2u   // a destination index >= R reached the replay
 #define CR_FLAG_TIMEOUT 4u   // a bounded wait gave up
 #define CR_FLAG_BADSIZE 8u   // token-weighted replay: a key came back with another prefix length
+#define CR_FLAG_INTERNAL 16u // a kernel found its own state inconsistent and skipped the access
 
 // ---- scratch slots owned by the context ------------------------------------
 enum cr_scratch_slot {

@@ -4,9 +4,9 @@
 //              (replica, destination) stream's (key, prefix, suffix) records
 //              in arrival order
 //   replay     one warp per (stream, chunk); the stream's LRU at the LARGEST
-//              capacity lives in shared memory as keys in recency order with
-//              a hash index, and 32 requests are simulated per step, one per
-//              lane.  A request's depth (its LRU stack distance) decides the
+//              capacity lives in shared memory as keys with recency stamps, a
+//              bitmap of live stamps and a hash index, and 32 requests are
+//              simulated per step, one per lane.  A request's depth (its LRU stack distance) decides the
 //              hit at every smaller capacity at once, because LRU caches are
 //              nested (Mattson et al. 1970): the cache of capacity c is the c
 //              most recent entries of any larger one.
@@ -156,121 +156,258 @@ struct replay_state {
     uint32_t *fill_out;
 };
 
-// ---- replay: batched stack distances ------------------------------------------
-// One warp per (stream, chunk) holds the LRU of the largest capacity as keys in
-// recency order, K[0] most recent, in shared memory, with an open-addressing
-// index key -> physical slot (u16, slot + 1, 0 = empty, tombstones for evicted
-// keys, rebuilt when a quarter of it is tombstones).  The keys form a ring:
-// recency position q (0 = most recent) is slot (H + q) mod cmax.  A batch is
-// 32 consecutive requests, one per lane.  The depth of
+// ---- replay: batched stack distances over recency stamps -----------------------
+// One warp per (stream, chunk) holds the LRU of the LARGEST capacity in shared
+// memory.  Each resident key has a slot holding the key and its STAMP, the
+// time of its last access, and an entry in an open-addressing index
+// key -> slot.  Time advances by one 32-bit word per step of 32 requests (the
+// request on lane l of the step at word w has time 32 w + l), and a bitmap
+// over the times of a window marks the live stamps: bit t is set iff t is the
+// stamp of a resident key.  The recency position of a resident key (0 = most
+// recent) is the number of live bits above its stamp, which one warp-wide scan
+// of the words' popcounts gives for every lane of a step at once.  Nothing
+// moves when a key is accessed: its old bit is cleared and its bit in the new
+// word set.  When the window's words are used up, the stamps are renumbered
+// 0 .. fill-1 in recency order (compaction).
+//
+// A step is 32 consecutive requests of the stream, one per lane.  The depth of
 // request i (its LRU stack distance, Mattson et al. 1970) follows from the
-// state before the batch and the batch itself:
-//   - key seen earlier in the batch, last at lane j: 1 + the number of
-//     distinct keys among lanes (j, i);
-//   - first time in the batch, at position d0 before it: d0 + 1 + the number
-//     of distinct keys among lanes < i that were deeper than d0 or absent;
-//   - absent before the batch: a miss at every capacity.
-// A request hits capacity c iff its depth <= c.  The state after the batch is
-// the batch's distinct keys by last access (latest first) followed by the
-// untouched old keys in their old order, cut at cmax.  Old keys below the
-// deepest one the batch touched move (in place); those beyond it all shift by
-// the same amount, which moving the head H does, so they stay where they are.
+// state before the step and the step itself:
+//   - key seen earlier in the step, last at lane j: 1 + the number of distinct
+//     keys among lanes (j, i), at most 31;
+//   - first time in the step, at recency position d0 before it: d0 + 1 + the
+//     number of distinct keys among lanes < i that were deeper than d0 or
+//     absent;
+//   - absent before the step: a miss at every capacity.
+// A request hits capacity c iff its depth <= c.  The state after the step is
+// the step's distinct keys by last access, then the untouched old keys in
+// their old order, cut at cmax: when the step brings m new keys and the cache
+// would exceed cmax, the oldest untouched keys (the lowest live bits) leave
+// and the new keys take their slots.
 constexpr uint32_t kNone = 0xffffffffu;
-constexpr uint16_t kTomb = 0xffffu;  // index slot whose key was evicted
+constexpr uint16_t kTomb = 0xffffu;    // index entry whose key was evicted
+constexpr uint32_t kAbsent = 2047u;    // depth code of a key not resident (above every position < 1024)
 
-struct lru_index {
-    unsigned long long *K;  // [cmax] keys: a ring, recency position q at slot (H + q) mod cmax
-    uint16_t *TS;           // [cmax] index slot of the key in each ring slot
-    uint16_t *tab;          // [tsz] ring slot + 1; 0 = empty, kTomb = evicted
-    uint32_t *bm;           // [32] bitmap of old positions touched by the batch
+struct stamp_lru {
+    unsigned long long *K;  // [cmax] key of each slot
+    uint32_t *BM;           // [nw] live-stamp bits, word w = times 32 w .. 32 w + 31
+    uint16_t *tab;          // [tsz] slot + 1; 0 = empty, kTomb = evicted
+    uint16_t *ST;           // [cmax] stamp of each slot
+    uint16_t *T2S;          // [32 nw] slot whose stamp is each time (where the bit is set)
+    uint16_t *EV;           // [32] slots the step's evictions freed
     uint32_t mask;
     int tbits;
 };
 
-__device__ __forceinline__ uint32_t lru_home(unsigned long long key, int tbits) { return (uint32_t)(key >> (64 - tbits)); }
-
-// Ring slot of `key` (kNone if absent); *slot gets its index slot.
-__device__ __forceinline__ uint32_t lru_lookup(const lru_index &X, unsigned long long key, uint32_t *slot)
+// Per-warp layout: K at 0 (8-byte entries), BM after it, the index at the next
+// 16-byte boundary (it is cleared with 16-byte stores), then ST, T2S and EV.
+__host__ __device__ inline size_t stamp_tab_offset(uint32_t cmax, uint32_t nw)
 {
-    uint32_t s = lru_home(key, X.tbits);
-    for (;;) {
-        const uint32_t e = X.tab[s];
-        if (e == 0) return kNone;
-        if (e != kTomb && X.K[e - 1] == key) {
-            *slot = s;
-            return e - 1;
-        }
-        s = (s + 1) & X.mask;
-    }
+    return ((size_t)cmax * 8 + (size_t)nw * 4 + 15) & ~(size_t)15;
 }
 
-// Claim an empty or evicted slot for an absent key; returns the slot.
-__device__ __forceinline__ uint32_t lru_insert(const lru_index &X, unsigned long long key, uint32_t pos)
+__host__ __device__ inline size_t stamp_lru_bytes(uint32_t cmax, uint32_t nw, uint32_t tsz)
+{
+    return (stamp_tab_offset(cmax, nw) + (size_t)tsz * 2 + (size_t)cmax * 2 + (size_t)nw * 64 + 64 + 15) &
+           ~(size_t)15;
+}
+
+__device__ __forceinline__ stamp_lru stamp_lru_at(unsigned char *base, uint32_t cmax, uint32_t nw, int tbits)
+{
+    const uint32_t tsz = 1u << tbits;
+    stamp_lru X;
+    X.K = reinterpret_cast<unsigned long long *>(base);
+    X.BM = reinterpret_cast<uint32_t *>(base + (size_t)cmax * 8);
+    X.tab = reinterpret_cast<uint16_t *>(base + stamp_tab_offset(cmax, nw));
+    X.ST = X.tab + tsz;
+    X.T2S = X.ST + cmax;
+    X.EV = X.T2S + (size_t)nw * 32;
+    X.mask = tsz - 1;
+    X.tbits = tbits;
+    return X;
+}
+
+__device__ __forceinline__ uint32_t lru_home(unsigned long long key, int tbits) { return (uint32_t)(key >> (64 - tbits)); }
+
+// Slot of `key`, or kNone.  The index always has empty entries (at most three
+// quarters are live or evicted when a step starts), so the probe ends at one;
+// the bound only guards against a corrupted index.
+__device__ __forceinline__ uint32_t sl_lookup(const stamp_lru &X, unsigned long long key)
+{
+    uint32_t s = lru_home(key, X.tbits);
+    for (uint32_t it = 0; it <= X.mask; ++it) {
+        const uint32_t e = X.tab[s];
+        if (e == 0) return kNone;
+        if (e != kTomb && X.K[e - 1] == key) return e - 1;
+        s = (s + 1) & X.mask;
+    }
+    return kNone;
+}
+
+// Index an absent key held in slot q; returns 1 when it took an evicted entry's
+// place.  A lost compare-and-swap means another lane filled the entry, so the
+// next look moves on; the bound only guards against a corrupted index.
+__device__ __forceinline__ uint32_t sl_insert(const stamp_lru &X, unsigned long long key, uint32_t q)
 {
     unsigned short *t = reinterpret_cast<unsigned short *>(X.tab);
     uint32_t s = lru_home(key, X.tbits);
-    for (;;) {
+    for (uint32_t it = 0; it <= 2 * X.mask + 1; ++it) {
         const unsigned short v = t[s];
         if (v == 0 || v == kTomb) {
-            if (atomicCAS(&t[s], v, (unsigned short)(pos + 1)) == v) return s;
-            continue;  // lost the slot to another lane: look at it again
+            if (atomicCAS(&t[s], v, (unsigned short)(q + 1)) == v) return v == kTomb ? 1u : 0u;
+            continue;  // another lane took it: look at it again
+        }
+        s = (s + 1) & X.mask;
+    }
+    return 0;
+}
+
+// Turn the index entry of slot q (key K[q]) into a tombstone.
+__device__ __forceinline__ void sl_erase(const stamp_lru &X, uint32_t q)
+{
+    uint32_t s = lru_home(X.K[q], X.tbits);
+    for (uint32_t it = 0; it <= X.mask; ++it) {
+        if (X.tab[s] == q + 1) {
+            X.tab[s] = kTomb;
+            return;
         }
         s = (s + 1) & X.mask;
     }
 }
 
-__device__ __forceinline__ uint32_t ring_slot(uint32_t H, uint32_t q, uint32_t cmax)
-{
-    const uint32_t x = H + q;  // H < cmax, q < 2 cmax
-    return x >= cmax ? (x - cmax >= cmax ? x - 2 * cmax : x - cmax) : x;
-}
-
-// Index of the fill keys from ring slot H on, from scratch (warp-cooperative);
-// clears every tombstone.
-__device__ __forceinline__ void lru_reindex(const lru_index &X, uint32_t H, uint32_t fill, uint32_t cmax,
-                                            uint32_t lane)
+// Index of slots 0 .. fill-1 from scratch (warp-cooperative); clears every tombstone.
+__device__ __forceinline__ void sl_reindex(const stamp_lru &X, uint32_t fill, uint32_t lane)
 {
     uint4 *t4 = reinterpret_cast<uint4 *>(X.tab);
     for (uint32_t x = lane; x < (X.mask + 1) / 8; x += 32) t4[x] = make_uint4(0, 0, 0, 0);
     __syncwarp();
-    for (uint32_t q = lane; q < fill; q += 32) {
-        const uint32_t ph = ring_slot(H, q, cmax);
-        X.TS[ph] = (uint16_t)lru_insert(X, X.K[ph], ph);
-    }
+    for (uint32_t q = lane; q < fill; q += 32) sl_insert(X, X.K[q], q);
     __syncwarp();
 }
 
-template <int NC>
+// Stamps for keys K[0 .. fill) held in recency order (K[0] most recent): times
+// fill-1 .. 0, bits 0 .. fill-1 set, the next step at the first word above them.
+__device__ __forceinline__ void sl_stamps_in_order(const stamp_lru &X, uint32_t fill, uint32_t nw, uint32_t lane,
+                                                   uint32_t &wnow, uint32_t &lo)
+{
+    for (uint32_t q = lane; q < fill; q += 32) {
+        const uint32_t t = fill - 1u - q;
+        X.ST[q] = (uint16_t)t;
+        X.T2S[t] = (uint16_t)q;
+    }
+    for (uint32_t w = lane; w < nw; w += 32)
+        X.BM[w] = 32u * w + 32u <= fill ? 0xffffffffu : (32u * w < fill ? (1u << (fill - 32u * w)) - 1u : 0u);
+    wnow = (fill + 31u) / 32u;
+    lo = 0;
+    __syncwarp();
+}
+
+__device__ __forceinline__ uint32_t warp_incl_scan(uint32_t v, uint32_t lane)
+{
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        const uint32_t y = __shfl_up_sync(0xffffffffu, v, o);
+        if (lane >= (uint32_t)o) v += y;
+    }
+    return v;
+}
+
+// Position of the k-th (from 0) set bit of w, which has more than k set bits.
+__device__ __forceinline__ uint32_t nth_set_bit(uint32_t w, uint32_t k)
+{
+    uint32_t pos = 0;
+#pragma unroll
+    for (int sh = 16; sh >= 1; sh >>= 1) {
+        const uint32_t lowc = (uint32_t)__popc(w & ((1u << sh) - 1u));
+        if (k >= lowc) {
+            k -= lowc;
+            w >>= sh;
+            pos += (uint32_t)sh;
+        }
+    }
+    return pos;
+}
+
+// Live stamps below any time of the window: lane l keeps word 32 g + l of every
+// group g of 32 words and the number of live bits in the words before it.
+template <int NG>
+struct live_prefix {
+    uint32_t w[NG], ex[NG];
+    __device__ __forceinline__ void load(const uint32_t *BM, uint32_t nw, uint32_t lane)
+    {
+        uint32_t run = 0;
+#pragma unroll
+        for (int g = 0; g < NG; ++g) {
+            const uint32_t wi = 32u * g + lane;
+            w[g] = wi < nw ? BM[wi] : 0u;
+            const uint32_t pc = (uint32_t)__popc(w[g]);
+            const uint32_t incl = warp_incl_scan(pc, lane);
+            ex[g] = run + incl - pc;
+            run += __shfl_sync(0xffffffffu, incl, 31);
+        }
+    }
+    // live stamps < s; every lane of the warp must call it
+    __device__ __forceinline__ uint32_t below(uint32_t s) const
+    {
+        const uint32_t src = (s >> 5) & 31u, g = s >> 10;
+        uint32_t e = 0, b = 0;
+#pragma unroll
+        for (int gg = 0; gg < NG; ++gg) {
+            const uint32_t ee = __shfl_sync(0xffffffffu, ex[gg], src), bb = __shfl_sync(0xffffffffu, w[gg], src);
+            if (g == (uint32_t)gg) {
+                e = ee;
+                b = bb;
+            }
+        }
+        return e + (uint32_t)__popc(b & ((1u << (s & 31u)) - 1u));
+    }
+};
+
+// Renumber the stamps of slots 0 .. fill-1 to 0 .. fill-1 keeping their order.
+template <int NG>
+__device__ __forceinline__ void sl_compact(const stamp_lru &X, uint32_t fill, uint32_t nw, uint32_t lane,
+                                           uint32_t &wnow, uint32_t &lo)
+{
+    live_prefix<NG> LP;
+    LP.load(X.BM, nw, lane);
+    for (uint32_t q0 = 0; q0 < fill; q0 += 32) {
+        const uint32_t q = q0 + lane;
+        const uint32_t nb = LP.below(q < fill ? (uint32_t)X.ST[q] : 0u);
+        if (q < fill) {
+            X.ST[q] = (uint16_t)nb;
+            X.T2S[nb] = (uint16_t)q;
+        }
+    }
+    for (uint32_t w = lane; w < nw; w += 32)
+        X.BM[w] = 32u * w + 32u <= fill ? 0xffffffffu : (32u * w < fill ? (1u << (fill - 32u * w)) - 1u : 0u);
+    wnow = (fill + 31u) / 32u;
+    lo = 0;
+    __syncwarp();
+}
+
+template <int NC, int NG, bool SMALL>
 __global__ void __launch_bounds__(128)
-k_lru_batch(const replay_caps caps, uint32_t cmax, uint32_t R, uint32_t ns, uint32_t CL, int tbits,
+k_lru_stamp(const replay_caps caps, uint32_t cmax, uint32_t nw, uint32_t R, uint32_t ns, uint32_t CL, int tbits,
             const uint32_t *__restrict__ start, const uint32_t *__restrict__ coff, const uint32_t *__restrict__ total,
-            const rec16 *__restrict__ rec, const replay_state st, unsigned long long *__restrict__ ctr)
+            const rec16 *__restrict__ rec, const replay_state st, unsigned long long *__restrict__ ctr,
+            uint32_t *status)
 {
     extern __shared__ uint4 smb[];
     const uint32_t lane = cr_lane(), warp = threadIdx.x >> 5, wpb = blockDim.x >> 5;
-    const uint32_t tsz = 1u << tbits;
-    // per-warp region: index (2*tsz bytes), bitmap (128), keys (8*cmax), slots (2*cmax)
-    const size_t per_warp = ((size_t)tsz * 2 + 128 + (size_t)cmax * 10 + 15) & ~(size_t)15;
-    unsigned char *base = reinterpret_cast<unsigned char *>(smb) + per_warp * warp;
-    lru_index X;
-    X.tab = reinterpret_cast<uint16_t *>(base);
-    X.bm = reinterpret_cast<uint32_t *>(base + (size_t)tsz * 2);
-    X.K = reinterpret_cast<unsigned long long *>(base + (size_t)tsz * 2 + 128);
-    X.TS = reinterpret_cast<uint16_t *>(base + (size_t)tsz * 2 + 128 + (size_t)cmax * 8);
-    X.mask = tsz - 1;
-    X.tbits = tbits;
+    const size_t per_warp = stamp_lru_bytes(cmax, nw, 1u << tbits);
+    const stamp_lru X = stamp_lru_at(reinterpret_cast<unsigned char *>(smb) + per_warp * warp, cmax, nw, tbits);
 
     const uint32_t w = blockIdx.x * wpb + warp;
     if (w >= *total) return;
-    uint32_t lo = 0, hi = ns;
-    while (hi - lo > 1) {
-        const uint32_t mid = (lo + hi) >> 1;
+    uint32_t lo_s = 0, hi_s = ns;
+    while (hi_s - lo_s > 1) {
+        const uint32_t mid = (lo_s + hi_s) >> 1;
         if (coff[mid] <= w)
-            lo = mid;
+            lo_s = mid;
         else
-            hi = mid;
+            hi_s = mid;
     }
-    const uint32_t s = lo, ci = w - coff[s];
+    const uint32_t s = lo_s, ci = w - coff[s];
     const uint32_t b = start[s], e = start[s + 1];
     const uint32_t p0 = b + ci * CL;
     const uint32_t p1 = (e - p0) < CL ? e : p0 + CL;
@@ -286,16 +423,16 @@ k_lru_batch(const replay_caps caps, uint32_t cmax, uint32_t R, uint32_t ns, uint
         return;
     }
 
-    // ---- state at p0 ------------------------------------------------------------
+    // ---- state at p0, in recency order in K[0 .. fill) ------------------------------
     uint32_t fill = 0;
+    sl_reindex(X, 0, lane);
     if (ci == 0) {
         for (uint32_t q = lane; q < fill_in; q += 32) X.K[q] = kin[q];
         fill = fill_in;
         __syncwarp();
-        lru_reindex(X, 0, fill, cmax, lane);
+        for (uint32_t q = lane; q < fill; q += 32) sl_insert(X, X.K[q], q);
     } else {
         // walk backwards collecting distinct keys, most recent first
-        lru_reindex(X, 0, 0, cmax, lane);
         const uint32_t back = p0 - b;
         const uint32_t vtot = back + fill_in;
         for (uint32_t v0 = 0; v0 < vtot && fill < cmax; v0 += 32) {
@@ -305,29 +442,29 @@ k_lru_batch(const replay_caps caps, uint32_t cmax, uint32_t R, uint32_t ns, uint
             if (valid) key = v < back ? rec[p0 - 1 - v].key : kin[v - back];
             const uint32_t vm = __ballot_sync(0xffffffffu, valid);
             const uint32_t peers = __match_any_sync(0xffffffffu, key) & vm;
-            uint32_t sl;
-            const bool fresh = valid && (peers & lt) == 0 && lru_lookup(X, key, &sl) == kNone;
+            const bool fresh = valid && (peers & lt) == 0 && sl_lookup(X, key) == kNone;
             const uint32_t bal = __ballot_sync(0xffffffffu, fresh);
             const uint32_t pos = fill + __popc(bal & lt);
             __syncwarp();
             if (fresh && pos < cmax) {
                 X.K[pos] = key;
-                X.TS[pos] = (uint16_t)lru_insert(X, key, pos);
+                sl_insert(X, key, pos);
             }
             fill = min(cmax, fill + (uint32_t)__popc(bal));
             __syncwarp();
         }
     }
+    __syncwarp();
+    uint32_t wnow, lo;
+    sl_stamps_in_order(X, fill, nw, lane, wnow, lo);
+    uint32_t tomb = 0;  // tombstones in the index
 
     unsigned long long my_req = 0, my_prompt = 0;
     unsigned long long my_hit[NC], my_tok[NC];
 #pragma unroll
     for (int c = 0; c < NC; ++c) my_hit[c] = my_tok[c] = 0;
-    const uint32_t nwords = (cmax + 31) / 32;
-    uint32_t tomb = 0;  // tombstones in the index
-    uint32_t H = 0;     // ring slot of recency position 0
 
-    rec16 ahead = {0ull, 0u, 0u};  // the next batch's records, loaded one batch early
+    rec16 ahead = {0ull, 0u, 0u};  // the next step's records, loaded one step early
     if (p0 + lane < p1) ahead = rec[p0 + lane];
     for (uint32_t t0 = p0; t0 < p1; t0 += 32) {
         const uint32_t cnt = (p1 - t0) < 32u ? (p1 - t0) : 32u;
@@ -342,19 +479,28 @@ k_lru_batch(const replay_caps caps, uint32_t cmax, uint32_t R, uint32_t ns, uint
         const uint32_t grp = __match_any_sync(0xffffffffu, mine.key) & vm;
         const uint32_t below = grp & lt, above = grp & gt;
         const bool first = valid && below == 0;
-        const uint32_t next = above ? (uint32_t)__ffs(above) - 1u : 32u;
-        uint32_t slot0 = kNone, d0 = kNone;
-        if (first) {
-            const uint32_t ph = lru_lookup(X, mine.key, &slot0);
-            if (ph != kNone) d0 = ph >= H ? ph - H : ph + cmax - H;  // recency position
+        const bool last = valid && above == 0;
+        uint32_t slot = first ? sl_lookup(X, mine.key) : kNone;
+        const bool res = slot != kNone;  // first occurrence of a resident key
+        uint32_t s_old = res ? (uint32_t)X.ST[slot] : 0u;
+        if (s_old >= 32u * nw) {  // never: stamps stay inside the window (guards the bitmap)
+            atomicOr(status, CR_FLAG_INTERNAL);
+            s_old = 0;
         }
+
+        // recency position at the step's start: live stamps above the key's
+        live_prefix<NG> LP;
+        LP.load(X.BM, nw, lane);
+        const uint32_t bl = LP.below(s_old);
+        const uint32_t D = res ? fill - 1u - bl : kAbsent;
         // lanes that push request i deeper, for every lane at once, by comparing
         // bit-sliced values from the most significant bit down (per bit: lanes
         // still equal keep the ones with the same bit; a lane whose bit is 1
         // where this lane's is 0 is decided greater):
-        //   repeat i: lanes whose key does not recur before i (next_l > i);
         //   first i:  first occurrences whose old position is deeper (D_l > D_i)
-        const uint32_t D = first ? (d0 < cmax ? d0 : 2047u) : 2047u;  // 2047: absent
+        //   repeat i: lanes whose key does not recur before i (next_l > i); only
+        //             needed below capacity 32 (a repeat's depth is at most 31)
+        const uint32_t next = above ? (uint32_t)__ffs(above) - 1u : 32u;
         uint32_t gN = 0, eN = 0xffffffffu, gD = 0, eD = 0xffffffffu;
 #pragma unroll
         for (int bt = 10; bt >= 0; --bt) {
@@ -362,7 +508,7 @@ k_lru_batch(const replay_caps caps, uint32_t cmax, uint32_t R, uint32_t ns, uint
             const uint32_t MD = 0u - ((D >> bt) & 1u);
             gD |= eD & BD & ~MD;
             eD &= ~(BD ^ MD);
-            if (bt <= 5) {
+            if (SMALL && bt <= 5) {
                 const uint32_t BN = __ballot_sync(0xffffffffu, (next >> bt) & 1u);
                 const uint32_t MN = 0u - ((lane >> bt) & 1u);
                 gN |= eN & BN & ~MN;
@@ -370,10 +516,12 @@ k_lru_batch(const replay_caps caps, uint32_t cmax, uint32_t R, uint32_t ns, uint
             }
         }
         const uint32_t firstm = __ballot_sync(0xffffffffu, first);
-        // repeat: lanes strictly between the previous occurrence and this one
-        const uint32_t win = lt & ~((2u << (31u - (uint32_t)__clz(below | 1u))) - 1u);
-        const uint32_t dep_rep = 1u + (uint32_t)__popc(gN & win);
-        const uint32_t dep_first = d0 < cmax ? d0 + 1u + (uint32_t)__popc(gD & firstm & lt) : kNone;
+        uint32_t dep_rep = 1u;
+        if (SMALL) {  // repeat: lanes strictly between the previous occurrence and this one
+            const uint32_t win = lt & ~((2u << (31u - (uint32_t)__clz(below | 1u))) - 1u);
+            dep_rep = 1u + (uint32_t)__popc(gN & win);
+        }
+        const uint32_t dep_first = res ? D + 1u + (uint32_t)__popc(gD & firstm & lt) : kNone;
         const uint32_t depth = !valid ? kNone : (first ? dep_first : dep_rep);
 #pragma unroll
         for (int c = 0; c < NC; ++c) {
@@ -383,89 +531,103 @@ k_lru_batch(const replay_caps caps, uint32_t cmax, uint32_t R, uint32_t ns, uint
             }
         }
 
-        // ---- state after the batch ------------------------------------------------
-        const uint32_t lastm = __ballot_sync(0xffffffffu, valid && above == 0);
+        // ---- state after the step ------------------------------------------------------
+        const uint32_t lastm = __ballot_sync(0xffffffffu, last);
         const uint32_t u = (uint32_t)__popc(lastm);
-        if (lane < nwords) X.bm[lane] = 0;
-        __syncwarp();
-        if (d0 != kNone) atomicOr(&X.bm[d0 >> 5], 1u << (d0 & 31));
-        __syncwarp();
-        const uint32_t wv = lane < nwords ? X.bm[lane] : 0u;
-        uint32_t pre = (uint32_t)__popc(wv);  // inclusive prefix over words
-#pragma unroll
-        for (int o = 1; o < 32; o <<= 1) {
-            const uint32_t y = __shfl_up_sync(0xffffffffu, pre, o);
-            if (lane >= (uint32_t)o) pre += y;
-        }
-        const uint32_t touched = __shfl_sync(0xffffffffu, pre, 31);
-        pre -= (uint32_t)__popc(wv);  // exclusive
-        // old keys up to the deepest touched one move back (never forward),
-        // highest block first, in place; each rewrites its index slot.  Those
-        // beyond it shift by delta = u - touched, done by moving the head.
-        const uint32_t pmax = __reduce_max_sync(0xffffffffu, d0 != kNone ? d0 + 1u : 0u);  // deepest + 1
-        const uint32_t delta = u - touched;
-        const uint32_t H2 = H >= delta % cmax ? H - delta % cmax : H + cmax - delta % cmax;
-        uint32_t evicted = 0;
-        for (int tb = (int)((pmax + 31) / 32) - 1; tb >= 0; --tb) {
-            const uint32_t p = (uint32_t)tb * 32u + lane;
-            const uint32_t wt = __shfl_sync(0xffffffffu, wv, tb), pt = __shfl_sync(0xffffffffu, pre, tb);
-            unsigned long long v = 0;
-            uint32_t np = kNone, ts = 0;
-            if (p < pmax && !((wt >> lane) & 1u)) {
-                const uint32_t ph = ring_slot(H, p, cmax);
-                v = X.K[ph];
-                ts = X.TS[ph];
-                np = p + u - (pt + (uint32_t)__popc(wt & lt));
-            }
+        const uint32_t absm = __ballot_sync(0xffffffffu, first && !res);
+        const uint32_t mnew = (uint32_t)__popc(absm);
+        if (SMALL && u > cmax) {
+            // more distinct keys than the capacity: every old key leaves and the
+            // cmax most recently used keys of the step form the cache
             __syncwarp();
-            if (np < cmax) {
-                const uint32_t ph = ring_slot(H2, np, cmax);
-                X.K[ph] = v;
-                X.TS[ph] = (uint16_t)ts;
-                X.tab[ts] = (uint16_t)(ph + 1);
-            } else if (np != kNone) {
-                X.tab[ts] = kTomb;
-                ++evicted;
+            sl_reindex(X, 0, lane);
+            for (uint32_t x = lane; x < nw; x += 32) X.BM[x] = 0;
+            __syncwarp();
+            const uint32_t rk = (uint32_t)__popc(lastm & gt);  // 0 = most recent
+            const bool keep = last && rk < cmax;
+            const uint32_t keepm = __ballot_sync(0xffffffffu, keep);
+            if (keep) {
+                const uint32_t t = wnow * 32u + lane;
+                X.K[rk] = mine.key;
+                sl_insert(X, mine.key, rk);
+                X.ST[rk] = (uint16_t)t;
+                X.T2S[t] = (uint16_t)rk;
             }
-        }
-        // old keys beyond the deepest touched one that the shift pushes past cmax
-        {
-            const uint32_t from = max(pmax, cmax > delta ? cmax - delta : 0u);
-            const uint32_t p = from + lane;
-            if (p < fill) {  // at most delta <= 32 of them
-                X.tab[X.TS[ring_slot(H, p, cmax)]] = kTomb;
-                ++evicted;
-            }
-        }
-        __syncwarp();
-        // the batch's distinct keys go to the front; a key already resident keeps
-        // its slot (taken from the lane of its first occurrence), a new one claims one
-        const uint32_t fl = (uint32_t)__ffs(grp ? grp : 1u) - 1u;
-        const uint32_t kslot = __shfl_sync(0xffffffffu, slot0, fl);
-        const uint32_t rank = (uint32_t)__popc(lastm & gt);
-        if (valid && above == 0) {
-            if (kslot != kNone) {
-                if (rank < cmax) {
-                    const uint32_t ph = ring_slot(H2, rank, cmax);
-                    X.K[ph] = mine.key;
-                    X.TS[ph] = (uint16_t)kslot;
-                    X.tab[kslot] = (uint16_t)(ph + 1);
-                } else {
-                    X.tab[kslot] = kTomb;
-                    ++evicted;
+            if (lane == 0) X.BM[wnow] = keepm;
+            fill = cmax;
+            tomb = 0;
+            lo = wnow;
+            ++wnow;
+        } else {
+            // touched keys leave their old time
+            if (res) atomicAnd(&X.BM[s_old >> 5], ~(1u << (s_old & 31u)));
+            __syncwarp();
+            // the oldest untouched keys leave until the cache fits: the lowest live
+            // bits, found 32 words at a time from the lowest word that has any
+            uint32_t need = fill + mnew > cmax ? fill + mnew - cmax : 0u;
+            uint32_t done = 0;
+            while (need && lo < wnow) {  // each pass ends the loop or moves lo up
+                const uint32_t wd = lo + lane;
+                const uint32_t word = wd < wnow ? X.BM[wd] : 0u;
+                const uint32_t pc = (uint32_t)__popc(word);
+                const uint32_t incl = warp_incl_scan(pc, lane);
+                const uint32_t tot = __shfl_sync(0xffffffffu, incl, 31);
+                const uint32_t take = min(need, tot);
+                uint32_t o = 0;  // the word holding this lane's bit: first lane whose prefix exceeds lane
+#pragma unroll
+                for (uint32_t stp = 16; stp >= 1; stp >>= 1) {
+                    const uint32_t v = __shfl_sync(0xffffffffu, incl, o + stp - 1u);
+                    if (v <= lane) o += stp;
                 }
-            } else if (rank < cmax) {
-                const uint32_t ph = ring_slot(H2, rank, cmax);
-                X.K[ph] = mine.key;
-                X.TS[ph] = (uint16_t)lru_insert(X, mine.key, ph);
+                const uint32_t exo = __shfl_sync(0xffffffffu, incl - pc, o & 31u);
+                const uint32_t wo = __shfl_sync(0xffffffffu, word, o & 31u);
+                const uint32_t olast = __shfl_sync(0xffffffffu, o, (take + 31u) & 31u);
+                __syncwarp();
+                if (lane < take) {
+                    const uint32_t bit = nth_set_bit(wo, lane - exo);
+                    uint32_t q = X.T2S[(lo + o) * 32u + bit];
+                    atomicAnd(&X.BM[lo + o], ~(1u << bit));
+                    if (q < cmax) {
+                        sl_erase(X, q);
+                    } else {  // never: a live time always maps to a slot (guards the arrays)
+                        atomicOr(status, CR_FLAG_INTERNAL);
+                        q = 0;
+                    }
+                    X.EV[done + lane] = (uint16_t)q;
+                }
+                lo = take == tot ? min(lo + 32u, wnow) : lo + olast;
+                need -= take;
+                done += take;
+                __syncwarp();
             }
+            tomb += done;
+            // new keys take the never-used slots, then the freed ones
+            uint32_t reused = 0;
+            if (first && !res) {
+                const uint32_t a = (uint32_t)__popc(absm & lt);
+                const uint32_t freecnt = cmax - fill;
+                const uint32_t q = a < freecnt ? fill + a : (uint32_t)X.EV[a - freecnt];
+                X.K[q] = mine.key;
+                reused = sl_insert(X, mine.key, q);
+                slot = q;
+            }
+            tomb -= __reduce_add_sync(0xffffffffu, reused);
+            // every key of the step takes the time of its last access
+            const uint32_t fl = (uint32_t)__ffs(grp ? grp : 1u) - 1u;
+            const uint32_t ks = __shfl_sync(0xffffffffu, slot, fl);
+            if (last) {
+                const uint32_t t = wnow * 32u + lane;
+                X.ST[ks] = (uint16_t)t;
+                X.T2S[t] = (uint16_t)ks;
+            }
+            if (lane == 0) X.BM[wnow] = lastm;
+            fill = min(cmax, fill + mnew);
+            ++wnow;
         }
-        H = H2;
-        fill = min(cmax, fill - touched + u);
-        tomb += __reduce_add_sync(0xffffffffu, evicted);
         __syncwarp();
+        if (wnow == nw) sl_compact<NG>(X, fill, nw, lane, wnow, lo);
         if (4 * (fill + tomb) > 3 * (X.mask + 1)) {  // too many tombstones: index afresh
-            lru_reindex(X, H, fill, cmax, lane);
+            sl_reindex(X, fill, lane);
             tomb = 0;
         }
     }
@@ -491,19 +653,33 @@ k_lru_batch(const replay_caps caps, uint32_t cmax, uint32_t R, uint32_t ns, uint
     // ---- the stream's last chunk hands the state to the next call, most recent first
     if (p1 == e) {
         unsigned long long *kout = st.keys_out + (unsigned long long)s * cmax;
-        for (uint32_t q = lane; q < fill; q += 32) kout[q] = X.K[ring_slot(H, q, cmax)];
+        live_prefix<NG> LP;
+        LP.load(X.BM, nw, lane);
+        for (uint32_t q0 = 0; q0 < fill; q0 += 32) {
+            const uint32_t q = q0 + lane;
+            const uint32_t nb = LP.below(q < fill ? (uint32_t)X.ST[q] : 0u);
+            if (q < fill && nb < fill) kout[fill - 1u - nb] = X.K[q];
+        }
         if (lane == 0) st.fill_out[s] = fill;
     }
 }
 
-template <int NC>
-int launch_batch_nc(cr_ctx *ctx, cr_replay *rp, const replay_caps &caps, uint32_t CL, const uint32_t *start,
-                    const uint32_t *coff, const uint32_t *total, uint64_t m, const rec16 *rec, uint64_t *d_ctr)
+// Words of the stamp window: the cmax stamps a compaction leaves plus at least
+// as many steps (and at least 8) before the next one.
+inline uint32_t stamp_words(uint32_t cmax)
 {
-    const uint32_t cmax = rp->cmax;
+    const uint32_t w0 = (cmax + 31) / 32;
+    return w0 + (w0 > 8 ? w0 : 8);
+}
+
+template <int NC, int NG, bool SMALL>
+int launch_stamp(cr_ctx *ctx, cr_replay *rp, const replay_caps &caps, uint32_t CL, const uint32_t *start,
+                 const uint32_t *coff, const uint32_t *total, uint64_t m, const rec16 *rec, uint64_t *d_ctr)
+{
+    const uint32_t cmax = rp->cmax, nw = stamp_words(cmax);
     int tbits = 6;
     while ((1u << tbits) < 4 * cmax) ++tbits;  // index at most a quarter full of live keys
-    const size_t per_warp = ((size_t)(1u << tbits) * 2 + 128 + (size_t)cmax * 10 + 15) & ~(size_t)15;
+    const size_t per_warp = stamp_lru_bytes(cmax, nw, 1u << tbits);
     // warps per block: the most warps per SM that shared memory allows
     const size_t sm_bytes = 227 * 1024;
     uint32_t wpb = 4, best = 0;
@@ -517,7 +693,8 @@ int launch_batch_nc(cr_ctx *ctx, cr_replay *rp, const replay_caps &caps, uint32_
     }
     const size_t smem = per_warp * wpb;
     if (smem > 48 * 1024)
-        CR_CUDA(ctx, cudaFuncSetAttribute(k_lru_batch<NC>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
+        CR_CUDA(ctx, cudaFuncSetAttribute(k_lru_stamp<NC, NG, SMALL>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                          (int)smem));
     const uint32_t ns = rp->n_rep * rp->R;
     const uint64_t items = (uint64_t)ns + (m + CL - 1) / CL;  // upper bound on work items
     replay_state st;
@@ -525,18 +702,32 @@ int launch_batch_nc(cr_ctx *ctx, cr_replay *rp, const replay_caps &caps, uint32_
     st.fill_in = rp->d_fill[rp->cur];
     st.keys_out = rp->d_keys[rp->cur ^ 1];
     st.fill_out = rp->d_fill[rp->cur ^ 1];
-    CR_LAUNCH(ctx, k_lru_batch<NC>, (unsigned int)((items + wpb - 1) / wpb), wpb * 32, smem, caps, cmax, rp->R, ns,
-              CL, tbits, start, coff, total, rec, st, (unsigned long long *)d_ctr);
+    CR_LAUNCH(ctx, (k_lru_stamp<NC, NG, SMALL>), (unsigned int)((items + wpb - 1) / wpb), wpb * 32, smem, caps, cmax,
+              nw, rp->R, ns, CL, tbits, start, coff, total, rec, st, (unsigned long long *)d_ctr, ctx->d_status);
     rp->cur ^= 1;
     return CR_OK;
+}
+
+template <int NC>
+int launch_stamp_nc(cr_ctx *ctx, cr_replay *rp, const replay_caps &caps, uint32_t CL, const uint32_t *start,
+                    const uint32_t *coff, const uint32_t *total, uint64_t m, const rec16 *rec, uint64_t *d_ctr)
+{
+    uint32_t cmin = 0xffffffffu;
+    for (uint32_t c = 0; c < caps.n_caps; ++c) cmin = caps.cap[c] < cmin ? caps.cap[c] : cmin;
+    const bool small = cmin < 32;  // a repeat within a step can miss only below capacity 32
+    if (stamp_words(rp->cmax) <= 32)
+        return small ? launch_stamp<NC, 1, true>(ctx, rp, caps, CL, start, coff, total, m, rec, d_ctr)
+                     : launch_stamp<NC, 1, false>(ctx, rp, caps, CL, start, coff, total, m, rec, d_ctr);
+    return small ? launch_stamp<NC, 2, true>(ctx, rp, caps, CL, start, coff, total, m, rec, d_ctr)
+                 : launch_stamp<NC, 2, false>(ctx, rp, caps, CL, start, coff, total, m, rec, d_ctr);
 }
 
 int launch_batch(cr_ctx *ctx, cr_replay *rp, const replay_caps &caps, uint32_t CL, const uint32_t *start,
                  const uint32_t *coff, const uint32_t *total, uint64_t m, const rec16 *rec, uint64_t *d_ctr)
 {
-    if (caps.n_caps == 1) return launch_batch_nc<1>(ctx, rp, caps, CL, start, coff, total, m, rec, d_ctr);
-    if (caps.n_caps <= 3) return launch_batch_nc<3>(ctx, rp, caps, CL, start, coff, total, m, rec, d_ctr);
-    return launch_batch_nc<CR_MAX_CAPS>(ctx, rp, caps, CL, start, coff, total, m, rec, d_ctr);
+    if (caps.n_caps == 1) return launch_stamp_nc<1>(ctx, rp, caps, CL, start, coff, total, m, rec, d_ctr);
+    if (caps.n_caps <= 3) return launch_stamp_nc<3>(ctx, rp, caps, CL, start, coff, total, m, rec, d_ctr);
+    return launch_stamp_nc<CR_MAX_CAPS>(ctx, rp, caps, CL, start, coff, total, m, rec, d_ctr);
 }
 
 // ---- token-weighted variant ---------------------------------------------------

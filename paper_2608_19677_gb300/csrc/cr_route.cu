@@ -76,7 +76,8 @@ __device__ __forceinline__ uint32_t p2c_pair(unsigned long long seed, uint32_t p
 {
     cr_u64x4 u = cr_philox4x64_10(g, 0ull, 0ull, 0ull, seed, (unsigned long long)policy);
     uint32_t d1 = cr_scale(u.x, R);
-    uint32_t d2 = (uint32_t)((d1 + 1ull + cr_scale(u.y, (unsigned long long)(R - 1))) % R);
+    uint32_t d2 = d1 + 1u + cr_scale(u.y, (unsigned long long)(R - 1));  // < 2R: one subtraction is mod R
+    if (d2 >= R) d2 -= R;
     return kPair | d1 | (d2 << 13);
 }
 

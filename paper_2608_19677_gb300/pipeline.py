@@ -345,3 +345,175 @@ class Pipeline:
     @property
     def launches(self) -> int:
         return sum(c.launches for c in self.contexts)
+
+
+class TracePipeline:
+    """Offline shadow replay of a whole trace whose routing keys are already on the device.
+
+    The plan of interval t depends only on interval t-1's keys, and routing
+    starts every interval from zero loads, so plans and routes of different
+    intervals are independent; only the replay, whose LRU state carries over,
+    must take the intervals in order.  This driver therefore keeps ``depth``
+    intervals in flight: plan builds go round-robin to ``plan_streams``
+    streams (each with its own library context and scratch), routing to
+    ``route_streams`` streams, and the replay of interval t follows its route
+    on one replay stream.  Plan and destination buffers are reused every
+    ``depth`` intervals, each reuse ordered by the event of its last reader.
+    The results equal the per-interval ``Pipeline``'s (same plans, routes and
+    counters); only the schedule differs.
+    """
+
+    def __init__(self, ctx: Context, R: int, W: int, caps: Sequence[int],
+                 replicas: Sequence[Tuple[str, int]], qcap: Callable[[int], Tuple[int, int]],
+                 max_n: int, batch_B: int = 1024, depth: int = 8, plan_streams: int = 4,
+                 route_streams: int = 4, vnodes: int = 64, fresh: bool = False, lru_tokens: bool = False):
+        import torch
+        self.ctx, self.R, self.W, self.caps = ctx, R, W, list(caps)
+        self.replicas = list(replicas)
+        self.qcap, self.B, self.fresh = qcap, batch_B, fresh
+        self.policies = [ROUTE_AS.get(p, p) for p, _ in self.replicas]
+        self.seeds = [s for _, s in self.replicas]
+        self.dev = torch.device("cuda", ctx.device)
+        self.plan_keys: List[Tuple[str, int]] = []
+        self.rep_plan: List[Optional[int]] = []
+        for p, s in self.replicas:
+            v = VARIANT_OF.get(p)
+            if v is None:
+                self.rep_plan.append(None)
+                continue
+            k = (v, s if v == "RANDOM" else 0)
+            if k not in self.plan_keys:
+                self.plan_keys.append(k)
+            self.rep_plan.append(self.plan_keys.index(k))
+        self.depth = max(1, depth)
+        self.mstream = ctx._stream_obj
+        lo, hi = torch.cuda.Stream.priority_range() if hasattr(torch.cuda.Stream, "priority_range") else (0, -1)
+        self.pstreams = [torch.cuda.Stream(self.dev, priority=hi) for _ in range(max(1, plan_streams))]
+        self.pctxs = [Context(ctx.device, s) for s in self.pstreams]
+        self.rstreams = [torch.cuda.Stream(self.dev) for _ in range(max(1, route_streams))]
+        self.rctxs = [Context(ctx.device, s) for s in self.rstreams]
+        self.ystream = torch.cuda.Stream(self.dev)
+        self.yctx = Context(ctx.device, self.ystream)
+        self.plans = [[Plan(self.pctxs[0]) for _ in self.plan_keys] for _ in range(self.depth)]
+        self.replay = Replay(ctx, len(self.replicas), R, self.caps, tokens=lru_tokens)
+        self.rings = [Ring(ctx, R, vnodes, s) if p == "CHWBL" else None for p, s in self.replicas]
+        nrep = len(self.replicas)
+        self.ctr = torch.zeros((nrep, len(self.caps), R, 5), dtype=torch.int64, device=self.dev)
+        self.loads = [torch.zeros((nrep, R), dtype=torch.int64, device=self.dev) for _ in self.rstreams]
+        self.max_n = max_n
+        self.dests = [torch.empty(nrep * max_n, dtype=torch.int16, device=self.dev) for _ in range(self.depth)]
+        ctx.sync()
+        self._reset_events()
+        self.plan_marks, self.route_marks, self.replay_marks = [], [], []
+
+    def _reset_events(self):
+        self._plan_free = [None] * self.depth   # route that last read plans buffer b
+        self._dest_free = [None] * self.depth   # replay that last read destinations buffer b
+        self._load_free = [None] * len(self.rstreams)
+
+    @property
+    def contexts(self):
+        return [self.ctx] + self.pctxs + self.rctxs + [self.yctx]
+
+    @property
+    def launches(self) -> int:
+        return sum(c.launches for c in self.contexts)
+
+    def _event(self, stream, timing=False):
+        import torch
+        e = torch.cuda.Event(enable_timing=timing)
+        e.record(stream)
+        return e
+
+    def dest_view(self, b: int, n: int):
+        return self.dests[b][:len(self.replicas) * n].view(len(self.replicas), n)
+
+    def run(self, keys, plens, slens, g0s, mark: bool = False, on_interval=None):
+        """Enqueue every interval of the trace (lists of device tensors and first request
+        indices) after the work already on the main stream; the main stream then waits for
+        all of it.  Counters accumulate in ``ctr`` (call ``reset`` between runs).
+        ``on_interval(t, dest, plans)``, when given, is called after interval t is enqueued
+        with its destinations view and plans (a test hook: the caller must order its reads
+        after the pipeline's streams, e.g. by ``sync``, before the buffer's reuse)."""
+        import torch
+        T = len(keys)
+        start = self._event(self.mstream)
+        for s in self.pstreams + self.rstreams + [self.ystream]:
+            s.wait_event(start)
+        self.plan_marks, self.route_marks, self.replay_marks = [], [], []
+        for t in range(T):
+            n = int(keys[t].shape[0])
+            if n > self.max_n:
+                raise ValueError(f"interval {t} has {n} requests, more than max_n={self.max_n}")
+            b = t % self.depth
+            # ---- plans of interval t (from interval t-1's keys; interval 0 from its own) ----
+            plans = None
+            if self.plan_keys:
+                ps = self.pstreams[t % len(self.pstreams)]
+                pc = self.pctxs[t % len(self.pctxs)]
+                if self._plan_free[b] is not None:
+                    ps.wait_event(self._plan_free[b])
+                pk = keys[t] if (t == 0 or self.fresh) else keys[t - 1]
+                num, den = self.qcap(int(pk.shape[0]))
+                params = [plan_params(self.R, self.W, num, den, v, seed=s, epoch=t) for v, s in self.plan_keys]
+                p0 = self._event(ps, True) if mark else None
+                build_plans(pc, pk, params, self.plans[b])
+                ready = self._event(ps, mark)
+                if mark:
+                    self.plan_marks.append((p0, ready))
+                plans = [self.plans[b][i] if i is not None else None for i in self.rep_plan]
+            # ---- route of interval t ---------------------------------------------------
+            q = t % len(self.rstreams)
+            rs, rc = self.rstreams[q], self.rctxs[q]
+            if plans is not None:
+                rs.wait_event(ready)
+            if self._dest_free[b] is not None:
+                rs.wait_event(self._dest_free[b])
+            dest = self.dest_view(b, n)
+            r0 = self._event(rs, True) if mark else None
+            with torch.cuda.stream(rs):
+                self.loads[q].zero_()
+            route_batch(rc, plans if plans is not None else [None] * len(self.replicas), self.policies,
+                        self.seeds, self.R, keys[t], g0s[t], self.B, self.loads[q], dest, rings=self.rings)
+            routed = self._event(rs, mark)
+            if mark:
+                self.route_marks.append((r0, routed))
+            self._plan_free[b] = routed
+            # ---- replay, in interval order ----------------------------------------------
+            self.ystream.wait_event(routed)
+            y0 = self._event(self.ystream, True) if mark else None
+            shadow_replay(self.yctx, self.replay, keys[t], plens[t], slens[t], dest, self.ctr)
+            replayed = self._event(self.ystream, mark)
+            if mark:
+                self.replay_marks.append((y0, replayed))
+            self._dest_free[b] = replayed
+            if on_interval is not None:
+                on_interval(t, dest, self.plans[b] if self.plan_keys else [])
+        for s in self.pstreams + self.rstreams + [self.ystream]:
+            self.mstream.wait_event(self._event(s))
+
+    def reset(self):
+        """Empty the simulators and counters (ordered on the main stream after earlier work)."""
+        import torch
+        self.sync()
+        self.replay.reset()
+        with torch.cuda.stream(self.mstream):
+            self.ctr.zero_()
+        self.ctx.sync()
+        self._reset_events()
+
+    def sync(self):
+        for c in self.contexts:
+            c.sync()
+
+    def close(self):
+        self.sync()
+        for buf in self.plans:
+            for pl in buf:
+                pl.close()
+        self.replay.close()
+        for g in self.rings:
+            if g is not None:
+                g.close()
+        for c in self.pctxs + self.rctxs + [self.yctx]:
+            c.close()

@@ -497,6 +497,42 @@ def test_pipeline_parity(P, ctx, name, n, nint, overlap):
         assert (h_u64(pipe.ctr) == ref["ctr"]).all()
 
 
+@pytest.mark.parametrize("name,n,nint,depth,ps,rs", [("70b", 40000, 6, 3, 2, 2), ("8b", 8000, 9, 4, 3, 2),
+                                                      ("burst", 40000, 4, 2, 1, 3), ("large", 200000, 3, 8, 4, 4),
+                                                      ("tiny", 20000, 1, 8, 4, 4)])
+def test_trace_pipeline_parity(P, ctx, name, n, nint, depth, ps, rs):
+    # several intervals in flight (plans and routes on several streams, the replay in order):
+    # every interval's plans and destinations, and the counters, equal the oracle's
+    from paper_2608_19677_gb300.pipeline import TracePipeline
+    cfg = tg.CONFIGS[name]
+    if name != "tiny":
+        cfg = cfg.scaled(n, nint)
+    tr = tg.Trace(cfg)
+    ref = OP.run_trace(tr, B=1024, keep=True)
+    ivs = [tr.interval(t) for t in range(cfg.n_intervals)]
+    keys = [d_u64(k) for k in ref["keys"]]
+    plens = [d_u32(iv.plen) for iv in ivs]
+    slens = [d_u32(iv.slen) for iv in ivs]
+    pipe = TracePipeline(ctx, cfg.R, cfg.W, cfg.caps, cfg.replicas, tr.qcap, max_n=max(iv.n for iv in ivs),
+                         batch_B=1024, depth=depth, plan_streams=ps, route_streams=rs, vnodes=cfg.vnodes)
+    for rep in range(2):   # twice: reset() restores the initial state
+        pipe.reset()
+        seen = []
+
+        def check(t, dest, plans):
+            pipe.sync()
+            seen.append(t)
+            assert (h_u16(dest) == ref["dest"][t]).all(), f"interval {t}: destinations differ"
+            for (v, s_), pl in zip(pipe.plan_keys, plans):
+                opl = ref["plans"][t][(v, s_)]
+                got = pl.export()
+                assert got["n_adm"] == opl.n_adm and (got["members"] == opl.members).all()
+        pipe.run(keys, plens, slens, [iv.g0 for iv in ivs], on_interval=check if rep == 0 else None)
+        pipe.sync()
+        assert (h_u64(pipe.ctr) == ref["ctr"]).all()
+    pipe.close()
+
+
 @pytest.mark.parametrize("B", [1, 7, 1024])
 def test_pipeline_parity_bounded_load_and_small_batches(P, ctx, B):
     # the 70B shape with the bounded-load comparison policy added, routed in
