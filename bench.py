@@ -39,7 +39,9 @@ def parse_args(argv=None):
     ap.add_argument("--steps", type=int, default=20)
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
-    ap.add_argument("--config", default="70b")
+    ap.add_argument("--config", default="large")
+    ap.add_argument("--cpu-sample", type=int, default=262144,
+                    help="keys mode: requests of interval 0 in the CPU oracle's timed sample")
     ap.add_argument("--batch", type=int, default=1024)
     ap.add_argument("--sm-split", type=int, default=0,
                     help="run hashing and candidates on all but N SMs and the load-dependent route resolution on "
@@ -67,6 +69,14 @@ def parse_args(argv=None):
     ap.add_argument("--keys-mode", action="store_true",
                     help="hash each interval's arena on its own and time plans + route + replay over resident keys "
                          "(automatic when the arenas do not fit in HBM)")
+    ap.add_argument("--per-interval", action="store_true",
+                    help="keys mode: drive one interval at a time (Pipeline) instead of keeping several intervals' "
+                         "plans and routes in flight (TracePipeline)")
+    ap.add_argument("--depth", type=int, default=8, help="keys mode: intervals in flight")
+    ap.add_argument("--plan-streams", type=int, default=4, help="keys mode: streams building plans")
+    ap.add_argument("--route-streams", type=int, default=4, help="keys mode: streams routing")
+    ap.add_argument("--replay-priority", choices=["high", "low"], default="high",
+                    help="keys mode: priority of the replay stream (plans get the other one)")
     ap.add_argument("--intervals", type=int, default=0,
                     help="profiling aid: run only the first N intervals (the JSON line says so)")
     return ap.parse_args(argv)
@@ -197,6 +207,28 @@ def hash_traffic(alg_bytes_per_launch: float):
         return None
 
 
+def lru_traffic(alg_bytes_per_launch: float, pairs_per_launch: float):
+    """DRAM bytes per LRU replay launch from the committed ncu capture (bytes per (request,
+    replica) pair there, times this launch's pairs); None when the replay source has changed
+    since the capture."""
+    import hashlib
+    path = os.path.join(ROOT, "profiles", "k_lru_stamp_traffic.txt")
+    src = os.path.join(ROOT, "paper_2608_19677_gb300", "csrc", "cr_replay.cu")
+    try:
+        kv = {}
+        for line in open(path):
+            line = line.strip()
+            if line and not line.startswith("#"):
+                k, v = line.split(None, 1)
+                kv[k] = v
+        if kv.get("source_sha256") != hashlib.sha256(open(src, "rb").read()).hexdigest():
+            return None
+        per_pair = (float(kv["dram_bytes_read"]) + float(kv["dram_bytes_write"])) / float(kv["pairs"])
+        return per_pair * pairs_per_launch
+    except Exception:
+        return None
+
+
 # ----------------------------------------------------------------- oracle ---
 def oracle_sample(trace, n_intervals: int = 1, B: int = 1024):
     """Time the CPU oracle (hash, plans, route, replay) on the first intervals of the trace."""
@@ -226,6 +258,85 @@ def oracle_sample(trace, n_intervals: int = 1, B: int = 1024):
     return reqs, busy
 
 
+def token_bytes(trace) -> float:
+    """Bytes of the token arenas of every interval of the trace."""
+    cfg = trace.cfg
+    rec_tokens = float(trace.key_plen.astype(np.float64).mean()) + cfg.suffix + 3
+    return 4.0 * rec_tokens * float(sum(trace.counts[:cfg.n_intervals]))
+
+
+def keys_mode_for(args, trace, free_bytes: float = 280e9) -> bool:
+    """Keys mode when asked, or when the arenas would not fit in (60% of) free device memory."""
+    return bool(args.keys_mode) or token_bytes(trace) > 0.6 * free_bytes
+
+
+def oracle_keys_sample(trace, S: int):
+    """Input preparation for the keys-mode oracle baseline (untimed): the first S requests of
+    interval 0 with their routing keys, hashed by the oracle from the prefix tokens (each
+    distinct key's prefix once, since requests that carry a key share its prefix)."""
+    import oracle as O
+    import tracegen as tg
+    iv = trace.interval(0)
+    S = min(S, iv.n)
+    kid = iv.key_id[:S]
+    ids = np.unique(kid)
+    keys = np.empty(S, np.uint64)
+    kv = np.empty(ids.size, np.uint64)
+    chunk = 50000
+    for a in range(0, ids.size, chunk):
+        tok, off, pl = tg.prefix_spans(trace, ids[a:a + chunk])
+        kv[a:a + chunk] = O.hash_prefixes(tok, off, pl)
+    keys[:] = kv[np.searchsorted(ids, kid)]
+    return {"keys": keys, "plen": iv.plen[:S].copy(), "slen": iv.slen[:S].copy(), "g0": iv.g0, "n": S,
+            "of": iv.n}
+
+
+def oracle_keys_step(trace, sample, threads: int, B: int) -> float:
+    """One timed pass of the CPU oracle, as it stands, over a keys-mode sample: the plans of
+    interval 0 (from its own keys), then routing and replay of every replica; independent plan
+    variants and replicas run on `threads` host threads (each oracle call is plain
+    single-threaded C and releases the interpreter lock).  Returns seconds."""
+    import concurrent.futures as cf
+    import oracle as O
+    import oracle.pipeline as OP
+    cfg = trace.cfg
+    reps = cfg.replicas
+    keys, plen, slen = sample["keys"], sample["plen"], sample["slen"]
+    rings = OP.rings_for(cfg)
+    num, den = trace.qcap(sample["n"])
+    variants = sorted({(OP.VARIANT_OF[p], s if OP.VARIANT_OF[p] == "RANDOM" else 0)
+                       for p, s in reps if p in OP.VARIANT_OF})
+    t0 = time.perf_counter()
+
+    def build(vs):
+        v, sd = vs
+        return vs, O.build_plan(keys, cfg.R, cfg.W, num, den, variant=v, seed=sd, epoch=0)
+
+    with cf.ThreadPoolExecutor(threads) as ex:
+        built = dict(ex.map(build, variants))
+
+    def one(i):
+        p, sd = reps[i]
+        v = OP.VARIANT_OF.get(p)
+        plan = built[(v, sd if v == "RANDOM" else 0)] if v is not None else None
+        d, _ = O.route([plan], [OP.ROUTE_AS.get(p, p)], [sd], cfg.R, keys, sample["g0"], B, rings=[rings[i]])
+        rp = O.Replay(1, cfg.R, cfg.caps, tokens=cfg.lru_tokens)
+        rp.step(keys, plen, slen, d)
+        return int(rp.ctr[..., 0].sum())
+
+    with cf.ThreadPoolExecutor(threads) as ex:
+        done = list(ex.map(one, range(len(reps))))
+    assert all(x == sample["n"] * len(cfg.caps) for x in done)
+    return time.perf_counter() - t0
+
+
+def keys_sample_text(cfg, sample, threads):
+    return (f"first {sample['n']} of the {sample['of']} requests of interval 0 (of {cfg.n_intervals}), all "
+            f"{len(cfg.replicas)} replicas x {len(cfg.caps)} capacities: plans from their keys + route + replay, "
+            f"keys hashed beforehand (the device step also starts from resident keys); C oracle, "
+            f"{threads} host thread(s) over independent plan variants and replicas")
+
+
 def run_reference(args):
     rank = int(os.environ.get("RANK", "0"))
     if rank != 0:
@@ -233,6 +344,8 @@ def run_reference(args):
     import tracegen as tg
     cfg = with_policies(tg.CONFIGS[args.config], args)
     trace = tg.Trace(cfg)
+    if keys_mode_for(args, trace):
+        return run_reference_keys(args, cfg, trace)
     import oracle as O
     import oracle.pipeline as OP
     iv = trace.interval(0)
@@ -263,6 +376,26 @@ def run_reference(args):
             "scaling": "weak", "vs_baseline": None, "dtype": "u64", "data": "synthetic",
             "config": workload_config(cfg, args.batch, args.fresh_plans),
             "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "kind": "oracle", "sample": sample},
+            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+def run_reference_keys(args, cfg, trace):
+    """Reference arm of a keys-mode configuration: each step is one oracle pass over the
+    bounded sample, on all host cores."""
+    threads = os.cpu_count() or 1
+    sample = oracle_keys_sample(trace, args.cpu_sample)
+    for _ in range(args.warmup):
+        oracle_keys_step(trace, sample, threads, args.batch)
+    each = [oracle_keys_step(trace, sample, threads, args.batch) for _ in range(args.steps)]
+    dt = float(np.mean(each)) if each else 0.0
+    value = sample["n"] / dt if dt > 0 else 0.0
+    cb = {"value": value, "unit": UNIT, "cores": threads, "kind": "oracle",
+          "sample": keys_sample_text(cfg, sample, threads)}
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": dt * 1e3, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "u64", "data": "synthetic",
+            "config": workload_config(cfg, args.batch, args.fresh_plans), "cpu_baseline": cb,
             "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     print(json.dumps(line), flush=True)
 
@@ -355,10 +488,8 @@ def main():
     # large configuration holds ~600 GB of tokens), every interval's arena is
     # generated and hashed one at a time (each hash launch timed on its own),
     # and the timed steps run plans + route + replay over the resident keys.
-    rec_tokens = float(trace.key_plen.astype(np.float64).mean()) + cfg.suffix + 3
-    tok_bytes = 4.0 * rec_tokens * float(sum(trace.counts[:cfg.n_intervals]))
     free, _total = torch.cuda.mem_get_info(dev)
-    if args.keys_mode or tok_bytes > 0.6 * free:
+    if keys_mode_for(args, trace, float(free)):
         return run_keys_mode(args, cfg, trace, dev, stream, world, rank, barrier, resolve_stream, part)
 
     # inputs resident in HBM (generated on the device, untimed)
@@ -600,7 +731,7 @@ def run_keys_mode(args, cfg, trace, dev, stream, world, rank, barrier, resolve_s
     import torch.distributed as dist
     import paper_2608_19677_gb300 as P
     import tracegen as tg
-    from paper_2608_19677_gb300.pipeline import Pipeline
+    from paper_2608_19677_gb300.pipeline import Pipeline, TracePipeline
 
     ctx = P.Context(dev.index if dev.index is not None else 0, stream)
     keys, plens, slens, g0s, ns = [], [], [], [], []
@@ -627,9 +758,16 @@ def run_keys_mode(args, cfg, trace, dev, stream, world, rank, barrier, resolve_s
     torch.cuda.synchronize()
     torch.cuda.empty_cache()  # the arenas are gone: only keys and lengths stay on the device
     n_step = sum(ns)
-    pipe = Pipeline(ctx, cfg.R, cfg.W, cfg.caps, cfg.replicas, trace.qcap, batch_B=args.batch, max_n=max(ns),
-                    overlap=not args.no_overlap, vnodes=cfg.vnodes, fresh=args.fresh_plans,
-                    lru_tokens=cfg.lru_tokens, resolve_stream=resolve_stream)
+    trace_mode = not args.per_interval and resolve_stream is None
+    if trace_mode:
+        pipe = TracePipeline(ctx, cfg.R, cfg.W, cfg.caps, cfg.replicas, trace.qcap, max_n=max(ns),
+                             batch_B=args.batch, depth=args.depth, plan_streams=args.plan_streams,
+                             route_streams=args.route_streams, vnodes=cfg.vnodes, fresh=args.fresh_plans,
+                             lru_tokens=cfg.lru_tokens, replay_first=args.replay_priority == "high")
+    else:
+        pipe = Pipeline(ctx, cfg.R, cfg.W, cfg.caps, cfg.replicas, trace.qcap, batch_B=args.batch, max_n=max(ns),
+                        overlap=not args.no_overlap, vnodes=cfg.vnodes, fresh=args.fresh_plans,
+                        lru_tokens=cfg.lru_tokens, resolve_stream=resolve_stream)
     marks = [[[torch.cuda.Event(enable_timing=True) for _ in range(5)] for _ in range(cfg.n_intervals)]
              for _ in range(max(args.steps, 1))]
     plan_marks = [[] for _ in range(max(args.steps, 1))]
@@ -638,10 +776,14 @@ def run_keys_mode(args, cfg, trace, dev, stream, world, rank, barrier, resolve_s
 
     def step(k=None):
         pipe.reset()
-        for t in range(cfg.n_intervals):
-            pipe.interval(t, None, None, plens[t], slens[t], g0s[t], marks=marks[k][t] if k is not None else None,
-                          plan_next=t + 1 < cfg.n_intervals, keys=keys[t])
-        pipe.finish()
+        if trace_mode:
+            pipe.run(keys, plens, slens, g0s, mark=k is not None)
+        else:
+            for t in range(cfg.n_intervals):
+                pipe.interval(t, None, None, plens[t], slens[t], g0s[t],
+                              marks=marks[k][t] if k is not None else None,
+                              plan_next=t + 1 < cfg.n_intervals, keys=keys[t])
+            pipe.finish()
         if k is not None:
             plan_marks[k] = list(pipe.plan_marks)
             route_marks[k] = list(pipe.route_marks)
@@ -660,6 +802,11 @@ def run_keys_mode(args, cfg, trace, dev, stream, world, rank, barrier, resolve_s
         graph_launches = pipe.launches - lc0
         graph.replay()
         torch.cuda.synchronize()
+    # per-launch CUDA events around the library's main kernels, on the streams they run on
+    # (graphs: from one ordinary step after the timed region)
+    prof_ctxs = pipe.contexts
+    for c in prof_ctxs:
+        c.profile_enable(0 if graph is not None else 16 * cfg.n_intervals * max(args.steps, 1) + 64)
     clocks = ClockSampler(dev.index or 0, args.clocks_out)
     clocks.start()
     time.sleep(0.3)
@@ -681,19 +828,31 @@ def run_keys_mode(args, cfg, trace, dev, stream, world, rank, barrier, resolve_s
     clk = clocks.stop()
     if graph is not None:  # stage and plan times from one ordinary step after the timed region
         pipe.quiesce()
+        for c in prof_ctxs:
+            c.profile_enable(16 * cfg.n_intervals + 64)
         step(0)
     pipe.sync()
+    kern = {}
+    for tag in ("plan", "route_cand", "route_resolve", "partition", "replay"):
+        n_, ms_ = 0, 0.0
+        for c in prof_ctxs:
+            a, b = c.profile_read(tag)
+            n_, ms_ = n_ + a, ms_ + b
+        kern[tag] = {"launches": n_, "avg_ms": ms_ / n_ if n_ else None}
+    for c in prof_ctxs:
+        c.profile_enable(0)
     ms = ev0.elapsed_time(ev1) / args.steps
     ms_max = max_over_ranks(ms, world, dev)
     marked = [0] if graph is not None else list(range(args.steps))
     plan_marks = [plan_marks[k] for k in marked]
     route_marks, replay_marks = [route_marks[k] for k in marked], [replay_marks[k] for k in marked]
     stage = np.zeros((len(marked), cfg.n_intervals, 4))
-    for j, k in enumerate(marked):
-        for t in range(cfg.n_intervals):
-            m = marks[k][t]
-            for s_ in range(4):
-                stage[j, t, s_] = m[s_].elapsed_time(m[s_ + 1])
+    if not trace_mode:
+        for j, k in enumerate(marked):
+            for t in range(cfg.n_intervals):
+                m = marks[k][t]
+                for s_ in range(4):
+                    stage[j, t, s_] = m[s_].elapsed_time(m[s_ + 1])
     plan_ms = np.array([[a.elapsed_time(b) for a, b in pm] for pm in plan_marks])
     # route and replay calls timed on their own streams, after their waits
     route_ms = float(np.array([[a.elapsed_time(b) for a, b in rm] for rm in route_marks]).sum(1).mean())
@@ -716,6 +875,11 @@ def run_keys_mode(args, cfg, trace, dev, stream, world, rank, barrier, resolve_s
     # route + replay's (plans overlap them on their own stream)
     rr_rps = n_step / (ms_max / 1e3)
     rr_gbs = rr_bytes * rr_rps / 1e9
+    # the dominant kernel of the step: the LRU simulation (a9), one launch per interval; its
+    # algorithmic bytes per launch are SURVEY 8(d)'s 20 per (request, replica, capacity)
+    a9_bytes = 20.0 * reps * ncaps * n_step / cfg.n_intervals
+    lru_ms = kern["replay"]["avg_ms"]
+    lru_gbs = a9_bytes / (lru_ms / 1e3) / 1e9 if lru_ms else None
     line = {
         "metric": METRIC, "value": job_throughput(n_step, world, ms_max), "unit": UNIT, "n_gpus": world,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_max, "higher_is_better": True,
@@ -724,11 +888,24 @@ def run_keys_mode(args, cfg, trace, dev, stream, world, rank, barrier, resolve_s
                        step="plans + route + replay over resident keys (the token arenas of all intervals do "
                             "not fit in HBM: each interval's arena was generated and hashed one at a time, each "
                             "hash launch timed alone)",
+                       schedule=(f"{args.depth} intervals in flight: plans on {args.plan_streams} streams, routes "
+                                 f"on {args.route_streams} streams, the replay in interval order on one stream"
+                                 if trace_mode else "one interval at a time (plans of the next interval overlap)"),
                        l2="inputs larger than L2 (keys, prefix and suffix lengths of all intervals resident)"),
-        "roofline": {"kernel": "k_hash_prefixes", "bound": "hbm", "achieved": hash_gbs, "peak": hbm_peak,
-                     "peak_source": "measured" if "hbm_gbs" in peaks else "fallback", "unit": "GB/s",
-                     "frac": hash_gbs / hbm_peak, "traffic": hash_traffic(float(hb.mean())),
-                     "algorithmic_bytes_per_launch_mean": float(hb.mean()), "avg_launch_ms": float(hms.mean())},
+        "roofline": {"kernel": "k_lru_stamp (a9 LRU replay)", "bound": "hbm", "achieved": lru_gbs,
+                     "peak": hbm_peak, "peak_source": "measured" if "hbm_gbs" in peaks else "fallback",
+                     "unit": "GB/s", "frac": lru_gbs / hbm_peak if lru_gbs else None,
+                     "traffic": lru_traffic(a9_bytes, reps * n_step / cfg.n_intervals),
+                     "algorithmic_bytes_per_launch_mean": a9_bytes, "avg_launch_ms": lru_ms,
+                     "launches_timed": kern["replay"]["launches"],
+                     "note": "20 B per (request, replica, capacity) as SURVEY 8(d) counts a9; the kernel reads "
+                             "one 16 B record per (request, replica) and decides every capacity from it; the "
+                             "kernel is bound by the latency of its per-step dependence chain, not by bytes"},
+        "hash_roofline": {"kernel": "k_hash_prefixes", "bound": "hbm", "achieved": hash_gbs, "peak": hbm_peak,
+                          "unit": "GB/s", "frac": hash_gbs / hbm_peak, "traffic": hash_traffic(float(hb.mean())),
+                          "algorithmic_bytes_per_launch_mean": float(hb.mean()), "avg_launch_ms": float(hms.mean()),
+                          "note": "keys mode: each interval's hash timed alone before the timed step"},
+        "kernels_ms_per_launch": kern,
         "route_replay": {"requests_per_s": rr_rps, "route_call_ms_per_step": route_ms,
                          "replay_call_ms_per_step": replay_ms,
                          "note": "route and replay run overlapped on two streams; call times are under contention",
@@ -742,11 +919,80 @@ def run_keys_mode(args, cfg, trace, dev, stream, world, rank, barrier, resolve_s
     if graph is not None:
         line["cuda_graph"] = ("the timed steps replay one CUDA graph of the whole step; stage, route, replay "
                               "and plan-build times come from one ordinary step after the timed region")
+    # ---- end to end through the public API with pinned host buffers -------
+    if not args.no_e2e and trace_mode:
+        line["e2e"] = e2e_keys(args, pipe, keys, plens, slens, g0s, dev, stream, n_step, world)
+    # ---- CPU baseline (rank 0, N = 1): the oracle on a bounded sample -------
+    if not args.no_cpu_baseline and world == 1:
+        sample = oracle_keys_sample(trace, args.cpu_sample)
+        nproc = os.cpu_count() or 1
+        t1 = oracle_keys_step(trace, sample, 1, args.batch)
+        tn = oracle_keys_step(trace, sample, nproc, args.batch)
+        line["cpu_baseline"] = {"value": sample["n"] / tn, "unit": UNIT, "cores": nproc, "kind": "oracle",
+                                "sample": keys_sample_text(cfg, sample, nproc),
+                                "single_thread": {"value": sample["n"] / t1, "unit": UNIT, "cores": 1},
+                                "nproc": nproc}
     if rank == 0:
         print(json.dumps(line), flush=True)
     close_in_order(pipe, ctx, part)
     if world > 1:
         dist.destroy_process_group()
+
+
+def e2e_keys(args, pipe, keys, plens, slens, g0s, dev, stream, n_step, world):
+    """Keys mode end to end through the public API: every step copies each interval's keys,
+    prefix and suffix lengths from pinned host memory (a copy stream, one event per
+    interval, so routing of interval t starts once its inputs have landed), runs the whole
+    trace and reads the counters back."""
+    import torch
+    host = []
+    for k, pl, sl in zip(keys, plens, slens):
+        h = []
+        for x in (k, pl, sl):
+            p = torch.empty(x.shape, dtype=x.dtype, pin_memory=True)
+            p.copy_(x)
+            h.append(p)
+        host.append(h)
+    h2d = sum(x.numel() * x.element_size() for h in host for x in h)
+    dbuf = [[torch.empty_like(x, device=dev) for x in h] for h in host]
+    copy_stream = torch.cuda.Stream(dev)
+    out = torch.empty(pipe.ctr.shape, dtype=torch.int64, pin_memory=True)
+    d2h = out.numel() * out.element_size()
+
+    def step():
+        pipe.reset()
+        start = torch.cuda.Event()
+        start.record(stream)
+        copy_stream.wait_event(start)  # the previous step's readers are done with the buffers
+        ready = []
+        with torch.cuda.stream(copy_stream):
+            for h, d in zip(host, dbuf):
+                for a, b in zip(h, d):
+                    b.copy_(a, non_blocking=True)
+                e = torch.cuda.Event()
+                e.record(copy_stream)
+                ready.append(e)
+        pipe.run([d[0] for d in dbuf], [d[1] for d in dbuf], [d[2] for d in dbuf], g0s, ready=ready)
+        out.copy_(pipe.ctr, non_blocking=True)
+
+    for _ in range(2):
+        step()
+    torch.cuda.synchronize()
+    each = []
+    for _ in range(args.e2e_steps):
+        e0 = torch.cuda.Event(enable_timing=True)
+        e1 = torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        step()
+        e1.record(stream)  # after the counters' read-back on this stream
+        e1.synchronize()
+        each.append(e0.elapsed_time(e1))
+    ms = max_over_ranks(float(np.median(each)), world, dev)
+    return {"value": job_throughput(n_step, world, ms), "unit": UNIT, "h2d_bytes_per_step": h2d,
+            "d2h_bytes_per_step": d2h, "ms_per_step": ms, "ms_per_step_each": [round(x, 2) for x in each],
+            "note": "keys, prefix and suffix lengths of every interval copied from pinned host memory on a copy "
+                    "stream each step (routing of an interval waits for its copy), counters read back; median "
+                    "of the timed steps"}
 
 
 def e2e(args, ctx, pipe, inputs, dev, stream, n_step, world):

@@ -143,6 +143,31 @@ CR_API const char *cr_last_error(const cr_ctx *ctx);
 /* Number of kernel launches this context has issued since it was created. */
 CR_API uint64_t cr_launch_count(const cr_ctx *ctx);
 
+/* ---- per-launch timing (tracing aid; no counterpart in the paper) --------
+ * With profiling enabled, the calls below bracket their main kernels with
+ * CUDA timing events on the stream the kernels run on, one pair per launch:
+ *   CR_PROF_HASH           k_hash_prefixes (cr_hash_prefixes)
+ *   CR_PROF_PLAN           the whole plan build (cr_build_plans)
+ *   CR_PROF_ROUTE_CAND     the load-independent pass of cr_route_batch
+ *   CR_PROF_ROUTE_RESOLVE  its load-dependent pass (on the resolve stream if split)
+ *   CR_PROF_PARTITION      the per-destination partition of cr_shadow_replay
+ *   CR_PROF_REPLAY         its LRU simulation kernel
+ * Every call also opens an NVTX range named after it (visible to profilers).
+ * cr_profile_enable(ctx, n) keeps room for n launches (0 turns timing off) and
+ * forgets earlier ones; launches beyond n are not timed.  cr_profile_read is
+ * blocking: it waits for the recorded events and returns the number of timed
+ * launches with `tag` and their summed duration in milliseconds.  Errors:
+ * CR_EINVAL (tag out of range), CR_ENOMEM, CR_ECUDA. */
+#define CR_PROF_HASH 0
+#define CR_PROF_PLAN 1
+#define CR_PROF_ROUTE_CAND 2
+#define CR_PROF_ROUTE_RESOLVE 3
+#define CR_PROF_PARTITION 4
+#define CR_PROF_REPLAY 5
+#define CR_PROF_TAGS 6
+CR_API int cr_profile_enable(cr_ctx *ctx, uint32_t max_launches);
+CR_API int cr_profile_read(cr_ctx *ctx, uint32_t tag, uint64_t *launches, double *total_ms);
+
 /* ==== a1: prefix-span routing key ==================================== */
 /*
  * The paper routes on an opaque business key b, which it allows to be salted

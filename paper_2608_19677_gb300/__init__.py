@@ -38,7 +38,9 @@ EXPORTS = ("cr_create", "cr_destroy", "cr_set_stream", "cr_sync", "cr_last_error
            "cr_plan_get_info", "cr_plan_export", "cr_route_batch", "cr_replay_create", "cr_replay_reset",
            "cr_replay_destroy", "cr_shadow_replay", "cr_replay_export_state", "cr_key_histogram_noalloc",
            "cr_ring_create", "cr_ring_destroy", "cr_ring_export", "cr_plan_diff",
-           "cr_replay_create_tokens", "cr_set_resolve_stream", "cr_partition_create", "cr_partition_destroy")
+           "cr_replay_create_tokens", "cr_set_resolve_stream", "cr_partition_create", "cr_partition_destroy",
+           "cr_profile_enable", "cr_profile_read")
+PROF = {"hash": 0, "plan": 1, "route_cand": 2, "route_resolve": 3, "partition": 4, "replay": 5}
 CR_NOALLOC_MAX_KEYS = 65536
 
 
@@ -117,6 +119,8 @@ def lib() -> C.CDLL:
         "cr_set_resolve_stream": ([vp, vp], i32),
         "cr_partition_create": ([i32, u32, C.POINTER(vp), C.POINTER(vp), C.POINTER(vp)], i32),
         "cr_partition_destroy": ([vp], i32),
+        "cr_profile_enable": ([vp, u32], i32),
+        "cr_profile_read": ([vp, u32, C.POINTER(C.c_uint64), C.POINTER(C.c_double)], i32),
     }
     for name, (args, res) in sig.items():
         f = getattr(L, name)
@@ -165,6 +169,16 @@ class Context:
     @property
     def launches(self) -> int:
         return int(lib().cr_launch_count(self._h))
+
+    def profile_enable(self, max_launches: int):
+        """Time the library's main kernels per launch with CUDA events (0: off); forgets earlier launches."""
+        self.check(lib().cr_profile_enable(self._h, max_launches), "cr_profile_enable")
+
+    def profile_read(self, tag: str):
+        """(timed launches, summed milliseconds) of one kind of launch (blocking)."""
+        n, ms = C.c_uint64(), C.c_double()
+        self.check(lib().cr_profile_read(self._h, PROF[tag], C.byref(n), C.byref(ms)), "cr_profile_read")
+        return int(n.value), float(ms.value)
 
     def close(self):
         if getattr(self, "_h", None):

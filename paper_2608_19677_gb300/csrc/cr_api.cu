@@ -82,10 +82,72 @@ extern "C" int cr_create(cr_ctx **out, int device, void *cuda_stream)
     return CR_OK;
 }
 
+static void prof_free(cr_ctx *ctx)
+{
+    cr_prof &P = ctx->prof;
+    if (P.ev) {
+        for (uint32_t i = 0; i < 2 * P.cap; ++i)
+            if (P.ev[i]) cudaEventDestroy(P.ev[i]);
+        free(P.ev);
+    }
+    free(P.tag);
+    memset(&P, 0, sizeof(P));
+}
+
+extern "C" int cr_profile_enable(cr_ctx *ctx, uint32_t max_launches)
+{
+    if (!ctx) return CR_EINVAL;
+    CR_CUDA(ctx, cudaStreamSynchronize(ctx->stream));
+    if (ctx->resolve_stream) CR_CUDA(ctx, cudaStreamSynchronize(ctx->resolve_stream));
+    if (max_launches == ctx->prof.cap && ctx->prof.ev) {  // same size: keep the events, forget the launches
+        ctx->prof.used = 0;
+        return CR_OK;
+    }
+    prof_free(ctx);
+    if (max_launches == 0) return CR_OK;
+    cr_prof &P = ctx->prof;
+    P.ev = (cudaEvent_t *)calloc(2 * (size_t)max_launches, sizeof(cudaEvent_t));
+    P.tag = (uint8_t *)calloc(max_launches, 1);
+    if (!P.ev || !P.tag) {
+        prof_free(ctx);
+        return cr_fail(ctx, CR_ENOMEM, "cr_profile_enable: host allocation failed");
+    }
+    P.cap = max_launches;
+    for (uint32_t i = 0; i < 2 * max_launches; ++i) {
+        if (cudaEventCreate(&P.ev[i]) != cudaSuccess) {
+            cudaGetLastError();
+            prof_free(ctx);
+            return cr_fail(ctx, CR_ECUDA, "cr_profile_enable: cannot create events");
+        }
+    }
+    return CR_OK;
+}
+
+extern "C" int cr_profile_read(cr_ctx *ctx, uint32_t tag, uint64_t *launches, double *total_ms)
+{
+    if (!ctx || !launches || !total_ms) return CR_EINVAL;
+    if (tag >= CR_PROF_TAGS) return cr_fail(ctx, CR_EINVAL, "cr_profile_read: tag %u", tag);
+    uint64_t n = 0;
+    double ms = 0.0;
+    const cr_prof &P = ctx->prof;
+    for (uint32_t i = 0; i < P.used; ++i) {
+        if (P.tag[i] != tag) continue;
+        CR_CUDA(ctx, cudaEventSynchronize(P.ev[2 * i + 1]));
+        float x = 0.f;
+        CR_CUDA(ctx, cudaEventElapsedTime(&x, P.ev[2 * i], P.ev[2 * i + 1]));
+        ms += x;
+        ++n;
+    }
+    *launches = n;
+    *total_ms = ms;
+    return CR_OK;
+}
+
 extern "C" int cr_destroy(cr_ctx *ctx)
 {
     if (!ctx) return CR_OK;
     cudaStreamSynchronize(ctx->stream);
+    prof_free(ctx);
     if (ctx->resolve_stream) cudaStreamSynchronize(ctx->resolve_stream);
     if (ctx->ev_cand) cudaEventDestroy(ctx->ev_cand);
     if (ctx->ev_resolve) cudaEventDestroy(ctx->ev_resolve);

@@ -131,6 +131,7 @@ k_hash_prefixes(const int32_t *__restrict__ tok, const unsigned long long *__res
 extern "C" int cr_hash_prefixes(cr_ctx *ctx, const int32_t *d_tokens, const uint64_t *d_off,
                                 const uint32_t *d_plen, uint64_t n, uint64_t salt, uint64_t *d_key_out)
 {
+    cr_nvtx_range nv("cr_hash_prefixes");
     if (!ctx) return CR_EINVAL;
     if (n == 0) return CR_OK;
     if (!d_tokens || !d_off || !d_plen || !d_key_out)
@@ -139,7 +140,9 @@ extern "C" int cr_hash_prefixes(cr_ctx *ctx, const int32_t *d_tokens, const uint
     // many more blocks than fit at once (32 per SM): blocks start as others
     // finish, which evens out the widely varying span lengths across the SMs
     unsigned int grid = cr_blocks(n, warps_per_block, (unsigned int)ctx->num_sms * 32u);
+    const int pi = cr_prof_begin(ctx, ctx->stream, CR_PROF_HASH);
     CR_LAUNCH(ctx, k_hash_prefixes, grid, kHashBlock, 0, d_tokens, (const unsigned long long *)d_off,
               d_plen, (unsigned long long)n, (unsigned long long)salt, (unsigned long long *)d_key_out);
+    cr_prof_end(ctx, ctx->stream, pi);
     return CR_OK;
 }

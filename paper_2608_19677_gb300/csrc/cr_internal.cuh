@@ -6,7 +6,15 @@
 #include <stdint.h>
 #include <stdio.h>
 
+#include <nvtx3/nvToolsExt.h>
+
 #include "cacheroute.h"
+
+// NVTX range over one C ABI call (free unless a profiler is attached).
+struct cr_nvtx_range {
+    explicit cr_nvtx_range(const char *name) { nvtxRangePushA(name); }
+    ~cr_nvtx_range() { nvtxRangePop(); }
+};
 
 // ---- device error flags (a bitmask in device memory, read by cr_sync) ------
 #define CR_FLAG_OVERFLOW 1u  // a load reached 2^47, or a stamp counter overflowed
@@ -35,7 +43,15 @@ enum cr_scratch_slot {
     SCR_NUM
 };
 
+// ---- per-launch timing of selected kernels (cr_profile_enable) ---------------
+struct cr_prof {
+    uint32_t cap, used;  // event pairs available / recorded
+    cudaEvent_t *ev;     // [2 cap]: start, end of each timed launch
+    uint8_t *tag;        // [cap]: CR_PROF_* of each
+};
+
 struct cr_ctx {
+    cr_prof prof;
     int device;
     int num_sms;
     cudaStream_t stream;
@@ -139,6 +155,22 @@ int cr_check_launch(cr_ctx *ctx, const char *what);
         (ctx)->launches++;                                                 \
         CR_TRY(cr_check_launch((ctx), #kern));                             \
     } while (0)
+
+// Bracket work enqueued on `st` with a timed event pair when profiling is on;
+// returns the pair's index (or -1) for cr_prof_end.
+static inline int cr_prof_begin(cr_ctx *ctx, cudaStream_t st, int tag)
+{
+    cr_prof &P = ctx->prof;
+    if (!P.ev || P.used >= P.cap) return -1;
+    const uint32_t i = P.used++;
+    P.tag[i] = (uint8_t)tag;
+    cudaEventRecord(P.ev[2 * i], st);
+    return (int)i;
+}
+static inline void cr_prof_end(cr_ctx *ctx, cudaStream_t st, int i)
+{
+    if (i >= 0) cudaEventRecord(ctx->prof.ev[2 * i + 1], st);
+}
 
 static inline unsigned int cr_blocks(uint64_t work, unsigned int per_block, unsigned int cap)
 {

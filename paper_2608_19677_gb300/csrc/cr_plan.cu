@@ -1465,8 +1465,22 @@ static int check_params(cr_ctx *ctx, const cr_plan_params *pp)
     return CR_OK;
 }
 
+static int build_plans(cr_ctx *ctx, const uint64_t *d_key, uint64_t n, const cr_plan_params *params,
+                       uint32_t n_plans, cr_plan *const *plans);
+
 extern "C" int cr_build_plans(cr_ctx *ctx, const uint64_t *d_key, uint64_t n, const cr_plan_params *params,
                               uint32_t n_plans, cr_plan *const *plans)
+{
+    if (!ctx) return CR_EINVAL;
+    cr_nvtx_range nv("cr_build_plans");
+    const int pi = cr_prof_begin(ctx, ctx->stream, CR_PROF_PLAN);
+    const int st = build_plans(ctx, d_key, n, params, n_plans, plans);
+    cr_prof_end(ctx, ctx->stream, pi);
+    return st;
+}
+
+static int build_plans(cr_ctx *ctx, const uint64_t *d_key, uint64_t n, const cr_plan_params *params,
+                       uint32_t n_plans, cr_plan *const *plans)
 {
     if (!ctx) return CR_EINVAL;
     if (!params || !plans || n_plans == 0) return cr_fail(ctx, CR_EINVAL, "cr_build_plans: no plans");

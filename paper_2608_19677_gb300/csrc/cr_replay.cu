@@ -185,101 +185,177 @@ struct replay_state {
 // would exceed cmax, the oldest untouched keys (the lowest live bits) leave
 // and the new keys take their slots.
 constexpr uint32_t kNone = 0xffffffffu;
-constexpr uint16_t kTomb = 0xffffu;    // index entry whose key was evicted
 constexpr uint32_t kAbsent = 2047u;    // depth code of a key not resident (above every position < 1024)
 
+constexpr uint32_t kStash = 32;              // index entries that found both buckets full
+constexpr uint32_t kDegraded = 0x80000000u;  // stash overflowed: lookups scan the keys
+
 struct stamp_lru {
-    unsigned long long *K;  // [cmax] key of each slot
-    uint32_t *BM;           // [nw] live-stamp bits, word w = times 32 w .. 32 w + 31
-    uint16_t *tab;          // [tsz] slot + 1; 0 = empty, kTomb = evicted
-    uint16_t *ST;           // [cmax] stamp of each slot
-    uint16_t *T2S;          // [32 nw] slot whose stamp is each time (where the bit is set)
-    uint16_t *EV;           // [32] slots the step's evictions freed
-    uint32_t mask;
-    int tbits;
+    unsigned long long *K;    // [cmax] key of each slot
+    uint32_t *BM;             // [nw] live-stamp bits, word w = times 32 w .. 32 w + 31
+    uint32_t *stash_n;        // stash entries claimed (| kDegraded once it overflowed)
+    unsigned long long *bkt;  // [2^nbb] index buckets of four 16-bit entries (0 = empty)
+    uint16_t *ST;             // [cmax] stamp of each slot
+    uint16_t *T2S;            // [32 nw] slot whose stamp is each time (where the bit is set)
+    uint16_t *EV;             // [32] slots the step's evictions freed
+    uint16_t *stash;          // [kStash] slot + 1 of keys indexed outside their buckets (0 = free)
+    uint32_t nbb;             // log2 of the bucket count
 };
 
-// Per-warp layout: K at 0 (8-byte entries), BM after it, the index at the next
-// 16-byte boundary (it is cleared with 16-byte stores), then ST, T2S and EV.
-__host__ __device__ inline size_t stamp_tab_offset(uint32_t cmax, uint32_t nw)
+// Per-warp layout: K at 0 (8-byte entries), BM and the stash count after it, the
+// buckets at the next 16-byte boundary (cleared with 16-byte stores), then ST,
+// T2S, EV and the stash.
+__host__ __device__ inline size_t stamp_bkt_offset(uint32_t cmax, uint32_t nw)
 {
-    return ((size_t)cmax * 8 + (size_t)nw * 4 + 15) & ~(size_t)15;
+    return ((size_t)cmax * 8 + (size_t)(nw + 1) * 4 + 15) & ~(size_t)15;
 }
 
-__host__ __device__ inline size_t stamp_lru_bytes(uint32_t cmax, uint32_t nw, uint32_t tsz)
+__host__ __device__ inline size_t stamp_lru_bytes(uint32_t cmax, uint32_t nw, uint32_t nbb)
 {
-    return (stamp_tab_offset(cmax, nw) + (size_t)tsz * 2 + (size_t)cmax * 2 + (size_t)nw * 64 + 64 + 15) &
+    return (stamp_bkt_offset(cmax, nw) + ((size_t)8 << nbb) + (size_t)cmax * 2 + (size_t)nw * 64 + 64 +
+            (size_t)kStash * 2 + 15) &
            ~(size_t)15;
 }
 
-__device__ __forceinline__ stamp_lru stamp_lru_at(unsigned char *base, uint32_t cmax, uint32_t nw, int tbits)
+__device__ __forceinline__ stamp_lru stamp_lru_at(unsigned char *base, uint32_t cmax, uint32_t nw, uint32_t nbb)
 {
-    const uint32_t tsz = 1u << tbits;
     stamp_lru X;
     X.K = reinterpret_cast<unsigned long long *>(base);
     X.BM = reinterpret_cast<uint32_t *>(base + (size_t)cmax * 8);
-    X.tab = reinterpret_cast<uint16_t *>(base + stamp_tab_offset(cmax, nw));
-    X.ST = X.tab + tsz;
+    X.stash_n = X.BM + nw;
+    X.bkt = reinterpret_cast<unsigned long long *>(base + stamp_bkt_offset(cmax, nw));
+    X.ST = reinterpret_cast<uint16_t *>(X.bkt + (1u << nbb));
     X.T2S = X.ST + cmax;
     X.EV = X.T2S + (size_t)nw * 32;
-    X.mask = tsz - 1;
-    X.tbits = tbits;
+    X.stash = X.EV + 32;
+    X.nbb = nbb;
     return X;
 }
 
-__device__ __forceinline__ uint32_t lru_home(unsigned long long key, int tbits) { return (uint32_t)(key >> (64 - tbits)); }
+// Index: two candidate buckets of four 16-bit entries per key, each entry
+// (5-bit tag << 11) | (slot + 1).  A key goes into the emptier of its buckets
+// (the first when equal); a key whose buckets are both full goes to a small
+// stash (with at most a quarter of the entries live that is rare); if even the
+// stash is full the index is marked degraded and lookups scan every key.
+// Entries never move, so concurrent lanes only need compare-and-swap on the
+// 64-bit bucket words, and a deleted entry becomes empty (no tombstones).
+struct bkt_hash {
+    uint32_t b1, b2, tag;
+};
 
-// Slot of `key`, or kNone.  The index always has empty entries (at most three
-// quarters are live or evicted when a step starts), so the probe ends at one;
-// the bound only guards against a corrupted index.
-__device__ __forceinline__ uint32_t sl_lookup(const stamp_lru &X, unsigned long long key)
+__device__ __forceinline__ bkt_hash sl_hash(unsigned long long key, uint32_t nbb)
 {
-    uint32_t s = lru_home(key, X.tbits);
-    for (uint32_t it = 0; it <= X.mask; ++it) {
-        const uint32_t e = X.tab[s];
-        if (e == 0) return kNone;
-        if (e != kTomb && X.K[e - 1] == key) return e - 1;
-        s = (s + 1) & X.mask;
+    const unsigned long long h = key * 0x9e3779b97f4a7c15ull;  // an odd multiplier spreads every key bit upwards
+    bkt_hash r;
+    r.b1 = (uint32_t)(h >> (64 - nbb));
+    r.b2 = (uint32_t)(h >> (64 - 2 * nbb)) & ((1u << nbb) - 1u);
+    r.tag = (uint32_t)(h >> (59 - 2 * nbb)) & 31u;
+    return r;
+}
+
+__device__ __forceinline__ uint32_t bkt_entry(unsigned long long w, int p) { return (uint32_t)(w >> (16 * p)) & 0xffffu; }
+
+// Slot of `key`, or kNone (fill: resident keys, scanned only when the index is degraded).
+__device__ __forceinline__ uint32_t sl_lookup(const stamp_lru &X, unsigned long long key, uint32_t fill, uint32_t cmax)
+{
+    const bkt_hash H = sl_hash(key, X.nbb);
+    const unsigned long long w1 = X.bkt[H.b1], w2 = X.bkt[H.b2];
+#pragma unroll
+    for (int p = 0; p < 8; ++p) {
+        const uint32_t e = bkt_entry(p < 4 ? w1 : w2, p & 3);
+        if (e != 0 && (e >> 11) == H.tag) {
+            const uint32_t q = (e & 0x7ffu) - 1u;
+            if (q < cmax && X.K[q] == key) return q;
+        }
+    }
+    const uint32_t sn = *X.stash_n;
+    if (sn) {
+        if (sn & kDegraded) {
+            for (uint32_t q = 0; q < fill; ++q)
+                if (X.K[q] == key) return q;
+            return kNone;
+        }
+        for (uint32_t i = 0; i < sn && i < kStash; ++i) {
+            const uint32_t e = X.stash[i];
+            if (e != 0 && e <= cmax && X.K[e - 1] == key) return e - 1;
+        }
     }
     return kNone;
 }
 
-// Index an absent key held in slot q; returns 1 when it took an evicted entry's
-// place.  A lost compare-and-swap means another lane filled the entry, so the
-// next look moves on; the bound only guards against a corrupted index.
-__device__ __forceinline__ uint32_t sl_insert(const stamp_lru &X, unsigned long long key, uint32_t q)
+// Index an absent key held in slot q.  A lost compare-and-swap means another lane
+// changed the bucket, so the next look sees it; the bound only guards the loop.
+__device__ __forceinline__ void sl_insert(const stamp_lru &X, unsigned long long key, uint32_t q)
 {
-    unsigned short *t = reinterpret_cast<unsigned short *>(X.tab);
-    uint32_t s = lru_home(key, X.tbits);
-    for (uint32_t it = 0; it <= 2 * X.mask + 1; ++it) {
-        const unsigned short v = t[s];
-        if (v == 0 || v == kTomb) {
-            if (atomicCAS(&t[s], v, (unsigned short)(q + 1)) == v) return v == kTomb ? 1u : 0u;
-            continue;  // another lane took it: look at it again
+    const bkt_hash H = sl_hash(key, X.nbb);
+    const unsigned long long ent = (unsigned long long)((H.tag << 11) | (q + 1u));
+    for (int it = 0; it < 64; ++it) {
+        const unsigned long long w1 = X.bkt[H.b1], w2 = X.bkt[H.b2];
+        int f1 = -1, f2 = -1, n1 = 0, n2 = 0;
+#pragma unroll
+        for (int p = 3; p >= 0; --p) {
+            if (bkt_entry(w1, p) == 0) {
+                f1 = p;
+                ++n1;
+            }
+            if (bkt_entry(w2, p) == 0) {
+                f2 = p;
+                ++n2;
+            }
         }
-        s = (s + 1) & X.mask;
+        uint32_t b;
+        unsigned long long w;
+        int p;
+        if (f1 >= 0 && (n1 >= n2 || f2 < 0)) {
+            b = H.b1;
+            w = w1;
+            p = f1;
+        } else if (f2 >= 0) {
+            b = H.b2;
+            w = w2;
+            p = f2;
+        } else {
+            break;  // both buckets full
+        }
+        if (atomicCAS(&X.bkt[b], w, w | (ent << (16 * p))) == w) return;
     }
-    return 0;
+    const uint32_t i = atomicAdd(X.stash_n, 1u);
+    if (i < kStash)
+        X.stash[i] = (uint16_t)(q + 1u);
+    else
+        atomicOr(X.stash_n, kDegraded);
 }
 
-// Turn the index entry of slot q (key K[q]) into a tombstone.
+// Remove the index entry of slot q (key K[q]).
 __device__ __forceinline__ void sl_erase(const stamp_lru &X, uint32_t q)
 {
-    uint32_t s = lru_home(X.K[q], X.tbits);
-    for (uint32_t it = 0; it <= X.mask; ++it) {
-        if (X.tab[s] == q + 1) {
-            X.tab[s] = kTomb;
+    const bkt_hash H = sl_hash(X.K[q], X.nbb);
+    const uint32_t ent = (H.tag << 11) | (q + 1u);
+#pragma unroll
+    for (int x = 0; x < 2; ++x) {
+        const uint32_t b = x ? H.b2 : H.b1;
+        const unsigned long long w = X.bkt[b];
+#pragma unroll
+        for (int p = 0; p < 4; ++p)
+            if (bkt_entry(w, p) == ent) {
+                atomicAnd(&X.bkt[b], ~(0xffffull << (16 * p)));
+                return;
+            }
+    }
+    const uint32_t sn = *X.stash_n & ~kDegraded;
+    for (uint32_t i = 0; i < sn && i < kStash; ++i)
+        if (X.stash[i] == q + 1u) {
+            X.stash[i] = 0;
             return;
         }
-        s = (s + 1) & X.mask;
-    }
 }
 
-// Index of slots 0 .. fill-1 from scratch (warp-cooperative); clears every tombstone.
+// Index of slots 0 .. fill-1 from scratch (warp-cooperative).
 __device__ __forceinline__ void sl_reindex(const stamp_lru &X, uint32_t fill, uint32_t lane)
 {
-    uint4 *t4 = reinterpret_cast<uint4 *>(X.tab);
-    for (uint32_t x = lane; x < (X.mask + 1) / 8; x += 32) t4[x] = make_uint4(0, 0, 0, 0);
+    uint4 *t4 = reinterpret_cast<uint4 *>(X.bkt);
+    for (uint32_t x = lane; x < (1u << X.nbb) / 2; x += 32) t4[x] = make_uint4(0, 0, 0, 0);
+    if (lane == 0) *X.stash_n = 0;
     __syncwarp();
     for (uint32_t q = lane; q < fill; q += 32) sl_insert(X, X.K[q], q);
     __syncwarp();
@@ -387,15 +463,15 @@ __device__ __forceinline__ void sl_compact(const stamp_lru &X, uint32_t fill, ui
 
 template <int NC, int NG, bool SMALL>
 __global__ void __launch_bounds__(128)
-k_lru_stamp(const replay_caps caps, uint32_t cmax, uint32_t nw, uint32_t R, uint32_t ns, uint32_t CL, int tbits,
+k_lru_stamp(const replay_caps caps, uint32_t cmax, uint32_t nw, uint32_t R, uint32_t ns, uint32_t CL, uint32_t nbb,
             const uint32_t *__restrict__ start, const uint32_t *__restrict__ coff, const uint32_t *__restrict__ total,
             const rec16 *__restrict__ rec, const replay_state st, unsigned long long *__restrict__ ctr,
             uint32_t *status)
 {
     extern __shared__ uint4 smb[];
     const uint32_t lane = cr_lane(), warp = threadIdx.x >> 5, wpb = blockDim.x >> 5;
-    const size_t per_warp = stamp_lru_bytes(cmax, nw, 1u << tbits);
-    const stamp_lru X = stamp_lru_at(reinterpret_cast<unsigned char *>(smb) + per_warp * warp, cmax, nw, tbits);
+    const size_t per_warp = stamp_lru_bytes(cmax, nw, nbb);
+    const stamp_lru X = stamp_lru_at(reinterpret_cast<unsigned char *>(smb) + per_warp * warp, cmax, nw, nbb);
 
     const uint32_t w = blockIdx.x * wpb + warp;
     if (w >= *total) return;
@@ -442,7 +518,7 @@ k_lru_stamp(const replay_caps caps, uint32_t cmax, uint32_t nw, uint32_t R, uint
             if (valid) key = v < back ? rec[p0 - 1 - v].key : kin[v - back];
             const uint32_t vm = __ballot_sync(0xffffffffu, valid);
             const uint32_t peers = __match_any_sync(0xffffffffu, key) & vm;
-            const bool fresh = valid && (peers & lt) == 0 && sl_lookup(X, key) == kNone;
+            const bool fresh = valid && (peers & lt) == 0 && sl_lookup(X, key, fill, cmax) == kNone;
             const uint32_t bal = __ballot_sync(0xffffffffu, fresh);
             const uint32_t pos = fill + __popc(bal & lt);
             __syncwarp();
@@ -457,7 +533,6 @@ k_lru_stamp(const replay_caps caps, uint32_t cmax, uint32_t nw, uint32_t R, uint
     __syncwarp();
     uint32_t wnow, lo;
     sl_stamps_in_order(X, fill, nw, lane, wnow, lo);
-    uint32_t tomb = 0;  // tombstones in the index
 
     unsigned long long my_req = 0, my_prompt = 0;
     unsigned long long my_hit[NC], my_tok[NC];
@@ -480,7 +555,7 @@ k_lru_stamp(const replay_caps caps, uint32_t cmax, uint32_t nw, uint32_t R, uint
         const uint32_t below = grp & lt, above = grp & gt;
         const bool first = valid && below == 0;
         const bool last = valid && above == 0;
-        uint32_t slot = first ? sl_lookup(X, mine.key) : kNone;
+        uint32_t slot = first ? sl_lookup(X, mine.key, fill, cmax) : kNone;
         const bool res = slot != kNone;  // first occurrence of a resident key
         uint32_t s_old = res ? (uint32_t)X.ST[slot] : 0u;
         if (s_old >= 32u * nw) {  // never: stamps stay inside the window (guards the bitmap)
@@ -493,35 +568,44 @@ k_lru_stamp(const replay_caps caps, uint32_t cmax, uint32_t nw, uint32_t R, uint
         LP.load(X.BM, nw, lane);
         const uint32_t bl = LP.below(s_old);
         const uint32_t D = res ? fill - 1u - bl : kAbsent;
-        // lanes that push request i deeper, for every lane at once, by comparing
-        // bit-sliced values from the most significant bit down (per bit: lanes
-        // still equal keep the ones with the same bit; a lane whose bit is 1
-        // where this lane's is 0 is decided greater):
-        //   first i:  first occurrences whose old position is deeper (D_l > D_i)
-        //   repeat i: lanes whose key does not recur before i (next_l > i); only
-        //             needed below capacity 32 (a repeat's depth is at most 31)
-        const uint32_t next = above ? (uint32_t)__ffs(above) - 1u : 32u;
-        uint32_t gN = 0, eN = 0xffffffffu, gD = 0, eD = 0xffffffffu;
+        // a first occurrence at old position D is pushed deeper by the step's earlier
+        // first occurrences that were deeper or absent: between the absent ones
+        // (jlo) and all of them (jhi).  Where that range straddles a capacity the
+        // exact count decides the hit: those lanes (a few per step) are counted one
+        // at a time against every lane; any count in the range decides the others.
+        const uint32_t firstm = __ballot_sync(0xffffffffu, first);
+        const uint32_t absm = __ballot_sync(0xffffffffu, first && !res);
+        const uint32_t jlo = (uint32_t)__popc(absm & lt), jhi = (uint32_t)__popc(firstm & lt);
+        bool amb = false;
 #pragma unroll
-        for (int bt = 10; bt >= 0; --bt) {
-            const uint32_t BD = __ballot_sync(0xffffffffu, (D >> bt) & 1u);
-            const uint32_t MD = 0u - ((D >> bt) & 1u);
-            gD |= eD & BD & ~MD;
-            eD &= ~(BD ^ MD);
-            if (SMALL && bt <= 5) {
+        for (int c = 0; c < NC; ++c)
+            if (c < (int)caps.n_caps && D + 1u + jlo <= caps.cap[c] && caps.cap[c] < D + 1u + jhi) amb = true;
+        uint32_t jx = jhi;
+        for (uint32_t am = __ballot_sync(0xffffffffu, res && amb); am; am &= am - 1u) {  // uniform
+            const uint32_t a = (uint32_t)__ffs(am) - 1u;
+            const uint32_t Da = __shfl_sync(0xffffffffu, D, a);
+            const uint32_t deeper = __ballot_sync(0xffffffffu, first && (!res || D > Da));
+            if (lane == a) jx = (uint32_t)__popc(deeper & lt);
+        }
+        uint32_t dep_rep = 1u;
+        if (SMALL) {
+            // a repeat of lane j: 1 + the distinct keys of lanes (j, i), i.e. the lanes
+            // there whose key does not recur before i (next occurrence lane > i);
+            // compared bit-sliced over the 6-bit next-occurrence lane; only needed
+            // below capacity 32 (a repeat's depth is at most 31)
+            const uint32_t next = above ? (uint32_t)__ffs(above) - 1u : 32u;
+            uint32_t gN = 0, eN = 0xffffffffu;
+#pragma unroll
+            for (int bt = 5; bt >= 0; --bt) {
                 const uint32_t BN = __ballot_sync(0xffffffffu, (next >> bt) & 1u);
                 const uint32_t MN = 0u - ((lane >> bt) & 1u);
                 gN |= eN & BN & ~MN;
                 eN &= ~(BN ^ MN);
             }
-        }
-        const uint32_t firstm = __ballot_sync(0xffffffffu, first);
-        uint32_t dep_rep = 1u;
-        if (SMALL) {  // repeat: lanes strictly between the previous occurrence and this one
             const uint32_t win = lt & ~((2u << (31u - (uint32_t)__clz(below | 1u))) - 1u);
             dep_rep = 1u + (uint32_t)__popc(gN & win);
         }
-        const uint32_t dep_first = res ? D + 1u + (uint32_t)__popc(gD & firstm & lt) : kNone;
+        const uint32_t dep_first = res ? D + 1u + jx : kNone;
         const uint32_t depth = !valid ? kNone : (first ? dep_first : dep_rep);
 #pragma unroll
         for (int c = 0; c < NC; ++c) {
@@ -534,7 +618,6 @@ k_lru_stamp(const replay_caps caps, uint32_t cmax, uint32_t nw, uint32_t R, uint
         // ---- state after the step ------------------------------------------------------
         const uint32_t lastm = __ballot_sync(0xffffffffu, last);
         const uint32_t u = (uint32_t)__popc(lastm);
-        const uint32_t absm = __ballot_sync(0xffffffffu, first && !res);
         const uint32_t mnew = (uint32_t)__popc(absm);
         if (SMALL && u > cmax) {
             // more distinct keys than the capacity: every old key leaves and the
@@ -555,7 +638,6 @@ k_lru_stamp(const replay_caps caps, uint32_t cmax, uint32_t nw, uint32_t R, uint
             }
             if (lane == 0) X.BM[wnow] = keepm;
             fill = cmax;
-            tomb = 0;
             lo = wnow;
             ++wnow;
         } else {
@@ -600,18 +682,15 @@ k_lru_stamp(const replay_caps caps, uint32_t cmax, uint32_t nw, uint32_t R, uint
                 done += take;
                 __syncwarp();
             }
-            tomb += done;
             // new keys take the never-used slots, then the freed ones
-            uint32_t reused = 0;
             if (first && !res) {
                 const uint32_t a = (uint32_t)__popc(absm & lt);
                 const uint32_t freecnt = cmax - fill;
                 const uint32_t q = a < freecnt ? fill + a : (uint32_t)X.EV[a - freecnt];
                 X.K[q] = mine.key;
-                reused = sl_insert(X, mine.key, q);
+                sl_insert(X, mine.key, q);
                 slot = q;
             }
-            tomb -= __reduce_add_sync(0xffffffffu, reused);
             // every key of the step takes the time of its last access
             const uint32_t fl = (uint32_t)__ffs(grp ? grp : 1u) - 1u;
             const uint32_t ks = __shfl_sync(0xffffffffu, slot, fl);
@@ -626,10 +705,6 @@ k_lru_stamp(const replay_caps caps, uint32_t cmax, uint32_t nw, uint32_t R, uint
         }
         __syncwarp();
         if (wnow == nw) sl_compact<NG>(X, fill, nw, lane, wnow, lo);
-        if (4 * (fill + tomb) > 3 * (X.mask + 1)) {  // too many tombstones: index afresh
-            sl_reindex(X, fill, lane);
-            tomb = 0;
-        }
     }
 
     // ---- counters -------------------------------------------------------------
@@ -677,9 +752,9 @@ int launch_stamp(cr_ctx *ctx, cr_replay *rp, const replay_caps &caps, uint32_t C
                  const uint32_t *coff, const uint32_t *total, uint64_t m, const rec16 *rec, uint64_t *d_ctr)
 {
     const uint32_t cmax = rp->cmax, nw = stamp_words(cmax);
-    int tbits = 6;
-    while ((1u << tbits) < 4 * cmax) ++tbits;  // index at most a quarter full of live keys
-    const size_t per_warp = stamp_lru_bytes(cmax, nw, 1u << tbits);
+    uint32_t nbb = 4;
+    while ((1u << nbb) < cmax) ++nbb;  // a bucket of four entries per resident key at most
+    const size_t per_warp = stamp_lru_bytes(cmax, nw, nbb);
     // warps per block: the most warps per SM that shared memory allows
     const size_t sm_bytes = 227 * 1024;
     uint32_t wpb = 4, best = 0;
@@ -702,8 +777,10 @@ int launch_stamp(cr_ctx *ctx, cr_replay *rp, const replay_caps &caps, uint32_t C
     st.fill_in = rp->d_fill[rp->cur];
     st.keys_out = rp->d_keys[rp->cur ^ 1];
     st.fill_out = rp->d_fill[rp->cur ^ 1];
+    const int pr = cr_prof_begin(ctx, ctx->stream, CR_PROF_REPLAY);
     CR_LAUNCH(ctx, (k_lru_stamp<NC, NG, SMALL>), (unsigned int)((items + wpb - 1) / wpb), wpb * 32, smem, caps, cmax,
-              nw, rp->R, ns, CL, tbits, start, coff, total, rec, st, (unsigned long long *)d_ctr, ctx->d_status);
+              nw, rp->R, ns, CL, nbb, start, coff, total, rec, st, (unsigned long long *)d_ctr, ctx->d_status);
+    cr_prof_end(ctx, ctx->stream, pr);
     rp->cur ^= 1;
     return CR_OK;
 }
@@ -1022,6 +1099,7 @@ extern "C" int cr_shadow_replay(cr_ctx *ctx, cr_replay *rp, const uint64_t *d_ke
                                 const uint32_t *d_slen, const uint16_t *d_dest, uint64_t n, uint64_t *d_ctr)
 {
     if (!ctx || !rp) return CR_EINVAL;
+    cr_nvtx_range nv("cr_shadow_replay");
     if (n == 0) return CR_OK;
     if (!d_key || !d_plen || !d_slen || !d_dest || !d_ctr)
         return cr_fail(ctx, CR_EINVAL, "cr_shadow_replay: NULL pointer");
@@ -1047,6 +1125,7 @@ extern "C" int cr_shadow_replay(cr_ctx *ctx, cr_replay *rp, const uint64_t *d_ke
         CR_CUDA(ctx, cudaFuncSetAttribute(k_part_count, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)csmem));
     if (ssmem > 48 * 1024)
         CR_CUDA(ctx, cudaFuncSetAttribute(k_part_scatter, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)ssmem));
+    const int pp = cr_prof_begin(ctx, ctx->stream, CR_PROF_PARTITION);
     CR_LAUNCH(ctx, k_part_count, pgrid, kPartBlock, csmem, d_dest, (unsigned long long)n, R, ntiles, cnt,
               ctx->d_status);
     CR_TRY(cr_scan_u32(ctx, cnt, cnt, ncnt, nrec));
@@ -1054,6 +1133,7 @@ extern "C" int cr_shadow_replay(cr_ctx *ctx, cr_replay *rp, const uint64_t *d_ke
               (const uint32_t *)nrec, start);
     CR_LAUNCH(ctx, k_part_scatter, pgrid, kPartBlock, ssmem, d_dest, (unsigned long long)n, R, ntiles,
               (const uint32_t *)cnt, (const unsigned long long *)d_key, d_plen, d_slen, rec);
+    cr_prof_end(ctx, ctx->stream, pp);
     replay_caps caps;
     caps.n_caps = rp->n_caps;
     for (uint32_t c = 0; c < CR_MAX_CAPS; ++c) caps.cap[c] = c < rp->n_caps ? rp->caps[c] : 0;
@@ -1062,9 +1142,11 @@ extern "C" int cr_shadow_replay(cr_ctx *ctx, cr_replay *rp, const uint64_t *d_ke
         const size_t tsmem = (size_t)kTokWarps * kTokMax * (sizeof(unsigned long long) + sizeof(uint32_t));
         if (tsmem > 48 * 1024)
             CR_CUDA(ctx, cudaFuncSetAttribute(k_lru_tokens, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)tsmem));
+        const int pt = cr_prof_begin(ctx, ctx->stream, CR_PROF_REPLAY);
         CR_LAUNCH(ctx, k_lru_tokens, (ns + kTokWarps - 1) / kTokWarps, kTokWarps * 32, tsmem, caps, ns, R,
                   (const uint32_t *)start, (const rec16 *)rec, (unsigned long long *)rp->d_keys[0], rp->d_size,
                   rp->d_fill[0], (unsigned long long *)d_ctr, ctx->d_status);
+        cr_prof_end(ctx, ctx->stream, pt);
         return CR_OK;
     }
     // chunk length: long enough that rebuilding an LRU state of cmax entries is amortised

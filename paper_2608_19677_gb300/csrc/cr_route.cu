@@ -623,6 +623,7 @@ extern "C" int cr_route_batch(cr_ctx *ctx, const cr_plan *const *plans, const cr
                               uint32_t batch_B, uint64_t *d_load, uint16_t *d_dest)
 {
     if (!ctx) return CR_EINVAL;
+    cr_nvtx_range nv("cr_route_batch");
     if (R == 0 || R > CR_MAX_R) return cr_fail(ctx, CR_EINVAL, "cr_route_batch: R=%u outside 1..%u", R, CR_MAX_R);
     if (n_rep == 0 || n_rep > CR_MAX_REPLICAS || !reps)
         return cr_fail(ctx, CR_EINVAL, "cr_route_batch: n_rep=%u outside 1..%u", n_rep, CR_MAX_REPLICAS);
@@ -679,9 +680,11 @@ extern "C" int cr_route_batch(cr_ctx *ctx, const cr_plan *const *plans, const cr
     CR_TRY(cr_scratch(ctx, SCR_ROUTE_DESC, (size_t)n * n_rep * sizeof(uint32_t), &pc));
     uint32_t *cand = (uint32_t *)pc;
     const unsigned int gcap = (unsigned int)ctx->num_sms * 16u;
+    const int pcand = cr_prof_begin(ctx, ctx->stream, CR_PROF_ROUTE_CAND);
     CR_LAUNCH(ctx, k_route_cand, cr_blocks(n * n_rep, 256, gcap), 256, 0, args, n_rep,
               (const unsigned long long *)d_key, (unsigned long long)n, (unsigned long long)first_req_index, R, cand,
               d_dest);
+    cr_prof_end(ctx, ctx->stream, pcand);
     // load counts of RR / HASH replicas (their choices never read the load)
     for (uint32_t i = 0; i < n_rep; ++i) {
         if (reps[i].policy != CR_POLICY_RR && reps[i].policy != CR_POLICY_HASH) continue;
@@ -696,7 +699,11 @@ extern "C" int cr_route_batch(cr_ctx *ctx, const cr_plan *const *plans, const cr
         CR_CUDA(ctx, cudaEventRecord(ctx->ev_cand, ctx->stream));
         CR_CUDA(ctx, cudaStreamWaitEvent(rs, ctx->ev_cand, 0));
     }
-    if (n_dep) CR_TRY(launch_resolve(ctx, rs, args, cand, n, batch_B, R, mc, n_dep, d_load, d_dest));
+    if (n_dep) {
+        const int pr = cr_prof_begin(ctx, rs, CR_PROF_ROUTE_RESOLVE);
+        CR_TRY(launch_resolve(ctx, rs, args, cand, n, batch_B, R, mc, n_dep, d_load, d_dest));
+        cr_prof_end(ctx, rs, pr);
+    }
     if (split) {
         CR_CUDA(ctx, cudaEventRecord(ctx->ev_resolve, rs));
         ctx->resolve_recorded = 1;

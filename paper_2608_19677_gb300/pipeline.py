@@ -366,7 +366,8 @@ class TracePipeline:
     def __init__(self, ctx: Context, R: int, W: int, caps: Sequence[int],
                  replicas: Sequence[Tuple[str, int]], qcap: Callable[[int], Tuple[int, int]],
                  max_n: int, batch_B: int = 1024, depth: int = 8, plan_streams: int = 4,
-                 route_streams: int = 4, vnodes: int = 64, fresh: bool = False, lru_tokens: bool = False):
+                 route_streams: int = 4, vnodes: int = 64, fresh: bool = False, lru_tokens: bool = False,
+                 replay_first: bool = True):
         import torch
         self.ctx, self.R, self.W, self.caps = ctx, R, W, list(caps)
         self.replicas = list(replicas)
@@ -387,12 +388,16 @@ class TracePipeline:
             self.rep_plan.append(self.plan_keys.index(k))
         self.depth = max(1, depth)
         self.mstream = ctx._stream_obj
+        # The replay is the one serial chain (interval after interval); with
+        # ``replay_first`` its stream has the high priority, so that its kernels take
+        # SMs ahead of the plans and routes of later intervals, which have slack.
         lo, hi = torch.cuda.Stream.priority_range() if hasattr(torch.cuda.Stream, "priority_range") else (0, -1)
-        self.pstreams = [torch.cuda.Stream(self.dev, priority=hi) for _ in range(max(1, plan_streams))]
+        self.pstreams = [torch.cuda.Stream(self.dev, priority=lo if replay_first else hi)
+                         for _ in range(max(1, plan_streams))]
         self.pctxs = [Context(ctx.device, s) for s in self.pstreams]
-        self.rstreams = [torch.cuda.Stream(self.dev) for _ in range(max(1, route_streams))]
+        self.rstreams = [torch.cuda.Stream(self.dev, priority=lo) for _ in range(max(1, route_streams))]
         self.rctxs = [Context(ctx.device, s) for s in self.rstreams]
-        self.ystream = torch.cuda.Stream(self.dev)
+        self.ystream = torch.cuda.Stream(self.dev, priority=hi if replay_first else lo)
         self.yctx = Context(ctx.device, self.ystream)
         self.plans = [[Plan(self.pctxs[0]) for _ in self.plan_keys] for _ in range(self.depth)]
         self.replay = Replay(ctx, len(self.replicas), R, self.caps, tokens=lru_tokens)
@@ -428,10 +433,12 @@ class TracePipeline:
     def dest_view(self, b: int, n: int):
         return self.dests[b][:len(self.replicas) * n].view(len(self.replicas), n)
 
-    def run(self, keys, plens, slens, g0s, mark: bool = False, on_interval=None):
+    def run(self, keys, plens, slens, g0s, mark: bool = False, on_interval=None, ready=None):
         """Enqueue every interval of the trace (lists of device tensors and first request
         indices) after the work already on the main stream; the main stream then waits for
         all of it.  Counters accumulate in ``ctr`` (call ``reset`` between runs).
+        ``ready[t]``, when given, is an event after which interval t's tensors may be read
+        (e.g. the end of their host-to-device copy).
         ``on_interval(t, dest, plans)``, when given, is called after interval t is enqueued
         with its destinations view and plans (a test hook: the caller must order its reads
         after the pipeline's streams, e.g. by ``sync``, before the buffer's reuse)."""
@@ -453,22 +460,27 @@ class TracePipeline:
                 pc = self.pctxs[t % len(self.pctxs)]
                 if self._plan_free[b] is not None:
                     ps.wait_event(self._plan_free[b])
-                pk = keys[t] if (t == 0 or self.fresh) else keys[t - 1]
+                pt = t if (t == 0 or self.fresh) else t - 1
+                pk = keys[pt]
+                if ready is not None:
+                    ps.wait_event(ready[pt])
                 num, den = self.qcap(int(pk.shape[0]))
                 params = [plan_params(self.R, self.W, num, den, v, seed=s, epoch=t) for v, s in self.plan_keys]
                 p0 = self._event(ps, True) if mark else None
                 build_plans(pc, pk, params, self.plans[b])
-                ready = self._event(ps, mark)
+                built = self._event(ps, mark)
                 if mark:
-                    self.plan_marks.append((p0, ready))
+                    self.plan_marks.append((p0, built))
                 plans = [self.plans[b][i] if i is not None else None for i in self.rep_plan]
             # ---- route of interval t ---------------------------------------------------
             q = t % len(self.rstreams)
             rs, rc = self.rstreams[q], self.rctxs[q]
             if plans is not None:
-                rs.wait_event(ready)
+                rs.wait_event(built)
             if self._dest_free[b] is not None:
                 rs.wait_event(self._dest_free[b])
+            if ready is not None:
+                rs.wait_event(ready[t])  # the replay follows the route, so it sees the inputs too
             dest = self.dest_view(b, n)
             r0 = self._event(rs, True) if mark else None
             with torch.cuda.stream(rs):
@@ -493,18 +505,24 @@ class TracePipeline:
             self.mstream.wait_event(self._event(s))
 
     def reset(self):
-        """Empty the simulators and counters (ordered on the main stream after earlier work)."""
+        """Empty the simulators and counters.  Both are enqueued on the main stream, which
+        ``run`` left waiting for all of the pipeline's streams and which the next ``run``
+        makes every stream wait for: no host synchronisation is needed."""
         import torch
-        self.sync()
         self.replay.reset()
         with torch.cuda.stream(self.mstream):
             self.ctr.zero_()
-        self.ctx.sync()
         self._reset_events()
 
     def sync(self):
         for c in self.contexts:
             c.sync()
+
+    def quiesce(self):
+        """Wait for all enqueued work and forget the events that ordered it (e.g. before
+        capturing a CUDA graph of ``run``)."""
+        self.sync()
+        self._reset_events()
 
     def close(self):
         self.sync()

@@ -858,3 +858,35 @@ def test_split_route_error_reported_by_sync(P):
         ring.close()
     finally:
         c.close()
+
+
+def test_profile_events_time_each_launch(P):
+    # per-launch timing: every timed kind of launch is counted once per call, with a positive duration
+    c = P.Context(0)
+    try:
+        c.profile_enable(64)
+        cfg = tg.CONFIGS["70b"].scaled(20000, 1)
+        tr = tg.Trace(cfg)
+        iv = tr.interval(0)
+        tok, off = tg.arena_host(tr, iv, 4)
+        keys = P.hash_prefixes(c, torch.from_numpy(tok).to(DEV), d_u64(off), d_u32(iv.plen))
+        num, den = tr.qcap(iv.n)
+        plan = P.build_plan(c, keys, P.plan_params(cfg.R, cfg.W, num, den, "LPT"))
+        load = torch.zeros((2, cfg.R), dtype=torch.int64, device=DEV)
+        dest = P.route_batch(c, [plan, None], ["CR", "P2C"], [0, 0], cfg.R, keys, iv.g0, 1024, load)
+        rp = P.Replay(c, 2, cfg.R, cfg.caps)
+        ctr = torch.zeros((2, 1, cfg.R, 5), dtype=torch.int64, device=DEV)
+        P.shadow_replay(c, rp, keys, d_u32(iv.plen), d_u32(iv.slen), dest, ctr)
+        c.sync()
+        for tag in ("hash", "plan", "route_cand", "route_resolve", "partition", "replay"):
+            n, ms = c.profile_read(tag)
+            assert n == 1 and ms > 0.0, tag
+        c.profile_enable(0)
+        assert c.profile_read("replay") == (0, 0.0)
+        import ctypes
+        n_, ms_ = ctypes.c_uint64(), ctypes.c_double()
+        assert P.lib().cr_profile_read(c.handle, 99, ctypes.byref(n_), ctypes.byref(ms_)) == P.CR_EINVAL
+        rp.close()
+        plan.close()
+    finally:
+        c.close()

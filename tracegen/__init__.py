@@ -418,7 +418,7 @@ def _tokens_lib():
         L = ctypes.CDLL(lib)
         L.tg_prefix_tokens.restype = None
         L.tg_prefix_tokens.argtypes = [ctypes.c_void_p, ctypes.c_void_p, ctypes.c_uint64, ctypes.c_int64,
-                                       ctypes.c_int64, ctypes.c_void_p, ctypes.c_void_p]
+                                       ctypes.c_int64, ctypes.c_void_p, ctypes.c_void_p, ctypes.c_uint64]
         _ctok = L
     return _ctok
 
@@ -430,8 +430,23 @@ def prefix_spans(trace: Trace, key_ids) -> Tuple[np.ndarray, np.ndarray, np.ndar
     total = int(pl.astype(np.int64).sum())
     tok = np.empty(max(total, 1), dtype=np.int32)
     off = np.empty(max(ids.size, 1), dtype=np.uint64)
-    _tokens_lib().tg_prefix_tokens(ids.ctypes.data, pl.ctypes.data, ids.size, trace.cfg.trace_seed,
-                                   trace.cfg.vocab, tok.ctypes.data, off.ctypes.data)
+    start = np.zeros(ids.size + 1, dtype=np.int64)
+    np.cumsum(pl, out=start[1:])
+    L = _tokens_lib()
+
+    def fill(ab):  # keys [a, b) into their slice of the arena (the C call releases the GIL)
+        a, b = ab
+        if b > a:
+            L.tg_prefix_tokens(ids.ctypes.data + 8 * a, pl.ctypes.data + 4 * a, b - a, trace.cfg.trace_seed,
+                               trace.cfg.vocab, tok.ctypes.data + 4 * int(start[a]), off.ctypes.data + 8 * a,
+                               int(start[a]))
+
+    import concurrent.futures as cf
+    import os
+    nt = max(1, min(os.cpu_count() or 1, 16, ids.size // 256 + 1))
+    cuts = [ids.size * i // nt for i in range(nt + 1)]
+    with cf.ThreadPoolExecutor(nt) as ex:
+        list(ex.map(fill, zip(cuts[:-1], cuts[1:])))
     return tok[:total], off[:ids.size], pl
 
 
