@@ -264,6 +264,22 @@ CR_API int cr_plan_export(cr_ctx *ctx, const cr_plan *plan, uint64_t *ukey, uint
                    uint64_t *adm_key, uint64_t *adm_cnt, uint32_t *adm_k, uint32_t *koff,
                    uint16_t *members, uint64_t *jobs, uint64_t *load);
 
+/* Blocking: install a plan computed elsewhere -- for example one exported by
+ * cr_plan_export from another process, or a host planner's table (the paper's
+ * planner runs on the host, sec. 3.1) -- so that cr_route_batch can route
+ * with it.  Host arrays in admission order, as cr_plan_export gives them:
+ *   adm_key[n_adm], adm_cnt[n_adm], adm_k[n_adm]   keys, their rates, k_b
+ *   members[sum k_b]   T(b) of each key in turn (uint16; the first member of
+ *                      a key breaks ties first, as in dispatch)
+ *   jobs[sum k_b], load[R]   optional (NULL: zeros); kept for export only
+ * The plan's histogram becomes the admitted keys with their rates.  Errors:
+ * CR_EINVAL (R or W out of range, n_adm or sum k_b above R*W, k_b of 0 or
+ * above R, a member >= R or repeated within a key, a repeated key, NULL
+ * arrays), CR_ENOMEM, CR_ECUDA. */
+CR_API int cr_plan_import(cr_ctx *ctx, cr_plan *plan, uint32_t R, uint32_t W, uint64_t n_adm, const uint64_t *adm_key,
+                          const uint64_t *adm_cnt, const uint32_t *adm_k, const uint16_t *members,
+                          const uint64_t *jobs, const uint64_t *load);
+
 /* ==== f2: plan difference (replanning under drift) ===================== */
 
 /* Integer counts describing how plan b differs from plan a (supplement
@@ -416,6 +432,16 @@ CR_API int cr_shadow_replay(cr_ctx *ctx, cr_replay *rp, const uint64_t *d_key, c
  * The state at a smaller capacity c is the first min(c, fill) of them. */
 CR_API int cr_replay_export_state(cr_ctx *ctx, const cr_replay *rp, uint32_t rep, uint32_t r,
                            uint64_t *keys_out, uint32_t *fill_out);
+
+/* Blocking: set one simulator's resident keys (host array, most recent
+ * first, distinct, at most the largest capacity), e.g. from
+ * cr_replay_export_state, so that a replay can resume from saved state; the
+ * simulators of smaller capacities hold the first min(c, fill) of them.
+ * Prefix-count replays only (a token-weighted replay also keeps each prefix's
+ * size).  Errors: CR_EINVAL (bad stream, too many keys, repeated key, token
+ * replay), CR_ECUDA. */
+CR_API int cr_replay_import_state(cr_ctx *ctx, cr_replay *rp, uint32_t rep, uint32_t r, const uint64_t *keys,
+                                  uint32_t fill);
 
 /* ==== allocation-free key histogram ================================== */
 /*

@@ -39,7 +39,7 @@ EXPORTS = ("cr_create", "cr_destroy", "cr_set_stream", "cr_sync", "cr_last_error
            "cr_replay_destroy", "cr_shadow_replay", "cr_replay_export_state", "cr_key_histogram_noalloc",
            "cr_ring_create", "cr_ring_destroy", "cr_ring_export", "cr_plan_diff",
            "cr_replay_create_tokens", "cr_set_resolve_stream", "cr_partition_create", "cr_partition_destroy",
-           "cr_profile_enable", "cr_profile_read")
+           "cr_profile_enable", "cr_profile_read", "cr_plan_import", "cr_replay_import_state")
 PROF = {"hash": 0, "plan": 1, "route_cand": 2, "route_resolve": 3, "partition": 4, "replay": 5}
 CR_NOALLOC_MAX_KEYS = 65536
 
@@ -119,6 +119,8 @@ def lib() -> C.CDLL:
         "cr_set_resolve_stream": ([vp, vp], i32),
         "cr_partition_create": ([i32, u32, C.POINTER(vp), C.POINTER(vp), C.POINTER(vp)], i32),
         "cr_partition_destroy": ([vp], i32),
+        "cr_plan_import": ([vp, vp, u32, u32, u64, vp, vp, vp, vp, vp, vp], i32),
+        "cr_replay_import_state": ([vp, vp, u32, u32, vp, u32], i32),
         "cr_profile_enable": ([vp, u32], i32),
         "cr_profile_read": ([vp, u32, C.POINTER(C.c_uint64), C.POINTER(C.c_double)], i32),
     }
@@ -248,6 +250,19 @@ class Plan:
                    adm_k=a["adm_k"][:na], koff=a["koff"], members=a["members"][:sk], jobs=a["jobs"][:sk],
                    load=a["load"])
         return out
+
+    def load(self, R: int, W: int, adm_key, adm_cnt, adm_k, members, jobs=None, load=None):
+        """Install a plan given as host arrays in admission order (cr_plan_import)."""
+        ak = np.ascontiguousarray(adm_key, np.uint64)
+        ac = np.ascontiguousarray(adm_cnt, np.uint64)
+        kk = np.ascontiguousarray(adm_k, np.uint32)
+        mm = np.ascontiguousarray(members, np.uint16)
+        jb = None if jobs is None else np.ascontiguousarray(jobs, np.uint64)
+        ld = None if load is None else np.ascontiguousarray(load, np.uint64)
+        self.ctx.check(lib().cr_plan_import(self.ctx.handle, self._h, R, W, ak.size, _np_ptr(ak), _np_ptr(ac),
+                                            _np_ptr(kk), _np_ptr(mm), None if jb is None else _np_ptr(jb),
+                                            None if ld is None else _np_ptr(ld)), "cr_plan_import")
+        return self
 
     def close(self):
         if getattr(self, "_h", None):
@@ -409,6 +424,12 @@ class Replay:
 
     def reset(self):
         self.ctx.check(lib().cr_replay_reset(self.ctx.handle, self._h), "cr_replay_reset")
+
+    def set_state(self, rep: int, r: int, keys):
+        """Resident keys of one simulator, most recent first (cr_replay_import_state)."""
+        k = np.ascontiguousarray(keys, np.uint64)
+        self.ctx.check(lib().cr_replay_import_state(self.ctx.handle, self._h, rep, r,
+                                                    _np_ptr(k) if k.size else None, k.size), "cr_replay_import_state")
 
     def state(self, rep: int, r: int) -> np.ndarray:
         out = np.zeros(MAX_CAP, np.uint64)

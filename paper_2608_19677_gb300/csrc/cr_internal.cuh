@@ -36,7 +36,8 @@ enum cr_scratch_slot {
     SCR_PLAN_C,
     SCR_REPLAY_IDX,    // partitioned request indices
     SCR_REPLAY_START,  // per-stream start offsets
-    SCR_REPLAY_REC,    // gathered (key, prefix, suffix) records in stream order
+    SCR_REPLAY_REC,    // request indices in stream order
+    SCR_REPLAY_RECS,   // (key, prefix, suffix) record of each request
     SCR_REPLAY_CHUNK,  // per-stream chunk counts -> offsets, and their total
     SCR_ROUTE_DESC,    // per-replica route descriptors
     SCR_DIFF,          // plan-difference counters

@@ -1977,3 +1977,126 @@ extern "C" int cr_key_histogram_noalloc(const uint64_t *d_key, uint64_t n, uint6
         return cr_fail(NULL, CR_ECUDA, "cr_key_histogram_noalloc: launch failed: %s", cudaGetErrorString(e));
     return CR_OK;
 }
+
+// ---- plan import (a table computed elsewhere, e.g. exported earlier) --------
+namespace {
+struct imp_ent {
+    unsigned long long key, cnt;
+};
+int cmp_imp(const void *a, const void *b)
+{
+    const unsigned long long x = ((const imp_ent *)a)->key, y = ((const imp_ent *)b)->key;
+    return x < y ? -1 : (x > y ? 1 : 0);
+}
+}  // namespace
+
+extern "C" int cr_plan_import(cr_ctx *ctx, cr_plan *p, uint32_t R, uint32_t W, uint64_t n_adm, const uint64_t *adm_key,
+                              const uint64_t *adm_cnt, const uint32_t *adm_k, const uint16_t *members,
+                              const uint64_t *jobs, const uint64_t *load)
+{
+    if (!ctx || !p) return CR_EINVAL;
+    cr_nvtx_range nv("cr_plan_import");
+    if (R == 0 || R > CR_MAX_R || W == 0) return cr_fail(ctx, CR_EINVAL, "cr_plan_import: R=%u W=%u", R, W);
+    const uint64_t C = (uint64_t)R * W;
+    if (n_adm > C) return cr_fail(ctx, CR_EINVAL, "cr_plan_import: %llu keys exceed C = R*W", (unsigned long long)n_adm);
+    if (n_adm && (!adm_key || !adm_cnt || !adm_k || !members))
+        return cr_fail(ctx, CR_EINVAL, "cr_plan_import: NULL array");
+    // host checks: every k in 1..R, sum of k <= C, members < R and distinct per key, keys distinct
+    uint64_t sum_k = 0, max_k = 0, adm_lam = 0;
+    for (uint64_t a = 0; a < n_adm; ++a) {
+        if (adm_k[a] == 0 || adm_k[a] > R)
+            return cr_fail(ctx, CR_EINVAL, "cr_plan_import: key %llu has k=%u", (unsigned long long)a, adm_k[a]);
+        sum_k += adm_k[a];
+        max_k = adm_k[a] > max_k ? adm_k[a] : max_k;
+        adm_lam += adm_cnt[a];
+    }
+    if (sum_k > C) return cr_fail(ctx, CR_EINVAL, "cr_plan_import: sum of k exceeds C = R*W");
+    uint32_t *koff = (uint32_t *)malloc((n_adm + 1) * sizeof(uint32_t));
+    imp_ent *srt = (imp_ent *)malloc((n_adm + 1) * sizeof(imp_ent));
+    uint8_t *seen = (uint8_t *)calloc(R, 1);
+    int bad = !koff || !srt || !seen;
+    if (!bad) {
+        koff[0] = 0;
+        for (uint64_t a = 0; a < n_adm && !bad; ++a) {
+            koff[a + 1] = koff[a] + adm_k[a];
+            for (uint32_t j = koff[a]; j < koff[a + 1]; ++j) {
+                if (members[j] >= R || seen[members[j]]) bad = 2;
+                else seen[members[j]] = 1;
+            }
+            for (uint32_t j = koff[a]; j < koff[a + 1]; ++j)
+                if (members[j] < R) seen[members[j]] = 0;
+            srt[a].key = adm_key[a];
+            srt[a].cnt = adm_cnt[a];
+        }
+        if (!bad) {
+            qsort(srt, n_adm, sizeof(imp_ent), cmp_imp);
+            for (uint64_t a = 1; a < n_adm; ++a)
+                if (srt[a].key == srt[a - 1].key) bad = 3;
+        }
+    }
+    int st = CR_OK;
+    if (bad == 1) st = cr_fail(ctx, CR_ENOMEM, "cr_plan_import: host allocation failed");
+    else if (bad == 2) st = cr_fail(ctx, CR_EINVAL, "cr_plan_import: a member is >= R or repeated within a key");
+    else if (bad == 3) st = cr_fail(ctx, CR_EINVAL, "cr_plan_import: a key is listed twice");
+    if (st == CR_OK) st = plan_reserve(ctx, p, n_adm, R, W);
+    if (st == CR_OK) {
+        cudaStream_t s = ctx->stream;
+        // the histogram of an imported plan is its admitted keys, ascending
+        unsigned long long *hk = (unsigned long long *)malloc((n_adm + 1) * 16);
+        if (!hk) st = cr_fail(ctx, CR_ENOMEM, "cr_plan_import: host allocation failed");
+        for (uint64_t a = 0; hk && a < n_adm; ++a) {
+            hk[a] = srt[a].key;
+            hk[n_adm + 1 + a] = srt[a].cnt;
+        }
+        cr_plan_info_dev d;
+        memset(&d, 0, sizeof(d));
+        d.n = adm_lam;
+        d.U = n_adm;
+        d.S = n_adm;
+        d.n_adm = n_adm;
+        d.sum_k = sum_k;
+        d.max_k = max_k;
+        d.adm_lam = adm_lam;
+        auto up = [&](void *dst, const void *src, size_t bytes) -> int {
+            if (bytes && cudaMemcpyAsync(dst, src, bytes, cudaMemcpyHostToDevice, s) != cudaSuccess)
+                return cr_fail(ctx, CR_ECUDA, "cr_plan_import: copy failed");
+            return CR_OK;
+        };
+        if (st == CR_OK) st = up(p->d_ukey, hk, n_adm * 8);
+        if (st == CR_OK) st = up(p->d_ucnt, hk + n_adm + 1, n_adm * 8);
+        if (st == CR_OK) st = up(p->d_adm_key, adm_key, n_adm * 8);
+        if (st == CR_OK) st = up(p->d_adm_cnt, adm_cnt, n_adm * 8);
+        if (st == CR_OK) st = up(p->d_adm_k, adm_k, n_adm * 4);
+        if (st == CR_OK) st = up(p->d_koff, koff, (n_adm + 1) * 4);
+        if (st == CR_OK) st = up(p->d_members, members, sum_k * 2);
+        if (st == CR_OK && jobs) st = up(p->d_jobs, jobs, sum_k * 8);
+        if (st == CR_OK && !jobs && sum_k && cudaMemsetAsync(p->d_jobs, 0, sum_k * 8, s) != cudaSuccess)
+            st = cr_fail(ctx, CR_ECUDA, "cr_plan_import: memset failed");
+        if (st == CR_OK && load) st = up(p->d_load, load, (size_t)R * 8);
+        if (st == CR_OK && !load && cudaMemsetAsync(p->d_load, 0, (size_t)R * 8, s) != cudaSuccess)
+            st = cr_fail(ctx, CR_ECUDA, "cr_plan_import: memset failed");
+        if (st == CR_OK) st = up(p->d_info, &d, sizeof(d));
+        if (st == CR_OK && cudaMemsetAsync(p->d_table, 0xff, p->table_slots * sizeof(cr_table_slot), s) != cudaSuccess)
+            st = cr_fail(ctx, CR_ECUDA, "cr_plan_import: memset failed");
+        if (st == CR_OK && n_adm) {
+            const int bits = bits_for(p->table_slots - 1);
+            CR_LAUNCH(ctx, k_table_insert, cr_blocks(n_adm, 256, (unsigned int)ctx->num_sms * 8u), 256, 0,
+                      (const cr_plan_info_dev *)p->d_info, (const unsigned long long *)p->d_adm_key,
+                      (const uint32_t *)p->d_adm_k, (const uint32_t *)p->d_koff, (const uint16_t *)p->d_members,
+                      p->d_table, bits);
+        }
+        if (st == CR_OK) {
+            p->n = adm_lam;
+            p->qnum = 1;
+            p->qden = 1;
+            p->variant = CR_VARIANT_LPT;
+            p->built = 1;
+            st = cr_sync(ctx);  // the host arrays may be reused as soon as the call returns
+        }
+        free(hk);
+    }
+    free(koff);
+    free(srt);
+    free(seen);
+    return st;
+}

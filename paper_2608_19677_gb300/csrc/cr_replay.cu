@@ -1,8 +1,9 @@
 // a8, a9: shadow replay (cr_shadow_replay).
 //
 //   partition  one stable counting sort per replica by destination: each
-//              (replica, destination) stream's (key, prefix, suffix) records
-//              in arrival order
+//              (replica, destination) stream's request indices in arrival
+//              order; the replay gathers each request's (key, prefix, suffix)
+//              record, packed once per call, through them
 //   replay     one warp per (stream, chunk); the stream's LRU at the LARGEST
 //              capacity lives in shared memory as keys with recency stamps, a
 //              bitmap of live stamps and a hash index, and 32 requests are
@@ -31,15 +32,31 @@ struct rec16 {
     uint32_t P, S;
 };
 
+__device__ __forceinline__ uint32_t warp_incl_scan(uint32_t v, uint32_t lane)
+{
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        const uint32_t y = __shfl_up_sync(0xffffffffu, v, o);
+        if (lane >= (uint32_t)o) v += y;
+    }
+    return v;
+}
+
 // ---- partition: one stable counting sort per replica, by destination --------
-// Tiles of 2048 requests.  k_part_count writes each tile's destination counts
+// Tiles of 8192 requests.  k_part_count writes each tile's destination counts
 // at [(replica * R + r) * ntiles + tile]; one exclusive scan of that array
 // gives every (stream, tile) its output base, in stream-major order.
-// k_part_scatter ranks each tile's requests stably and writes their
-// (key, prefix, suffix) records straight to their place in stream order.
+// k_part_scatter ranks each tile's requests stably (warp-private counters),
+// stages their request indices in shared memory in (destination, arrival)
+// order, and writes them out so that consecutive threads write consecutive
+// positions of a destination's run.  The replay reads each request's
+// (key, prefix, suffix) record, packed once per call by k_part_records,
+// through these indices.
 constexpr int kPartBlock = 256;
 constexpr int kPartWarps = kPartBlock / 32;
-constexpr int kPartTile = kPartBlock * 8;
+constexpr int kPartPer = 32;                      // requests per thread
+constexpr int kPartTile = kPartBlock * kPartPer;  // 8192
+constexpr uint32_t kNoDest = 0xffffu;
 
 __global__ void __launch_bounds__(kPartBlock) k_part_count(const uint16_t *__restrict__ dest, unsigned long long n,
                                                            uint32_t R, uint32_t ntiles, uint32_t *__restrict__ cnt,
@@ -52,16 +69,16 @@ __global__ void __launch_bounds__(kPartBlock) k_part_count(const uint16_t *__res
     const uint16_t *D = dest + (unsigned long long)rep * n;
     const unsigned long long base = (unsigned long long)tile * kPartTile;
     bool bad = false;
-#pragma unroll
-    for (int j = 0; j < 8; ++j) {
+#pragma unroll 4
+    for (int j = 0; j < kPartPer; ++j) {
         const unsigned long long i = base + (unsigned long long)j * kPartBlock + threadIdx.x;
-        uint32_t d = i < n ? D[i] : 0xffffu;
+        uint32_t d = i < n ? D[i] : kNoDest;
         if (i < n && d >= R) {
             bad = true;
-            d = 0xffffu;  // skipped: reported through the status word
+            d = kNoDest;  // skipped: reported through the status word
         }
         const uint32_t peers = __match_any_sync(0xffffffffu, d);
-        if (d != 0xffffu && (peers & ((1u << lane) - 1u)) == 0) atomicAdd(&hist[d], (uint32_t)__popc(peers));
+        if (d != kNoDest && (peers & ((1u << lane) - 1u)) == 0) atomicAdd(&hist[d], (uint32_t)__popc(peers));
     }
     __syncthreads();
     for (uint32_t r = threadIdx.x; r < R; r += kPartBlock)
@@ -77,66 +94,128 @@ __global__ void k_part_starts(const uint32_t *__restrict__ off, uint32_t ns, uin
         start[s] = s < ns ? off[(unsigned long long)s * ntiles] : *total;
 }
 
-// Warp w ranks items [256w, 256w+256) of the tile in 8 rounds against
-// warp-private counters (u16, destination-major); one pass over the
-// destinations turns them into per-warp offsets.
+// Shared memory of k_part_scatter: per-warp counters wc[R][8] (u16), the
+// tile's destination offsets toff[R] (u32), each item's (destination << 16 |
+// rank among its warp's items of that destination) (u32), and the tile's items
+// in (destination, arrival) order (u16 item numbers).
+__host__ __device__ inline size_t part_scatter_smem(uint32_t R)
+{
+    return (size_t)R * kPartWarps * 2 + (size_t)R * 4 + (size_t)kPartTile * 6;
+}
+
 __global__ void __launch_bounds__(kPartBlock) k_part_scatter(const uint16_t *__restrict__ dest, unsigned long long n,
                                                              uint32_t R, uint32_t ntiles,
                                                              const uint32_t *__restrict__ off,
-                                                             const unsigned long long *__restrict__ keys,
-                                                             const uint32_t *__restrict__ plen,
-                                                             const uint32_t *__restrict__ slen,
-                                                             rec16 *__restrict__ rec)
+                                                             uint32_t *__restrict__ out, unsigned long long m)
 {
-    extern __shared__ uint16_t wc[];  // [R][8]
+    extern __shared__ uint4 psm[];
+    uint16_t *wc = reinterpret_cast<uint16_t *>(psm);                            // [R][8]
+    uint32_t *toff = reinterpret_cast<uint32_t *>(wc + (size_t)R * kPartWarps);  // [R]
+    uint32_t *spk = toff + R;                                                    // [kPartTile]
+    uint16_t *sitem = reinterpret_cast<uint16_t *>(spk + kPartTile);            // [kPartTile]
+    __shared__ uint32_t part[kPartBlock];
+    __shared__ uint32_t s_valid;
     const uint32_t rep = blockIdx.y, tile = blockIdx.x, lane = cr_lane(), warp = threadIdx.x >> 5;
     const uint32_t lt = (1u << lane) - 1u;
     uint4 *wc4 = reinterpret_cast<uint4 *>(wc);
     for (uint32_t r = threadIdx.x; r < R; r += kPartBlock) wc4[r] = make_uint4(0, 0, 0, 0);
     __syncthreads();
     const uint16_t *D = dest + (unsigned long long)rep * n;
-    const unsigned long long base = (unsigned long long)tile * kPartTile + (unsigned long long)warp * 256;
-    uint32_t dig[8], rank[8];
-#pragma unroll
-    for (int j = 0; j < 8; ++j) {
-        const unsigned long long i = base + (unsigned long long)j * 32 + lane;
-        uint32_t d = i < n ? D[i] : 0xffffu;
-        if (d >= R) d = 0xffffu;
+    const unsigned long long base = (unsigned long long)tile * kPartTile;
+    const uint32_t cnt = (uint32_t)min((unsigned long long)kPartTile, n - base);
+    // ranks: warp w takes items [1024 w, 1024 w + 1024) of the tile, 32 at a time
+    constexpr uint32_t kPerWarp = kPartTile / kPartWarps;
+    for (uint32_t j = 0; j < (uint32_t)kPartPer; ++j) {
+        const uint32_t it = warp * kPerWarp + j * 32u + lane;
+        uint32_t d = it < cnt ? D[base + it] : kNoDest;
+        if (d >= R) d = kNoDest;
         const uint32_t peers = __match_any_sync(0xffffffffu, d);
-        const uint32_t before = d != 0xffffu ? wc[d * kPartWarps + warp] : 0u;
-        rank[j] = before + __popc(peers & lt);
-        dig[j] = d;
+        const uint32_t before = d != kNoDest ? wc[d * kPartWarps + warp] : 0u;
+        spk[it] = (d << 16) | (before + (uint32_t)__popc(peers & lt));
         __syncwarp();
-        if (d != 0xffffu && (peers & lt) == 0) wc[d * kPartWarps + warp] = (uint16_t)(before + __popc(peers));
+        if (d != kNoDest && (peers & lt) == 0) wc[d * kPartWarps + warp] = (uint16_t)(before + __popc(peers));
         __syncwarp();
     }
     __syncthreads();
-    for (uint32_t r = threadIdx.x; r < R; r += kPartBlock) {  // exclusive prefix over the 8 warps
+    // per destination: exclusive prefix over the 8 warps and its total; then the
+    // tile's destination offsets by a block scan over thread-contiguous ranges of R
+    const uint32_t per = (R + kPartBlock - 1) / kPartBlock, r0 = threadIdx.x * per;
+    uint32_t run = 0;
+    for (uint32_t r = r0; r < r0 + per && r < R; ++r) {
         uint4 v = wc4[r];
         uint16_t c[8];
         memcpy(c, &v, 16);
-        uint16_t run = 0;
+        uint16_t acc = 0;
 #pragma unroll
         for (int w = 0; w < kPartWarps; ++w) {
             const uint16_t x = c[w];
-            c[w] = run;
-            run = (uint16_t)(run + x);
+            c[w] = acc;
+            acc = (uint16_t)(acc + x);
         }
         memcpy(&v, c, 16);
         wc4[r] = v;
+        toff[r] = acc;  // the destination's total until the scan below
+        run += acc;
+    }
+    part[threadIdx.x] = run;
+    __syncthreads();
+    if (threadIdx.x < 32) {  // exclusive scan of the 256 partials by one warp
+        constexpr int kPer = kPartBlock / 32;
+        uint32_t x[kPer], sum = 0;
+#pragma unroll
+        for (int k = 0; k < kPer; ++k) {
+            x[k] = part[threadIdx.x * kPer + k];
+            sum += x[k];
+        }
+        const uint32_t incl = warp_incl_scan(sum, lane);
+        uint32_t ex = incl - sum;
+#pragma unroll
+        for (int k = 0; k < kPer; ++k) {
+            part[threadIdx.x * kPer + k] = ex;
+            ex += x[k];
+        }
+        if (threadIdx.x == 31) s_valid = incl;
     }
     __syncthreads();
-#pragma unroll
-    for (int j = 0; j < 8; ++j) {
-        if (dig[j] == 0xffffu) continue;
-        const unsigned long long i = base + (unsigned long long)j * 32 + lane;
-        const uint32_t pos = off[((unsigned long long)rep * R + dig[j]) * ntiles + tile] +
-                             wc[dig[j] * kPartWarps + warp] + rank[j];
-        rec16 rr;
-        rr.key = keys[i];
-        rr.P = plen[i];
-        rr.S = slen[i];
-        rec[pos] = rr;
+    run = part[threadIdx.x];
+    for (uint32_t r = r0; r < r0 + per && r < R; ++r) {
+        const uint32_t t = toff[r];
+        toff[r] = run;
+        run += t;
+    }
+    __syncthreads();
+    // staging: every valid item at its place in (destination, arrival) order
+    for (uint32_t it = threadIdx.x; it < cnt; it += kPartBlock) {
+        const uint32_t pk = spk[it];
+        const uint32_t d = pk >> 16;
+        if (d == kNoDest) continue;
+        const uint32_t pos = toff[d] + wc[d * kPartWarps + it / kPerWarp] + (pk & 0xffffu);
+        sitem[pos] = (uint16_t)it;
+    }
+    __syncthreads();
+    // output: consecutive threads write consecutive positions of each destination's run
+    const uint32_t valid = s_valid;
+    const uint32_t *O = off + (unsigned long long)rep * R * ntiles;
+    for (uint32_t j = threadIdx.x; j < valid; j += kPartBlock) {
+        const uint32_t it = sitem[j];
+        const uint32_t d = spk[it] >> 16;
+        if (d >= R || j < toff[d]) continue;  // never: every staged item is valid (guards the writes)
+        const unsigned long long o = (unsigned long long)O[(unsigned long long)d * ntiles + tile] + (j - toff[d]);
+        if (o < m) out[o] = (uint32_t)(base + it);
+    }
+}
+
+// One (key, prefix, suffix) record per request, read by the replay through the indices.
+__global__ void k_part_records(const unsigned long long *__restrict__ keys, const uint32_t *__restrict__ plen,
+                               const uint32_t *__restrict__ slen, unsigned long long n, rec16 *__restrict__ recs)
+{
+    for (unsigned long long i = (unsigned long long)blockIdx.x * blockDim.x + threadIdx.x; i < n;
+         i += (unsigned long long)gridDim.x * blockDim.x) {
+        rec16 r;
+        r.key = keys[i];
+        r.P = plen[i];
+        r.S = slen[i];
+        recs[i] = r;
     }
 }
 
@@ -378,15 +457,6 @@ __device__ __forceinline__ void sl_stamps_in_order(const stamp_lru &X, uint32_t 
     __syncwarp();
 }
 
-__device__ __forceinline__ uint32_t warp_incl_scan(uint32_t v, uint32_t lane)
-{
-#pragma unroll
-    for (int o = 1; o < 32; o <<= 1) {
-        const uint32_t y = __shfl_up_sync(0xffffffffu, v, o);
-        if (lane >= (uint32_t)o) v += y;
-    }
-    return v;
-}
 
 // Position of the k-th (from 0) set bit of w, which has more than k set bits.
 __device__ __forceinline__ uint32_t nth_set_bit(uint32_t w, uint32_t k)
@@ -465,7 +535,8 @@ template <int NC, int NG, bool SMALL>
 __global__ void __launch_bounds__(128)
 k_lru_stamp(const replay_caps caps, uint32_t cmax, uint32_t nw, uint32_t R, uint32_t ns, uint32_t CL, uint32_t nbb,
             const uint32_t *__restrict__ start, const uint32_t *__restrict__ coff, const uint32_t *__restrict__ total,
-            const rec16 *__restrict__ rec, const replay_state st, unsigned long long *__restrict__ ctr,
+            const uint32_t *__restrict__ idx, const rec16 *__restrict__ recs, uint32_t nrec,
+            const replay_state st, unsigned long long *__restrict__ ctr,
             uint32_t *status)
 {
     extern __shared__ uint4 smb[];
@@ -515,7 +586,7 @@ k_lru_stamp(const replay_caps caps, uint32_t cmax, uint32_t nw, uint32_t R, uint
             const uint32_t v = v0 + lane;
             const bool valid = v < vtot;
             unsigned long long key = 0;
-            if (valid) key = v < back ? rec[p0 - 1 - v].key : kin[v - back];
+            if (valid) key = v < back ? recs[min(idx[p0 - 1 - v], nrec - 1u)].key : kin[v - back];
             const uint32_t vm = __ballot_sync(0xffffffffu, valid);
             const uint32_t peers = __match_any_sync(0xffffffffu, key) & vm;
             const bool fresh = valid && (peers & lt) == 0 && sl_lookup(X, key, fill, cmax) == kNone;
@@ -540,12 +611,12 @@ k_lru_stamp(const replay_caps caps, uint32_t cmax, uint32_t nw, uint32_t R, uint
     for (int c = 0; c < NC; ++c) my_hit[c] = my_tok[c] = 0;
 
     rec16 ahead = {0ull, 0u, 0u};  // the next step's records, loaded one step early
-    if (p0 + lane < p1) ahead = rec[p0 + lane];
+    if (p0 + lane < p1) ahead = recs[min(idx[p0 + lane], nrec - 1u)];  // (the bound guards the gather)
     for (uint32_t t0 = p0; t0 < p1; t0 += 32) {
         const uint32_t cnt = (p1 - t0) < 32u ? (p1 - t0) : 32u;
         const bool valid = lane < cnt;
         const rec16 mine = ahead;
-        if (t0 + 32u + lane < p1) ahead = rec[t0 + 32u + lane];
+        if (t0 + 32u + lane < p1) ahead = recs[min(idx[t0 + 32u + lane], nrec - 1u)];
         if (valid) {
             my_req += 1;
             my_prompt += (unsigned long long)mine.P + mine.S;
@@ -749,7 +820,8 @@ inline uint32_t stamp_words(uint32_t cmax)
 
 template <int NC, int NG, bool SMALL>
 int launch_stamp(cr_ctx *ctx, cr_replay *rp, const replay_caps &caps, uint32_t CL, const uint32_t *start,
-                 const uint32_t *coff, const uint32_t *total, uint64_t m, const rec16 *rec, uint64_t *d_ctr)
+                 const uint32_t *coff, const uint32_t *total, uint64_t m, const uint32_t *idx,
+                 const rec16 *recs, uint64_t *d_ctr)
 {
     const uint32_t cmax = rp->cmax, nw = stamp_words(cmax);
     uint32_t nbb = 4;
@@ -779,7 +851,9 @@ int launch_stamp(cr_ctx *ctx, cr_replay *rp, const replay_caps &caps, uint32_t C
     st.fill_out = rp->d_fill[rp->cur ^ 1];
     const int pr = cr_prof_begin(ctx, ctx->stream, CR_PROF_REPLAY);
     CR_LAUNCH(ctx, (k_lru_stamp<NC, NG, SMALL>), (unsigned int)((items + wpb - 1) / wpb), wpb * 32, smem, caps, cmax,
-              nw, rp->R, ns, CL, nbb, start, coff, total, rec, st, (unsigned long long *)d_ctr, ctx->d_status);
+              nw, rp->R, ns, CL, nbb, start, coff, total, idx, recs, (uint32_t)(m / rp->n_rep), st,
+              (unsigned long long *)d_ctr,
+              ctx->d_status);
     cr_prof_end(ctx, ctx->stream, pr);
     rp->cur ^= 1;
     return CR_OK;
@@ -787,24 +861,26 @@ int launch_stamp(cr_ctx *ctx, cr_replay *rp, const replay_caps &caps, uint32_t C
 
 template <int NC>
 int launch_stamp_nc(cr_ctx *ctx, cr_replay *rp, const replay_caps &caps, uint32_t CL, const uint32_t *start,
-                    const uint32_t *coff, const uint32_t *total, uint64_t m, const rec16 *rec, uint64_t *d_ctr)
+                    const uint32_t *coff, const uint32_t *total, uint64_t m, const uint32_t *idx,
+                 const rec16 *recs, uint64_t *d_ctr)
 {
     uint32_t cmin = 0xffffffffu;
     for (uint32_t c = 0; c < caps.n_caps; ++c) cmin = caps.cap[c] < cmin ? caps.cap[c] : cmin;
     const bool small = cmin < 32;  // a repeat within a step can miss only below capacity 32
     if (stamp_words(rp->cmax) <= 32)
-        return small ? launch_stamp<NC, 1, true>(ctx, rp, caps, CL, start, coff, total, m, rec, d_ctr)
-                     : launch_stamp<NC, 1, false>(ctx, rp, caps, CL, start, coff, total, m, rec, d_ctr);
-    return small ? launch_stamp<NC, 2, true>(ctx, rp, caps, CL, start, coff, total, m, rec, d_ctr)
-                 : launch_stamp<NC, 2, false>(ctx, rp, caps, CL, start, coff, total, m, rec, d_ctr);
+        return small ? launch_stamp<NC, 1, true>(ctx, rp, caps, CL, start, coff, total, m, idx, recs, d_ctr)
+                     : launch_stamp<NC, 1, false>(ctx, rp, caps, CL, start, coff, total, m, idx, recs, d_ctr);
+    return small ? launch_stamp<NC, 2, true>(ctx, rp, caps, CL, start, coff, total, m, idx, recs, d_ctr)
+                 : launch_stamp<NC, 2, false>(ctx, rp, caps, CL, start, coff, total, m, idx, recs, d_ctr);
 }
 
 int launch_batch(cr_ctx *ctx, cr_replay *rp, const replay_caps &caps, uint32_t CL, const uint32_t *start,
-                 const uint32_t *coff, const uint32_t *total, uint64_t m, const rec16 *rec, uint64_t *d_ctr)
+                 const uint32_t *coff, const uint32_t *total, uint64_t m, const uint32_t *idx,
+                 const rec16 *recs, uint64_t *d_ctr)
 {
-    if (caps.n_caps == 1) return launch_stamp_nc<1>(ctx, rp, caps, CL, start, coff, total, m, rec, d_ctr);
-    if (caps.n_caps <= 3) return launch_stamp_nc<3>(ctx, rp, caps, CL, start, coff, total, m, rec, d_ctr);
-    return launch_stamp_nc<CR_MAX_CAPS>(ctx, rp, caps, CL, start, coff, total, m, rec, d_ctr);
+    if (caps.n_caps == 1) return launch_stamp_nc<1>(ctx, rp, caps, CL, start, coff, total, m, idx, recs, d_ctr);
+    if (caps.n_caps <= 3) return launch_stamp_nc<3>(ctx, rp, caps, CL, start, coff, total, m, idx, recs, d_ctr);
+    return launch_stamp_nc<CR_MAX_CAPS>(ctx, rp, caps, CL, start, coff, total, m, idx, recs, d_ctr);
 }
 
 // ---- token-weighted variant ---------------------------------------------------
@@ -833,7 +909,8 @@ __device__ __forceinline__ uint32_t sat_add(uint32_t a, uint32_t b)
 
 __global__ void __launch_bounds__(kTokWarps * 32) k_lru_tokens(const __grid_constant__ replay_caps caps, uint32_t ns,
                                                                uint32_t R, const uint32_t *__restrict__ start,
-                                                               const rec16 *__restrict__ rec,
+                                                               const uint32_t *__restrict__ idx,
+                                                               const rec16 *__restrict__ recs, uint32_t nrec,
                                                                unsigned long long *__restrict__ keys_state,
                                                                uint32_t *__restrict__ cum_state,
                                                                uint32_t *__restrict__ fill_state,
@@ -867,10 +944,10 @@ __global__ void __launch_bounds__(kTokWarps * 32) k_lru_tokens(const __grid_cons
     unsigned long long c_hit = 0, c_hit_tok = 0, c_prompt = 0;  // lane = capacity (prompt: every lane)
     const uint32_t i0 = start[s], i1 = start[s + 1];
     rec16 nx = {0ull, 0u, 0u};
-    if (i0 + lane < i1) nx = rec[i0 + lane];
+    if (i0 + lane < i1) nx = recs[min(idx[i0 + lane], nrec - 1u)];
     for (uint32_t b0 = i0; b0 < i1; b0 += 32) {
         const rec16 cur = nx;
-        if (b0 + 32 + lane < i1) nx = rec[b0 + 32 + lane];  // next 32 records in flight
+        if (b0 + 32 + lane < i1) nx = recs[min(idx[b0 + 32 + lane], nrec - 1u)];  // next 32 in flight
         const uint32_t nb = i1 - b0 < 32 ? i1 - b0 : 32;
         if (lane < nb) c_prompt += (unsigned long long)cur.P + cur.S;
         for (uint32_t q = 0; q < nb; ++q) {
@@ -1110,29 +1187,33 @@ extern "C" int cr_shadow_replay(cr_ctx *ctx, cr_replay *rp, const uint64_t *d_ke
     const uint32_t ntiles = (uint32_t)((n + kPartTile - 1) / kPartTile);
     const uint64_t ncnt = (uint64_t)ns * ntiles;
     if (ncnt >= 0xffffffffull) return cr_fail(ctx, CR_EINVAL, "cr_shadow_replay: too many (stream, tile) pairs");
-    void *pk, *ps, *prec, *pch;
+    void *pk, *ps, *pidx, *pch, *precs;
     CR_TRY(cr_scratch(ctx, SCR_REPLAY_IDX, (ncnt + 2) * sizeof(uint32_t), &pk));
     CR_TRY(cr_scratch(ctx, SCR_REPLAY_START, ((size_t)ns + 1) * sizeof(uint32_t), &ps));
-    CR_TRY(cr_scratch(ctx, SCR_REPLAY_REC, m * sizeof(rec16), &prec));
+    CR_TRY(cr_scratch(ctx, SCR_REPLAY_REC, m * sizeof(uint32_t), &pidx));
+    CR_TRY(cr_scratch(ctx, SCR_REPLAY_RECS, n * sizeof(rec16), &precs));
     CR_TRY(cr_scratch(ctx, SCR_REPLAY_CHUNK, ((size_t)ns + 2) * sizeof(uint32_t), &pch));
     uint32_t *cnt = (uint32_t *)pk, *nrec = cnt + ncnt, *start = (uint32_t *)ps;
-    rec16 *rec = (rec16 *)prec;
+    uint32_t *idx = (uint32_t *)pidx;
+    rec16 *recs = (rec16 *)precs;
     uint32_t *coff = (uint32_t *)pch, *total = coff + ns;
     const unsigned int gcap = (unsigned int)ctx->num_sms * 8u;
     const dim3 pgrid(ntiles, rp->n_rep);
-    const size_t csmem = (size_t)R * sizeof(uint32_t), ssmem = (size_t)R * kPartWarps * sizeof(uint16_t);
+    const size_t csmem = (size_t)R * sizeof(uint32_t), ssmem = part_scatter_smem(R);
     if (csmem > 48 * 1024)
         CR_CUDA(ctx, cudaFuncSetAttribute(k_part_count, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)csmem));
     if (ssmem > 48 * 1024)
         CR_CUDA(ctx, cudaFuncSetAttribute(k_part_scatter, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)ssmem));
     const int pp = cr_prof_begin(ctx, ctx->stream, CR_PROF_PARTITION);
+    CR_LAUNCH(ctx, k_part_records, cr_blocks(n, 256, gcap), 256, 0, (const unsigned long long *)d_key, d_plen, d_slen,
+              (unsigned long long)n, recs);
     CR_LAUNCH(ctx, k_part_count, pgrid, kPartBlock, csmem, d_dest, (unsigned long long)n, R, ntiles, cnt,
               ctx->d_status);
     CR_TRY(cr_scan_u32(ctx, cnt, cnt, ncnt, nrec));
     CR_LAUNCH(ctx, k_part_starts, cr_blocks((uint64_t)ns + 1, 256, gcap), 256, 0, (const uint32_t *)cnt, ns, ntiles,
               (const uint32_t *)nrec, start);
     CR_LAUNCH(ctx, k_part_scatter, pgrid, kPartBlock, ssmem, d_dest, (unsigned long long)n, R, ntiles,
-              (const uint32_t *)cnt, (const unsigned long long *)d_key, d_plen, d_slen, rec);
+              (const uint32_t *)cnt, idx, (unsigned long long)m);
     cr_prof_end(ctx, ctx->stream, pp);
     replay_caps caps;
     caps.n_caps = rp->n_caps;
@@ -1144,7 +1225,8 @@ extern "C" int cr_shadow_replay(cr_ctx *ctx, cr_replay *rp, const uint64_t *d_ke
             CR_CUDA(ctx, cudaFuncSetAttribute(k_lru_tokens, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)tsmem));
         const int pt = cr_prof_begin(ctx, ctx->stream, CR_PROF_REPLAY);
         CR_LAUNCH(ctx, k_lru_tokens, (ns + kTokWarps - 1) / kTokWarps, kTokWarps * 32, tsmem, caps, ns, R,
-                  (const uint32_t *)start, (const rec16 *)rec, (unsigned long long *)rp->d_keys[0], rp->d_size,
+                  (const uint32_t *)start, (const uint32_t *)idx, (const rec16 *)recs, (uint32_t)n,
+                  (unsigned long long *)rp->d_keys[0], rp->d_size,
                   rp->d_fill[0], (unsigned long long *)d_ctr, ctx->d_status);
         cr_prof_end(ctx, ctx->stream, pt);
         return CR_OK;
@@ -1153,7 +1235,7 @@ extern "C" int cr_shadow_replay(cr_ctx *ctx, cr_replay *rp, const uint64_t *d_ke
     const uint32_t CL = rp->cmax * 16u > 256u ? rp->cmax * 16u : 256u;
     CR_LAUNCH(ctx, k_chunk_counts, cr_blocks(ns, 256, gcap), 256, 0, (const uint32_t *)start, ns, CL, coff);
     CR_TRY(cr_scan_u32(ctx, coff, coff, ns, total));
-    return launch_batch(ctx, rp, caps, CL, start, coff, total, m, rec, d_ctr);
+    return launch_batch(ctx, rp, caps, CL, start, coff, total, m, idx, recs, d_ctr);
 }
 
 extern "C" int cr_replay_export_state(cr_ctx *ctx, const cr_replay *rp, uint32_t rep, uint32_t r,
@@ -1171,4 +1253,32 @@ extern "C" int cr_replay_export_state(cr_ctx *ctx, const cr_replay *rp, uint32_t
                                      cudaMemcpyDeviceToHost, ctx->stream));
     *fill_out = fill;
     return cr_sync(ctx);
+}
+
+extern "C" int cr_replay_import_state(cr_ctx *ctx, cr_replay *rp, uint32_t rep, uint32_t r, const uint64_t *keys,
+                                      uint32_t fill)
+{
+    if (!ctx || !rp || (fill && !keys)) return CR_EINVAL;
+    if (rp->tokens) return cr_fail(ctx, CR_EINVAL, "import_state: token-weighted replays keep prefix sizes too");
+    if (rep >= rp->n_rep || r >= rp->R) return cr_fail(ctx, CR_EINVAL, "import_state: bad stream");
+    if (fill > rp->cmax) return cr_fail(ctx, CR_EINVAL, "import_state: %u keys exceed capacity %u", fill, rp->cmax);
+    // the keys of one LRU are distinct
+    uint64_t *tmp = (uint64_t *)malloc((size_t)(fill ? fill : 1) * sizeof(uint64_t));
+    if (!tmp) return cr_fail(ctx, CR_ENOMEM, "import_state: host allocation failed");
+    memcpy(tmp, keys, (size_t)fill * sizeof(uint64_t));
+    qsort(tmp, fill, sizeof(uint64_t), [](const void *a, const void *b) {
+        const uint64_t x = *(const uint64_t *)a, y = *(const uint64_t *)b;
+        return x < y ? -1 : (x > y ? 1 : 0);
+    });
+    int dup = 0;
+    for (uint32_t i = 1; i < fill; ++i) dup |= tmp[i] == tmp[i - 1];
+    free(tmp);
+    if (dup) return cr_fail(ctx, CR_EINVAL, "import_state: a key is listed twice");
+    const uint64_t s = (uint64_t)rep * rp->R + r;
+    if (fill)
+        CR_CUDA(ctx, cudaMemcpyAsync(rp->d_keys[rp->cur] + s * rp->cmax, keys, (size_t)fill * sizeof(uint64_t),
+                                     cudaMemcpyHostToDevice, ctx->stream));
+    CR_CUDA(ctx, cudaMemcpyAsync(rp->d_fill[rp->cur] + s, &fill, sizeof(uint32_t), cudaMemcpyHostToDevice,
+                                 ctx->stream));
+    return cr_sync(ctx);  // blocking: the host arrays may be reused when the call returns
 }

@@ -890,3 +890,72 @@ def test_profile_events_time_each_launch(P):
         plan.close()
     finally:
         c.close()
+
+
+def test_plan_import_routes_like_the_built_plan(P, ctx):
+    # a plan exported from the device and installed again (as a host planner's table would
+    # be) routes exactly as the plan it came from; bad tables are refused
+    rng = np.random.default_rng(21)
+    R, W = 64, 8
+    keys = _rates_keys(rng, 3000, 60000)
+    n = keys.size
+    built = P.build_plan(ctx, d_u64(keys), P.plan_params(R, W, 5 * n, 4 * R, "LPT"))
+    ex = built.export()
+    imp = P.Plan(ctx).load(R, W, ex["adm_key"], ex["adm_cnt"], ex["adm_k"], ex["members"], ex["jobs"], ex["load"])
+    got = imp.export()
+    for f in ("adm_key", "adm_cnt", "adm_k", "koff", "members", "jobs", "load"):
+        assert (got[f] == ex[f]).all(), f
+    assert got["n_adm"] == ex["n_adm"] and got["sum_k"] == ex["sum_k"]
+    load = torch.zeros((2, R), dtype=torch.int64, device=DEV)
+    dk = d_u64(keys)
+    d = P.route_batch(ctx, [built, imp], ["CR", "CR"], [3, 3], R, dk, 0, 1024, load)
+    ctx.sync()
+    h = h_u16(d)
+    assert (h[0] == h[1]).all()
+    # the oracle agrees with the imported plan's routes
+    opl = O.build_plan(keys, R, W, 5 * n, 4 * R)
+    od, _ = O.route([opl], ["CR"], [3], R, keys, 0, 1024)
+    assert (h[1] == od[0]).all()
+    for bad in (dict(adm_k=np.zeros_like(ex["adm_k"])),                       # k = 0
+                dict(members=np.full_like(ex["members"], R)),                 # member >= R
+                dict(adm_key=np.zeros_like(ex["adm_key"]))):                  # repeated key
+        args = dict(adm_key=ex["adm_key"], adm_cnt=ex["adm_cnt"], adm_k=ex["adm_k"], members=ex["members"])
+        args.update(bad)
+        with pytest.raises(P.CacheRouteError):
+            P.Plan(ctx).load(R, W, **args)
+
+
+def test_replay_state_import_resumes(P, ctx):
+    # replay two calls in one simulator set; export every state after the first, import
+    # it into a fresh set, and the second call's counters match
+    rng = np.random.default_rng(5)
+    caps, n_rep, R = [8, 64, 256], 2, 6
+    keys = _rates_keys(rng, 2000, 30000)
+    n = keys.size
+    plen = rng.integers(16, 4000, size=n).astype(np.uint32)
+    slen = np.full(n, 64, np.uint32)
+    dest = tg.random_dest(n_rep, n, R, 9)
+    cut = n // 2
+    dk, dp, ds, dd = d_u64(keys), d_u32(plen), d_u32(slen), d_u16(dest)
+    a = P.Replay(ctx, n_rep, R, caps)
+    ctr_a = torch.zeros((n_rep, len(caps), R, 5), dtype=torch.int64, device=DEV)
+    P.shadow_replay(ctx, a, dk[:cut].contiguous(), dp[:cut].contiguous(), ds[:cut].contiguous(),
+                    dd[:, :cut].contiguous(), ctr_a)
+    ctx.sync()
+    b = P.Replay(ctx, n_rep, R, caps)
+    for rep in range(n_rep):
+        for r in range(R):
+            b.set_state(rep, r, a.state(rep, r))
+    ctr_a.zero_()
+    ctr_b = torch.zeros_like(ctr_a)
+    for rp, ctr in ((a, ctr_a), (b, ctr_b)):
+        P.shadow_replay(ctx, rp, dk[cut:].contiguous(), dp[cut:].contiguous(), ds[cut:].contiguous(),
+                        dd[:, cut:].contiguous(), ctr)
+    ctx.sync()
+    assert (h_u64(ctr_a) == h_u64(ctr_b)).all()
+    with pytest.raises(P.CacheRouteError):
+        b.set_state(0, 0, np.array([1, 2, 1], np.uint64))     # repeated key
+    with pytest.raises(P.CacheRouteError):
+        b.set_state(0, R, np.array([1], np.uint64))            # no such destination
+    a.close()
+    b.close()
