@@ -70,12 +70,14 @@ def parse_args(argv=None):
                     help="hash each interval's arena on its own and time plans + route + replay over resident keys "
                          "(automatic when the arenas do not fit in HBM)")
     ap.add_argument("--per-interval", action="store_true",
-                    help="keys mode: drive one interval at a time (Pipeline) instead of keeping several intervals' "
-                         "plans and routes in flight (TracePipeline)")
+                    help="drive one interval at a time (Pipeline) instead of keeping several intervals' plans and "
+                         "routes in flight (TracePipeline)")
     ap.add_argument("--depth", type=int, default=8, help="keys mode: intervals in flight")
     ap.add_argument("--plan-streams", type=int, default=4, help="keys mode: streams building plans")
     ap.add_argument("--route-streams", type=int, default=4, help="keys mode: streams routing")
-    ap.add_argument("--replay-priority", choices=["high", "low"], default="high",
+    ap.add_argument("--replay-group", type=int, default=2,
+                    help="keys mode: consecutive intervals replayed by one call")
+    ap.add_argument("--replay-priority", choices=["high", "low"], default="low",
                     help="keys mode: priority of the replay stream (plans get the other one)")
     ap.add_argument("--intervals", type=int, default=0,
                     help="profiling aid: run only the first N intervals (the JSON line says so)")
@@ -230,32 +232,61 @@ def lru_traffic(alg_bytes_per_launch: float, pairs_per_launch: float):
 
 
 # ----------------------------------------------------------------- oracle ---
-def oracle_sample(trace, n_intervals: int = 1, B: int = 1024):
-    """Time the CPU oracle (hash, plans, route, replay) on the first intervals of the trace."""
+def oracle_interval_step(trace, sample, threads: int, B: int) -> float:
+    """One timed pass of the CPU oracle, as it stands, over interval 0 of a resident-arena
+    configuration: hash every request (the arena split in `threads` request ranges), the
+    plans (from interval 0's own keys), then route and replay every replica; independent
+    ranges, plan variants and replicas run on `threads` host threads (each oracle call is
+    plain single-threaded C and releases the interpreter lock).  Returns seconds."""
+    import concurrent.futures as cf
     import oracle as O
     import oracle.pipeline as OP
-    import tracegen as tg
     cfg = trace.cfg
     reps = cfg.replicas
-    pols = [OP.ROUTE_AS.get(p, p) for p, _ in reps]
-    seeds = [s for _, s in reps]
-    rp = O.Replay(len(reps), cfg.R, cfg.caps, tokens=cfg.lru_tokens)
+    tok, off, iv = sample["tok"], sample["off"], sample["iv"]
     rings = OP.rings_for(cfg)
-    prev = None
-    busy = 0.0
-    reqs = 0
-    for t in range(n_intervals):
-        iv = trace.interval(t)
-        tok, off = tg.arena_host(trace, iv, 4)
-        t0 = time.perf_counter()
-        keys = O.hash_prefixes(tok, off, iv.plen)
-        per_rep, _ = OP.plans_for_interval(trace, keys if prev is None else prev, t)
-        dest, _ = O.route(per_rep, pols, seeds, cfg.R, keys, iv.g0, B, rings=rings)
-        rp.step(keys, iv.plen, iv.slen, dest)
-        busy += time.perf_counter() - t0
-        reqs += iv.n
-        prev = keys
-    return reqs, busy
+    n = iv.n
+    t0 = time.perf_counter()
+    cuts = [n * i // threads for i in range(threads + 1)]
+
+    def hash_range(ab):
+        a, b = ab
+        return O.hash_prefixes(tok, off[a:b], iv.plen[a:b]) if b > a else np.zeros(0, np.uint64)
+
+    with cf.ThreadPoolExecutor(threads) as ex:
+        keys = np.concatenate(list(ex.map(hash_range, zip(cuts[:-1], cuts[1:]))))
+    num, den = trace.qcap(n)
+    variants = sorted({(OP.VARIANT_OF[p], sd if OP.VARIANT_OF[p] == "RANDOM" else 0)
+                       for p, sd in reps if p in OP.VARIANT_OF})
+
+    def build(vs):
+        v, sd = vs
+        return vs, O.build_plan(keys, cfg.R, cfg.W, num, den, variant=v, seed=sd, epoch=0)
+
+    with cf.ThreadPoolExecutor(threads) as ex:
+        built = dict(ex.map(build, variants))
+
+    def one(i):
+        p, sd = reps[i]
+        v = OP.VARIANT_OF.get(p)
+        plan = built[(v, sd if v == "RANDOM" else 0)] if v is not None else None
+        d, _ = O.route([plan], [OP.ROUTE_AS.get(p, p)], [sd], cfg.R, keys, iv.g0, B, rings=[rings[i]])
+        rp = O.Replay(1, cfg.R, cfg.caps, tokens=cfg.lru_tokens)
+        rp.step(keys, iv.plen, iv.slen, d)
+        return int(rp.ctr[..., 0].sum())
+
+    with cf.ThreadPoolExecutor(threads) as ex:
+        done = list(ex.map(one, range(len(reps))))
+    assert all(x == n * len(cfg.caps) for x in done)
+    return time.perf_counter() - t0
+
+
+def oracle_interval_sample(trace):
+    """Input preparation (untimed): interval 0's token arena on the host."""
+    import tracegen as tg
+    iv = trace.interval(0)
+    tok, off = tg.arena_host(trace, iv, 4)
+    return {"tok": tok, "off": off, "iv": iv, "n": iv.n}
 
 
 def token_bytes(trace) -> float:
@@ -346,36 +377,21 @@ def run_reference(args):
     trace = tg.Trace(cfg)
     if keys_mode_for(args, trace):
         return run_reference_keys(args, cfg, trace)
-    import oracle as O
-    import oracle.pipeline as OP
-    iv = trace.interval(0)
-    tok, off = tg.arena_host(trace, iv, 4)
-    reps = cfg.replicas
-    pols = [OP.ROUTE_AS.get(p, p) for p, _ in reps]
-    seeds = [s for _, s in reps]
-    rings = OP.rings_for(cfg)
-
-    def step():
-        rp = O.Replay(len(reps), cfg.R, cfg.caps, tokens=cfg.lru_tokens)
-        keys = O.hash_prefixes(tok, off, iv.plen)
-        per_rep, _ = OP.plans_for_interval(trace, keys, 0)
-        dest, _ = O.route(per_rep, pols, seeds, cfg.R, keys, iv.g0, args.batch, rings=rings)
-        rp.step(keys, iv.plen, iv.slen, dest)
-
+    threads = os.cpu_count() or 1
+    sample = oracle_interval_sample(trace)
     for _ in range(args.warmup):
-        step()
-    t0 = time.perf_counter()
-    for _ in range(args.steps):
-        step()
-    dt = (time.perf_counter() - t0) / max(args.steps, 1)
-    value = iv.n / dt
-    sample = (f"interval 0 of {cfg.n_intervals} ({iv.n} requests, all {len(reps)} replicas) per step, "
-              f"single-threaded C oracle")
+        oracle_interval_step(trace, sample, threads, args.batch)
+    each = [oracle_interval_step(trace, sample, threads, args.batch) for _ in range(args.steps)]
+    dt = float(np.mean(each)) if each else 0.0
+    value = sample["n"] / dt if dt > 0 else 0.0
+    text = (f"interval 0 of {cfg.n_intervals} ({sample['n']} requests, all {len(cfg.replicas)} replicas) per step, "
+            f"hash+plan+route+replay, C oracle on {threads} host threads over request ranges, plan variants and "
+            f"replicas")
     line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": dt * 1e3, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "u64", "data": "synthetic",
             "config": workload_config(cfg, args.batch, args.fresh_plans),
-            "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "kind": "oracle", "sample": sample},
+            "cpu_baseline": {"value": value, "unit": UNIT, "cores": threads, "kind": "oracle", "sample": text},
             "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     print(json.dumps(line), flush=True)
 
@@ -506,6 +522,11 @@ def main():
     torch.cuda.synchronize()
     n_step = sum(x[6] for x in inputs)
     max_n = max(x[6] for x in inputs)
+    # several intervals in flight pay off when intervals are large; many small intervals are
+    # bound by launches from the host, which the one-interval driver issues fewer of
+    big = n_step / max(cfg.n_intervals, 1) >= 65536
+    if big and not (args.per_interval or args.graph or part is not None or cfg.drift or args.no_overlap):
+        return run_resident_trace(args, cfg, trace, inputs, hash_bytes, dev, stream, world, rank, barrier)
 
     ctx = P.Context(local, stream)
     pipe = Pipeline(ctx, cfg.R, cfg.W, cfg.caps, cfg.replicas, trace.qcap, batch_B=args.batch, max_n=max_n,
@@ -648,11 +669,16 @@ def main():
         line["e2e"] = e2e(args, ctx, pipe, inputs, dev, stream, n_step, world)
     # ---- CPU baseline (rank 0, N = 1) ---------------------------------------
     if not args.no_cpu_baseline and world == 1:
-        reqs, busy = oracle_sample(trace, 1, args.batch)
-        line["cpu_baseline"] = {"value": reqs / busy, "unit": UNIT, "cores": 1, "kind": "oracle",
-                                "sample": f"interval 0 of {cfg.n_intervals} ({reqs} requests, all "
-                                          f"{len(cfg.replicas)} replicas), hash+plan+route+replay, "
-                                          f"single-threaded C oracle"}
+        sample = oracle_interval_sample(trace)
+        nproc = os.cpu_count() or 1
+        t1 = oracle_interval_step(trace, sample, 1, args.batch)
+        tn = oracle_interval_step(trace, sample, nproc, args.batch)
+        line["cpu_baseline"] = {"value": sample["n"] / tn, "unit": UNIT, "cores": nproc, "kind": "oracle",
+                                "sample": f"interval 0 of {cfg.n_intervals} ({sample['n']} requests, all "
+                                          f"{len(cfg.replicas)} replicas), hash+plan+route+replay, C oracle on "
+                                          f"{nproc} host threads over request ranges, plan variants and replicas",
+                                "single_thread": {"value": sample["n"] / t1, "unit": UNIT, "cores": 1},
+                                "nproc": nproc}
     if rank == 0:
         print(json.dumps(line), flush=True)
     close_in_order(pipe, ctx, part)
@@ -763,7 +789,8 @@ def run_keys_mode(args, cfg, trace, dev, stream, world, rank, barrier, resolve_s
         pipe = TracePipeline(ctx, cfg.R, cfg.W, cfg.caps, cfg.replicas, trace.qcap, max_n=max(ns),
                              batch_B=args.batch, depth=args.depth, plan_streams=args.plan_streams,
                              route_streams=args.route_streams, vnodes=cfg.vnodes, fresh=args.fresh_plans,
-                             lru_tokens=cfg.lru_tokens, replay_first=args.replay_priority == "high")
+                             lru_tokens=cfg.lru_tokens, replay_first=args.replay_priority == "high",
+                             replay_group=args.replay_group)
     else:
         pipe = Pipeline(ctx, cfg.R, cfg.W, cfg.caps, cfg.replicas, trace.qcap, batch_B=args.batch, max_n=max(ns),
                         overlap=not args.no_overlap, vnodes=cfg.vnodes, fresh=args.fresh_plans,
@@ -877,7 +904,9 @@ def run_keys_mode(args, cfg, trace, dev, stream, world, rank, barrier, resolve_s
     rr_gbs = rr_bytes * rr_rps / 1e9
     # the dominant kernel of the step: the LRU simulation (a9), one launch per interval; its
     # algorithmic bytes per launch are SURVEY 8(d)'s 20 per (request, replica, capacity)
-    a9_bytes = 20.0 * reps * ncaps * n_step / cfg.n_intervals
+    steps_profiled = 1 if graph is not None else args.steps
+    req_per_launch = n_step * steps_profiled / max(kern["replay"]["launches"], 1)
+    a9_bytes = 20.0 * reps * ncaps * req_per_launch
     lru_ms = kern["replay"]["avg_ms"]
     lru_gbs = a9_bytes / (lru_ms / 1e3) / 1e9 if lru_ms else None
     line = {
@@ -889,13 +918,15 @@ def run_keys_mode(args, cfg, trace, dev, stream, world, rank, barrier, resolve_s
                             "not fit in HBM: each interval's arena was generated and hashed one at a time, each "
                             "hash launch timed alone)",
                        schedule=(f"{args.depth} intervals in flight: plans on {args.plan_streams} streams, routes "
-                                 f"on {args.route_streams} streams, the replay in interval order on one stream"
+                                 f"on {args.route_streams} streams, the replay in interval order on one stream, "
+                                 f"{args.replay_group} intervals per replay call"
                                  if trace_mode else "one interval at a time (plans of the next interval overlap)"),
                        l2="inputs larger than L2 (keys, prefix and suffix lengths of all intervals resident)"),
         "roofline": {"kernel": "k_lru_stamp (a9 LRU replay)", "bound": "hbm", "achieved": lru_gbs,
                      "peak": hbm_peak, "peak_source": "measured" if "hbm_gbs" in peaks else "fallback",
                      "unit": "GB/s", "frac": lru_gbs / hbm_peak if lru_gbs else None,
-                     "traffic": lru_traffic(a9_bytes, reps * n_step / cfg.n_intervals),
+                     "traffic": lru_traffic(a9_bytes, reps * req_per_launch),
+                     "requests_per_launch": req_per_launch,
                      "algorithmic_bytes_per_launch_mean": a9_bytes, "avg_launch_ms": lru_ms,
                      "launches_timed": kern["replay"]["launches"],
                      "note": "20 B per (request, replica, capacity) as SURVEY 8(d) counts a9; the kernel reads "
@@ -993,6 +1024,204 @@ def e2e_keys(args, pipe, keys, plens, slens, g0s, dev, stream, n_step, world):
             "note": "keys, prefix and suffix lengths of every interval copied from pinned host memory on a copy "
                     "stream each step (routing of an interval waits for its copy), counters read back; median "
                     "of the timed steps"}
+
+
+def run_resident_trace(args, cfg, trace, inputs, hash_bytes, dev, stream, world, rank, barrier):
+    """Resident-arena configurations with the multi-interval driver: every interval's prefix
+    spans are hashed on a stream of their own (one event per interval), and TracePipeline
+    plans and routes each interval as soon as its keys (and the previous interval's) exist,
+    the replay following in interval order."""
+    import torch
+    import torch.distributed as dist
+    import paper_2608_19677_gb300 as P
+    from paper_2608_19677_gb300.pipeline import TracePipeline
+
+    ctx = P.Context(dev.index if dev.index is not None else 0, stream)
+    n_step = sum(x[6] for x in inputs)
+    max_n = max(x[6] for x in inputs)
+    pipe = TracePipeline(ctx, cfg.R, cfg.W, cfg.caps, cfg.replicas, trace.qcap, max_n=max_n, batch_B=args.batch,
+                         depth=args.depth, plan_streams=args.plan_streams, route_streams=args.route_streams,
+                         vnodes=cfg.vnodes, fresh=args.fresh_plans, lru_tokens=cfg.lru_tokens,
+                         replay_first=args.replay_priority == "high", replay_group=args.replay_group)
+    hstream = torch.cuda.Stream(dev)
+    hctx = P.Context(ctx.device, hstream)
+    keys = [torch.empty(x[6], dtype=torch.int64, device=dev) for x in inputs]
+    g0s = [x[5] for x in inputs]
+
+    def enqueue(arenas, ready_in=None):
+        """Hash every interval (after its copy when ready_in is given), then the trace;
+        arenas[i] = (tokens, offsets, prefix lengths, suffix lengths) of interval i."""
+        pipe.reset()
+        start = torch.cuda.Event()
+        start.record(stream)
+        hstream.wait_event(start)
+        hashed = []
+        for i, (tok, off, plen, _) in enumerate(arenas):
+            if ready_in is not None:
+                hstream.wait_event(ready_in[i])
+            P.hash_prefixes(hctx, tok, off, plen, 0, out=keys[i])
+            e = torch.cuda.Event()
+            e.record(hstream)
+            hashed.append(e)
+        pipe.run(keys, [a[2] for a in arenas], [a[3] for a in arenas], g0s, ready=hashed)
+        stream.wait_event(hashed[-1])
+
+    resident = [(x[1], x[2], x[3], x[4]) for x in inputs]
+    for _ in range(max(args.warmup, 0)):
+        enqueue(resident)
+    pipe.sync()
+    hctx.sync()
+    prof = pipe.contexts + [hctx]
+    for c in prof:
+        c.profile_enable(16 * cfg.n_intervals * max(args.steps, 1) + 64)
+    clocks = ClockSampler(dev.index or 0, args.clocks_out)
+    clocks.start()
+    time.sleep(0.3)
+    barrier()
+    torch.cuda.synchronize()
+    l0 = pipe.launches + hctx.launches
+    ev0 = torch.cuda.Event(enable_timing=True)
+    ev1 = torch.cuda.Event(enable_timing=True)
+    ev0.record(stream)
+    for _ in range(args.steps):
+        enqueue(resident)
+    ev1.record(stream)
+    torch.cuda.synchronize()
+    barrier()
+    n_launch = pipe.launches + hctx.launches - l0
+    clk = clocks.stop()
+    pipe.sync()
+    kern = {}
+    for tag in ("hash", "plan", "route_cand", "route_resolve", "partition", "replay"):
+        n_, ms_ = 0, 0.0
+        for c in prof:
+            a, b = c.profile_read(tag)
+            n_, ms_ = n_ + a, ms_ + b
+        kern[tag] = {"launches": n_, "avg_ms": ms_ / n_ if n_ else None, "ms_per_step": ms_ / max(args.steps, 1)}
+    for c in prof:
+        c.profile_enable(0)
+    ms = ev0.elapsed_time(ev1) / args.steps
+    ms_max = max_over_ranks(ms, world, dev)
+    peaks = {}
+    try:
+        peaks = json.load(open(os.path.join(ROOT, "MEASURED_PEAKS.json")))
+    except Exception:
+        pass
+    hbm_peak = float(peaks.get("hbm_gbs", 6800.0))
+    peak_src = "measured" if "hbm_gbs" in peaks else "fallback"
+    reps, ncaps = len(cfg.replicas), len(cfg.caps)
+    hb = float(np.mean(hash_bytes))
+    hash_ms = kern["hash"]["avg_ms"]
+    hash_rf = {"kernel": "k_hash_prefixes", "bound": "hbm", "achieved": hb / (hash_ms / 1e3) / 1e9,
+               "peak": hbm_peak, "peak_source": peak_src, "unit": "GB/s",
+               "frac": hb / (hash_ms / 1e3) / 1e9 / hbm_peak, "traffic": hash_traffic(hb),
+               "algorithmic_bytes_per_launch_mean": hb, "avg_launch_ms": hash_ms,
+               "launches_timed": kern["hash"]["launches"]}
+    req_per_launch = n_step * args.steps / max(kern["replay"]["launches"], 1)
+    a9_bytes = 20.0 * reps * ncaps * req_per_launch
+    lru_ms = kern["replay"]["avg_ms"]
+    lru_rf = {"kernel": "k_lru_stamp (a9 LRU replay)" if not cfg.lru_tokens else "k_lru_tokens (a9 byte-aware replay)",
+              "bound": "hbm", "achieved": a9_bytes / (lru_ms / 1e3) / 1e9, "peak": hbm_peak,
+              "peak_source": peak_src, "unit": "GB/s", "frac": a9_bytes / (lru_ms / 1e3) / 1e9 / hbm_peak,
+              "traffic": lru_traffic(a9_bytes, reps * req_per_launch) if not cfg.lru_tokens else None,
+              "algorithmic_bytes_per_launch_mean": a9_bytes, "avg_launch_ms": lru_ms,
+              "requests_per_launch": req_per_launch, "launches_timed": kern["replay"]["launches"],
+              "note": "20 B per (request, replica, capacity) as SURVEY 8(d) counts a9"}
+    # the roofline object names the kernel with the larger share of the step
+    dom_lru = kern["replay"]["ms_per_step"] >= kern["hash"]["ms_per_step"]
+    rr_bytes = 8 + 2 * reps + 6 * reps + 20 * reps * ncaps
+    line = {
+        "metric": METRIC, "value": job_throughput(n_step, world, ms_max), "unit": UNIT, "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_max, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "u64", "data": "synthetic",
+        "config": dict(workload_config(cfg, args.batch, args.fresh_plans),
+                       schedule=(f"hashing on its own stream, one event per interval; {args.depth} intervals in "
+                                 f"flight: plans on {args.plan_streams} streams, routes on {args.route_streams} "
+                                 f"streams, the replay in interval order, {args.replay_group} intervals per call")),
+        "roofline": lru_rf if dom_lru else hash_rf,
+        ("hash_roofline" if dom_lru else "replay_roofline"): hash_rf if dom_lru else lru_rf,
+        "kernels_ms_per_launch": kern,
+        "route_replay": {"algorithmic_bytes_per_request": rr_bytes,
+                         "achieved_GBps": rr_bytes * n_step / (ms_max / 1e3) / 1e9,
+                         "hbm_frac": rr_bytes * n_step / (ms_max / 1e3) / 1e9 / hbm_peak,
+                         "note": "SURVEY 8(d) route + replay bytes over the whole step (hashing and plans included "
+                                 "in the time)"},
+        "gpu_launches": int(n_launch), "clocks": clk,
+    }
+    if not args.no_e2e:
+        line["e2e"] = e2e_resident(args, pipe, enqueue, inputs, dev, stream, n_step, world)
+    if not args.no_cpu_baseline and world == 1:
+        sample = oracle_interval_sample(trace)
+        nproc = os.cpu_count() or 1
+        t1 = oracle_interval_step(trace, sample, 1, args.batch)
+        tn = oracle_interval_step(trace, sample, nproc, args.batch)
+        line["cpu_baseline"] = {"value": sample["n"] / tn, "unit": UNIT, "cores": nproc, "kind": "oracle",
+                                "sample": f"interval 0 of {cfg.n_intervals} ({sample['n']} requests, all "
+                                          f"{len(cfg.replicas)} replicas), hash+plan+route+replay, C oracle on "
+                                          f"{nproc} host threads over request ranges, plan variants and replicas",
+                                "single_thread": {"value": sample["n"] / t1, "unit": UNIT, "cores": 1},
+                                "nproc": nproc}
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    pipe.close()
+    hctx.close()
+    if world > 1:
+        dist.destroy_process_group()
+
+
+def e2e_resident(args, pipe, enqueue, inputs, dev, stream, n_step, world):
+    """End to end through the public API: every step copies each interval's token arena,
+    offsets and lengths from pinned host memory (a copy stream, one event per interval, so
+    hashing of interval t starts once its inputs have landed), runs the trace and reads
+    the counters back."""
+    import torch
+    host, dbuf = [], []
+    for (t, tok, off, plen, slen, g0, n) in inputs:
+        h = []
+        for x in (tok, off, plen, slen):
+            p = torch.empty(x.shape, dtype=x.dtype, pin_memory=True)
+            p.copy_(x)
+            h.append(p)
+        host.append(h)
+        dbuf.append([torch.empty_like(x, device=dev) for x in h])
+    h2d = sum(x.numel() * x.element_size() for h in host for x in h)
+    copy_stream = torch.cuda.Stream(dev)
+    out = torch.empty(pipe.ctr.shape, dtype=torch.int64, pin_memory=True)
+    d2h = out.numel() * out.element_size()
+
+    def step():
+        start = torch.cuda.Event()
+        start.record(stream)
+        copy_stream.wait_event(start)
+        ready = []
+        with torch.cuda.stream(copy_stream):
+            for h, d in zip(host, dbuf):
+                for a, b in zip(h, d):
+                    b.copy_(a, non_blocking=True)
+                e = torch.cuda.Event()
+                e.record(copy_stream)
+                ready.append(e)
+        enqueue([(d[0], d[1], d[2], d[3]) for d in dbuf], ready_in=ready)
+        out.copy_(pipe.ctr, non_blocking=True)
+
+    for _ in range(2):
+        step()
+    torch.cuda.synchronize()
+    each = []
+    for _ in range(args.e2e_steps):
+        e0 = torch.cuda.Event(enable_timing=True)
+        e1 = torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        step()
+        e1.record(stream)
+        e1.synchronize()
+        each.append(e0.elapsed_time(e1))
+    ms = max_over_ranks(float(np.median(each)), world, dev)
+    return {"value": job_throughput(n_step, world, ms), "unit": UNIT, "h2d_bytes_per_step": h2d,
+            "d2h_bytes_per_step": d2h, "ms_per_step": ms, "ms_per_step_each": [round(x, 2) for x in each],
+            "note": "token arenas, offsets, prefix and suffix lengths of every interval copied from pinned host "
+                    "memory on a copy stream each step (hashing of an interval waits for its copy), counters read "
+                    "back; median of the timed steps"}
 
 
 def e2e(args, ctx, pipe, inputs, dev, stream, n_step, world):

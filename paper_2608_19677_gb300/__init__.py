@@ -23,7 +23,9 @@ from typing import List, Optional, Sequence
 import numpy as np
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
-LIB_PATH = os.path.join(_HERE, "libcacheroute.so")
+# CR_DEBUG_LIB=1 loads the bounds-checking build (buildlib.build(debug=True)) instead
+LIB_PATH = os.path.join(_HERE, "libcacheroute_debug.so" if os.environ.get("CR_DEBUG_LIB") == "1"
+                        else "libcacheroute.so")
 
 CR_OK, CR_EINVAL, CR_ENOMEM, CR_ECUDA, CR_ETIMEOUT, CR_EOVERFLOW = range(6)
 STATUS_NAMES = {0: "CR_OK", 1: "CR_EINVAL", 2: "CR_ENOMEM", 3: "CR_ECUDA", 4: "CR_ETIMEOUT",

@@ -307,6 +307,9 @@ extern "C" int cr_sync(cr_ctx *ctx)
             return cr_fail(ctx, CR_EOVERFLOW, "a load or counter exceeded its documented range");
         if (flags & CR_FLAG_TIMEOUT)
             return cr_fail(ctx, CR_ETIMEOUT, "a bounded device-side wait gave up");
+        if (flags & CR_FLAG_BOUNDS)
+            return cr_fail(ctx, CR_EINVAL, "debug build: an index outside its array was skipped (results of that "
+                                           "call are not meaningful)");
         if (flags & CR_FLAG_INTERNAL)
             return cr_fail(ctx, CR_ECUDA, "a kernel found its state inconsistent (results of that call are not "
                                           "meaningful)");

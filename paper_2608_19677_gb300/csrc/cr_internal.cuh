@@ -22,6 +22,17 @@ struct cr_nvtx_range {
 #define CR_FLAG_TIMEOUT 4u   // a bounded wait gave up
 #define CR_FLAG_BADSIZE 8u   // token-weighted replay: a key came back with another prefix length
 #define CR_FLAG_INTERNAL 16u // a kernel found its own state inconsistent and skipped the access
+#define CR_FLAG_BOUNDS 32u   // debug build: an index outside its array was skipped
+
+// Debug build (compiled with -DCR_DEBUG_CHECKS, see buildlib.py): data-dependent
+// indices are checked before use; a failing check raises CR_FLAG_BOUNDS in the
+// status word and the caller skips the access.  In the normal build the check
+// is the constant true and costs nothing.
+#ifdef CR_DEBUG_CHECKS
+#define CR_DCHECK(ok, status) ((ok) || (atomicOr((status), CR_FLAG_BOUNDS), false))
+#else
+#define CR_DCHECK(ok, status) (true)
+#endif
 
 // ---- scratch slots owned by the context ------------------------------------
 enum cr_scratch_slot {
@@ -115,7 +126,7 @@ struct cr_ring {
 struct cr_replay {
     uint32_t n_rep, R, n_caps, cmax;  // cmax: largest capacity, or CR_MAX_CAP entries in token mode
     int tokens;                       // capacities in prefix tokens (one state buffer, d_size used)
-    uint32_t *d_size;                // token mode: [stream][cmax] tokens of the listed keys up to each one
+    uint32_t *d_size[2];             // token mode: [stream][cmax] tokens of the listed keys up to each one
     uint32_t caps[CR_MAX_CAPS];
     uint64_t n_streams;              // n_rep * R
     unsigned long long *d_keys[2];   // [stream][cmax], most recent first; double-buffered

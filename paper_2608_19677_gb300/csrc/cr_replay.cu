@@ -481,16 +481,19 @@ struct live_prefix {
     uint32_t w[NG], ex[NG];
     __device__ __forceinline__ void load(const uint32_t *BM, uint32_t nw, uint32_t lane)
     {
-        uint32_t run = 0;
+        // both groups' popcounts in one scan: group g in bits 16 g .. 16 g + 15
+        // (a group holds at most 1024 live bits, so the halves never carry)
+        uint32_t pc = 0;
 #pragma unroll
         for (int g = 0; g < NG; ++g) {
             const uint32_t wi = 32u * g + lane;
             w[g] = wi < nw ? BM[wi] : 0u;
-            const uint32_t pc = (uint32_t)__popc(w[g]);
-            const uint32_t incl = warp_incl_scan(pc, lane);
-            ex[g] = run + incl - pc;
-            run += __shfl_sync(0xffffffffu, incl, 31);
+            pc |= (uint32_t)__popc(w[g]) << (16 * g);
         }
+        const uint32_t incl = warp_incl_scan(pc, lane);
+        const uint32_t ex2 = incl - pc;
+        ex[0] = ex2 & 0xffffu;
+        if (NG > 1) ex[NG - 1] = (ex2 >> 16) + (__shfl_sync(0xffffffffu, incl, 31) & 0xffffu);
     }
     // live stamps < s; every lane of the warp must call it
     __device__ __forceinline__ uint32_t below(uint32_t s) const
@@ -611,12 +614,20 @@ k_lru_stamp(const replay_caps caps, uint32_t cmax, uint32_t nw, uint32_t R, uint
     for (int c = 0; c < NC; ++c) my_hit[c] = my_tok[c] = 0;
 
     rec16 ahead = {0ull, 0u, 0u};  // the next step's records, loaded one step early
-    if (p0 + lane < p1) ahead = recs[min(idx[p0 + lane], nrec - 1u)];  // (the bound guards the gather)
+    if (p0 + lane < p1) {
+        const uint32_t ix = idx[p0 + lane];
+        CR_DCHECK(ix < nrec, status);
+        ahead = recs[min(ix, nrec - 1u)];  // (the bound guards the gather)
+    }
     for (uint32_t t0 = p0; t0 < p1; t0 += 32) {
         const uint32_t cnt = (p1 - t0) < 32u ? (p1 - t0) : 32u;
         const bool valid = lane < cnt;
         const rec16 mine = ahead;
-        if (t0 + 32u + lane < p1) ahead = recs[min(idx[t0 + 32u + lane], nrec - 1u)];
+        if (t0 + 32u + lane < p1) {
+            const uint32_t ix = idx[t0 + 32u + lane];
+            CR_DCHECK(ix < nrec, status);
+            ahead = recs[min(ix, nrec - 1u)];
+        }
         if (valid) {
             my_req += 1;
             my_prompt += (unsigned long long)mine.P + mine.S;
@@ -907,42 +918,117 @@ __device__ __forceinline__ uint32_t sat_add(uint32_t a, uint32_t b)
     return v > 0xffffffffull ? 0xffffffffu : (uint32_t)v;
 }
 
+struct token_state {
+    const unsigned long long *keys_in;  // [stream][kTokMax], most recent first
+    const uint32_t *cum_in;             // [stream][kTokMax], tokens of entries 0..j
+    const uint32_t *fill_in;
+    unsigned long long *keys_out;
+    uint32_t *cum_out;
+    uint32_t *fill_out;
+};
+
 __global__ void __launch_bounds__(kTokWarps * 32) k_lru_tokens(const __grid_constant__ replay_caps caps, uint32_t ns,
-                                                               uint32_t R, const uint32_t *__restrict__ start,
+                                                               uint32_t R, uint32_t CL, const uint32_t *__restrict__ start,
+                                                               const uint32_t *__restrict__ coff,
+                                                               const uint32_t *__restrict__ total,
                                                                const uint32_t *__restrict__ idx,
                                                                const rec16 *__restrict__ recs, uint32_t nrec,
-                                                               unsigned long long *__restrict__ keys_state,
-                                                               uint32_t *__restrict__ cum_state,
-                                                               uint32_t *__restrict__ fill_state,
+                                                               const token_state st,
                                                                unsigned long long *__restrict__ ctr, uint32_t *status)
 {
     extern __shared__ unsigned long long tok_sh[];
     const uint32_t lane = threadIdx.x & 31, w = threadIdx.x >> 5;
-    const uint32_t s = blockIdx.x * kTokWarps + w;
-    if (s >= ns) return;  // whole warps only; the kernel has no block-wide barrier
+    const uint32_t wi = blockIdx.x * kTokWarps + w;
+    if (wi >= *total) return;  // whole warps only; the kernel has no block-wide barrier
+    // work item -> (stream, chunk)
+    uint32_t lo_s = 0, hi_s = ns;
+    while (hi_s - lo_s > 1) {
+        const uint32_t mid = (lo_s + hi_s) >> 1;
+        if (coff[mid] <= wi)
+            lo_s = mid;
+        else
+            hi_s = mid;
+    }
+    const uint32_t s = lo_s, ci = wi - coff[s];
+    const uint32_t b = start[s], e = start[s + 1];
     unsigned long long *K = tok_sh + (size_t)w * kTokMax;
     uint32_t *Cm = reinterpret_cast<uint32_t *>(tok_sh + (size_t)kTokWarps * kTokMax) + (size_t)w * kTokMax;
     uint32_t capmax = 0;
     for (uint32_t c = 0; c < caps.n_caps; ++c) capmax = caps.cap[c] > capmax ? caps.cap[c] : capmax;
     const uint32_t mycap = lane < caps.n_caps ? caps.cap[lane] : 0u;
-    uint32_t f = fill_state[s];
-    unsigned long long kr = 0;  // register list: entry `lane`
-    uint32_t cr = 0;
-    bool inreg = f <= 32;
-    if (inreg) {
-        if (lane < f) {
-            kr = keys_state[(size_t)s * kTokMax + lane];
-            cr = cum_state[(size_t)s * kTokMax + lane];
+    const uint32_t fin = st.fill_in[s];
+    const unsigned long long *kin = st.keys_in + (size_t)s * kTokMax;
+    const uint32_t *cin = st.cum_in + (size_t)s * kTokMax;
+    if (b == e) {  // nothing routed here: carry the state over unchanged
+        for (uint32_t j = lane; j < fin; j += 32) {
+            st.keys_out[(size_t)s * kTokMax + j] = kin[j];
+            st.cum_out[(size_t)s * kTokMax + j] = cin[j];
+        }
+        if (lane == 0) st.fill_out[s] = fin;
+        return;
+    }
+    const uint32_t i0 = b + ci * CL;
+    const uint32_t i1 = (e - i0) < CL ? e : i0 + CL;
+    uint32_t f = 0;
+    if (ci == 0) {
+        f = fin;
+        for (uint32_t j = lane; j < f; j += 32) {
+            K[j] = kin[j];
+            Cm[j] = cin[j];
         }
     } else {
-        for (uint32_t j = lane; j < f; j += 32) {
-            K[j] = keys_state[(size_t)s * kTokMax + j];
-            Cm[j] = cum_state[(size_t)s * kTokMax + j];
+        // the state at i0 is the longest run of most recent distinct prefixes that fits
+        // (tokens <= the largest capacity, at most kTokMax of them): walk back over the
+        // stream, then over the carried-in list, keeping each key's most recent access
+        const uint32_t back = i0 - b;
+        uint32_t tot = 0;
+        bool stop = false;
+        for (uint32_t v0 = 0; v0 < back + fin && !stop; v0 += 32) {
+            const uint32_t v = v0 + lane;
+            unsigned long long ck = 0;
+            uint32_t cp = 0;
+            if (v < back) {
+                const rec16 rr = recs[min(idx[i0 - 1 - v], nrec - 1u)];
+                ck = rr.key;
+                cp = rr.P;
+            } else if (v < back + fin) {
+                const uint32_t j = v - back;
+                ck = kin[j];
+                cp = cin[j] - (j ? cin[j - 1] : 0u);
+            }
+            const uint32_t nb = min(32u, back + fin - v0);
+            for (uint32_t q = 0; q < nb; ++q) {  // uniform over the warp
+                const unsigned long long x = __shfl_sync(0xffffffffu, ck, q);
+                const uint32_t P = __shfl_sync(0xffffffffu, cp, q);
+                bool seen = false;
+                for (uint32_t c0 = 0; c0 < f && !seen; c0 += 32)
+                    seen = __ballot_sync(0xffffffffu, c0 + lane < f && K[c0 + lane] == x) != 0;
+                if (seen) continue;
+                const unsigned long long nt = (unsigned long long)tot + P;
+                if (f == kTokMax || nt > capmax) {  // the first distinct prefix that does not fit ends the run
+                    stop = true;
+                    break;
+                }
+                tot = (uint32_t)nt;
+                if (lane == 0) {
+                    K[f] = x;
+                    Cm[f] = tot;
+                }
+                ++f;
+                __syncwarp();
+            }
         }
     }
     __syncwarp();
+    unsigned long long kr = 0;  // register list: entry `lane`
+    uint32_t cr = 0;
+    bool inreg = f <= 32;
+    if (inreg && lane < f) {
+        kr = K[lane];
+        cr = Cm[lane];
+    }
+    __syncwarp();
     unsigned long long c_hit = 0, c_hit_tok = 0, c_prompt = 0;  // lane = capacity (prompt: every lane)
-    const uint32_t i0 = start[s], i1 = start[s + 1];
     rec16 nx = {0ull, 0u, 0u};
     if (i0 + lane < i1) nx = recs[min(idx[i0 + lane], nrec - 1u)];
     for (uint32_t b0 = i0; b0 < i1; b0 += 32) {
@@ -1054,27 +1140,29 @@ __global__ void __launch_bounds__(kTokWarps * 32) k_lru_tokens(const __grid_cons
             }
         }
     }
-    if (inreg) {
-        if (lane < f) {
-            keys_state[(size_t)s * kTokMax + lane] = kr;
-            cum_state[(size_t)s * kTokMax + lane] = cr;
+    if (i1 == e) {  // the stream's last chunk hands the state to the next call
+        if (inreg) {
+            if (lane < f) {
+                st.keys_out[(size_t)s * kTokMax + lane] = kr;
+                st.cum_out[(size_t)s * kTokMax + lane] = cr;
+            }
+        } else {
+            for (uint32_t j = lane; j < f; j += 32) {
+                st.keys_out[(size_t)s * kTokMax + j] = K[j];
+                st.cum_out[(size_t)s * kTokMax + j] = Cm[j];
+            }
         }
-    } else {
-        for (uint32_t j = lane; j < f; j += 32) {
-            keys_state[(size_t)s * kTokMax + j] = K[j];
-            cum_state[(size_t)s * kTokMax + j] = Cm[j];
-        }
+        if (lane == 0) st.fill_out[s] = f;
     }
-    if (lane == 0) fill_state[s] = f;
     for (int o = 16; o > 0; o >>= 1) c_prompt += __shfl_xor_sync(0xffffffffu, c_prompt, o);
     if (lane < caps.n_caps) {
         const uint32_t rep = s / R, r = s - rep * R;
         unsigned long long *C = ctr + (((unsigned long long)rep * caps.n_caps + lane) * R + r) * CR_CTR_FIELDS;
-        C[0] += i1 - i0;
-        C[1] += c_hit;
-        C[2] += c_hit_tok;
-        C[3] += c_prompt;
-        C[4] += c_prompt - c_hit_tok;
+        atomicAdd(&C[0], (unsigned long long)(i1 - i0));
+        if (c_hit) atomicAdd(&C[1], c_hit);
+        if (c_hit_tok) atomicAdd(&C[2], c_hit_tok);
+        atomicAdd(&C[3], c_prompt);
+        atomicAdd(&C[4], c_prompt - c_hit_tok);
     }
 }
 
@@ -1139,12 +1227,14 @@ extern "C" int cr_replay_create_tokens(cr_ctx *ctx, uint32_t n_rep, uint32_t R, 
     rp->tokens = 1;
     memcpy(rp->caps, token_caps, n_caps * sizeof(uint32_t));
     rp->n_streams = (uint64_t)n_rep * R;
-    if (cudaMalloc(&rp->d_keys[0], rp->n_streams * kTokMax * sizeof(unsigned long long)) != cudaSuccess ||
-        cudaMalloc(&rp->d_size, rp->n_streams * kTokMax * sizeof(uint32_t)) != cudaSuccess ||
-        cudaMalloc(&rp->d_fill[0], rp->n_streams * sizeof(uint32_t)) != cudaSuccess) {
-        cudaGetLastError();
-        cr_replay_destroy(ctx, rp);
-        return cr_fail(ctx, CR_ENOMEM, "replay: cannot allocate state");
+    for (int x = 0; x < 2; ++x) {  // double-buffered: chunks of a stream read the old state
+        if (cudaMalloc(&rp->d_keys[x], rp->n_streams * kTokMax * sizeof(unsigned long long)) != cudaSuccess ||
+            cudaMalloc(&rp->d_size[x], rp->n_streams * kTokMax * sizeof(uint32_t)) != cudaSuccess ||
+            cudaMalloc(&rp->d_fill[x], rp->n_streams * sizeof(uint32_t)) != cudaSuccess) {
+            cudaGetLastError();
+            cr_replay_destroy(ctx, rp);
+            return cr_fail(ctx, CR_ENOMEM, "replay: cannot allocate state");
+        }
     }
     *out = rp;
     return cr_replay_reset(ctx, rp);
@@ -1167,7 +1257,8 @@ extern "C" int cr_replay_destroy(cr_ctx *ctx, cr_replay *rp)
         if (rp->d_keys[b]) cudaFree(rp->d_keys[b]);
         if (rp->d_fill[b]) cudaFree(rp->d_fill[b]);
     }
-    if (rp->d_size) cudaFree(rp->d_size);
+    for (int b = 0; b < 2; ++b)
+        if (rp->d_size[b]) cudaFree(rp->d_size[b]);
     free(rp);
     return CR_OK;
 }
@@ -1219,16 +1310,31 @@ extern "C" int cr_shadow_replay(cr_ctx *ctx, cr_replay *rp, const uint64_t *d_ke
     caps.n_caps = rp->n_caps;
     for (uint32_t c = 0; c < CR_MAX_CAPS; ++c) caps.cap[c] = c < rp->n_caps ? rp->caps[c] : 0;
     if (rp->tokens) {
-        // token-weighted: one warp per stream, its list in shared memory, state updated in place
+        // token-weighted: one warp per (stream, chunk), its list in registers or shared memory
+        uint32_t capmax = 0;
+        for (uint32_t c = 0; c < rp->n_caps; ++c) capmax = rp->caps[c] > capmax ? rp->caps[c] : capmax;
+        // chunks long against the rebuild walk, which reaches back until the largest capacity fills
+        const uint32_t TCL = capmax <= (1u << 16) ? 1024u : (capmax <= (1u << 17) ? 4096u : 16384u);
+        CR_LAUNCH(ctx, k_chunk_counts, cr_blocks(ns, 256, gcap), 256, 0, (const uint32_t *)start, ns, TCL, coff);
+        CR_TRY(cr_scan_u32(ctx, coff, coff, ns, total));
         const size_t tsmem = (size_t)kTokWarps * kTokMax * (sizeof(unsigned long long) + sizeof(uint32_t));
         if (tsmem > 48 * 1024)
             CR_CUDA(ctx, cudaFuncSetAttribute(k_lru_tokens, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)tsmem));
+        token_state tst;
+        tst.keys_in = rp->d_keys[rp->cur];
+        tst.cum_in = rp->d_size[rp->cur];
+        tst.fill_in = rp->d_fill[rp->cur];
+        tst.keys_out = rp->d_keys[rp->cur ^ 1];
+        tst.cum_out = rp->d_size[rp->cur ^ 1];
+        tst.fill_out = rp->d_fill[rp->cur ^ 1];
+        const uint64_t items = (uint64_t)ns + (m + TCL - 1) / TCL;  // upper bound on work items
         const int pt = cr_prof_begin(ctx, ctx->stream, CR_PROF_REPLAY);
-        CR_LAUNCH(ctx, k_lru_tokens, (ns + kTokWarps - 1) / kTokWarps, kTokWarps * 32, tsmem, caps, ns, R,
-                  (const uint32_t *)start, (const uint32_t *)idx, (const rec16 *)recs, (uint32_t)n,
-                  (unsigned long long *)rp->d_keys[0], rp->d_size,
-                  rp->d_fill[0], (unsigned long long *)d_ctr, ctx->d_status);
+        CR_LAUNCH(ctx, k_lru_tokens, (unsigned int)((items + kTokWarps - 1) / kTokWarps), kTokWarps * 32, tsmem,
+                  caps, ns, R, TCL, (const uint32_t *)start, (const uint32_t *)coff, (const uint32_t *)total,
+                  (const uint32_t *)idx, (const rec16 *)recs, (uint32_t)n, tst, (unsigned long long *)d_ctr,
+                  ctx->d_status);
         cr_prof_end(ctx, ctx->stream, pt);
+        rp->cur ^= 1;
         return CR_OK;
     }
     // chunk length: long enough that rebuilding an LRU state of cmax entries is amortised

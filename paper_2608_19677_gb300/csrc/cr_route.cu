@@ -243,6 +243,11 @@ __device__ __forceinline__ uint32_t resolve(uint32_t c, const route_desc &rd, co
         return L[d1] <= L[d2] ? d1 : d2;
     }
     const cr_table_slot slot = rd.table[c & kLow30];
+#ifdef CR_DEBUG_CHECKS
+    // the member list of the slot lies inside the plan's members (sum of k_b)
+    if (!CR_DCHECK(rd.n_members == nullptr || (unsigned long long)slot.koff + slot.k <= *rd.n_members, status))
+        return 0;
+#endif
     return set_min(mem, slot.koff, slot.k, slot.m0, load_of);
 }
 
@@ -280,6 +285,7 @@ __device__ __forceinline__ void resolve_batches(const route_desc &rd, const uint
             const unsigned long long b1 = (b0 + B < n) ? b0 + B : n;
             for (unsigned long long i = b0 + tid; i < b1; i += blockDim.x) {
                 const uint32_t d = resolve<RING>(Cd[i], rd, mem, L, tot0 + b0, R, status);
+                if (!CR_DCHECK(d < R, status)) continue;
                 D[i] = (uint16_t)d;
                 atomicAdd(&delta[d], 1u);
             }
@@ -309,6 +315,7 @@ __device__ __forceinline__ void resolve_batches(const route_desc &rd, const uint
             const unsigned long long b1 = (b0 + B < c1) ? b0 + B : c1;
             for (unsigned long long i = b0 + tid; i < b1; i += blockDim.x) {
                 const uint32_t d = resolve<RING>(cb[i - c0], rd, mem, L, tot0 + b0, R, status);
+                if (!CR_DCHECK(d < R, status)) continue;
                 D[i] = (uint16_t)d;
                 atomicAdd(&delta[d], 1u);
             }
@@ -466,12 +473,14 @@ __global__ void __launch_bounds__(32) k_route_resolve_warp(const __grid_constant
             const unsigned long long cap = ring ? chwbl_cap(tot + bstart, R) : 0ull;
             const prep_cand pq = ps[q * 32 + lane];
             uint32_t d = decide(pq, rd, mem, L, mask, 0u, cap, status);
+            if (!CR_DCHECK(d < R, status)) d = 0;
             if (active) atomicOr(&mask[d], bit);
             __syncwarp();
             if (several) {
                 // fixed point: after iteration t the first t batches of the step are final
                 for (uint32_t it = 0;; ++it) {
-                    const uint32_t nd = active ? decide(pq, rd, mem, L, mask, earlier, cap, status) : d;
+                    uint32_t nd = active ? decide(pq, rd, mem, L, mask, earlier, cap, status) : d;
+                    if (!CR_DCHECK(nd < R, status)) nd = 0;
                     const uint32_t moved = __ballot_sync(0xffffffffu, nd != d);
                     if (!moved) break;
                     if (it >= S) {  // unreachable: S iterations always settle the step

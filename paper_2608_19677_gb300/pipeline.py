@@ -367,7 +367,7 @@ class TracePipeline:
                  replicas: Sequence[Tuple[str, int]], qcap: Callable[[int], Tuple[int, int]],
                  max_n: int, batch_B: int = 1024, depth: int = 8, plan_streams: int = 4,
                  route_streams: int = 4, vnodes: int = 64, fresh: bool = False, lru_tokens: bool = False,
-                 replay_first: bool = True):
+                 replay_first: bool = False, replay_group: int = 1):
         import torch
         self.ctx, self.R, self.W, self.caps = ctx, R, W, list(caps)
         self.replicas = list(replicas)
@@ -407,6 +407,18 @@ class TracePipeline:
         self.loads = [torch.zeros((nrep, R), dtype=torch.int64, device=self.dev) for _ in self.rstreams]
         self.max_n = max_n
         self.dests = [torch.empty(nrep * max_n, dtype=torch.int16, device=self.dev) for _ in range(self.depth)]
+        # grouped replay: `replay_group` consecutive intervals are staged into one buffer
+        # (inputs and destinations, [replica][request of the group]) and replayed by one
+        # call, which pays the per-stream setup of the replay once per group
+        self.group = max(1, replay_group)
+        self.gbuf = []
+        if self.group > 1:
+            G = self.group * max_n
+            for _ in range(2):
+                self.gbuf.append((torch.empty(G, dtype=torch.int64, device=self.dev),
+                                  torch.empty(G, dtype=torch.int32, device=self.dev),
+                                  torch.empty(G, dtype=torch.int32, device=self.dev),
+                                  torch.empty(nrep * G, dtype=torch.int16, device=self.dev)))
         ctx.sync()
         self._reset_events()
         self.plan_marks, self.route_marks, self.replay_marks = [], [], []
@@ -415,6 +427,7 @@ class TracePipeline:
         self._plan_free = [None] * self.depth   # route that last read plans buffer b
         self._dest_free = [None] * self.depth   # replay that last read destinations buffer b
         self._load_free = [None] * len(self.rstreams)
+        self._gfree = [None, None]              # replay that last read group buffer k
 
     @property
     def contexts(self):
@@ -448,6 +461,17 @@ class TracePipeline:
         for s in self.pstreams + self.rstreams + [self.ystream]:
             s.wait_event(start)
         self.plan_marks, self.route_marks, self.replay_marks = [], [], []
+        # replay groups: [g0, g1) intervals, their request count, and each interval's column
+        sizes = [int(k.shape[0]) for k in keys]
+        groups, col = [], [0] * T
+        for g0 in range(0, T, self.group):
+            g1 = min(T, g0 + self.group)
+            c = 0
+            for t in range(g0, g1):
+                col[t] = c
+                c += sizes[t]
+            groups.append((g0, g1, c))
+        staged = []
         for t in range(T):
             n = int(keys[t].shape[0])
             if n > self.max_n:
@@ -491,16 +515,43 @@ class TracePipeline:
             if mark:
                 self.route_marks.append((r0, routed))
             self._plan_free[b] = routed
-            # ---- replay, in interval order ----------------------------------------------
-            self.ystream.wait_event(routed)
-            y0 = self._event(self.ystream, True) if mark else None
-            shadow_replay(self.yctx, self.replay, keys[t], plens[t], slens[t], dest, self.ctr)
-            replayed = self._event(self.ystream, mark)
-            if mark:
-                self.replay_marks.append((y0, replayed))
-            self._dest_free[b] = replayed
             if on_interval is not None:
                 on_interval(t, dest, self.plans[b] if self.plan_keys else [])
+            # ---- replay, in interval order ----------------------------------------------
+            if self.group == 1:
+                self.ystream.wait_event(routed)
+                y0 = self._event(self.ystream, True) if mark else None
+                shadow_replay(self.yctx, self.replay, keys[t], plens[t], slens[t], dest, self.ctr)
+                replayed = self._event(self.ystream, mark)
+                if mark:
+                    self.replay_marks.append((y0, replayed))
+                self._dest_free[b] = replayed
+                continue
+            gi = t // self.group
+            g0, g1, N = groups[gi]
+            gk, gp, gs, gd = self.gbuf[gi % 2]
+            if self._gfree[gi % 2] is not None:
+                rs.wait_event(self._gfree[gi % 2])   # the group before last has been replayed
+            with torch.cuda.stream(rs):  # stage the interval into the group buffer
+                c = col[t]
+                gk[c:c + n].copy_(keys[t])
+                gp[c:c + n].copy_(plens[t])
+                gs[c:c + n].copy_(slens[t])
+                gd[:len(self.replicas) * N].view(len(self.replicas), N)[:, c:c + n].copy_(dest)
+            st_ev = self._event(rs)
+            staged.append(st_ev)
+            self._dest_free[b] = st_ev
+            if t == g1 - 1:
+                for e in staged:
+                    self.ystream.wait_event(e)
+                staged = []
+                y0 = self._event(self.ystream, True) if mark else None
+                shadow_replay(self.yctx, self.replay, gk[:N], gp[:N], gs[:N],
+                              gd[:len(self.replicas) * N].view(len(self.replicas), N), self.ctr)
+                replayed = self._event(self.ystream, mark)
+                if mark:
+                    self.replay_marks.append((y0, replayed))
+                self._gfree[gi % 2] = replayed
         for s in self.pstreams + self.rstreams + [self.ystream]:
             self.mstream.wait_event(self._event(s))
 

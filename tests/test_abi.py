@@ -59,3 +59,13 @@ def test_product_never_imports_the_oracle():
                 txt = open(os.path.join(dirpath, f)).read()
                 assert not re.search(r"^\s*(import|from)\s+oracle\b", txt, flags=re.M), f
                 assert "cr_oracle" not in txt and "libcr_oracle" not in txt, f
+
+
+def test_debug_build_compiles_and_exports_every_symbol():
+    # the bounds-checking variant (-DCR_DEBUG_CHECKS) builds for sm_103a and exports the same ABI
+    from paper_2608_19677_gb300 import buildlib
+    path = buildlib.build(debug=True)
+    assert path.endswith("libcacheroute_debug.so") and os.path.exists(path)
+    lib = ctypes.CDLL(path)
+    missing = [s for s in _declared() if not hasattr(lib, s)]
+    assert not missing, missing

@@ -497,10 +497,13 @@ def test_pipeline_parity(P, ctx, name, n, nint, overlap):
         assert (h_u64(pipe.ctr) == ref["ctr"]).all()
 
 
-@pytest.mark.parametrize("name,n,nint,depth,ps,rs", [("70b", 40000, 6, 3, 2, 2), ("8b", 8000, 9, 4, 3, 2),
-                                                      ("burst", 40000, 4, 2, 1, 3), ("large", 200000, 3, 8, 4, 4),
-                                                      ("tiny", 20000, 1, 8, 4, 4)])
-def test_trace_pipeline_parity(P, ctx, name, n, nint, depth, ps, rs):
+@pytest.mark.parametrize("name,n,nint,depth,ps,rs,grp", [("70b", 40000, 6, 3, 2, 2, 1), ("8b", 8000, 9, 4, 3, 2, 1),
+                                                          ("burst", 40000, 4, 2, 1, 3, 1),
+                                                          ("large", 200000, 3, 8, 4, 4, 1),
+                                                          ("tiny", 20000, 1, 8, 4, 4, 1),
+                                                          ("70b", 40000, 7, 4, 2, 3, 3), ("8b", 8000, 9, 6, 2, 2, 4),
+                                                          ("large", 200000, 3, 8, 4, 4, 2)])
+def test_trace_pipeline_parity(P, ctx, name, n, nint, depth, ps, rs, grp):
     # several intervals in flight (plans and routes on several streams, the replay in order):
     # every interval's plans and destinations, and the counters, equal the oracle's
     from paper_2608_19677_gb300.pipeline import TracePipeline
@@ -514,7 +517,8 @@ def test_trace_pipeline_parity(P, ctx, name, n, nint, depth, ps, rs):
     plens = [d_u32(iv.plen) for iv in ivs]
     slens = [d_u32(iv.slen) for iv in ivs]
     pipe = TracePipeline(ctx, cfg.R, cfg.W, cfg.caps, cfg.replicas, tr.qcap, max_n=max(iv.n for iv in ivs),
-                         batch_B=1024, depth=depth, plan_streams=ps, route_streams=rs, vnodes=cfg.vnodes)
+                         batch_B=1024, depth=depth, plan_streams=ps, route_streams=rs, vnodes=cfg.vnodes,
+                         replay_group=grp)
     for rep in range(2):   # twice: reset() restores the initial state
         pipe.reset()
         seen = []
@@ -653,6 +657,38 @@ def test_token_replay_parity(P, ctx, caps, lo, hi):
     dk, dp, ds, dd = d_u64(keys), d_u32(plen), d_u32(slen), d_u16(dest)
     cut = n // 3
     for a, b in ((0, cut), (cut, n)):  # state persists across calls
+        orp.step(keys[a:b], plen[a:b], slen[a:b], dest[:, a:b])
+        P.shadow_replay(ctx, rp, dk[a:b].contiguous(), dp[a:b].contiguous(), ds[a:b].contiguous(),
+                        dd[:, a:b].contiguous(), ctr)
+        ctx.sync()
+        assert (h_u64(ctr) == orp.ctr).all()
+    ci = caps.index(max(caps))
+    for rep in range(n_rep):
+        for r in range(R):
+            assert (rp.state(rep, r) == orp.state(rep, ci, r)).all()
+
+
+@pytest.mark.parametrize("caps,lo,hi,nkeys", [([24576], 16, 5000, 400), ([1, 100, 3000], 16, 5000, 2000),
+                                              ([4096, 65536, 2 ** 31], 16, 200, 3000)])
+def test_token_replay_parity_long_streams(P, ctx, caps, lo, hi, nkeys):
+    # streams much longer than the chunks the byte-aware replay splits them into: every chunk
+    # after a stream's first rebuilds its starting list by walking back over the stream and
+    # the carried-in list, in both calls
+    rng = np.random.default_rng(nkeys + lo)
+    n_rep, R, n = 2, 2, 80000
+    keys, plen = _fixed_len_stream(rng, n, nkeys, lo, hi)
+    n = keys.size
+    slen = rng.integers(0, 200, size=n).astype(np.uint32)
+    dest = tg.random_dest(n_rep, n, R, 8)
+    orp = O.Replay(n_rep, R, caps, tokens=True)
+    rp = P.Replay(ctx, n_rep, R, caps, tokens=True)
+    ctr = torch.zeros((n_rep, len(caps), R, 5), dtype=torch.int64, device=DEV)
+    dk, dp, ds, dd = d_u64(keys), d_u32(plen), d_u32(slen), d_u16(dest)
+    cut = n // 3
+    for a, b in ((0, cut), (cut, n)):
+        if a == cut:  # the second call's streams span several chunks at every capacity tested
+            assert np.bincount(dest[0, a:b], minlength=R).min() > (16384 if max(caps) > (1 << 17) else 4096)
+            # (capacities up to 2^16 tokens use chunks of 1,024 requests, up to 2^17 of 4,096)
         orp.step(keys[a:b], plen[a:b], slen[a:b], dest[:, a:b])
         P.shadow_replay(ctx, rp, dk[a:b].contiguous(), dp[a:b].contiguous(), ds[a:b].contiguous(),
                         dd[:, a:b].contiguous(), ctr)
@@ -959,3 +995,20 @@ def test_replay_state_import_resumes(P, ctx):
         b.set_state(0, R, np.array([1], np.uint64))            # no such destination
     a.close()
     b.close()
+
+
+def test_debug_build_runs_the_smoke_check_clean():
+    # the bounds-checking build gives the oracle's results and raises no flag on a small
+    # pass of the whole path (run in a child process that loads the debug library)
+    import os
+    import subprocess
+    import sys
+    from paper_2608_19677_gb300 import buildlib
+    buildlib.build(debug=True)
+    root = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+    env = dict(os.environ, CR_DEBUG_LIB="1")
+    code = ("import paper_2608_19677_gb300 as P, __graft_entry__ as g; "
+            "assert P.LIB_PATH.endswith('libcacheroute_debug.so'); g.smoke()")
+    r = subprocess.run([sys.executable, "-c", code], cwd=root, env=env, capture_output=True, text=True, timeout=900)
+    assert r.returncode == 0, r.stdout[-2000:] + r.stderr[-2000:]
+    assert "smoke ok" in r.stdout
