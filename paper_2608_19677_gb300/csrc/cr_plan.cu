@@ -1222,8 +1222,13 @@ __global__ void __launch_bounds__(32) k_plan_lpt_reg(const __grid_constant__ lpt
     if (__any_sync(0xffffffffu, overflow) && lane == 0) atomicOr(status, CR_FLAG_OVERFLOW);
 }
 
-// RANDOM placement: one warp per admitted key; the first k steps of a
-// Fisher-Yates shuffle of 0..R-1 held in shared memory.
+// RANDOM placement: T(b) = the first k_b entries of a Fisher-Yates shuffle of
+// 0..R-1 (step s swaps position s with s + floor(u R_s / 2^64), R_s = R - s).
+// A key with k_b = 1 needs no array: its member is the first draw itself, so
+// every lane of a warp places one such key.  Keys with k_b > 1 are shuffled by
+// the warp's lane 0 over a shared-memory array that is never reset: an entry
+// counts only when its stamp equals the key being placed, otherwise position x
+// holds x.  Every key therefore costs O(k_b), not O(R).
 constexpr int kRandWarps = 4;
 
 __device__ __forceinline__ void random_body(const cr_plan_info_dev *info,
@@ -1237,34 +1242,56 @@ __device__ __forceinline__ void random_body(const cr_plan_info_dev *info,
                                                                  uint32_t *status, uint16_t *perm_all)
 {
     const uint32_t lane = cr_lane(), warp = threadIdx.x >> 5;
-    uint16_t *perm = perm_all + (size_t)warp * R;
+    const uint32_t Rp = (R + 1u) & ~1u;                                  // keeps the stamps 4-byte aligned
+    uint16_t *val = perm_all + (size_t)warp * Rp * 3;                  // [R] values of touched positions
+    uint32_t *stamp = reinterpret_cast<uint32_t *>(val + Rp);           // [R] key (+1) that touched each
+    for (uint32_t r = lane; r < R; r += 32) stamp[r] = 0;
+    __syncwarp();
     const unsigned long long na = info->n_adm;
     const unsigned long long nw = (unsigned long long)gridDim.x * kRandWarps;
-    for (unsigned long long a = (unsigned long long)blockIdx.x * kRandWarps + warp; a < na; a += nw) {
-        const uint32_t k = adm_k[a], base = koff[a];
-        const unsigned long long lam = adm_cnt[a];
-        const unsigned long long q = lam / k, rem = lam % k;
-        for (uint32_t r = lane; r < R; r += 32) perm[r] = (uint16_t)r;
-        __syncwarp();
-        if (lane == 0) {
-            for (uint32_t s = 0; s < k; ++s) {
-                cr_u64x4 u = cr_philox4x64_10(a, s, 1ull, epoch, seed, (unsigned long long)CR_POLICY_CR_NOLPT);
-                uint32_t t = s + cr_scale(u.x, (unsigned long long)(R - s));
-                uint16_t tmp = perm[s];
-                perm[s] = perm[t];
-                perm[t] = tmp;
+    for (unsigned long long a0 = ((unsigned long long)blockIdx.x * kRandWarps + warp) * 32; a0 < na; a0 += nw * 32) {
+        const unsigned long long a = a0 + lane;
+        const bool live = a < na;
+        const uint32_t k = live ? adm_k[a] : 0u;
+        if (live && k == 1) {
+            const cr_u64x4 u = cr_philox4x64_10(a, 0ull, 1ull, epoch, seed, (unsigned long long)CR_POLICY_CR_NOLPT);
+            const uint32_t m = cr_scale(u.x, (unsigned long long)R);
+            const unsigned long long lam = adm_cnt[a];
+            members[koff[a]] = (uint16_t)m;
+            jobs[koff[a]] = lam;
+            const unsigned long long old = atomicAdd(&load_g[m], lam);
+            if (old + lam >= kLoadLimit) atomicOr(status, CR_FLAG_OVERFLOW);
+        }
+        for (unsigned mk = __ballot_sync(0xffffffffu, live && k > 1); mk; mk &= mk - 1) {  // uniform
+            const uint32_t src = (uint32_t)__ffs(mk) - 1u;
+            const unsigned long long b = a0 + src;
+            const uint32_t kb = __shfl_sync(0xffffffffu, k, src), base = koff[b];
+            const unsigned long long lam = adm_cnt[b];
+            const unsigned long long q = lam / kb, rem = lam % kb;
+            const uint32_t tag = (uint32_t)b + 1u;
+            if (lane == 0) {
+                for (uint32_t s2 = 0; s2 < kb; ++s2) {
+                    const cr_u64x4 u = cr_philox4x64_10(b, s2, 1ull, epoch, seed, (unsigned long long)CR_POLICY_CR_NOLPT);
+                    const uint32_t t = s2 + cr_scale(u.x, (unsigned long long)(R - s2));
+                    const uint32_t vs = stamp[s2] == tag ? val[s2] : s2;
+                    const uint32_t vt = stamp[t] == tag ? val[t] : t;
+                    val[t] = (uint16_t)vs;
+                    stamp[t] = tag;
+                    val[s2] = (uint16_t)vt;
+                    stamp[s2] = tag;
+                    members[base + s2] = (uint16_t)vt;  // later steps only swap positions above s2
+                }
             }
+            __syncwarp();
+            for (uint32_t s2 = lane; s2 < kb; s2 += 32) {
+                const unsigned long long job = q + (s2 < rem ? 1ull : 0ull);
+                const uint32_t m = val[s2];
+                jobs[base + s2] = job;
+                const unsigned long long old = atomicAdd(&load_g[m], job);
+                if (old + job >= kLoadLimit) atomicOr(status, CR_FLAG_OVERFLOW);
+            }
+            __syncwarp();
         }
-        __syncwarp();
-        for (uint32_t s = lane; s < k; s += 32) {
-            const unsigned long long job = q + (s < rem ? 1ull : 0ull);
-            uint16_t m = perm[s];
-            members[base + s] = m;
-            jobs[base + s] = job;
-            unsigned long long old = atomicAdd(&load_g[m], job);
-            if (old + job >= kLoadLimit) atomicOr(status, CR_FLAG_OVERFLOW);
-        }
-        __syncwarp();
     }
 }
 
@@ -1632,11 +1659,11 @@ static int build_plans(cr_ctx *ctx, const uint64_t *d_key, uint64_t n, const cr_
         uint64_t radm = 0;
         auto flush_random = [&]() -> int {
             if (!nr) return CR_OK;
-            const size_t smem = (size_t)kRandWarps * rmaxR * sizeof(uint16_t);
+            const size_t smem = (size_t)kRandWarps * (rmaxR + 1) * 3 * sizeof(uint16_t);
             if (smem > 48 * 1024)
                 CR_CUDA(ctx, cudaFuncSetAttribute(k_plan_random_multi, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                                   (int)smem));
-            CR_LAUNCH(ctx, k_plan_random_multi, dim3(cr_blocks(radm, kRandWarps, gcap), nr), kRandWarps * 32, smem,
+            CR_LAUNCH(ctx, k_plan_random_multi, dim3(cr_blocks(radm, kRandWarps * 32, gcap), nr), kRandWarps * 32, smem,
                       rj, ctx->d_status);
             nr = 0;
             rmaxR = 0;
@@ -1766,12 +1793,12 @@ static int build_plans(cr_ctx *ctx, const uint64_t *d_key, uint64_t n, const cr_
                 CR_LAUNCH(ctx, k_plan_lpt_capped, 1, 32, smem, p->d_info, (const unsigned long long *)p->d_adm_cnt,
                           p->d_adm_k, p->d_koff, pp.R, pp.W, p->d_load, p->d_members, p->d_jobs, ctx->d_status);
             } else if (pp.variant == CR_VARIANT_RANDOM) {
-                size_t smem = (size_t)kRandWarps * pp.R * sizeof(uint16_t);
+                size_t smem = (size_t)kRandWarps * (pp.R + 1) * 3 * sizeof(uint16_t);
                 if (smem > 48 * 1024)
                     CR_CUDA(ctx, cudaFuncSetAttribute(k_plan_random, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                                       (int)smem));
                 uint64_t adm = n < C ? n : C;
-                CR_LAUNCH(ctx, k_plan_random, cr_blocks(adm, kRandWarps, gcap), kRandWarps * 32, smem,
+                CR_LAUNCH(ctx, k_plan_random, cr_blocks(adm, kRandWarps * 32, gcap), kRandWarps * 32, smem,
                           (const cr_plan_info_dev *)p->d_info, (const unsigned long long *)p->d_adm_cnt,
                           (const uint32_t *)p->d_adm_k, (const uint32_t *)p->d_koff, pp.R,
                           (unsigned long long)pp.seed, (unsigned long long)pp.epoch, p->d_load, p->d_members,
