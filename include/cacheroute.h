@@ -89,6 +89,7 @@ typedef struct cr_plan cr_plan;
 typedef struct cr_replay cr_replay;
 typedef struct cr_ring cr_ring;
 typedef struct cr_partition cr_partition;
+typedef struct cr_replay_input cr_replay_input;
 
 /* ==== context ============================================================ */
 
@@ -426,6 +427,28 @@ CR_API int cr_replay_destroy(cr_ctx *ctx, cr_replay *rp);
 CR_API int cr_shadow_replay(cr_ctx *ctx, cr_replay *rp, const uint64_t *d_key, const uint32_t *d_plen,
                      const uint32_t *d_slen, const uint16_t *d_dest, uint64_t n,
                      uint64_t *d_ctr);
+
+/*
+ * cr_shadow_replay in two calls, so that the partition (a8) of later requests
+ * can run on another stream while the simulators (a9), which must take the
+ * requests in arrival order, work through earlier ones:
+ *   cr_replay_partition  splits n routed requests (same arguments as
+ *       cr_shadow_replay) into every (replica, destination) stream in arrival
+ *       order, into a library-owned input object `in` (its device buffers grow on
+ *       demand; growing waits for the whole device).  Enqueued on ctx's stream.
+ *   cr_replay_simulate   runs the simulators of `rp` over `in` and accumulates
+ *       the counters exactly as cr_shadow_replay does.  Enqueued on ctx's stream,
+ *       which the caller orders after the partition (same stream, or an event)
+ *       and before any later partition into the same `in`.
+ * `in` must have been partitioned for a replay of the same n_rep, R and
+ * capacity kind.  cr_shadow_replay is exactly partition + simulate.  Errors:
+ * CR_EINVAL (shape mismatch, NULL pointers, n * n_rep >= 2^32 - 1), CR_ENOMEM,
+ * CR_ECUDA. */
+CR_API int cr_replay_input_create(cr_ctx *ctx, cr_replay_input **out);
+CR_API int cr_replay_input_destroy(cr_ctx *ctx, cr_replay_input *in);
+CR_API int cr_replay_partition(cr_ctx *ctx, const cr_replay *rp, const uint64_t *d_key, const uint32_t *d_plen,
+                               const uint32_t *d_slen, const uint16_t *d_dest, uint64_t n, cr_replay_input *in);
+CR_API int cr_replay_simulate(cr_ctx *ctx, cr_replay *rp, const cr_replay_input *in, uint64_t *d_ctr);
 
 /* Blocking: resident keys of one simulator at the largest capacity, most
  * recent first, into keys_out[CR_MAX_CAP] (host); *fill_out = their count.

@@ -41,7 +41,8 @@ EXPORTS = ("cr_create", "cr_destroy", "cr_set_stream", "cr_sync", "cr_last_error
            "cr_replay_destroy", "cr_shadow_replay", "cr_replay_export_state", "cr_key_histogram_noalloc",
            "cr_ring_create", "cr_ring_destroy", "cr_ring_export", "cr_plan_diff",
            "cr_replay_create_tokens", "cr_set_resolve_stream", "cr_partition_create", "cr_partition_destroy",
-           "cr_profile_enable", "cr_profile_read", "cr_plan_import", "cr_replay_import_state")
+           "cr_profile_enable", "cr_profile_read", "cr_plan_import", "cr_replay_import_state",
+           "cr_replay_input_create", "cr_replay_input_destroy", "cr_replay_partition", "cr_replay_simulate")
 PROF = {"hash": 0, "plan": 1, "route_cand": 2, "route_resolve": 3, "partition": 4, "replay": 5}
 CR_NOALLOC_MAX_KEYS = 65536
 
@@ -123,6 +124,10 @@ def lib() -> C.CDLL:
         "cr_partition_destroy": ([vp], i32),
         "cr_plan_import": ([vp, vp, u32, u32, u64, vp, vp, vp, vp, vp, vp], i32),
         "cr_replay_import_state": ([vp, vp, u32, u32, vp, u32], i32),
+        "cr_replay_input_create": ([vp, C.POINTER(vp)], i32),
+        "cr_replay_input_destroy": ([vp, vp], i32),
+        "cr_replay_partition": ([vp, vp, vp, vp, vp, vp, u64, vp], i32),
+        "cr_replay_simulate": ([vp, vp, vp, vp], i32),
         "cr_profile_enable": ([vp, u32], i32),
         "cr_profile_read": ([vp, u32, C.POINTER(C.c_uint64), C.POINTER(C.c_double)], i32),
     }
@@ -450,6 +455,52 @@ class Replay:
             self.close()
         except Exception:
             pass
+
+
+class ReplayInput:
+    """A partitioned batch of routed requests (cr_replay_partition), read by replay_simulate."""
+
+    def __init__(self, ctx: Context):
+        self.ctx = ctx
+        h = C.c_void_p()
+        ctx.check(lib().cr_replay_input_create(ctx.handle, C.byref(h)), "cr_replay_input_create")
+        self._h = h
+
+    @property
+    def handle(self):
+        return self._h
+
+    def close(self):
+        if getattr(self, "_h", None):
+            lib().cr_replay_input_destroy(self.ctx.handle, self._h)
+            self._h = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+
+def replay_partition(ctx: Context, replay: Replay, keys, plen, slen, dest, inp: ReplayInput):
+    """Partition routed requests for `replay` into `inp` (a8 alone), on ctx's stream."""
+    import torch
+    n = int(keys.shape[0])
+    _need_cuda("keys", keys, torch.int64)
+    _need_cuda("plen", plen, torch.int32)
+    _need_cuda("slen", slen, torch.int32)
+    _need_cuda("dest", dest, torch.int16)
+    ctx.check(lib().cr_replay_partition(ctx.handle, replay.handle, _ptr(keys), _ptr(plen), _ptr(slen), _ptr(dest),
+                                        n, inp.handle), "cr_replay_partition")
+    return inp
+
+
+def replay_simulate(ctx: Context, replay: Replay, inp: ReplayInput, ctr):
+    """Run the simulators over a partitioned input (a9 alone), accumulating into ``ctr``."""
+    import torch
+    _need_cuda("ctr", ctr, torch.int64)
+    ctx.check(lib().cr_replay_simulate(ctx.handle, replay.handle, inp.handle, _ptr(ctr)), "cr_replay_simulate")
+    return ctr
 
 
 def shadow_replay(ctx: Context, replay: Replay, keys, plen, slen, dest, ctr):

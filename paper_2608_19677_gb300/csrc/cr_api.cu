@@ -148,6 +148,7 @@ extern "C" int cr_destroy(cr_ctx *ctx)
     if (!ctx) return CR_OK;
     cudaStreamSynchronize(ctx->stream);
     prof_free(ctx);
+    cr_replay_input_destroy(nullptr, ctx->replay_in);
     if (ctx->resolve_stream) cudaStreamSynchronize(ctx->resolve_stream);
     if (ctx->ev_cand) cudaEventDestroy(ctx->ev_cand);
     if (ctx->ev_resolve) cudaEventDestroy(ctx->ev_resolve);

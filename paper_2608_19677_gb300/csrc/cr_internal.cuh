@@ -64,6 +64,7 @@ struct cr_prof {
 
 struct cr_ctx {
     cr_prof prof;
+    cr_replay_input *replay_in;  // partition of cr_shadow_replay (library-owned)
     int device;
     int num_sms;
     cudaStream_t stream;

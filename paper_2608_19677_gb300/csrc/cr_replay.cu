@@ -1263,31 +1263,103 @@ extern "C" int cr_replay_destroy(cr_ctx *ctx, cr_replay *rp)
     return CR_OK;
 }
 
-extern "C" int cr_shadow_replay(cr_ctx *ctx, cr_replay *rp, const uint64_t *d_key, const uint32_t *d_plen,
-                                const uint32_t *d_slen, const uint16_t *d_dest, uint64_t n, uint64_t *d_ctr)
+// ---- a8 / a9 as separate calls --------------------------------------------------
+// A partitioned input: every (replica, destination) stream's request indices in
+// arrival order, the packed records, the streams' starts and their chunking.
+struct cr_replay_input {
+    uint32_t n_rep, R, tokens;   // shape of the replay it was built for
+    uint32_t CL;                 // chunk length of the work items
+    uint64_t n, m;               // requests, (request, replica) pairs
+    uint32_t ns, ntiles;
+    uint32_t *d_idx;             // [m]
+    rec16 *d_recs;               // [n]
+    uint32_t *d_cnt;             // [ns * ntiles + 2]: tile counts -> offsets, and their total
+    uint32_t *d_start;           // [ns + 1]
+    uint32_t *d_coff;            // [ns + 2]: work-item offsets and their total
+    uint64_t cap_m, cap_n, cap_cnt, cap_ns;
+};
+
+static int grow_u32(cr_ctx *ctx, uint32_t **p, uint64_t *cap, uint64_t need)
 {
-    if (!ctx || !rp) return CR_EINVAL;
-    cr_nvtx_range nv("cr_shadow_replay");
-    if (n == 0) return CR_OK;
-    if (!d_key || !d_plen || !d_slen || !d_dest || !d_ctr)
-        return cr_fail(ctx, CR_EINVAL, "cr_shadow_replay: NULL pointer");
+    if (*cap >= need && *p) return CR_OK;
+    if (*p) {
+        // the old buffer may still be read by work on any stream (a simulation ordered after
+        // the partition by an event): wait for the whole device before freeing it
+        CR_CUDA(ctx, cudaDeviceSynchronize());
+        cudaFree(*p);
+        *p = nullptr;
+    }
+    const uint64_t c = need + need / 4 + 64;
+    if (cudaMalloc((void **)p, c * sizeof(uint32_t)) != cudaSuccess) {
+        cudaGetLastError();
+        *cap = 0;
+        return cr_fail(ctx, CR_ENOMEM, "replay input: cannot allocate %llu words", (unsigned long long)c);
+    }
+    *cap = c;
+    return CR_OK;
+}
+
+extern "C" int cr_replay_input_create(cr_ctx *ctx, cr_replay_input **out)
+{
+    if (!ctx || !out) return CR_EINVAL;
+    *out = (cr_replay_input *)calloc(1, sizeof(cr_replay_input));
+    return *out ? CR_OK : cr_fail(ctx, CR_ENOMEM, "replay input: host allocation failed");
+}
+
+extern "C" int cr_replay_input_destroy(cr_ctx *ctx, cr_replay_input *in)
+{
+    if (!in) return CR_OK;
+    if (ctx) cudaStreamSynchronize(ctx->stream);
+    cudaFree(in->d_idx);
+    cudaFree(in->d_recs);
+    cudaFree(in->d_cnt);
+    cudaFree(in->d_start);
+    cudaFree(in->d_coff);
+    free(in);
+    return CR_OK;
+}
+
+extern "C" int cr_replay_partition(cr_ctx *ctx, const cr_replay *rp, const uint64_t *d_key, const uint32_t *d_plen,
+                                   const uint32_t *d_slen, const uint16_t *d_dest, uint64_t n, cr_replay_input *in)
+{
+    if (!ctx || !rp || !in) return CR_EINVAL;
+    cr_nvtx_range nv("cr_replay_partition");
     const uint64_t m = n * rp->n_rep;
     if (n >= (1ull << 31) || m >= 0xffffffffull)
-        return cr_fail(ctx, CR_EINVAL, "cr_shadow_replay: n * n_rep must be < 2^32 - 1");
+        return cr_fail(ctx, CR_EINVAL, "cr_replay_partition: n * n_rep must be < 2^32 - 1");
+    if (n && (!d_key || !d_plen || !d_slen || !d_dest))
+        return cr_fail(ctx, CR_EINVAL, "cr_replay_partition: NULL pointer");
     const uint32_t R = rp->R, ns = (uint32_t)rp->n_streams;
     const uint32_t ntiles = (uint32_t)((n + kPartTile - 1) / kPartTile);
     const uint64_t ncnt = (uint64_t)ns * ntiles;
-    if (ncnt >= 0xffffffffull) return cr_fail(ctx, CR_EINVAL, "cr_shadow_replay: too many (stream, tile) pairs");
-    void *pk, *ps, *pidx, *pch, *precs;
-    CR_TRY(cr_scratch(ctx, SCR_REPLAY_IDX, (ncnt + 2) * sizeof(uint32_t), &pk));
-    CR_TRY(cr_scratch(ctx, SCR_REPLAY_START, ((size_t)ns + 1) * sizeof(uint32_t), &ps));
-    CR_TRY(cr_scratch(ctx, SCR_REPLAY_REC, m * sizeof(uint32_t), &pidx));
-    CR_TRY(cr_scratch(ctx, SCR_REPLAY_RECS, n * sizeof(rec16), &precs));
-    CR_TRY(cr_scratch(ctx, SCR_REPLAY_CHUNK, ((size_t)ns + 2) * sizeof(uint32_t), &pch));
-    uint32_t *cnt = (uint32_t *)pk, *nrec = cnt + ncnt, *start = (uint32_t *)ps;
-    uint32_t *idx = (uint32_t *)pidx;
-    rec16 *recs = (rec16 *)precs;
-    uint32_t *coff = (uint32_t *)pch, *total = coff + ns;
+    if (ncnt >= 0xffffffffull) return cr_fail(ctx, CR_EINVAL, "cr_replay_partition: too many (stream, tile) pairs");
+    in->n_rep = rp->n_rep;
+    in->R = R;
+    in->tokens = (uint32_t)rp->tokens;
+    in->n = n;
+    in->m = m;
+    in->ns = ns;
+    in->ntiles = ntiles;
+    if (rp->tokens) {
+        uint32_t capmax = 0;
+        for (uint32_t c = 0; c < rp->n_caps; ++c) capmax = rp->caps[c] > capmax ? rp->caps[c] : capmax;
+        // chunks long against the rebuild walk, which reaches back until the largest capacity fills
+        in->CL = capmax <= (1u << 16) ? 1024u : (capmax <= (1u << 17) ? 4096u : 16384u);
+    } else {
+        // long enough that rebuilding an LRU state of cmax entries is amortised
+        in->CL = rp->cmax * 16u > 256u ? rp->cmax * 16u : 256u;
+    }
+    if (n == 0) return CR_OK;
+    CR_TRY(grow_u32(ctx, &in->d_idx, &in->cap_m, m));
+    CR_TRY(grow_u32(ctx, (uint32_t **)&in->d_recs, &in->cap_n, n * (sizeof(rec16) / sizeof(uint32_t))));
+    CR_TRY(grow_u32(ctx, &in->d_cnt, &in->cap_cnt, ncnt + 2));
+    if (in->cap_ns < (uint64_t)ns + 2 || !in->d_start) {
+        uint64_t c0 = in->cap_ns;
+        CR_TRY(grow_u32(ctx, &in->d_start, &c0, (uint64_t)ns + 2));
+        CR_TRY(grow_u32(ctx, &in->d_coff, &in->cap_ns, (uint64_t)ns + 2));
+    }
+    uint32_t *cnt = in->d_cnt, *nrec = cnt + ncnt, *start = in->d_start;
+    uint32_t *coff = in->d_coff, *total = coff + ns;
     const unsigned int gcap = (unsigned int)ctx->num_sms * 8u;
     const dim3 pgrid(ntiles, rp->n_rep);
     const size_t csmem = (size_t)R * sizeof(uint32_t), ssmem = part_scatter_smem(R);
@@ -1297,26 +1369,37 @@ extern "C" int cr_shadow_replay(cr_ctx *ctx, cr_replay *rp, const uint64_t *d_ke
         CR_CUDA(ctx, cudaFuncSetAttribute(k_part_scatter, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)ssmem));
     const int pp = cr_prof_begin(ctx, ctx->stream, CR_PROF_PARTITION);
     CR_LAUNCH(ctx, k_part_records, cr_blocks(n, 256, gcap), 256, 0, (const unsigned long long *)d_key, d_plen, d_slen,
-              (unsigned long long)n, recs);
+              (unsigned long long)n, in->d_recs);
     CR_LAUNCH(ctx, k_part_count, pgrid, kPartBlock, csmem, d_dest, (unsigned long long)n, R, ntiles, cnt,
               ctx->d_status);
     CR_TRY(cr_scan_u32(ctx, cnt, cnt, ncnt, nrec));
     CR_LAUNCH(ctx, k_part_starts, cr_blocks((uint64_t)ns + 1, 256, gcap), 256, 0, (const uint32_t *)cnt, ns, ntiles,
               (const uint32_t *)nrec, start);
     CR_LAUNCH(ctx, k_part_scatter, pgrid, kPartBlock, ssmem, d_dest, (unsigned long long)n, R, ntiles,
-              (const uint32_t *)cnt, idx, (unsigned long long)m);
+              (const uint32_t *)cnt, in->d_idx, (unsigned long long)m);
+    CR_LAUNCH(ctx, k_chunk_counts, cr_blocks(ns, 256, gcap), 256, 0, (const uint32_t *)start, ns, in->CL, coff);
+    CR_TRY(cr_scan_u32(ctx, coff, coff, ns, total));
     cr_prof_end(ctx, ctx->stream, pp);
+    return CR_OK;
+}
+
+extern "C" int cr_replay_simulate(cr_ctx *ctx, cr_replay *rp, const cr_replay_input *in, uint64_t *d_ctr)
+{
+    if (!ctx || !rp || !in) return CR_EINVAL;
+    cr_nvtx_range nv("cr_replay_simulate");
+    if (in->n_rep != rp->n_rep || in->R != rp->R || in->tokens != (uint32_t)rp->tokens)
+        return cr_fail(ctx, CR_EINVAL, "cr_replay_simulate: the input was partitioned for another replay shape");
+    if (in->n == 0) return CR_OK;
+    if (!d_ctr) return cr_fail(ctx, CR_EINVAL, "cr_replay_simulate: d_ctr is NULL");
+    const uint32_t R = rp->R, ns = in->ns;
+    const uint64_t m = in->m, n = in->n;
+    const uint32_t *start = in->d_start, *coff = in->d_coff, *total = in->d_coff + ns;
     replay_caps caps;
     caps.n_caps = rp->n_caps;
     for (uint32_t c = 0; c < CR_MAX_CAPS; ++c) caps.cap[c] = c < rp->n_caps ? rp->caps[c] : 0;
     if (rp->tokens) {
         // token-weighted: one warp per (stream, chunk), its list in registers or shared memory
-        uint32_t capmax = 0;
-        for (uint32_t c = 0; c < rp->n_caps; ++c) capmax = rp->caps[c] > capmax ? rp->caps[c] : capmax;
-        // chunks long against the rebuild walk, which reaches back until the largest capacity fills
-        const uint32_t TCL = capmax <= (1u << 16) ? 1024u : (capmax <= (1u << 17) ? 4096u : 16384u);
-        CR_LAUNCH(ctx, k_chunk_counts, cr_blocks(ns, 256, gcap), 256, 0, (const uint32_t *)start, ns, TCL, coff);
-        CR_TRY(cr_scan_u32(ctx, coff, coff, ns, total));
+        const uint32_t TCL = in->CL;
         const size_t tsmem = (size_t)kTokWarps * kTokMax * (sizeof(unsigned long long) + sizeof(uint32_t));
         if (tsmem > 48 * 1024)
             CR_CUDA(ctx, cudaFuncSetAttribute(k_lru_tokens, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)tsmem));
@@ -1330,18 +1413,26 @@ extern "C" int cr_shadow_replay(cr_ctx *ctx, cr_replay *rp, const uint64_t *d_ke
         const uint64_t items = (uint64_t)ns + (m + TCL - 1) / TCL;  // upper bound on work items
         const int pt = cr_prof_begin(ctx, ctx->stream, CR_PROF_REPLAY);
         CR_LAUNCH(ctx, k_lru_tokens, (unsigned int)((items + kTokWarps - 1) / kTokWarps), kTokWarps * 32, tsmem,
-                  caps, ns, R, TCL, (const uint32_t *)start, (const uint32_t *)coff, (const uint32_t *)total,
-                  (const uint32_t *)idx, (const rec16 *)recs, (uint32_t)n, tst, (unsigned long long *)d_ctr,
-                  ctx->d_status);
+                  caps, ns, R, TCL, start, coff, total, (const uint32_t *)in->d_idx, (const rec16 *)in->d_recs,
+                  (uint32_t)n, tst, (unsigned long long *)d_ctr, ctx->d_status);
         cr_prof_end(ctx, ctx->stream, pt);
         rp->cur ^= 1;
         return CR_OK;
     }
-    // chunk length: long enough that rebuilding an LRU state of cmax entries is amortised
-    const uint32_t CL = rp->cmax * 16u > 256u ? rp->cmax * 16u : 256u;
-    CR_LAUNCH(ctx, k_chunk_counts, cr_blocks(ns, 256, gcap), 256, 0, (const uint32_t *)start, ns, CL, coff);
-    CR_TRY(cr_scan_u32(ctx, coff, coff, ns, total));
-    return launch_batch(ctx, rp, caps, CL, start, coff, total, m, idx, recs, d_ctr);
+    return launch_batch(ctx, rp, caps, in->CL, start, coff, total, m, in->d_idx, in->d_recs, d_ctr);
+}
+
+extern "C" int cr_shadow_replay(cr_ctx *ctx, cr_replay *rp, const uint64_t *d_key, const uint32_t *d_plen,
+                                const uint32_t *d_slen, const uint16_t *d_dest, uint64_t n, uint64_t *d_ctr)
+{
+    if (!ctx || !rp) return CR_EINVAL;
+    cr_nvtx_range nv("cr_shadow_replay");
+    if (n == 0) return CR_OK;
+    if (!d_key || !d_plen || !d_slen || !d_dest || !d_ctr)
+        return cr_fail(ctx, CR_EINVAL, "cr_shadow_replay: NULL pointer");
+    if (!ctx->replay_in) CR_TRY(cr_replay_input_create(ctx, &ctx->replay_in));
+    CR_TRY(cr_replay_partition(ctx, rp, d_key, d_plen, d_slen, d_dest, n, ctx->replay_in));
+    return cr_replay_simulate(ctx, rp, ctx->replay_in, d_ctr);
 }
 
 extern "C" int cr_replay_export_state(cr_ctx *ctx, const cr_replay *rp, uint32_t rep, uint32_t r,

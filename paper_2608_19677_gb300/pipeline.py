@@ -31,8 +31,8 @@ from __future__ import annotations
 
 from typing import Callable, List, Optional, Sequence, Tuple
 
-from . import (Context, Plan, Replay, Ring, build_plans, hash_prefixes, plan_params, route_batch,
-               set_resolve_stream, shadow_replay)
+from . import (Context, Plan, Replay, ReplayInput, Ring, build_plans, hash_prefixes, plan_params, replay_partition,
+               replay_simulate, route_batch, set_resolve_stream, shadow_replay)
 
 VARIANT_OF = {"CR": "LPT", "CR_NOLPT": "RANDOM", "CR_NOREPL": "NOREPL", "CR_SLOTCAP": "SLOTCAP"}
 # CacheRoute on a slot-capped plan routes as CacheRoute (same fallback draws as CR, seed for seed)
@@ -411,6 +411,7 @@ class TracePipeline:
         # (inputs and destinations, [replica][request of the group]) and replayed by one
         # call, which pays the per-stream setup of the replay once per group
         self.group = max(1, replay_group)
+        self.inputs = [ReplayInput(ctx) for _ in range(2)]  # partitioned groups, double-buffered
         self.gbuf = []
         if self.group > 1:
             G = self.group * max_n
@@ -460,7 +461,7 @@ class TracePipeline:
         start = self._event(self.mstream)
         for s in self.pstreams + self.rstreams + [self.ystream]:
             s.wait_event(start)
-        self.plan_marks, self.route_marks, self.replay_marks = [], [], []
+        self.plan_marks, self.route_marks, self.replay_marks, self.part_marks = [], [], [], []
         # replay groups: [g0, g1) intervals, their request count, and each interval's column
         sizes = [int(k.shape[0]) for k in keys]
         groups, col = [], [0] * T
@@ -517,37 +518,43 @@ class TracePipeline:
             self._plan_free[b] = routed
             if on_interval is not None:
                 on_interval(t, dest, self.plans[b] if self.plan_keys else [])
-            # ---- replay, in interval order ----------------------------------------------
-            if self.group == 1:
-                self.ystream.wait_event(routed)
-                y0 = self._event(self.ystream, True) if mark else None
-                shadow_replay(self.yctx, self.replay, keys[t], plens[t], slens[t], dest, self.ctr)
-                replayed = self._event(self.ystream, mark)
-                if mark:
-                    self.replay_marks.append((y0, replayed))
-                self._dest_free[b] = replayed
-                continue
+            # ---- replay: partition on the route stream, simulation in interval order ---------
+            # (the partition of later intervals runs while the simulators work through
+            # earlier ones; only the simulation carries state from interval to interval)
             gi = t // self.group
             g0, g1, N = groups[gi]
-            gk, gp, gs, gd = self.gbuf[gi % 2]
+            inp = self.inputs[gi % 2]
             if self._gfree[gi % 2] is not None:
-                rs.wait_event(self._gfree[gi % 2])   # the group before last has been replayed
-            with torch.cuda.stream(rs):  # stage the interval into the group buffer
-                c = col[t]
-                gk[c:c + n].copy_(keys[t])
-                gp[c:c + n].copy_(plens[t])
-                gs[c:c + n].copy_(slens[t])
-                gd[:len(self.replicas) * N].view(len(self.replicas), N)[:, c:c + n].copy_(dest)
+                rs.wait_event(self._gfree[gi % 2])   # the group before last has been simulated
+            if self.group == 1:
+                rk, rp_, rsl, rd = keys[t], plens[t], slens[t], dest
+            else:
+                gk, gp, gs, gd = self.gbuf[gi % 2]
+                with torch.cuda.stream(rs):  # stage the interval into the group buffer
+                    c = col[t]
+                    gk[c:c + n].copy_(keys[t])
+                    gp[c:c + n].copy_(plens[t])
+                    gs[c:c + n].copy_(slens[t])
+                    gd[:len(self.replicas) * N].view(len(self.replicas), N)[:, c:c + n].copy_(dest)
+                rk, rp_, rsl = gk[:N], gp[:N], gs[:N]
+                rd = gd[:len(self.replicas) * N].view(len(self.replicas), N)
             st_ev = self._event(rs)
             staged.append(st_ev)
-            self._dest_free[b] = st_ev
+            self._dest_free[b] = st_ev if self.group > 1 else None
             if t == g1 - 1:
-                for e in staged:
-                    self.ystream.wait_event(e)
+                for e in staged[:-1]:
+                    rs.wait_event(e)                 # the other intervals of the group are staged
                 staged = []
+                p0 = self._event(rs, True) if mark else None
+                replay_partition(rc, self.replay, rk, rp_, rsl, rd, inp)
+                parted = self._event(rs, mark)
+                if mark:
+                    self.part_marks.append((p0, parted))
+                if self.group == 1:
+                    self._dest_free[b] = parted
+                self.ystream.wait_event(parted)
                 y0 = self._event(self.ystream, True) if mark else None
-                shadow_replay(self.yctx, self.replay, gk[:N], gp[:N], gs[:N],
-                              gd[:len(self.replicas) * N].view(len(self.replicas), N), self.ctr)
+                replay_simulate(self.yctx, self.replay, inp, self.ctr)
                 replayed = self._event(self.ystream, mark)
                 if mark:
                     self.replay_marks.append((y0, replayed))
@@ -584,5 +591,7 @@ class TracePipeline:
         for g in self.rings:
             if g is not None:
                 g.close()
+        for i in self.inputs:
+            i.close()
         for c in self.pctxs + self.rctxs + [self.yctx]:
             c.close()

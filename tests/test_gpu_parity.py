@@ -1012,3 +1012,45 @@ def test_debug_build_runs_the_smoke_check_clean():
     r = subprocess.run([sys.executable, "-c", code], cwd=root, env=env, capture_output=True, text=True, timeout=900)
     assert r.returncode == 0, r.stdout[-2000:] + r.stderr[-2000:]
     assert "smoke ok" in r.stdout
+
+
+def test_replay_partition_then_simulate_equals_shadow_replay(P, ctx):
+    # the two-call form (partition on one stream, simulation on another, ordered by an
+    # event) gives the same counters and states as cr_shadow_replay, over two calls; an
+    # input partitioned for another replay shape is refused
+    rng = np.random.default_rng(17)
+    caps, n_rep, R = [16, 64], 3, 9
+    keys = _rates_keys(rng, 800, 24000)
+    n = keys.size
+    plen = rng.integers(16, 3000, size=n).astype(np.uint32)
+    slen = np.full(n, 64, np.uint32)
+    dest = tg.random_dest(n_rep, n, R, 4)
+    dk, dp, ds, dd = d_u64(keys), d_u32(plen), d_u32(slen), d_u16(dest)
+    a = P.Replay(ctx, n_rep, R, caps)
+    b = P.Replay(ctx, n_rep, R, caps)
+    ctr_a = torch.zeros((n_rep, len(caps), R, 5), dtype=torch.int64, device=DEV)
+    ctr_b = torch.zeros_like(ctr_a)
+    side = torch.cuda.Stream(DEV)
+    pctx = P.Context(0, side)
+    inp = P.ReplayInput(pctx)
+    cut = n // 2
+    for lo, hi in ((0, cut), (cut, n)):
+        args = (dk[lo:hi].contiguous(), dp[lo:hi].contiguous(), ds[lo:hi].contiguous(), dd[:, lo:hi].contiguous())
+        P.shadow_replay(ctx, a, *args, ctr_a)
+        side.wait_stream(torch.cuda.current_stream(DEV))
+        P.replay_partition(pctx, b, *args, inp)
+        ev = torch.cuda.Event()
+        ev.record(side)
+        torch.cuda.current_stream(DEV).wait_event(ev)
+        P.replay_simulate(ctx, b, inp, ctr_b)
+        ctx.sync()
+        pctx.sync()
+    assert (h_u64(ctr_a) == h_u64(ctr_b)).all()
+    for rep in range(n_rep):
+        for r in range(R):
+            assert (a.state(rep, r) == b.state(rep, r)).all()
+    other = P.Replay(ctx, n_rep, R + 1, caps)
+    with pytest.raises(P.CacheRouteError):
+        P.replay_simulate(ctx, other, inp, torch.zeros((n_rep, len(caps), R + 1, 5), dtype=torch.int64, device=DEV))
+    inp.close()
+    pctx.close()
