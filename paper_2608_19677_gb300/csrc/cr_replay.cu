@@ -58,31 +58,75 @@ constexpr int kPartPer = 32;                      // requests per thread
 constexpr int kPartTile = kPartBlock * kPartPer;  // 8192
 constexpr uint32_t kNoDest = 0xffffu;
 
+// Counts per warp in private u16 bins ([R][8], destination-major, as in
+// k_part_scatter): the leader of each group of equal destinations in a round
+// adds the group's size with a plain read-modify-write (no other lane touches
+// its warp's bins), then the 8 warps' bins are summed per destination.
 __global__ void __launch_bounds__(kPartBlock) k_part_count(const uint16_t *__restrict__ dest, unsigned long long n,
                                                            uint32_t R, uint32_t ntiles, uint32_t *__restrict__ cnt,
                                                            uint32_t *status)
 {
-    extern __shared__ uint32_t hist[];
-    const uint32_t rep = blockIdx.y, tile = blockIdx.x, lane = cr_lane();
-    for (uint32_t r = threadIdx.x; r < R; r += kPartBlock) hist[r] = 0;
+    extern __shared__ uint4 pcm[];
+    uint16_t *wc = reinterpret_cast<uint16_t *>(pcm);  // [R][8]
+    const uint32_t rep = blockIdx.y, tile = blockIdx.x, lane = cr_lane(), warp = threadIdx.x >> 5;
+    const uint32_t lt = (1u << lane) - 1u;
+    for (uint32_t r = threadIdx.x; r < R; r += kPartBlock) pcm[r] = make_uint4(0, 0, 0, 0);
     __syncthreads();
     const uint16_t *D = dest + (unsigned long long)rep * n;
     const unsigned long long base = (unsigned long long)tile * kPartTile;
+    const uint32_t cnt_t = (uint32_t)min((unsigned long long)kPartTile, n - base);
+    // counting needs no order: lane l of warp w takes the 32 consecutive items
+    // 1024 w + 32 l .. + 31, read up front with four 16-byte loads, one per round
+    constexpr uint32_t kPerWarp = kPartTile / kPartWarps;
+    const uint32_t first = warp * kPerWarp + lane * 32u;
+    uint32_t dv[16];  // two destinations per word
+    const bool whole = base + first + 32u <= n && ((base + first) & 7u) == 0 &&
+                       ((reinterpret_cast<uintptr_t>(D) & 15u) == 0);
+    if (whole) {
+        const uint4 *src = reinterpret_cast<const uint4 *>(D + base + first);
+#pragma unroll
+        for (int x = 0; x < 4; ++x) {
+            const uint4 v = src[x];
+            dv[4 * x] = v.x;
+            dv[4 * x + 1] = v.y;
+            dv[4 * x + 2] = v.z;
+            dv[4 * x + 3] = v.w;
+        }
+    } else {
+#pragma unroll
+        for (int x = 0; x < 16; ++x) {
+            const uint32_t i0 = first + 2u * x, i1 = i0 + 1u;
+            const uint32_t a = i0 < cnt_t ? D[base + i0] : kNoDest, c = i1 < cnt_t ? D[base + i1] : kNoDest;
+            dv[x] = a | (c << 16);
+        }
+    }
     bool bad = false;
-#pragma unroll 4
-    for (int j = 0; j < kPartPer; ++j) {
-        const unsigned long long i = base + (unsigned long long)j * kPartBlock + threadIdx.x;
-        uint32_t d = i < n ? D[i] : kNoDest;
-        if (i < n && d >= R) {
+#pragma unroll
+    for (uint32_t j = 0; j < (uint32_t)kPartPer; ++j) {
+        const uint32_t it = first + j;
+        uint32_t d = (dv[j >> 1] >> (16 * (j & 1))) & 0xffffu;
+        if (it >= cnt_t) d = kNoDest;
+        if (it < cnt_t && d >= R) {
             bad = true;
             d = kNoDest;  // skipped: reported through the status word
         }
         const uint32_t peers = __match_any_sync(0xffffffffu, d);
-        if (d != kNoDest && (peers & ((1u << lane) - 1u)) == 0) atomicAdd(&hist[d], (uint32_t)__popc(peers));
+        if (d != kNoDest && (peers & lt) == 0) {
+            uint16_t *c = &wc[d * kPartWarps + warp];
+            *c = (uint16_t)(*c + __popc(peers));
+        }
+        __syncwarp();
     }
     __syncthreads();
-    for (uint32_t r = threadIdx.x; r < R; r += kPartBlock)
-        cnt[((unsigned long long)rep * R + r) * ntiles + tile] = hist[r];
+    for (uint32_t r = threadIdx.x; r < R; r += kPartBlock) {
+        const uint4 v = pcm[r];
+        uint16_t c[8];
+        memcpy(c, &v, 16);
+        uint32_t t = 0;
+#pragma unroll
+        for (int w = 0; w < kPartWarps; ++w) t += c[w];
+        cnt[((unsigned long long)rep * R + r) * ntiles + tile] = t;
+    }
     if (__any_sync(0xffffffffu, bad) && lane == 0) atomicOr(status, CR_FLAG_BADDEST);
 }
 
@@ -124,10 +168,18 @@ __global__ void __launch_bounds__(kPartBlock) k_part_scatter(const uint16_t *__r
     const unsigned long long base = (unsigned long long)tile * kPartTile;
     const uint32_t cnt = (uint32_t)min((unsigned long long)kPartTile, n - base);
     // ranks: warp w takes items [1024 w, 1024 w + 1024) of the tile, 32 at a time
+    // (lane order is arrival order); all 32 rounds' destinations are read up front
     constexpr uint32_t kPerWarp = kPartTile / kPartWarps;
+    uint32_t dv[kPartPer / 2];
+#pragma unroll
+    for (int x = 0; x < kPartPer / 2; ++x) {
+        const uint32_t i0 = warp * kPerWarp + (2u * x) * 32u + lane, i1 = i0 + 32u;
+        const uint32_t a = i0 < cnt ? D[base + i0] : kNoDest, c = i1 < cnt ? D[base + i1] : kNoDest;
+        dv[x] = a | (c << 16);
+    }
     for (uint32_t j = 0; j < (uint32_t)kPartPer; ++j) {
         const uint32_t it = warp * kPerWarp + j * 32u + lane;
-        uint32_t d = it < cnt ? D[base + it] : kNoDest;
+        uint32_t d = (dv[j >> 1] >> (16 * (j & 1))) & 0xffffu;
         if (d >= R) d = kNoDest;
         const uint32_t peers = __match_any_sync(0xffffffffu, d);
         const uint32_t before = d != kNoDest ? wc[d * kPartWarps + warp] : 0u;
@@ -268,6 +320,7 @@ constexpr uint32_t kAbsent = 2047u;    // depth code of a key not resident (abov
 
 constexpr uint32_t kStash = 32;              // index entries that found both buckets full
 constexpr uint32_t kDegraded = 0x80000000u;  // stash overflowed: lookups scan the keys
+constexpr uint16_t kInStash = 0xffffu;       // TS of a slot whose entry is in the stash
 
 struct stamp_lru {
     unsigned long long *K;    // [cmax] key of each slot
@@ -278,6 +331,7 @@ struct stamp_lru {
     uint16_t *T2S;            // [32 nw] slot whose stamp is each time (where the bit is set)
     uint16_t *EV;             // [32] slots the step's evictions freed
     uint16_t *stash;          // [kStash] slot + 1 of keys indexed outside their buckets (0 = free)
+    uint16_t *TS;             // [cmax] where each slot's index entry is: bucket << 2 | entry, or kInStash
     uint32_t nbb;             // log2 of the bucket count
 };
 
@@ -291,7 +345,7 @@ __host__ __device__ inline size_t stamp_bkt_offset(uint32_t cmax, uint32_t nw)
 
 __host__ __device__ inline size_t stamp_lru_bytes(uint32_t cmax, uint32_t nw, uint32_t nbb)
 {
-    return (stamp_bkt_offset(cmax, nw) + ((size_t)8 << nbb) + (size_t)cmax * 2 + (size_t)nw * 64 + 64 +
+    return (stamp_bkt_offset(cmax, nw) + ((size_t)8 << nbb) + (size_t)cmax * 4 + (size_t)nw * 64 + 64 +
             (size_t)kStash * 2 + 15) &
            ~(size_t)15;
 }
@@ -307,6 +361,7 @@ __device__ __forceinline__ stamp_lru stamp_lru_at(unsigned char *base, uint32_t 
     X.T2S = X.ST + cmax;
     X.EV = X.T2S + (size_t)nw * 32;
     X.stash = X.EV + 32;
+    X.TS = X.stash + kStash;
     X.nbb = nbb;
     return X;
 }
@@ -396,8 +451,12 @@ __device__ __forceinline__ void sl_insert(const stamp_lru &X, unsigned long long
         } else {
             break;  // both buckets full
         }
-        if (atomicCAS(&X.bkt[b], w, w | (ent << (16 * p))) == w) return;
+        if (atomicCAS(&X.bkt[b], w, w | (ent << (16 * p))) == w) {
+            X.TS[q] = (uint16_t)((b << 2) | (uint32_t)p);
+            return;
+        }
     }
+    X.TS[q] = kInStash;
     const uint32_t i = atomicAdd(X.stash_n, 1u);
     if (i < kStash)
         X.stash[i] = (uint16_t)(q + 1u);
@@ -405,21 +464,13 @@ __device__ __forceinline__ void sl_insert(const stamp_lru &X, unsigned long long
         atomicOr(X.stash_n, kDegraded);
 }
 
-// Remove the index entry of slot q (key K[q]).
+// Remove the index entry of slot q: its place is recorded in TS[q].
 __device__ __forceinline__ void sl_erase(const stamp_lru &X, uint32_t q)
 {
-    const bkt_hash H = sl_hash(X.K[q], X.nbb);
-    const uint32_t ent = (H.tag << 11) | (q + 1u);
-#pragma unroll
-    for (int x = 0; x < 2; ++x) {
-        const uint32_t b = x ? H.b2 : H.b1;
-        const unsigned long long w = X.bkt[b];
-#pragma unroll
-        for (int p = 0; p < 4; ++p)
-            if (bkt_entry(w, p) == ent) {
-                atomicAnd(&X.bkt[b], ~(0xffffull << (16 * p)));
-                return;
-            }
+    const uint32_t loc = X.TS[q];
+    if (loc != kInStash) {
+        atomicAnd(&X.bkt[loc >> 2], ~(0xffffull << (16 * (loc & 3u))));
+        return;
     }
     const uint32_t sn = *X.stash_n & ~kDegraded;
     for (uint32_t i = 0; i < sn && i < kStash; ++i)
@@ -1362,7 +1413,7 @@ extern "C" int cr_replay_partition(cr_ctx *ctx, const cr_replay *rp, const uint6
     uint32_t *coff = in->d_coff, *total = coff + ns;
     const unsigned int gcap = (unsigned int)ctx->num_sms * 8u;
     const dim3 pgrid(ntiles, rp->n_rep);
-    const size_t csmem = (size_t)R * sizeof(uint32_t), ssmem = part_scatter_smem(R);
+    const size_t csmem = (size_t)R * kPartWarps * sizeof(uint16_t), ssmem = part_scatter_smem(R);
     if (csmem > 48 * 1024)
         CR_CUDA(ctx, cudaFuncSetAttribute(k_part_count, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)csmem));
     if (ssmem > 48 * 1024)
