@@ -106,6 +106,33 @@ def plan_stats(plan_ms):
             "builds_per_step": int(plan_ms.shape[1])}
 
 
+def isolated_plan_ms(pipe, keys, n_max: int = 8):
+    """Plan build timed alone on an otherwise idle device: for intervals 1..n_max, one
+    cr_build_plans call (every plan variant the replicas need, from the previous
+    interval's keys) between two events on the plan stream; median and max in ms."""
+    import torch
+    from paper_2608_19677_gb300 import build_plans, plan_params
+    if not pipe.plan_keys or len(keys) < 2:
+        return {"median": None, "max": None, "intervals": 0}
+    torch.cuda.synchronize()
+    ps, pc = pipe.pstreams[0], pipe.pctxs[0]
+    out = []
+    for t in range(1, min(len(keys), n_max + 1)):
+        pk = keys[t - 1]
+        num, den = pipe.qcap(int(pk.shape[0]))
+        params = [plan_params(pipe.R, pipe.W, num, den, v, seed=s, epoch=t) for v, s in pipe.plan_keys]
+        e0 = torch.cuda.Event(enable_timing=True)
+        e1 = torch.cuda.Event(enable_timing=True)
+        e0.record(ps)
+        build_plans(pc, pk, params, pipe.plans[0])
+        e1.record(ps)
+        e1.synchronize()
+        out.append(e0.elapsed_time(e1))
+    pc.sync()
+    return {"median": float(np.median(out)), "max": float(np.max(out)), "intervals": len(out),
+            "variants_per_build": len(pipe.plan_keys)}
+
+
 def workload_config(cfg, B, fresh=False):
     return {
         "workload": (f"{cfg.name}: {cfg.R} destinations, {cfg.total_keys} keys Zipf s={cfg.zipf_s}"
@@ -903,7 +930,7 @@ def run_keys_mode(args, cfg, trace, dev, stream, world, rank, barrier, resolve_s
     rr_rps = n_step / (ms_max / 1e3)
     rr_gbs = rr_bytes * rr_rps / 1e9
     # the dominant kernel of the step: the LRU simulation (a9), one launch per interval; its
-    # algorithmic bytes per launch are SURVEY 8(d)'s 20 per (request, replica, capacity)
+    # algorithmic bytes per launch are 20 per (request, replica, capacity): the replay's algorithmic count
     steps_profiled = 1 if graph is not None else args.steps
     req_per_launch = n_step * steps_profiled / max(kern["replay"]["launches"], 1)
     a9_bytes = 20.0 * reps * ncaps * req_per_launch
@@ -929,7 +956,7 @@ def run_keys_mode(args, cfg, trace, dev, stream, world, rank, barrier, resolve_s
                      "requests_per_launch": req_per_launch,
                      "algorithmic_bytes_per_launch_mean": a9_bytes, "avg_launch_ms": lru_ms,
                      "launches_timed": kern["replay"]["launches"],
-                     "note": "20 B per (request, replica, capacity) as SURVEY 8(d) counts a9; the kernel reads "
+                     "note": "20 B per (request, replica, capacity), the algorithmic bytes of the replay step; the kernel reads "
                              "one 16 B record per (request, replica) and decides every capacity from it; the "
                              "kernel is bound by the latency of its per-step dependence chain, not by bytes"},
         "hash_roofline": {"kernel": "k_hash_prefixes", "bound": "hbm", "achieved": hash_gbs, "peak": hbm_peak,
@@ -943,7 +970,8 @@ def run_keys_mode(args, cfg, trace, dev, stream, world, rank, barrier, resolve_s
                          "algorithmic_bytes_per_request": rr_bytes,
                          "achieved_GBps": rr_gbs, "hbm_frac": rr_gbs / hbm_peak},
         "hash_ms_per_pass": float(hms.sum()),
-        "plan_build_ms": plan_stats(plan_ms),
+        "plan_build_ms": dict(plan_stats(plan_ms), note="in the step, under contention with routes and replay",
+                              isolated=isolated_plan_ms(pipe, keys) if trace_mode else None),
         "main_wait_for_plans_ms_per_step": float((stage[:, :, 0] + stage[:, :, 1]).sum(1).mean()),
         "gpu_launches": int(n_launch), "clocks": clk,
     }
@@ -1126,7 +1154,7 @@ def run_resident_trace(args, cfg, trace, inputs, hash_bytes, dev, stream, world,
               "traffic": lru_traffic(a9_bytes, reps * req_per_launch) if not cfg.lru_tokens else None,
               "algorithmic_bytes_per_launch_mean": a9_bytes, "avg_launch_ms": lru_ms,
               "requests_per_launch": req_per_launch, "launches_timed": kern["replay"]["launches"],
-              "note": "20 B per (request, replica, capacity) as SURVEY 8(d) counts a9"}
+              "note": "20 B per (request, replica, capacity), the algorithmic bytes of the replay step"}
     # the roofline object names the kernel with the larger share of the step
     dom_lru = kern["replay"]["ms_per_step"] >= kern["hash"]["ms_per_step"]
     rr_bytes = 8 + 2 * reps + 6 * reps + 20 * reps * ncaps
@@ -1141,10 +1169,12 @@ def run_resident_trace(args, cfg, trace, inputs, hash_bytes, dev, stream, world,
         "roofline": lru_rf if dom_lru else hash_rf,
         ("hash_roofline" if dom_lru else "replay_roofline"): hash_rf if dom_lru else lru_rf,
         "kernels_ms_per_launch": kern,
+        "plan_build_ms": {"mean_in_step": kern["plan"]["avg_ms"],
+                          "isolated": isolated_plan_ms(pipe, keys)},
         "route_replay": {"algorithmic_bytes_per_request": rr_bytes,
                          "achieved_GBps": rr_bytes * n_step / (ms_max / 1e3) / 1e9,
                          "hbm_frac": rr_bytes * n_step / (ms_max / 1e3) / 1e9 / hbm_peak,
-                         "note": "SURVEY 8(d) route + replay bytes over the whole step (hashing and plans included "
+                         "note": "algorithmic route + replay bytes over the whole step (hashing and plans included "
                                  "in the time)"},
         "gpu_launches": int(n_launch), "clocks": clk,
     }

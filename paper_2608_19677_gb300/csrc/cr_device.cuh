@@ -90,3 +90,17 @@ __device__ __forceinline__ unsigned long long cr_warp_min_u64(unsigned long long
 }
 
 __device__ __forceinline__ uint32_t cr_lane() { return threadIdx.x & 31u; }
+
+// Lanes of the warp holding the same 64-bit key (every lane must call it).  The
+// lanes are grouped on a 32-bit fold of the key, and each group is checked
+// against its lowest lane's full key; only if some fold collided between
+// different keys (rare for hashed keys) is the 64-bit match taken.  A 64-bit
+// match costs several times the latency of a 32-bit one on this GPU.
+__device__ __forceinline__ uint32_t cr_match_u64(unsigned long long key)
+{
+    const uint32_t fold = (uint32_t)key ^ (uint32_t)(key >> 32);
+    const uint32_t grp = __match_any_sync(0xffffffffu, fold);
+    const unsigned long long lead = __shfl_sync(0xffffffffu, key, __ffs(grp) - 1);
+    if (__all_sync(0xffffffffu, lead == key)) return grp;
+    return __match_any_sync(0xffffffffu, key);
+}

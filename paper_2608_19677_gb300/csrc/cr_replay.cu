@@ -58,25 +58,20 @@ constexpr int kPartPer = 32;                      // requests per thread
 constexpr int kPartTile = kPartBlock * kPartPer;  // 8192
 constexpr uint32_t kNoDest = 0xffffu;
 
-// Counts per warp in private u16 bins ([R][8], destination-major, as in
-// k_part_scatter): the leader of each group of equal destinations in a round
-// adds the group's size with a plain read-modify-write (no other lane touches
-// its warp's bins), then the 8 warps' bins are summed per destination.
+// Counts of one tile in u32 bins [R], one shared-memory atomic add per item:
+// counting needs no order, so lane l of warp w takes the 32 consecutive items
+// 1024 w + 32 l .. + 31, read up front with four 16-byte loads.
 __global__ void __launch_bounds__(kPartBlock) k_part_count(const uint16_t *__restrict__ dest, unsigned long long n,
                                                            uint32_t R, uint32_t ntiles, uint32_t *__restrict__ cnt,
                                                            uint32_t *status)
 {
-    extern __shared__ uint4 pcm[];
-    uint16_t *wc = reinterpret_cast<uint16_t *>(pcm);  // [R][8]
+    extern __shared__ uint32_t pcb[];  // [R]
     const uint32_t rep = blockIdx.y, tile = blockIdx.x, lane = cr_lane(), warp = threadIdx.x >> 5;
-    const uint32_t lt = (1u << lane) - 1u;
-    for (uint32_t r = threadIdx.x; r < R; r += kPartBlock) pcm[r] = make_uint4(0, 0, 0, 0);
+    for (uint32_t r = threadIdx.x; r < R; r += kPartBlock) pcb[r] = 0;
     __syncthreads();
     const uint16_t *D = dest + (unsigned long long)rep * n;
     const unsigned long long base = (unsigned long long)tile * kPartTile;
     const uint32_t cnt_t = (uint32_t)min((unsigned long long)kPartTile, n - base);
-    // counting needs no order: lane l of warp w takes the 32 consecutive items
-    // 1024 w + 32 l .. + 31, read up front with four 16-byte loads, one per round
     constexpr uint32_t kPerWarp = kPartTile / kPartWarps;
     const uint32_t first = warp * kPerWarp + lane * 32u;
     uint32_t dv[16];  // two destinations per word
@@ -103,30 +98,16 @@ __global__ void __launch_bounds__(kPartBlock) k_part_count(const uint16_t *__res
     bool bad = false;
 #pragma unroll
     for (uint32_t j = 0; j < (uint32_t)kPartPer; ++j) {
-        const uint32_t it = first + j;
-        uint32_t d = (dv[j >> 1] >> (16 * (j & 1))) & 0xffffu;
-        if (it >= cnt_t) d = kNoDest;
-        if (it < cnt_t && d >= R) {
-            bad = true;
-            d = kNoDest;  // skipped: reported through the status word
+        const uint32_t d = (dv[j >> 1] >> (16 * (j & 1))) & 0xffffu;
+        if (first + j < cnt_t) {
+            if (d < R)
+                atomicAdd(&pcb[d], 1u);
+            else
+                bad = true;  // skipped: reported through the status word
         }
-        const uint32_t peers = __match_any_sync(0xffffffffu, d);
-        if (d != kNoDest && (peers & lt) == 0) {
-            uint16_t *c = &wc[d * kPartWarps + warp];
-            *c = (uint16_t)(*c + __popc(peers));
-        }
-        __syncwarp();
     }
     __syncthreads();
-    for (uint32_t r = threadIdx.x; r < R; r += kPartBlock) {
-        const uint4 v = pcm[r];
-        uint16_t c[8];
-        memcpy(c, &v, 16);
-        uint32_t t = 0;
-#pragma unroll
-        for (int w = 0; w < kPartWarps; ++w) t += c[w];
-        cnt[((unsigned long long)rep * R + r) * ntiles + tile] = t;
-    }
+    for (uint32_t r = threadIdx.x; r < R; r += kPartBlock) cnt[((unsigned long long)rep * R + r) * ntiles + tile] = pcb[r];
     if (__any_sync(0xffffffffu, bad) && lane == 0) atomicOr(status, CR_FLAG_BADDEST);
 }
 
@@ -138,7 +119,7 @@ __global__ void k_part_starts(const uint32_t *__restrict__ off, uint32_t ns, uin
         start[s] = s < ns ? off[(unsigned long long)s * ntiles] : *total;
 }
 
-// Shared memory of k_part_scatter: per-warp counters wc[R][8] (u16), the
+// Shared memory of k_part_scatter: per-warp counters wc[8][R] (u16), the
 // tile's destination offsets toff[R] (u32), each item's (destination << 16 |
 // rank among its warp's items of that destination) (u32), and the tile's items
 // in (destination, arrival) order (u16 item numbers).
@@ -153,7 +134,7 @@ __global__ void __launch_bounds__(kPartBlock) k_part_scatter(const uint16_t *__r
                                                              uint32_t *__restrict__ out, unsigned long long m)
 {
     extern __shared__ uint4 psm[];
-    uint16_t *wc = reinterpret_cast<uint16_t *>(psm);                            // [R][8]
+    uint16_t *wc = reinterpret_cast<uint16_t *>(psm);                            // [8][R]
     uint32_t *toff = reinterpret_cast<uint32_t *>(wc + (size_t)R * kPartWarps);  // [R]
     uint32_t *spk = toff + R;                                                    // [kPartTile]
     uint16_t *sitem = reinterpret_cast<uint16_t *>(spk + kPartTile);            // [kPartTile]
@@ -168,8 +149,12 @@ __global__ void __launch_bounds__(kPartBlock) k_part_scatter(const uint16_t *__r
     const unsigned long long base = (unsigned long long)tile * kPartTile;
     const uint32_t cnt = (uint32_t)min((unsigned long long)kPartTile, n - base);
     // ranks: warp w takes items [1024 w, 1024 w + 1024) of the tile, 32 at a time
-    // (lane order is arrival order); all 32 rounds' destinations are read up front
+    // (lane order is arrival order); all 32 rounds' destinations are read up front.
+    // The lanes of a round with equal destinations are found from one ballot per
+    // bit of the destination (R stands for "no item").
     constexpr uint32_t kPerWarp = kPartTile / kPartWarps;
+    const uint32_t nb = 32u - (uint32_t)__clz(R);
+    uint16_t *wcw = wc + (size_t)warp * R;
     uint32_t dv[kPartPer / 2];
 #pragma unroll
     for (int x = 0; x < kPartPer / 2; ++x) {
@@ -177,15 +162,22 @@ __global__ void __launch_bounds__(kPartBlock) k_part_scatter(const uint16_t *__r
         const uint32_t a = i0 < cnt ? D[base + i0] : kNoDest, c = i1 < cnt ? D[base + i1] : kNoDest;
         dv[x] = a | (c << 16);
     }
+#pragma unroll
     for (uint32_t j = 0; j < (uint32_t)kPartPer; ++j) {
         const uint32_t it = warp * kPerWarp + j * 32u + lane;
         uint32_t d = (dv[j >> 1] >> (16 * (j & 1))) & 0xffffu;
+        const uint32_t dd = d < R ? d : R;
         if (d >= R) d = kNoDest;
-        const uint32_t peers = __match_any_sync(0xffffffffu, d);
-        const uint32_t before = d != kNoDest ? wc[d * kPartWarps + warp] : 0u;
+        uint32_t peers = 0xffffffffu;
+        for (uint32_t bt = 0; bt < nb; ++bt) {
+            const uint32_t bit = (dd >> bt) & 1u;
+            const uint32_t B = __ballot_sync(0xffffffffu, bit);
+            peers &= bit ? B : ~B;
+        }
+        const uint32_t before = d != kNoDest ? wcw[d] : 0u;
         spk[it] = (d << 16) | (before + (uint32_t)__popc(peers & lt));
         __syncwarp();
-        if (d != kNoDest && (peers & lt) == 0) wc[d * kPartWarps + warp] = (uint16_t)(before + __popc(peers));
+        if (d != kNoDest && (peers & lt) == 0) wcw[d] = (uint16_t)(before + __popc(peers));
         __syncwarp();
     }
     __syncthreads();
@@ -194,18 +186,13 @@ __global__ void __launch_bounds__(kPartBlock) k_part_scatter(const uint16_t *__r
     const uint32_t per = (R + kPartBlock - 1) / kPartBlock, r0 = threadIdx.x * per;
     uint32_t run = 0;
     for (uint32_t r = r0; r < r0 + per && r < R; ++r) {
-        uint4 v = wc4[r];
-        uint16_t c[8];
-        memcpy(c, &v, 16);
         uint16_t acc = 0;
 #pragma unroll
         for (int w = 0; w < kPartWarps; ++w) {
-            const uint16_t x = c[w];
-            c[w] = acc;
+            const uint16_t x = wc[(size_t)w * R + r];
+            wc[(size_t)w * R + r] = acc;
             acc = (uint16_t)(acc + x);
         }
-        memcpy(&v, c, 16);
-        wc4[r] = v;
         toff[r] = acc;  // the destination's total until the scan below
         run += acc;
     }
@@ -241,18 +228,23 @@ __global__ void __launch_bounds__(kPartBlock) k_part_scatter(const uint16_t *__r
         const uint32_t pk = spk[it];
         const uint32_t d = pk >> 16;
         if (d == kNoDest) continue;
-        const uint32_t pos = toff[d] + wc[d * kPartWarps + it / kPerWarp] + (pk & 0xffffu);
+        const uint32_t pos = toff[d] + wc[(size_t)(it / kPerWarp) * R + d] + (pk & 0xffffu);
         sitem[pos] = (uint16_t)it;
     }
+    // each destination's output position minus its staging position (mod 2^32), in
+    // the counters' space, which the staging no longer needs
+    uint32_t *gb = reinterpret_cast<uint32_t *>(wc);  // [R]
+    const uint32_t *O = off + (unsigned long long)rep * R * ntiles;
+    __syncthreads();
+    for (uint32_t r = threadIdx.x; r < R; r += kPartBlock) gb[r] = O[(unsigned long long)r * ntiles + tile] - toff[r];
     __syncthreads();
     // output: consecutive threads write consecutive positions of each destination's run
     const uint32_t valid = s_valid;
-    const uint32_t *O = off + (unsigned long long)rep * R * ntiles;
     for (uint32_t j = threadIdx.x; j < valid; j += kPartBlock) {
         const uint32_t it = sitem[j];
         const uint32_t d = spk[it] >> 16;
-        if (d >= R || j < toff[d]) continue;  // never: every staged item is valid (guards the writes)
-        const unsigned long long o = (unsigned long long)O[(unsigned long long)d * ntiles + tile] + (j - toff[d]);
+        if (d >= R) continue;  // never: every staged item is valid (guards the writes)
+        const uint32_t o = gb[d] + j;
         if (o < m) out[o] = (uint32_t)(base + it);
     }
 }
@@ -269,6 +261,15 @@ __global__ void k_part_records(const unsigned long long *__restrict__ keys, cons
         r.S = slen[i];
         recs[i] = r;
     }
+}
+
+// The stream of every work item: items coff[s] .. coff[s + 1] - 1 belong to stream s
+// (coff[ns] is the total), written at wmap[item].
+__global__ void k_item_streams(const uint32_t *__restrict__ coff, uint32_t ns, uint32_t *__restrict__ wmap,
+                               uint64_t items_max)
+{
+    for (uint32_t s = blockIdx.x * blockDim.x + threadIdx.x; s < ns; s += gridDim.x * blockDim.x)
+        for (uint32_t w = coff[s]; w < coff[s + 1] && w < items_max; ++w) wmap[w] = s;
 }
 
 // Chunks per stream (an empty stream still gets one work item that carries its state over).
@@ -600,15 +601,7 @@ k_lru_stamp(const replay_caps caps, uint32_t cmax, uint32_t nw, uint32_t R, uint
 
     const uint32_t w = blockIdx.x * wpb + warp;
     if (w >= *total) return;
-    uint32_t lo_s = 0, hi_s = ns;
-    while (hi_s - lo_s > 1) {
-        const uint32_t mid = (lo_s + hi_s) >> 1;
-        if (coff[mid] <= w)
-            lo_s = mid;
-        else
-            hi_s = mid;
-    }
-    const uint32_t s = lo_s, ci = w - coff[s];
+    const uint32_t s = min(coff[ns + 2 + w], ns - 1u), ci = w - coff[s];  // the item's stream and chunk
     const uint32_t b = start[s], e = start[s + 1];
     const uint32_t p0 = b + ci * CL;
     const uint32_t p1 = (e - p0) < CL ? e : p0 + CL;
@@ -628,10 +621,24 @@ k_lru_stamp(const replay_caps caps, uint32_t cmax, uint32_t nw, uint32_t R, uint
     uint32_t fill = 0;
     sl_reindex(X, 0, lane);
     if (ci == 0) {
-        for (uint32_t q = lane; q < fill_in; q += 32) X.K[q] = kin[q];
+        // the carried-in keys, eight loads in flight per lane
+        for (uint32_t q0 = 0; q0 < fill_in; q0 += 256) {
+            unsigned long long kk[8];
+#pragma unroll
+            for (uint32_t x = 0; x < 8; ++x) {
+                const uint32_t q = q0 + 32u * x + lane;
+                kk[x] = q < fill_in ? kin[q] : 0ull;
+            }
+#pragma unroll
+            for (uint32_t x = 0; x < 8; ++x) {
+                const uint32_t q = q0 + 32u * x + lane;
+                if (q < fill_in) {
+                    X.K[q] = kk[x];
+                    sl_insert(X, kk[x], q);
+                }
+            }
+        }
         fill = fill_in;
-        __syncwarp();
-        for (uint32_t q = lane; q < fill; q += 32) sl_insert(X, X.K[q], q);
     } else {
         // walk backwards collecting distinct keys, most recent first
         const uint32_t back = p0 - b;
@@ -664,21 +671,24 @@ k_lru_stamp(const replay_caps caps, uint32_t cmax, uint32_t nw, uint32_t R, uint
 #pragma unroll
     for (int c = 0; c < NC; ++c) my_hit[c] = my_tok[c] = 0;
 
-    rec16 ahead = {0ull, 0u, 0u};  // the next step's records, loaded one step early
+    // the next step's records are gathered one step early, through request
+    // indices read two steps early
+    rec16 ahead = {0ull, 0u, 0u};
     if (p0 + lane < p1) {
         const uint32_t ix = idx[p0 + lane];
-        CR_DCHECK(ix < nrec, status);
+        (void)CR_DCHECK(ix < nrec, status);
         ahead = recs[min(ix, nrec - 1u)];  // (the bound guards the gather)
     }
+    uint32_t ix_next = p0 + 32u + lane < p1 ? idx[p0 + 32u + lane] : 0u;
     for (uint32_t t0 = p0; t0 < p1; t0 += 32) {
         const uint32_t cnt = (p1 - t0) < 32u ? (p1 - t0) : 32u;
         const bool valid = lane < cnt;
         const rec16 mine = ahead;
         if (t0 + 32u + lane < p1) {
-            const uint32_t ix = idx[t0 + 32u + lane];
-            CR_DCHECK(ix < nrec, status);
-            ahead = recs[min(ix, nrec - 1u)];
+            (void)CR_DCHECK(ix_next < nrec, status);
+            ahead = recs[min(ix_next, nrec - 1u)];
         }
+        ix_next = t0 + 64u + lane < p1 ? idx[t0 + 64u + lane] : 0u;
         if (valid) {
             my_req += 1;
             my_prompt += (unsigned long long)mine.P + mine.S;
@@ -992,15 +1002,7 @@ __global__ void __launch_bounds__(kTokWarps * 32) k_lru_tokens(const __grid_cons
     const uint32_t wi = blockIdx.x * kTokWarps + w;
     if (wi >= *total) return;  // whole warps only; the kernel has no block-wide barrier
     // work item -> (stream, chunk)
-    uint32_t lo_s = 0, hi_s = ns;
-    while (hi_s - lo_s > 1) {
-        const uint32_t mid = (lo_s + hi_s) >> 1;
-        if (coff[mid] <= wi)
-            lo_s = mid;
-        else
-            hi_s = mid;
-    }
-    const uint32_t s = lo_s, ci = wi - coff[s];
+    const uint32_t s = min(coff[ns + 2 + wi], ns - 1u), ci = wi - coff[s];
     const uint32_t b = start[s], e = start[s + 1];
     unsigned long long *K = tok_sh + (size_t)w * kTokMax;
     uint32_t *Cm = reinterpret_cast<uint32_t *>(tok_sh + (size_t)kTokWarps * kTokMax) + (size_t)w * kTokMax;
@@ -1326,8 +1328,8 @@ struct cr_replay_input {
     rec16 *d_recs;               // [n]
     uint32_t *d_cnt;             // [ns * ntiles + 2]: tile counts -> offsets, and their total
     uint32_t *d_start;           // [ns + 1]
-    uint32_t *d_coff;            // [ns + 2]: work-item offsets and their total
-    uint64_t cap_m, cap_n, cap_cnt, cap_ns;
+    uint32_t *d_coff;            // [ns + 2 + items]: work-item offsets, their total, then each item's stream
+    uint64_t cap_m, cap_n, cap_cnt, cap_ns, cap_coff;
 };
 
 static int grow_u32(cr_ctx *ctx, uint32_t **p, uint64_t *cap, uint64_t need)
@@ -1404,16 +1406,14 @@ extern "C" int cr_replay_partition(cr_ctx *ctx, const cr_replay *rp, const uint6
     CR_TRY(grow_u32(ctx, &in->d_idx, &in->cap_m, m));
     CR_TRY(grow_u32(ctx, (uint32_t **)&in->d_recs, &in->cap_n, n * (sizeof(rec16) / sizeof(uint32_t))));
     CR_TRY(grow_u32(ctx, &in->d_cnt, &in->cap_cnt, ncnt + 2));
-    if (in->cap_ns < (uint64_t)ns + 2 || !in->d_start) {
-        uint64_t c0 = in->cap_ns;
-        CR_TRY(grow_u32(ctx, &in->d_start, &c0, (uint64_t)ns + 2));
-        CR_TRY(grow_u32(ctx, &in->d_coff, &in->cap_ns, (uint64_t)ns + 2));
-    }
+    CR_TRY(grow_u32(ctx, &in->d_start, &in->cap_ns, (uint64_t)ns + 2));
+    const uint64_t items_max = (uint64_t)ns + m / in->CL + 1;  // every stream's chunks, at least one each
+    CR_TRY(grow_u32(ctx, &in->d_coff, &in->cap_coff, (uint64_t)ns + 2 + items_max));
     uint32_t *cnt = in->d_cnt, *nrec = cnt + ncnt, *start = in->d_start;
     uint32_t *coff = in->d_coff, *total = coff + ns;
     const unsigned int gcap = (unsigned int)ctx->num_sms * 8u;
     const dim3 pgrid(ntiles, rp->n_rep);
-    const size_t csmem = (size_t)R * kPartWarps * sizeof(uint16_t), ssmem = part_scatter_smem(R);
+    const size_t csmem = (size_t)R * sizeof(uint32_t), ssmem = part_scatter_smem(R);
     if (csmem > 48 * 1024)
         CR_CUDA(ctx, cudaFuncSetAttribute(k_part_count, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)csmem));
     if (ssmem > 48 * 1024)
@@ -1430,6 +1430,8 @@ extern "C" int cr_replay_partition(cr_ctx *ctx, const cr_replay *rp, const uint6
               (const uint32_t *)cnt, in->d_idx, (unsigned long long)m);
     CR_LAUNCH(ctx, k_chunk_counts, cr_blocks(ns, 256, gcap), 256, 0, (const uint32_t *)start, ns, in->CL, coff);
     CR_TRY(cr_scan_u32(ctx, coff, coff, ns, total));
+    CR_LAUNCH(ctx, k_item_streams, cr_blocks(ns, 256, gcap), 256, 0, (const uint32_t *)coff, ns, coff + ns + 2,
+              items_max);
     cr_prof_end(ctx, ctx->stream, pp);
     return CR_OK;
 }

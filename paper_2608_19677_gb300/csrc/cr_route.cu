@@ -96,36 +96,55 @@ __device__ __forceinline__ unsigned long long chwbl_cap(unsigned long long m, ui
     return (5ull * (m + 1ull) + den - 1ull) / den;
 }
 
-// Everything that does not depend on the live load, for every (replica, request).
+// Everything that does not depend on the live load, for every (replica, request):
+// blockIdx.y is the replica, so every block runs one policy's loop.
 // Load-independent replicas (RR, HASH) write their destinations directly.
 __global__ void __launch_bounds__(256) k_route_cand(const __grid_constant__ route_args args, uint32_t n_rep,
                                                     const unsigned long long *__restrict__ keys,
                                                     unsigned long long n, unsigned long long g0, uint32_t R,
                                                     uint32_t *__restrict__ cand, uint16_t *__restrict__ dest)
 {
-    const unsigned long long total = n * n_rep;
-    for (unsigned long long j = (unsigned long long)blockIdx.x * blockDim.x + threadIdx.x; j < total;
-         j += (unsigned long long)gridDim.x * blockDim.x) {
-        const uint32_t rep = (uint32_t)(j / n);
-        const unsigned long long i = j - (unsigned long long)rep * n;
-        const route_desc &rd = args.d[rep];
-        const unsigned long long g = g0 + i;
-        switch (rd.policy) {
-        case CR_POLICY_RR:
-            dest[j] = (uint16_t)((g + rd.seed) % R);
-            break;
-        case CR_POLICY_HASH:
-            dest[j] = (uint16_t)cr_jump_hash(cr_fmix64(keys[i] ^ rd.seed), R);
-            break;
-        case CR_POLICY_P2C:
-            cand[j] = p2c_pair(rd.seed, rd.policy, g, R);
-            break;
-        case CR_POLICY_CHWBL:
-            cand[j] = kRing | ring_start(rd, cr_fmix64(keys[i] ^ rd.seed));
-            break;
-        default: {
+    const uint32_t rep = blockIdx.y;
+    if (rep >= n_rep) return;
+    const route_desc &rd = args.d[rep];
+    uint32_t *C = cand + (unsigned long long)rep * n;
+    uint16_t *Dst = dest + (unsigned long long)rep * n;
+    const unsigned long long stride = (unsigned long long)gridDim.x * blockDim.x;
+    const unsigned long long i0 = (unsigned long long)blockIdx.x * blockDim.x + threadIdx.x;
+    switch (rd.policy) {
+    case CR_POLICY_RR: {
+        // (g0 + i + seed) mod 2^64 mod R.  Until the sum wraps (i < wrap) that is
+        // (base mod R + i mod R) mod R, which needs only 32-bit remainders while i < 2^32.
+        const unsigned long long base = g0 + rd.seed;
+        const unsigned long long wrap = base ? 0ull - base : ~0ull;
+        const uint32_t b0 = (uint32_t)(base % R);
+        for (unsigned long long i = i0; i < n; i += stride) {
+            uint32_t r;
+            if (i < wrap && i < (1ull << 32)) {
+                r = b0 + (uint32_t)i % R;
+                if (r >= R) r -= R;
+            } else {
+                r = (uint32_t)((base + i) % R);
+            }
+            Dst[i] = (uint16_t)r;
+        }
+        break;
+    }
+    case CR_POLICY_HASH:
+        for (unsigned long long i = i0; i < n; i += stride)
+            Dst[i] = (uint16_t)cr_jump_hash(cr_fmix64(keys[i] ^ rd.seed), R);
+        break;
+    case CR_POLICY_P2C:
+        for (unsigned long long i = i0; i < n; i += stride) C[i] = p2c_pair(rd.seed, rd.policy, g0 + i, R);
+        break;
+    case CR_POLICY_CHWBL:
+        for (unsigned long long i = i0; i < n; i += stride)
+            C[i] = kRing | ring_start(rd, cr_fmix64(keys[i] ^ rd.seed));
+        break;
+    default: {
+        const unsigned long long mask = (1ull << rd.tbits) - 1ull;
+        for (unsigned long long i = i0; i < n; i += stride) {
             const unsigned long long key = keys[i];
-            const unsigned long long mask = (1ull << rd.tbits) - 1ull;
             unsigned long long sl = key >> (64 - rd.tbits);
             uint32_t c = 0xffffffffu;
             for (;;) {
@@ -137,9 +156,9 @@ __global__ void __launch_bounds__(256) k_route_cand(const __grid_constant__ rout
                 }
                 sl = (sl + 1) & mask;
             }
-            cand[j] = c != 0xffffffffu ? c : p2c_pair(rd.seed, rd.policy, g, R);
+            C[i] = c != 0xffffffffu ? c : p2c_pair(rd.seed, rd.policy, g0 + i, R);
         }
-        }
+    }
     }
 }
 
@@ -690,7 +709,8 @@ extern "C" int cr_route_batch(cr_ctx *ctx, const cr_plan *const *plans, const cr
     uint32_t *cand = (uint32_t *)pc;
     const unsigned int gcap = (unsigned int)ctx->num_sms * 16u;
     const int pcand = cr_prof_begin(ctx, ctx->stream, CR_PROF_ROUTE_CAND);
-    CR_LAUNCH(ctx, k_route_cand, cr_blocks(n * n_rep, 256, gcap), 256, 0, args, n_rep,
+    const dim3 cgrid(cr_blocks(n, 256, std::max(1u, gcap / n_rep)), n_rep);
+    CR_LAUNCH(ctx, k_route_cand, cgrid, 256, 0, args, n_rep,
               (const unsigned long long *)d_key, (unsigned long long)n, (unsigned long long)first_req_index, R, cand,
               d_dest);
     cr_prof_end(ctx, ctx->stream, pcand);

@@ -295,6 +295,23 @@ def test_route_parity(P, ctx, R, B):
     assert (h_u64(load) == ref_load).all()
 
 
+@pytest.mark.parametrize("R", [1, 30, 1024, 8191])
+@pytest.mark.parametrize("g0,seed", [(0, 2**64 - 1000), (2**40 + 3, 2**64 - 2**40 - 2500), (2**33, 7), (0, 0)])
+def test_route_rr_hash_index_edges(P, ctx, R, g0, seed):
+    # round robin is (g0 + i + seed) mod 2^64 mod R: the sum wraps inside the call for the
+    # first two seeds, and request indices start above 2^32 for the second and third
+    rng = np.random.default_rng(R)
+    keys = rng.integers(0, 2**63, 5000, dtype=np.int64).astype(np.uint64)
+    pols, seeds = ["RR", "HASH", "P2C"], [seed, seed ^ 5, seed]
+    ref_dest, ref_load = O.route([None] * 3, pols, seeds, R, keys, g0, 1024)
+    load = torch.zeros((3, R), dtype=torch.int64, device=DEV)
+    dest = P.route_batch(ctx, [None] * 3, pols, seeds, R, d_u64(keys), g0, 1024, load)
+    ctx.sync()
+    for i, p in enumerate(pols):
+        assert (h_u16(dest[i]) == ref_dest[i]).all(), p
+    assert (h_u64(load) == ref_load).all()
+
+
 @pytest.mark.parametrize("R,V,seed", [(1, 1, 0), (3, 1, 0), (7, 5, 123), (1024, 64, 9), (8192, 16, 2**64 - 1),
                                       (5, 1024, 77)])
 def test_ring_parity(P, ctx, R, V, seed):
