@@ -48,10 +48,13 @@ __device__ __forceinline__ uint32_t cr_scale(unsigned long long u, unsigned long
 
 // Jump consistent hash (Lamping and Veach 2014) with the jump evaluated exactly
 // in integers: j = floor((b + 1) * 2^31 / d), d = (k >> 33) + 1 in [1, 2^31].
-// No 64-bit division: a single-precision estimate of the quotient (relative
-// error below 2^-21) settles j >= R whenever it exceeds R + 2; otherwise it is
-// at most R + 2 <= 8194, its error is below 0.01, and one integer step either
-// way (products below 2^46) gives the exact floor.
+// No 64-bit division: a single-precision estimate of the quotient settles
+// j >= R whenever it exceeds R + 2; otherwise it is at most R + 2 <= 8194, and
+// one integer step either way (products below 2^46) gives the exact floor.  The
+// estimate is the numerator (exact in float) over d rounded to float (relative
+// error 2^-24), divided by the fast approximate division (at most 2 ulp for
+// divisors below 2^126): relative error below 2^-21, so an error below 0.01
+// wherever the estimate is at most R + 2.
 __device__ __forceinline__ uint32_t cr_jump_hash(unsigned long long k, uint32_t R)
 {
     uint32_t b = 0, j = 0;
@@ -60,7 +63,7 @@ __device__ __forceinline__ uint32_t cr_jump_hash(unsigned long long k, uint32_t 
         k = k * 2862933555777941757ull + 1ull;
         const uint32_t d = (uint32_t)(k >> 33) + 1u;
         const unsigned long long num = (unsigned long long)(b + 1u) << 31;
-        const float est = (float)(b + 1u) * (2147483648.0f / (float)d);
+        const float est = __fdividef((float)(b + 1u) * 2147483648.0f, (float)d);
         if (est > (float)R + 2.0f) break;  // the exact quotient is above R as well
         uint32_t q = (uint32_t)est;
         if ((unsigned long long)q * d > num)
@@ -90,17 +93,3 @@ __device__ __forceinline__ unsigned long long cr_warp_min_u64(unsigned long long
 }
 
 __device__ __forceinline__ uint32_t cr_lane() { return threadIdx.x & 31u; }
-
-// Lanes of the warp holding the same 64-bit key (every lane must call it).  The
-// lanes are grouped on a 32-bit fold of the key, and each group is checked
-// against its lowest lane's full key; only if some fold collided between
-// different keys (rare for hashed keys) is the 64-bit match taken.  A 64-bit
-// match costs several times the latency of a 32-bit one on this GPU.
-__device__ __forceinline__ uint32_t cr_match_u64(unsigned long long key)
-{
-    const uint32_t fold = (uint32_t)key ^ (uint32_t)(key >> 32);
-    const uint32_t grp = __match_any_sync(0xffffffffu, fold);
-    const unsigned long long lead = __shfl_sync(0xffffffffu, key, __ffs(grp) - 1);
-    if (__all_sync(0xffffffffu, lead == key)) return grp;
-    return __match_any_sync(0xffffffffu, key);
-}

@@ -57,7 +57,7 @@ __global__ void k_hist_insert(const unsigned long long *__restrict__ keys, uint6
         const bool valid = i < n;
         const unsigned long long key = valid ? keys[i] : kEmptyKey;
         const uint32_t vmask = __ballot_sync(0xffffffffu, valid);
-        const uint32_t peers = cr_match_u64(key) & vmask;
+        const uint32_t peers = __match_any_sync(0xffffffffu, key) & vmask;
         if (!valid || (peers & lt) != 0) continue;  // one leader per distinct key in the warp
         const uint32_t c = __popc(peers);
         if (key == kEmptyKey) {

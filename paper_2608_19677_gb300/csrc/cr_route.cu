@@ -142,21 +142,47 @@ __global__ void __launch_bounds__(256) k_route_cand(const __grid_constant__ rout
             C[i] = kRing | ring_start(rd, cr_fmix64(keys[i] ^ rd.seed));
         break;
     default: {
+        // Table probes for every lane; the requests whose key is not in the table
+        // queue per warp, and the warp draws their power-of-two choices 32 at a time,
+        // so the Philox rounds run with every lane busy.
+        __shared__ unsigned long long q_req[256 / 32][64];
+        const uint32_t lane = threadIdx.x & 31u, lt = (1u << lane) - 1u;
+        unsigned long long *Q = q_req[threadIdx.x >> 5];
+        uint32_t qn = 0;  // queued, < 32 between rounds
         const unsigned long long mask = (1ull << rd.tbits) - 1ull;
-        for (unsigned long long i = i0; i < n; i += stride) {
-            const unsigned long long key = keys[i];
-            unsigned long long sl = key >> (64 - rd.tbits);
+        for (unsigned long long wb = i0 - lane; wb < n; wb += stride) {  // uniform over the warp
+            const unsigned long long i = wb + lane;
+            const bool valid = i < n;
             uint32_t c = 0xffffffffu;
-            for (;;) {
-                const cr_table_slot slot = rd.table[sl];
-                if (slot.koff == kEmpty) break;
-                if (slot.key == key) {
-                    c = slot.k == 1 ? (kFixed | slot.m0) : (kSet | (uint32_t)sl);
-                    break;
+            if (valid) {
+                const unsigned long long key = keys[i];
+                unsigned long long sl = key >> (64 - rd.tbits);
+                for (;;) {
+                    const cr_table_slot slot = rd.table[sl];
+                    if (slot.koff == kEmpty) break;
+                    if (slot.key == key) {
+                        c = slot.k == 1 ? (kFixed | slot.m0) : (kSet | (uint32_t)sl);
+                        break;
+                    }
+                    sl = (sl + 1) & mask;
                 }
-                sl = (sl + 1) & mask;
+                if (c != 0xffffffffu) C[i] = c;
             }
-            C[i] = c != 0xffffffffu ? c : p2c_pair(rd.seed, rd.policy, g0 + i, R);
+            const bool miss = valid && c == 0xffffffffu;
+            const uint32_t mm = __ballot_sync(0xffffffffu, miss);
+            if (miss) Q[qn + (uint32_t)__popc(mm & lt)] = i;
+            qn += (uint32_t)__popc(mm);
+            __syncwarp();
+            if (qn >= 32u) {
+                const unsigned long long j = Q[qn - 32u + lane];
+                C[j] = p2c_pair(rd.seed, rd.policy, g0 + j, R);
+                qn -= 32u;
+                __syncwarp();
+            }
+        }
+        if (lane < qn) {
+            const unsigned long long j = Q[lane];
+            C[j] = p2c_pair(rd.seed, rd.policy, g0 + j, R);
         }
     }
     }
