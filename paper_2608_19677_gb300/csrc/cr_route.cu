@@ -274,13 +274,22 @@ __device__ __forceinline__ const uint16_t *stage_aux(const route_desc &rd, uint1
 // candidates are all RING; every other replica's are FIXED, PAIR or SET, so
 // the two cases are compiled apart.  m: requests in the load vector the batch
 // sees (the bounded-load rule's m).
-template <bool RING>
+// Replica classes of the resolution loop, compiled apart: a plan replica's
+// candidates are FIXED, PAIR or SET, a power-of-two-choices replica's only PAIR,
+// a bounded-load replica's only RING.
+constexpr int kResolvePlan = 0, kResolveRing = 1, kResolvePair = 2;
+
+template <int MODE>
 __device__ __forceinline__ uint32_t resolve(uint32_t c, const route_desc &rd, const uint16_t *mem,
                                             const unsigned long long *L, unsigned long long m, uint32_t R,
                                             uint32_t *status)
 {
     auto load_of = [&](uint32_t d) { return L[d]; };
-    if (RING) return ring_walk(rd, mem, c & kLow30, chwbl_cap(m, R), load_of, status);
+    if (MODE == kResolveRing) return ring_walk(rd, mem, c & kLow30, chwbl_cap(m, R), load_of, status);
+    if (MODE == kResolvePair) {
+        const uint32_t d1 = c & 0x1fffu, d2 = (c >> 13) & 0x1fffu;
+        return L[d1] <= L[d2] ? d1 : d2;
+    }
     const uint32_t kind = c & kKindMask;
     if (kind == kFixed) return c & 0xffffu;
     if (kind == kPair) {
@@ -317,7 +326,7 @@ __device__ __forceinline__ unsigned long long block_load_sum(const unsigned long
 }
 
 // The batch loop of one replica (L already holds its loads; ends with a barrier).
-template <bool RING>
+template <int MODE>
 __device__ __forceinline__ void resolve_batches(const route_desc &rd, const uint16_t *mem, unsigned long long *L,
                                                 uint32_t *delta, uint32_t *cbuf, const uint32_t *__restrict__ Cd,
                                                 uint16_t *__restrict__ D, unsigned long long n, uint32_t B,
@@ -329,7 +338,7 @@ __device__ __forceinline__ void resolve_batches(const route_desc &rd, const uint
         for (unsigned long long b0 = 0; b0 < n; b0 += B) {
             const unsigned long long b1 = (b0 + B < n) ? b0 + B : n;
             for (unsigned long long i = b0 + tid; i < b1; i += blockDim.x) {
-                const uint32_t d = resolve<RING>(Cd[i], rd, mem, L, tot0 + b0, R, status);
+                const uint32_t d = resolve<MODE>(Cd[i], rd, mem, L, tot0 + b0, R, status);
                 if (!CR_DCHECK(d < R, status)) continue;
                 D[i] = (uint16_t)d;
                 atomicAdd(&delta[d], 1u);
@@ -356,12 +365,14 @@ __device__ __forceinline__ void resolve_batches(const route_desc &rd, const uint
             nx[q] = (q * blockDim.x + tid < CH && i < n) ? Cd[i] : 0u;
         }
         const uint32_t *cb = cbuf + (size_t)cur * CH;
-        for (unsigned long long b0 = c0; b0 < c1; b0 += B) {
-            const unsigned long long b1 = (b0 + B < c1) ? b0 + B : c1;
-            for (unsigned long long i = b0 + tid; i < b1; i += blockDim.x) {
-                const uint32_t d = resolve<RING>(cb[i - c0], rd, mem, L, tot0 + b0, R, status);
+        uint16_t *Dc = D + c0;
+        const uint32_t len = (uint32_t)(c1 - c0);  // chunk offsets fit 32 bits
+        for (uint32_t o0 = 0; o0 < len; o0 += B) {
+            const uint32_t o1 = (o0 + B < len) ? o0 + B : len;
+            for (uint32_t o = o0 + tid; o < o1; o += blockDim.x) {
+                const uint32_t d = resolve<MODE>(cb[o], rd, mem, L, tot0 + c0 + o0, R, status);
                 if (!CR_DCHECK(d < R, status)) continue;
-                D[i] = (uint16_t)d;
+                Dc[o] = (uint16_t)d;
                 atomicAdd(&delta[d], 1u);
             }
             __syncthreads();
@@ -404,10 +415,13 @@ __global__ void __launch_bounds__(kRouteBlock) k_route_resolve(const __grid_cons
     const uint16_t *mem = stage_aux(rd, smem_aux, MC);
     if (rd.policy == CR_POLICY_CHWBL) {  // uniform over the block
         const unsigned long long tot0 = block_load_sum(L, R);
-        resolve_batches<true>(rd, mem, L, delta, cbuf, Cd, D, n, B, CH, R, tot0, status);
-    } else {
+        resolve_batches<kResolveRing>(rd, mem, L, delta, cbuf, Cd, D, n, B, CH, R, tot0, status);
+    } else if (rd.policy == CR_POLICY_P2C) {
         __syncthreads();  // orders the copies above
-        resolve_batches<false>(rd, mem, L, delta, cbuf, Cd, D, n, B, CH, R, 0ull, status);
+        resolve_batches<kResolvePair>(rd, mem, L, delta, cbuf, Cd, D, n, B, CH, R, 0ull, status);
+    } else {
+        __syncthreads();
+        resolve_batches<kResolvePlan>(rd, mem, L, delta, cbuf, Cd, D, n, B, CH, R, 0ull, status);
     }
     for (uint32_t r = threadIdx.x; r < R; r += blockDim.x) Lg[r] = L[r];
 }
