@@ -77,6 +77,9 @@ def parse_args(argv=None):
     ap.add_argument("--route-streams", type=int, default=4, help="keys mode: streams routing")
     ap.add_argument("--replay-group", type=int, default=2,
                     help="keys mode: consecutive intervals replayed by one call")
+    ap.add_argument("--trace-min-interval", type=int, default=65536,
+                    help="resident inputs: mean requests per interval from which the multi-interval "
+                         "driver runs the trace (0: always)")
     ap.add_argument("--replay-priority", choices=["high", "low"], default="low",
                     help="keys mode: priority of the replay stream (plans get the other one)")
     ap.add_argument("--intervals", type=int, default=0,
@@ -551,7 +554,7 @@ def main():
     max_n = max(x[6] for x in inputs)
     # several intervals in flight pay off when intervals are large; many small intervals are
     # bound by launches from the host, which the one-interval driver issues fewer of
-    big = n_step / max(cfg.n_intervals, 1) >= 65536
+    big = n_step / max(cfg.n_intervals, 1) >= args.trace_min_interval
     if big and not (args.per_interval or args.graph or part is not None or cfg.drift or args.no_overlap):
         return run_resident_trace(args, cfg, trace, inputs, hash_bytes, dev, stream, world, rank, barrier)
 

@@ -309,7 +309,22 @@ __device__ __forceinline__ uint32_t resolve(uint32_t c, const route_desc &rd, co
 // batch, at most kStage requests) ahead: while chunk c is resolved from one
 // buffer, chunk c+1's loads are in flight into registers and land in the other.
 constexpr uint32_t kStage = 16384;
-constexpr int kStageRegs = kStage / kRouteBlock;  // 16
+
+// 4-byte asynchronous global -> shared copies (the next chunk lands while this
+// one is resolved, without holding registers)
+__device__ __forceinline__ void cp_async4(void *smem, const void *gmem)
+{
+    const unsigned sa = (unsigned)__cvta_generic_to_shared(smem);
+    asm volatile("cp.async.ca.shared.global [%0], [%1], 4;\n" ::"r"(sa), "l"(gmem) : "memory");
+}
+__device__ __forceinline__ void cp_async_wait_all() { asm volatile("cp.async.wait_all;\n" ::: "memory"); }
+
+// Start copying chunk [c1, c1 + CH) of the candidates into buffer nb.
+__device__ __forceinline__ void stage_next(uint32_t *nb, const uint32_t *__restrict__ Cd, unsigned long long c1,
+                                           unsigned long long n, uint32_t CH)
+{
+    for (uint32_t q = threadIdx.x; q < CH && c1 + q < n; q += blockDim.x) cp_async4(&nb[q], &Cd[c1 + q]);
+}
 
 // Sum of a replica's load vector on entry (the m of the bounded-load rule).
 __device__ __forceinline__ unsigned long long block_load_sum(const unsigned long long *L, uint32_t R)
@@ -357,13 +372,7 @@ __device__ __forceinline__ void resolve_batches(const route_desc &rd, const uint
     int cur = 0;
     for (unsigned long long c0 = 0; c0 < n; c0 += CH) {
         const unsigned long long c1 = (c0 + CH < n) ? c0 + CH : n;
-        // next chunk in flight
-        uint32_t nx[kStageRegs];
-#pragma unroll
-        for (int q = 0; q < kStageRegs; ++q) {
-            const unsigned long long i = c1 + (unsigned long long)q * blockDim.x + tid;
-            nx[q] = (q * blockDim.x + tid < CH && i < n) ? Cd[i] : 0u;
-        }
+        stage_next(cbuf + (size_t)(cur ^ 1) * CH, Cd, c1, n, CH);  // next chunk in flight
         const uint32_t *cb = cbuf + (size_t)cur * CH;
         uint16_t *Dc = D + c0;
         const uint32_t len = (uint32_t)(c1 - c0);  // chunk offsets fit 32 bits
@@ -382,13 +391,204 @@ __device__ __forceinline__ void resolve_batches(const route_desc &rd, const uint
             }
             __syncthreads();
         }
-        uint32_t *nb = cbuf + (size_t)(cur ^ 1) * CH;
-#pragma unroll
-        for (int q = 0; q < kStageRegs; ++q)
-            if (q * blockDim.x + tid < CH) nb[q * blockDim.x + tid] = nx[q];
+        cp_async_wait_all();
         __syncthreads();
         cur ^= 1;
     }
+}
+
+// ---- plan replicas: keys with several members decided once per batch ---------
+// Inside a batch every request of a key with k_b > 1 goes to the same member:
+// the least loaded of T(b) at the batch start (ties to the earlier member).  So
+// the CTA keeps the member lists of those keys in shared memory, collected as
+// the staging meets them, and finds each key's member once per batch, at the
+// boundary; a request then reads its key's answer.  Loads and batch counts are
+// double-buffered so that the answers for batch b + 1 (loads of batch b plus
+// its counts) are computed while the loads are being updated, behind the same
+// two barriers per batch.
+constexpr uint32_t kSetCap = 256;      // keys with k_b > 1 tracked per replica
+constexpr uint32_t kSetMapCap = 512;   // open-addressing map: table slot -> key index
+constexpr uint32_t kSetPool = 4096;    // member entries of the tracked keys
+
+struct set_cache {
+    uint32_t map_slot[kSetMapCap];  // table slot of each map entry, kEmpty when free
+    uint16_t map_j[kSetMapCap];     // key index of each map entry
+    uint32_t off[kSetCap];          // first member of key j in the pool
+    uint16_t k[kSetCap];
+    uint16_t res[2][kSetCap];       // least-loaded member of each key, per batch parity
+    uint16_t pool[kSetPool];
+    uint32_t n, used, ready, overflow;
+};
+
+__host__ __device__ inline size_t set_cache_bytes() { return (sizeof(set_cache) + 15) & ~(size_t)15; }
+
+// Shared-memory layout of k_route_resolve: loads [R] u64, counts [R] u32, two
+// staging buffers [CH] u32, member lists / ring owners [MC] u16, then (plan
+// replicas) the second loads and counts and the key cache, 16-byte aligned.
+__host__ __device__ inline size_t resolve_plan_extra_at(uint32_t R, uint32_t CH, unsigned long long MC)
+{
+    return ((size_t)R * 12 + (size_t)CH * 8 + (size_t)MC * 2 + 15) & ~(size_t)15;
+}
+__host__ __device__ inline size_t resolve_plan_extra_bytes(uint32_t R)
+{
+    return (((size_t)R * 12 + 15) & ~(size_t)15) + set_cache_bytes();
+}
+
+__device__ __forceinline__ uint32_t set_hash(uint32_t slot) { return (slot * 0x9E3779B1u) >> 23; }  // 9 bits
+
+// Record the key of table slot `slot` (a SET candidate) unless it is known.
+__device__ void set_discover(set_cache &S, const route_desc &rd, const uint16_t *mem, uint32_t slot)
+{
+    uint32_t h = set_hash(slot);
+    for (uint32_t it = 0; it < kSetMapCap; ++it, h = (h + 1) & (kSetMapCap - 1)) {
+        const uint32_t cur = *(volatile uint32_t *)&S.map_slot[h];
+        if (cur == slot) return;
+        if (cur != kEmpty) continue;
+        const uint32_t prev = atomicCAS(&S.map_slot[h], kEmpty, slot);
+        if (prev == slot) return;
+        if (prev != kEmpty) continue;
+        const uint32_t j = atomicAdd(&S.n, 1u);
+        const cr_table_slot ts = rd.table[slot];
+        const uint32_t off = atomicAdd(&S.used, (uint32_t)ts.k);
+        if (j >= kSetCap || off + ts.k > kSetPool) {
+            S.overflow = 1u;
+            return;
+        }
+        for (uint32_t m = 0; m < ts.k; ++m) S.pool[off + m] = mem[(size_t)ts.koff + m];
+        S.off[j] = off;
+        S.k[j] = ts.k;
+        S.map_j[h] = (uint16_t)j;
+        return;
+    }
+    S.overflow = 1u;
+}
+
+// Key index of a discovered slot, or kEmpty.
+__device__ __forceinline__ uint32_t set_find(const set_cache &S, uint32_t slot)
+{
+    uint32_t h = set_hash(slot);
+    for (uint32_t it = 0; it < kSetMapCap; ++it, h = (h + 1) & (kSetMapCap - 1)) {
+        const uint32_t cur = S.map_slot[h];
+        if (cur == slot) return S.map_j[h];
+        if (cur == kEmpty) return kEmpty;
+    }
+    return kEmpty;
+}
+
+// res[j] for keys j0 .. j1-1: the first member with the least load Lb[m] (+ db[m]),
+// one warp per key.
+__device__ __forceinline__ void set_results(set_cache &S, uint16_t *res, const unsigned long long *Lb,
+                                            const uint32_t *db, uint32_t j0, uint32_t j1)
+{
+    const uint32_t lane = threadIdx.x & 31u, warp = threadIdx.x >> 5, nw = blockDim.x >> 5;
+    for (uint32_t j = j0 + warp; j < j1; j += nw) {
+        const uint32_t off = S.off[j], k = S.k[j];
+        unsigned long long bl = ~0ull;
+        uint32_t bp = 0xffffffffu;
+        for (uint32_t p = lane; p < k; p += 32) {
+            const uint32_t m = S.pool[off + p];
+            const unsigned long long l = Lb[m] + (db ? db[m] : 0u);
+            if (l < bl) {  // positions rise within a lane: the first minimum stays
+                bl = l;
+                bp = p;
+            }
+        }
+        // the lexicographic minimum of (load, position) over the warp, by three 32-bit
+        // warp reductions: high word of the load, low word among those, position among those
+        const uint32_t hi = (uint32_t)(bl >> 32), lo = (uint32_t)bl;
+        const uint32_t mhi = __reduce_min_sync(0xffffffffu, hi);
+        const uint32_t mlo = __reduce_min_sync(0xffffffffu, hi == mhi ? lo : 0xffffffffu);
+        const uint32_t mp = __reduce_min_sync(0xffffffffu, (hi == mhi && lo == mlo) ? bp : 0xffffffffu);
+        if (lane == 0) res[j] = S.pool[off + mp];
+    }
+}
+
+// The batch loop of a plan replica with staging (CH > 0).  L0/dl0 hold the loads
+// and zero counts on entry; returns the buffer (0 or 1) that holds the loads at
+// the end.  Falls back to per-request member scans once the cache overflows.
+__device__ int resolve_batches_plan(const route_desc &rd, const uint16_t *mem, unsigned long long *L0,
+                                    unsigned long long *L1, uint32_t *dl0, uint32_t *dl1, set_cache &S,
+                                    uint32_t *cbuf, const uint32_t *__restrict__ Cd, uint16_t *__restrict__ D,
+                                    unsigned long long n, uint32_t B, uint32_t CH, uint32_t R, uint32_t *status)
+{
+    const uint32_t tid = threadIdx.x;
+    for (uint32_t x = tid; x < kSetMapCap; x += blockDim.x) S.map_slot[x] = kEmpty;
+    if (tid == 0) {
+        S.n = 0;
+        S.used = 0;
+        S.ready = 0;
+        S.overflow = 0;
+    }
+    for (uint32_t r = tid; r < R; r += blockDim.x) dl1[r] = 0;
+    __syncthreads();
+    for (uint32_t x = tid; x < CH && x < n; x += blockDim.x) {
+        const uint32_t c = Cd[x];
+        cbuf[x] = c;
+        if ((c & kKindMask) == kSet) set_discover(S, rd, mem, c & kLow30);
+    }
+    __syncthreads();
+    if (!S.overflow) set_results(S, S.res[0], L0, nullptr, 0, min(S.n, kSetCap));
+    if (tid == 0) S.ready = min(S.n, kSetCap);  // read by nobody before the barrier
+    __syncthreads();
+    int par = 0, cur = 0;
+    for (unsigned long long c0 = 0; c0 < n; c0 += CH) {
+        const unsigned long long c1 = (c0 + CH < n) ? c0 + CH : n;
+        uint32_t *nb = cbuf + (size_t)(cur ^ 1) * CH;
+        stage_next(nb, Cd, c1, n, CH);
+        const uint32_t *cb = cbuf + (size_t)cur * CH;
+        uint16_t *Dc = D + c0;
+        const uint32_t len = (uint32_t)(c1 - c0);
+        const bool ovf = S.overflow != 0u;  // uniform: written only while staging
+        for (uint32_t o0 = 0; o0 < len; o0 += B) {
+            const uint32_t o1 = (o0 + B < len) ? o0 + B : len;
+            unsigned long long *Lc = par ? L1 : L0, *Ln = par ? L0 : L1;
+            uint32_t *dc = par ? dl1 : dl0, *dn = par ? dl0 : dl1;
+            const uint16_t *res = S.res[par];
+            for (uint32_t o = o0 + tid; o < o1; o += blockDim.x) {
+                const uint32_t c = cb[o], kind = c & kKindMask;
+                // FIXED and PAIR without a branch: for FIXED the two fields read are the
+                // destination (< R <= 8192) and 0, in range as well; a SET reads entry 0
+                const bool two = kind < kSet;
+                const uint32_t d1 = two ? (c & 0x1fffu) : 0u, d2 = two ? ((c >> 13) & 0x1fffu) : 0u;
+                const bool p1 = Lc[d1] <= Lc[d2];
+                uint32_t d = kind == kFixed ? (c & 0xffffu) : (p1 ? d1 : d2);
+                if (!two) {
+                    const uint32_t j = ovf ? kEmpty : set_find(S, c & kLow30);
+                    if (j < kSetCap) {
+                        d = res[j];
+                    } else {
+                        const cr_table_slot slot = rd.table[c & kLow30];
+                        auto load_of = [&](uint32_t x) { return Lc[x]; };
+                        d = set_min(mem, slot.koff, slot.k, slot.m0, load_of);
+                    }
+                }
+                if (!CR_DCHECK(d < R, status)) continue;
+                Dc[o] = (uint16_t)d;
+                atomicAdd(&dc[d], 1u);
+            }
+            __syncthreads();
+            for (uint32_t r = tid; r < R; r += blockDim.x) {
+                Ln[r] = Lc[r] + dc[r];
+                dn[r] = 0;
+            }
+            if (!ovf) set_results(S, S.res[par ^ 1], Lc, dc, 0, min(S.ready, kSetCap));
+            __syncthreads();
+            par ^= 1;
+        }
+        cp_async_wait_all();
+        __syncthreads();
+        for (uint32_t q = tid; q < CH && c1 + q < n; q += blockDim.x)
+            if ((nb[q] & kKindMask) == kSet) set_discover(S, rd, mem, nb[q] & kLow30);
+        __syncthreads();
+        // keys met for the first time: their answers for the next batch, from its loads
+        const uint32_t nn = min(S.n, kSetCap), rd0 = S.ready;
+        if (nn > rd0 && !S.overflow) set_results(S, S.res[par], par ? L1 : L0, nullptr, rd0, nn);  // uniform
+        __syncthreads();  // every thread has read S.ready
+        if (tid == 0) S.ready = S.overflow ? rd0 : nn;
+        __syncthreads();
+        cur ^= 1;
+    }
+    return par;
 }
 
 __global__ void __launch_bounds__(kRouteBlock) k_route_resolve(const __grid_constant__ route_args args,
@@ -396,13 +596,15 @@ __global__ void __launch_bounds__(kRouteBlock) k_route_resolve(const __grid_cons
                                                                unsigned long long n, uint32_t B, uint32_t CH,
                                                                uint32_t R, unsigned long long *__restrict__ load,
                                                                uint16_t *__restrict__ dest, uint32_t *status,
-                                                               unsigned long long MC)
+                                                               unsigned long long MC, int plan_x)
 {
     extern __shared__ unsigned long long sh[];
     unsigned long long *L = sh;                              // [R] live load
     uint32_t *delta = reinterpret_cast<uint32_t *>(sh + R);  // [R] this batch
     uint32_t *cbuf = delta + R;                              // [2][CH] staged candidates
     uint16_t *smem_aux = reinterpret_cast<uint16_t *>(cbuf + 2 * (size_t)CH);  // [MC] members or ring owners
+    // plan replicas (when the launch reserved it): the second load and count buffers and the key cache
+    unsigned char *px = reinterpret_cast<unsigned char *>(sh) + resolve_plan_extra_at(R, CH, MC);
     const uint32_t rep = args.dep[blockIdx.x];
     const route_desc rd = args.d[rep];
     unsigned long long *Lg = load + (unsigned long long)rep * R;
@@ -419,6 +621,14 @@ __global__ void __launch_bounds__(kRouteBlock) k_route_resolve(const __grid_cons
     } else if (rd.policy == CR_POLICY_P2C) {
         __syncthreads();  // orders the copies above
         resolve_batches<kResolvePair>(rd, mem, L, delta, cbuf, Cd, D, n, B, CH, R, 0ull, status);
+    } else if (plan_x && CH > 0) {
+        __syncthreads();
+        unsigned long long *L1 = reinterpret_cast<unsigned long long *>(px);
+        uint32_t *dl1 = reinterpret_cast<uint32_t *>(L1 + R);
+        set_cache &S = *reinterpret_cast<set_cache *>(px + (((size_t)R * 12 + 15) & ~(size_t)15));
+        if (resolve_batches_plan(rd, mem, L, L1, delta, dl1, S, cbuf, Cd, D, n, B, CH, R, status))
+            for (uint32_t r = threadIdx.x; r < R; r += blockDim.x) L[r] = L1[r];
+        __syncthreads();
     } else {
         __syncthreads();
         resolve_batches<kResolvePlan>(rd, mem, L, delta, cbuf, Cd, D, n, B, CH, R, 0ull, status);
@@ -802,12 +1012,33 @@ static int launch_resolve(cr_ctx *ctx, cudaStream_t rs, const route_args &args, 
         return CR_OK;
     }
     // staging chunk: a whole number of batches, at most kStage requests
-    const uint32_t CH = batch_B <= kStage ? (kStage / batch_B) * batch_B : 0u;  // 0: no staging
-    const size_t smem = with_members(
-        (size_t)R * (sizeof(unsigned long long) + sizeof(uint32_t)) + 2ull * CH * sizeof(uint32_t), &MC);
+    uint32_t CH = batch_B <= kStage ? (kStage / batch_B) * batch_B : 0u;  // 0: no staging
+    const size_t loads = (size_t)R * (sizeof(unsigned long long) + sizeof(uint32_t));
+    // plan replicas take the second load and count buffers and the key cache when they
+    // fit beside a stage of at least one batch (the stage shrinks by whole batches)
+    bool any_plan = false;
+    for (uint32_t i = 0; i < n_dep; ++i) any_plan |= args.d[args.dep[i]].policy <= CR_POLICY_CR_NOREPL;
+    const size_t px = resolve_plan_extra_bytes(R);
+    int plan_x = 0;
+    if (any_plan && CH) {
+        uint32_t ch = CH;
+        while (ch >= batch_B && loads + (size_t)ch * 8 + 16 + px > kSmemBudget) ch -= batch_B;
+        if (ch >= batch_B) {
+            CH = ch;
+            plan_x = 1;
+        }
+    }
+    size_t smem;
+    if (plan_x) {
+        const size_t fixed = loads + (size_t)CH * 8 + 16 + px;
+        MC = (mc && fixed + mc * sizeof(uint16_t) <= kSmemBudget) ? mc : 0;
+        smem = resolve_plan_extra_at(R, CH, MC) + px;
+    } else {
+        smem = with_members(loads + 2ull * CH * sizeof(uint32_t), &MC);
+    }
     if (smem > 48 * 1024)
         CR_CUDA(ctx, cudaFuncSetAttribute(k_route_resolve, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
     CR_LAUNCH_ON(ctx, rs, k_route_resolve, n_dep, kRouteBlock, smem, args, (const uint32_t *)cand, (unsigned long long)n,
-              batch_B, CH, R, (unsigned long long *)d_load, d_dest, ctx->d_status, (unsigned long long)MC);
+              batch_B, CH, R, (unsigned long long *)d_load, d_dest, ctx->d_status, (unsigned long long)MC, plan_x);
     return CR_OK;
 }

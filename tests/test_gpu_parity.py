@@ -380,6 +380,36 @@ def test_route_small_batches_one_hot_key(P, ctx, B):
     assert (h_u64(load) == ref_load).all()
 
 
+@pytest.mark.parametrize("case", ["few", "many", "pool", "wide"])
+@pytest.mark.parametrize("B", [100, 1024])
+def test_route_replicated_keys_per_batch(P, ctx, case, B):
+    # keys with k_b > 1 decided once per batch from a shared-memory cache of their member
+    # lists: a few such keys; more keys than the cache holds (300); member lists larger than
+    # its pool (two keys on every one of 4096 destinations); and R = 8192, where the cache
+    # does not fit beside the loads.  q_cap = 1, so a key seen c times gets k_b = min(c, R).
+    rng = np.random.default_rng(B + len(case))
+    R, W = {"few": (64, 64), "many": (64, 64), "pool": (4096, 2), "wide": (8192, 1)}[case]
+    counts = {"few": [2, 3, 5, 8, 13, 21, 34, 55, 64, 64], "many": [2] * 300 + [3] * 20,
+              "pool": [4096, 4096], "wide": [7, 300, 2]}[case]
+    ks = rng.integers(1, 2**63, len(counts) + 30000, dtype=np.int64).astype(np.uint64)
+    keys = np.concatenate([np.repeat(ks[: len(counts)], counts), ks[len(counts):]])
+    rng.shuffle(keys)
+    pols, seeds = ["CR", "CR_NOLPT", "CR_NOREPL", "P2C", "CR"], [0, 1, 0, 2, 3]
+    vmap = {"CR": ("LPT", 0), "CR_NOLPT": ("RANDOM", 1), "CR_NOREPL": ("NOREPL", 0)}
+    opl = {p: O.build_plan(keys, R, W, 1, 1, variant=v, seed=s, epoch=0) for p, (v, s) in vmap.items()}
+    dpl = {p: P.build_plan(ctx, d_u64(keys), P.plan_params(R, W, 1, 1, v, seed=s, epoch=0))
+           for p, (v, s) in vmap.items()}
+    assert (np.asarray(opl["CR"].adm_k) > 1).sum() >= min(len(counts), 2)
+    init = rng.integers(0, 9, size=(len(pols), R)).astype(np.uint64)
+    ref_dest, ref_load = O.route([opl.get(p) for p in pols], pols, seeds, R, keys, 11, B, load=init)
+    load = d_u64(init.reshape(-1)).view(len(pols), R).contiguous()
+    dest = P.route_batch(ctx, [dpl.get(p) for p in pols], pols, seeds, R, d_u64(keys), 11, B, load)
+    ctx.sync()
+    for i, p in enumerate(pols):
+        assert (h_u16(dest[i]) == ref_dest[i]).all(), (i, p)
+    assert (h_u64(load) == ref_load).all()
+
+
 def test_route_rejects_bad_args(P, ctx):
     keys = d_u64(np.array([1, 2, 3], np.uint64))
     load = torch.zeros((1, 4), dtype=torch.int64, device=DEV)
