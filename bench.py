@@ -46,9 +46,12 @@ def parse_args(argv=None):
     ap.add_argument("--sm-split", type=int, default=0,
                     help="run hashing and candidates on all but N SMs and the load-dependent route resolution on "
                          "the other N (green contexts), so that it overlaps the next interval's hashing")
-    ap.add_argument("--graph", action="store_true",
-                    help="capture the whole step (every interval) once as a CUDA graph and replay it; stage "
-                         "times and the roofline then come from one ordinary step after the timed region")
+    ap.add_argument("--graph", action=argparse.BooleanOptionalAction, default=None,
+                    help="capture the whole step (every interval) once as a CUDA graph and replay it, so that the "
+                         "host enqueues one graph per step instead of every launch (default: on for configurations "
+                         "whose inputs stay resident, off in keys mode, whose few large intervals the host "
+                         "enqueues in a fraction of the step, and with --sm-split or --per-interval); kernel times "
+                         "and the roofline then come from one ordinary step after the timed region")
     ap.add_argument("--fresh-plans", action="store_true",
                     help="plan every interval from its own keys (the fresh plan of the replanning study) "
                          "instead of from the previous interval's")
@@ -72,19 +75,28 @@ def parse_args(argv=None):
     ap.add_argument("--per-interval", action="store_true",
                     help="drive one interval at a time (Pipeline) instead of keeping several intervals' plans and "
                          "routes in flight (TracePipeline)")
-    ap.add_argument("--depth", type=int, default=8, help="keys mode: intervals in flight")
-    ap.add_argument("--plan-streams", type=int, default=4, help="keys mode: streams building plans")
-    ap.add_argument("--route-streams", type=int, default=4, help="keys mode: streams routing")
-    ap.add_argument("--replay-group", type=int, default=2,
-                    help="keys mode: consecutive intervals replayed by one call")
-    ap.add_argument("--trace-min-interval", type=int, default=65536,
+    ap.add_argument("--depth", type=int, default=16, help="multi-interval driver: intervals in flight")
+    ap.add_argument("--plan-streams", type=int, default=8, help="multi-interval driver: streams building plans")
+    ap.add_argument("--route-streams", type=int, default=4, help="multi-interval driver: streams routing")
+    ap.add_argument("--replay-group", type=int, default=None,
+                    help="multi-interval driver: consecutive intervals replayed by one call (default: "
+                         "max(2, min(16, 65536 // mean requests per interval)))")
+    ap.add_argument("--trace-min-interval", type=int, default=None,
                     help="resident inputs: mean requests per interval from which the multi-interval "
-                         "driver runs the trace (0: always)")
+                         "driver runs the trace (default: 0 with a CUDA graph, 65536 without, where many "
+                         "small intervals are bound by the host's launch rate)")
     ap.add_argument("--replay-priority", choices=["high", "low"], default="low",
                     help="keys mode: priority of the replay stream (plans get the other one)")
     ap.add_argument("--intervals", type=int, default=0,
                     help="profiling aid: run only the first N intervals (the JSON line says so)")
-    return ap.parse_args(argv)
+    args = ap.parse_args(argv)
+    args.graph_auto = args.graph is None
+    if args.graph is None:
+        args.graph = not (args.sm_split or args.per_interval)
+    args.trace_min_interval_auto = args.trace_min_interval is None
+    if args.trace_min_interval is None:
+        args.trace_min_interval = 0 if args.graph else 65536
+    return args
 
 
 def with_policies(cfg, args):
@@ -326,6 +338,22 @@ def token_bytes(trace) -> float:
     return 4.0 * rec_tokens * float(sum(trace.counts[:cfg.n_intervals]))
 
 
+def auto_schedule(args, trace):
+    """Defaults that depend on the interval size (mean requests per interval, m): a CUDA
+    graph of the step when m < 262,144 (many intervals, each too short to hide the host's
+    launches; the Large sweep's ~1M-request intervals run better without one), and
+    max(2, min(16, 65536 // m)) consecutive intervals per replay call (the replay is the
+    one serial chain; grouping short intervals shortens it)."""
+    cfg = trace.cfg
+    m = sum(int(c) for c in trace.counts[:cfg.n_intervals]) / max(cfg.n_intervals, 1)
+    if args.graph_auto:
+        args.graph = bool(m < 262144 and not (args.sm_split or args.per_interval))
+        if args.trace_min_interval_auto:
+            args.trace_min_interval = 0 if args.graph else 65536
+    if args.replay_group is None:
+        args.replay_group = int(max(2, min(16, 65536 // max(int(m), 1))))
+
+
 def keys_mode_for(args, trace, free_bytes: float = 280e9) -> bool:
     """Keys mode when asked, or when the arenas would not fit in (60% of) free device memory."""
     return bool(args.keys_mode) or token_bytes(trace) > 0.6 * free_bytes
@@ -511,6 +539,12 @@ def main():
     cfg = with_policies(tg.CONFIGS[args.config], args)
     cfg = replica_cfg(cfg, rank, world)  # independent replica per rank
     trace = tg.Trace(cfg)
+    if args.intervals:
+        import dataclasses
+        cfg = dataclasses.replace(cfg, n_intervals=args.intervals, name=f"{cfg.name} (first {args.intervals} "
+                                  f"intervals only)", n_requests=int(sum(trace.counts[:args.intervals])))
+        trace.cfg = cfg
+    auto_schedule(args, trace)
     dev = torch.device("cuda", local)
     part = None
     if args.sm_split and args.graph:
@@ -523,12 +557,6 @@ def main():
         torch.cuda.set_stream(torch.cuda.Stream(dev))
     stream = torch.cuda.current_stream(dev)
     resolve_stream = part.small if part is not None else None
-
-    if args.intervals:
-        import dataclasses
-        cfg = dataclasses.replace(cfg, n_intervals=args.intervals, name=f"{cfg.name} (first {args.intervals} "
-                                  f"intervals only)", n_requests=int(sum(trace.counts[:args.intervals])))
-        trace.cfg = cfg
 
     # keys mode: when the token arenas of all intervals do not fit in HBM (the
     # large configuration holds ~600 GB of tokens), every interval's arena is
@@ -555,7 +583,7 @@ def main():
     # several intervals in flight pay off when intervals are large; many small intervals are
     # bound by launches from the host, which the one-interval driver issues fewer of
     big = n_step / max(cfg.n_intervals, 1) >= args.trace_min_interval
-    if big and not (args.per_interval or args.graph or part is not None or cfg.drift or args.no_overlap):
+    if big and not (args.per_interval or part is not None or cfg.drift or args.no_overlap):
         return run_resident_trace(args, cfg, trace, inputs, hash_bytes, dev, stream, world, rank, barrier)
 
     ctx = P.Context(local, stream)
@@ -1103,8 +1131,21 @@ def run_resident_trace(args, cfg, trace, inputs, hash_bytes, dev, stream, world,
     pipe.sync()
     hctx.sync()
     prof = pipe.contexts + [hctx]
-    for c in prof:
-        c.profile_enable(16 * cfg.n_intervals * max(args.steps, 1) + 64)
+    # optional CUDA graph of the whole step (every interval's hash, plans, routes and
+    # replay): the host then enqueues one graph per step instead of every launch
+    graph, graph_launches = None, 0
+    if args.graph:
+        pipe.quiesce()
+        lc0 = pipe.launches + hctx.launches
+        graph = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(graph, stream=stream):
+            enqueue(resident)
+        graph_launches = pipe.launches + hctx.launches - lc0
+        graph.replay()
+        torch.cuda.synchronize()
+    else:
+        for c in prof:
+            c.profile_enable(16 * cfg.n_intervals * max(args.steps, 1) + 64)
     clocks = ClockSampler(dev.index or 0, args.clocks_out)
     clocks.start()
     time.sleep(0.3)
@@ -1115,12 +1156,22 @@ def run_resident_trace(args, cfg, trace, inputs, hash_bytes, dev, stream, world,
     ev1 = torch.cuda.Event(enable_timing=True)
     ev0.record(stream)
     for _ in range(args.steps):
-        enqueue(resident)
+        if graph is not None:
+            graph.replay()
+        else:
+            enqueue(resident)
     ev1.record(stream)
     torch.cuda.synchronize()
     barrier()
-    n_launch = pipe.launches + hctx.launches - l0
+    n_launch = graph_launches * args.steps if graph is not None else pipe.launches + hctx.launches - l0
     clk = clocks.stop()
+    steps_profiled = args.steps
+    if graph is not None:  # kernel times from one ordinary step after the timed region
+        pipe.quiesce()
+        for c in prof:
+            c.profile_enable(16 * cfg.n_intervals + 64)
+        enqueue(resident)
+        steps_profiled = 1
     pipe.sync()
     kern = {}
     for tag in ("hash", "plan", "route_cand", "route_resolve", "partition", "replay"):
@@ -1128,7 +1179,7 @@ def run_resident_trace(args, cfg, trace, inputs, hash_bytes, dev, stream, world,
         for c in prof:
             a, b = c.profile_read(tag)
             n_, ms_ = n_ + a, ms_ + b
-        kern[tag] = {"launches": n_, "avg_ms": ms_ / n_ if n_ else None, "ms_per_step": ms_ / max(args.steps, 1)}
+        kern[tag] = {"launches": n_, "avg_ms": ms_ / n_ if n_ else None, "ms_per_step": ms_ / steps_profiled}
     for c in prof:
         c.profile_enable(0)
     ms = ev0.elapsed_time(ev1) / args.steps
@@ -1148,7 +1199,7 @@ def run_resident_trace(args, cfg, trace, inputs, hash_bytes, dev, stream, world,
                "frac": hb / (hash_ms / 1e3) / 1e9 / hbm_peak, "traffic": hash_traffic(hb),
                "algorithmic_bytes_per_launch_mean": hb, "avg_launch_ms": hash_ms,
                "launches_timed": kern["hash"]["launches"]}
-    req_per_launch = n_step * args.steps / max(kern["replay"]["launches"], 1)
+    req_per_launch = n_step * steps_profiled / max(kern["replay"]["launches"], 1)
     a9_bytes = 20.0 * reps * ncaps * req_per_launch
     lru_ms = kern["replay"]["avg_ms"]
     lru_rf = {"kernel": "k_lru_stamp (a9 LRU replay)" if not cfg.lru_tokens else "k_lru_tokens (a9 byte-aware replay)",
@@ -1168,7 +1219,9 @@ def run_resident_trace(args, cfg, trace, inputs, hash_bytes, dev, stream, world,
         "config": dict(workload_config(cfg, args.batch, args.fresh_plans),
                        schedule=(f"hashing on its own stream, one event per interval; {args.depth} intervals in "
                                  f"flight: plans on {args.plan_streams} streams, routes on {args.route_streams} "
-                                 f"streams, the replay in interval order, {args.replay_group} intervals per call")),
+                                 f"streams, the replay in interval order, {args.replay_group} intervals per call"
+                                 + ("; the step captured once as a CUDA graph and replayed" if graph is not None
+                                    else ""))),
         "roofline": lru_rf if dom_lru else hash_rf,
         ("hash_roofline" if dom_lru else "replay_roofline"): hash_rf if dom_lru else lru_rf,
         "kernels_ms_per_launch": kern,

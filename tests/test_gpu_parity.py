@@ -584,6 +584,40 @@ def test_trace_pipeline_parity(P, ctx, name, n, nint, depth, ps, rs, grp):
     pipe.close()
 
 
+@pytest.mark.parametrize("name,grp", [("8b", 4), ("70b", 2)])
+def test_trace_pipeline_cuda_graph(P, ctx, name, grp):
+    # the whole trace (reset + every interval's plans, routes and replay, on many streams)
+    # captured once as a CUDA graph: each replay gives the oracle's counters again
+    from paper_2608_19677_gb300.pipeline import TracePipeline
+    cfg = tg.CONFIGS[name].scaled(40000, 8)
+    tr = tg.Trace(cfg)
+    ref = OP.run_trace(tr, B=1024, keep=True)
+    ivs = [tr.interval(t) for t in range(cfg.n_intervals)]
+    keys = [d_u64(k) for k in ref["keys"]]
+    plens = [d_u32(iv.plen) for iv in ivs]
+    slens = [d_u32(iv.slen) for iv in ivs]
+    g0s = [iv.g0 for iv in ivs]
+    stream = torch.cuda.Stream()       # a graph is captured on a stream other than the default one
+    gctx = P.Context(0, stream)
+    pipe = TracePipeline(gctx, cfg.R, cfg.W, cfg.caps, cfg.replicas, tr.qcap, max_n=max(iv.n for iv in ivs),
+                         batch_B=1024, depth=4, plan_streams=3, route_streams=2, vnodes=cfg.vnodes,
+                         replay_group=grp)
+    pipe.reset()
+    pipe.run(keys, plens, slens, g0s)   # warm-up: scratch and inputs reach their sizes
+    pipe.quiesce()
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(graph, stream=stream):
+        pipe.reset()
+        pipe.run(keys, plens, slens, g0s)
+    for _ in range(2):
+        graph.replay()
+        torch.cuda.synchronize()
+        assert (h_u64(pipe.ctr) == ref["ctr"]).all()
+    del graph
+    pipe.close()
+    gctx.close()
+
+
 @pytest.mark.parametrize("B", [1, 7, 1024])
 def test_pipeline_parity_bounded_load_and_small_batches(P, ctx, B):
     # the 70B shape with the bounded-load comparison policy added, routed in
