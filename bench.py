@@ -614,7 +614,7 @@ def main():
     def launches():
         return pipe.launches
 
-    for _ in range(max(args.warmup, 0)):
+    for _ in range(max(args.warmup, 1 if args.graph else 0)):  # a graph captures warm buffers only
         step()
     ctx.sync()
     torch.cuda.synchronize()
@@ -874,7 +874,7 @@ def run_keys_mode(args, cfg, trace, dev, stream, world, rank, barrier, resolve_s
             route_marks[k] = list(pipe.route_marks)
             replay_marks[k] = list(pipe.replay_marks)
 
-    for _ in range(max(args.warmup, 0)):
+    for _ in range(max(args.warmup, 1 if args.graph else 0)):  # a graph captures warm buffers only
         step()
     pipe.sync()
     graph, graph_launches = None, 0
@@ -1126,7 +1126,7 @@ def run_resident_trace(args, cfg, trace, inputs, hash_bytes, dev, stream, world,
         stream.wait_event(hashed[-1])
 
     resident = [(x[1], x[2], x[3], x[4]) for x in inputs]
-    for _ in range(max(args.warmup, 0)):
+    for _ in range(max(args.warmup, 1 if args.graph else 0)):  # a graph captures warm buffers only
         enqueue(resident)
     pipe.sync()
     hctx.sync()
