@@ -1,12 +1,13 @@
-"""The allocation-free key histogram, checked against the plan builder's.
+"""The allocation-free key histogram, checked against the oracle's and the plan builder's.
 
 cr_key_histogram_noalloc serves callers that cannot allocate device memory
 when they call in (device memory owned by another runtime's pool, or a
 latency-critical path that cannot afford cudaMalloc).  It must give exactly
-the histogram that cr_build_plans computes for the same keys, on repeated
-calls (its scratch array is shared and keeps the previous call's contents),
-and reject inputs larger than its fixed scratch.  This file is collected
-last so that a failure here never hides the results of the other tests.
+the oracle's histogram (and the one cr_build_plans computes) for the same
+keys, on repeated calls (its scratch array is shared and keeps the previous
+call's contents), and reject inputs larger than its fixed scratch.  This file
+is collected last so that a failure here never hides the results of the
+other tests.
 """
 import ctypes
 
@@ -67,10 +68,13 @@ def _reference(P, ctx, keys):
 
 
 def test_noalloc_histogram_matches_plan_builder_twice(P):
+    import oracle as O
     ctx = P.Context(0)
     for seed, nkeys, n in ((1, 3000, 60000), (2, 50, 700)):   # second call smaller: stale contents must not leak
         keys = _keys(seed, nkeys, n)
         uk, uc = _noalloc(P, keys)
+        ok, oc = O.histogram(keys)                # the oracle's (key ascending, count)
+        assert uk.size == ok.size and (uk == ok).all() and (uc == oc).all()
         rk, rc = _reference(P, ctx, keys)
         assert uk.size == rk.size and (uk == rk).all() and (uc == rc).all()
         assert int(uc.sum()) == n
