@@ -61,6 +61,7 @@ static_assert(sizeof(route_desc) == 48, "route_desc layout");
 struct route_args {
     route_desc d[CR_MAX_REPLICAS];
     uint32_t dep[CR_MAX_REPLICAS];    // load-dependent replicas, one CTA each in the resolve pass
+    uint32_t cand[CR_MAX_REPLICAS];   // candidate pass: the replica of each grid row, costliest first
 };
 
 // Candidate encoding, one u32 per (replica, request):
@@ -104,8 +105,8 @@ __global__ void __launch_bounds__(256) k_route_cand(const __grid_constant__ rout
                                                     unsigned long long n, unsigned long long g0, uint32_t R,
                                                     uint32_t *__restrict__ cand, uint16_t *__restrict__ dest)
 {
-    const uint32_t rep = blockIdx.y;
-    if (rep >= n_rep) return;
+    if (blockIdx.y >= n_rep) return;
+    const uint32_t rep = args.cand[blockIdx.y];  // rows of the costliest policies are scheduled first
     const route_desc &rd = args.d[rep];
     uint32_t *C = cand + (unsigned long long)rep * n;
     uint16_t *Dst = dest + (unsigned long long)rep * n;
@@ -950,6 +951,19 @@ extern "C" int cr_route_batch(cr_ctx *ctx, const cr_plan *const *plans, const cr
     uint32_t n_dep = 0;
     for (uint32_t i = 0; i < n_rep; ++i)
         if (reps[i].policy != CR_POLICY_RR && reps[i].policy != CR_POLICY_HASH) args.dep[n_dep++] = i;
+    // candidate rows, costliest policy first, so that the grid's last wave holds cheap rows
+    // (per request: jump hash ~8 jumps, Philox ~10 rounds, plan probe + Philox for misses,
+    // ring lookup, round robin)
+    {
+        auto cost = [&](uint32_t p) {
+            return p == CR_POLICY_HASH ? 0 : p == CR_POLICY_P2C ? 1 : p <= CR_POLICY_CR_NOREPL ? 2
+                 : p == CR_POLICY_CHWBL ? 3 : 4;
+        };
+        uint32_t k = 0;
+        for (uint32_t c = 0; c <= 4; ++c)
+            for (uint32_t i = 0; i < n_rep; ++i)
+                if ((uint32_t)cost(reps[i].policy) == c) args.cand[k++] = i;
+    }
     // split routing: the candidates scratch is free once the last resolution has read it
     const cudaStream_t rs = ctx->resolve_stream ? ctx->resolve_stream : ctx->stream;
     const bool split = rs != ctx->stream;
