@@ -1754,11 +1754,22 @@ static int build_plans(cr_ctx *ctx, const uint64_t *d_key, uint64_t n, const cr_
         }
         return CR_OK;
     }
-    // large intervals (and empty ones): plan by plan
+    // large intervals (and empty ones): plan by plan.  Eq. 1 and the admission depend only
+    // on (R, W, q_cap, single copy or not): a plan equal in those to an earlier one of the
+    // build (the random placements of several seeds, say) copies its admitted arrays and
+    // counters instead of recomputing them.
+    auto same_admission = [&](uint32_t a, uint32_t b) {
+        const cr_plan_params &x = params[a], &y = params[b];
+        return x.R == y.R && x.W == y.W && x.qcap_num == y.qcap_num && x.qcap_den == y.qcap_den &&
+               (x.variant == CR_VARIANT_NOREPL) == (y.variant == CR_VARIANT_NOREPL);
+    };
     for (uint32_t j = 0; j < n_plans; ++j) {
         cr_plan *p = plans[j];
         const cr_plan_params &pp = params[j];
         const uint64_t C = (uint64_t)pp.R * pp.W;
+        uint32_t src = j;
+        for (uint32_t i = 0; i < j && src == j; ++i)
+            if (same_admission(i, j)) src = i;
         if (j > 0 && n > 0) {
             CR_CUDA(ctx, cudaMemcpyAsync(p->d_ukey, p0->d_ukey, n * sizeof(unsigned long long),
                                          cudaMemcpyDeviceToDevice, ctx->stream));
@@ -1768,7 +1779,20 @@ static int build_plans(cr_ctx *ctx, const uint64_t *d_key, uint64_t n, const cr_
                                          cudaMemcpyDeviceToDevice, ctx->stream));  // U and S
         }
         CR_CUDA(ctx, cudaMemsetAsync(p->d_table, 0xff, p->table_slots * sizeof(cr_table_slot), ctx->stream));
-        if (n > 0) {
+        if (n > 0 && src != j) {
+            const cr_plan *q = plans[src];
+            const uint64_t na = n < C ? n : C;  // a bound on the admitted keys
+            CR_CUDA(ctx, cudaMemcpyAsync(p->d_info, q->d_info, sizeof(cr_plan_info_dev), cudaMemcpyDeviceToDevice,
+                                         ctx->stream));
+            CR_CUDA(ctx, cudaMemcpyAsync(p->d_adm_key, q->d_adm_key, na * sizeof(unsigned long long),
+                                         cudaMemcpyDeviceToDevice, ctx->stream));
+            CR_CUDA(ctx, cudaMemcpyAsync(p->d_adm_cnt, q->d_adm_cnt, na * sizeof(unsigned long long),
+                                         cudaMemcpyDeviceToDevice, ctx->stream));
+            CR_CUDA(ctx, cudaMemcpyAsync(p->d_adm_k, q->d_adm_k, na * sizeof(uint32_t), cudaMemcpyDeviceToDevice,
+                                         ctx->stream));
+            CR_CUDA(ctx, cudaMemcpyAsync(p->d_koff, q->d_koff, (na + 1) * sizeof(uint32_t), cudaMemcpyDeviceToDevice,
+                                         ctx->stream));
+        } else if (n > 0) {
             void *pk;
             CR_TRY(cr_scratch(ctx, SCR_PLAN_B, (n + 2) * sizeof(unsigned long long), &pk));
             unsigned long long *kk = (unsigned long long *)pk;
