@@ -81,24 +81,40 @@ __global__ void k_hist_insert(const unsigned long long *__restrict__ keys, uint6
 }
 
 // Occupied slots -> a dense list (order immaterial: it is sorted next).
+// Occupied slots appended to a dense list (order free: the list is sorted next).
+// A warp takes 8 x 32 consecutive slots and claims their places with one atomic:
+// one atomic per 32 slots on the single counter serialised the launch.
+constexpr int kCompactRounds = 8;
 __global__ void k_hist_compact(const unsigned long long *__restrict__ tkey, const uint32_t *__restrict__ tcnt,
                                uint64_t slots, unsigned long long *__restrict__ lkey, uint32_t *__restrict__ lcnt,
                                cr_plan_info_dev *info)
 {
-    const uint32_t lane = cr_lane();
-    for (uint64_t base = ((uint64_t)blockIdx.x * blockDim.x + threadIdx.x) & ~31ull; base < slots;
-         base += (uint64_t)gridDim.x * blockDim.x) {
-        const uint64_t s = base + lane;
-        const bool occ = s < slots && tkey[s] != kEmptyKey;
-        const uint32_t bal = __ballot_sync(0xffffffffu, occ);
-        if (!bal) continue;
+    const uint32_t lane = cr_lane(), lt = (1u << lane) - 1u;
+    constexpr uint64_t kSpan = 32ull * kCompactRounds;
+    const uint64_t w0 = ((uint64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+    const uint64_t nwarps = ((uint64_t)gridDim.x * blockDim.x) >> 5;
+    for (uint64_t base = w0 * kSpan; base < slots; base += nwarps * kSpan) {
+        unsigned long long k[kCompactRounds];
+        uint32_t bal[kCompactRounds], tot = 0;
+#pragma unroll
+        for (int r = 0; r < kCompactRounds; ++r) {
+            const uint64_t s = base + 32ull * r + lane;
+            k[r] = s < slots ? tkey[s] : kEmptyKey;
+            bal[r] = __ballot_sync(0xffffffffu, k[r] != kEmptyKey);
+            tot += (uint32_t)__popc(bal[r]);
+        }
+        if (!tot) continue;
         unsigned long long at = 0;
-        if (lane == 0) at = atomicAdd(&info->U, (unsigned long long)__popc(bal));
+        if (lane == 0) at = atomicAdd(&info->U, (unsigned long long)tot);
         at = __shfl_sync(0xffffffffu, at, 0);
-        if (occ) {
-            const unsigned long long pos = at + __popc(bal & ((1u << lane) - 1u));
-            lkey[pos] = tkey[s];
-            lcnt[pos] = tcnt[s];
+#pragma unroll
+        for (int r = 0; r < kCompactRounds; ++r) {
+            if (k[r] != kEmptyKey) {
+                const unsigned long long pos = at + (uint32_t)__popc(bal[r] & lt);
+                lkey[pos] = k[r];
+                lcnt[pos] = tcnt[base + 32ull * r + lane];
+            }
+            at += (uint32_t)__popc(bal[r]);
         }
     }
     if (blockIdx.x == 0 && threadIdx.x == 0 && info->special) {

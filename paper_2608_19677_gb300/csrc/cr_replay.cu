@@ -896,20 +896,43 @@ int launch_stamp(cr_ctx *ctx, cr_replay *rp, const replay_caps &caps, uint32_t C
                  const rec16 *recs, uint64_t *d_ctr)
 {
     const uint32_t cmax = rp->cmax, nw = stamp_words(cmax);
-    uint32_t nbb = 4;
-    while ((1u << nbb) < cmax) ++nbb;  // a bucket of four entries per resident key at most
-    const size_t per_warp = stamp_lru_bytes(cmax, nw, nbb);
-    // warps per block: the most warps per SM that shared memory allows
+    // warps per block: the most warps per SM that shared memory allows (at most 32
+    // blocks and 64 warps per SM, and what the registers allow)
     const size_t sm_bytes = 227 * 1024;
-    uint32_t wpb = 4, best = 0;
-    for (uint32_t x = 4; x >= 1; --x) {
-        const size_t blk = per_warp * x + 1024;
-        const uint32_t nb = blk <= sm_bytes ? (uint32_t)(sm_bytes / blk) : 0u;
-        if (nb * x > best) {
-            best = nb * x;
-            wpb = x;
+    cudaFuncAttributes fa;
+    uint32_t warps_regs = 64;
+    if (cudaFuncGetAttributes(&fa, k_lru_stamp<NC, NG, SMALL>) == cudaSuccess && fa.numRegs > 0)
+        warps_regs = 65536u / ((((uint32_t)fa.numRegs * 32u + 255u) / 256u) * 256u);
+    else
+        cudaGetLastError();
+    auto fit = [&](uint32_t nb_bits, uint32_t *wpb_out) {
+        const size_t pw = stamp_lru_bytes(cmax, nw, nb_bits);
+        uint32_t best = 0;
+        for (uint32_t x = 4; x >= 1; --x) {
+            const size_t blk = pw * x + 1024;
+            uint32_t nb = blk <= sm_bytes ? (uint32_t)(sm_bytes / blk) : 0u;
+            nb = nb < 32u ? nb : 32u;
+            nb = nb < warps_regs / x ? nb : warps_regs / x;
+            const uint32_t wps = nb * x < 64u ? nb * x : 64u;
+            if (wps > best) {
+                best = wps;
+                *wpb_out = x;
+            }
         }
+        return best;
+    };
+    // index buckets: one per resident key at most (a quarter of the entries live); half
+    // as many (half the entries live: a few more probes and inserts) when that fits more
+    // warps on an SM, i.e. when the state of the largest capacities bounds the occupancy
+    uint32_t nbb = 4;
+    while ((1u << nbb) < cmax) ++nbb;
+    uint32_t wpb = 1, wpb_half = 1;
+    const uint32_t w_full = fit(nbb, &wpb);
+    if (nbb > 4 && fit(nbb - 1, &wpb_half) * 10u >= w_full * 11u) {  // at least 10% more warps
+        --nbb;
+        wpb = wpb_half;
     }
+    const size_t per_warp = stamp_lru_bytes(cmax, nw, nbb);
     const size_t smem = per_warp * wpb;
     if (smem > 48 * 1024)
         CR_CUDA(ctx, cudaFuncSetAttribute(k_lru_stamp<NC, NG, SMALL>, cudaFuncAttributeMaxDynamicSharedMemorySize,
