@@ -68,3 +68,23 @@ def test_plan_stats_without_plans():
     assert bench.plan_stats(np.zeros((3, 0))) == {"median": None, "max": None, "builds_per_step": 0}
     st = bench.plan_stats(np.array([[1.0, 3.0], [2.0, 5.0]]))
     assert st == {"median": 2.5, "max": 5.0, "builds_per_step": 2}
+
+
+def test_schedule_defaults_follow_interval_size():
+    # a CUDA graph and long replay groups for many short intervals; the Large sweep's
+    # ~1M-request intervals run without a graph, two intervals per replay call
+    import tracegen as tg
+    import bench
+    got = {}
+    for name in ("tiny", "70b", "8b", "burst", "large"):
+        args = bench.parse_args(["--config", name])
+        bench.auto_schedule(args, tg.Trace(tg.CONFIGS[name]))
+        got[name] = (args.graph, args.trace_min_interval, args.replay_group)
+    assert got["large"] == (False, 65536, 2)
+    assert got["8b"] == (True, 0, 13)
+    assert got["70b"][0] and got["burst"][0] and got["tiny"][0]
+    args = bench.parse_args(["--config", "8b", "--no-graph", "--replay-group", "1"])
+    bench.auto_schedule(args, tg.Trace(tg.CONFIGS["8b"]))
+    assert (args.graph, args.trace_min_interval, args.replay_group) == (False, 65536, 1)
+    args = bench.parse_args(["--sm-split", "8"])
+    assert args.graph is False
