@@ -36,6 +36,10 @@
  *     reported by the next blocking call (cr_sync, *_export, *_info).
  *   - All quantities are unsigned integers: results are exact and
  *     deterministic (bit-identical run to run).
+ *   - A call whose scratch buffers are already large enough allocates
+ *     nothing and does not synchronise, so a sequence of non-blocking calls
+ *     can be captured into a CUDA graph after one pass over the same sizes
+ *     (stream capture on a stream other than the legacy default one).
  */
 #ifndef CACHEROUTE_H
 #define CACHEROUTE_H
