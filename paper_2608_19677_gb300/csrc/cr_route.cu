@@ -61,7 +61,9 @@ static_assert(sizeof(route_desc) == 48, "route_desc layout");
 struct route_args {
     route_desc d[CR_MAX_REPLICAS];
     uint32_t dep[CR_MAX_REPLICAS];    // load-dependent replicas, one CTA each in the resolve pass
-    uint32_t cand[CR_MAX_REPLICAS];   // candidate pass: the replica of each grid row, costliest first
+    uint32_t cand[CR_MAX_REPLICAS];   // candidate pass: replica order, costliest policy first
+    uint32_t rr_b0[CR_MAX_REPLICAS];  // round robin: (g0 + seed) mod 2^64 mod R
+    unsigned long long rr_wrap[CR_MAX_REPLICAS];  // round robin: first i where g0 + seed + i wraps (~0: never)
 };
 
 // Candidate encoding, one u32 per (replica, request):
@@ -97,95 +99,95 @@ __device__ __forceinline__ unsigned long long chwbl_cap(unsigned long long m, ui
     return (5ull * (m + 1ull) + den - 1ull) / den;
 }
 
-// Everything that does not depend on the live load, for every (replica, request):
-// blockIdx.y is the replica, so every block runs one policy's loop.
-// Load-independent replicas (RR, HASH) write their destinations directly.
+// Everything that does not depend on the live load, for every (replica, request).
+// A warp takes 32 consecutive requests, reads their keys once and computes the
+// candidates of the replicas of its group for them (blockIdx.y = group g of
+// gridDim.y: replicas args.cand[g], args.cand[g + G], ..., so every group mixes
+// costly and cheap policies; one group when the requests alone fill the GPU);
+// round robin and sticky-hash replicas write their destinations directly.
+// Plan replicas' table misses queue per warp in shared memory, and the warp draws
+// their power-of-two choices 32 at a time, so the Philox rounds run with every lane
+// busy.
 __global__ void __launch_bounds__(256) k_route_cand(const __grid_constant__ route_args args, uint32_t n_rep,
                                                     const unsigned long long *__restrict__ keys,
                                                     unsigned long long n, unsigned long long g0, uint32_t R,
                                                     uint32_t *__restrict__ cand, uint16_t *__restrict__ dest)
 {
-    if (blockIdx.y >= n_rep) return;
-    const uint32_t rep = args.cand[blockIdx.y];  // rows of the costliest policies are scheduled first
-    const route_desc &rd = args.d[rep];
-    uint32_t *C = cand + (unsigned long long)rep * n;
-    uint16_t *Dst = dest + (unsigned long long)rep * n;
+    __shared__ unsigned long long q_req[256 / 32][64];  // replica << 40 | request
+    const uint32_t lane = threadIdx.x & 31u, lt = (1u << lane) - 1u;
+    unsigned long long *Q = q_req[threadIdx.x >> 5];
+    uint32_t qn = 0;  // queued, < 32 between rounds
     const unsigned long long stride = (unsigned long long)gridDim.x * blockDim.x;
-    const unsigned long long i0 = (unsigned long long)blockIdx.x * blockDim.x + threadIdx.x;
-    switch (rd.policy) {
-    case CR_POLICY_RR: {
-        // (g0 + i + seed) mod 2^64 mod R.  Until the sum wraps (i < wrap) that is
-        // (base mod R + i mod R) mod R, which needs only 32-bit remainders while i < 2^32.
-        const unsigned long long base = g0 + rd.seed;
-        const unsigned long long wrap = base ? 0ull - base : ~0ull;
-        const uint32_t b0 = (uint32_t)(base % R);
-        for (unsigned long long i = i0; i < n; i += stride) {
-            uint32_t r;
-            if (i < wrap && i < (1ull << 32)) {
-                r = b0 + (uint32_t)i % R;
-                if (r >= R) r -= R;
-            } else {
-                r = (uint32_t)((base + i) % R);
-            }
-            Dst[i] = (uint16_t)r;
-        }
-        break;
-    }
-    case CR_POLICY_HASH:
-        for (unsigned long long i = i0; i < n; i += stride)
-            Dst[i] = (uint16_t)cr_jump_hash(cr_fmix64(keys[i] ^ rd.seed), R);
-        break;
-    case CR_POLICY_P2C:
-        for (unsigned long long i = i0; i < n; i += stride) C[i] = p2c_pair(rd.seed, rd.policy, g0 + i, R);
-        break;
-    case CR_POLICY_CHWBL:
-        for (unsigned long long i = i0; i < n; i += stride)
-            C[i] = kRing | ring_start(rd, cr_fmix64(keys[i] ^ rd.seed));
-        break;
-    default: {
-        // Table probes for every lane; the requests whose key is not in the table
-        // queue per warp, and the warp draws their power-of-two choices 32 at a time,
-        // so the Philox rounds run with every lane busy.
-        __shared__ unsigned long long q_req[256 / 32][64];
-        const uint32_t lane = threadIdx.x & 31u, lt = (1u << lane) - 1u;
-        unsigned long long *Q = q_req[threadIdx.x >> 5];
-        uint32_t qn = 0;  // queued, < 32 between rounds
-        const unsigned long long mask = (1ull << rd.tbits) - 1ull;
-        for (unsigned long long wb = i0 - lane; wb < n; wb += stride) {  // uniform over the warp
-            const unsigned long long i = wb + lane;
-            const bool valid = i < n;
-            uint32_t c = 0xffffffffu;
-            if (valid) {
-                const unsigned long long key = keys[i];
-                unsigned long long sl = key >> (64 - rd.tbits);
-                for (;;) {
-                    const cr_table_slot slot = rd.table[sl];
-                    if (slot.koff == kEmpty) break;
-                    if (slot.key == key) {
-                        c = slot.k == 1 ? (kFixed | slot.m0) : (kSet | (uint32_t)sl);
-                        break;
+    for (unsigned long long wb = (unsigned long long)blockIdx.x * blockDim.x + (threadIdx.x & ~31u); wb < n;
+         wb += stride) {  // uniform over the warp
+        const unsigned long long i = wb + lane;
+        const bool valid = i < n;
+        const unsigned long long key = valid ? keys[i] : 0ull;
+        for (uint32_t x = blockIdx.y; x < n_rep; x += gridDim.y) {  // uniform
+            const uint32_t rep = args.cand[x];
+            const route_desc &rd = args.d[rep];
+            const unsigned long long o = (unsigned long long)rep * n + i;
+            switch (rd.policy) {
+            case CR_POLICY_RR:
+                // (g0 + i + seed) mod 2^64 mod R: before the sum wraps, (b0 + i mod R) mod R
+                if (valid) {
+                    uint32_t r;
+                    if (i < args.rr_wrap[rep] && i < (1ull << 32)) {
+                        r = args.rr_b0[rep] + (uint32_t)i % R;
+                        if (r >= R) r -= R;
+                    } else {
+                        r = (uint32_t)((g0 + rd.seed + i) % R);
                     }
-                    sl = (sl + 1) & mask;
+                    dest[o] = (uint16_t)r;
                 }
-                if (c != 0xffffffffu) C[i] = c;
-            }
-            const bool miss = valid && c == 0xffffffffu;
-            const uint32_t mm = __ballot_sync(0xffffffffu, miss);
-            if (miss) Q[qn + (uint32_t)__popc(mm & lt)] = i;
-            qn += (uint32_t)__popc(mm);
-            __syncwarp();
-            if (qn >= 32u) {
-                const unsigned long long j = Q[qn - 32u + lane];
-                C[j] = p2c_pair(rd.seed, rd.policy, g0 + j, R);
-                qn -= 32u;
+                break;
+            case CR_POLICY_HASH:
+                if (valid) dest[o] = (uint16_t)cr_jump_hash(cr_fmix64(key ^ rd.seed), R);
+                break;
+            case CR_POLICY_P2C:
+                if (valid) cand[o] = p2c_pair(rd.seed, rd.policy, g0 + i, R);
+                break;
+            case CR_POLICY_CHWBL:
+                if (valid) cand[o] = kRing | ring_start(rd, cr_fmix64(key ^ rd.seed));
+                break;
+            default: {
+                uint32_t c = 0xffffffffu;
+                if (valid) {
+                    const unsigned long long mask = (1ull << rd.tbits) - 1ull;
+                    unsigned long long sl = key >> (64 - rd.tbits);
+                    for (;;) {
+                        const cr_table_slot slot = rd.table[sl];
+                        if (slot.koff == kEmpty) break;
+                        if (slot.key == key) {
+                            c = slot.k == 1 ? (kFixed | slot.m0) : (kSet | (uint32_t)sl);
+                            break;
+                        }
+                        sl = (sl + 1) & mask;
+                    }
+                    if (c != 0xffffffffu) cand[o] = c;
+                }
+                const bool miss = valid && c == 0xffffffffu;
+                const uint32_t mm = __ballot_sync(0xffffffffu, miss);
+                if (miss) Q[qn + (uint32_t)__popc(mm & lt)] = ((unsigned long long)rep << 40) | i;
+                qn += (uint32_t)__popc(mm);
                 __syncwarp();
+                if (qn >= 32u) {
+                    const unsigned long long e = Q[qn - 32u + lane];
+                    const uint32_t er = (uint32_t)(e >> 40);
+                    const unsigned long long j = e & ((1ull << 40) - 1ull);
+                    cand[(unsigned long long)er * n + j] = p2c_pair(args.d[er].seed, args.d[er].policy, g0 + j, R);
+                    qn -= 32u;
+                    __syncwarp();
+                }
             }
-        }
-        if (lane < qn) {
-            const unsigned long long j = Q[lane];
-            C[j] = p2c_pair(rd.seed, rd.policy, g0 + j, R);
+            }
         }
     }
+    if (lane < qn) {
+        const unsigned long long e = Q[lane];
+        const uint32_t er = (uint32_t)(e >> 40);
+        const unsigned long long j = e & ((1ull << 40) - 1ull);
+        cand[(unsigned long long)er * n + j] = p2c_pair(args.d[er].seed, args.d[er].policy, g0 + j, R);
     }
 }
 
@@ -971,10 +973,18 @@ extern "C" int cr_route_batch(cr_ctx *ctx, const cr_plan *const *plans, const cr
     void *pc;
     CR_TRY(cr_scratch(ctx, SCR_ROUTE_DESC, (size_t)n * n_rep * sizeof(uint32_t), &pc));
     uint32_t *cand = (uint32_t *)pc;
-    const unsigned int gcap = (unsigned int)ctx->num_sms * 16u;
     const int pcand = cr_prof_begin(ctx, ctx->stream, CR_PROF_ROUTE_CAND);
-    const dim3 cgrid(cr_blocks(n, 256, std::max(1u, gcap / n_rep)), n_rep);
-    CR_LAUNCH(ctx, k_route_cand, cgrid, 256, 0, args, n_rep,
+    for (uint32_t i = 0; i < n_rep; ++i) {
+        const uint64_t base = (uint64_t)first_req_index + reps[i].seed;  // wraps mod 2^64 as the policy does
+        args.rr_b0[i] = (uint32_t)(base % R);
+        args.rr_wrap[i] = base ? 0ull - base : ~0ull;
+    }
+    // request blocks; replica groups only as many as it takes to reach ~16 blocks per SM
+    const unsigned int cbx = cr_blocks(n, 256, (unsigned int)ctx->num_sms * 32u);
+    const unsigned int want = (unsigned int)ctx->num_sms * 16u;
+    unsigned int cgy = (want + cbx - 1) / cbx;
+    cgy = cgy < 1 ? 1 : (cgy > n_rep ? n_rep : cgy);
+    CR_LAUNCH(ctx, k_route_cand, dim3(cbx, cgy), 256, 0, args, n_rep,
               (const unsigned long long *)d_key, (unsigned long long)n, (unsigned long long)first_req_index, R, cand,
               d_dest);
     cr_prof_end(ctx, ctx->stream, pcand);
